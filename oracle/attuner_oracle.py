@@ -1,0 +1,215 @@
+"""Plain float64 definitions of the artifact-KV read path (test infrastructure).
+
+Only tests, the smoke check and the benchmark's CPU-baseline leg use this
+module.  It is deliberately slow and literal: no blocking, no fusion, no
+reordering beyond what each definition states.
+
+Notation follows the paper: h (here x) is the projection input, W^Q the base
+query projection, A in R^{r x d_model}, B in R^{d_q x r}, s = alpha / r.
+"""
+
+from __future__ import annotations
+
+import math
+from typing import Iterable, List, Optional, Sequence, Tuple
+
+import numpy as np
+
+
+def bf16_to_f64(t) -> np.ndarray:
+    """Exact widening of a bf16 tensor (torch, any device) to float64 numpy."""
+    import torch  # local: the oracle itself is numpy-only
+    if isinstance(t, np.ndarray):
+        return t.astype(np.float64)
+    return t.detach().to("cpu").to(torch.float64).numpy()
+
+
+# ---------------------------------------------------------------------------
+# Sec. 3, Eq. (query-adaptation): q~ = W^Q h + (alpha/r) B A h
+# ---------------------------------------------------------------------------
+def lora_q_projection(x: np.ndarray, w_q: np.ndarray, a: Optional[np.ndarray],
+                      b: Optional[np.ndarray], s: float) -> np.ndarray:
+    """Unmerged adapted query projection, one row per token.
+
+    x [M, d_model], w_q [d_q, d_model] (output x input), a [r, d_model],
+    b [d_q, r].  Returns q_raw [M, d_q] = x W^T + s * (x A^T) B^T.
+    a = b = None (or r = 0) is the merged / base path.
+    """
+    base = x @ w_q.T
+    if a is None or b is None or a.shape[0] == 0:
+        return base
+    down = x @ a.T            # A h        [M, r]
+    up = down @ b.T           # B (A h)    [M, d_q]
+    return base + s * up
+
+
+def merged_q_weight(w_q: np.ndarray, a: np.ndarray, b: np.ndarray, s: float) -> np.ndarray:
+    """App. A.5 (Deployment): W^Q <- W^Q + (alpha/r) B A."""
+    return w_q + s * (b @ a)
+
+
+# ---------------------------------------------------------------------------
+# Sec. 3 (after Eq. query-adaptation): the model's original query
+# normalisation (Qwen3 per-head RMSNorm over head_dim), then RoPE.
+# ---------------------------------------------------------------------------
+def rms_norm_heads(q: np.ndarray, w: np.ndarray, eps: float) -> np.ndarray:
+    """q [M, H, d] -> q / sqrt(mean_j q_j^2 + eps) * w, per (token, head)."""
+    ms = np.mean(q * q, axis=-1, keepdims=True)
+    return q / np.sqrt(ms + eps) * w
+
+
+def rope_rotate_half(q: np.ndarray, pos: np.ndarray, theta: float) -> np.ndarray:
+    """Rotary embedding, rotate-half pairing.
+
+    Element j < d/2 is paired with j + d/2 and the pair is rotated by the angle
+    pos * theta^(-2j/d).  q [M, H, d], pos [M] (integer positions).
+    """
+    d = q.shape[-1]
+    half = d // 2
+    j = np.arange(half, dtype=np.float64)
+    inv_freq = theta ** (-2.0 * j / d)                     # [d/2]
+    ang = np.asarray(pos, dtype=np.float64)[:, None] * inv_freq[None, :]   # [M, d/2]
+    c = np.cos(ang)[:, None, :]
+    sn = np.sin(ang)[:, None, :]
+    x1 = q[..., :half]
+    x2 = q[..., half:]
+    out = np.empty_like(q)
+    out[..., :half] = x1 * c - x2 * sn
+    out[..., half:] = x2 * c + x1 * sn
+    return out
+
+
+def query_positions(t_art: int, S: int, S_kv: int) -> np.ndarray:
+    """App. A.5: position ids of the assembled context.
+
+    Artifacts occupy assembled positions 0..T_art-1; the suffix KV occupies
+    T_art..T_art+S_kv-1 and the S query tokens are its last S entries.
+    """
+    return t_art + (S_kv - S) + np.arange(S, dtype=np.int64)
+
+
+# ---------------------------------------------------------------------------
+# Sec. 2 (PIC box, Eq. full-vs-pic) and App. A.3 "Cache construction and
+# reuse": cached blocks are assembled in prompt order without re-encoding.
+# Paging in 64-token blocks is this library's storage, not the paper's.
+# ---------------------------------------------------------------------------
+def assemble(art_lengths: Sequence[int], request: Sequence[int], block_tokens: int = 64) -> dict:
+    """Block table and index map of one request.
+
+    Storage rule (bump allocation in registration order): artifact j owns the
+    consecutive block ids starting at sum_{i<j} ceil(L_i / block_tokens);
+    local token p of artifact j lives in block first_j + p // block_tokens,
+    slot p % block_tokens.
+
+    Returns block_table, valid_len (per block of the request, runtime order),
+    index_map[t] = block * block_tokens + slot for assembled token t,
+    token_art[t], token_off[t] (artifact id and local offset of token t).
+    """
+    first = []
+    nxt = 0
+    for L in art_lengths:
+        first.append(nxt)
+        nxt += -(-int(L) // block_tokens)
+    block_table: List[int] = []
+    valid_len: List[int] = []
+    index_map: List[int] = []
+    token_art: List[int] = []
+    token_off: List[int] = []
+    for a in request:
+        L = int(art_lengths[a])
+        nb = -(-L // block_tokens)
+        for bi in range(nb):
+            block_table.append(first[a] + bi)
+            valid_len.append(min(block_tokens, L - bi * block_tokens))
+        for p in range(L):
+            index_map.append((first[a] + p // block_tokens) * block_tokens + p % block_tokens)
+            token_art.append(a)
+            token_off.append(p)
+    i32 = lambda v: np.asarray(v, dtype=np.int32)
+    return dict(block_table=i32(block_table), valid_len=i32(valid_len), index_map=i32(index_map),
+                token_art=i32(token_art), token_off=i32(token_off), first_block=i32(first),
+                total_blocks=nxt)
+
+
+# ---------------------------------------------------------------------------
+# Sec. 2.2, Eq. (routing-oracle): softmax(q K^T / sqrt(d_k) + M_t) V
+# ---------------------------------------------------------------------------
+def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, n_visible: Sequence[int],
+              pairs: Optional[Iterable[Tuple[int, int]]] = None):
+    """Grouped-query attention with a prefix-visibility mask.
+
+    q [S, Hq, d]; k, v [T, Hkv, d]; query head h reads KV head h // (Hq/Hkv).
+    Query i sees keys 0..n_visible[i]-1 (M_t = 0 there, -inf elsewhere).
+    Returns (o [S, Hq, d], lse [S, Hq]) or, with pairs = [(i, h), ...],
+    (o [P, d], lse [P]).  lse is the natural log of the softmax denominator
+    of the scaled logits.
+    """
+    S, Hq, d = q.shape
+    Hkv = k.shape[1]
+    G = Hq // Hkv
+    scale = 1.0 / math.sqrt(d)
+
+    def one(i, h):
+        n = int(n_visible[i])
+        kh = k[:n, h // G, :]
+        vh = v[:n, h // G, :]
+        logits = (kh @ q[i, h, :]) * scale
+        m = np.max(logits)
+        e = np.exp(logits - m)
+        z = np.sum(e)
+        return (e / z) @ vh, m + math.log(z)
+
+    if pairs is None:
+        o = np.zeros((S, Hq, d))
+        lse = np.zeros((S, Hq))
+        for i in range(S):
+            for h in range(Hq):
+                o[i, h], lse[i, h] = one(i, h)
+        return o, lse
+    pairs = list(pairs)
+    o = np.zeros((len(pairs), d))
+    lse = np.zeros(len(pairs))
+    for p, (i, h) in enumerate(pairs):
+        o[p], lse[p] = one(i, h)
+    return o, lse
+
+
+# ---------------------------------------------------------------------------
+# One request end to end: adapted Q -> q_norm -> RoPE -> attention over the
+# assembled artifact KV followed by the suffix's own KV.
+# ---------------------------------------------------------------------------
+def request_forward(x, w_q, a, b, s, q_norm_w, eps, theta, art_k: List[np.ndarray],
+                    art_v: List[np.ndarray], suffix_k, suffix_v, n_q_heads: int,
+                    pairs=None, q_only: bool = False):
+    """x [S, d_model]; art_k/art_v: per-artifact [L, Hkv, d] in runtime order;
+    suffix_k/suffix_v [S_kv, Hkv, d].  All float64.
+
+    Suffix query i sits at position T_art + (S_kv - S) + i and sees every
+    artifact token plus suffix keys j <= (S_kv - S) + i.
+    """
+    S = x.shape[0]
+    S_kv = suffix_k.shape[0]
+    d = suffix_k.shape[2]
+    t_art = int(sum(t.shape[0] for t in art_k))
+    q_raw = lora_q_projection(x, w_q, a, b, s).reshape(S, n_q_heads, d)
+    q_n = rms_norm_heads(q_raw, q_norm_w, eps)
+    q = rope_rotate_half(q_n, query_positions(t_art, S, S_kv), theta)
+    if q_only:
+        return q
+    k_all = np.concatenate(list(art_k) + [suffix_k], axis=0)
+    v_all = np.concatenate(list(art_v) + [suffix_v], axis=0)
+    n_visible = t_art + (S_kv - S) + np.arange(S) + 1
+    return attention(q, k_all, v_all, n_visible, pairs)
+
+
+def workload_reference(wl, req: int, pairs=None, q_only: bool = False):
+    """Run request_forward on request `req` of a seeded workload object."""
+    g = wl.geom
+    f = bf16_to_f64
+    a = None if wl.lora_a is None else f(wl.lora_a)
+    b = None if wl.lora_b is None else f(wl.lora_b)
+    ids = wl.requests[req]
+    return request_forward(
+        f(wl.x[req]), f(wl.w_q), a, b, g.scale, f(wl.q_norm_w), g.rms_eps, g.rope_theta,
+        [f(wl.art_k[i]) for i in ids], [f(wl.art_v[i]) for i in ids],
+        f(wl.suffix_k[req]), f(wl.suffix_v[req]), g.n_q_heads, pairs=pairs, q_only=q_only)

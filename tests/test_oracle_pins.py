@@ -1,0 +1,323 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+None of these tests needs a GPU.  Each oracle function is checked against
+something other than itself: hand-derived closed forms (tests/golden/),
+invariants the paper states (B = 0 gives base PIC, merged = unmerged, the
+artifact order does not matter, one artifact at global positions is full
+causal attention), and an fp64 library routine
+(torch.nn.functional.scaled_dot_product_attention on the CPU).
+"""
+
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from conftest import GOLDEN
+import oracle
+from oracle import attuner_oracle as O
+
+
+def _golden(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def _runs(runs, total):
+    out = np.full(total, -1, dtype=np.int64)
+    for start, count, first in runs:
+        out[start:start + count] = first + np.arange(count)
+    return out
+
+
+def _const_runs(runs, total):
+    out = np.full(total, -1, dtype=np.int64)
+    for start, count, val in runs:
+        out[start:start + count] = val
+    return out
+
+
+# --------------------------------------------------------------------------
+# Eq. (query-adaptation) and the merged deployment form
+# --------------------------------------------------------------------------
+def test_lora_projection_hand_example():
+    g = _golden("lora_q_projection_2x2.json")
+    w, a, b = (np.array(g[k]) for k in ("w_q", "lora_a", "lora_b"))
+    x = np.array(g["x"])
+    q = O.lora_q_projection(x, w, a, b, g["s"])
+    np.testing.assert_allclose(q, np.array(g["q_raw"]), atol=1e-14)
+    np.testing.assert_allclose(O.merged_q_weight(w, a, b, g["s"]), np.array(g["merged_w"]), atol=1e-14)
+
+
+def test_b_zero_is_base_pic():
+    # App. A.5: B starts at zero, so the initial update is zero.
+    rng = np.random.default_rng(11)
+    x = rng.standard_normal((5, 24))
+    w = rng.standard_normal((12, 24))
+    a = rng.standard_normal((4, 24))
+    b0 = np.zeros((12, 4))
+    np.testing.assert_array_equal(O.lora_q_projection(x, w, a, b0, 2.0), O.lora_q_projection(x, w, None, None, 2.0))
+
+
+def test_merged_equals_unmerged_and_scale_linear():
+    rng = np.random.default_rng(12)
+    x = rng.standard_normal((7, 32))
+    w = rng.standard_normal((16, 32))
+    a = rng.standard_normal((4, 32))
+    b = rng.standard_normal((16, 4))
+    un = O.lora_q_projection(x, w, a, b, 2.0)
+    mg = x @ O.merged_q_weight(w, a, b, 2.0).T
+    np.testing.assert_allclose(un, mg, rtol=1e-12, atol=1e-12)
+    # the update is linear in s: f(2) - f(0) = 2 (f(1) - f(0))
+    f0 = O.lora_q_projection(x, w, a, b, 0.0)
+    f1 = O.lora_q_projection(x, w, a, b, 1.0)
+    np.testing.assert_allclose(un - f0, 2.0 * (f1 - f0), rtol=1e-12, atol=1e-12)
+    # superposition over the rows of x: projecting unit vectors gives the columns
+    eye = np.eye(32)
+    cols = O.lora_q_projection(eye, w, a, b, 2.0)          # [32, 16]
+    np.testing.assert_allclose(x @ cols, un, rtol=1e-12, atol=1e-11)
+
+
+# --------------------------------------------------------------------------
+# q RMSNorm
+# --------------------------------------------------------------------------
+def test_rmsnorm_hand_example():
+    g = _golden("rms_norm_d2.json")
+    q = np.array(g["q"]).reshape(1, 1, 2)
+    for c in g["cases"]:
+        out = O.rms_norm_heads(q, np.array(g["w"]), c["eps"])
+        np.testing.assert_allclose(out.reshape(-1), c["out"], atol=1e-14)
+
+
+def test_rmsnorm_invariants():
+    rng = np.random.default_rng(13)
+    q = rng.standard_normal((6, 3, 16)) * 5
+    out = O.rms_norm_heads(q, np.ones(16), 1e-6)
+    rms = np.sqrt(np.mean(out ** 2, axis=-1))
+    assert np.all(rms <= 1.0) and np.all(rms > 1.0 - 1e-6)
+    # scale invariance and per-head independence (a wrong axis breaks one of these)
+    np.testing.assert_allclose(O.rms_norm_heads(3.0 * q, np.ones(16), 0.0), O.rms_norm_heads(q, np.ones(16), 0.0), atol=1e-13)
+    q2 = q.copy()
+    q2[:, 1, :] *= 100.0
+    q2[:, 2, :] = rng.standard_normal((6, 16))
+    np.testing.assert_array_equal(O.rms_norm_heads(q2, np.ones(16), 1e-6)[:, 0], O.rms_norm_heads(q, np.ones(16), 1e-6)[:, 0])
+
+
+# --------------------------------------------------------------------------
+# RoPE
+# --------------------------------------------------------------------------
+def test_rope_hand_example():
+    g = _golden("rope_d4.json")
+    q = np.array(g["q"]).reshape(1, 1, 4)
+    out = O.rope_rotate_half(q, np.array([g["pos"]]), g["theta"])
+    np.testing.assert_allclose(out.reshape(-1), g["out"], atol=1e-13)
+
+
+def test_rope_invariants():
+    rng = np.random.default_rng(14)
+    d, theta = 64, 1.0e6
+    q = rng.standard_normal((5, 2, d))
+    k = rng.standard_normal((5, 2, d))
+    p = np.array([0, 3, 17, 201, 131071])
+    # R(0) = I
+    np.testing.assert_array_equal(O.rope_rotate_half(q, np.zeros(5, dtype=np.int64), theta), q)
+    # norm preserving
+    np.testing.assert_allclose(np.linalg.norm(O.rope_rotate_half(q, p, theta), axis=-1), np.linalg.norm(q, axis=-1), rtol=1e-12)
+    # relative position: <R(p) q, R(p') k> = <R(p + c) q, R(p' + c) k>
+    p2 = np.array([5, 9, 1, 60, 100])
+    for c in (1, 37, 4096):
+        lhs = np.sum(O.rope_rotate_half(q, p, theta) * O.rope_rotate_half(k, p2, theta), axis=-1)
+        rhs = np.sum(O.rope_rotate_half(q, p + c, theta) * O.rope_rotate_half(k, p2 + c, theta), axis=-1)
+        np.testing.assert_allclose(lhs, rhs, rtol=1e-9, atol=1e-9)
+    # composition R(a) R(b) = R(a + b)
+    np.testing.assert_allclose(O.rope_rotate_half(O.rope_rotate_half(q, p, theta), p2, theta),
+                               O.rope_rotate_half(q, p + p2, theta), atol=1e-9)
+
+
+def test_query_positions():
+    # tiny workload: 201 artifact tokens, S = S_kv = 16 -> positions 201..216
+    np.testing.assert_array_equal(O.query_positions(201, 16, 16), np.arange(201, 217))
+    # decode: 128 prior suffix entries + the new token; the query is the last one
+    np.testing.assert_array_equal(O.query_positions(1000, 1, 129), [1128])
+
+
+# --------------------------------------------------------------------------
+# Assembly / index map
+# --------------------------------------------------------------------------
+def test_assemble_hand_example():
+    g = _golden("assemble_37_64_100.json")
+    for c in g["cases"]:
+        r = O.assemble(g["art_lengths"], c["request"], g["block_tokens"])
+        np.testing.assert_array_equal(r["block_table"], c["block_table"])
+        np.testing.assert_array_equal(r["valid_len"], c["valid_len"])
+        T = sum(g["art_lengths"][a] for a in c["request"])
+        np.testing.assert_array_equal(r["index_map"], _runs(c["index_map_runs"], T))
+        np.testing.assert_array_equal(r["token_art"], _const_runs(c["token_art_runs"], T))
+
+
+def test_assemble_brute_force_against_flat_storage():
+    # the index map must point at the same bytes as a flat concatenation
+    rng = np.random.default_rng(15)
+    lengths = rng.integers(1, 200, size=9).tolist()
+    r = O.assemble(lengths, [4, 0, 8, 4, 2])
+    pool = np.full(r["total_blocks"] * 64, -1, dtype=np.int64)
+    for a, L in enumerate(lengths):
+        for p in range(L):
+            pool[(r["first_block"][a] + p // 64) * 64 + p % 64] = a * 10000 + p
+    flat = np.concatenate([a * 10000 + np.arange(lengths[a]) for a in [4, 0, 8, 4, 2]])
+    np.testing.assert_array_equal(pool[r["index_map"]], flat)
+    assert np.sum(r["valid_len"]) == len(flat)
+
+
+# --------------------------------------------------------------------------
+# Attention, Eq. (routing-oracle)
+# --------------------------------------------------------------------------
+def test_attention_hand_example():
+    g = _golden("softmax_3keys.json")
+    q = np.array(g["q"]).reshape(1, 1, 2)
+    k = np.array([[math.sqrt(2.0) * math.log(i), 0.0] for i in g["k_from_log"]]).reshape(3, 1, 2)
+    v = np.array(g["v"]).reshape(3, 1, 2)
+    for c in g["cases"]:
+        o, lse = O.attention(q, k, v, [c["n_visible"]])
+        np.testing.assert_allclose(o.reshape(-1), c["o"], atol=1e-13)
+        np.testing.assert_allclose(lse.reshape(-1), [c["lse"]], atol=1e-13)
+
+
+def _sdpa_f64(q, k, v, n_visible):
+    """fp64 SDPA on CPU with GQA expanded (kv head = q head // G) and a prefix mask."""
+    S, Hq, d = q.shape
+    T, Hkv, _ = k.shape
+    G = Hq // Hkv
+    qt = torch.from_numpy(q).permute(1, 0, 2)[None]
+    kt = torch.from_numpy(k).repeat_interleave(G, dim=1).permute(1, 0, 2)[None]
+    vt = torch.from_numpy(v).repeat_interleave(G, dim=1).permute(1, 0, 2)[None]
+    mask = torch.from_numpy(np.arange(T)[None, :] < np.asarray(n_visible)[:, None])
+    o = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, attn_mask=mask)
+    return o[0].permute(1, 0, 2).numpy()
+
+
+def test_attention_matches_sdpa_f64_gqa():
+    rng = np.random.default_rng(16)
+    S, Hq, Hkv, d, T = 9, 8, 2, 32, 70
+    q = rng.standard_normal((S, Hq, d))
+    k = rng.standard_normal((T, Hkv, d))
+    v = rng.standard_normal((T, Hkv, d))
+    n_vis = T - S + np.arange(S) + 1
+    o, lse = O.attention(q, k, v, n_vis)
+    np.testing.assert_allclose(o, _sdpa_f64(q, k, v, n_vis), atol=1e-12)
+    # lse against an independent log-sum-exp of the scaled logits
+    from scipy.special import logsumexp
+    for i in (0, S - 1):
+        for h in (0, 5):
+            lg = k[:n_vis[i], h // 4] @ q[i, h] / math.sqrt(d)
+            assert abs(lse[i, h] - logsumexp(lg)) < 1e-12
+    # sampled pairs agree with the full evaluation
+    pairs = [(0, 0), (3, 7), (8, 2)]
+    op, lp = O.attention(q, k, v, n_vis, pairs)
+    for p, (i, h) in enumerate(pairs):
+        np.testing.assert_array_equal(op[p], o[i, h])
+        assert lp[p] == lse[i, h]
+
+
+def test_softmax_rows_sum_to_one_and_convex_hull():
+    rng = np.random.default_rng(17)
+    q = rng.standard_normal((4, 2, 8)) * 3
+    k = rng.standard_normal((30, 1, 8))
+    v = np.ones((30, 1, 8))
+    n_vis = [5, 12, 29, 30]
+    o, _ = O.attention(q, k, v, n_vis)
+    np.testing.assert_allclose(o, 1.0, atol=1e-14)
+    v = rng.standard_normal((30, 1, 8))
+    o, _ = O.attention(q, k, v, n_vis)
+    for i, n in enumerate(n_vis):
+        lo = v[:n, 0].min(axis=0)
+        hi = v[:n, 0].max(axis=0)
+        assert np.all(o[i] >= lo[None] - 1e-12) and np.all(o[i] <= hi[None] + 1e-12)
+
+
+def test_gqa_equals_mha_with_duplicated_heads():
+    rng = np.random.default_rng(18)
+    q = rng.standard_normal((5, 4, 16))
+    k = rng.standard_normal((20, 2, 16))
+    v = rng.standard_normal((20, 2, 16))
+    n_vis = [16, 17, 18, 19, 20]
+    o_gqa, l_gqa = O.attention(q, k, v, n_vis)
+    k_mha = k[:, [0, 0, 1, 1]]
+    v_mha = v[:, [0, 0, 1, 1]]
+    o_mha, l_mha = O.attention(q, k_mha, v_mha, n_vis)
+    np.testing.assert_array_equal(o_gqa, o_mha)
+    np.testing.assert_array_equal(l_gqa, l_mha)
+
+
+# --------------------------------------------------------------------------
+# End-to-end properties of one request
+# --------------------------------------------------------------------------
+def _small_inputs(rng, hidden=32, hq=4, hkv=2, d=16, r=4):
+    return dict(
+        w_q=rng.standard_normal((hq * d, hidden)) / math.sqrt(hidden),
+        a=rng.standard_normal((r, hidden)) / math.sqrt(hidden),
+        b=rng.standard_normal((hq * d, r)) / math.sqrt(r),
+        qn=1.0 + 0.1 * rng.standard_normal(d))
+
+
+def test_single_artifact_equals_full_causal():
+    # Eq. (full-vs-pic) with m = 1 and an empty prefix: the cached artifact is
+    # the full prefill of its own tokens, so the suffix rows equal causal
+    # attention over the whole L + S sequence.
+    rng = np.random.default_rng(19)
+    hidden, hq, hkv, d, theta, eps, s = 32, 4, 2, 16, 1.0e4, 1e-6, 2.0
+    L, S = 50, 7
+    w = _small_inputs(rng, hidden, hq, hkv, d)
+    k_raw = rng.standard_normal((L + S, hkv, d))
+    v = rng.standard_normal((L + S, hkv, d))
+    k_rot = O.rope_rotate_half(k_raw, np.arange(L + S), theta)   # global positions 0..L+S-1
+    x = rng.standard_normal((S, hidden))
+    o, lse = O.request_forward(x, w["w_q"], w["a"], w["b"], s, w["qn"], eps, theta,
+                               [k_rot[:L]], [v[:L]], k_rot[L:], v[L:], hq)
+    # Full side: queries built step by step at positions L..L+S-1, random
+    # queries for the artifact tokens, plain causal SDPA over L + S tokens.
+    q_raw = O.lora_q_projection(x, w["w_q"], w["a"], w["b"], s).reshape(S, hq, d)
+    q_suf = O.rope_rotate_half(O.rms_norm_heads(q_raw, w["qn"], eps), np.arange(L, L + S), theta)
+    q_full = np.concatenate([rng.standard_normal((L, hq, d)), q_suf], axis=0)
+    qt = torch.from_numpy(q_full).permute(1, 0, 2)[None]
+    kt = torch.from_numpy(k_rot).repeat_interleave(hq // hkv, dim=1).permute(1, 0, 2)[None]
+    vt = torch.from_numpy(v).repeat_interleave(hq // hkv, dim=1).permute(1, 0, 2)[None]
+    full = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True)[0].permute(1, 0, 2).numpy()
+    np.testing.assert_allclose(o, full[L:], atol=1e-12)
+
+
+def test_artifact_order_invariance():
+    # keys are pre-rotated at local positions and every artifact token is
+    # visible to every suffix query, so the output is a softmax over a set.
+    rng = np.random.default_rng(20)
+    hidden, hq, hkv, d = 32, 4, 2, 16
+    w = _small_inputs(rng, hidden, hq, hkv, d)
+    lens = [13, 64, 40]
+    ak = [rng.standard_normal((L, hkv, d)) for L in lens]
+    av = [rng.standard_normal((L, hkv, d)) for L in lens]
+    x = rng.standard_normal((6, hidden))
+    sk = rng.standard_normal((9, hkv, d))
+    sv = rng.standard_normal((9, hkv, d))
+    args = (x, w["w_q"], w["a"], w["b"], 2.0, w["qn"], 1e-6, 1e6)
+    o0, l0 = O.request_forward(*args, ak, av, sk, sv, hq)
+    for perm in ([2, 0, 1], [1, 2, 0], [2, 1, 0]):
+        o1, l1 = O.request_forward(*args, [ak[i] for i in perm], [av[i] for i in perm], sk, sv, hq)
+        np.testing.assert_allclose(o1, o0, atol=1e-12)
+        np.testing.assert_allclose(l1, l0, atol=1e-12)
+
+
+def test_tiny_workload_against_sdpa():
+    # the tiny parity workload, end to end, against fp64 SDPA
+    from gen import make_workload
+    wl = make_workload("tiny")
+    o, lse = O.workload_reference(wl, 0)
+    q = O.workload_reference(wl, 0, q_only=True)
+    f = O.bf16_to_f64
+    k = np.concatenate([f(t) for t in wl.art_k] + [f(wl.suffix_k[0])])
+    v = np.concatenate([f(t) for t in wl.art_v] + [f(wl.suffix_v[0])])
+    n_vis = 201 + np.arange(16) + 1
+    np.testing.assert_allclose(o, _sdpa_f64(q, k, v, n_vis), atol=1e-12)
+    assert o.shape == (16, 4, 64) and np.all(np.isfinite(lse))
