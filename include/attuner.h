@@ -1,0 +1,207 @@
+/*
+ * attuner.h - C ABI of the artifact-KV read path (libattuner.so).
+ *
+ * The library implements, for one decoder layer on one GB300 (sm_103a), the
+ * request-time read of a frozen, independently cached artifact KV store as
+ * the paper describes it:
+ *
+ *   Sec. 2, Eq. (1) and Eq. (full-vs-pic): every artifact A_j is encoded on
+ *     its own, at local positions 0..L_j-1, and its K/V are stored for reuse;
+ *     at request time the cached blocks are assembled in prompt order without
+ *     re-encoding (App. A.3 "Cache construction and reuse", App. C.1 PIC).
+ *   Sec. 3, Eq. (query-adaptation): the online tokens use the adapted query
+ *     q = W^Q h + (alpha/r) B A h, then the model's original query RMSNorm
+ *     and RoPE; artifact K/V never change.
+ *   Sec. 2.2, Eq. (routing-oracle) and App. A.5 (Deployment): attention is
+ *     softmax(q K^T / sqrt(d_k) + M_t) V with a causal mask and position ids
+ *     of the assembled context.
+ *
+ * Conventions shared by every entry point
+ *   - All tensors are row-major (last index fastest).  "bf16" is IEEE
+ *     bfloat16 stored as 16-bit words.  Pointers are DEVICE pointers on the
+ *     context's device unless the argument name ends in _host.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Device work is enqueued on it; the call returns before that
+ *     work finishes unless the documentation says otherwise.
+ *   - Every function returns an attuner_status and never throws.  On error a
+ *     thread-local message is available from attuner_last_error().
+ *   - The caller owns every input and output buffer; the library owns the
+ *     context, the paged pool, plans and its per-call scratch (drawn from a
+ *     stream-ordered memory pool of the context).
+ *   - A context is not thread-safe: calls on one context must come from one
+ *     host thread at a time.  Calls on different streams may overlap on the
+ *     GPU; each call's scratch is private to it.
+ *   - Device-side checks (bounded waits on mbarriers, block ids inside the
+ *     pool) never trap: they set a status word in the context, which
+ *     attuner_sync_status() returns and clears.
+ */
+#ifndef ATTUNER_H_
+#define ATTUNER_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t attuner_status;
+
+#define ATTUNER_OK                    0
+#define ATTUNER_ERR_INVALID_ARG      (-1) /* a size, pointer or id is out of range      */
+#define ATTUNER_ERR_OOM              (-2) /* pool full or a device allocation failed     */
+#define ATTUNER_ERR_UNKNOWN_ARTIFACT (-3) /* an artifact id was never registered         */
+#define ATTUNER_ERR_CUDA             (-4) /* a CUDA runtime or driver call failed        */
+#define ATTUNER_ERR_TIMEOUT          (-5) /* a kernel's bounded wait ran out             */
+#define ATTUNER_ERR_UNSUPPORTED      (-6) /* geometry this build has no kernel for       */
+#define ATTUNER_ERR_DEVICE_CHECK     (-7) /* a kernel's bounds check rejected an index   */
+
+/* Tokens per paged KV block.  Paging is this library's storage; the paper
+ * only says that cached blocks are assembled (Sec. 2). */
+#define ATTUNER_BLOCK_TOKENS 64
+
+typedef struct attuner_config {
+    int32_t hidden;        /* d_model of the projection input h (multiple of 64)          */
+    int32_t n_q_heads;     /* Hq                                                           */
+    int32_t n_kv_heads;    /* Hkv; Hq % Hkv == 0, G = Hq / Hkv in {1, 2, 4, 8}             */
+    int32_t head_dim;      /* d in {64, 128}                                               */
+    int32_t block_tokens;  /* must be ATTUNER_BLOCK_TOKENS                                 */
+    int32_t pool_blocks;   /* capacity of the paged K/V pool, in blocks                    */
+    float   rope_theta;    /* RoPE base (1e6 for Qwen3)                                    */
+    float   rms_eps;       /* q RMSNorm epsilon (1e-6 for Qwen3)                           */
+    int32_t device;        /* CUDA device ordinal the context lives on                     */
+} attuner_config;
+
+typedef struct attuner_ctx attuner_ctx;
+typedef struct attuner_plan attuner_plan;
+
+/* Create a context: allocates the paged K/V pool of cfg->pool_blocks blocks,
+ * each [Hkv][64][d] bf16 for K and the same for V (16 KiB per block and head
+ * at d = 128).  Errors: INVALID_ARG for an unsupported field, OOM, CUDA. */
+attuner_status attuner_create(const attuner_config* cfg, attuner_ctx** out);
+
+/* Free the context, its pool and every stream-ordered scratch it cached.
+ * The caller must have finished all work it enqueued with this context and
+ * freed its plans first. NULL is accepted. */
+attuner_status attuner_destroy(attuner_ctx* ctx);
+
+/* Register one artifact (Sec. 2, Eq. full-vs-pic: Z^PIC = C(A | P_cache),
+ * encoded alone at local positions 0..L-1, K already rotated there).
+ *   k, v : [L, Hkv, d] bf16, device.  Copied into ceil(L/64) consecutive pool
+ *          blocks on `stream`; the caller's buffers are free once that copy
+ *          has run.
+ *   Blocks are handed out in registration order by a bump allocator:
+ *   artifact j owns blocks first_j .. first_j + ceil(L_j/64) - 1 with
+ *   first_j = sum_{i<j} ceil(L_i/64), and artifact ids are 0, 1, 2, ...
+ * Errors: INVALID_ARG (L <= 0, NULL pointers), OOM (pool full). */
+attuner_status attuner_register_artifact(attuner_ctx* ctx, const void* k, const void* v,
+                                         int32_t L, void* stream, int32_t* artifact_id_out);
+
+/* Assemble a batch of requests (Sec. 2 PIC box: cached blocks in prompt
+ * order; App. A.3).  artifact_ids_host lists every request's artifacts in
+ * runtime order, CSR-indexed by req_offsets_host[0..n_req] (host arrays).
+ * Duplicates are allowed (assembled twice); an empty list is allowed (the
+ * request then attends to its suffix only).  The plan holds, per request,
+ * the block table (pool block, valid length) and the assembled index map
+ * index_map[t] = block * 64 + slot for t in [0, T_art).  Synchronous: the
+ * plan is on the device when the call returns.
+ * Errors: INVALID_ARG, UNKNOWN_ARTIFACT, OOM, CUDA. */
+attuner_status attuner_assemble(attuner_ctx* ctx, const int32_t* artifact_ids_host,
+                                const int32_t* req_offsets_host, int32_t n_req,
+                                attuner_plan** out);
+
+/* Copy a plan's layout to host arrays (for bit-exact tests).
+ * sizes_inout[0..4] on input: capacities of block_table, valid_len,
+ * index_map, token_art, token_off (elements); on output: the lengths used,
+ * and sizes_inout[5] = number of requests.  Per request the arrays are
+ * concatenated in request order (blocks first by request, then tokens).
+ * Any output pointer may be NULL to skip it.  Errors: INVALID_ARG when a
+ * capacity is too small. */
+attuner_status attuner_plan_export(const attuner_plan* plan, int32_t* block_table_host,
+                                   int32_t* valid_len_host, int32_t* index_map_host,
+                                   int32_t* token_art_host, int32_t* token_off_host,
+                                   int64_t* sizes_inout);
+
+/* Per-request assembled artifact length T_art (host array of n_req). */
+attuner_status attuner_plan_t_art(const attuner_plan* plan, int32_t* t_art_host, int32_t n_req);
+
+/* Free a plan. The caller must have finished all work that reads it. */
+attuner_status attuner_plan_free(attuner_plan* plan);
+
+/* Adapted query of the online tokens (Sec. 3, Eq. query-adaptation, then
+ * the query RMSNorm and RoPE):
+ *   q[m] = RoPE( RMSNorm_head( W_q x_m + s * B (A x_m) ) * q_norm_w, pos_m )
+ *   x        [n_req, S, hidden] bf16
+ *   w_q      [Hq*d, hidden] bf16 (output x input, as stored by HF q_proj)
+ *   lora_a   [r, hidden] bf16, lora_b [Hq*d, r] bf16; r in {0, 8, 16, ..., 64};
+ *            r = 0 or NULL A/B is the merged deployment form (App. A.5).
+ *            A x is rounded to bf16 before B is applied (as a bf16 PEFT layer
+ *            does); everything else accumulates in fp32.
+ *   q_norm_w [d] bf16; eps and theta come from the context config.
+ *   pos_m    = T_art(req) + (S_kv - S) + i for suffix token i.
+ *   q_out    [n_req, S, Hq, d] bf16.
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+attuner_status attuner_q_project(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
+                                 const void* w_q, const void* lora_a, const void* lora_b,
+                                 int32_t r, float s, const void* q_norm_w, int32_t S,
+                                 int32_t S_kv, void* q_out, void* stream);
+
+/* Attention of the online queries over the assembled artifact KV followed
+ * by the suffix's own KV (Eq. routing-oracle with the causal mask M_t):
+ *   q        [n_req, S, Hq, d] bf16 (already normalised and rotated)
+ *   suffix_k, suffix_v [n_req, S_kv, Hkv, d] bf16, K rotated at positions
+ *            T_art .. T_art + S_kv - 1.
+ *   Query i of a request sees all T_art artifact tokens and suffix keys
+ *   j <= (S_kv - S) + i; q head h reads KV head h / (Hq/Hkv).
+ *   out      [n_req, S, Hq, d] bf16, softmax(q k^T / sqrt(d)) v.
+ *   lse_out  [n_req, S, Hq] fp32 natural-log softmax denominator, or NULL.
+ * A plan with no artifacts gives plain causal attention over the suffix.
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+attuner_status attuner_attend(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
+                              const void* suffix_k, const void* suffix_v, int32_t S,
+                              int32_t S_kv, void* out, float* lse_out, void* stream);
+
+/* The whole path: attuner_q_project into stream-ordered scratch, then
+ * attuner_attend.  Arguments as in those two calls. */
+attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
+                                    const void* w_q, const void* lora_a, const void* lora_b,
+                                    int32_t r, float s, const void* q_norm_w,
+                                    const void* suffix_k, const void* suffix_v, int32_t S,
+                                    int32_t S_kv, void* out, float* lse_out, void* stream);
+
+/* The paged pool: device base pointers of K and V ([pool_blocks][Hkv][64][d]
+ * bf16 each), blocks in use and capacity.  Any output may be NULL. */
+attuner_status attuner_pool_info(const attuner_ctx* ctx, void** k_pool, void** v_pool,
+                                 int32_t* used_blocks, int32_t* capacity_blocks);
+
+/* Synchronise `stream`, then return and clear the device status word:
+ * OK, TIMEOUT (a bounded wait ran out) or DEVICE_CHECK (an index failed a
+ * bounds check), or CUDA if the synchronisation itself failed. */
+attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
+
+/* Tuning and test options (value 0 restores the default):
+ *   ATTUNER_OPT_PREFILL_KERNEL  0 auto, 1 tcgen05 tile kernel, 2 warp-MMA kernel
+ *   ATTUNER_OPT_SPLIT_BLOCKS    KV blocks per split-KV chunk (0 = automatic)
+ *   ATTUNER_OPT_WAIT_LIMIT      clock cycles a device wait may spin before it
+ *                               gives up and sets TIMEOUT (0 = about 2 s)
+ *   ATTUNER_OPT_TEST_STUCK_WAIT see below */
+#define ATTUNER_OPT_PREFILL_KERNEL 1
+#define ATTUNER_OPT_SPLIT_BLOCKS   2
+#define ATTUNER_OPT_WAIT_LIMIT     3
+/* Test hook (failure detection without a GPU fault): while non-zero, one
+ * role of every attention launch waits on an mbarrier that nothing arrives
+ * at; its bounded wait runs out, the kernel drains its own copies, frees its
+ * tensor memory and returns, and attuner_sync_status() reports TIMEOUT. */
+#define ATTUNER_OPT_TEST_STUCK_WAIT 1000
+attuner_status attuner_set_option(attuner_ctx* ctx, int32_t option, int64_t value);
+
+/* Number of kernel launches the last call on this context enqueued. */
+int32_t attuner_last_launch_count(const attuner_ctx* ctx);
+
+/* Message of the last error on this host thread ("" if none). */
+const char* attuner_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ATTUNER_H_ */

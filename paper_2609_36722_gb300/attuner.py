@@ -1,0 +1,294 @@
+"""ctypes binding of libattuner (include/attuner.h).
+
+Argument marshalling only: every step of the path runs in the library's CUDA
+kernels.  PyTorch supplies device memory (``tensor.data_ptr()``) and streams
+(``torch.cuda.current_stream().cuda_stream``).  There is no fallback: if the
+shared library is missing, importing this module raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import List, Optional, Sequence
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libattuner.so")
+
+OK = 0
+ERR_INVALID_ARG = -1
+ERR_OOM = -2
+ERR_UNKNOWN_ARTIFACT = -3
+ERR_CUDA = -4
+ERR_TIMEOUT = -5
+ERR_UNSUPPORTED = -6
+ERR_DEVICE_CHECK = -7
+
+OPT_PREFILL_KERNEL = 1
+OPT_SPLIT_BLOCKS = 2
+OPT_WAIT_LIMIT = 3
+OPT_TEST_STUCK_WAIT = 1000
+
+BLOCK_TOKENS = 64
+
+# every symbol include/attuner.h declares
+EXPORTS = [
+    "attuner_create", "attuner_destroy", "attuner_register_artifact", "attuner_assemble",
+    "attuner_plan_export", "attuner_plan_t_art", "attuner_plan_free", "attuner_q_project",
+    "attuner_attend", "attuner_query_attend", "attuner_pool_info", "attuner_sync_status",
+    "attuner_set_option", "attuner_last_launch_count", "attuner_last_error",
+]
+
+
+class AttunerError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"attuner status {status}: {msg}")
+        self.status = status
+
+
+class Config(ctypes.Structure):
+    _fields_ = [
+        ("hidden", ctypes.c_int32), ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32), ("block_tokens", ctypes.c_int32), ("pool_blocks", ctypes.c_int32),
+        ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float), ("device", ctypes.c_int32),
+    ]
+
+
+_vp = ctypes.c_void_p
+_i32 = ctypes.c_int32
+_p_i32 = ctypes.POINTER(ctypes.c_int32)
+_p_i64 = ctypes.POINTER(ctypes.c_int64)
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    if not os.path.exists(path):
+        raise ImportError(f"libattuner.so is not built ({path}); run __graft_entry__.build() "
+                          "or python -m paper_2609_36722_gb300.build")
+    lib = ctypes.CDLL(path)
+    sig = {
+        "attuner_create": ([ctypes.POINTER(Config), ctypes.POINTER(_vp)], _i32),
+        "attuner_destroy": ([_vp], _i32),
+        "attuner_register_artifact": ([_vp, _vp, _vp, _i32, _vp, _p_i32], _i32),
+        "attuner_assemble": ([_vp, _p_i32, _p_i32, _i32, ctypes.POINTER(_vp)], _i32),
+        "attuner_plan_export": ([_vp, _p_i32, _p_i32, _p_i32, _p_i32, _p_i32, _p_i64], _i32),
+        "attuner_plan_t_art": ([_vp, _p_i32, _i32], _i32),
+        "attuner_plan_free": ([_vp], _i32),
+        "attuner_q_project": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _i32, _i32, _vp, _vp], _i32),
+        "attuner_attend": ([_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
+        "attuner_query_attend": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _vp, _vp, _i32, _i32,
+                                  _vp, _vp, _vp], _i32),
+        "attuner_pool_info": ([_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _p_i32, _p_i32], _i32),
+        "attuner_sync_status": ([_vp, _vp], _i32),
+        "attuner_set_option": ([_vp, _i32, ctypes.c_int64], _i32),
+        "attuner_last_launch_count": ([_vp], _i32),
+        "attuner_last_error": ([], ctypes.c_char_p),
+    }
+    for name, (args, ret) in sig.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = ret
+    return lib
+
+
+_LIB: Optional[ctypes.CDLL] = None
+
+
+def lib() -> ctypes.CDLL:
+    global _LIB
+    if _LIB is None:
+        _LIB = load_library()
+    return _LIB
+
+
+def _check(status: int):
+    if status != OK:
+        raise AttunerError(status, lib().attuner_last_error().decode())
+
+
+def _ptr(t: Optional[torch.Tensor], name: str, dtype=torch.bfloat16) -> Optional[int]:
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+class Plan:
+    """Assembled requests: block tables and index maps on the device."""
+
+    def __init__(self, ctx: "Context", handle: ctypes.c_void_p, requests: List[List[int]]):
+        self.ctx = ctx
+        self.handle = handle
+        self.requests = requests
+        self.n_req = len(requests)
+
+    def t_art(self) -> List[int]:
+        arr = (ctypes.c_int32 * self.n_req)()
+        _check(lib().attuner_plan_t_art(self.handle, arr, self.n_req))
+        return list(arr)
+
+    def export(self):
+        """Host copies of block table, valid lengths, index map, token artifact and offset."""
+        import numpy as np
+        sizes = (ctypes.c_int64 * 6)(0, 0, 0, 0, 0, 0)
+        _check(lib().attuner_plan_export(self.handle, None, None, None, None, None, sizes))
+        nb, nt = sizes[0], sizes[2]
+        arrs = [np.zeros(max(n, 1), dtype=np.int32) for n in (nb, nb, nt, nt, nt)]
+        ptrs = [a.ctypes.data_as(_p_i32) for a in arrs]
+        _check(lib().attuner_plan_export(self.handle, *ptrs, sizes))
+        bt, vl, im, ta, to = (a[:n] for a, n in zip(arrs, (nb, nb, nt, nt, nt)))
+        return dict(block_table=bt, valid_len=vl, index_map=im, token_art=ta, token_off=to)
+
+    def free(self):
+        if self.handle:
+            lib().attuner_plan_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+class Context:
+    """One layer's artifact KV store on one GPU (attuner_create)."""
+
+    def __init__(self, hidden: int, n_q_heads: int, n_kv_heads: int, head_dim: int, pool_blocks: int,
+                 rope_theta: float = 1.0e6, rms_eps: float = 1.0e-6, device: int = 0):
+        cfg = Config(hidden, n_q_heads, n_kv_heads, head_dim, BLOCK_TOKENS, pool_blocks, rope_theta, rms_eps,
+                     device)
+        h = ctypes.c_void_p()
+        _check(lib().attuner_create(ctypes.byref(cfg), ctypes.byref(h)))
+        self.handle = h
+        self.cfg = cfg
+        self.device = torch.device("cuda", device)
+
+    @classmethod
+    def for_geometry(cls, geom, pool_blocks: int, device: int = 0) -> "Context":
+        return cls(geom.hidden, geom.n_q_heads, geom.n_kv_heads, geom.head_dim, pool_blocks,
+                   geom.rope_theta, geom.rms_eps, device)
+
+    def close(self):
+        if getattr(self, "handle", None):
+            lib().attuner_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # --- artifacts and plans
+    def register_artifact(self, k: torch.Tensor, v: torch.Tensor, stream=None) -> int:
+        if k.shape != v.shape or k.dim() != 3:
+            raise ValueError("k and v must both be [L, Hkv, d]")
+        aid = ctypes.c_int32(-1)
+        _check(lib().attuner_register_artifact(self.handle, _ptr(k, "k"), _ptr(v, "v"), k.shape[0],
+                                               _stream(stream), ctypes.byref(aid)))
+        return aid.value
+
+    def assemble(self, requests: Sequence[Sequence[int]]) -> Plan:
+        reqs = [list(map(int, r)) for r in requests]
+        flat = [a for r in reqs for a in r]
+        offs = [0]
+        for r in reqs:
+            offs.append(offs[-1] + len(r))
+        ids = (ctypes.c_int32 * max(len(flat), 1))(*flat)
+        off_arr = (ctypes.c_int32 * len(offs))(*offs)
+        h = ctypes.c_void_p()
+        _check(lib().attuner_assemble(self.handle, ids, off_arr, len(reqs), ctypes.byref(h)))
+        return Plan(self, h, reqs)
+
+    # --- compute
+    def q_project(self, plan: Plan, x, w_q, lora_a, lora_b, s: float, q_norm_w, S_kv: Optional[int] = None,
+                  out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+        n_req, S, _ = x.shape
+        S_kv = S if S_kv is None else S_kv
+        r = 0 if lora_a is None else lora_a.shape[0]
+        if out is None:
+            out = torch.empty(n_req, S, self.cfg.n_q_heads, self.cfg.head_dim, dtype=torch.bfloat16, device=x.device)
+        _check(lib().attuner_q_project(self.handle, plan.handle, _ptr(x, "x"), _ptr(w_q, "w_q"),
+                                       _ptr(lora_a, "lora_a"), _ptr(lora_b, "lora_b"), r, float(s),
+                                       _ptr(q_norm_w, "q_norm_w"), S, S_kv, _ptr(out, "out"), _stream(stream)))
+        return out
+
+    def attend(self, plan: Plan, q, suffix_k, suffix_v, out: Optional[torch.Tensor] = None,
+               lse: Optional[torch.Tensor] = None, want_lse: bool = True, stream=None):
+        n_req, S, Hq, d = q.shape
+        S_kv = suffix_k.shape[1]
+        if out is None:
+            out = torch.empty_like(q)
+        if lse is None and want_lse:
+            lse = torch.empty(n_req, S, Hq, dtype=torch.float32, device=q.device)
+        _check(lib().attuner_attend(self.handle, plan.handle, _ptr(q, "q"), _ptr(suffix_k, "suffix_k"),
+                                    _ptr(suffix_v, "suffix_v"), S, S_kv, _ptr(out, "out"),
+                                    _ptr(lse, "lse", torch.float32), _stream(stream)))
+        return out, lse
+
+    def query_attend(self, plan: Plan, x, w_q, lora_a, lora_b, s: float, q_norm_w, suffix_k, suffix_v,
+                     out: Optional[torch.Tensor] = None, lse: Optional[torch.Tensor] = None,
+                     want_lse: bool = True, stream=None):
+        n_req, S, _ = x.shape
+        S_kv = suffix_k.shape[1]
+        r = 0 if lora_a is None else lora_a.shape[0]
+        if out is None:
+            out = torch.empty(n_req, S, self.cfg.n_q_heads, self.cfg.head_dim, dtype=torch.bfloat16, device=x.device)
+        if lse is None and want_lse:
+            lse = torch.empty(n_req, S, self.cfg.n_q_heads, dtype=torch.float32, device=x.device)
+        _check(lib().attuner_query_attend(self.handle, plan.handle, _ptr(x, "x"), _ptr(w_q, "w_q"),
+                                          _ptr(lora_a, "lora_a"), _ptr(lora_b, "lora_b"), r, float(s),
+                                          _ptr(q_norm_w, "q_norm_w"), _ptr(suffix_k, "suffix_k"),
+                                          _ptr(suffix_v, "suffix_v"), S, S_kv, _ptr(out, "out"),
+                                          _ptr(lse, "lse", torch.float32), _stream(stream)))
+        return out, lse
+
+    # --- misc
+    def pool_tensors(self):
+        """(K pool, V pool) as torch views [pool_blocks, Hkv, 64, d] of the library's memory, and blocks used."""
+        k = ctypes.c_void_p()
+        v = ctypes.c_void_p()
+        used = ctypes.c_int32()
+        cap = ctypes.c_int32()
+        _check(lib().attuner_pool_info(self.handle, ctypes.byref(k), ctypes.byref(v), ctypes.byref(used),
+                                       ctypes.byref(cap)))
+        shape = (cap.value, self.cfg.n_kv_heads, BLOCK_TOKENS, self.cfg.head_dim)
+        return _wrap(k.value, shape, self.device), _wrap(v.value, shape, self.device), used.value
+
+    def sync_status(self, stream=None) -> int:
+        """Synchronise and return the device status (0 = OK) without raising."""
+        return lib().attuner_sync_status(self.handle, _stream(stream))
+
+    def set_option(self, option: int, value: int):
+        _check(lib().attuner_set_option(self.handle, option, int(value)))
+
+    def last_launch_count(self) -> int:
+        return lib().attuner_last_launch_count(self.handle)
+
+
+def _wrap(ptr: int, shape, device) -> torch.Tensor:
+    """A non-owning torch view of library-owned bf16 device memory."""
+    n = 1
+    for s in shape:
+        n *= s
+
+    class _Arr:
+        __cuda_array_interface__ = {
+            "shape": (n,), "typestr": "<i2", "data": (ptr, False), "version": 3, "strides": None,
+        }
+
+    t = torch.as_tensor(_Arr(), device=device)
+    return t.view(torch.bfloat16).view(*shape)

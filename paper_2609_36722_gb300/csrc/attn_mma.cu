@@ -1,0 +1,391 @@
+// attn_mma.cu - K3: split-KV attention for few query rows per (request, KV
+// head), the decode step of Sec. 3 (generated tokens read the frozen
+// artifact KV plus the online KV through the adapted query) and, as a
+// second kernel for any S, the same attention as attn_tc.cu;
+// K4: the log-sum-exp merge of split-KV partial results.
+//
+// K3 is bound by HBM: every (request, KV head) streams its assembled K/V
+// once (4 KiB per token at Hkv = 8, d = 128).  One CTA owns 16 packed query
+// rows (token * G + head_in_group) of one request and KV head, and one
+// chunk of its virtual block list.  Warp 4 streams 64-token K/V blocks with
+// TMA (128-byte swizzle) into a 4-stage ring; warps 0..3 each take 16 of the
+// 64 keys of every block (intra-CTA split over keys), run QK^T and PV with
+// m16n8k16 warp MMAs (tensor work is ~5% of the memory time here), keep an
+// online softmax in registers, and merge their partial results through
+// shared memory at the end.
+#include <math.h>
+
+#include "kernels.h"
+
+namespace att {
+
+template <int D>
+struct MmaLayout {
+  static constexpr int NH = D / 64;
+  static constexpr int NS = 4;
+  static constexpr int BLK = kBlockTokens * 128;      // one 64-row x 128 B box
+  static constexpr int STAGE = 2 * NH * BLK;          // K halves then V halves
+  static constexpr int BAR_OFF = NS * STAGE;
+  static constexpr int LIST_OFF = BAR_OFF + 256;
+  static constexpr int MERGE_BYTES = 4 * 16 * (D + 2) * 4;   // per warp: O[16][D], m[16], l[16]
+  static constexpr int SMEM = LIST_OFF + kMaxChunkBlocks * 4 + 1024;
+  static_assert(MERGE_BYTES <= BAR_OFF, "merge area aliases the stage ring");
+};
+
+template <int D>
+__global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ AttnParams p) {
+  using L = MmaLayout<D>;
+  constexpr int NT = D / 8;           // n8 tiles of the output
+  constexpr int KS = D / 16;          // k16 steps of QK^T
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t sbase = smem_u32(smem);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);   // full[NS], empty[NS], never
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 8 * (2 * L::NS + 1));
+  int* list = reinterpret_cast<int*>(smem + L::LIST_OFF);
+  auto bar = [&](int i) { return smem_u32(&bars[i]); };
+  const int B_FULL = 0, B_EMPTY = L::NS, B_NEVER = 2 * L::NS;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int G = p.G;
+  const int cta = blockIdx.x;
+  const int req = find_req(p.work, cta);
+  int rel = cta - p.work.base[req];
+  const int rt = rel % p.work.row_tiles;
+  rel /= p.work.row_tiles;
+  const int kvh = rel % p.Hkv;
+  const int split = rel / p.Hkv;
+  const int nsplit = p.work.nsplit[req];
+  const int boff = p.plan.blk_off[req];
+  const int nab = p.plan.blk_off[req + 1] - boff;
+  const int nsuf = (p.S_kv + kBlockTokens - 1) / kBlockTokens;
+  const int row0 = rt * kMmaRows;
+  const int last_row = min(row0 + kMmaRows - 1, p.S * G - 1);
+  const int last_vis = nab + ((p.S_kv - p.S) + last_row / G) / kBlockTokens;
+  const int b0 = split * p.work.chunk_blocks;
+  const int b1 = min(min(b0 + p.work.chunk_blocks, nab + nsuf), last_vis + 1);
+  const int nblk = max(0, b1 - b0);
+
+  for (int i = threadIdx.x; i < nblk; i += blockDim.x) {
+    const int b = b0 + i;
+    int e;
+    if (b < nab) {
+      e = p.plan.blocks[boff + b];
+      const int blk = e >> 7, valid = e & 127;
+      if (blk < 0 || blk >= p.plan.pool_blocks || valid < 1 || valid > kBlockTokens) {
+        set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
+        e = 0;
+      }
+    } else {
+      e = -(b - nab + 1);
+    }
+    list[i] = e;
+  }
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < L::NS; ++i) {
+      mbar_init(bar(B_FULL + i), 1);
+      mbar_init(bar(B_EMPTY + i), 4);
+    }
+    mbar_init(bar(B_NEVER), 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  if (warp == 4) {
+    // ================= TMA producer =================
+    if (lane == 0) {
+      const int pool_rows = p.plan.pool_blocks * p.Hkv * kBlockTokens;
+      int issued = 0;
+      for (int j = 0; j < nblk; ++j) {
+        const int st = j % L::NS;
+        if (j >= L::NS &&
+            !mbar_wait(bar(B_EMPTY + st), ((j / L::NS) - 1) & 1, abort_flag, p.wait_limit, p.status))
+          break;
+        const uint32_t dst = sbase + st * L::STAGE;
+        const uint32_t fb = bar(B_FULL + st);
+        mbar_expect_tx(fb, L::STAGE);
+        const int e = list[j];
+#pragma unroll
+        for (int h = 0; h < L::NH; ++h) {
+          if (e < 0) {
+            const int c = (-e - 1) * kBlockTokens;
+            tma_load_4d(dst + h * L::BLK, &p.tm_ksuf, fb, h * 64, kvh, c, req);
+            tma_load_4d(dst + (L::NH + h) * L::BLK, &p.tm_vsuf, fb, h * 64, kvh, c, req);
+          } else {
+            const int row = (e == 0) ? pool_rows : ((e >> 7) * p.Hkv + kvh) * kBlockTokens;
+            tma_load_2d(dst + h * L::BLK, &p.tm_kpool, fb, h * 64, row);
+            tma_load_2d(dst + (L::NH + h) * L::BLK, &p.tm_vpool, fb, h * 64, row);
+          }
+        }
+        issued = j + 1;
+      }
+      if (*abort_flag) {
+        for (int j = (issued > L::NS ? issued - L::NS : 0); j < issued; ++j)
+          mbar_drain(bar(B_FULL + j % L::NS), (j / L::NS) & 1, p.status);
+      }
+    }
+    return;   // the producer takes no part in the merge below
+  }
+
+  // ================= consumers: warps 0..3 =================
+  const int g = lane >> 2, t = lane & 3;
+  // Q fragments of rows g and g+8 (A operand of m16n8k16, row-major)
+  uint32_t qa[KS][4];
+  int tok_r[2];
+  long long qrow[2];
+#pragma unroll
+  for (int hr = 0; hr < 2; ++hr) {
+    const int pr = row0 + g + 8 * hr;
+    tok_r[hr] = pr / G;
+    qrow[hr] = (tok_r[hr] < p.S) ? (((long long)req * p.S + tok_r[hr]) * p.Hq + kvh * G + pr % G) : -1;
+  }
+#pragma unroll
+  for (int ks = 0; ks < KS; ++ks) {
+#pragma unroll
+    for (int hr = 0; hr < 2; ++hr) {
+#pragma unroll
+      for (int kh = 0; kh < 2; ++kh) {
+        uint32_t v = 0;
+        if (qrow[hr] >= 0)
+          v = *reinterpret_cast<const uint32_t*>(p.q + qrow[hr] * D + ks * 16 + kh * 8 + 2 * t);
+        qa[ks][hr + 2 * kh] = v;
+      }
+    }
+  }
+  const int lim0 = (p.S_kv - p.S) + tok_r[0];
+  const int lim1 = (p.S_kv - p.S) + tok_r[1];
+
+  float o[NT][4];
+#pragma unroll
+  for (int n = 0; n < NT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+  float m_r[2] = {-INFINITY, -INFINITY}, l_r[2] = {0.f, 0.f};
+  bool ok = true;
+  if (p.inject_stuck && warp == 0)
+    ok = warp_wait(bar(B_NEVER), 0, abort_flag, p.wait_limit, p.status);   // nothing arrives: times out
+
+  for (int j = 0; ok && j < nblk; ++j) {
+    const int st = j % L::NS;
+    if (!warp_wait(bar(B_FULL + st), (j / L::NS) & 1, abort_flag, p.wait_limit, p.status)) { ok = false; break; }
+    const uint32_t ks_base = sbase + st * L::STAGE;
+    const uint32_t vs_base = ks_base + L::NH * L::BLK;
+    // ---- S = Q K^T for keys 16*warp .. +15 (two n8 tiles)
+    float s[2][4];
+#pragma unroll
+    for (int n = 0; n < 2; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
+    {
+      const int mi = lane >> 3, ri = lane & 7;
+      const int key = 16 * warp + 8 * (mi >> 1) + ri;
+#pragma unroll
+      for (int ks = 0; ks < KS; ++ks) {
+        const int chunk = 2 * ks + (mi & 1);
+        uint32_t b0r, b1r, b2r, b3r;
+        ldmatrix_x4(ks_base + (chunk >> 3) * L::BLK + sw128_off(key, chunk & 7), b0r, b1r, b2r, b3r);
+        mma_16816(s[0], qa[ks], b0r, b1r);
+        mma_16816(s[1], qa[ks], b2r, b3r);
+      }
+    }
+    // ---- mask
+    const int e = list[j];
+#pragma unroll
+    for (int n = 0; n < 2; ++n) {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int kb = 16 * warp + 8 * n + 2 * t + (c & 1);
+        bool vis;
+        if (e > 0) vis = kb < (e & 127);
+        else if (e < 0) vis = ((-e - 1) * kBlockTokens + kb) <= ((c < 2) ? lim0 : lim1);
+        else vis = false;
+        if (!vis) s[n][c] = -INFINITY;
+      }
+    }
+    // ---- online softmax (rows g: c = 0,1; row g+8: c = 2,3)
+    float alpha[2];
+#pragma unroll
+    for (int hr = 0; hr < 2; ++hr) {
+      float mx = fmaxf(fmaxf(s[0][2 * hr], s[0][2 * hr + 1]), fmaxf(s[1][2 * hr], s[1][2 * hr + 1]));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      mx *= p.scale_log2;
+      const float m_new = fmaxf(m_r[hr], mx);
+      const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
+      alpha[hr] = ex2(m_r[hr] - m_use);
+      m_r[hr] = m_new;
+      float rs = 0.f;
+#pragma unroll
+      for (int n = 0; n < 2; ++n) {
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const float pv = ex2(fmaf(s[n][2 * hr + c], p.scale_log2, -m_use));
+          s[n][2 * hr + c] = pv;
+          rs += pv;
+        }
+      }
+      l_r[hr] = l_r[hr] * alpha[hr] + rs;
+    }
+#pragma unroll
+    for (int n = 0; n < NT; ++n) {
+      o[n][0] *= alpha[0]; o[n][1] *= alpha[0];
+      o[n][2] *= alpha[1]; o[n][3] *= alpha[1];
+    }
+    // ---- O += P V (A = P from the S fragments; B = V via ldmatrix.trans)
+    uint32_t pa[4];
+    pa[0] = pack_bf16(s[0][0], s[0][1]);
+    pa[1] = pack_bf16(s[0][2], s[0][3]);
+    pa[2] = pack_bf16(s[1][0], s[1][1]);
+    pa[3] = pack_bf16(s[1][2], s[1][3]);
+    {
+      const int mi = lane >> 3, ri = lane & 7;
+      const int key = 16 * warp + ri + 8 * (mi & 1);
+#pragma unroll
+      for (int np = 0; np < NT / 2; ++np) {
+        const int chunk = 2 * np + (mi >> 1);
+        uint32_t b0r, b1r, b2r, b3r;
+        ldmatrix_x4_trans(vs_base + (chunk >> 3) * L::BLK + sw128_off(key, chunk & 7), b0r, b1r, b2r, b3r);
+        mma_16816(o[2 * np], pa, b0r, b1r);
+        mma_16816(o[2 * np + 1], pa, b2r, b3r);
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar(B_EMPTY + st));
+  }
+
+  // ---- merge the four warps (the stage ring is reused once every warp is done)
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+  if (*abort_flag) return;
+#pragma unroll
+  for (int hr = 0; hr < 2; ++hr) {
+    l_r[hr] += __shfl_xor_sync(0xffffffffu, l_r[hr], 1);
+    l_r[hr] += __shfl_xor_sync(0xffffffffu, l_r[hr], 2);
+  }
+  float* mo = reinterpret_cast<float*>(smem) + warp * 16 * (D + 2);
+#pragma unroll
+  for (int n = 0; n < NT; ++n) {
+    *reinterpret_cast<float2*>(mo + g * (D + 2) + 8 * n + 2 * t) = make_float2(o[n][0], o[n][1]);
+    *reinterpret_cast<float2*>(mo + (g + 8) * (D + 2) + 8 * n + 2 * t) = make_float2(o[n][2], o[n][3]);
+  }
+  if (t == 0) {
+    mo[g * (D + 2) + D] = m_r[0];
+    mo[g * (D + 2) + D + 1] = l_r[0];
+    mo[(g + 8) * (D + 2) + D] = m_r[1];
+    mo[(g + 8) * (D + 2) + D + 1] = l_r[1];
+  }
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+  const float* mb = reinterpret_cast<const float*>(smem);
+  const int tid = threadIdx.x;
+  constexpr int CPT = D / 8;                    // columns per thread: 16 rows x 8 threads
+  const int row = tid >> 3, c0 = (tid & 7) * CPT;
+  float mw[4], lw[4];
+  float M = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    mw[w] = mb[(w * 16 + row) * (D + 2) + D];
+    lw[w] = mb[(w * 16 + row) * (D + 2) + D + 1];
+    M = fmaxf(M, mw[w]);
+  }
+  const float Mu = (M == -INFINITY) ? 0.f : M;
+  float wsum = 0.f, wt[4];
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    wt[w] = ex2(mw[w] - Mu);
+    wsum += wt[w] * lw[w];
+  }
+  const float inv = (wsum > 0.f) ? 1.f / wsum : 0.f;
+  const float lse = (wsum > 0.f) ? (Mu + log2f(wsum)) * 0.69314718055994531f : -INFINITY;
+  const int pr = row0 + row;
+  const int tok = pr / G;
+  if (tok >= p.S) return;
+  float acc[CPT];
+#pragma unroll
+  for (int c = 0; c < CPT; ++c) {
+    float a = 0.f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) a += wt[w] * mb[(w * 16 + row) * (D + 2) + c0 + c];
+    acc[c] = a * inv;
+  }
+  if (nsplit > 1) {
+    float* po = p.part_o + ((long long)cta * kMmaRows + row) * D + c0;
+#pragma unroll
+    for (int c = 0; c < CPT; c += 4) *reinterpret_cast<float4*>(po + c) = make_float4(acc[c], acc[c + 1], acc[c + 2], acc[c + 3]);
+    if ((tid & 7) == 0) p.part_lse[(long long)cta * kMmaRows + row] = lse;
+  } else {
+    const long long orow = ((long long)req * p.S + tok) * p.Hq + kvh * G + pr % G;
+    uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D + c0);
+#pragma unroll
+    for (int c = 0; c < CPT; c += 8)
+      dst[c / 8] = make_uint4(pack_bf16(acc[c], acc[c + 1]), pack_bf16(acc[c + 2], acc[c + 3]),
+                              pack_bf16(acc[c + 4], acc[c + 5]), pack_bf16(acc[c + 6], acc[c + 7]));
+    if ((tid & 7) == 0 && p.lse_out) p.lse_out[orow] = lse;
+  }
+}
+
+template <int D>
+static cudaError_t launch_attn_mma_t(const AttnParams& p, cudaStream_t st) {
+  using L = MmaLayout<D>;
+  cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
+  if (e != cudaSuccess) return e;
+  attn_mma_kernel<D><<<p.work.n_cta, 160, L::SMEM, st>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st) {
+  if (D == 128) return launch_attn_mma_t<128>(p, st);
+  if (D == 64) return launch_attn_mma_t<64>(p, st);
+  return cudaErrorInvalidValue;
+}
+
+// ---------------------------------------------------------------------------
+// K4: merge split-KV partials: lse = log sum_s exp(lse_s),
+// O = sum_s exp(lse_s - lse) O_s.  One warp per output row.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ CombineParams p,
+                                                      long long total_rows) {
+  const long long gw = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (gw >= total_rows) return;
+  const int R = p.rows_per_tile;
+  const long long per_req = (long long)p.Hkv * p.work.row_tiles * R;
+  const int req = (int)(gw / per_req);
+  long long rem = gw % per_req;
+  const int r = (int)(rem % R);
+  rem /= R;
+  const int rt = (int)(rem % p.work.row_tiles);
+  const int kvh = (int)(rem / p.work.row_tiles);
+  const int ns = p.work.nsplit[req];
+  if (ns <= 1) return;
+  const int pr = rt * R + r;
+  const int tok = pr / p.G;
+  if (tok >= p.S) return;
+  float M = -INFINITY;
+  for (int s = 0; s < ns; ++s) {
+    const long long c = p.work.base[req] + ((long long)s * p.Hkv + kvh) * p.work.row_tiles + rt;
+    M = fmaxf(M, p.part_lse[c * R + r]);
+  }
+  float W = 0.f;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  const int cpl = p.D / 32;   // columns per lane (2 or 4)
+  for (int s = 0; s < ns; ++s) {
+    const long long c = p.work.base[req] + ((long long)s * p.Hkv + kvh) * p.work.row_tiles + rt;
+    const float ls = p.part_lse[c * R + r];
+    if (ls == -INFINITY) continue;
+    const float w = __expf(ls - M);
+    W += w;
+    const float* po = p.part_o + (c * R + r) * p.D + lane * cpl;
+    for (int k = 0; k < cpl; ++k) acc[k] += w * po[k];
+  }
+  const float inv = (W > 0.f) ? 1.f / W : 0.f;
+  const long long orow = ((long long)req * p.S + tok) * p.Hq + kvh * p.G + pr % p.G;
+  __nv_bfloat16* dst = p.out + orow * p.D + lane * cpl;
+  for (int k = 0; k < cpl; ++k) dst[k] = __float2bfloat16_rn(acc[k] * inv);
+  if (lane == 0 && p.lse_out) p.lse_out[orow] = (W > 0.f) ? M + logf(W) : -INFINITY;
+}
+
+cudaError_t launch_combine(const CombineParams& p, cudaStream_t st) {
+  const long long total_rows = (long long)p.work.n_req * p.Hkv * p.work.row_tiles * p.rows_per_tile;
+  const long long threads = total_rows * 32;
+  const int grid = (int)((threads + 255) / 256);
+  combine_kernel<<<grid, 256, 0, st>>>(p, total_rows);
+  return cudaGetLastError();
+}
+
+}  // namespace att

@@ -1,0 +1,719 @@
+// capi.cu - the C ABI of libattuner (declared in include/attuner.h):
+// context and paged pool, artifact registration (bump allocation in
+// registration order), request assembly into block tables and index maps,
+// tensor-map encoding, split-KV work decomposition and kernel dispatch.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "kernels.h"
+
+using namespace att;
+
+// ---------------------------------------------------------------------------
+// errors
+// ---------------------------------------------------------------------------
+static thread_local std::string g_err;
+
+static attuner_status fail(attuner_status s, const std::string& msg) {
+  g_err = msg;
+  return s;
+}
+
+#define CUDA_TRY(call)                                                                        \
+  do {                                                                                        \
+    cudaError_t e_ = (call);                                                                  \
+    if (e_ != cudaSuccess)                                                                    \
+      return fail(ATTUNER_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_));      \
+  } while (0)
+
+#define CHECK_ARG(cond, msg)                                  \
+  do {                                                        \
+    if (!(cond)) return fail(ATTUNER_ERR_INVALID_ARG, msg);   \
+  } while (0)
+
+// ---------------------------------------------------------------------------
+// objects
+// ---------------------------------------------------------------------------
+struct Artifact {
+  int32_t first_block;
+  int32_t L;
+  int32_t n_blocks;
+};
+
+struct attuner_ctx {
+  attuner_config cfg{};
+  __nv_bfloat16* kpool = nullptr;
+  __nv_bfloat16* vpool = nullptr;
+  int32_t used_blocks = 0;
+  std::vector<Artifact> arts;
+  CUtensorMap tm_kpool{}, tm_vpool{};
+  int* d_status = nullptr;
+  cudaMemPool_t mempool = nullptr;
+  int num_sms = 0;
+  int opt_prefill = 0;
+  int opt_split = 0;
+  long long wait_limit = 1ll << 32;
+  int inject_stuck = 0;
+  int last_launches = 0;
+};
+
+struct attuner_plan {
+  int32_t n_req = 0;
+  int32_t device = 0;
+  int32_t pool_blocks = 0;
+  std::vector<int32_t> req_off;   // CSR over artifact ids
+  std::vector<int32_t> art_ids;
+  std::vector<int32_t> blk_off;   // CSR over blocks
+  std::vector<int32_t> blocks;    // (pool block << 7) | valid
+  std::vector<int32_t> t_art;
+  std::vector<Artifact> arts;     // snapshot of the registry entries used
+  int32_t* d_buf = nullptr;       // blk_off | blocks | t_art
+};
+
+// ---------------------------------------------------------------------------
+// driver entry point for tensor maps (no link-time dependency on libcuda)
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// bf16 tensor map, 128-byte swizzle, zero fill out of bounds.
+// dims[0] is the innermost (contiguous) dimension; strides[i] is the byte
+// stride of dims[i+1].
+static attuner_status make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
+                               const uint64_t* strides, const uint32_t* box, const char* what) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return fail(ATTUNER_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  if ((reinterpret_cast<uintptr_t>(base) & 15) != 0)
+    return fail(ATTUNER_ERR_INVALID_ARG, std::string(what) + ": base address must be 16-byte aligned");
+  cuuint64_t d[5];
+  cuuint64_t s[4];
+  cuuint32_t b[5], e[5];
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    b[i] = box[i];
+    e[i] = 1;
+    if (i + 1 < rank) s[i] = strides[i];
+  }
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base), d, s, b, e,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return fail(ATTUNER_ERR_CUDA, std::string("cuTensorMapEncodeTiled failed for ") + what +
+                                      " (CUresult " + std::to_string((int)r) + ")");
+  return ATTUNER_OK;
+}
+
+static attuner_status set_device(const attuner_ctx* ctx) {
+  int cur = -1;
+  CUDA_TRY(cudaGetDevice(&cur));
+  if (cur != ctx->cfg.device) CUDA_TRY(cudaSetDevice(ctx->cfg.device));
+  return ATTUNER_OK;
+}
+
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// stream-ordered scratch of one call
+struct Scratch {
+  attuner_ctx* ctx;
+  cudaStream_t st;
+  void* base = nullptr;
+  size_t used = 0, cap = 0;
+  size_t take(size_t bytes) {
+    size_t off = used;
+    used += (bytes + 255) & ~size_t(255);
+    return off;
+  }
+};
+
+// ---------------------------------------------------------------------------
+// context
+// ---------------------------------------------------------------------------
+extern "C" attuner_status attuner_create(const attuner_config* cfg, attuner_ctx** out) {
+  CHECK_ARG(cfg != nullptr && out != nullptr, "attuner_create: cfg and out must not be NULL");
+  *out = nullptr;
+  CHECK_ARG(cfg->head_dim == 64 || cfg->head_dim == 128, "head_dim must be 64 or 128");
+  CHECK_ARG(cfg->n_kv_heads >= 1 && cfg->n_q_heads >= 1 && cfg->n_q_heads % cfg->n_kv_heads == 0,
+            "n_q_heads must be a positive multiple of n_kv_heads");
+  const int G = cfg->n_q_heads / cfg->n_kv_heads;
+  CHECK_ARG(G == 1 || G == 2 || G == 4 || G == 8, "group size n_q_heads / n_kv_heads must be 1, 2, 4 or 8");
+  CHECK_ARG(cfg->hidden >= 64 && cfg->hidden % 64 == 0, "hidden must be a positive multiple of 64");
+  CHECK_ARG(cfg->block_tokens == ATTUNER_BLOCK_TOKENS, "block_tokens must be 64");
+  CHECK_ARG(cfg->pool_blocks >= 1, "pool_blocks must be >= 1");
+  CHECK_ARG((long long)cfg->pool_blocks * cfg->n_kv_heads * 64 < (1ll << 31),
+            "pool too large: pool_blocks * n_kv_heads * 64 must be < 2^31");
+  CHECK_ARG(cfg->pool_blocks < (1 << 24), "pool_blocks must be < 2^24");
+  CHECK_ARG(cfg->rope_theta > 1.0f && cfg->rms_eps >= 0.0f, "rope_theta must be > 1 and rms_eps >= 0");
+  int ndev = 0;
+  CUDA_TRY(cudaGetDeviceCount(&ndev));
+  CHECK_ARG(cfg->device >= 0 && cfg->device < ndev, "device ordinal out of range");
+
+  attuner_ctx* ctx = new attuner_ctx();
+  ctx->cfg = *cfg;
+  attuner_status st = set_device(ctx);
+  if (st != ATTUNER_OK) { delete ctx; return st; }
+  const size_t pool_bytes = (size_t)cfg->pool_blocks * cfg->n_kv_heads * 64 * cfg->head_dim * 2;
+  cudaError_t e1 = cudaMalloc(&ctx->kpool, pool_bytes);
+  cudaError_t e2 = (e1 == cudaSuccess) ? cudaMalloc(&ctx->vpool, pool_bytes) : e1;
+  cudaError_t e3 = (e2 == cudaSuccess) ? cudaMalloc(&ctx->d_status, sizeof(int)) : e2;
+  if (e3 != cudaSuccess) {
+    attuner_destroy(ctx);
+    cudaGetLastError();
+    return fail(ATTUNER_ERR_OOM, std::string("pool allocation failed: ") + cudaGetErrorString(e3));
+  }
+  if (cudaMemset(ctx->kpool, 0, pool_bytes) != cudaSuccess || cudaMemset(ctx->vpool, 0, pool_bytes) != cudaSuccess ||
+      cudaMemset(ctx->d_status, 0, sizeof(int)) != cudaSuccess ||
+      cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, cfg->device) != cudaSuccess) {
+    attuner_destroy(ctx);
+    return fail(ATTUNER_ERR_CUDA, "context initialisation failed");
+  }
+  cudaMemPoolProps props{};
+  props.allocType = cudaMemAllocationTypePinned;
+  props.location.type = cudaMemLocationTypeDevice;
+  props.location.id = cfg->device;
+  if (cudaMemPoolCreate(&ctx->mempool, &props) != cudaSuccess) {
+    attuner_destroy(ctx);
+    return fail(ATTUNER_ERR_CUDA, "cudaMemPoolCreate failed");
+  }
+  uint64_t thresh = ~0ull;
+  cudaMemPoolSetAttribute(ctx->mempool, cudaMemPoolAttrReleaseThreshold, &thresh);
+
+  const uint64_t D = cfg->head_dim;
+  const uint64_t rows = (uint64_t)cfg->pool_blocks * cfg->n_kv_heads * 64;
+  const uint64_t dims[2] = {D, rows};
+  const uint64_t strides[1] = {D * 2};
+  const uint32_t box[2] = {64, 64};
+  st = make_map(&ctx->tm_kpool, ctx->kpool, 2, dims, strides, box, "K pool");
+  if (st == ATTUNER_OK) st = make_map(&ctx->tm_vpool, ctx->vpool, 2, dims, strides, box, "V pool");
+  if (st != ATTUNER_OK) {
+    attuner_destroy(ctx);
+    return st;
+  }
+  *out = ctx;
+  return ATTUNER_OK;
+}
+
+extern "C" attuner_status attuner_destroy(attuner_ctx* ctx) {
+  if (!ctx) return ATTUNER_OK;
+  set_device(ctx);
+  if (ctx->kpool) cudaFree(ctx->kpool);
+  if (ctx->vpool) cudaFree(ctx->vpool);
+  if (ctx->d_status) cudaFree(ctx->d_status);
+  if (ctx->mempool) cudaMemPoolDestroy(ctx->mempool);
+  delete ctx;
+  return ATTUNER_OK;
+}
+
+extern "C" attuner_status attuner_register_artifact(attuner_ctx* ctx, const void* k, const void* v,
+                                                    int32_t L, void* stream, int32_t* artifact_id_out) {
+  CHECK_ARG(ctx != nullptr, "ctx must not be NULL");
+  CHECK_ARG(k != nullptr && v != nullptr, "k and v must not be NULL");
+  CHECK_ARG(L > 0, "artifact length L must be > 0");
+  CHECK_ARG(aligned16(k) && aligned16(v), "k and v must be 16-byte aligned");
+  const int nb = (L + 63) / 64;
+  if ((long long)ctx->used_blocks + nb > ctx->cfg.pool_blocks)
+    return fail(ATTUNER_ERR_OOM, "artifact pool is full: " + std::to_string(ctx->used_blocks) + " of " +
+                                     std::to_string(ctx->cfg.pool_blocks) + " blocks used, " +
+                                     std::to_string(nb) + " more needed");
+  attuner_status s = set_device(ctx);
+  if (s != ATTUNER_OK) return s;
+  CUDA_TRY(launch_pool_write(static_cast<const __nv_bfloat16*>(k), static_cast<const __nv_bfloat16*>(v),
+                             ctx->kpool, ctx->vpool, L, ctx->cfg.n_kv_heads, ctx->cfg.head_dim,
+                             ctx->used_blocks, static_cast<cudaStream_t>(stream)));
+  ctx->arts.push_back(Artifact{ctx->used_blocks, L, nb});
+  ctx->used_blocks += nb;
+  if (artifact_id_out) *artifact_id_out = (int32_t)ctx->arts.size() - 1;
+  ctx->last_launches = 1;
+  return ATTUNER_OK;
+}
+
+// ---------------------------------------------------------------------------
+// plans
+// ---------------------------------------------------------------------------
+extern "C" attuner_status attuner_assemble(attuner_ctx* ctx, const int32_t* ids, const int32_t* offs,
+                                           int32_t n_req, attuner_plan** out) {
+  CHECK_ARG(ctx != nullptr && out != nullptr, "ctx and out must not be NULL");
+  *out = nullptr;
+  CHECK_ARG(n_req >= 1 && n_req <= kMaxReq, "n_req must be in [1, " + std::to_string(kMaxReq) + "]");
+  CHECK_ARG(offs != nullptr, "req_offsets_host must not be NULL");
+  CHECK_ARG(offs[0] == 0, "req_offsets_host[0] must be 0");
+  for (int i = 0; i < n_req; ++i) CHECK_ARG(offs[i + 1] >= offs[i], "req_offsets_host must be non-decreasing");
+  CHECK_ARG(offs[n_req] == 0 || ids != nullptr, "artifact_ids_host must not be NULL");
+  attuner_plan* p = new attuner_plan();
+  p->n_req = n_req;
+  p->device = ctx->cfg.device;
+  p->pool_blocks = ctx->cfg.pool_blocks;
+  p->req_off.assign(offs, offs + n_req + 1);
+  p->art_ids.assign(ids, ids + offs[n_req]);
+  p->blk_off.push_back(0);
+  for (int r = 0; r < n_req; ++r) {
+    long long t = 0;
+    for (int i = offs[r]; i < offs[r + 1]; ++i) {
+      const int a = ids[i];
+      if (a < 0 || a >= (int)ctx->arts.size()) {
+        delete p;
+        return fail(ATTUNER_ERR_UNKNOWN_ARTIFACT, "artifact id " + std::to_string(a) + " was never registered");
+      }
+      const Artifact& A = ctx->arts[a];
+      for (int b = 0; b < A.n_blocks; ++b)
+        p->blocks.push_back(((A.first_block + b) << 7) | std::min(64, A.L - 64 * b));
+      t += A.L;
+    }
+    if (t >= (1ll << 30)) {
+      delete p;
+      return fail(ATTUNER_ERR_INVALID_ARG, "assembled length of a request must be < 2^30 tokens");
+    }
+    p->blk_off.push_back((int32_t)p->blocks.size());
+    p->t_art.push_back((int32_t)t);
+  }
+  p->arts = ctx->arts;
+  attuner_status s = set_device(ctx);
+  if (s != ATTUNER_OK) { delete p; return s; }
+  const size_t n = p->blk_off.size() + p->blocks.size() + p->t_art.size();
+  std::vector<int32_t> h;
+  h.reserve(n);
+  h.insert(h.end(), p->blk_off.begin(), p->blk_off.end());
+  h.insert(h.end(), p->blocks.begin(), p->blocks.end());
+  h.insert(h.end(), p->t_art.begin(), p->t_art.end());
+  if (cudaMalloc(&p->d_buf, n * sizeof(int32_t)) != cudaSuccess) {
+    cudaGetLastError();
+    delete p;
+    return fail(ATTUNER_ERR_OOM, "plan allocation failed");
+  }
+  if (cudaMemcpy(p->d_buf, h.data(), n * sizeof(int32_t), cudaMemcpyHostToDevice) != cudaSuccess) {
+    cudaFree(p->d_buf);
+    delete p;
+    return fail(ATTUNER_ERR_CUDA, "plan upload failed");
+  }
+  *out = p;
+  return ATTUNER_OK;
+}
+
+extern "C" attuner_status attuner_plan_export(const attuner_plan* p, int32_t* block_table, int32_t* valid_len,
+                                              int32_t* index_map, int32_t* token_art, int32_t* token_off,
+                                              int64_t* sizes) {
+  CHECK_ARG(p != nullptr && sizes != nullptr, "plan and sizes_inout must not be NULL");
+  const int64_t nb = (int64_t)p->blocks.size();
+  int64_t nt = 0;
+  for (int32_t t : p->t_art) nt += t;
+  CHECK_ARG(!block_table || sizes[0] >= nb, "block_table capacity too small");
+  CHECK_ARG(!valid_len || sizes[1] >= nb, "valid_len capacity too small");
+  CHECK_ARG(!index_map || sizes[2] >= nt, "index_map capacity too small");
+  CHECK_ARG(!token_art || sizes[3] >= nt, "token_art capacity too small");
+  CHECK_ARG(!token_off || sizes[4] >= nt, "token_off capacity too small");
+  for (int64_t i = 0; i < nb; ++i) {
+    if (block_table) block_table[i] = p->blocks[i] >> 7;
+    if (valid_len) valid_len[i] = p->blocks[i] & 127;
+  }
+  int64_t t = 0;
+  for (int r = 0; r < p->n_req; ++r) {
+    for (int i = p->req_off[r]; i < p->req_off[r + 1]; ++i) {
+      const int a = p->art_ids[i];
+      const Artifact& A = p->arts[a];
+      for (int q = 0; q < A.L; ++q, ++t) {
+        if (index_map) index_map[t] = (A.first_block + q / 64) * 64 + q % 64;
+        if (token_art) token_art[t] = a;
+        if (token_off) token_off[t] = q;
+      }
+    }
+  }
+  sizes[0] = nb;
+  sizes[1] = nb;
+  sizes[2] = nt;
+  sizes[3] = nt;
+  sizes[4] = nt;
+  sizes[5] = p->n_req;
+  return ATTUNER_OK;
+}
+
+extern "C" attuner_status attuner_plan_t_art(const attuner_plan* p, int32_t* t_art, int32_t n_req) {
+  CHECK_ARG(p != nullptr && t_art != nullptr, "plan and t_art_host must not be NULL");
+  CHECK_ARG(n_req == p->n_req, "n_req does not match the plan");
+  for (int i = 0; i < n_req; ++i) t_art[i] = p->t_art[i];
+  return ATTUNER_OK;
+}
+
+extern "C" attuner_status attuner_plan_free(attuner_plan* p) {
+  if (!p) return ATTUNER_OK;
+  if (p->d_buf) {
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != p->device) cudaSetDevice(p->device);
+    cudaFree(p->d_buf);
+    if (cur != p->device && cur >= 0) cudaSetDevice(cur);
+  }
+  delete p;
+  return ATTUNER_OK;
+}
+
+static PlanDev plan_dev(const attuner_plan* p) {
+  PlanDev d;
+  d.blk_off = p->d_buf;
+  d.blocks = p->d_buf + p->blk_off.size();
+  d.t_art = p->d_buf + p->blk_off.size() + p->blocks.size();
+  d.pool_blocks = p->pool_blocks;
+  return d;
+}
+
+// ---------------------------------------------------------------------------
+// Q projection
+// ---------------------------------------------------------------------------
+static attuner_status check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv) {
+  CHECK_ARG(ctx != nullptr && plan != nullptr, "ctx and plan must not be NULL");
+  CHECK_ARG(plan->device == ctx->cfg.device && plan->pool_blocks == ctx->cfg.pool_blocks,
+            "plan belongs to another context");
+  CHECK_ARG(S >= 1 && S_kv >= S, "need 1 <= S <= S_kv");
+  CHECK_ARG((long long)plan->n_req * S * ctx->cfg.n_q_heads < (1ll << 31) && S_kv < (1 << 30),
+            "n_req * S * n_q_heads must be < 2^31");
+  return ATTUNER_OK;
+}
+
+static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan, const void* x, const void* w_q,
+                                     const void* lora_a, const void* lora_b, int32_t r, float s,
+                                     const void* q_norm_w, int32_t S, int32_t S_kv, void* q_out,
+                                     cudaStream_t st, Scratch& sc, int& launches) {
+  const attuner_config& c = ctx->cfg;
+  CHECK_ARG(x && w_q && q_norm_w && q_out, "x, w_q, q_norm_w and q_out must not be NULL");
+  CHECK_ARG(aligned16(x) && aligned16(w_q) && aligned16(q_out) && aligned16(q_norm_w),
+            "x, w_q, q_norm_w and q_out must be 16-byte aligned");
+  const bool lora = (r > 0 && lora_a != nullptr && lora_b != nullptr);
+  CHECK_ARG(r >= 0 && r <= 64 && r % 8 == 0, "LoRA rank r must be 0 or a multiple of 8 up to 64");
+  if (lora) CHECK_ARG(aligned16(lora_a) && aligned16(lora_b), "lora_a and lora_b must be 16-byte aligned");
+  const int M = plan->n_req * S;
+  const int D = c.head_dim, Hq = c.n_q_heads, dq = Hq * D;
+  const size_t off_u = sc.take((size_t)M * 64 * 2);
+  const size_t off_b = sc.take((size_t)dq * 64 * 2);
+  const size_t off_rope = sc.take((size_t)M * (D / 2) * 8);
+  char* base = static_cast<char*>(sc.base);
+  __nv_bfloat16* u_pad = reinterpret_cast<__nv_bfloat16*>(base + off_u);
+  __nv_bfloat16* b_pad = reinterpret_cast<__nv_bfloat16*>(base + off_b);
+  float2* rope = reinterpret_cast<float2*>(base + off_rope);
+
+  PrepParams pp{};
+  pp.x = static_cast<const __nv_bfloat16*>(x);
+  pp.lora_a = lora ? static_cast<const __nv_bfloat16*>(lora_a) : nullptr;
+  pp.lora_b = lora ? static_cast<const __nv_bfloat16*>(lora_b) : nullptr;
+  pp.u_pad = u_pad;
+  pp.b_pad = b_pad;
+  pp.rope = rope;
+  pp.t_art = plan_dev(plan).t_art;
+  pp.M = M;
+  pp.hidden = c.hidden;
+  pp.r = lora ? r : 0;
+  pp.d_q = dq;
+  pp.D = D;
+  pp.S = S;
+  pp.S_kv = S_kv;
+  pp.s = s;
+  pp.theta = (double)c.rope_theta;
+  CUDA_TRY(launch_prep(pp, st));
+  ++launches;
+
+  QprojParams qp{};
+  attuner_status e;
+  {
+    const uint64_t dims[2] = {(uint64_t)c.hidden, (uint64_t)M};
+    const uint64_t strides[1] = {(uint64_t)c.hidden * 2};
+    const uint32_t box[2] = {64, 128};
+    if ((e = make_map(&qp.tm_x, x, 2, dims, strides, box, "x")) != ATTUNER_OK) return e;
+  }
+  {
+    const uint64_t dims[2] = {(uint64_t)c.hidden, (uint64_t)dq};
+    const uint64_t strides[1] = {(uint64_t)c.hidden * 2};
+    const uint32_t box[2] = {64, (uint32_t)D};
+    if ((e = make_map(&qp.tm_w, w_q, 2, dims, strides, box, "w_q")) != ATTUNER_OK) return e;
+  }
+  {
+    const uint64_t dims[2] = {64, (uint64_t)M};
+    const uint64_t strides[1] = {128};
+    const uint32_t box[2] = {64, 128};
+    if ((e = make_map(&qp.tm_u, u_pad, 2, dims, strides, box, "u")) != ATTUNER_OK) return e;
+  }
+  {
+    const uint64_t dims[2] = {64, (uint64_t)dq};
+    const uint64_t strides[1] = {128};
+    const uint32_t box[2] = {64, (uint32_t)D};
+    if ((e = make_map(&qp.tm_b, b_pad, 2, dims, strides, box, "B")) != ATTUNER_OK) return e;
+  }
+  qp.q_out = static_cast<__nv_bfloat16*>(q_out);
+  qp.qnorm_w = static_cast<const __nv_bfloat16*>(q_norm_w);
+  qp.rope = rope;
+  qp.M = M;
+  qp.hidden = c.hidden;
+  qp.Hq = Hq;
+  qp.lora_ksteps = lora ? (r + 15) / 16 : 0;
+  qp.eps = c.rms_eps;
+  qp.status = ctx->d_status;
+  qp.wait_limit = ctx->wait_limit;
+  CUDA_TRY(launch_qproj(qp, D, st));
+  ++launches;
+  return ATTUNER_OK;
+}
+
+static size_t q_project_scratch(const attuner_ctx* ctx, int M) {
+  const int D = ctx->cfg.head_dim, dq = ctx->cfg.n_q_heads * D;
+  auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
+  return al((size_t)M * 64 * 2) + al((size_t)dq * 64 * 2) + al((size_t)M * (D / 2) * 8);
+}
+
+// ---------------------------------------------------------------------------
+// attention
+// ---------------------------------------------------------------------------
+static void make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc,
+                      WorkTable& w) {
+  const int G = ctx->cfg.n_q_heads / ctx->cfg.n_kv_heads, Hkv = ctx->cfg.n_kv_heads;
+  const int rows = tc ? kTcRows : kMmaRows;
+  const int row_tiles = (S * G + rows - 1) / rows;
+  const int nsuf = (S_kv + 63) / 64;
+  long long total = 0;
+  int maxv = 0;
+  for (int r = 0; r < plan->n_req; ++r) {
+    const int nv = plan->blk_off[r + 1] - plan->blk_off[r] + nsuf;
+    total += (long long)nv * Hkv * row_tiles;
+    maxv = std::max(maxv, nv);
+  }
+  const long long units = (long long)plan->n_req * Hkv * row_tiles;
+  int chunk;
+  if (ctx->opt_split > 0) {
+    chunk = ctx->opt_split;
+  } else if (tc) {
+    // one CTA per SM: split only when the natural grid leaves SMs idle
+    const long long target = 2ll * ctx->num_sms;
+    chunk = (units >= target) ? maxv : (int)((total + target - 1) / target);
+    chunk = std::max(chunk, 8);
+  } else {
+    const long long target = 8ll * ctx->num_sms;
+    chunk = (int)std::max<long long>(16, (total + target - 1) / target);
+  }
+  chunk = std::min(chunk, kMaxChunkBlocks);
+  if (tc) chunk = (chunk + 1) & ~1;   // whole 128-key tiles per split
+  w.n_req = plan->n_req;
+  w.row_tiles = row_tiles;
+  w.chunk_blocks = chunk;
+  int base = 0;
+  for (int r = 0; r < plan->n_req; ++r) {
+    const int nv = plan->blk_off[r + 1] - plan->blk_off[r] + nsuf;
+    const int ns = (nv + chunk - 1) / chunk;
+    w.base[r] = base;
+    w.nsplit[r] = ns;
+    base += ns * Hkv * row_tiles;
+  }
+  w.n_cta = base;
+}
+
+static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
+                                  const void* suffix_k, const void* suffix_v, int32_t S, int32_t S_kv,
+                                  void* out, float* lse_out, cudaStream_t st, Scratch* sc_outer,
+                                  int& launches) {
+  const attuner_config& c = ctx->cfg;
+  CHECK_ARG(q && suffix_k && suffix_v && out, "q, suffix_k, suffix_v and out must not be NULL");
+  CHECK_ARG(aligned16(q) && aligned16(suffix_k) && aligned16(suffix_v) && aligned16(out),
+            "q, suffix_k, suffix_v and out must be 16-byte aligned");
+  const int D = c.head_dim, Hq = c.n_q_heads, Hkv = c.n_kv_heads, G = Hq / Hkv;
+  bool tc;
+  if (ctx->opt_prefill == 1) tc = true;
+  else if (ctx->opt_prefill == 2) tc = false;
+  else tc = (S * G > kMmaRows);
+  WorkTable* w = new WorkTable();
+  make_work(ctx, plan, S, S_kv, tc, *w);
+  bool need_combine = false;
+  for (int r = 0; r < plan->n_req; ++r) need_combine |= (w->nsplit[r] > 1);
+  const int rows = tc ? kTcRows : kMmaRows;
+
+  AttnParams* ap = new AttnParams();
+  attuner_status e = ATTUNER_OK;
+  auto done = [&](attuner_status s) { delete ap; delete w; return s; };
+  if (tc) {
+    const uint64_t dims[5] = {(uint64_t)D, (uint64_t)G, (uint64_t)Hkv, (uint64_t)S, (uint64_t)plan->n_req};
+    const uint64_t strides[4] = {(uint64_t)D * 2, (uint64_t)G * D * 2, (uint64_t)Hq * D * 2,
+                                 (uint64_t)S * Hq * D * 2};
+    const uint32_t box[5] = {64, (uint32_t)G, 1, (uint32_t)(kTcRows / G), 1};
+    if ((e = make_map(&ap->tm_q, q, 5, dims, strides, box, "q")) != ATTUNER_OK) return done(e);
+  }
+  {
+    const uint64_t dims[4] = {(uint64_t)D, (uint64_t)Hkv, (uint64_t)S_kv, (uint64_t)plan->n_req};
+    const uint64_t strides[3] = {(uint64_t)D * 2, (uint64_t)Hkv * D * 2, (uint64_t)S_kv * Hkv * D * 2};
+    const uint32_t box[4] = {64, 1, 64, 1};
+    if ((e = make_map(&ap->tm_ksuf, suffix_k, 4, dims, strides, box, "suffix_k")) != ATTUNER_OK) return done(e);
+    if ((e = make_map(&ap->tm_vsuf, suffix_v, 4, dims, strides, box, "suffix_v")) != ATTUNER_OK) return done(e);
+  }
+  ap->tm_kpool = ctx->tm_kpool;
+  ap->tm_vpool = ctx->tm_vpool;
+  ap->plan = plan_dev(plan);
+  ap->work = *w;
+  ap->q = static_cast<const __nv_bfloat16*>(q);
+  ap->out = static_cast<__nv_bfloat16*>(out);
+  ap->lse_out = lse_out;
+  ap->S = S;
+  ap->S_kv = S_kv;
+  ap->Hq = Hq;
+  ap->Hkv = Hkv;
+  ap->G = G;
+  ap->scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
+  ap->status = ctx->d_status;
+  ap->wait_limit = ctx->wait_limit;
+  ap->inject_stuck = ctx->inject_stuck;
+
+  Scratch local{ctx, st};
+  Scratch& sc = sc_outer ? *sc_outer : local;
+  void* part = nullptr;
+  size_t part_bytes = 0;
+  if (need_combine) {
+    part_bytes = (size_t)w->n_cta * rows * (D + 1) * 4;
+    if (cudaMallocFromPoolAsync(&part, part_bytes, ctx->mempool, st) != cudaSuccess) {
+      cudaGetLastError();
+      return done(fail(ATTUNER_ERR_OOM, "split-KV scratch allocation failed"));
+    }
+    ap->part_o = static_cast<float*>(part);
+    ap->part_lse = static_cast<float*>(part) + (size_t)w->n_cta * rows * D;
+  }
+  cudaError_t ce = tc ? launch_attn_tc(*ap, D, st) : launch_attn_mma(*ap, D, st);
+  if (ce == cudaSuccess) ++launches;
+  if (ce == cudaSuccess && need_combine) {
+    CombineParams cp{};
+    cp.work = *w;
+    cp.part_o = ap->part_o;
+    cp.part_lse = ap->part_lse;
+    cp.out = ap->out;
+    cp.lse_out = lse_out;
+    cp.S = S;
+    cp.Hq = Hq;
+    cp.Hkv = Hkv;
+    cp.G = G;
+    cp.D = D;
+    cp.rows_per_tile = rows;
+    ce = launch_combine(cp, st);
+    if (ce == cudaSuccess) ++launches;
+  }
+  if (part) cudaFreeAsync(part, st);
+  if (ce != cudaSuccess) return done(fail(ATTUNER_ERR_CUDA, std::string("attention launch failed: ") + cudaGetErrorString(ce)));
+  return done(ATTUNER_OK);
+}
+
+extern "C" attuner_status attuner_q_project(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
+                                            const void* w_q, const void* lora_a, const void* lora_b, int32_t r,
+                                            float s, const void* q_norm_w, int32_t S, int32_t S_kv, void* q_out,
+                                            void* stream) {
+  attuner_status e = check_common(ctx, plan, S, S_kv);
+  if (e != ATTUNER_OK) return e;
+  if ((e = set_device(ctx)) != ATTUNER_OK) return e;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  Scratch sc{ctx, st};
+  sc.cap = q_project_scratch(ctx, plan->n_req * S);
+  CUDA_TRY(cudaMallocFromPoolAsync(&sc.base, sc.cap, ctx->mempool, st));
+  int launches = 0;
+  e = q_project_impl(ctx, plan, x, w_q, lora_a, lora_b, r, s, q_norm_w, S, S_kv, q_out, st, sc, launches);
+  cudaFreeAsync(sc.base, st);
+  ctx->last_launches = launches;
+  return e;
+}
+
+extern "C" attuner_status attuner_attend(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
+                                         const void* suffix_k, const void* suffix_v, int32_t S, int32_t S_kv,
+                                         void* out, float* lse_out, void* stream) {
+  attuner_status e = check_common(ctx, plan, S, S_kv);
+  if (e != ATTUNER_OK) return e;
+  if ((e = set_device(ctx)) != ATTUNER_OK) return e;
+  int launches = 0;
+  e = attend_impl(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, static_cast<cudaStream_t>(stream),
+                  nullptr, launches);
+  ctx->last_launches = launches;
+  return e;
+}
+
+extern "C" attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
+                                               const void* w_q, const void* lora_a, const void* lora_b,
+                                               int32_t r, float s, const void* q_norm_w, const void* suffix_k,
+                                               const void* suffix_v, int32_t S, int32_t S_kv, void* out,
+                                               float* lse_out, void* stream) {
+  attuner_status e = check_common(ctx, plan, S, S_kv);
+  if (e != ATTUNER_OK) return e;
+  if ((e = set_device(ctx)) != ATTUNER_OK) return e;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int M = plan->n_req * S;
+  const size_t q_bytes = ((size_t)M * ctx->cfg.n_q_heads * ctx->cfg.head_dim * 2 + 255) & ~size_t(255);
+  Scratch sc{ctx, st};
+  sc.cap = q_bytes + q_project_scratch(ctx, M);
+  CUDA_TRY(cudaMallocFromPoolAsync(&sc.base, sc.cap, ctx->mempool, st));
+  const size_t off_q = sc.take(q_bytes);
+  void* q = static_cast<char*>(sc.base) + off_q;
+  int launches = 0;
+  e = q_project_impl(ctx, plan, x, w_q, lora_a, lora_b, r, s, q_norm_w, S, S_kv, q, st, sc, launches);
+  if (e == ATTUNER_OK)
+    e = attend_impl(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, st, &sc, launches);
+  cudaFreeAsync(sc.base, st);
+  ctx->last_launches = launches;
+  return e;
+}
+
+// ---------------------------------------------------------------------------
+// misc
+// ---------------------------------------------------------------------------
+extern "C" attuner_status attuner_pool_info(const attuner_ctx* ctx, void** k_pool, void** v_pool,
+                                            int32_t* used_blocks, int32_t* capacity_blocks) {
+  CHECK_ARG(ctx != nullptr, "ctx must not be NULL");
+  if (k_pool) *k_pool = ctx->kpool;
+  if (v_pool) *v_pool = ctx->vpool;
+  if (used_blocks) *used_blocks = ctx->used_blocks;
+  if (capacity_blocks) *capacity_blocks = ctx->cfg.pool_blocks;
+  return ATTUNER_OK;
+}
+
+extern "C" attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream) {
+  CHECK_ARG(ctx != nullptr, "ctx must not be NULL");
+  attuner_status e = set_device(ctx);
+  if (e != ATTUNER_OK) return e;
+  CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  int h = 0;
+  CUDA_TRY(cudaMemcpy(&h, ctx->d_status, sizeof(int), cudaMemcpyDeviceToHost));
+  CUDA_TRY(cudaMemset(ctx->d_status, 0, sizeof(int)));
+  if (h == ATTUNER_ERR_TIMEOUT) return fail(ATTUNER_ERR_TIMEOUT, "a kernel's bounded wait ran out");
+  if (h == ATTUNER_ERR_DEVICE_CHECK) return fail(ATTUNER_ERR_DEVICE_CHECK, "a kernel rejected an out-of-range index");
+  if (h != 0) return fail(ATTUNER_ERR_CUDA, "device status " + std::to_string(h));
+  return ATTUNER_OK;
+}
+
+extern "C" attuner_status attuner_set_option(attuner_ctx* ctx, int32_t option, int64_t value) {
+  CHECK_ARG(ctx != nullptr, "ctx must not be NULL");
+  switch (option) {
+    case ATTUNER_OPT_PREFILL_KERNEL:
+      CHECK_ARG(value >= 0 && value <= 2, "prefill kernel must be 0, 1 or 2");
+      ctx->opt_prefill = (int)value;
+      return ATTUNER_OK;
+    case ATTUNER_OPT_SPLIT_BLOCKS:
+      CHECK_ARG(value >= 0 && value <= kMaxChunkBlocks, "split blocks must be in [0, 4096]");
+      ctx->opt_split = (int)value;
+      return ATTUNER_OK;
+    case ATTUNER_OPT_WAIT_LIMIT:
+      CHECK_ARG(value >= 0, "wait limit must be >= 0");
+      ctx->wait_limit = value ? value : (1ll << 32);
+      return ATTUNER_OK;
+    case ATTUNER_OPT_TEST_STUCK_WAIT:
+      ctx->inject_stuck = value ? 1 : 0;
+      return ATTUNER_OK;
+    default:
+      return fail(ATTUNER_ERR_INVALID_ARG, "unknown option " + std::to_string(option));
+  }
+}
+
+extern "C" int32_t attuner_last_launch_count(const attuner_ctx* ctx) { return ctx ? ctx->last_launches : 0; }
+
+extern "C" const char* attuner_last_error(void) { return g_err.c_str(); }
