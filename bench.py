@@ -1,0 +1,412 @@
+"""Benchmark of the artifact-KV read path on GB300.
+
+One step = one pass of the whole path over one batch: adapted Q projection
+(LoRA, RMSNorm, RoPE) and attention over the assembled artifact blocks plus
+the suffix KV (split-KV combine included).  Default workload: the Qwen3-4B
+layer (hidden 2560, 32/8 heads, d 128, r 16, 8 artifacts of 512-2048 tokens,
+256 suffix tokens).  Inputs are seeded synthetic tensors of that shape.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the fp64 CPU oracle, timed on host cores
+
+Prints ONE JSON line (rank 0).  value = algorithmic attention FLOPs (or KV
+bytes for the decode workload) per step / device time per step, with the
+inputs resident in HBM; e2e = the same metric through the public API with
+the step's inputs copied from pinned host memory and its output copied back.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "artifact-KV attention TFLOP/s (prefill) & KV GB/s (decode), % of roofline"
+L2_FLUSH_BYTES = 512 << 20
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d["bf16_tflops_sustained"], src="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+# ---------------------------------------------------------------------------
+# work accounting (algorithmic, per step)
+# ---------------------------------------------------------------------------
+def attention_flops(wl) -> float:
+    """4 d Hq per visible (query, key) pair: 2d for q.k and 2d for p.v."""
+    g = wl.geom
+    pairs = 0
+    for r in range(wl.n_req):
+        t = wl.t_art(r)
+        pairs += wl.S * t + wl.S * (wl.S_kv - wl.S) + wl.S * (wl.S + 1) // 2
+    return 4.0 * g.head_dim * g.n_q_heads * pairs
+
+
+def qproj_flops(wl) -> float:
+    g = wl.geom
+    M = wl.n_req * wl.S
+    return 2.0 * M * g.hidden * g.d_q + 2.0 * M * g.hidden * g.rank + 2.0 * M * g.rank * g.d_q
+
+
+def kv_bytes(wl) -> float:
+    """Each request reads its assembled K and V once: (T_art + S_kv) * 2 * Hkv * d * 2 bytes."""
+    g = wl.geom
+    return float(sum((wl.t_art(r) + wl.S_kv) * 2 * g.n_kv_heads * g.head_dim * 2 for r in range(wl.n_req)))
+
+
+def is_decode(wl) -> bool:
+    return wl.S * wl.geom.group <= 16
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", str(device_index)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        load = [s for s in sm if s > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(load), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# the oracle timed on host cores (cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------
+def _oracle_inputs(wl, req):
+    import oracle
+    f = oracle.bf16_to_f64
+    g = wl.geom
+    ids = wl.requests[req]
+    return dict(x=f(wl.x[req]), w_q=f(wl.w_q), a=None if wl.lora_a is None else f(wl.lora_a),
+                b=None if wl.lora_b is None else f(wl.lora_b), s=g.scale, q_norm_w=f(wl.q_norm_w),
+                eps=g.rms_eps, theta=g.rope_theta, art_k=[f(wl.art_k[i]) for i in ids],
+                art_v=[f(wl.art_v[i]) for i in ids], suffix_k=f(wl.suffix_k[req]),
+                suffix_v=f(wl.suffix_v[req]), n_q_heads=g.n_q_heads)
+
+
+def oracle_sample(wl, inputs, tokens, decode: bool):
+    """Run the oracle on every head of the given suffix tokens of request 0.
+    Returns (seconds, work) with work in FLOPs (prefill) or bytes (decode)."""
+    import oracle
+    g = wl.geom
+    pairs = [(i, h) for i in tokens for h in range(g.n_q_heads)]
+    t0 = time.perf_counter()
+    oracle.request_forward(**inputs, pairs=pairs)
+    dt = time.perf_counter() - t0
+    t_art = wl.t_art(0)
+    vis = sum(t_art + (wl.S_kv - wl.S) + i + 1 for i in tokens)
+    if decode:
+        # every KV head's keys and values of the request are read once per token
+        work = float(sum(t_art + (wl.S_kv - wl.S) + i + 1 for i in tokens) * 2 * g.n_kv_heads * g.head_dim * 2)
+    else:
+        work = 4.0 * g.head_dim * g.n_q_heads * vis
+    return dt, work
+
+
+def _single_thread_env():
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
+        os.environ.setdefault(k, "1")
+
+
+def cpu_baseline(wl, budget_s: float = 12.0, seed: int = 0):
+    import numpy as np
+    decode = is_decode(wl)
+    inputs = _oracle_inputs(wl, 0)
+    rng = np.random.default_rng(seed)
+    tokens_all = list(range(wl.S))
+    done_t, done_w, n_tok = 0.0, 0.0, 0
+    chunk = max(1, min(8, wl.S))
+    while done_t < budget_s and n_tok < wl.S:
+        toks = sorted(rng.choice(tokens_all, size=min(chunk, wl.S), replace=False).tolist())
+        dt, w = oracle_sample(wl, inputs, toks, decode)
+        done_t += dt
+        done_w += w
+        n_tok += len(toks)
+    scale = 1e9 if decode else 1e12
+    return {"value": done_w / done_t / scale, "unit": "GB/s" if decode else "TFLOP/s",
+            "cores": int(os.environ.get("OPENBLAS_NUM_THREADS", "1")), "kind": "oracle",
+            "sample": f"request 0, {n_tok} suffix tokens x all {wl.geom.n_q_heads} q heads "
+                      f"(fp64 numpy, single-threaded BLAS), {done_t:.1f} s of CPU work"}
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import paper_2609_36722_gb300 as pkg
+    from gen import make_workload
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    wl = make_workload(args.workload, device=dev)
+    g = wl.geom
+    decode = is_decode(wl)
+    ctx = pkg.Context.for_geometry(g, pool_blocks=sum(-(-L // 64) for L in wl.art_lengths) + 1, device=local_rank)
+    for k, v in zip(wl.art_k, wl.art_v):
+        ctx.register_artifact(k, v)
+    plan = ctx.assemble(wl.requests)
+    stream = torch.cuda.current_stream()
+    out = torch.empty(wl.n_req, wl.S, g.n_q_heads, g.head_dim, dtype=torch.bfloat16, device=dev)
+    lse = torch.empty(wl.n_req, wl.S, g.n_q_heads, dtype=torch.float32, device=dev)
+    q = torch.empty_like(out)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def step():
+        ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv, out=q)
+        n1 = ctx.last_launch_count()
+        ev_a.record(stream)
+        ctx.attend(plan, q, wl.suffix_k, wl.suffix_v, out=out, lse=lse)
+        ev_b.record(stream)
+        return n1 + ctx.last_launch_count()
+
+    ev_a = torch.cuda.Event(enable_timing=True)
+    ev_b = torch.cuda.Event(enable_timing=True)
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    assert ctx.sync_status() == 0
+
+    sampler = ClockSampler(local_rank) if rank == 0 else None
+    # keep the GPU busy ~1 s before timing so the clock samples describe the timed region
+    t_end = time.perf_counter() + 1.0
+    while time.perf_counter() < t_end:
+        step()
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    attn_ms = []
+    launches = 0
+    for i in range(args.steps):
+        flush.zero_()                                   # L2 flush between steps, outside the timed events
+        starts[i].record(stream)
+        launches += step()
+        ends[i].record(stream)
+        ends[i].synchronize()
+        attn_ms.append(ev_a.elapsed_time(ev_b))
+    torch.cuda.synchronize()
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    total_ms = sum(step_ms)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    clocks = sampler.stop() if sampler else None
+    st = ctx.sync_status()
+    if st != 0:
+        raise RuntimeError(f"device status {st} after the timed region")
+
+    # ---- end to end through the public API with host buffers
+    x_h = wl.x.cpu().pin_memory()
+    sk_h = wl.suffix_k.cpu().pin_memory()
+    sv_h = wl.suffix_v.cpu().pin_memory()
+    out_h = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
+    x_d = torch.empty_like(wl.x)
+    sk_d = torch.empty_like(wl.suffix_k)
+    sv_d = torch.empty_like(wl.suffix_v)
+
+    def e2e_step():
+        p = ctx.assemble(wl.requests)
+        x_d.copy_(x_h, non_blocking=True)
+        sk_d.copy_(sk_h, non_blocking=True)
+        sv_d.copy_(sv_h, non_blocking=True)
+        ctx.query_attend(p, x_d, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, sk_d, sv_d, out=out,
+                         want_lse=False)
+        out_h.copy_(out, non_blocking=True)
+        torch.cuda.synchronize()
+        p.free()
+
+    for _ in range(max(3, args.warmup)):
+        e2e_step()
+    e2e_times = []
+    for _ in range(args.steps):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        e2e_step()
+        e2e_times.append(time.perf_counter() - t0)
+    e2e_s = sum(e2e_times)
+    if world > 1:
+        t = torch.tensor([e2e_s], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    h2d = (x_h.numel() + sk_h.numel() + sv_h.numel()) * 2
+    d2h = out_h.numel() * 2
+
+    peaks = _peaks()
+    work = kv_bytes(wl) if decode else attention_flops(wl)
+    scale = 1e9 if decode else 1e12
+    unit = "GB/s" if decode else "TFLOP/s"
+    value = work * world * args.steps / (total_ms * 1e-3) / scale
+    attn_avg_ms = statistics.mean(attn_ms)
+    achieved = work / (attn_avg_ms * 1e-3) / scale
+    peak = peaks["hbm"] if decode else peaks["bf16"]
+    traffic = load_traffic(args.workload)
+    result = {
+        "metric": METRIC, "value": round(value, 3), "unit": unit, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.workload, "hidden": g.hidden, "n_q_heads": g.n_q_heads,
+                   "n_kv_heads": g.n_kv_heads, "head_dim": g.head_dim, "lora_rank": g.rank, "s": g.scale,
+                   "n_req": wl.n_req, "S": wl.S, "S_kv": wl.S_kv,
+                   "t_art": [wl.t_art(r) for r in range(wl.n_req)][:8],
+                   "artifacts_per_req": [len(r) for r in wl.requests][:8],
+                   "parallelism": f"replicas x{world}",
+                   "l2": f"flushed between timed steps ({L2_FLUSH_BYTES >> 20} MiB write, outside the events)",
+                   "attention_kernel": "tcgen05 (attn_tc)" if not decode else "split-KV warp-MMA (attn_mma)"},
+        "roofline": {"bound": "hbm" if decode else "tensor", "achieved": round(achieved, 3), "peak": peak,
+                     "unit": unit, "frac": round(achieved / peak, 4), "traffic": traffic,
+                     "kernel": ("attn_mma_kernel + combine_kernel" if decode else "attn_tc_kernel (+ combine_kernel when split)"),
+                     "peak_source": f"{peaks['src']} ({'hbm_gbs' if decode else 'bf16_tflops burst'})",
+                     "avg_launch_ms": round(attn_avg_ms, 5)},
+        "path_work": {"attention_flops": attention_flops(wl), "qproj_flops": qproj_flops(wl),
+                      "kv_bytes": kv_bytes(wl)},
+        "e2e": {"value": round(work * world * args.steps / e2e_s / scale, 3), "unit": unit,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "includes": "assemble (host block table + H2D), H2D of x and suffix K/V, query_attend, D2H of O"},
+        "gpu_launches": launches,
+        "clocks": clocks,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(wl)
+    plan.free()
+    ctx.close()
+    return result
+
+
+def load_traffic(workload):
+    """dram bytes per launch of the dominant kernel, from the committed ncu summary (or None)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    return d.get(workload)
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the fp64 oracle on host cores
+# ---------------------------------------------------------------------------
+def run_reference(args):
+    import numpy as np
+    import torch
+    from gen import make_workload
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    wl = make_workload(args.workload, device=dev).to("cpu")
+    decode = is_decode(wl)
+    inputs = _oracle_inputs(wl, 0)
+    rng = np.random.default_rng(0)
+    toks_per_step = max(1, min(4, wl.S))
+    for _ in range(args.warmup):
+        oracle_sample(wl, inputs, sorted(rng.choice(wl.S, size=toks_per_step, replace=False).tolist()), decode)
+    tot_t, tot_w = 0.0, 0.0
+    for _ in range(args.steps):
+        dt, w = oracle_sample(wl, inputs, sorted(rng.choice(wl.S, size=toks_per_step, replace=False).tolist()),
+                              decode)
+        tot_t += dt
+        tot_w += w
+    scale = 1e9 if decode else 1e12
+    unit = "GB/s" if decode else "TFLOP/s"
+    value = tot_w / tot_t / scale
+    sample = (f"per step: request 0, {toks_per_step} random suffix tokens x all {wl.geom.n_q_heads} q heads "
+              f"(fp64 numpy oracle, single-threaded BLAS)")
+    return {"metric": METRIC, "value": value, "unit": unit, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": tot_t * 1e3 / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": args.workload, "parallelism": "host cores"},
+            "cpu_baseline": {"value": value, "unit": unit, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="qwen3_4b_prefill")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        _single_thread_env()
+        if rank != 0:
+            return
+        print(json.dumps(run_reference(args)))
+        return
+
+    _single_thread_env()
+    if world > 1:
+        import torch
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    res = run_ours(args, rank, world, local_rank)
+    if rank == 0:
+        print(json.dumps(res))
+    if world > 1:
+        import torch
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -149,10 +149,14 @@ def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, n_visible: Sequence[i
     G = Hq // Hkv
     scale = 1.0 / math.sqrt(d)
 
+    # one contiguous [T, d] copy per KV head, so each query row reads a prefix
+    k_heads = [np.ascontiguousarray(k[:, j, :]) for j in range(Hkv)]
+    v_heads = [np.ascontiguousarray(v[:, j, :]) for j in range(Hkv)]
+
     def one(i, h):
         n = int(n_visible[i])
-        kh = k[:n, h // G, :]
-        vh = v[:n, h // G, :]
+        kh = k_heads[h // G][:n]
+        vh = v_heads[h // G][:n]
         logits = (kh @ q[i, h, :]) * scale
         m = np.max(logits)
         e = np.exp(logits - m)

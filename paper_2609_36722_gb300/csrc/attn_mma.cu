@@ -362,7 +362,7 @@ __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ Co
     M = fmaxf(M, p.part_lse[c * R + r]);
   }
   float W = 0.f;
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   const int cpl = p.D / 32;   // columns per lane (2 or 4)
   for (int s = 0; s < ns; ++s) {
     const long long c = p.work.base[req] + ((long long)s * p.Hkv + kvh) * p.work.row_tiles + rt;
@@ -371,12 +371,22 @@ __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ Co
     const float w = __expf(ls - M);
     W += w;
     const float* po = p.part_o + (c * R + r) * p.D + lane * cpl;
-    for (int k = 0; k < cpl; ++k) acc[k] += w * po[k];
+    if (cpl == 4) {
+      const float4 v = *reinterpret_cast<const float4*>(po);
+      acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+    } else {
+      const float2 v = *reinterpret_cast<const float2*>(po);
+      acc.x += w * v.x; acc.y += w * v.y;
+    }
   }
   const float inv = (W > 0.f) ? 1.f / W : 0.f;
   const long long orow = ((long long)req * p.S + tok) * p.Hq + kvh * p.G + pr % p.G;
   __nv_bfloat16* dst = p.out + orow * p.D + lane * cpl;
-  for (int k = 0; k < cpl; ++k) dst[k] = __float2bfloat16_rn(acc[k] * inv);
+  if (cpl == 4) {
+    *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16(acc.x * inv, acc.y * inv), pack_bf16(acc.z * inv, acc.w * inv));
+  } else {
+    *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc.x * inv, acc.y * inv);
+  }
   if (lane == 0 && p.lse_out) p.lse_out[orow] = (W > 0.f) ? M + logf(W) : -INFINITY;
 }
 

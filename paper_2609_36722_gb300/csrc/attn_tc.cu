@@ -275,9 +275,16 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
           for (int c = 0; c < 64; ++c) s[64 * b + c] = -INFINITY;
         }
       }
-      float mx = s[0];
+      // row max: eight independent chains of 3-input max, then a small tree
+      float mk[8];
 #pragma unroll
-      for (int c = 1; c < 128; ++c) mx = fmaxf(mx, s[c]);
+      for (int k = 0; k < 8; ++k) mk[k] = fmaxf(s[k], s[k + 8]);
+#pragma unroll
+      for (int c = 16; c < 128; c += 16) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) mk[k] = fmax3(mk[k], s[c + k], s[c + k + 8]);
+      }
+      float mx = fmax3(fmax3(mk[0], mk[1], mk[2]), fmax3(mk[3], mk[4], mk[5]), fmaxf(mk[6], mk[7]));
       mx *= p.scale_log2;
       float alpha = 1.f;
       if (mx > m_run + 8.f) {              // move the reference max only when it grows past 2^8
@@ -285,11 +292,22 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
         m_run = mx;
       }
       const float neg = (m_run == -INFINITY) ? 0.f : -m_run;
-      float rs = 0.f;
+      // p = 2^(s * log2(e)/sqrt(d) - m): packed fp32 FMA, then ex2; row sum in 8 packed chains
+      const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2), ng2 = f2_pack(neg, neg);
+      uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-      for (int c = 0; c < 128; ++c) {
-        s[c] = ex2(fmaf(s[c], p.scale_log2, neg));
-        rs += s[c];
+      for (int c = 0; c < 128; c += 2) {
+        float a, b;
+        f2_unpack(f2_fma(f2_pack(s[c], s[c + 1]), sc2, ng2), a, b);
+        s[c] = ex2(a);
+        s[c + 1] = ex2(b);
+        acc2[(c >> 1) & 3] = f2_add(acc2[(c >> 1) & 3], f2_pack(s[c], s[c + 1]));
+      }
+      float rs;
+      {
+        float a0, a1;
+        f2_unpack(f2_add(f2_add(acc2[0], acc2[1]), f2_add(acc2[2], acc2[3])), a0, a1);
+        rs = a0 + a1;
       }
       l_run = l_run * alpha + rs;
 

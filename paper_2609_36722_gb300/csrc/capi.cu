@@ -423,7 +423,7 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
   pp.S = S;
   pp.S_kv = S_kv;
   pp.s = s;
-  pp.theta = (double)c.rope_theta;
+  for (int j = 0; j < D / 2; ++j) pp.inv_freq[j] = std::pow((double)c.rope_theta, -2.0 * j / (double)D);
   CUDA_TRY(launch_prep(pp, st));
   ++launches;
 
@@ -495,14 +495,33 @@ static void make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, i
   if (ctx->opt_split > 0) {
     chunk = ctx->opt_split;
   } else if (tc) {
-    // one CTA per SM: split only when the natural grid leaves SMs idle
-    const long long target = 2ll * ctx->num_sms;
-    chunk = (units >= target) ? maxv : (int)((total + target - 1) / target);
-    chunk = std::max(chunk, 8);
+    // One CTA per SM.  Cost of a chunk size = waves x (tiles per CTA + a fixed
+    // per-CTA overhead of ~4 tiles for the prologue, epilogue and combine);
+    // pick the number of splits of the longest request that minimises it.
+    const int maxt = (maxv + 1) / 2;
+    double best = 1e30;
+    chunk = maxv;
+    for (int sp = 1; sp <= 32; ++sp) {
+      const int ct = (maxt + sp - 1) / sp;
+      long long ncta = 0;
+      for (int r = 0; r < plan->n_req; ++r) {
+        const int nv = plan->blk_off[r + 1] - plan->blk_off[r] + nsuf;
+        ncta += (long long)((nv + 2 * ct - 1) / (2 * ct)) * Hkv * row_tiles;
+      }
+      const long long waves = (ncta + ctx->num_sms - 1) / ctx->num_sms;
+      const double cost = (double)waves * (ct + 4.0 + (sp > 1 ? 2.0 : 0.0));
+      if (cost < best - 1e-9) {
+        best = cost;
+        chunk = 2 * ct;
+      }
+    }
   } else {
+    // decode: several small CTAs per SM keep the HBM queues full and balance
+    // requests of different lengths
     const long long target = 8ll * ctx->num_sms;
     chunk = (int)std::max<long long>(16, (total + target - 1) / target);
   }
+  (void)units;
   chunk = std::min(chunk, kMaxChunkBlocks);
   if (tc) chunk = (chunk + 1) & ~1;   // whole 128-key tiles per split
   w.n_req = plan->n_req;

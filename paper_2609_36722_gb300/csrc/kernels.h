@@ -23,7 +23,7 @@ struct PrepParams {
   const int32_t* t_art;          // [n_req]
   int32_t M, hidden, r, d_q, D, S, S_kv;
   float s;
-  double theta;
+  double inv_freq[64];           // theta^(-2j/D), j < D/2 (computed on the host in double)
 };
 
 // K1b: Q = RoPE(RMSNorm([x | u] [W_q | B]^T) * w)  (tcgen05 GEMM + epilogue)

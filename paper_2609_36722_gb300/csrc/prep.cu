@@ -54,85 +54,80 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float* f) {
   }
 }
 
-// One warp per query row: u_pad row, rope row.  Extra blocks: b_pad.
-__global__ void __launch_bounds__(128) prep_kernel(const PrepParams p, int row_blocks) {
-  if ((int)blockIdx.x >= row_blocks) {
-    // b_pad[n][0..63] = B[n][0..r-1], zeros beyond
-    const long long idx = (long long)(blockIdx.x - row_blocks) * blockDim.x + threadIdx.x;
-    if (p.lora_b == nullptr || idx >= (long long)p.d_q * 8) return;
-    const int n = (int)(idx / 8), c = (int)(idx % 8);
-    uint4 val = make_uint4(0, 0, 0, 0);
-    if (c * 8 < p.r) val = *reinterpret_cast<const uint4*>(p.lora_b + (long long)n * p.r + c * 8);
-    *reinterpret_cast<uint4*>(p.b_pad + (long long)n * 64 + c * 8) = val;
+// One launch, three independent jobs selected by block index:
+//   [0, nb_lora)            one warp per (query row, 4 LoRA outputs): u = s * (A x)
+//   [nb_lora, +nb_rope)     one thread per (query row, rotary pair): cos/sin table
+//   [.., +nb_b)             one thread per 16 bytes of b_pad
+__global__ void __launch_bounds__(256) prep_kernel(const __grid_constant__ PrepParams p, int nb_lora,
+                                                   int nb_rope) {
+  const int bid = blockIdx.x;
+  if (bid < nb_lora) {
+    const int warp = (bid * 256 + (int)threadIdx.x) >> 5, lane = threadIdx.x & 31;
+    const int groups = 16;                       // 64 padded columns / 4 per warp
+    const int m = warp / groups, jg = warp % groups;
+    if (m >= p.M) return;
+    const int j0 = jg * 4;
+    if (j0 >= p.r) {                             // zero padding columns r..63
+      if (lane < 4) p.u_pad[(long long)m * 64 + j0 + lane] = __float2bfloat16_rn(0.f);
+      return;
+    }
+    const __nv_bfloat16* xr = p.x + (long long)m * p.hidden;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 2
+    for (int k = lane * 8; k < p.hidden; k += 256) {
+      float xf[8];
+      bf16x8_to_f32(*reinterpret_cast<const uint4*>(xr + k), xf);
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        float af[8];
+        bf16x8_to_f32(*reinterpret_cast<const uint4*>(p.lora_a + (long long)(j0 + jj) * p.hidden + k), af);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[jj] = fmaf(af[e], xf[e], acc[jj]);
+      }
+    }
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc[jj] += __shfl_xor_sync(0xffffffffu, acc[jj], o);
+    }
+    if (lane < 4) {
+      float v = lane == 0 ? acc[0] : lane == 1 ? acc[1] : lane == 2 ? acc[2] : acc[3];
+      p.u_pad[(long long)m * 64 + j0 + lane] = __float2bfloat16_rn(p.s * v);
+    }
     return;
   }
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int m = blockIdx.x * 4 + warp;
-  if (m >= p.M) return;
-
-  if (p.lora_a != nullptr && p.r > 0) {
-    float acc[64];
-#pragma unroll
-    for (int j = 0; j < 64; ++j) acc[j] = 0.f;
-    const __nv_bfloat16* xr = p.x + (long long)m * p.hidden;
-    for (int k0 = 0; k0 < p.hidden; k0 += 256) {
-      const int k = k0 + lane * 8;
-      if (k < p.hidden) {
-        float xf[8];
-        bf16x8_to_f32(*reinterpret_cast<const uint4*>(xr + k), xf);
-#pragma unroll
-        for (int j = 0; j < 64; ++j) {
-          if (j < p.r) {
-            float af[8];
-            bf16x8_to_f32(*reinterpret_cast<const uint4*>(p.lora_a + (long long)j * p.hidden + k), af);
-            float s = 0.f;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) s = fmaf(af[e], xf[e], s);
-            acc[j] += s;
-          }
-        }
-      }
-    }
-#pragma unroll
-    for (int j = 0; j < 64; ++j) {
-      if (j < p.r) {
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc[j] += __shfl_xor_sync(0xffffffffu, acc[j], o);
-      }
-    }
-    // lane writes columns 2*lane, 2*lane+1
-    float lo = 0.f, hi = 0.f;
-#pragma unroll
-    for (int j = 0; j < 64; ++j) {
-      if (j == 2 * lane) lo = (j < p.r) ? p.s * acc[j] : 0.f;
-      if (j == 2 * lane + 1) hi = (j < p.r) ? p.s * acc[j] : 0.f;
-    }
-    reinterpret_cast<__nv_bfloat162*>(p.u_pad + (long long)m * 64)[lane] =
-        __floats2bfloat162_rn(lo, hi);
-  }
-
-  // RoPE angles of this row: pos = T_art(req) + (S_kv - S) + i, pairs (j, j + D/2)
-  // turned by pos * theta^(-2j/D).  The angle is formed and reduced modulo
-  // 2*pi in double, then sin/cos are taken in float on |angle| <= pi.
-  const int req = m / p.S, i = m % p.S;
-  const long long pos = (long long)p.t_art[req] + (p.S_kv - p.S) + i;
-  const int half = p.D / 2;
-  const double two_pi = 6.283185307179586476925286766559;
-  for (int j = lane; j < half; j += 32) {
-    const double inv_freq = pow(p.theta, -2.0 * (double)j / (double)p.D);
-    double ang = (double)pos * inv_freq;
-    ang -= two_pi * floor(ang / two_pi);
-    if (ang > 3.14159265358979323846) ang -= two_pi;
+  if (bid < nb_lora + nb_rope) {
+    // RoPE angle of (row m, pair j): pos * theta^(-2j/D), pos = T_art(req) + (S_kv - S) + i.
+    // Formed and reduced modulo 2*pi in double, then sin/cos in float on |angle| <= pi.
+    const int half = p.D / 2;
+    const long long idx = (long long)(bid - nb_lora) * 256 + threadIdx.x;
+    if (idx >= (long long)p.M * half) return;
+    const int m = (int)(idx / half), j = (int)(idx % half);
+    const int req = m / p.S, i = m % p.S;
+    const long long pos = (long long)p.t_art[req] + (p.S_kv - p.S) + i;
+    const double ang = (double)pos * p.inv_freq[j];
+    const double k = rint(ang * 0.15915494309189533577);   // 1 / (2 pi)
+    const double red = fma(-k, 6.283185307179586232, ang);
     float sn, cs;
-    sincosf((float)ang, &sn, &cs);
-    p.rope[(long long)m * half + j] = make_float2(cs, sn);
+    sincosf((float)red, &sn, &cs);
+    p.rope[idx] = make_float2(cs, sn);
+    return;
   }
+  // b_pad[n][0..63] = B[n][0..r-1], zeros beyond
+  const long long idx = (long long)(bid - nb_lora - nb_rope) * 256 + threadIdx.x;
+  if (idx >= (long long)p.d_q * 8) return;
+  const int n = (int)(idx / 8), c = (int)(idx % 8);
+  uint4 val = make_uint4(0, 0, 0, 0);
+  if (c * 8 < p.r) val = *reinterpret_cast<const uint4*>(p.lora_b + (long long)n * p.r + c * 8);
+  *reinterpret_cast<uint4*>(p.b_pad + (long long)n * 64 + c * 8) = val;
 }
 
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st) {
-  const int row_blocks = (p.M + 3) / 4;
-  const int b_blocks = (p.lora_b != nullptr && p.r > 0) ? (p.d_q * 8 + 127) / 128 : 0;
-  prep_kernel<<<row_blocks + b_blocks, 128, 0, st>>>(p, row_blocks);
+  const bool lora = p.lora_a != nullptr && p.lora_b != nullptr && p.r > 0;
+  const int nb_lora = lora ? (p.M * 16 * 32 + 255) / 256 : 0;
+  const int nb_rope = (int)(((long long)p.M * (p.D / 2) + 255) / 256);
+  const int nb_b = lora ? (p.d_q * 8 + 255) / 256 : 0;
+  prep_kernel<<<nb_lora + nb_rope + nb_b, 256, 0, st>>>(p, nb_lora, nb_rope);
   return cudaGetLastError();
 }
 
