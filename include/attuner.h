@@ -160,6 +160,31 @@ attuner_status attuner_attend(attuner_ctx* ctx, const attuner_plan* plan, const 
                               const void* suffix_k, const void* suffix_v, int32_t S,
                               int32_t S_kv, void* out, float* lse_out, void* stream);
 
+/* attuner_attend for callers that cannot allocate GPU memory (no
+ * counterpart in the paper).  Some callers own the whole device: a serving
+ * engine whose allocator reserves the GPU up front, or a runtime that bars
+ * other libraries from cudaMalloc or stream-ordered pools because such an
+ * allocation can synchronise the device or fail in the middle of a request.
+ * This call runs the same kernels with the same split-KV decomposition as
+ * attuner_attend, with the same arguments and results, but keeps the split
+ * partial results in one fixed 32 MiB array in device memory that the library
+ * declares at file scope; it calls no allocator of any kind.
+ *   - The array exists on every GPU that loads the library until the process
+ *     exits.  The first call on a device looks up its device address once
+ *     (cudaGetSymbolAddress), so make that first call outside any stream
+ *     capture.
+ *   - Every call shares the array and it keeps the last call's contents
+ *     (nothing in it needs to start at zero).  Calls whose kernels overlap on
+ *     the GPU race on it: order them (one stream, or events).
+ *   - A call whose partial results would need more than 32 MiB
+ *     (n_split_ctas * rows_per_cta * (d + 1) * 4 bytes) is rejected with
+ *     INVALID_ARG before anything is launched; use attuner_attend for it.
+ * Errors: as attuner_attend, plus INVALID_ARG for a call beyond the limit. */
+attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const attuner_plan* plan,
+                                             const void* q, const void* suffix_k,
+                                             const void* suffix_v, int32_t S, int32_t S_kv,
+                                             void* out, float* lse_out, void* stream);
+
 /* The whole path: attuner_q_project into stream-ordered scratch, then
  * attuner_attend.  Arguments as in those two calls. */
 attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, const void* x,

@@ -39,6 +39,7 @@ EXPORTS = [
     "attuner_plan_export", "attuner_plan_t_art", "attuner_plan_free", "attuner_q_project",
     "attuner_attend", "attuner_query_attend", "attuner_pool_info", "attuner_sync_status",
     "attuner_set_option", "attuner_last_launch_count", "attuner_last_error",
+    "attuner_attend_static_scratch",
 ]
 
 
@@ -77,6 +78,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "attuner_plan_free": ([_vp], _i32),
         "attuner_q_project": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _i32, _i32, _vp, _vp], _i32),
         "attuner_attend": ([_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
+        "attuner_attend_static_scratch": ([_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
         "attuner_query_attend": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _vp, _vp, _i32, _i32,
                                   _vp, _vp, _vp], _i32),
         "attuner_pool_info": ([_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _p_i32, _p_i32], _i32),
@@ -237,6 +239,21 @@ class Context:
         _check(lib().attuner_attend(self.handle, plan.handle, _ptr(q, "q"), _ptr(suffix_k, "suffix_k"),
                                     _ptr(suffix_v, "suffix_v"), S, S_kv, _ptr(out, "out"),
                                     _ptr(lse, "lse", torch.float32), _stream(stream)))
+        return out, lse
+
+    def attend_static_scratch(self, plan: Plan, q, suffix_k, suffix_v, out: Optional[torch.Tensor] = None,
+                              lse: Optional[torch.Tensor] = None, want_lse: bool = True, stream=None):
+        """attend() without any allocation inside the library (fixed device scratch)."""
+        n_req, S, Hq, d = q.shape
+        S_kv = suffix_k.shape[1]
+        if out is None:
+            out = torch.empty_like(q)
+        if lse is None and want_lse:
+            lse = torch.empty(n_req, S, Hq, dtype=torch.float32, device=q.device)
+        _check(lib().attuner_attend_static_scratch(self.handle, plan.handle, _ptr(q, "q"),
+                                                   _ptr(suffix_k, "suffix_k"), _ptr(suffix_v, "suffix_v"), S,
+                                                   S_kv, _ptr(out, "out"), _ptr(lse, "lse", torch.float32),
+                                                   _stream(stream)))
         return out, lse
 
     def query_attend(self, plan: Plan, x, w_q, lora_a, lora_b, s: float, q_norm_w, suffix_k, suffix_v,

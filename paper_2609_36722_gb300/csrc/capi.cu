@@ -9,7 +9,7 @@
 #include <string>
 #include <vector>
 
-#include "kernels.h"
+#include "internal.h"
 
 using namespace att;
 
@@ -18,61 +18,10 @@ using namespace att;
 // ---------------------------------------------------------------------------
 static thread_local std::string g_err;
 
-static attuner_status fail(attuner_status s, const std::string& msg) {
+attuner_status att::fail(attuner_status s, const std::string& msg) {
   g_err = msg;
   return s;
 }
-
-#define CUDA_TRY(call)                                                                        \
-  do {                                                                                        \
-    cudaError_t e_ = (call);                                                                  \
-    if (e_ != cudaSuccess)                                                                    \
-      return fail(ATTUNER_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_));      \
-  } while (0)
-
-#define CHECK_ARG(cond, msg)                                  \
-  do {                                                        \
-    if (!(cond)) return fail(ATTUNER_ERR_INVALID_ARG, msg);   \
-  } while (0)
-
-// ---------------------------------------------------------------------------
-// objects
-// ---------------------------------------------------------------------------
-struct Artifact {
-  int32_t first_block;
-  int32_t L;
-  int32_t n_blocks;
-};
-
-struct attuner_ctx {
-  attuner_config cfg{};
-  __nv_bfloat16* kpool = nullptr;
-  __nv_bfloat16* vpool = nullptr;
-  int32_t used_blocks = 0;
-  std::vector<Artifact> arts;
-  CUtensorMap tm_kpool{}, tm_vpool{};
-  int* d_status = nullptr;
-  cudaMemPool_t mempool = nullptr;
-  int num_sms = 0;
-  int opt_prefill = 0;
-  int opt_split = 0;
-  long long wait_limit = 1ll << 32;
-  int inject_stuck = 0;
-  int last_launches = 0;
-};
-
-struct attuner_plan {
-  int32_t n_req = 0;
-  int32_t device = 0;
-  int32_t pool_blocks = 0;
-  std::vector<int32_t> req_off;   // CSR over artifact ids
-  std::vector<int32_t> art_ids;
-  std::vector<int32_t> blk_off;   // CSR over blocks
-  std::vector<int32_t> blocks;    // (pool block << 7) | valid
-  std::vector<int32_t> t_art;
-  std::vector<Artifact> arts;     // snapshot of the registry entries used
-  int32_t* d_buf = nullptr;       // blk_off | blocks | t_art
-};
 
 // ---------------------------------------------------------------------------
 // driver entry point for tensor maps (no link-time dependency on libcuda)
@@ -98,7 +47,7 @@ static EncodeTiledFn encode_fn() {
 // bf16 tensor map, 128-byte swizzle, zero fill out of bounds.
 // dims[0] is the innermost (contiguous) dimension; strides[i] is the byte
 // stride of dims[i+1].
-static attuner_status make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
+attuner_status att::make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
                                const uint64_t* strides, const uint32_t* box, const char* what) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return fail(ATTUNER_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
@@ -122,14 +71,14 @@ static attuner_status make_map(CUtensorMap* m, const void* base, int rank, const
   return ATTUNER_OK;
 }
 
-static attuner_status set_device(const attuner_ctx* ctx) {
+attuner_status att::set_device(const attuner_ctx* ctx) {
   int cur = -1;
   CUDA_TRY(cudaGetDevice(&cur));
   if (cur != ctx->cfg.device) CUDA_TRY(cudaSetDevice(ctx->cfg.device));
   return ATTUNER_OK;
 }
 
-static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+bool att::aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 // stream-ordered scratch of one call
 struct Scratch {
@@ -364,7 +313,7 @@ extern "C" attuner_status attuner_plan_free(attuner_plan* p) {
   return ATTUNER_OK;
 }
 
-static PlanDev plan_dev(const attuner_plan* p) {
+PlanDev att::plan_dev(const attuner_plan* p) {
   PlanDev d;
   d.blk_off = p->d_buf;
   d.blocks = p->d_buf + p->blk_off.size();
@@ -376,7 +325,7 @@ static PlanDev plan_dev(const attuner_plan* p) {
 // ---------------------------------------------------------------------------
 // Q projection
 // ---------------------------------------------------------------------------
-static attuner_status check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv) {
+attuner_status att::check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv) {
   CHECK_ARG(ctx != nullptr && plan != nullptr, "ctx and plan must not be NULL");
   CHECK_ARG(plan->device == ctx->cfg.device && plan->pool_blocks == ctx->cfg.pool_blocks,
             "plan belongs to another context");
@@ -477,7 +426,7 @@ static size_t q_project_scratch(const attuner_ctx* ctx, int M) {
 // ---------------------------------------------------------------------------
 // attention
 // ---------------------------------------------------------------------------
-static void make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc,
+void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc,
                       WorkTable& w) {
   const int G = ctx->cfg.n_q_heads / ctx->cfg.n_kv_heads, Hkv = ctx->cfg.n_kv_heads;
   const int rows = tc ? kTcRows : kMmaRows;

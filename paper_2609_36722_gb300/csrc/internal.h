@@ -1,0 +1,73 @@
+// internal.h - host-side objects and helpers shared by the translation units
+// that implement the C ABI (capi.cu and attend_static.cu).  Not part of the
+// public boundary, which is include/attuner.h.
+#pragma once
+
+#include <string>
+#include <vector>
+
+#include "kernels.h"
+
+#define CUDA_TRY(call)                                                                        \
+  do {                                                                                        \
+    cudaError_t e_ = (call);                                                                  \
+    if (e_ != cudaSuccess)                                                                    \
+      return att::fail(ATTUNER_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+#define CHECK_ARG(cond, msg)                                       \
+  do {                                                             \
+    if (!(cond)) return att::fail(ATTUNER_ERR_INVALID_ARG, msg);   \
+  } while (0)
+
+struct Artifact {
+  int32_t first_block;
+  int32_t L;
+  int32_t n_blocks;
+};
+
+struct attuner_ctx {
+  attuner_config cfg{};
+  __nv_bfloat16* kpool = nullptr;
+  __nv_bfloat16* vpool = nullptr;
+  int32_t used_blocks = 0;
+  std::vector<Artifact> arts;
+  CUtensorMap tm_kpool{}, tm_vpool{};
+  int* d_status = nullptr;
+  cudaMemPool_t mempool = nullptr;
+  int num_sms = 0;
+  int opt_prefill = 0;
+  int opt_split = 0;
+  long long wait_limit = 1ll << 32;
+  int inject_stuck = 0;
+  int last_launches = 0;
+};
+
+struct attuner_plan {
+  int32_t n_req = 0;
+  int32_t device = 0;
+  int32_t pool_blocks = 0;
+  std::vector<int32_t> req_off;   // CSR over artifact ids
+  std::vector<int32_t> art_ids;
+  std::vector<int32_t> blk_off;   // CSR over blocks
+  std::vector<int32_t> blocks;    // (pool block << 7) | valid
+  std::vector<int32_t> t_art;
+  std::vector<Artifact> arts;     // snapshot of the registry entries used
+  int32_t* d_buf = nullptr;       // blk_off | blocks | t_art
+};
+
+namespace att {
+
+// record `msg` as this thread's last error and return `s`
+attuner_status fail(attuner_status s, const std::string& msg);
+// bf16 tensor map with 128-byte swizzle and zero fill out of bounds
+attuner_status make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
+                        const uint64_t* strides, const uint32_t* box, const char* what);
+attuner_status set_device(const attuner_ctx* ctx);
+bool aligned16(const void* p);
+PlanDev plan_dev(const attuner_plan* p);
+attuner_status check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv);
+// split-KV decomposition of one attention launch (tc: tcgen05 kernel, else warp-MMA kernel)
+void make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc, WorkTable& w);
+
+}  // namespace att

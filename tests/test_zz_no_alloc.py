@@ -1,0 +1,63 @@
+"""attuner_attend_static_scratch: the attention entry point for callers that
+cannot allocate GPU memory (a serving engine that owns the whole device, a
+runtime that bars other libraries from allocating because an allocation can
+synchronise the device).  Its split-KV partial results live in a fixed
+device array of the library instead of a stream-ordered pool.
+
+The test calls it through the C ABI twice in a row on a layout that splits
+the KV (so the fixed array is really used, and the second call finds the
+first call's contents there) and compares each result with attuner_attend
+on the same inputs.  It must pass alone in a fresh process and after every
+other test; pytest collects this file last."""
+
+import numpy as np
+import pytest
+import torch
+
+from gen import Geometry, make_custom
+from helpers import LSE_MAX_ABS, O_MAX_ABS, O_MEAN_ABS, load_context
+
+pytestmark = pytest.mark.gpu
+
+DEV = torch.device("cuda", 0) if torch.cuda.is_available() else None
+
+
+def _close(a, b):
+    d = (a.double() - b.double()).abs()
+    return d.max().item() <= O_MAX_ABS and d.mean().item() <= O_MEAN_ABS
+
+
+@pytest.mark.parametrize("kernel,split,S,S_kv", [(1, 4, 96, 96), (2, 0, 1, 129)])
+def test_static_scratch_matches_attend_twice(kernel, split, S, S_kv):
+    import paper_2609_36722_gb300 as pkg
+    geom = Geometry(hidden=256, n_q_heads=16, n_kv_heads=4, head_dim=128, rank=16)
+    wl = make_custom("noalloc", geom, 41, [700, 333, 1200, 64], [[2, 0, 3], [1, 3], [0, 1, 2, 3]], S, S_kv,
+                     device=DEV)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, kernel)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, split)
+    g = wl.geom
+    q = ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=S_kv)
+    ref_o, ref_l = ctx.attend(plan, q, wl.suffix_k, wl.suffix_v)
+    assert ctx.sync_status() == 0
+    assert ctx.last_launch_count() == 2, "the layout must split the KV so the scratch is used"
+    for _ in range(2):
+        out, lse = ctx.attend_static_scratch(plan, q, wl.suffix_k, wl.suffix_v)
+        assert ctx.sync_status() == 0
+        assert ctx.last_launch_count() == 2
+        assert _close(out, ref_o)
+        assert (lse - ref_l).abs().max().item() <= LSE_MAX_ABS
+
+
+def test_static_scratch_rejects_calls_beyond_its_size():
+    import paper_2609_36722_gb300 as pkg
+    geom = Geometry(hidden=256, n_q_heads=32, n_kv_heads=8, head_dim=128, rank=16)
+    # 8 KV heads x 64 row tiles x 8 splits of 128-row fp32 partials is far over 32 MiB
+    wl = make_custom("big", geom, 43, [4096], [[0]], 2048, 2048, device=DEV)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, 16)
+    q = torch.zeros(1, 2048, 32, 128, dtype=torch.bfloat16, device=DEV)
+    with pytest.raises(pkg.AttunerError) as e:
+        ctx.attend_static_scratch(plan, q, wl.suffix_k, wl.suffix_v)
+    assert e.value.status == pkg.attuner.ERR_INVALID_ARG
+    assert "32" in str(e.value) or "bytes" in str(e.value)
