@@ -328,13 +328,23 @@ def run_ours(args, rank, world, local_rank):
 
 
 def load_traffic(workload):
-    """dram bytes per launch of the dominant kernel, from the committed ncu summary (or None)."""
+    """DRAM bytes per launch of the dominant kernel from the committed ncu summary,
+    or None when there is none or the kernel source changed since it was taken."""
+    import hashlib
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
     with open(p) as f:
-        d = json.load(f)
-    return d.get(workload)
+        d = json.load(f).get(workload)
+    if not d:
+        return None
+    src = os.path.join(ROOT, d["source"])
+    if not os.path.exists(src):
+        return None
+    with open(src, "rb") as f:
+        if hashlib.sha256(f.read()).hexdigest()[:16] != d["sha256_16"]:
+            return None
+    return d["bytes_per_launch"]
 
 
 # ---------------------------------------------------------------------------
