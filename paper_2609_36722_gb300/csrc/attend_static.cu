@@ -91,7 +91,7 @@ extern "C" attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const 
     const uint64_t dims[5] = {(uint64_t)D, (uint64_t)G, (uint64_t)Hkv, (uint64_t)S, (uint64_t)plan->n_req};
     const uint64_t strides[4] = {(uint64_t)D * 2, (uint64_t)G * D * 2, (uint64_t)Hq * D * 2,
                                  (uint64_t)S * Hq * D * 2};
-    const uint32_t box[5] = {64, (uint32_t)G, 1, (uint32_t)(kTcRows / G), 1};
+    const uint32_t box[5] = {64, (uint32_t)G, 1, (uint32_t)(kTcTileRows / G), 1};
     if ((e = make_map(&ap.tm_q, q, 5, dims, strides, box, "q")) != ATTUNER_OK) return e;
   }
   {

@@ -3,23 +3,31 @@
 // the causal mask M_t; App. A.5: SDPA with position ids of the assembled
 // context), as a tcgen05 / TMEM / TMA flash-attention kernel.
 //
-// One CTA = 128 "packed" query rows of one request and one KV head: the G
-// query heads that share the KV head are stacked into the M dimension
-// (packed row = token * G + head_in_group), and one split-KV chunk of the
-// request's virtual block list (artifact blocks from the block table in
-// runtime order, then 64-token chunks of the suffix KV).
+// One CTA = 256 "packed" query rows of one request and one KV head, as two
+// 128-row query tiles Q0 and Q1 (packed row = token * G + head_in_group: the
+// G query heads that share a KV head are stacked into the MMA M dimension),
+// and one split-KV chunk of the request's virtual block list (artifact blocks
+// from the block table in runtime order, then 64-token chunks of the suffix).
 //
-// Per 128-key tile (two 64-token blocks, each one 16 KiB TMA box pair):
-//   S  = Q K^T     tcgen05.mma M=128 N=128 K=D   -> TMEM (double buffered)
-//   P  = exp2(S * log2(e)/sqrt(D) - m)           softmax warps, fp32, -> bf16 smem
-//   O += P V       tcgen05.mma M=128 N=D K=128   -> TMEM
-// The MMA warp issues QK^T of tile j+1 before PV of tile j, so the tensor
-// pipe computes while the softmax warps work on tile j.  The running max is
-// only moved when it grows by more than 2^8 (then O in TMEM is rescaled), so
-// most tiles need no O round trip.
+// Per 128-key tile j (two 64-token blocks, each one TMA box per 64 columns):
+//   S_i = Q_i K_j^T     tcgen05.mma M=128 N=128 K=D, A and B from SMEM -> TMEM
+//   P_i = exp2(S_i * log2(e)/sqrt(D) - m_i)    softmax warpgroup i, written as
+//                       bf16 back into the TMEM columns of S_i
+//   O_i += P_i V_j      tcgen05.mma M=128 N=D K=128, A = P_i from TMEM, B = V
+// The single MMA thread issues  PV_0(j), QK_0(j+1), PV_1(j), QK_1(j+1), so
+// each softmax warpgroup works on its tile while the tensor pipe runs the
+// other tile's products: every K/V tile feeds 4 MMAs, and the softmax of a
+// tile has the time of two MMAs to finish.  A commit after QK_i(j+1) also
+// covers every earlier MMA, so one barrier per tile tells softmax i that S_i
+// is ready, that PV_i(j) has consumed P_i and that O_i is current.  The
+// running max only moves when it grows by more than 2^8 (then O_i in TMEM is
+// rescaled), so most tiles need no O round trip.
 //
-// Warp 0: TMA producer.  Warp 1: TMEM owner and single-thread MMA issuer.
-// Warps 2..5: softmax + epilogue, one query row per thread (TMEM lane).
+// Warps 0..3: softmax of Q0; warps 4..7: softmax of Q1 (one query row per
+// thread = one TMEM lane; warp w reaches lanes 32*(w%4)..+31).  Warp 8: TMA
+// producer.  Warp 9: TMEM owner and single-thread MMA issuer.  The softmax
+// walks the two 64-key halves of a tile one at a time so that it fits the
+// 168 registers a 320-thread block gets.
 #include <math.h>
 
 #include "kernels.h"
@@ -29,25 +37,42 @@ namespace att {
 template <int D>
 struct TcLayout {
   static constexpr int NH = D / 64;                 // 64-column (128-byte) halves
-  static constexpr int NS = 2;                      // K/V pipeline stages
+  static constexpr int NS = 2;                      // K and V pipeline stages
   static constexpr int HALF = 128 * 128;            // 128 rows x 128 B
-  static constexpr int Q_OFF = 0;
-  static constexpr int K_OFF = Q_OFF + NH * HALF;
+  static constexpr int Q_OFF = 0;                   // Q0 then Q1, NH halves each
+  static constexpr int K_OFF = Q_OFF + 2 * NH * HALF;
   static constexpr int V_OFF = K_OFF + NS * NH * HALF;
-  static constexpr int P_OFF = V_OFF + NS * NH * HALF;
-  static constexpr int BAR_OFF = P_OFF + 2 * HALF;
+  static constexpr int BAR_OFF = V_OFF + NS * NH * HALF;
   static constexpr int LIST_OFF = BAR_OFF + 1024;
-  static constexpr int SMEM = LIST_OFF + kMaxChunkBlocks * 4 + 1024;
-  static constexpr uint32_t TMEM_COLS = 512;        // S0 | S1 | O
-  static constexpr uint32_t S_COL0 = 0, S_COL1 = 128, O_COL = 256;
+  static constexpr int SMEM_MIN = LIST_OFF + kMaxChunkBlocks * 4 + 1024;
+  // at least 116 KiB so that two CTAs never share an SM (each holds all of TMEM)
+  static constexpr int SMEM = SMEM_MIN > 118784 ? SMEM_MIN : 118784;
+  static constexpr uint32_t TMEM_COLS = 512;        // S0/P0 | S1/P1 | O0 | O1
 };
+
+__device__ __forceinline__ uint32_t s_col_of(int qt) { return qt ? 128u : 0u; }
+__device__ __forceinline__ uint32_t o_col_of(int qt) { return qt ? 384u : 256u; }
+
+constexpr int kProducerWarp = 8, kMmaWarp = 9;
 
 enum : int {
-  B_Q = 0, B_KF = 1, B_VF = 3, B_KE = 5, B_VE = 7, B_SF = 9, B_SE = 11,
-  B_PF = 13, B_PV = 14, B_O = 15, B_DRAIN = 16, B_NEVER = 17, B_COUNT = 18
+  B_Q = 0, B_KF = 1, B_VF = 3, B_KE = 5, B_VE = 7, B_SF = 9, B_PF = 11,
+  B_O = 13, B_DRAIN = 14, B_NEVER = 15, B_COUNT = 16
 };
 
-// load the K (or V) half-tiles of block slot `e` into `dst` (two 64-column halves at +HALF)
+// D[tmem] (+)= A[tmem] * B[smem desc]: A (M x 16 bf16 per step) read from TMEM,
+// lane = row, each 32-bit column two consecutive K elements.
+ATT_DEV void umma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// load the K (or V) half-tiles of block slot `e` into `dst` (64-column halves at +HALF)
 template <int D>
 __device__ __forceinline__ void load_slot(uint32_t dst, int e, const CUtensorMap* pool,
                                           const CUtensorMap* suf, uint32_t bar, int kvh, int Hkv,
@@ -68,8 +93,29 @@ __device__ __forceinline__ void load_slot(uint32_t dst, int e, const CUtensorMap
   }
 }
 
+// Mask one 64-key block slot in place: artifact block tail (slot >= valid),
+// suffix causality (key > lim), or an empty slot.
+__device__ __forceinline__ void mask_slot(float* v, int e, int lim) {
+  if (e > 0) {
+    const int valid = e & 127;
+    if (valid < kBlockTokens) {
+#pragma unroll
+      for (int c = 0; c < 64; ++c) if (c >= valid) v[c] = -INFINITY;
+    }
+  } else if (e < 0) {
+    const int kbase = (-e - 1) * kBlockTokens;
+    if (kbase + kBlockTokens - 1 > lim) {
+#pragma unroll
+      for (int c = 0; c < 64; ++c) if (kbase + c > lim) v[c] = -INFINITY;
+    }
+  } else {
+#pragma unroll
+    for (int c = 0; c < 64; ++c) v[c] = -INFINITY;
+  }
+}
+
 template <int D>
-__global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__ AttnParams p) {
+__global__ void __launch_bounds__(320, 1) attn_tc_kernel(const __grid_constant__ AttnParams p) {
   using L = TcLayout<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -123,14 +169,11 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
     list[i] = e;
   }
   if (threadIdx.x == 0) {
-    for (int i = 0; i < B_COUNT; ++i) {
-      const bool multi = (i == B_SE || i == B_SE + 1 || i == B_PF);
-      mbar_init(bar(i), multi ? 4u : 1u);
-    }
+    for (int i = 0; i < B_COUNT; ++i) mbar_init(bar(i), (i == B_PF || i == B_PF + 1) ? 4u : 1u);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
     tmem_relinquish();
   }
@@ -139,17 +182,20 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0) {
+  if (warp == kProducerWarp) {
     // ================= TMA producer =================
     if (lane == 0 && ntile > 0) {
       tma_prefetch_desc(&p.tm_q);
       tma_prefetch_desc(&p.tm_kpool);
       tma_prefetch_desc(&p.tm_vpool);
-      mbar_expect_tx(bar(B_Q), L::NH * L::HALF);
+      mbar_expect_tx(bar(B_Q), 2 * L::NH * L::HALF);
 #pragma unroll
-      for (int h = 0; h < L::NH; ++h)
-        tma_load_5d(sbase + L::Q_OFF + h * L::HALF, &p.tm_q, bar(B_Q), h * 64, 0, kvh,
-                    rt * (kTcRows / G), req);
+      for (int qt = 0; qt < 2; ++qt) {
+#pragma unroll
+        for (int h = 0; h < L::NH; ++h)
+          tma_load_5d(sbase + L::Q_OFF + (qt * L::NH + h) * L::HALF, &p.tm_q, bar(B_Q), h * 64, 0, kvh,
+                      (row0 + qt * kTcTileRows) / G, req);
+      }
       int issued_k = 0, issued_v = 0;
       constexpr uint32_t tile_bytes = 2 * L::NH * (kBlockTokens * 128);
       for (int j = 0; j < ntile; ++j) {
@@ -182,47 +228,59 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
           mbar_drain(bar(B_VF + j % L::NS), (j / L::NS) & 1, p.status);
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == kMmaWarp) {
     // ================= MMA issuer (one thread) =================
     if (lane == 0 && ntile > 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(128, 128, 0, 0);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
-      bool ok = mbar_wait(bar(B_Q), 0, abort_flag, p.wait_limit, p.status);
       bool any = false;
-      auto issue_pv = [&](int i) -> bool {
-        const int st = i % L::NS;
-        if (!mbar_wait(bar(B_PF), i & 1, abort_flag, p.wait_limit, p.status)) return false;
-        if (!mbar_wait(bar(B_VF + st), (i / L::NS) & 1, abort_flag, p.wait_limit, p.status)) return false;
-        tc_fence_after();
-        const uint32_t v_s = sbase + L::V_OFF + st * L::NH * L::HALF;
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          const uint64_t a = sdesc_sw128(sbase + L::P_OFF + (k / 4) * L::HALF + (k % 4) * 32, 16, 1024);
-          const uint64_t b = sdesc_sw128(v_s + k * 2048, L::HALF, 1024);
-          umma_bf16(tmem + L::O_COL, a, b, idesc_pv, (i > 0 || k > 0) ? 1u : 0u);
-        }
-        umma_commit(bar(B_PV));
-        umma_commit(bar(B_VE + st));
-        return true;
-      };
-      for (int j = 0; ok && j < ntile; ++j) {
-        const int st = j % L::NS, sb = j & 1;
-        if (!mbar_wait(bar(B_KF + st), (j / L::NS) & 1, abort_flag, p.wait_limit, p.status)) { ok = false; break; }
-        if (j >= 2 && !mbar_wait(bar(B_SE + sb), ((j / 2) - 1) & 1, abort_flag, p.wait_limit, p.status)) { ok = false; break; }
-        tc_fence_after();
+      auto wait = [&](int b, uint32_t par) { return mbar_wait(bar(b), par, abort_flag, p.wait_limit, p.status); };
+      auto issue_qk = [&](int qt, int st) {
+        const uint32_t q_s = sbase + L::Q_OFF + qt * L::NH * L::HALF;
         const uint32_t k_s = sbase + L::K_OFF + st * L::NH * L::HALF;
 #pragma unroll
         for (int k = 0; k < D / 16; ++k) {
           const uint32_t off = (k / 4) * L::HALF + (k % 4) * 32;
-          umma_bf16(tmem + (sb ? L::S_COL1 : L::S_COL0), sdesc_sw128(sbase + L::Q_OFF + off, 16, 1024),
-                    sdesc_sw128(k_s + off, 16, 1024), idesc_qk, k > 0 ? 1u : 0u);
+          umma_bf16(tmem + s_col_of(qt), sdesc_sw128(q_s + off, 16, 1024), sdesc_sw128(k_s + off, 16, 1024),
+                    idesc_qk, k > 0 ? 1u : 0u);
         }
+        umma_commit(bar(B_SF + qt));
         any = true;
-        umma_commit(bar(B_SF + sb));
-        umma_commit(bar(B_KE + st));
-        if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
+      };
+      auto issue_pv = [&](int qt, int st, int j) {
+        const uint32_t v_s = sbase + L::V_OFF + st * L::NH * L::HALF;
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          umma_bf16_ts(tmem + o_col_of(qt), tmem + s_col_of(qt) + k * 8,
+                       sdesc_sw128(v_s + k * 2048, L::HALF, 1024), idesc_pv, (j > 0 || k > 0) ? 1u : 0u);
+      };
+      bool ok = wait(B_Q, 0) && wait(B_KF, 0);
+      if (ok) {
+        tc_fence_after();
+        issue_qk(0, 0);
+        issue_qk(1, 0);
+        umma_commit(bar(B_KE));
       }
-      if (ok) ok = issue_pv(ntile - 1);
+      for (int j = 0; ok && j < ntile; ++j) {
+        const int st = j % L::NS, st1 = (j + 1) % L::NS;
+        const bool more = j + 1 < ntile;
+        if (!(ok = wait(B_PF, j & 1) && wait(B_VF + st, (j / L::NS) & 1))) break;
+        tc_fence_after();
+        issue_pv(0, st, j);
+        if (more) {
+          if (!(ok = wait(B_KF + st1, ((j + 1) / L::NS) & 1))) break;
+          tc_fence_after();
+          issue_qk(0, st1);
+        }
+        if (!(ok = wait(B_PF + 1, j & 1))) break;
+        tc_fence_after();
+        issue_pv(1, st, j);
+        umma_commit(bar(B_VE + st));
+        if (more) {
+          issue_qk(1, st1);
+          umma_commit(bar(B_KE + st1));
+        }
+      }
       if (ok) {
         umma_commit(bar(B_O));
       } else if (any) {
@@ -230,59 +288,42 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
         mbar_drain(bar(B_DRAIN), 0, p.status);
       }
     }
-  } else {
-    // ================= softmax + epilogue (warps 2..5) =================
-    const int q = warp & 3;
-    const int r = q * 32 + lane;                 // tile row == TMEM lane
-    const int pr = row0 + r;                     // packed row
+  } else if (warp < 8) {
+    // ================= softmax + epilogue: warps 0..3 -> Q0, 4..7 -> Q1 =================
+    const int qt = warp / 4;
+    const int quad = warp & 3;
+    const int r = qt * kTcTileRows + quad * 32 + lane;   // CTA row
+    const int pr = row0 + r;                             // packed row
     const int tok = pr / G, jh = pr % G;
-    const int lim = (p.S_kv - p.S) + tok;        // last visible suffix key
-    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    const int lim = (p.S_kv - p.S) + tok;                // last visible suffix key
+    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    const uint32_t s_col = tmem + lane_base + s_col_of(qt);
+    const uint32_t o_col = tmem + lane_base + o_col_of(qt);
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    if (p.inject_stuck && q == 2)
+    if (p.inject_stuck && warp == 2)
       ok = warp_wait(bar(B_NEVER), 0, abort_flag, p.wait_limit, p.status);   // nothing arrives: times out
     for (int j = 0; ok && j < ntile; ++j) {
-      const int sb = j & 1;
-      if (!warp_wait(bar(B_SF + sb), (j / 2) & 1, abort_flag, p.wait_limit, p.status)) { ok = false; break; }
+      if (!warp_wait(bar(B_SF + qt), j & 1, abort_flag, p.wait_limit, p.status)) { ok = false; break; }
       tc_fence_after();
-      float s[128];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_base + (sb ? L::S_COL1 : L::S_COL0) + c * 32, s + c * 32);
-      tc_wait_ld();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar(B_SE + sb));
-
-      // mask: artifact block tails, suffix causality, empty slots
-#pragma unroll
-      for (int b = 0; b < 2; ++b) {
-        const int e = list[2 * j + b];
-        if (e > 0) {
-          const int valid = e & 127;
-          if (valid < kBlockTokens) {
-#pragma unroll
-            for (int c = 0; c < 64; ++c) if (c >= valid) s[64 * b + c] = -INFINITY;
-          }
-        } else if (e < 0) {
-          const int kbase = (-e - 1) * kBlockTokens;
-          if (kbase + kBlockTokens - 1 > lim) {
-#pragma unroll
-            for (int c = 0; c < 64; ++c) if (kbase + c > lim) s[64 * b + c] = -INFINITY;
-          }
-        } else {
-#pragma unroll
-          for (int c = 0; c < 64; ++c) s[64 * b + c] = -INFINITY;
-        }
-      }
-      // row max: eight independent chains of 3-input max, then a small tree
+      // Two passes over the two 64-key halves (one block slot each) keep only
+      // 64 scores live: pass 1 finds the masked row max, pass 2 re-reads each
+      // half from TMEM, exponentiates, sums and writes P back as bf16.
       float mk[8];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) mk[k] = fmaxf(s[k], s[k + 8]);
+      for (int k = 0; k < 8; ++k) mk[k] = -INFINITY;
+#pragma unroll 1
+      for (int b = 0; b < 2; ++b) {
+        float v[64];
+        tmem_ld32(s_col + 64 * b, v);
+        tmem_ld32(s_col + 64 * b + 32, v + 32);
+        tc_wait_ld();
+        mask_slot(v, list[2 * j + b], lim);
 #pragma unroll
-      for (int c = 16; c < 128; c += 16) {
+        for (int c = 0; c < 64; c += 16) {
 #pragma unroll
-        for (int k = 0; k < 8; ++k) mk[k] = fmax3(mk[k], s[c + k], s[c + k + 8]);
+          for (int k = 0; k < 8; ++k) mk[k] = fmax3(mk[k], v[c + k], v[c + k + 8]);
+        }
       }
       float mx = fmax3(fmax3(mk[0], mk[1], mk[2]), fmax3(mk[3], mk[4], mk[5]), fmaxf(mk[6], mk[7]));
       mx *= p.scale_log2;
@@ -292,53 +333,50 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
         m_run = mx;
       }
       const float neg = (m_run == -INFINITY) ? 0.f : -m_run;
-      // p = 2^(s * log2(e)/sqrt(d) - m): packed fp32 FMA, then ex2; row sum in 8 packed chains
+      // p = 2^(s * log2(e)/sqrt(d) - m): packed fp32 FMA, then ex2; row sum in packed chains
       const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2), ng2 = f2_pack(neg, neg);
       uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll 1
+      for (int b = 0; b < 2; ++b) {
+        float v[64];
+        tmem_ld32(s_col + 64 * b, v);
+        tmem_ld32(s_col + 64 * b + 32, v + 32);
+        tc_wait_ld();
+        mask_slot(v, list[2 * j + b], lim);
+        uint32_t pk[32];
 #pragma unroll
-      for (int c = 0; c < 128; c += 2) {
-        float a, b;
-        f2_unpack(f2_fma(f2_pack(s[c], s[c + 1]), sc2, ng2), a, b);
-        s[c] = ex2(a);
-        s[c + 1] = ex2(b);
-        acc2[(c >> 1) & 3] = f2_add(acc2[(c >> 1) & 3], f2_pack(s[c], s[c + 1]));
+        for (int c = 0; c < 64; c += 2) {
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(v[c], v[c + 1]), sc2, ng2), x0, x1);
+          x0 = ex2(x0);
+          x1 = ex2(x1);
+          acc2[(c >> 1) & 3] = f2_add(acc2[(c >> 1) & 3], f2_pack(x0, x1));
+          pk[c >> 1] = pack_bf16(x0, x1);
+        }
+        // P as bf16 pairs: keys 64b..64b+63 -> TMEM columns 32b..32b+31 of this tile's S region
+        tmem_st32(s_col + 32 * b, reinterpret_cast<const float*>(pk));
       }
-      float rs;
       {
         float a0, a1;
         f2_unpack(f2_add(f2_add(acc2[0], acc2[1]), f2_add(acc2[2], acc2[3])), a0, a1);
-        rs = a0 + a1;
+        l_run = l_run * alpha + (a0 + a1);
       }
-      l_run = l_run * alpha + rs;
-
-      // PV of the previous tile must be done: P buffer free, O current
-      if (j >= 1 && !warp_wait(bar(B_PV), (j - 1) & 1, abort_flag, p.wait_limit, p.status)) { ok = false; break; }
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const float* f = s + 64 * h + 8 * c;
-          st_shared_v4(sbase + L::P_OFF + h * L::HALF + sw128_off(r, c), pack_bf16(f[0], f[1]),
-                       pack_bf16(f[2], f[3]), pack_bf16(f[4], f[5]), pack_bf16(f[6], f[7]));
-        }
-      }
+      // O is current here (the commit that signalled S also covers the previous PV)
       if (j >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {
-        tc_fence_after();
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
-          tmem_ld32(tmem + lane_base + L::O_COL + c * 32, o);
+          tmem_ld32(o_col + c * 32, o);
           tc_wait_ld();
 #pragma unroll
           for (int k = 0; k < 32; ++k) o[k] *= alpha;
-          tmem_st32(tmem + lane_base + L::O_COL + c * 32, o);
+          tmem_st32(o_col + c * 32, o);
         }
-        tc_wait_st();
       }
-      fence_proxy_async_smem();
+      tc_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(bar(B_PF));
+      if (lane == 0) mbar_arrive(bar(B_PF + qt));
     }
 
     // ---- epilogue
@@ -355,7 +393,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
 #pragma unroll
           for (int c = 0; c < D / 32; ++c) {
             float o[32];
-            tmem_ld32(tmem + lane_base + L::O_COL + c * 32, o);
+            tmem_ld32(o_col + c * 32, o);
             tc_wait_ld();
             if (row_ok) {
 #pragma unroll
@@ -372,7 +410,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
-          tmem_ld32(tmem + lane_base + L::O_COL + c * 32, o);
+          tmem_ld32(o_col + c * 32, o);
           tc_wait_ld();
           if (row_ok) {
 #pragma unroll
@@ -388,7 +426,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc_kernel(const __grid_constant__
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, L::TMEM_COLS);
   }
@@ -399,7 +437,7 @@ static cudaError_t launch_attn_tc_t(const AttnParams& p, cudaStream_t st) {
   using L = TcLayout<D>;
   cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
-  attn_tc_kernel<D><<<p.work.n_cta, 192, L::SMEM, st>>>(p);
+  attn_tc_kernel<D><<<p.work.n_cta, 320, L::SMEM, st>>>(p);
   return cudaGetLastError();
 }
 

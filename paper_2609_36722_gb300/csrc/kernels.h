@@ -82,7 +82,8 @@ cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st);
 cudaError_t launch_combine(const CombineParams& p, cudaStream_t st);
 
 // rows per CTA of each attention kernel
-constexpr int kTcRows = 128;
+constexpr int kTcRows = 256;      // packed query rows per CTA of attn_tc (two tiles)
+constexpr int kTcTileRows = 128;  // rows per query tile (one MMA M)
 constexpr int kMmaRows = 16;
 // largest split chunk (virtual blocks) the kernels' shared-memory block list holds
 constexpr int kMaxChunkBlocks = 4096;
