@@ -23,11 +23,13 @@
 // running max only moves when it grows by more than 2^8 (then O_i in TMEM is
 // rescaled), so most tiles need no O round trip.
 //
-// Warps 0..3: softmax of Q0; warps 4..7: softmax of Q1 (one query row per
-// thread = one TMEM lane; warp w reaches lanes 32*(w%4)..+31).  Warp 8: TMA
-// producer.  Warp 9: TMEM owner and single-thread MMA issuer.  The softmax
-// walks the two 64-key halves of a tile one at a time so that it fits the
-// 168 registers a 320-thread block gets.
+// Warpgroup 0 (warps 0..3): softmax of Q0; warpgroup 1 (warps 4..7): softmax
+// of Q1 (one query row per thread = one TMEM lane; warp w reaches lanes
+// 32*(w%4)..+31).  Warpgroup 2: warp 8 TMA producer, warp 9 TMEM owner and
+// single-thread MMA issuer, warps 10..11 idle.  The block is launched with
+// 384 threads x 168 registers = 64512; warpgroup 2 drops to kCtrlRegs and the
+// softmax warpgroups rise to kSoftRegs: 128 x kCtrlRegs + 256 x kSoftRegs
+// <= 64512, so every score of a tile stays in registers.
 #include <math.h>
 
 #include "kernels.h"
@@ -54,6 +56,8 @@ __device__ __forceinline__ uint32_t s_col_of(int qt) { return qt ? 128u : 0u; }
 __device__ __forceinline__ uint32_t o_col_of(int qt) { return qt ? 384u : 256u; }
 
 constexpr int kProducerWarp = 8, kMmaWarp = 9;
+constexpr int kCtrlRegs = 80, kSoftRegs = 208;
+static_assert(128 * kCtrlRegs + 256 * kSoftRegs <= 384 * 168, "register split exceeds the launch budget");
 
 enum : int {
   B_Q = 0, B_KF = 1, B_VF = 3, B_KE = 5, B_VE = 7, B_SF = 9, B_PF = 11,
@@ -115,7 +119,7 @@ __device__ __forceinline__ void mask_slot(float* v, int e, int lim) {
 }
 
 template <int D>
-__global__ void __launch_bounds__(320, 1) attn_tc_kernel(const __grid_constant__ AttnParams p) {
+__global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__ AttnParams p) {
   using L = TcLayout<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -181,7 +185,8 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(const __grid_constant__
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-
+  if (warp >= 8) {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kCtrlRegs));
   if (warp == kProducerWarp) {
     // ================= TMA producer =================
     if (lane == 0 && ntile > 0) {
@@ -288,7 +293,9 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(const __grid_constant__
         mbar_drain(bar(B_DRAIN), 0, p.status);
       }
     }
-  } else if (warp < 8) {
+  }
+  } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kSoftRegs));
     // ================= softmax + epilogue: warps 0..3 -> Q0, 4..7 -> Q1 =================
     const int qt = warp / 4;
     const int quad = warp & 3;
@@ -306,24 +313,20 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(const __grid_constant__
     for (int j = 0; ok && j < ntile; ++j) {
       if (!warp_wait(bar(B_SF + qt), j & 1, abort_flag, p.wait_limit, p.status)) { ok = false; break; }
       tc_fence_after();
-      // Two passes over the two 64-key halves (one block slot each) keep only
-      // 64 scores live: pass 1 finds the masked row max, pass 2 re-reads each
-      // half from TMEM, exponentiates, sums and writes P back as bf16.
+      float sc[128];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(s_col + c * 32, sc + c * 32);
+      tc_wait_ld();
+      mask_slot(sc, list[2 * j], lim);
+      mask_slot(sc + 64, list[2 * j + 1], lim);
+      // row max: eight independent chains of 3-input max, then a small tree
       float mk[8];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) mk[k] = -INFINITY;
-#pragma unroll 1
-      for (int b = 0; b < 2; ++b) {
-        float v[64];
-        tmem_ld32(s_col + 64 * b, v);
-        tmem_ld32(s_col + 64 * b + 32, v + 32);
-        tc_wait_ld();
-        mask_slot(v, list[2 * j + b], lim);
+      for (int k = 0; k < 8; ++k) mk[k] = fmaxf(sc[k], sc[k + 8]);
 #pragma unroll
-        for (int c = 0; c < 64; c += 16) {
+      for (int c = 16; c < 128; c += 16) {
 #pragma unroll
-          for (int k = 0; k < 8; ++k) mk[k] = fmax3(mk[k], v[c + k], v[c + k + 8]);
-        }
+        for (int k = 0; k < 8; ++k) mk[k] = fmax3(mk[k], sc[c + k], sc[c + k + 8]);
       }
       float mx = fmax3(fmax3(mk[0], mk[1], mk[2]), fmax3(mk[3], mk[4], mk[5]), fmaxf(mk[6], mk[7]));
       mx *= p.scale_log2;
@@ -336,31 +339,24 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(const __grid_constant__
       // p = 2^(s * log2(e)/sqrt(d) - m): packed fp32 FMA, then ex2; row sum in packed chains
       const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2), ng2 = f2_pack(neg, neg);
       uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
-#pragma unroll 1
-      for (int b = 0; b < 2; ++b) {
-        float v[64];
-        tmem_ld32(s_col + 64 * b, v);
-        tmem_ld32(s_col + 64 * b + 32, v + 32);
-        tc_wait_ld();
-        mask_slot(v, list[2 * j + b], lim);
-        uint32_t pk[32];
+      uint32_t pk[64];
 #pragma unroll
-        for (int c = 0; c < 64; c += 2) {
-          float x0, x1;
-          f2_unpack(f2_fma(f2_pack(v[c], v[c + 1]), sc2, ng2), x0, x1);
-          x0 = ex2(x0);
-          x1 = ex2(x1);
-          acc2[(c >> 1) & 3] = f2_add(acc2[(c >> 1) & 3], f2_pack(x0, x1));
-          pk[c >> 1] = pack_bf16(x0, x1);
-        }
-        // P as bf16 pairs: keys 64b..64b+63 -> TMEM columns 32b..32b+31 of this tile's S region
-        tmem_st32(s_col + 32 * b, reinterpret_cast<const float*>(pk));
+      for (int c = 0; c < 128; c += 2) {
+        float x0, x1;
+        f2_unpack(f2_fma(f2_pack(sc[c], sc[c + 1]), sc2, ng2), x0, x1);
+        x0 = ex2(x0);
+        x1 = ex2(x1);
+        acc2[(c >> 1) & 3] = f2_add(acc2[(c >> 1) & 3], f2_pack(x0, x1));
+        pk[c >> 1] = pack_bf16(x0, x1);
       }
       {
         float a0, a1;
         f2_unpack(f2_add(f2_add(acc2[0], acc2[1]), f2_add(acc2[2], acc2[3])), a0, a1);
         l_run = l_run * alpha + (a0 + a1);
       }
+      // P as bf16 pairs (key k in column k/2) over the first 64 columns of this tile's S region
+      tmem_st32(s_col, reinterpret_cast<const float*>(pk));
+      tmem_st32(s_col + 32, reinterpret_cast<const float*>(pk + 32));
       // O is current here (the commit that signalled S also covers the previous PV)
       if (j >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll
@@ -435,9 +431,15 @@ __global__ void __launch_bounds__(320, 1) attn_tc_kernel(const __grid_constant__
 template <int D>
 static cudaError_t launch_attn_tc_t(const AttnParams& p, cudaStream_t st) {
   using L = TcLayout<D>;
-  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
+  // setmaxnreg.inc waits until the registers it asks for are free in the
+  // block's launch budget: never launch a split that exceeds that budget.
+  cudaFuncAttributes fa{};
+  cudaError_t e = cudaFuncGetAttributes(&fa, attn_tc_kernel<D>);
   if (e != cudaSuccess) return e;
-  attn_tc_kernel<D><<<p.work.n_cta, 320, L::SMEM, st>>>(p);
+  if (fa.numRegs * 384 < 128 * kCtrlRegs + 256 * kSoftRegs) return cudaErrorLaunchOutOfResources;
+  e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
+  if (e != cudaSuccess) return e;
+  attn_tc_kernel<D><<<p.work.n_cta, 384, L::SMEM, st>>>(p);
   return cudaGetLastError();
 }
 
