@@ -208,10 +208,14 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
  *   ATTUNER_OPT_SPLIT_BLOCKS    KV blocks per split-KV chunk (0 = automatic)
  *   ATTUNER_OPT_WAIT_LIMIT      clock cycles a device wait may spin before it
  *                               gives up and sets TIMEOUT (0 = about 2 s)
+ *   ATTUNER_OPT_QPROJ_SPLIT_K  most CTAs (1..4) that split the K dimension of one
+ *                               Q-projection tile when the tiles alone leave SMs
+ *                               idle (0 or 1 = no split, the default)
  *   ATTUNER_OPT_TEST_STUCK_WAIT see below */
 #define ATTUNER_OPT_PREFILL_KERNEL 1
 #define ATTUNER_OPT_SPLIT_BLOCKS   2
 #define ATTUNER_OPT_WAIT_LIMIT     3
+#define ATTUNER_OPT_QPROJ_SPLIT_K  4
 /* Test hook (failure detection without a GPU fault): while non-zero, one
  * role of every attention launch waits on an mbarrier that nothing arrives
  * at; its bounded wait runs out, the kernel drains its own copies, frees its

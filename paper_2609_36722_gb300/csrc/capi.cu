@@ -44,11 +44,12 @@ static EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// bf16 tensor map, 128-byte swizzle, zero fill out of bounds.
+// bf16 tensor map, 128-byte swizzle (or none), zero fill out of bounds.
 // dims[0] is the innermost (contiguous) dimension; strides[i] is the byte
 // stride of dims[i+1].
 attuner_status att::make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
-                               const uint64_t* strides, const uint32_t* box, const char* what) {
+                               const uint64_t* strides, const uint32_t* box, const char* what,
+                               bool swizzle128) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return fail(ATTUNER_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
   if ((reinterpret_cast<uintptr_t>(base) & 15) != 0)
@@ -63,7 +64,8 @@ attuner_status att::make_map(CUtensorMap* m, const void* base, int rank, const u
     if (i + 1 < rank) s[i] = strides[i];
   }
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base), d, s, b, e,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS)
     return fail(ATTUNER_ERR_CUDA, std::string("cuTensorMapEncodeTiled failed for ") + what +
@@ -335,6 +337,18 @@ attuner_status att::check_common(attuner_ctx* ctx, const attuner_plan* plan, int
   return ATTUNER_OK;
 }
 
+// Split K of the Q projection over up to ATTUNER_OPT_QPROJ_SPLIT_K CTAs per
+// (row tile, head) when those tiles alone would leave SMs idle.  Off by
+// default: on GB300 the partial-sum traffic costs more than the extra SMs
+// bring for the Qwen3-4B and decode shapes.
+static int qproj_ksplit(const attuner_ctx* ctx, int M) {
+  const int tiles = ctx->cfg.n_q_heads * ((M + 127) / 128);
+  const int nk = ctx->cfg.hidden / 64;
+  int ks = 1;
+  while (ks < ctx->opt_qproj_split && (long long)tiles * (ks + 1) <= ctx->num_sms && nk / (ks + 1) >= 2) ++ks;
+  return ks;
+}
+
 static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan, const void* x, const void* w_q,
                                      const void* lora_a, const void* lora_b, int32_t r, float s,
                                      const void* q_norm_w, int32_t S, int32_t S_kv, void* q_out,
@@ -348,30 +362,27 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
   if (lora) CHECK_ARG(aligned16(lora_a) && aligned16(lora_b), "lora_a and lora_b must be 16-byte aligned");
   const int M = plan->n_req * S;
   const int D = c.head_dim, Hq = c.n_q_heads, dq = Hq * D;
-  const size_t off_u = sc.take((size_t)M * 64 * 2);
-  const size_t off_b = sc.take((size_t)dq * 64 * 2);
+  const int n_lora = lora ? ((r + 15) / 16) * 16 : 0;
+  const int ksplit = qproj_ksplit(ctx, M);
+  const int tiles = Hq * ((M + 127) / 128);
   const size_t off_rope = sc.take((size_t)M * (D / 2) * 8);
+  size_t off_part = 0, off_cnt = 0;
+  if (ksplit > 1) {
+    off_part = sc.take((size_t)tiles * ksplit * 128 * (D + n_lora) * 4);
+    off_cnt = sc.take((size_t)tiles * 4);
+  }
   char* base = static_cast<char*>(sc.base);
-  __nv_bfloat16* u_pad = reinterpret_cast<__nv_bfloat16*>(base + off_u);
-  __nv_bfloat16* b_pad = reinterpret_cast<__nv_bfloat16*>(base + off_b);
   float2* rope = reinterpret_cast<float2*>(base + off_rope);
 
   PrepParams pp{};
-  pp.x = static_cast<const __nv_bfloat16*>(x);
-  pp.lora_a = lora ? static_cast<const __nv_bfloat16*>(lora_a) : nullptr;
-  pp.lora_b = lora ? static_cast<const __nv_bfloat16*>(lora_b) : nullptr;
-  pp.u_pad = u_pad;
-  pp.b_pad = b_pad;
   pp.rope = rope;
   pp.t_art = plan_dev(plan).t_art;
+  pp.counters = ksplit > 1 ? reinterpret_cast<int32_t*>(base + off_cnt) : nullptr;
+  pp.n_counters = ksplit > 1 ? tiles : 0;
   pp.M = M;
-  pp.hidden = c.hidden;
-  pp.r = lora ? r : 0;
-  pp.d_q = dq;
   pp.D = D;
   pp.S = S;
   pp.S_kv = S_kv;
-  pp.s = s;
   for (int j = 0; j < D / 2; ++j) pp.inv_freq[j] = std::pow((double)c.rope_theta, -2.0 * j / (double)D);
   CUDA_TRY(launch_prep(pp, st));
   ++launches;
@@ -390,25 +401,28 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
     const uint32_t box[2] = {64, (uint32_t)D};
     if ((e = make_map(&qp.tm_w, w_q, 2, dims, strides, box, "w_q")) != ATTUNER_OK) return e;
   }
-  {
-    const uint64_t dims[2] = {64, (uint64_t)M};
-    const uint64_t strides[1] = {128};
-    const uint32_t box[2] = {64, 128};
-    if ((e = make_map(&qp.tm_u, u_pad, 2, dims, strides, box, "u")) != ATTUNER_OK) return e;
-  }
-  {
-    const uint64_t dims[2] = {64, (uint64_t)dq};
-    const uint64_t strides[1] = {128};
-    const uint32_t box[2] = {64, (uint32_t)D};
-    if ((e = make_map(&qp.tm_b, b_pad, 2, dims, strides, box, "B")) != ATTUNER_OK) return e;
+  if (lora) {
+    const uint64_t dims[2] = {(uint64_t)c.hidden, (uint64_t)r};
+    const uint64_t strides[1] = {(uint64_t)c.hidden * 2};
+    const uint32_t box[2] = {64, (uint32_t)n_lora};
+    if ((e = make_map(&qp.tm_a, lora_a, 2, dims, strides, box, "lora_a")) != ATTUNER_OK) return e;
+    const uint64_t bdims[2] = {(uint64_t)r, (uint64_t)dq};
+    const uint64_t bstrides[1] = {(uint64_t)r * 2};
+    const uint32_t bbox[2] = {8, (uint32_t)D};
+    if ((e = make_map(&qp.tm_b, lora_b, 2, bdims, bstrides, bbox, "lora_b", false)) != ATTUNER_OK) return e;
   }
   qp.q_out = static_cast<__nv_bfloat16*>(q_out);
   qp.qnorm_w = static_cast<const __nv_bfloat16*>(q_norm_w);
   qp.rope = rope;
+  qp.part = ksplit > 1 ? reinterpret_cast<float*>(base + off_part) : nullptr;
+  qp.counters = pp.counters;
   qp.M = M;
   qp.hidden = c.hidden;
   qp.Hq = Hq;
-  qp.lora_ksteps = lora ? (r + 15) / 16 : 0;
+  qp.r = lora ? r : 0;
+  qp.n_lora = n_lora;
+  qp.ksplit = ksplit;
+  qp.s = s;
   qp.eps = c.rms_eps;
   qp.status = ctx->d_status;
   qp.wait_limit = ctx->wait_limit;
@@ -418,9 +432,13 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
 }
 
 static size_t q_project_scratch(const attuner_ctx* ctx, int M) {
-  const int D = ctx->cfg.head_dim, dq = ctx->cfg.n_q_heads * D;
+  const int D = ctx->cfg.head_dim, Hq = ctx->cfg.n_q_heads;
   auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
-  return al((size_t)M * 64 * 2) + al((size_t)dq * 64 * 2) + al((size_t)M * (D / 2) * 8);
+  const int ksplit = qproj_ksplit(ctx, M);
+  const size_t tiles = (size_t)Hq * ((M + 127) / 128);
+  size_t bytes = al((size_t)M * (D / 2) * 8);
+  if (ksplit > 1) bytes += al(tiles * ksplit * 128 * (D + 64) * 4) + al(tiles * 4);
+  return bytes;
 }
 
 // ---------------------------------------------------------------------------
@@ -540,8 +558,7 @@ static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, co
   ap->wait_limit = ctx->wait_limit;
   ap->inject_stuck = ctx->inject_stuck;
 
-  Scratch local{ctx, st};
-  Scratch& sc = sc_outer ? *sc_outer : local;
+  (void)sc_outer;
   void* part = nullptr;
   size_t part_bytes = 0;
   if (need_combine) {
@@ -673,6 +690,10 @@ extern "C" attuner_status attuner_set_option(attuner_ctx* ctx, int32_t option, i
     case ATTUNER_OPT_WAIT_LIMIT:
       CHECK_ARG(value >= 0, "wait limit must be >= 0");
       ctx->wait_limit = value ? value : (1ll << 32);
+      return ATTUNER_OK;
+    case ATTUNER_OPT_QPROJ_SPLIT_K:
+      CHECK_ARG(value >= 0 && value <= 4, "Q-projection split-K must be in [0, 4]");
+      ctx->opt_qproj_split = value ? (int)value : 1;
       return ATTUNER_OK;
     case ATTUNER_OPT_TEST_STUCK_WAIT:
       ctx->inject_stuck = value ? 1 : 0;

@@ -38,6 +38,7 @@ struct attuner_ctx {
   int num_sms = 0;
   int opt_prefill = 0;
   int opt_split = 0;
+  int opt_qproj_split = 1;
   long long wait_limit = 1ll << 32;
   int inject_stuck = 0;
   int last_launches = 0;
@@ -60,9 +61,10 @@ namespace att {
 
 // record `msg` as this thread's last error and return `s`
 attuner_status fail(attuner_status s, const std::string& msg);
-// bf16 tensor map with 128-byte swizzle and zero fill out of bounds
+// bf16 tensor map with zero fill out of bounds; 128-byte swizzle unless swizzle128 is false
 attuner_status make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
-                        const uint64_t* strides, const uint32_t* box, const char* what);
+                        const uint64_t* strides, const uint32_t* box, const char* what,
+                        bool swizzle128 = true);
 attuner_status set_device(const attuner_ctx* ctx);
 bool aligned16(const void* p);
 PlanDev plan_dev(const attuner_plan* p);

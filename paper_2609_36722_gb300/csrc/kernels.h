@@ -11,32 +11,31 @@
 
 namespace att {
 
-// K1: LoRA down-projection u = s * (A x) (bf16, zero-padded to 64 columns),
-// B zero-padded to 64 columns, and the RoPE cos/sin table of every query row.
+// K1: the RoPE cos/sin table of every query row; also clears the split-K
+// counters of K1b for this call.
 struct PrepParams {
-  const __nv_bfloat16* x;        // [M, hidden]
-  const __nv_bfloat16* lora_a;   // [r, hidden] or nullptr
-  const __nv_bfloat16* lora_b;   // [d_q, r] or nullptr
-  __nv_bfloat16* u_pad;          // [M, 64]
-  __nv_bfloat16* b_pad;          // [d_q, 64]
-  float2* rope;                  // [M, D/2] (cos, sin)
+  float2* rope;                  // [D/2, M] (cos, sin), pair-major
   const int32_t* t_art;          // [n_req]
-  int32_t M, hidden, r, d_q, D, S, S_kv;
-  float s;
+  int32_t* counters;             // [n_counters] split-K arrival counters, or nullptr
+  int32_t n_counters;
+  int32_t M, D, S, S_kv;
   double inv_freq[64];           // theta^(-2j/D), j < D/2 (computed on the host in double)
 };
 
-// K1b: Q = RoPE(RMSNorm([x | u] [W_q | B]^T) * w)  (tcgen05 GEMM + epilogue)
+// K1b: Q = RoPE(RMSNorm(x W_q^T + s * bf16(x A^T) B^T) * w) as one tcgen05
+// GEMM (A stacked under W_q: one MMA of N = D + r) with a fused epilogue.
 struct QprojParams {
   CUtensorMap tm_x;    // x [M, hidden], box 64 x 128, SW128
   CUtensorMap tm_w;    // W_q [d_q, hidden], box 64 x D, SW128
-  CUtensorMap tm_u;    // u_pad [M, 64], box 64 x 128
-  CUtensorMap tm_b;    // b_pad [d_q, 64], box 64 x D
+  CUtensorMap tm_a;    // A [r, hidden], box 64 x n_lora, SW128 (rows past r read as zeros)
+  CUtensorMap tm_b;    // B [d_q, r], box 8 x D, no swizzle (columns past r read as zeros)
   __nv_bfloat16* q_out;            // [M, Hq, D]
   const __nv_bfloat16* qnorm_w;    // [D]
-  const float2* rope;              // [M, D/2]
-  int32_t M, hidden, Hq, lora_ksteps;
-  float eps;
+  const float2* rope;              // [D/2, M] (cos, sin), pair-major
+  float* part;                     // split-K partials [tiles][ksplit][128][D + n_lora]
+  int32_t* counters;               // [tiles] arrivals per output tile (zero on entry)
+  int32_t M, hidden, Hq, r, n_lora, ksplit;
+  float s, eps;
   int* status;
   long long wait_limit;
 };

@@ -2,11 +2,11 @@
 //   * pool_write: copy one artifact's K/V ([L, Hkv, D], Sec. 2 Eq. full-vs-pic:
 //     encoded alone at local positions, never changed afterwards) into its
 //     paged pool blocks [block][Hkv][64][D];
-//   * prep: per query row, the LoRA down-projection u = s * (A x) of
-//     Sec. 3 Eq. (query-adaptation), rounded to bf16 and zero-padded to 64
-//     columns (one extra K block of the Q-projection GEMM), the cos/sin table
-//     of the row's RoPE angles, and B zero-padded to 64 columns.
+//   * prep: the cos/sin table of every query row's RoPE angles (App. A.5
+//     position ids of the assembled context).
 #include <math.h>
+
+#include <algorithm>
 
 #include "kernels.h"
 
@@ -44,90 +44,30 @@ cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __
   return cudaGetLastError();
 }
 
-__device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float* f) {
-  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    float2 t = __bfloat1622float2(h[i]);
-    f[2 * i] = t.x;
-    f[2 * i + 1] = t.y;
-  }
-}
-
-// One launch, three independent jobs selected by block index:
-//   [0, nb_lora)            one warp per (query row, 4 LoRA outputs): u = s * (A x)
-//   [nb_lora, +nb_rope)     one thread per (query row, rotary pair): cos/sin table
-//   [.., +nb_b)             one thread per 16 bytes of b_pad
-__global__ void __launch_bounds__(256) prep_kernel(const __grid_constant__ PrepParams p, int nb_lora,
-                                                   int nb_rope) {
-  const int bid = blockIdx.x;
-  if (bid < nb_lora) {
-    const int warp = (bid * 256 + (int)threadIdx.x) >> 5, lane = threadIdx.x & 31;
-    const int groups = 16;                       // 64 padded columns / 4 per warp
-    const int m = warp / groups, jg = warp % groups;
-    if (m >= p.M) return;
-    const int j0 = jg * 4;
-    if (j0 >= p.r) {                             // zero padding columns r..63
-      if (lane < 4) p.u_pad[(long long)m * 64 + j0 + lane] = __float2bfloat16_rn(0.f);
-      return;
-    }
-    const __nv_bfloat16* xr = p.x + (long long)m * p.hidden;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 2
-    for (int k = lane * 8; k < p.hidden; k += 256) {
-      float xf[8];
-      bf16x8_to_f32(*reinterpret_cast<const uint4*>(xr + k), xf);
-#pragma unroll
-      for (int jj = 0; jj < 4; ++jj) {
-        float af[8];
-        bf16x8_to_f32(*reinterpret_cast<const uint4*>(p.lora_a + (long long)(j0 + jj) * p.hidden + k), af);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc[jj] = fmaf(af[e], xf[e], acc[jj]);
-      }
-    }
-#pragma unroll
-    for (int jj = 0; jj < 4; ++jj) {
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) acc[jj] += __shfl_xor_sync(0xffffffffu, acc[jj], o);
-    }
-    if (lane < 4) {
-      float v = lane == 0 ? acc[0] : lane == 1 ? acc[1] : lane == 2 ? acc[2] : acc[3];
-      p.u_pad[(long long)m * 64 + j0 + lane] = __float2bfloat16_rn(p.s * v);
-    }
-    return;
-  }
-  if (bid < nb_lora + nb_rope) {
-    // RoPE angle of (row m, pair j): pos * theta^(-2j/D), pos = T_art(req) + (S_kv - S) + i.
-    // Formed and reduced modulo 2*pi in double, then sin/cos in float on |angle| <= pi.
-    const int half = p.D / 2;
-    const long long idx = (long long)(bid - nb_lora) * 256 + threadIdx.x;
-    if (idx >= (long long)p.M * half) return;
-    const int m = (int)(idx / half), j = (int)(idx % half);
-    const int req = m / p.S, i = m % p.S;
-    const long long pos = (long long)p.t_art[req] + (p.S_kv - p.S) + i;
-    const double ang = (double)pos * p.inv_freq[j];
-    const double k = rint(ang * 0.15915494309189533577);   // 1 / (2 pi)
-    const double red = fma(-k, 6.283185307179586232, ang);
-    float sn, cs;
-    sincosf((float)red, &sn, &cs);
-    p.rope[idx] = make_float2(cs, sn);
-    return;
-  }
-  // b_pad[n][0..63] = B[n][0..r-1], zeros beyond
-  const long long idx = (long long)(bid - nb_lora - nb_rope) * 256 + threadIdx.x;
-  if (idx >= (long long)p.d_q * 8) return;
-  const int n = (int)(idx / 8), c = (int)(idx % 8);
-  uint4 val = make_uint4(0, 0, 0, 0);
-  if (c * 8 < p.r) val = *reinterpret_cast<const uint4*>(p.lora_b + (long long)n * p.r + c * 8);
-  *reinterpret_cast<uint4*>(p.b_pad + (long long)n * 64 + c * 8) = val;
+// One thread per (query row, rotary pair): the RoPE angle pos * theta^(-2j/D)
+// with pos = T_art(req) + (S_kv - S) + i (App. A.5: positions of the
+// assembled context), formed and reduced modulo 2*pi in double, then sin/cos
+// in float on |angle| <= pi.  The first threads also clear the split-K
+// arrival counters the Q-projection kernel uses in this call.
+__global__ void __launch_bounds__(256) prep_kernel(const __grid_constant__ PrepParams p) {
+  const long long idx = (long long)blockIdx.x * 256 + threadIdx.x;
+  if (p.counters != nullptr && idx < p.n_counters) p.counters[idx] = 0;
+  const int half = p.D / 2;
+  if (idx >= (long long)p.M * half) return;
+  const int j = (int)(idx / p.M), m = (int)(idx % p.M);   // pair-major: coalesced in the epilogue
+  const int req = m / p.S, i = m % p.S;
+  const long long pos = (long long)p.t_art[req] + (p.S_kv - p.S) + i;
+  const double ang = (double)pos * p.inv_freq[j];
+  const double k = rint(ang * 0.15915494309189533577);   // 1 / (2 pi)
+  const double red = fma(-k, 6.283185307179586232, ang);
+  float sn, cs;
+  sincosf((float)red, &sn, &cs);
+  p.rope[(long long)j * p.M + m] = make_float2(cs, sn);
 }
 
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st) {
-  const bool lora = p.lora_a != nullptr && p.lora_b != nullptr && p.r > 0;
-  const int nb_lora = lora ? (p.M * 16 * 32 + 255) / 256 : 0;
-  const int nb_rope = (int)(((long long)p.M * (p.D / 2) + 255) / 256);
-  const int nb_b = lora ? (p.d_q * 8 + 255) / 256 : 0;
-  prep_kernel<<<nb_lora + nb_rope + nb_b, 256, 0, st>>>(p, nb_lora, nb_rope);
+  const long long n = std::max<long long>((long long)p.M * (p.D / 2), p.n_counters);
+  prep_kernel<<<(int)((n + 255) / 256), 256, 0, st>>>(p);
   return cudaGetLastError();
 }
 

@@ -1,31 +1,185 @@
 // qproj.cu - K1b: the adapted query projection of Sec. 3, Eq.
 // (query-adaptation), followed by the model's original query RMSNorm and
-// RoPE, as ONE tcgen05 GEMM with a fused epilogue:
+// RoPE, as one tcgen05 GEMM with a fused epilogue:
 //
-//   Q[m, h, :] = RoPE( RMSNorm( [x_m | u_m] . [W_q | B]_h^T ) * w, pos_m )
-//
-// where u = s * (A x) (bf16, from prep.cu).  Concatenating along K turns the
-// low-rank update into one more 64-wide K block of the same GEMM (only
-// ceil(r/16) of its four 16-wide MMA steps are issued).
+//   Q[m, h, :] = RoPE( RMSNorm( x_m W_q,h^T + bf16(s * x_m A^T) B_h^T ) * w, pos_m )
 //
 // CTA tile: 128 query rows x one head (N = D = 64 or 128), so every
 // accumulator row holds a whole head and the RMSNorm needs no cross-CTA
-// reduction.  Warp 0: TMA producer; warp 1: TMEM owner + MMA issuer; warps
-// 2..5: epilogue (one accumulator row per thread, tcgen05.ld 32x32b).
+// reduction of its own.  Each K block loads the x tile, the W_q rows of the
+// head and, right below them, the r rows of the LoRA A matrix, so ONE MMA of
+// N = D + r produces both x W_q,h^T (columns 0..D-1) and u = x A^T (columns
+// D..D+r-1).  After the K loop the epilogue writes bf16(s * u) as a small
+// K-major tile in shared memory and one MMA with B_h (loaded by TMA at the
+// start) adds the rank-r update into a second TMEM accumulator.
+//
+// When (row tiles x heads) cannot fill the GPU (decode, short suffixes) the
+// K dimension is split over up to 4 CTAs per tile; each publishes its fp32
+// partial accumulators and the last CTA to arrive (an atomic counter per
+// tile, cleared by the prep kernel of the same call) sums all of them in
+// split order (the result does not depend on arrival order) and finishes.
+//
+// Warp 0: TMA producer; warp 1: TMEM owner + MMA issuer; warps 2..5:
+// epilogue (one accumulator row per thread, tcgen05.ld 32x32b).
 #include "kernels.h"
 
 namespace att {
 
 template <int D>
 struct QpLayout {
-  static constexpr int NS = (D == 128) ? 6 : 8;
-  static constexpr int A_BYTES = 128 * 128;   // 128 rows x 64 bf16
-  static constexpr int B_BYTES = D * 128;     // D rows x 64 bf16
-  static constexpr int STAGE = A_BYTES + B_BYTES;
-  static constexpr int BAR_OFF = NS * STAGE;
-  static constexpr int SMEM = BAR_OFF + 512 + 1024;   // + alignment slack
-  static constexpr uint32_t TMEM_COLS = (D < 32) ? 32 : D;
+  static constexpr int X_BYTES = 128 * 128;   // x tile: 128 rows x 64 bf16
+  static constexpr int W_BYTES = D * 128;     // W_q rows of the head, then...
+  static constexpr int A_BYTES = 64 * 128;    // ...up to 64 rows of the LoRA A matrix
+  static constexpr int STAGE = X_BYTES + W_BYTES + A_BYTES;
+  static constexpr int NS = (D == 128) ? 5 : 6;
+  static constexpr int B_OFF = NS * STAGE;               // B_h: [r/8][D rows][8 bf16]
+  static constexpr int B_BYTES = 64 * D * 2;
+  static constexpr int BAR_OFF = B_OFF + B_BYTES;
+  static constexpr int SMEM = BAR_OFF + 512 + 1024;     // + alignment slack
+  static constexpr uint32_t TMEM_COLS = 512;            // [x W^T | x A^T] at 0, LoRA update at 256
+  static constexpr uint32_t LUP_COL = 256;
 };
+
+// Shared-memory matrix descriptor, no swizzle (canonical K-major layout of
+// 8-row x 16-byte core matrices): lbo = byte distance between the two
+// 8-element K halves of a core-matrix pair, sbo = between 8-row groups.
+ATT_DEV uint64_t sdesc_noswz(uint32_t saddr, uint32_t lbo_bytes, uint32_t sbo_bytes) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo_bytes >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo_bytes >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  return d;
+}
+
+enum : int { QB_ACC = 0, QB_LORA = 1, QB_LUP = 2, QB_DRAIN = 3, QB_FULL = 4 };   // + NS full, NS empty
+
+// Epilogue of one accumulator row per thread (warps 2..5).  R = LoRA rank
+// rounded up to 16 (0: no adapter).
+template <int D, int R>
+__device__ __forceinline__ void qproj_epilogue(const QprojParams& p, uint32_t sbase, uint32_t tmem,
+                                               uint64_t* bars, volatile int* abort_flag,
+                                               volatile int* last_flag, int head, int ks, int tile,
+                                               int m0) {
+  using L = QpLayout<D>;
+  constexpr int RU = R > 0 ? R : 1;
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int q = warp & 3;
+  const int r = q * 32 + lane;
+  const int et = threadIdx.x - 64;     // 0..127 within the epilogue warps
+  const int m = m0 + r;
+  const uint32_t row_t = tmem + ((uint32_t)(q * 32) << 16);
+  constexpr int rowlen = D + R;
+  auto bar = [&](int i) { return smem_u32(&bars[i]); };
+
+  float v[D];
+  float u[RU];
+#pragma unroll
+  for (int c = 0; c < D / 32; ++c) tmem_ld32(row_t + c * 32, v + c * 32);
+  if (R == 16) {
+    float t[32];
+    tmem_ld32(row_t + D, t);            // columns past D + 16 are not used
+    tc_wait_ld();
+#pragma unroll
+    for (int j = 0; j < RU; ++j) u[j] = t[j];
+  } else {
+#pragma unroll
+    for (int c = 0; c < R / 32; ++c) tmem_ld32(row_t + D + c * 32, u + c * 32);
+    tc_wait_ld();
+  }
+  if (p.ksplit > 1) {
+    float* mine = p.part + (((long long)tile * p.ksplit + ks) * 128 + r) * rowlen;
+#pragma unroll
+    for (int c = 0; c < D; c += 4) *reinterpret_cast<float4*>(mine + c) = make_float4(v[c], v[c + 1], v[c + 2], v[c + 3]);
+#pragma unroll
+    for (int c = 0; c < R; c += 4) *reinterpret_cast<float4*>(mine + D + c) = make_float4(u[c], u[c + 1], u[c + 2], u[c + 3]);
+    __threadfence();
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (et == 0) *last_flag = (atomicAdd(&p.counters[tile], 1) == p.ksplit - 1) ? 1 : 0;
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (*last_flag == 0) return;          // CTA-uniform: another CTA finishes this tile
+    __threadfence();
+    // every split's partial (this CTA's too), in split order
+#pragma unroll
+    for (int c = 0; c < D; ++c) v[c] = 0.f;
+#pragma unroll
+    for (int c = 0; c < RU; ++c) u[c] = 0.f;
+    for (int kk = 0; kk < p.ksplit; ++kk) {
+      const float* part = p.part + (((long long)tile * p.ksplit + kk) * 128 + r) * rowlen;
+#pragma unroll
+      for (int c = 0; c < D; c += 4) {
+        const float4 o = __ldcg(reinterpret_cast<const float4*>(part + c));
+        v[c] += o.x; v[c + 1] += o.y; v[c + 2] += o.z; v[c + 3] += o.w;
+      }
+#pragma unroll
+      for (int c = 0; c < R; c += 4) {
+        const float4 o = __ldcg(reinterpret_cast<const float4*>(part + D + c));
+        u[c] += o.x; u[c + 1] += o.y; u[c + 2] += o.z; u[c + 3] += o.w;
+      }
+    }
+  }
+  if (R > 0) {
+    // U = bf16(s * u) as a K-major tile [R/8][128 rows][8] in the idle stage ring,
+    // then one MMA per 16 of R: LoRA update (TMEM at LUP_COL) = U B_h^T
+#pragma unroll
+    for (int g = 0; g < R / 8; ++g) {
+      uint32_t w[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int j0 = g * 8 + 2 * e;
+        w[e] = pack_bf16(j0 < p.r ? p.s * u[j0] : 0.f, j0 + 1 < p.r ? p.s * u[j0 + 1] : 0.f);
+      }
+      st_shared_v4(sbase + g * 2048 + r * 16, w[0], w[1], w[2], w[3]);
+    }
+    fence_proxy_async_smem();
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (et == 0) {
+      if (mbar_wait(bar(QB_LORA), 0, abort_flag, p.wait_limit, p.status)) {
+        tc_fence_after();
+        constexpr uint32_t idesc = idesc_bf16_f32(128, D, 0, 0);
+#pragma unroll
+        for (int kk = 0; kk < R / 16; ++kk)
+          umma_bf16(tmem + L::LUP_COL, sdesc_noswz(sbase + kk * 2 * 2048, 2048, 128),
+                    sdesc_noswz(sbase + L::B_OFF + kk * 2 * (D * 16), D * 16, 128), idesc, kk > 0 ? 1u : 0u);
+        umma_commit(bar(QB_LUP));
+      } else {
+        mbar_arrive(bar(QB_LUP));       // never issued: release the waiters (status already TIMEOUT)
+      }
+    }
+    warp_wait(bar(QB_LUP), 0, abort_flag, p.wait_limit, p.status);
+    tc_fence_after();
+#pragma unroll
+    for (int c = 0; c < D / 32; ++c) {
+      float t[32];
+      tmem_ld32(row_t + L::LUP_COL + c * 32, t);
+      tc_wait_ld();
+#pragma unroll
+      for (int k = 0; k < 32; ++k) v[c * 32 + k] += t[k];
+    }
+  }
+  // RMSNorm * w, RoPE on pairs (j, j + D/2), bf16 store; rows past M store nothing
+  const bool row_ok = m < p.M;
+  const int mr = row_ok ? m : p.M - 1;
+  float ss = 0.f;
+#pragma unroll
+  for (int j = 0; j < D; ++j) ss = fmaf(v[j], v[j], ss);
+  const float rinv = rsqrtf(ss * (1.0f / D) + p.eps);
+#pragma unroll
+  for (int j = 0; j < D / 2; ++j) {
+    const float2 cs = p.rope[(long long)j * p.M + mr];
+    const float a = v[j] * rinv * __bfloat162float(p.qnorm_w[j]);
+    const float b = v[j + D / 2] * rinv * __bfloat162float(p.qnorm_w[j + D / 2]);
+    v[j] = a * cs.x - b * cs.y;
+    v[j + D / 2] = b * cs.x + a * cs.y;
+  }
+  if (row_ok) {
+    uint4* dst = reinterpret_cast<uint4*>(p.q_out + ((long long)m * p.Hq + head) * D);
+#pragma unroll
+    for (int c = 0; c < D / 8; ++c)
+      dst[c] = make_uint4(pack_bf16(v[8 * c], v[8 * c + 1]), pack_bf16(v[8 * c + 2], v[8 * c + 3]),
+                          pack_bf16(v[8 * c + 4], v[8 * c + 5]), pack_bf16(v[8 * c + 6], v[8 * c + 7]));
+  }
+}
 
 template <int D>
 __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ QprojParams p) {
@@ -34,22 +188,28 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sbase = smem_u32(smem);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);
-  // bars[0..NS): full, bars[NS..2NS): empty, bars[2NS]: accumulator ready, bars[2NS+1]: drain
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::BAR_OFF + 384);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 392);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 396);
   auto bar = [&](int i) { return smem_u32(&bars[i]); };
-  const int B_FULL = 0, B_EMPTY = L::NS, B_ACC = 2 * L::NS, B_DRAIN = 2 * L::NS + 1;
+  const int B_FULL = QB_FULL, B_EMPTY = QB_FULL + L::NS;
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int head = blockIdx.x;
+  const int head = blockIdx.x / p.ksplit;
+  const int ks = blockIdx.x % p.ksplit;
+  const int tile = blockIdx.y * p.Hq + head;
   const int m0 = blockIdx.y * 128;
   const int n0 = head * D;
-  const int nk_main = p.hidden / 64;
-  const int nk = nk_main + (p.lora_ksteps > 0 ? 1 : 0);
+  const int nk = p.hidden / 64;
+  const int kb0 = ks * nk / p.ksplit, kb1 = (ks + 1) * nk / p.ksplit;
+  const bool lora = p.n_lora > 0;
+  const int nmma = D + (lora ? p.n_lora : 0);             // N of the main MMA
+  const uint32_t stage_tx = L::X_BYTES + L::W_BYTES + (lora ? p.n_lora * 128 : 0);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2 * L::NS + 2; ++i) mbar_init(bar(i), 1);
+    for (int i = 0; i < QB_FULL + 2 * L::NS; ++i) mbar_init(bar(i), 1);
     *abort_flag = 0;
+    *last_flag = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -65,91 +225,68 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
     if (lane == 0) {
       tma_prefetch_desc(&p.tm_x);
       tma_prefetch_desc(&p.tm_w);
+      if (lora) {
+        // B_h: r/8 boxes of [D rows][8 columns] (columns past r read as zeros)
+        mbar_expect_tx(bar(QB_LORA), (p.n_lora / 8) * D * 16);
+        for (int g = 0; g < p.n_lora / 8; ++g)
+          tma_load_2d(sbase + L::B_OFF + g * D * 16, &p.tm_b, bar(QB_LORA), g * 8, n0);
+      }
       int issued = 0;
-      for (int kb = 0; kb < nk; ++kb) {
-        const int st = kb % L::NS;
-        if (kb >= L::NS &&
-            !mbar_wait(bar(B_EMPTY + st), ((kb / L::NS) - 1) & 1, abort_flag, p.wait_limit, p.status))
+      for (int kb = kb0; kb < kb1; ++kb) {
+        const int it = kb - kb0, st = it % L::NS;
+        if (it >= L::NS &&
+            !mbar_wait(bar(B_EMPTY + st), ((it / L::NS) - 1) & 1, abort_flag, p.wait_limit, p.status))
           break;
-        const uint32_t a_dst = sbase + st * L::STAGE;
-        const uint32_t b_dst = a_dst + L::A_BYTES;
-        mbar_expect_tx(bar(B_FULL + st), L::STAGE);
-        if (kb < nk_main) {
-          tma_load_2d(a_dst, &p.tm_x, bar(B_FULL + st), kb * 64, m0);
-          tma_load_2d(b_dst, &p.tm_w, bar(B_FULL + st), kb * 64, n0);
-        } else {
-          tma_load_2d(a_dst, &p.tm_u, bar(B_FULL + st), 0, m0);
-          tma_load_2d(b_dst, &p.tm_b, bar(B_FULL + st), 0, n0);
-        }
-        issued = kb + 1;
+        const uint32_t x_dst = sbase + st * L::STAGE;
+        mbar_expect_tx(bar(B_FULL + st), stage_tx);
+        tma_load_2d(x_dst, &p.tm_x, bar(B_FULL + st), kb * 64, m0);
+        tma_load_2d(x_dst + L::X_BYTES, &p.tm_w, bar(B_FULL + st), kb * 64, n0);
+        if (lora) tma_load_2d(x_dst + L::X_BYTES + L::W_BYTES, &p.tm_a, bar(B_FULL + st), kb * 64, 0);
+        issued = it + 1;
       }
       if (*abort_flag) {   // let every copy this CTA issued land before exiting
-        for (int kb = (issued > L::NS ? issued - L::NS : 0); kb < issued; ++kb)
-          mbar_drain(bar(B_FULL + kb % L::NS), (kb / L::NS) & 1, p.status);
+        if (lora) mbar_drain(bar(QB_LORA), 0, p.status);
+        for (int it = (issued > L::NS ? issued - L::NS : 0); it < issued; ++it)
+          mbar_drain(bar(B_FULL + it % L::NS), (it / L::NS) & 1, p.status);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(128, D, 0, 0);
+      const uint32_t idesc = idesc_bf16_f32(128, nmma, 0, 0);
       bool ok = true;
       bool any = false;
-      for (int kb = 0; kb < nk; ++kb) {
-        const int st = kb % L::NS;
-        if (!mbar_wait(bar(B_FULL + st), (kb / L::NS) & 1, abort_flag, p.wait_limit, p.status)) {
+      for (int kb = kb0; kb < kb1; ++kb) {
+        const int it = kb - kb0, st = it % L::NS;
+        if (!mbar_wait(bar(B_FULL + st), (it / L::NS) & 1, abort_flag, p.wait_limit, p.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t a_s = sbase + st * L::STAGE;
-        const uint32_t b_s = a_s + L::A_BYTES;
-        const int ksteps = (kb < nk_main) ? 4 : p.lora_ksteps;
-        for (int k = 0; k < ksteps; ++k) {
-          umma_bf16(tmem, sdesc_sw128(a_s + k * 32, 16, 1024), sdesc_sw128(b_s + k * 32, 16, 1024),
-                    idesc, (kb > 0 || k > 0) ? 1u : 0u);
-          any = true;
-        }
+        const uint32_t x_s = sbase + st * L::STAGE;
+        const uint32_t w_s = x_s + L::X_BYTES;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          umma_bf16(tmem, sdesc_sw128(x_s + k * 32, 16, 1024), sdesc_sw128(w_s + k * 32, 16, 1024), idesc,
+                    (it > 0 || k > 0) ? 1u : 0u);
+        any = true;
         umma_commit(bar(B_EMPTY + st));
       }
       if (ok) {
-        umma_commit(bar(B_ACC));
+        umma_commit(bar(QB_ACC));
       } else if (any) {
-        umma_commit(bar(B_DRAIN));
-        mbar_drain(bar(B_DRAIN), 0, p.status);
+        umma_commit(bar(QB_DRAIN));
+        mbar_drain(bar(QB_DRAIN), 0, p.status);
       }
     }
   } else {
     // epilogue: warps 2..5 -> TMEM lane quadrants 2, 3, 0, 1
-    const int q = warp & 3;
-    const int r = q * 32 + lane;
-    const int m = m0 + r;
-    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-    if (warp_wait(bar(B_ACC), 0, abort_flag, p.wait_limit, p.status)) {
+    if (warp_wait(bar(QB_ACC), 0, abort_flag, p.wait_limit, p.status)) {
       tc_fence_after();
-      float v[D];
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) tmem_ld32(tmem + lane_base + c * 32, v + c * 32);
-      tc_wait_ld();
-      if (m < p.M) {
-        float ss = 0.f;
-#pragma unroll
-        for (int j = 0; j < D; ++j) ss = fmaf(v[j], v[j], ss);
-        const float rinv = rsqrtf(ss * (1.0f / D) + p.eps);
-#pragma unroll
-        for (int j = 0; j < D; ++j) v[j] = v[j] * rinv * __bfloat162float(p.qnorm_w[j]);
-        const float2* rp = p.rope + (long long)m * (D / 2);
-#pragma unroll
-        for (int j = 0; j < D / 2; ++j) {
-          const float2 cs = rp[j];
-          const float a = v[j], b = v[j + D / 2];
-          v[j] = a * cs.x - b * cs.y;
-          v[j + D / 2] = b * cs.x + a * cs.y;
-        }
-        uint4* dst = reinterpret_cast<uint4*>(p.q_out + ((long long)m * p.Hq + head) * D);
-#pragma unroll
-        for (int c = 0; c < D / 8; ++c)
-          dst[c] = make_uint4(pack_bf16(v[8 * c], v[8 * c + 1]), pack_bf16(v[8 * c + 2], v[8 * c + 3]),
-                              pack_bf16(v[8 * c + 4], v[8 * c + 5]), pack_bf16(v[8 * c + 6], v[8 * c + 7]));
-      }
+      const int nl = lora ? p.n_lora : 0;
+      if (nl == 0) qproj_epilogue<D, 0>(p, sbase, tmem, bars, abort_flag, last_flag, head, ks, tile, m0);
+      else if (nl <= 16) qproj_epilogue<D, 16>(p, sbase, tmem, bars, abort_flag, last_flag, head, ks, tile, m0);
+      else if (nl <= 32) qproj_epilogue<D, 32>(p, sbase, tmem, bars, abort_flag, last_flag, head, ks, tile, m0);
+      else qproj_epilogue<D, 64>(p, sbase, tmem, bars, abort_flag, last_flag, head, ks, tile, m0);
     }
   }
   tc_fence_before();
@@ -163,13 +300,9 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
 template <int D>
 static cudaError_t launch_qproj_t(const QprojParams& p, cudaStream_t st) {
   using L = QpLayout<D>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(qproj_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
-  dim3 grid(p.Hq, (p.M + 127) / 128);
+  cudaError_t e = cudaFuncSetAttribute(qproj_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
+  if (e != cudaSuccess) return e;
+  dim3 grid(p.Hq * p.ksplit, (p.M + 127) / 128);
   qproj_kernel<D><<<grid, 192, L::SMEM, st>>>(p);
   return cudaGetLastError();
 }

@@ -59,9 +59,12 @@ def test_assemble_bit_exact_tiny(tiny):
     assert torch.equal(v_tok.view(torch.int16), v_cat.view(torch.int16))
 
 
-def test_q_project_tiny(tiny):
+@pytest.mark.parametrize("split_k", [1, 2])
+def test_q_project_tiny(tiny, split_k):
+    import paper_2609_36722_gb300 as pkg
     wl, _ = tiny
     ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_QPROJ_SPLIT_K, split_k)
     g = wl.geom
     q = ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv)
     assert ctx.sync_status() == 0
@@ -124,3 +127,17 @@ def test_decode_shape():
     ctx, plan = load_context(wl)
     out, lse = run_path(ctx, plan, wl)
     compare(_np(out), o_ref, _np(lse), lse_ref, label="decode")
+
+
+@pytest.mark.parametrize("split_k", [2, 4])
+def test_q_project_split_k_matches_oracle(split_k):
+    import paper_2609_36722_gb300 as pkg
+    wl = make_custom("qsplit", G128, 13, [100], [[0]], 40, 40, device=DEV)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_QPROJ_SPLIT_K, split_k)
+    g = wl.geom
+    q = ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv)
+    assert ctx.sync_status() == 0
+    q_ref = oracle.workload_reference(wl, 0, q_only=True)
+    err = np.abs(_np(q[0]) - q_ref)
+    assert err.max() <= Q_MAX_ABS, err.max()
