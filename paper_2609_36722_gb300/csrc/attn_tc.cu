@@ -97,25 +97,19 @@ __device__ __forceinline__ void load_slot(uint32_t dst, int e, const CUtensorMap
   }
 }
 
-// Mask one 64-key block slot in place: artifact block tail (slot >= valid),
-// suffix causality (key > lim), or an empty slot.
-__device__ __forceinline__ void mask_slot(float* v, int e, int lim) {
-  if (e > 0) {
-    const int valid = e & 127;
-    if (valid < kBlockTokens) {
+// Visible keys of one 64-key block slot for a query row: every slot reduces
+// to "the first n keys are visible" -- an artifact block's valid length, the
+// causal prefix of a suffix chunk (keys <= lim), or 0 for an empty slot.
+__device__ __forceinline__ int slot_visible(int e, int lim) {
+  if (e > 0) return e & 127;
+  if (e < 0) return min(max(lim - (-e - 1) * kBlockTokens + 1, 0), kBlockTokens);
+  return 0;
+}
+
+// -inf for keys past n_vis in a 64-key slot
+__device__ __forceinline__ void mask_tail(float* v, int n_vis) {
 #pragma unroll
-      for (int c = 0; c < 64; ++c) if (c >= valid) v[c] = -INFINITY;
-    }
-  } else if (e < 0) {
-    const int kbase = (-e - 1) * kBlockTokens;
-    if (kbase + kBlockTokens - 1 > lim) {
-#pragma unroll
-      for (int c = 0; c < 64; ++c) if (kbase + c > lim) v[c] = -INFINITY;
-    }
-  } else {
-#pragma unroll
-    for (int c = 0; c < 64; ++c) v[c] = -INFINITY;
-  }
+  for (int c = 0; c < 64; ++c) v[c] = (c < n_vis) ? v[c] : -INFINITY;
 }
 
 template <int D>
@@ -317,8 +311,14 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
 #pragma unroll
       for (int c = 0; c < 4; ++c) tmem_ld32(s_col + c * 32, sc + c * 32);
       tc_wait_ld();
-      mask_slot(sc, list[2 * j], lim);
-      mask_slot(sc + 64, list[2 * j + 1], lim);
+      {
+        // most tiles are fully visible: one warp vote skips the masking code
+        const int nv0 = slot_visible(list[2 * j], lim), nv1 = slot_visible(list[2 * j + 1], lim);
+        if (__any_sync(0xffffffffu, min(nv0, nv1) < kBlockTokens)) {
+          mask_tail(sc, nv0);
+          mask_tail(sc + 64, nv1);
+        }
+      }
       // row max: eight independent chains of 3-input max, then a small tree
       float mk[8];
 #pragma unroll
