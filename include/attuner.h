@@ -174,10 +174,13 @@ attuner_status attuner_attend(attuner_ctx* ctx, const attuner_plan* plan, const 
  *     (cudaGetSymbolAddress), so make that first call outside any stream
  *     capture.
  *   - Every call shares the array and it keeps the last call's contents
- *     (nothing in it needs to start at zero).  Calls whose kernels overlap on
- *     the GPU race on it: order them (one stream, or events).
+ *     (nothing in it needs to start at zero; the call clears the arrival
+ *     counters it keeps there with cudaMemsetAsync on `stream`).  Calls
+ *     whose kernels overlap on the GPU race on it: order them (one stream,
+ *     or events).
  *   - A call whose partial results would need more than 32 MiB
- *     (n_split_ctas * rows_per_cta * (d + 1) * 4 bytes) is rejected with
+ *     (n_split_ctas * rows_per_cta * (d + 1) * 4 bytes, plus 4 bytes per
+ *     (request, KV head, row tile) for the tcgen05 kernel) is rejected with
  *     INVALID_ARG before anything is launched; use attuner_attend for it.
  * Errors: as attuner_attend, plus INVALID_ARG for a call beyond the limit. */
 attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const attuner_plan* plan,
@@ -211,11 +214,18 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
  *   ATTUNER_OPT_QPROJ_SPLIT_K  most CTAs (1..4) that split the K dimension of one
  *                               Q-projection tile when the tiles alone leave SMs
  *                               idle (0 or 1 = no split, the default)
+ *   ATTUNER_OPT_SPLIT_MERGE     how the tcgen05 kernel merges the split-KV
+ *                               chunks of a row tile: 0 auto (cost model),
+ *                               1 independent CTAs merged through global memory
+ *                               by the last one to finish, 2 one thread-block
+ *                               cluster per row tile (2..8 chunks) merged
+ *                               through distributed shared memory
  *   ATTUNER_OPT_TEST_STUCK_WAIT see below */
 #define ATTUNER_OPT_PREFILL_KERNEL 1
 #define ATTUNER_OPT_SPLIT_BLOCKS   2
 #define ATTUNER_OPT_WAIT_LIMIT     3
 #define ATTUNER_OPT_QPROJ_SPLIT_K  4
+#define ATTUNER_OPT_SPLIT_MERGE    5
 /* Test hook (failure detection without a GPU fault): while non-zero, one
  * role of every attention launch waits on an mbarrier that nothing arrives
  * at; its bounded wait runs out, the kernel drains its own copies, frees its

@@ -16,8 +16,10 @@
 // exits.  All calls share it, so two calls whose kernels overlap on the GPU
 // (different streams, or different contexts on the same device) race on it;
 // the caller must order such calls.  It keeps the last call's contents:
-// nothing in it needs to start at zero, because every partial result the
-// combine kernel reads is written earlier in the same call.
+// nothing in it needs to start at zero, because every partial result a merge
+// reads is written earlier in the same call, and the call clears the few
+// arrival counters it keeps there itself (cudaMemsetAsync, which allocates
+// nothing).
 #include <mutex>
 
 #include "internal.h"
@@ -75,10 +77,14 @@ extern "C" attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const 
   const int rows = tc ? kTcRows : kMmaRows;
 
   AttnParams ap{};   // on the stack: this entry point touches no heap
+  if (tc) query_cluster_occupancy(ctx);
   make_work(ctx, plan, S, S_kv, tc, ap.work);
-  bool need_combine = false;
+  bool need_combine = false;   // split partial results in global memory
   for (int r = 0; r < plan->n_req; ++r) need_combine |= (ap.work.nsplit[r] > 1);
-  const size_t part_bytes = need_combine ? (size_t)ap.work.n_cta * rows * (D + 1) * 4 : 0;
+  if (ap.work.cluster > 0) need_combine = false;
+  const size_t pb = need_combine ? (size_t)ap.work.n_cta * rows * (D + 1) * 4 : 0;
+  const size_t units = (size_t)plan->n_req * Hkv * ap.work.row_tiles;
+  const size_t part_bytes = pb + ((need_combine && tc) ? units * 4 : 0);
   if (part_bytes > kStaticScratchBytes)
     return fail(ATTUNER_ERR_INVALID_ARG,
                 "attuner_attend_static_scratch: this call needs " + std::to_string(part_bytes) +
@@ -116,14 +122,19 @@ extern "C" attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const 
   ap.status = ctx->d_status;
   ap.wait_limit = ctx->wait_limit;
   ap.inject_stuck = ctx->inject_stuck;
+  cudaError_t ce = cudaSuccess;
   if (need_combine) {
     ap.part_o = static_cast<float*>(scratch);
     ap.part_lse = static_cast<float*>(scratch) + (size_t)ap.work.n_cta * rows * D;
+    if (tc) {   // arrival counters of the in-kernel split merge
+      ap.unit_cnt = reinterpret_cast<int*>(static_cast<char*>(scratch) + pb);
+      ce = cudaMemsetAsync(ap.unit_cnt, 0, units * 4, st);
+    }
   }
   int launches = 0;
-  cudaError_t ce = tc ? launch_attn_tc(ap, D, st) : launch_attn_mma(ap, D, st);
+  if (ce == cudaSuccess) ce = tc ? launch_attn_tc(ap, D, st) : launch_attn_mma(ap, D, st);
   if (ce == cudaSuccess) ++launches;
-  if (ce == cudaSuccess && need_combine) {
+  if (ce == cudaSuccess && need_combine && !tc) {
     CombineParams cp{};
     cp.work = ap.work;
     cp.part_o = ap.part_o;

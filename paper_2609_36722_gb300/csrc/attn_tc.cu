@@ -61,7 +61,9 @@ static_assert(128 * kCtrlRegs + 256 * kSoftRegs <= 384 * 168, "register split ex
 
 enum : int {
   B_Q = 0, B_KF = 1, B_VF = 3, B_KE = 5, B_VE = 7, B_SF = 9, B_PF = 11,
-  B_O = 13, B_DRAIN = 14, B_NEVER = 15, B_COUNT = 16
+  B_O = 13, B_DRAIN = 14, B_NEVER = 15,
+  B_MF = 16, B_ME = 24,   // split merge: full / empty barriers of up to 8 staging buffers
+  B_COUNT = 32
 };
 
 // D[tmem] (+)= A[tmem] * B[smem desc]: A (M x 16 bf16 per step) read from TMEM,
@@ -112,6 +114,46 @@ __device__ __forceinline__ void mask_tail(float* v, int n_vis) {
   for (int c = 0; c < 64; ++c) v[c] = (c < n_vis) ? v[c] : -INFINITY;
 }
 
+// Which (request, KV head, row tile, split) a CTA owns, and its KV chunk size
+// in blocks.  Independent splits: CTAs in [request][split][kv head][row tile]
+// order.  Cluster mode: one cluster per (request, kv head, row tile), split =
+// rank, every request cut into `cluster` chunks of whole 128-key tiles.
+struct TcCta {
+  int req, rt, kvh, split, nsplit, chunk;
+};
+__device__ __forceinline__ TcCta tc_cta(const AttnParams& p, int cta) {
+  TcCta c;
+  if (p.work.cluster > 0) {
+    const int ns = p.work.cluster, unit = cta / ns, per_req = p.Hkv * p.work.row_tiles;
+    c.split = cta % ns;
+    c.nsplit = ns;
+    c.req = unit / per_req;
+    const int rem = unit % per_req;
+    c.rt = rem % p.work.row_tiles;
+    c.kvh = rem / p.work.row_tiles;
+    const int nv = p.plan.blk_off[c.req + 1] - p.plan.blk_off[c.req] + (p.S_kv + kBlockTokens - 1) / kBlockTokens;
+    c.chunk = (((nv + ns - 1) / ns) + 1) & ~1;
+  } else {
+    c.req = find_req(p.work, cta);
+    int rel = cta - p.work.base[c.req];
+    c.rt = rel % p.work.row_tiles;
+    rel /= p.work.row_tiles;
+    c.kvh = rel % p.Hkv;
+    c.split = rel / p.Hkv;
+    c.nsplit = p.work.nsplit[c.req];
+    c.chunk = p.work.chunk_blocks;
+  }
+  return c;
+}
+
+// the CTA index, read so that the compiler recomputes what derives from it
+// instead of keeping it in registers across the main loop
+__device__ __forceinline__ int cta_index_fresh() {
+  int v;
+  asm volatile("mov.u32 %0, %%ctaid.x;" : "=r"(v));
+  return v;
+}
+
 template <int D>
 __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__ AttnParams p) {
   using L = TcLayout<D>;
@@ -121,6 +163,7 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::BAR_OFF + 512);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 520);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 524);
   int* list = reinterpret_cast<int*>(smem + L::LIST_OFF);
   auto bar = [&](int i) { return smem_u32(&bars[i]); };
 
@@ -129,21 +172,16 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
 
   // ---- which (request, kv head, row tile, split) this CTA owns
   const int cta = blockIdx.x;
-  const int req = find_req(p.work, cta);
-  int rel = cta - p.work.base[req];
-  const int rt = rel % p.work.row_tiles;
-  rel /= p.work.row_tiles;
-  const int kvh = rel % p.Hkv;
-  const int split = rel / p.Hkv;
-  const int nsplit = p.work.nsplit[req];
+  const TcCta cw = tc_cta(p, cta);
+  const int req = cw.req, rt = cw.rt, kvh = cw.kvh;
   const int boff = p.plan.blk_off[req];
   const int nab = p.plan.blk_off[req + 1] - boff;
   const int nsuf = (p.S_kv + kBlockTokens - 1) / kBlockTokens;
   const int row0 = rt * kTcRows;
   const int last_row = min(row0 + kTcRows - 1, p.S * G - 1);
   const int last_vis = nab + ((p.S_kv - p.S) + last_row / G) / kBlockTokens;
-  const int b0 = split * p.work.chunk_blocks;
-  const int b1 = min(min(b0 + p.work.chunk_blocks, nab + nsuf), last_vis + 1);
+  const int b0 = cw.split * cw.chunk;
+  const int b1 = min(min(b0 + cw.chunk, nab + nsuf), last_vis + 1);
   const int nblk = max(0, b1 - b0);
   const int ntile = (nblk + 1) / 2;
   const int pool_rows = p.plan.pool_blocks * p.Hkv * kBlockTokens;
@@ -167,7 +205,8 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
     list[i] = e;
   }
   if (threadIdx.x == 0) {
-    for (int i = 0; i < B_COUNT; ++i) mbar_init(bar(i), (i == B_PF || i == B_PF + 1) ? 4u : 1u);
+    for (int i = 0; i < B_COUNT; ++i)
+      mbar_init(bar(i), (i == B_PF || i == B_PF + 1) ? 4u : (i >= B_ME ? 8u : 1u));
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -288,6 +327,11 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
       }
     }
   }
+  // cluster mode: the softmax warps' two cluster barriers count every thread
+  if (p.work.cluster > 0) {
+    cluster_sync_all();
+    cluster_sync_all();
+  }
   } else {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kSoftRegs));
     // ================= softmax + epilogue: warps 0..3 -> Q0, 4..7 -> Q1 =================
@@ -295,7 +339,7 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
     const int quad = warp & 3;
     const int r = qt * kTcTileRows + quad * 32 + lane;   // CTA row
     const int pr = row0 + r;                             // packed row
-    const int tok = pr / G, jh = pr % G;
+    const int tok = pr / G;
     const int lim = (p.S_kv - p.S) + tok;                // last visible suffix key
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const uint32_t s_col = tmem + lane_base + s_col_of(qt);
@@ -310,14 +354,14 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
       float sc[128];
 #pragma unroll
       for (int c = 0; c < 4; ++c) tmem_ld32(s_col + c * 32, sc + c * 32);
+      // while the TMEM loads are in flight: visible keys of the two slots, and
+      // one warp vote (most tiles are fully visible and skip the masking code)
+      const int nv0 = slot_visible(list[2 * j], lim), nv1 = slot_visible(list[2 * j + 1], lim);
+      const bool need_mask = __any_sync(0xffffffffu, min(nv0, nv1) < kBlockTokens);
       tc_wait_ld();
-      {
-        // most tiles are fully visible: one warp vote skips the masking code
-        const int nv0 = slot_visible(list[2 * j], lim), nv1 = slot_visible(list[2 * j + 1], lim);
-        if (__any_sync(0xffffffffu, min(nv0, nv1) < kBlockTokens)) {
-          mask_tail(sc, nv0);
-          mask_tail(sc + 64, nv1);
-        }
+      if (need_mask) {
+        mask_tail(sc, nv0);
+        mask_tail(sc + 64, nv1);
       }
       // row max: eight independent chains of 3-input max, then a small tree
       float mk[8];
@@ -339,24 +383,27 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
       // p = 2^(s * log2(e)/sqrt(d) - m): packed fp32 FMA, then ex2; row sum in packed chains
       const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2), ng2 = f2_pack(neg, neg);
       uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
-      uint32_t pk[64];
+      // P as bf16 pairs (key k in column k/2) over the first 64 columns of this
+      // tile's S region; the first half is stored while the second is computed
 #pragma unroll
-      for (int c = 0; c < 128; c += 2) {
-        float x0, x1;
-        f2_unpack(f2_fma(f2_pack(sc[c], sc[c + 1]), sc2, ng2), x0, x1);
-        x0 = ex2(x0);
-        x1 = ex2(x1);
-        acc2[(c >> 1) & 3] = f2_add(acc2[(c >> 1) & 3], f2_pack(x0, x1));
-        pk[c >> 1] = pack_bf16(x0, x1);
+      for (int h = 0; h < 2; ++h) {
+        uint32_t pk[32];
+#pragma unroll
+        for (int c = 64 * h; c < 64 * h + 64; c += 2) {
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(sc[c], sc[c + 1]), sc2, ng2), x0, x1);
+          x0 = ex2(x0);
+          x1 = ex2(x1);
+          acc2[(c >> 1) & 3] = f2_add(acc2[(c >> 1) & 3], f2_pack(x0, x1));
+          pk[(c >> 1) & 31] = pack_bf16(x0, x1);
+        }
+        tmem_st32(s_col + 32 * h, reinterpret_cast<const float*>(pk));
       }
       {
         float a0, a1;
         f2_unpack(f2_add(f2_add(acc2[0], acc2[1]), f2_add(acc2[2], acc2[3])), a0, a1);
         l_run = l_run * alpha + (a0 + a1);
       }
-      // P as bf16 pairs (key k in column k/2) over the first 64 columns of this tile's S region
-      tmem_st32(s_col, reinterpret_cast<const float*>(pk));
-      tmem_st32(s_col + 32, reinterpret_cast<const float*>(pk + 32));
       // O is current here (the commit that signalled S also covers the previous PV)
       if (j >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll
@@ -375,49 +422,233 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
       if (lane == 0) mbar_arrive(bar(B_PF + qt));
     }
 
-    // ---- epilogue
-    const bool split_out = nsplit > 1;
+    // ---- epilogue (indices recomputed from the CTA and thread ids, so that
+    // nothing the main loop does not need stays live across it)
+    const TcCta ce = tc_cta(p, cta_index_fresh());
+    const int split = ce.split, nsplit = ce.nsplit;
+    const int erow = threadIdx.x;                               // CTA row = thread (warps 0..7)
+    const int epr = ce.rt * kTcRows + erow;                     // packed row
+    const bool row_ok = epr / G < p.S;
     if (ok && ntile > 0) ok = warp_wait(bar(B_O), 0, abort_flag, p.wait_limit, p.status);
-    if (ok) {
-      tc_fence_after();
-      const float inv_l = (l_run > 0.f) ? 1.f / l_run : 0.f;
-      const float lse = (l_run > 0.f) ? (m_run + log2f(l_run)) * 0.69314718055994531f : -INFINITY;
-      const bool row_ok = tok < p.S;
-      if (split_out) {
-        float* po = p.part_o + ((long long)cta * kTcRows + r) * D;
+    if (ok) tc_fence_after();
+    const float inv_l = (l_run > 0.f) ? 1.f / l_run : 0.f;
+    const float lse = (ok && l_run > 0.f) ? (m_run + log2f(l_run)) * 0.69314718055994531f : -INFINITY;
+    // output row of packed row `pr`: token pr / G, head kvh * G + pr % G
+    auto out_row = [&](int pr) {
+      return ((long long)ce.req * p.S + pr / G) * p.Hq + ce.kvh * G + pr % G;
+    };
+    // 32 columns of one output row, bf16
+    auto store_row32 = [&](long long orow, int c, const float* o, float scale) {
+      uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D) + c * 4;
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        dst[k] = make_uint4(pack_bf16(o[8 * k] * scale, o[8 * k + 1] * scale),
+                            pack_bf16(o[8 * k + 2] * scale, o[8 * k + 3] * scale),
+                            pack_bf16(o[8 * k + 4] * scale, o[8 * k + 5] * scale),
+                            pack_bf16(o[8 * k + 6] * scale, o[8 * k + 7] * scale));
+    };
+    // Split-KV partial results are staged column-major ([d][256 rows] fp32) in
+    // the Q/K/V area, free once the last MMA has completed: 32 columns are one
+    // contiguous 32 KiB piece, and a warp's accesses to one column are 128
+    // consecutive bytes.
+    constexpr int kPiece = 32 * kTcRows * 4;
+    float* stage = reinterpret_cast<float*>(smem);
+    auto stage_own = [&]() {
+      if (!ok) return;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        float* sb = stage + c * (kPiece / 4);
         if (ntile > 0) {
-#pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
-            float o[32];
-            tmem_ld32(o_col + c * 32, o);
-            tc_wait_ld();
-            if (row_ok) {
-#pragma unroll
-              for (int k = 0; k < 32; k += 4)
-                *reinterpret_cast<float4*>(po + c * 32 + k) =
-                    make_float4(o[k] * inv_l, o[k + 1] * inv_l, o[k + 2] * inv_l, o[k + 3] * inv_l);
-            }
-          }
-        }
-        if (row_ok) p.part_lse[(long long)cta * kTcRows + r] = lse;
-      } else if (ntile > 0) {
-        const long long orow = ((long long)req * p.S + tok) * p.Hq + kvh * G + jh;
-        uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D);
-#pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
           float o[32];
           tmem_ld32(o_col + c * 32, o);
           tc_wait_ld();
-          if (row_ok) {
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-              dst[c * 4 + k] = make_uint4(
-                  pack_bf16(o[8 * k] * inv_l, o[8 * k + 1] * inv_l), pack_bf16(o[8 * k + 2] * inv_l, o[8 * k + 3] * inv_l),
-                  pack_bf16(o[8 * k + 4] * inv_l, o[8 * k + 5] * inv_l), pack_bf16(o[8 * k + 6] * inv_l, o[8 * k + 7] * inv_l));
+          for (int k = 0; k < 32; ++k) sb[k * kTcRows + erow] = o[k] * inv_l;
+        } else {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) sb[k * kTcRows + erow] = 0.f;
+        }
+      }
+    };
+    if (p.work.cluster > 0) {
+      // Cluster mode: the nsplit CTAs of this row tile form one cluster.  Each
+      // stages its normalised O and LSE, then merges a slice of the 256 rows
+      // (whole 32-row groups) from all of them through distributed shared
+      // memory, in split order, so no partial result goes to global memory.
+      float* slse = stage + D * kTcRows;
+      stage_own();
+      slse[erow] = lse;
+      cluster_sync_all();   // 1: every CTA of the cluster has staged
+      const int g_lo = (split * 8) / nsplit, g_hi = ((split + 1) * 8) / nsplit;
+      const int nrows = (g_hi - g_lo) * 32;
+      const uint32_t own_base = smem_u32(stage);
+      if (!*abort_flag) {
+        for (int item = erow; item < nrows * (D / 32); item += 256) {
+          const int lr = g_lo * 32 + item % nrows, cb = item / nrows;
+          float w[8];
+          float mx = -INFINITY;
+#pragma unroll
+          for (int sp = 0; sp < 8; ++sp) {
+            w[sp] = sp < nsplit ? ld_dsmem(dsmem_addr(own_base + (D * kTcRows + lr) * 4, sp)) : -INFINITY;
+            mx = fmaxf(mx, w[sp]);
+          }
+          float wsum = 0.f;
+#pragma unroll
+          for (int sp = 0; sp < 8; ++sp) {
+            w[sp] = (w[sp] == -INFINITY) ? 0.f : __expf(w[sp] - mx);
+            wsum += w[sp];
+          }
+          float acc[32];
+#pragma unroll
+          for (int k = 0; k < 32; ++k) acc[k] = 0.f;
+#pragma unroll
+          for (int sp = 0; sp < 8; ++sp) {
+            if (sp < nsplit) {
+              const uint32_t src = dsmem_addr(own_base + ((cb * 32) * kTcRows + lr) * 4, sp);
+#pragma unroll
+              for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w[sp], ld_dsmem(src + k * kTcRows * 4), acc[k]);
+            }
+          }
+          const int pr = ce.rt * kTcRows + lr;
+          if (pr / G < p.S) {
+            const long long orow = out_row(pr);
+            store_row32(orow, cb, acc, wsum > 0.f ? 1.f / wsum : 0.f);
+            if (cb == 0 && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
           }
         }
-        if (row_ok && p.lse_out) p.lse_out[orow] = lse;
       }
+      cluster_sync_all();   // 2: no CTA leaves while a peer may still read its shared memory
+    } else if (nsplit > 1) {
+      // Independent splits: publish this chunk's normalised O and its
+      // log-sum-exp through global memory; the last CTA of the (request, KV
+      // head, row tile) to arrive merges all chunks.
+      const int cta = cta_index_fresh();
+      const int r = erow;
+      const long long orow = out_row(epr);
+      auto store_row32o = [&](int c, const float* o, float scale) { store_row32(orow, c, o, scale); };
+      const int req = ce.req, kvh = ce.kvh, rt = ce.rt;
+      constexpr int kBufs = L::BAR_OFF / kPiece;       // 6 (d = 128) or 3 (d = 64)
+      constexpr int kRing = kBufs - 1;                 // the last one holds the merge weights
+      static_assert(D / 32 <= kRing && kRing <= 8, "staging buffers");
+      static_assert(kMaxSplits * kTcRows * 4 <= kPiece, "merge weights buffer");
+      float* po = p.part_o + (long long)cta * kTcRows * D;
+      stage_own();
+      p.part_lse[(long long)cta * kTcRows + r] = lse;
+      fence_proxy_async_smem();
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      if (threadIdx.x == 0) {
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) bulk_store(po + c * 32 * kTcRows, sbase + c * kPiece, kPiece);
+        bulk_commit();
+        bulk_wait_all();
+        fence_proxy_async_all();
+      }
+      // every CTA arrives, also after a timeout, so the count always completes;
+      // the merge runs only without an abort (a warp whose wait failed raised
+      // the flag before the barrier above), decided once for all warps
+      __threadfence();
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      if (threadIdx.x == 0) {
+        const int unit = (req * p.Hkv + kvh) * p.work.row_tiles + rt;
+        const bool last = atomicAdd(&p.unit_cnt[unit], 1) == nsplit - 1;
+        bool fits = nsplit <= kMaxSplits;   // merge weights: one buffer of kMaxSplits x 256
+        if (last && !fits) set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
+        *last_flag = (last && fits && !*abort_flag) ? 1 : 0;
+      }
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      if (*last_flag) {
+        __threadfence();
+        fence_proxy_async_all();
+        const int c0 = p.work.base[req] + kvh * p.work.row_tiles + rt;   // CTA of split 0
+        const int cstride = p.Hkv * p.work.row_tiles;
+        // merge weights exp(lse_s - max) of this row, one per split, in the last buffer
+        float* wt = stage + kRing * (kPiece / 4);
+        float mx = -INFINITY;
+        for (int sp = 0; sp < nsplit; ++sp)
+          mx = fmaxf(mx, __ldcg(p.part_lse + (long long)(c0 + sp * cstride) * kTcRows + r));
+        float wsum = 0.f;
+        for (int sp = 0; sp < nsplit; ++sp) {
+          const float ls = __ldcg(p.part_lse + (long long)(c0 + sp * cstride) * kTcRows + r);
+          const float w = (ls == -INFINITY) ? 0.f : __expf(ls - mx);
+          wsum += w;
+          wt[sp * kTcRows + r] = w;
+        }
+        const float inv_w = wsum > 0.f ? 1.f / wsum : 0.f;
+        // the other splits' pieces stream through the ring: piece i = (column
+        // block i / (nsplit-1), i-th other split); warp 0 issues the copies.
+        // Splits are summed in split order with the same arithmetic for the
+        // own chunk (tensor memory) as for the others, so the result does not
+        // depend on which CTA arrived last.
+        const int others = nsplit - 1, n_pieces = (D / 32) * others;
+        auto issue = [&](int i) {
+          const int t = i % others, sp = t < split ? t : t + 1;
+          const int b = i % kRing;
+          mbar_expect_tx(bar(B_MF + b), kPiece);
+          bulk_load(sbase + b * kPiece,
+                    p.part_o + (long long)(c0 + sp * cstride) * kTcRows * D + (long long)(i / others) * 32 * kTcRows,
+                    kPiece, bar(B_MF + b));
+        };
+        int issued = 0;
+        if (warp == 0) {
+          if (lane == 0)
+            for (int i = 0; i < min(kRing, n_pieces); ++i) issue(i);
+          issued = min(kRing, n_pieces);
+        }
+        asm volatile("bar.sync 1, 256;" ::: "memory");   // weights visible to all rows' threads
+        bool mok = true;
+#pragma unroll 1
+        for (int c = 0; mok && c < D / 32; ++c) {
+          float own[32], acc[32];
+          if (ntile > 0) {
+            tmem_ld32(o_col + c * 32, own);
+            tc_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 32; ++k) own[k] = own[k] * inv_l;   // the value the other CTAs would read
+          } else {
+#pragma unroll
+            for (int k = 0; k < 32; ++k) own[k] = 0.f;
+          }
+#pragma unroll
+          for (int k = 0; k < 32; ++k) acc[k] = 0.f;
+#pragma unroll 1
+          for (int sp = 0; sp < nsplit; ++sp) {
+            const float w = wt[sp * kTcRows + r];
+            if (sp == split) {
+#pragma unroll
+              for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w, own[k], acc[k]);
+              continue;
+            }
+            const int i = c * others + (sp < split ? sp : sp - 1), b = i % kRing;
+            if (!(mok = warp_wait(bar(B_MF + b), (i / kRing) & 1, abort_flag, p.wait_limit, p.status))) break;
+            const float* src = stage + b * (kPiece / 4) + r;
+#pragma unroll
+            for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w, src[k * kTcRows], acc[k]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(B_ME + b));
+            if (warp == 0 && i + kRing < n_pieces) {
+              if (!(mok = warp_wait(bar(B_ME + b), (i / kRing) & 1, abort_flag, p.wait_limit, p.status))) break;
+              if (lane == 0) issue(i + kRing);
+              ++issued;
+            }
+          }
+          if (mok && row_ok) store_row32o(c, acc, inv_w);
+        }
+        if (warp == 0 && !mok && lane == 0) {   // let the copies this CTA issued land
+          for (int i = max(0, issued - kRing); i < issued; ++i)
+            mbar_drain(bar(B_MF + i % kRing), (i / kRing) & 1, p.status);
+        }
+        if (mok && row_ok && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
+      }
+    } else if (ok && ntile > 0) {
+      const long long orow = out_row(epr);
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        float o[32];
+        tmem_ld32(o_col + c * 32, o);
+        tc_wait_ld();
+        if (row_ok) store_row32(orow, c, o, inv_l);
+      }
+      if (row_ok && p.lse_out) p.lse_out[orow] = lse;
     }
   }
   tc_fence_before();
@@ -439,8 +670,54 @@ static cudaError_t launch_attn_tc_t(const AttnParams& p, cudaStream_t st) {
   if (fa.numRegs * 384 < 128 * kCtrlRegs + 256 * kSoftRegs) return cudaErrorLaunchOutOfResources;
   e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
+  if (p.work.cluster > 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.work.n_cta);
+    cfg.blockDim = dim3(384);
+    cfg.dynamicSmemBytes = L::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = p.work.cluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, attn_tc_kernel<D>, p);
+  }
   attn_tc_kernel<D><<<p.work.n_cta, 384, L::SMEM, st>>>(p);
   return cudaGetLastError();
+}
+
+// clusters of `ns` CTAs of this kernel that fit on the device at once (0: none)
+template <int D>
+static int attn_tc_max_clusters_t(int ns) {
+  using L = TcLayout<D>;
+  if (cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM) != cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(ns);
+  cfg.blockDim = dim3(384);
+  cfg.dynamicSmemBytes = L::SMEM;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = ns;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<D>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+int attn_tc_max_clusters(int D, int ns) {
+  if (D == 128) return attn_tc_max_clusters_t<128>(ns);
+  if (D == 64) return attn_tc_max_clusters_t<64>(ns);
+  return 0;
 }
 
 cudaError_t launch_attn_tc(const AttnParams& p, int D, cudaStream_t st) {

@@ -444,6 +444,11 @@ static size_t q_project_scratch(const attuner_ctx* ctx, int M) {
 // ---------------------------------------------------------------------------
 // attention
 // ---------------------------------------------------------------------------
+void att::query_cluster_occupancy(attuner_ctx* ctx) {
+  if (ctx->tc_clusters[2] >= 0) return;
+  for (int ns = 0; ns <= 8; ++ns) ctx->tc_clusters[ns] = ns >= 2 ? attn_tc_max_clusters(ctx->cfg.head_dim, ns) : 0;
+}
+
 void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc,
                       WorkTable& w) {
   const int G = ctx->cfg.n_q_heads / ctx->cfg.n_kv_heads, Hkv = ctx->cfg.n_kv_heads;
@@ -458,28 +463,55 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
     maxv = std::max(maxv, nv);
   }
   const long long units = (long long)plan->n_req * Hkv * row_tiles;
+  // Cluster mode (tcgen05 kernel): every row tile cut into ns chunks, one
+  // cluster of ns CTAs per row tile.  Cost in 128-key tile times: waves of
+  // co-resident clusters x (largest chunk + ~4 tiles of prologue and epilogue
+  // + ~1 for the merge).
+  auto cluster_cost = [&](int ns) -> double {
+    const int maxc = ctx->tc_clusters[ns];
+    if (maxc <= 0) return 1e30;
+    const int chunk = (((maxv + ns - 1) / ns) + 1) & ~1;
+    if (chunk > kMaxChunkBlocks) return 1e30;
+    const long long waves = (units + maxc - 1) / maxc;
+    return (double)waves * (chunk / 2 + 5.0);
+  };
+  int cluster_ns = 0;
   int chunk;
   if (ctx->opt_split > 0) {
     chunk = ctx->opt_split;
+    if (tc && ctx->opt_merge == 2 && maxv > chunk)
+      cluster_ns = std::min(8, std::max(2, (maxv + chunk - 1) / chunk));
   } else if (tc) {
-    // One CTA per SM.  Cost of a chunk size = waves x (tiles per CTA + a fixed
-    // per-CTA overhead of ~4 tiles for the prologue, epilogue and combine);
-    // pick the number of splits of the longest request that minimises it.
+    // Independent splits, one CTA per SM.  Cost of a chunk size = waves x
+    // (tiles per CTA + ~4 tiles for the prologue and epilogue + ~2 for the
+    // merge through global memory); pick the number of splits of the
+    // longest request that minimises it.
     const int maxt = (maxv + 1) / 2;
     double best = 1e30;
     chunk = maxv;
-    for (int sp = 1; sp <= 32; ++sp) {
-      const int ct = (maxt + sp - 1) / sp;
-      long long ncta = 0;
-      for (int r = 0; r < plan->n_req; ++r) {
-        const int nv = plan->blk_off[r + 1] - plan->blk_off[r] + nsuf;
-        ncta += (long long)((nv + 2 * ct - 1) / (2 * ct)) * Hkv * row_tiles;
+    if (ctx->opt_merge != 2) {
+      for (int sp = 1; sp <= kMaxSplits; ++sp) {
+        const int ct = (maxt + sp - 1) / sp;
+        long long ncta = 0;
+        for (int r = 0; r < plan->n_req; ++r) {
+          const int nv = plan->blk_off[r + 1] - plan->blk_off[r] + nsuf;
+          ncta += (long long)((nv + 2 * ct - 1) / (2 * ct)) * Hkv * row_tiles;
+        }
+        const long long waves = (ncta + ctx->num_sms - 1) / ctx->num_sms;
+        const double cost = (double)waves * (ct + 4.0 + (sp > 1 ? 2.0 : 0.0));
+        if (cost < best - 1e-9) {
+          best = cost;
+          chunk = 2 * ct;
+        }
       }
-      const long long waves = (ncta + ctx->num_sms - 1) / ctx->num_sms;
-      const double cost = (double)waves * (ct + 4.0 + (sp > 1 ? 2.0 : 0.0));
-      if (cost < best - 1e-9) {
-        best = cost;
-        chunk = 2 * ct;
+    }
+    if (ctx->opt_merge != 1) {
+      for (int ns = 2; ns <= 8; ++ns) {
+        const double cost = cluster_cost(ns);
+        if (cost < best - 1e-9) {
+          best = cost;
+          cluster_ns = ns;
+        }
       }
     }
   } else {
@@ -488,11 +520,25 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
     const long long target = 8ll * ctx->num_sms;
     chunk = (int)std::max<long long>(16, (total + target - 1) / target);
   }
-  (void)units;
-  chunk = std::min(chunk, kMaxChunkBlocks);
-  if (tc) chunk = (chunk + 1) & ~1;   // whole 128-key tiles per split
   w.n_req = plan->n_req;
   w.row_tiles = row_tiles;
+  if (cluster_ns > 0) {
+    w.cluster = cluster_ns;
+    w.chunk_blocks = 0;   // per request, ceil(blocks / cluster) rounded up to whole tiles
+    for (int r = 0; r < plan->n_req; ++r) {
+      w.base[r] = (int)(r * (long long)Hkv * row_tiles * cluster_ns);
+      w.nsplit[r] = cluster_ns;
+    }
+    w.n_cta = (int)(units * cluster_ns);
+    return;
+  }
+  w.cluster = 0;
+  chunk = std::min(chunk, kMaxChunkBlocks);
+  if (tc) {
+    // the kernel merges at most kMaxSplits chunks of one row tile
+    chunk = std::max(chunk, (maxv + kMaxSplits - 1) / kMaxSplits);
+    chunk = (chunk + 1) & ~1;   // whole 128-key tiles per split
+  }
   w.chunk_blocks = chunk;
   int base = 0;
   for (int r = 0; r < plan->n_req; ++r) {
@@ -519,9 +565,11 @@ static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, co
   else if (ctx->opt_prefill == 2) tc = false;
   else tc = (S * G > kMmaRows);
   WorkTable* w = new WorkTable();
+  if (tc) query_cluster_occupancy(ctx);
   make_work(ctx, plan, S, S_kv, tc, *w);
-  bool need_combine = false;
+  bool need_combine = false;   // split partial results in global memory
   for (int r = 0; r < plan->n_req; ++r) need_combine |= (w->nsplit[r] > 1);
+  if (w->cluster > 0) need_combine = false;
   const int rows = tc ? kTcRows : kMmaRows;
 
   AttnParams* ap = new AttnParams();
@@ -561,18 +609,27 @@ static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, co
   (void)sc_outer;
   void* part = nullptr;
   size_t part_bytes = 0;
+  cudaError_t ce = cudaSuccess;
   if (need_combine) {
-    part_bytes = (size_t)w->n_cta * rows * (D + 1) * 4;
+    // partial O and LSE of every split CTA; for the tcgen05 kernel also one
+    // arrival counter per (request, KV head, row tile), zeroed here
+    const size_t pb = (size_t)w->n_cta * rows * (D + 1) * 4;
+    const size_t units = (size_t)plan->n_req * Hkv * w->row_tiles;
+    part_bytes = pb + (tc ? units * 4 : 0);
     if (cudaMallocFromPoolAsync(&part, part_bytes, ctx->mempool, st) != cudaSuccess) {
       cudaGetLastError();
       return done(fail(ATTUNER_ERR_OOM, "split-KV scratch allocation failed"));
     }
     ap->part_o = static_cast<float*>(part);
     ap->part_lse = static_cast<float*>(part) + (size_t)w->n_cta * rows * D;
+    if (tc) {
+      ap->unit_cnt = reinterpret_cast<int*>(static_cast<char*>(part) + pb);
+      ce = cudaMemsetAsync(ap->unit_cnt, 0, units * 4, st);
+    }
   }
-  cudaError_t ce = tc ? launch_attn_tc(*ap, D, st) : launch_attn_mma(*ap, D, st);
+  if (ce == cudaSuccess) ce = tc ? launch_attn_tc(*ap, D, st) : launch_attn_mma(*ap, D, st);
   if (ce == cudaSuccess) ++launches;
-  if (ce == cudaSuccess && need_combine) {
+  if (ce == cudaSuccess && need_combine && !tc) {   // the tcgen05 kernel merges its splits itself
     CombineParams cp{};
     cp.work = *w;
     cp.part_o = ap->part_o;
@@ -694,6 +751,10 @@ extern "C" attuner_status attuner_set_option(attuner_ctx* ctx, int32_t option, i
     case ATTUNER_OPT_QPROJ_SPLIT_K:
       CHECK_ARG(value >= 0 && value <= 4, "Q-projection split-K must be in [0, 4]");
       ctx->opt_qproj_split = value ? (int)value : 1;
+      return ATTUNER_OK;
+    case ATTUNER_OPT_SPLIT_MERGE:
+      CHECK_ARG(value >= 0 && value <= 2, "split merge must be 0, 1 or 2");
+      ctx->opt_merge = (int)value;
       return ATTUNER_OK;
     case ATTUNER_OPT_TEST_STUCK_WAIT:
       ctx->inject_stuck = value ? 1 : 0;

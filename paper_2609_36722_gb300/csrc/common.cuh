@@ -32,6 +32,11 @@ struct WorkTable {
   int32_t row_tiles;      // row tiles per (request, kv head)
   int32_t chunk_blocks;   // virtual blocks per split
   int32_t n_cta;
+  // tcgen05 kernel only: 0 = splits of a row tile are independent CTAs merged
+  // through global memory; > 0 = every row tile has exactly this many splits,
+  // launched as one thread-block cluster (split = rank in the cluster) and
+  // merged through distributed shared memory.
+  int32_t cluster;
   int32_t base[kMaxReq];
   int32_t nsplit[kMaxReq];
 };
@@ -164,6 +169,52 @@ ATT_DEV void tma_load_5d(uint32_t dst, const CUtensorMap* m, uint32_t bar, int c
 // generic-proxy shared-memory writes -> visible to the async proxy (UMMA, TMA)
 ATT_DEV void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// the same, both directions, for every state space (global included)
+ATT_DEV void fence_proxy_async_all() {
+  asm volatile("fence.proxy.async;" ::: "memory");
+}
+
+// Untiled bulk copies (cp.async.bulk): both addresses 16-byte aligned and the
+// size a multiple of 16.  A load completes on an mbarrier (complete_tx); stores
+// are tracked per thread in bulk groups.
+ATT_DEV void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(dst), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+               : "memory");
+}
+ATT_DEV void bulk_store(void* dst, uint32_t src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
+               ::"l"(reinterpret_cast<uint64_t>(dst)), "r"(src), "r"(bytes)
+               : "memory");
+}
+ATT_DEV void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// waits until every committed bulk store of this thread has been performed
+ATT_DEV void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// ---------------------------------------------------------------------------
+// Thread-block clusters: barrier and distributed shared memory
+// ---------------------------------------------------------------------------
+// every thread of every CTA in the cluster; release/acquire orders the shared
+// memory writes before it with the peers' reads after it
+ATT_DEV void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// shared::cluster address of the same offset in the shared memory of CTA `rank`
+ATT_DEV uint32_t dsmem_addr(uint32_t saddr, uint32_t rank) {
+  uint32_t d;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(saddr), "r"(rank));
+  return d;
+}
+ATT_DEV float ld_dsmem(uint32_t caddr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
+  return v;
+}
+ATT_DEV uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
 }
 
 // ---------------------------------------------------------------------------

@@ -39,6 +39,8 @@ struct attuner_ctx {
   int opt_prefill = 0;
   int opt_split = 0;
   int opt_qproj_split = 1;
+  int opt_merge = 0;
+  int tc_clusters[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};   // co-resident clusters of n tcgen05 CTAs
   long long wait_limit = 1ll << 32;
   int inject_stuck = 0;
   int last_launches = 0;
@@ -71,5 +73,7 @@ PlanDev plan_dev(const attuner_plan* p);
 attuner_status check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv);
 // split-KV decomposition of one attention launch (tc: tcgen05 kernel, else warp-MMA kernel)
 void make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc, WorkTable& w);
+// fills ctx->tc_clusters on first use (queries the device)
+void query_cluster_occupancy(attuner_ctx* ctx);
 
 }  // namespace att

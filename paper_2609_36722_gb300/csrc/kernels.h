@@ -52,8 +52,9 @@ struct AttnParams {
   const __nv_bfloat16* q;        // (K3 reads Q directly)
   __nv_bfloat16* out;            // [n_req, S, Hq, D]
   float* lse_out;                // [n_req, S, Hq] or nullptr
-  float* part_o;                 // [n_cta, rows_per_tile, D] (split chunks only)
+  float* part_o;                 // split chunks only: K3 [n_cta, 16, D]; K2 [n_cta, D, 256] (column-major)
   float* part_lse;               // [n_cta, rows_per_tile]
+  int* unit_cnt;                 // K2: arrivals per (request, KV head, row tile); zero on entry, left zero
   int32_t S, S_kv, Hq, Hkv, G;
   float scale_log2;              // log2(e) / sqrt(D)
   int* status;
@@ -76,6 +77,8 @@ cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __
                               cudaStream_t st);
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st);
 cudaError_t launch_qproj(const QprojParams& p, int D, cudaStream_t st);
+// how many clusters of `ns` tcgen05 attention CTAs fit on the current device at once
+int attn_tc_max_clusters(int D, int ns);
 cudaError_t launch_attn_tc(const AttnParams& p, int D, cudaStream_t st);
 cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st);
 cudaError_t launch_combine(const CombineParams& p, cudaStream_t st);
@@ -86,5 +89,7 @@ constexpr int kTcTileRows = 128;  // rows per query tile (one MMA M)
 constexpr int kMmaRows = 16;
 // largest split chunk (virtual blocks) the kernels' shared-memory block list holds
 constexpr int kMaxChunkBlocks = 4096;
+// most split-KV chunks of one (request, KV head, row tile) in the tcgen05 kernel
+constexpr int kMaxSplits = 32;
 
 }  // namespace att

@@ -108,11 +108,16 @@ def test_error_paths_leave_context_usable():
     assert torch.isfinite(out.float()).all()
 
 
+@pytest.mark.parametrize("merge", [1, 2])
 @pytest.mark.parametrize("S,S_kv", [(1, 129), (40, 48), (300, 300)])
-def test_repeated_calls_are_bit_identical(S, S_kv):
-    # split-K partial sums and split-KV partials are combined in a fixed order
+def test_repeated_calls_are_bit_identical(S, S_kv, merge):
+    # split-K partial sums and split-KV partials are combined in a fixed order,
+    # whichever CTA finishes last and whichever merge path runs
+    import paper_2609_36722_gb300 as pkg
     wl = make_custom("det", GEOM, 27, [150, 64, 333, 20], [[3, 0, 2, 1], [1, 2]], S, S_kv, device=DEV)
     ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, 4)
+    ctx.set_option(pkg.OPT_SPLIT_MERGE, merge)
     o1, l1 = run_path(ctx, plan, wl)
     o2, l2 = run_path(ctx, plan, wl)
     assert torch.equal(o1, o2) and torch.equal(l1, l2)

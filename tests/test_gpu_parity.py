@@ -102,6 +102,23 @@ def test_ragged_multi_request(kernel, split):
     compare(_np(out), o_ref, _np(lse), lse_ref, label=f"ragged kernel={kernel} split={split}")
 
 
+@pytest.mark.parametrize("merge", [1, 2])
+@pytest.mark.parametrize("split,S,S_kv", [(2, 50, 70), (4, 300, 300), (6, 130, 200), (0, 300, 300)])
+def test_split_merge_modes(merge, split, S, S_kv):
+    # tcgen05 kernel, split-KV chunks merged through global memory (1) or inside
+    # one thread-block cluster per row tile (2); 300 suffix tokens x G = 4 give
+    # ragged 256-row tiles, and 2..8 chunks per row tile with uneven row slices
+    import paper_2609_36722_gb300 as pkg
+    wl = _ragged(seed=17, S=S, S_kv=S_kv, lengths=(37, 700, 64, 1, 1290))
+    o_ref, lse_ref = _full_reference(wl)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, 1)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, split)
+    ctx.set_option(pkg.OPT_SPLIT_MERGE, merge)
+    out, lse = run_path(ctx, plan, wl)
+    compare(_np(out), o_ref, _np(lse), lse_ref, label=f"merge={merge} split={split} S={S}")
+
+
 @pytest.mark.parametrize("G", [1, 2, 8])
 def test_group_sizes(G):
     geom = Geometry(hidden=256, n_q_heads=4 * G, n_kv_heads=4, head_dim=128, rank=8)
