@@ -154,6 +154,249 @@ __device__ __forceinline__ int cta_index_fresh() {
   return v;
 }
 
+// Epilogue of the softmax warps (warps 0..7, one CTA row per thread): O from
+// tensor memory, normalised, written as bf16 -- directly, or after merging the
+// split-KV chunks of the row tile.  A separate (not inlined) function, so that
+// its registers do not press on the main loop's.
+template <int D>
+__device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uint32_t o_col, bool ok,
+                                         float m_run, float l_run, int ntile) {
+  using L = TcLayout<D>;
+  const uint32_t sbase = smem_u32(smem);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 520);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 524);
+  auto bar = [&](int i) { return smem_u32(&bars[i]); };
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int G = p.G;
+  const TcCta ce = tc_cta(p, blockIdx.x);
+  const int split = ce.split, nsplit = ce.nsplit;
+  const int erow = threadIdx.x;                               // CTA row = thread (warps 0..7)
+  const int epr = ce.rt * kTcRows + erow;                     // packed row
+  const bool row_ok = epr / G < p.S;
+  if (ok && ntile > 0) ok = warp_wait(bar(B_O), 0, abort_flag, p.wait_limit, p.status);
+  if (ok) tc_fence_after();
+  const float inv_l = (l_run > 0.f) ? 1.f / l_run : 0.f;
+  const float lse = (ok && l_run > 0.f) ? (m_run + log2f(l_run)) * 0.69314718055994531f : -INFINITY;
+  // output row of packed row `pr`: token pr / G, head kvh * G + pr % G
+  auto out_row = [&](int pr) {
+    return ((long long)ce.req * p.S + pr / G) * p.Hq + ce.kvh * G + pr % G;
+  };
+  // 32 columns of one output row, bf16
+  auto store_row32 = [&](long long orow, int c, const float* o, float scale) {
+    uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D) + c * 4;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      dst[k] = make_uint4(pack_bf16(o[8 * k] * scale, o[8 * k + 1] * scale),
+                          pack_bf16(o[8 * k + 2] * scale, o[8 * k + 3] * scale),
+                          pack_bf16(o[8 * k + 4] * scale, o[8 * k + 5] * scale),
+                          pack_bf16(o[8 * k + 6] * scale, o[8 * k + 7] * scale));
+  };
+  // Split-KV partial results are staged in the Q/K/V area, free once the last
+  // MMA has completed.  Global mode stages them column-major ([d][256 rows]
+  // fp32): 32 columns are one contiguous 32 KiB piece for one bulk copy, and a
+  // warp's accesses to one column are 128 consecutive bytes.
+  constexpr int kPiece = 32 * kTcRows * 4;
+  float* stage = reinterpret_cast<float*>(smem);
+  auto stage_own = [&]() {
+    if (!ok) return;
+#pragma unroll
+    for (int c = 0; c < D / 32; ++c) {
+      float* sb = stage + c * (kPiece / 4);
+      if (ntile > 0) {
+        float o[32];
+        tmem_ld32(o_col + c * 32, o);
+        tc_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) sb[k * kTcRows + erow] = o[k] * inv_l;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 32; ++k) sb[k * kTcRows + erow] = 0.f;
+      }
+    }
+  };
+  if (p.work.cluster > 0) {
+    // Cluster mode: the nsplit CTAs of this row tile form one cluster.  Each
+    // stages its normalised O and LSE, then merges a slice of the 256 rows
+    // (whole 32-row groups) from all of them through distributed shared
+    // memory, in split order, so no partial result goes to global memory.
+    float* slse = stage + D * kTcRows;
+    stage_own();
+    slse[erow] = lse;
+    cluster_sync_all();   // 1: every CTA of the cluster has staged
+    const int g_lo = (split * 8) / nsplit, g_hi = ((split + 1) * 8) / nsplit;
+    const int nrows = (g_hi - g_lo) * 32;
+    const uint32_t own_base = smem_u32(stage);
+    if (!*abort_flag) {
+      for (int item = erow; item < nrows * (D / 32); item += 256) {
+        const int lr = g_lo * 32 + item % nrows, cb = item / nrows;
+        float w[8];
+        float mx = -INFINITY;
+#pragma unroll
+        for (int sp = 0; sp < 8; ++sp) {
+          w[sp] = sp < nsplit ? ld_dsmem(dsmem_addr(own_base + (D * kTcRows + lr) * 4, sp)) : -INFINITY;
+          mx = fmaxf(mx, w[sp]);
+        }
+        float wsum = 0.f;
+#pragma unroll
+        for (int sp = 0; sp < 8; ++sp) {
+          w[sp] = (w[sp] == -INFINITY) ? 0.f : __expf(w[sp] - mx);
+          wsum += w[sp];
+        }
+        float acc[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) acc[k] = 0.f;
+#pragma unroll
+        for (int sp = 0; sp < 8; ++sp) {
+          if (sp < nsplit) {
+            const uint32_t src = dsmem_addr(own_base + ((cb * 32) * kTcRows + lr) * 4, sp);
+#pragma unroll
+            for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w[sp], ld_dsmem(src + k * kTcRows * 4), acc[k]);
+          }
+        }
+        const int pr = ce.rt * kTcRows + lr;
+        if (pr / G < p.S) {
+          const long long orow = out_row(pr);
+          store_row32(orow, cb, acc, wsum > 0.f ? 1.f / wsum : 0.f);
+          if (cb == 0 && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
+        }
+      }
+    }
+    cluster_sync_all();   // 2: no CTA leaves while a peer may still read its shared memory
+  } else if (nsplit > 1) {
+    // Independent splits: publish this chunk's normalised O and its
+    // log-sum-exp through global memory; the last CTA of the (request, KV
+    // head, row tile) to arrive merges all chunks.
+    const int cta = cta_index_fresh();
+    const int r = erow;
+    const long long orow = out_row(epr);
+    auto store_row32o = [&](int c, const float* o, float scale) { store_row32(orow, c, o, scale); };
+    const int req = ce.req, kvh = ce.kvh, rt = ce.rt;
+    constexpr int kBufs = L::BAR_OFF / kPiece;       // 6 (d = 128) or 3 (d = 64)
+    constexpr int kRing = kBufs - 1;                 // the last one holds the merge weights
+    static_assert(D / 32 <= kRing && kRing <= 8, "staging buffers");
+    static_assert(kMaxSplits * kTcRows * 4 <= kPiece, "merge weights buffer");
+    float* po = p.part_o + (long long)cta * kTcRows * D;
+    stage_own();
+    p.part_lse[(long long)cta * kTcRows + r] = lse;
+    fence_proxy_async_smem();
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+    if (threadIdx.x == 0) {
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) bulk_store(po + c * 32 * kTcRows, sbase + c * kPiece, kPiece);
+      bulk_commit();
+      bulk_wait_all();
+      fence_proxy_async_all();
+    }
+    // every CTA arrives, also after a timeout, so the count always completes;
+    // the merge runs only without an abort (a warp whose wait failed raised
+    // the flag before the barrier above), decided once for all warps
+    __threadfence();
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+    if (threadIdx.x == 0) {
+      const int unit = (req * p.Hkv + kvh) * p.work.row_tiles + rt;
+      const bool last = atomicAdd(&p.unit_cnt[unit], 1) == nsplit - 1;
+      bool fits = nsplit <= kMaxSplits;   // merge weights: one buffer of kMaxSplits x 256
+      if (last && !fits) set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
+      *last_flag = (last && fits && !*abort_flag) ? 1 : 0;
+    }
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+    if (*last_flag) {
+      __threadfence();
+      fence_proxy_async_all();
+      const int c0 = p.work.base[req] + kvh * p.work.row_tiles + rt;   // CTA of split 0
+      const int cstride = p.Hkv * p.work.row_tiles;
+      // merge weights exp(lse_s - max) of this row, one per split, in the last buffer
+      float* wt = stage + kRing * (kPiece / 4);
+      float mx = -INFINITY;
+      for (int sp = 0; sp < nsplit; ++sp)
+        mx = fmaxf(mx, __ldcg(p.part_lse + (long long)(c0 + sp * cstride) * kTcRows + r));
+      float wsum = 0.f;
+      for (int sp = 0; sp < nsplit; ++sp) {
+        const float ls = __ldcg(p.part_lse + (long long)(c0 + sp * cstride) * kTcRows + r);
+        const float w = (ls == -INFINITY) ? 0.f : __expf(ls - mx);
+        wsum += w;
+        wt[sp * kTcRows + r] = w;
+      }
+      const float inv_w = wsum > 0.f ? 1.f / wsum : 0.f;
+      // the other splits' pieces stream through the ring: piece i = (column
+      // block i / (nsplit-1), i-th other split); warp 0 issues the copies.
+      // Splits are summed in split order with the same arithmetic for the
+      // own chunk (tensor memory) as for the others, so the result does not
+      // depend on which CTA arrived last.
+      const int others = nsplit - 1, n_pieces = (D / 32) * others;
+      auto issue = [&](int i) {
+        const int t = i % others, sp = t < split ? t : t + 1;
+        const int b = i % kRing;
+        mbar_expect_tx(bar(B_MF + b), kPiece);
+        bulk_load(sbase + b * kPiece,
+                  p.part_o + (long long)(c0 + sp * cstride) * kTcRows * D + (long long)(i / others) * 32 * kTcRows,
+                  kPiece, bar(B_MF + b));
+      };
+      int issued = 0;
+      if (warp == 0) {
+        if (lane == 0)
+          for (int i = 0; i < min(kRing, n_pieces); ++i) issue(i);
+        issued = min(kRing, n_pieces);
+      }
+      asm volatile("bar.sync 1, 256;" ::: "memory");   // weights visible to all rows' threads
+      bool mok = true;
+#pragma unroll 1
+      for (int c = 0; mok && c < D / 32; ++c) {
+        float own[32], acc[32];
+        if (ntile > 0) {
+          tmem_ld32(o_col + c * 32, own);
+          tc_wait_ld();
+#pragma unroll
+          for (int k = 0; k < 32; ++k) own[k] = own[k] * inv_l;   // the value the other CTAs would read
+        } else {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) own[k] = 0.f;
+        }
+#pragma unroll
+        for (int k = 0; k < 32; ++k) acc[k] = 0.f;
+#pragma unroll 1
+        for (int sp = 0; sp < nsplit; ++sp) {
+          const float w = wt[sp * kTcRows + r];
+          if (sp == split) {
+#pragma unroll
+            for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w, own[k], acc[k]);
+            continue;
+          }
+          const int i = c * others + (sp < split ? sp : sp - 1), b = i % kRing;
+          if (!(mok = warp_wait(bar(B_MF + b), (i / kRing) & 1, abort_flag, p.wait_limit, p.status))) break;
+          const float* src = stage + b * (kPiece / 4) + r;
+#pragma unroll
+          for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w, src[k * kTcRows], acc[k]);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar(B_ME + b));
+          if (warp == 0 && i + kRing < n_pieces) {
+            if (!(mok = warp_wait(bar(B_ME + b), (i / kRing) & 1, abort_flag, p.wait_limit, p.status))) break;
+            if (lane == 0) issue(i + kRing);
+            ++issued;
+          }
+        }
+        if (mok && row_ok) store_row32o(c, acc, inv_w);
+      }
+      if (warp == 0 && !mok && lane == 0) {   // let the copies this CTA issued land
+        for (int i = max(0, issued - kRing); i < issued; ++i)
+          mbar_drain(bar(B_MF + i % kRing), (i / kRing) & 1, p.status);
+      }
+      if (mok && row_ok && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
+    }
+  } else if (ok && ntile > 0) {
+    const long long orow = out_row(epr);
+#pragma unroll
+    for (int c = 0; c < D / 32; ++c) {
+      float o[32];
+      tmem_ld32(o_col + c * 32, o);
+      tc_wait_ld();
+      if (row_ok) store_row32(orow, c, o, inv_l);
+    }
+    if (row_ok && p.lse_out) p.lse_out[orow] = lse;
+  }
+}
+
 template <int D>
 __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__ AttnParams p) {
   using L = TcLayout<D>;
@@ -422,234 +665,7 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
       if (lane == 0) mbar_arrive(bar(B_PF + qt));
     }
 
-    // ---- epilogue (indices recomputed from the CTA and thread ids, so that
-    // nothing the main loop does not need stays live across it)
-    const TcCta ce = tc_cta(p, cta_index_fresh());
-    const int split = ce.split, nsplit = ce.nsplit;
-    const int erow = threadIdx.x;                               // CTA row = thread (warps 0..7)
-    const int epr = ce.rt * kTcRows + erow;                     // packed row
-    const bool row_ok = epr / G < p.S;
-    if (ok && ntile > 0) ok = warp_wait(bar(B_O), 0, abort_flag, p.wait_limit, p.status);
-    if (ok) tc_fence_after();
-    const float inv_l = (l_run > 0.f) ? 1.f / l_run : 0.f;
-    const float lse = (ok && l_run > 0.f) ? (m_run + log2f(l_run)) * 0.69314718055994531f : -INFINITY;
-    // output row of packed row `pr`: token pr / G, head kvh * G + pr % G
-    auto out_row = [&](int pr) {
-      return ((long long)ce.req * p.S + pr / G) * p.Hq + ce.kvh * G + pr % G;
-    };
-    // 32 columns of one output row, bf16
-    auto store_row32 = [&](long long orow, int c, const float* o, float scale) {
-      uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D) + c * 4;
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        dst[k] = make_uint4(pack_bf16(o[8 * k] * scale, o[8 * k + 1] * scale),
-                            pack_bf16(o[8 * k + 2] * scale, o[8 * k + 3] * scale),
-                            pack_bf16(o[8 * k + 4] * scale, o[8 * k + 5] * scale),
-                            pack_bf16(o[8 * k + 6] * scale, o[8 * k + 7] * scale));
-    };
-    // Split-KV partial results are staged column-major ([d][256 rows] fp32) in
-    // the Q/K/V area, free once the last MMA has completed: 32 columns are one
-    // contiguous 32 KiB piece, and a warp's accesses to one column are 128
-    // consecutive bytes.
-    constexpr int kPiece = 32 * kTcRows * 4;
-    float* stage = reinterpret_cast<float*>(smem);
-    auto stage_own = [&]() {
-      if (!ok) return;
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
-        float* sb = stage + c * (kPiece / 4);
-        if (ntile > 0) {
-          float o[32];
-          tmem_ld32(o_col + c * 32, o);
-          tc_wait_ld();
-#pragma unroll
-          for (int k = 0; k < 32; ++k) sb[k * kTcRows + erow] = o[k] * inv_l;
-        } else {
-#pragma unroll
-          for (int k = 0; k < 32; ++k) sb[k * kTcRows + erow] = 0.f;
-        }
-      }
-    };
-    if (p.work.cluster > 0) {
-      // Cluster mode: the nsplit CTAs of this row tile form one cluster.  Each
-      // stages its normalised O and LSE, then merges a slice of the 256 rows
-      // (whole 32-row groups) from all of them through distributed shared
-      // memory, in split order, so no partial result goes to global memory.
-      float* slse = stage + D * kTcRows;
-      stage_own();
-      slse[erow] = lse;
-      cluster_sync_all();   // 1: every CTA of the cluster has staged
-      const int g_lo = (split * 8) / nsplit, g_hi = ((split + 1) * 8) / nsplit;
-      const int nrows = (g_hi - g_lo) * 32;
-      const uint32_t own_base = smem_u32(stage);
-      if (!*abort_flag) {
-        for (int item = erow; item < nrows * (D / 32); item += 256) {
-          const int lr = g_lo * 32 + item % nrows, cb = item / nrows;
-          float w[8];
-          float mx = -INFINITY;
-#pragma unroll
-          for (int sp = 0; sp < 8; ++sp) {
-            w[sp] = sp < nsplit ? ld_dsmem(dsmem_addr(own_base + (D * kTcRows + lr) * 4, sp)) : -INFINITY;
-            mx = fmaxf(mx, w[sp]);
-          }
-          float wsum = 0.f;
-#pragma unroll
-          for (int sp = 0; sp < 8; ++sp) {
-            w[sp] = (w[sp] == -INFINITY) ? 0.f : __expf(w[sp] - mx);
-            wsum += w[sp];
-          }
-          float acc[32];
-#pragma unroll
-          for (int k = 0; k < 32; ++k) acc[k] = 0.f;
-#pragma unroll
-          for (int sp = 0; sp < 8; ++sp) {
-            if (sp < nsplit) {
-              const uint32_t src = dsmem_addr(own_base + ((cb * 32) * kTcRows + lr) * 4, sp);
-#pragma unroll
-              for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w[sp], ld_dsmem(src + k * kTcRows * 4), acc[k]);
-            }
-          }
-          const int pr = ce.rt * kTcRows + lr;
-          if (pr / G < p.S) {
-            const long long orow = out_row(pr);
-            store_row32(orow, cb, acc, wsum > 0.f ? 1.f / wsum : 0.f);
-            if (cb == 0 && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
-          }
-        }
-      }
-      cluster_sync_all();   // 2: no CTA leaves while a peer may still read its shared memory
-    } else if (nsplit > 1) {
-      // Independent splits: publish this chunk's normalised O and its
-      // log-sum-exp through global memory; the last CTA of the (request, KV
-      // head, row tile) to arrive merges all chunks.
-      const int cta = cta_index_fresh();
-      const int r = erow;
-      const long long orow = out_row(epr);
-      auto store_row32o = [&](int c, const float* o, float scale) { store_row32(orow, c, o, scale); };
-      const int req = ce.req, kvh = ce.kvh, rt = ce.rt;
-      constexpr int kBufs = L::BAR_OFF / kPiece;       // 6 (d = 128) or 3 (d = 64)
-      constexpr int kRing = kBufs - 1;                 // the last one holds the merge weights
-      static_assert(D / 32 <= kRing && kRing <= 8, "staging buffers");
-      static_assert(kMaxSplits * kTcRows * 4 <= kPiece, "merge weights buffer");
-      float* po = p.part_o + (long long)cta * kTcRows * D;
-      stage_own();
-      p.part_lse[(long long)cta * kTcRows + r] = lse;
-      fence_proxy_async_smem();
-      asm volatile("bar.sync 1, 256;" ::: "memory");
-      if (threadIdx.x == 0) {
-#pragma unroll
-        for (int c = 0; c < D / 32; ++c) bulk_store(po + c * 32 * kTcRows, sbase + c * kPiece, kPiece);
-        bulk_commit();
-        bulk_wait_all();
-        fence_proxy_async_all();
-      }
-      // every CTA arrives, also after a timeout, so the count always completes;
-      // the merge runs only without an abort (a warp whose wait failed raised
-      // the flag before the barrier above), decided once for all warps
-      __threadfence();
-      asm volatile("bar.sync 1, 256;" ::: "memory");
-      if (threadIdx.x == 0) {
-        const int unit = (req * p.Hkv + kvh) * p.work.row_tiles + rt;
-        const bool last = atomicAdd(&p.unit_cnt[unit], 1) == nsplit - 1;
-        bool fits = nsplit <= kMaxSplits;   // merge weights: one buffer of kMaxSplits x 256
-        if (last && !fits) set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
-        *last_flag = (last && fits && !*abort_flag) ? 1 : 0;
-      }
-      asm volatile("bar.sync 1, 256;" ::: "memory");
-      if (*last_flag) {
-        __threadfence();
-        fence_proxy_async_all();
-        const int c0 = p.work.base[req] + kvh * p.work.row_tiles + rt;   // CTA of split 0
-        const int cstride = p.Hkv * p.work.row_tiles;
-        // merge weights exp(lse_s - max) of this row, one per split, in the last buffer
-        float* wt = stage + kRing * (kPiece / 4);
-        float mx = -INFINITY;
-        for (int sp = 0; sp < nsplit; ++sp)
-          mx = fmaxf(mx, __ldcg(p.part_lse + (long long)(c0 + sp * cstride) * kTcRows + r));
-        float wsum = 0.f;
-        for (int sp = 0; sp < nsplit; ++sp) {
-          const float ls = __ldcg(p.part_lse + (long long)(c0 + sp * cstride) * kTcRows + r);
-          const float w = (ls == -INFINITY) ? 0.f : __expf(ls - mx);
-          wsum += w;
-          wt[sp * kTcRows + r] = w;
-        }
-        const float inv_w = wsum > 0.f ? 1.f / wsum : 0.f;
-        // the other splits' pieces stream through the ring: piece i = (column
-        // block i / (nsplit-1), i-th other split); warp 0 issues the copies.
-        // Splits are summed in split order with the same arithmetic for the
-        // own chunk (tensor memory) as for the others, so the result does not
-        // depend on which CTA arrived last.
-        const int others = nsplit - 1, n_pieces = (D / 32) * others;
-        auto issue = [&](int i) {
-          const int t = i % others, sp = t < split ? t : t + 1;
-          const int b = i % kRing;
-          mbar_expect_tx(bar(B_MF + b), kPiece);
-          bulk_load(sbase + b * kPiece,
-                    p.part_o + (long long)(c0 + sp * cstride) * kTcRows * D + (long long)(i / others) * 32 * kTcRows,
-                    kPiece, bar(B_MF + b));
-        };
-        int issued = 0;
-        if (warp == 0) {
-          if (lane == 0)
-            for (int i = 0; i < min(kRing, n_pieces); ++i) issue(i);
-          issued = min(kRing, n_pieces);
-        }
-        asm volatile("bar.sync 1, 256;" ::: "memory");   // weights visible to all rows' threads
-        bool mok = true;
-#pragma unroll 1
-        for (int c = 0; mok && c < D / 32; ++c) {
-          float own[32], acc[32];
-          if (ntile > 0) {
-            tmem_ld32(o_col + c * 32, own);
-            tc_wait_ld();
-#pragma unroll
-            for (int k = 0; k < 32; ++k) own[k] = own[k] * inv_l;   // the value the other CTAs would read
-          } else {
-#pragma unroll
-            for (int k = 0; k < 32; ++k) own[k] = 0.f;
-          }
-#pragma unroll
-          for (int k = 0; k < 32; ++k) acc[k] = 0.f;
-#pragma unroll 1
-          for (int sp = 0; sp < nsplit; ++sp) {
-            const float w = wt[sp * kTcRows + r];
-            if (sp == split) {
-#pragma unroll
-              for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w, own[k], acc[k]);
-              continue;
-            }
-            const int i = c * others + (sp < split ? sp : sp - 1), b = i % kRing;
-            if (!(mok = warp_wait(bar(B_MF + b), (i / kRing) & 1, abort_flag, p.wait_limit, p.status))) break;
-            const float* src = stage + b * (kPiece / 4) + r;
-#pragma unroll
-            for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w, src[k * kTcRows], acc[k]);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(B_ME + b));
-            if (warp == 0 && i + kRing < n_pieces) {
-              if (!(mok = warp_wait(bar(B_ME + b), (i / kRing) & 1, abort_flag, p.wait_limit, p.status))) break;
-              if (lane == 0) issue(i + kRing);
-              ++issued;
-            }
-          }
-          if (mok && row_ok) store_row32o(c, acc, inv_w);
-        }
-        if (warp == 0 && !mok && lane == 0) {   // let the copies this CTA issued land
-          for (int i = max(0, issued - kRing); i < issued; ++i)
-            mbar_drain(bar(B_MF + i % kRing), (i / kRing) & 1, p.status);
-        }
-        if (mok && row_ok && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
-      }
-    } else if (ok && ntile > 0) {
-      const long long orow = out_row(epr);
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
-        float o[32];
-        tmem_ld32(o_col + c * 32, o);
-        tc_wait_ld();
-        if (row_ok) store_row32(orow, c, o, inv_l);
-      }
-      if (row_ok && p.lse_out) p.lse_out[orow] = lse;
-    }
+    tc_epilogue<D>(p, smem, o_col, ok, m_run, l_run, ntile);
   }
   tc_fence_before();
   __syncthreads();

@@ -479,8 +479,9 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
   int chunk;
   if (ctx->opt_split > 0) {
     chunk = ctx->opt_split;
-    if (tc && ctx->opt_merge == 2 && maxv > chunk)
+    if (tc && ctx->opt_merge == 2 && maxv > chunk) {
       cluster_ns = std::min(8, std::max(2, (maxv + chunk - 1) / chunk));
+    }
   } else if (tc) {
     // Independent splits, one CTA per SM.  Cost of a chunk size = waves x
     // (tiles per CTA + ~4 tiles for the prologue and epilogue + ~2 for the
