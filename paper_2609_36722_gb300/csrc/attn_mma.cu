@@ -35,6 +35,8 @@ struct MmaLayout {
 template <int D>
 __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ AttnParams p) {
   using L = MmaLayout<D>;
+  grid_dep_wait();     // Q and the suffix K/V may come from the previous kernel
+  grid_dep_launch();   // the combine kernel may be scheduled as CTAs finish
   constexpr int NT = D / 8;           // n8 tiles of the output
   constexpr int KS = D / 16;          // k16 steps of QK^T
   extern __shared__ uint8_t smem_raw[];
@@ -324,8 +326,7 @@ static cudaError_t launch_attn_mma_t(const AttnParams& p, cudaStream_t st) {
   using L = MmaLayout<D>;
   cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
-  attn_mma_kernel<D><<<p.work.n_cta, 160, L::SMEM, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(attn_mma_kernel<D>, dim3(p.work.n_cta), dim3(160), (size_t)L::SMEM, st, 0, p);
 }
 
 cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st) {
@@ -340,6 +341,7 @@ cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st) {
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ CombineParams p,
                                                       long long total_rows) {
+  grid_dep_wait();   // the partial results of the attention kernel just before
   const long long gw = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (gw >= total_rows) return;
@@ -394,8 +396,7 @@ cudaError_t launch_combine(const CombineParams& p, cudaStream_t st) {
   const long long total_rows = (long long)p.work.n_req * p.Hkv * p.work.row_tiles * p.rows_per_tile;
   const long long threads = total_rows * 32;
   const int grid = (int)((threads + 255) / 256);
-  combine_kernel<<<grid, 256, 0, st>>>(p, total_rows);
-  return cudaGetLastError();
+  return launch_pdl(combine_kernel, dim3(grid), dim3(256), 0, st, 0, p, total_rows);
 }
 
 }  // namespace att

@@ -169,6 +169,7 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
   auto bar = [&](int i) { return smem_u32(&bars[i]); };
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int G = p.G;
+  grid_dep_wait();   // before the first global write (the producer thread has waited already)
   const TcCta ce = tc_cta(p, blockIdx.x);
   const int split = ce.split, nsplit = ce.nsplit;
   const int erow = threadIdx.x;                               // CTA row = thread (warps 0..7)
@@ -469,19 +470,31 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
       tma_prefetch_desc(&p.tm_q);
       tma_prefetch_desc(&p.tm_kpool);
       tma_prefetch_desc(&p.tm_vpool);
-      mbar_expect_tx(bar(B_Q), 2 * L::NH * L::HALF);
+      // Only kernels that never signal an early launch write the paged pool,
+      // so its blocks of the first tile may load while the previous kernel of
+      // the stream is still running; Q and suffix K/V wait for it.
+      bool dep_done = false;
+      auto dep = [&]() {
+        if (!dep_done) grid_dep_wait();
+        dep_done = true;
+      };
+      auto load_q = [&]() {
+        dep();
+        mbar_expect_tx(bar(B_Q), 2 * L::NH * L::HALF);
 #pragma unroll
-      for (int qt = 0; qt < 2; ++qt) {
+        for (int qt = 0; qt < 2; ++qt) {
 #pragma unroll
-        for (int h = 0; h < L::NH; ++h)
-          tma_load_5d(sbase + L::Q_OFF + (qt * L::NH + h) * L::HALF, &p.tm_q, bar(B_Q), h * 64, 0, kvh,
-                      (row0 + qt * kTcTileRows) / G, req);
-      }
+          for (int h = 0; h < L::NH; ++h)
+            tma_load_5d(sbase + L::Q_OFF + (qt * L::NH + h) * L::HALF, &p.tm_q, bar(B_Q), h * 64, 0, kvh,
+                        (row0 + qt * kTcTileRows) / G, req);
+        }
+      };
       int issued_k = 0, issued_v = 0;
       constexpr uint32_t tile_bytes = 2 * L::NH * (kBlockTokens * 128);
       for (int j = 0; j < ntile; ++j) {
         const int st = j % L::NS;
         const int e0 = list[2 * j], e1 = list[2 * j + 1];
+        if (e0 < 0 || e1 < 0) dep();
         if (j >= L::NS &&
             !mbar_wait(bar(B_KE + st), ((j / L::NS) - 1) & 1, abort_flag, p.wait_limit, p.status))
           break;
@@ -491,6 +504,7 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
         load_slot<D>(kd + kBlockTokens * 128, e1, &p.tm_kpool, &p.tm_ksuf, bar(B_KF + st), kvh,
                      p.Hkv, req, pool_rows);
         issued_k = j + 1;
+        if (j == 0) load_q();
         if (j >= L::NS &&
             !mbar_wait(bar(B_VE + st), ((j / L::NS) - 1) & 1, abort_flag, p.wait_limit, p.status))
           break;
@@ -686,23 +700,7 @@ static cudaError_t launch_attn_tc_t(const AttnParams& p, cudaStream_t st) {
   if (fa.numRegs * 384 < 128 * kCtrlRegs + 256 * kSoftRegs) return cudaErrorLaunchOutOfResources;
   e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
-  if (p.work.cluster > 0) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.work.n_cta);
-    cfg.blockDim = dim3(384);
-    cfg.dynamicSmemBytes = L::SMEM;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = p.work.cluster;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, attn_tc_kernel<D>, p);
-  }
-  attn_tc_kernel<D><<<p.work.n_cta, 384, L::SMEM, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(attn_tc_kernel<D>, dim3(p.work.n_cta), dim3(384), (size_t)L::SMEM, st, p.work.cluster, p);
 }
 
 // clusters of `ns` CTAs of this kernel that fit on the device at once (0: none)

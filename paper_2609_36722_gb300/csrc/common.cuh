@@ -193,6 +193,17 @@ ATT_DEV void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "mem
 ATT_DEV void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // ---------------------------------------------------------------------------
+// Programmatic dependent launch.  Kernels of this library are launched so
+// that they may start while the previous kernel in the stream is finishing.
+// A kernel calls grid_dep_wait() before it reads anything an earlier kernel
+// of the stream may still be writing, and before its first global write;
+// once the previous grid has completed it returns at once.
+// grid_dep_launch() lets the next kernel start its own prologue early.
+// ---------------------------------------------------------------------------
+ATT_DEV void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+ATT_DEV void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// ---------------------------------------------------------------------------
 // Thread-block clusters: barrier and distributed shared memory
 // ---------------------------------------------------------------------------
 // every thread of every CTA in the cluster; release/acquire orders the shared

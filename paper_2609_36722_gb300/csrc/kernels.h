@@ -77,6 +77,34 @@ cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __
                               cudaStream_t st);
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st);
 cudaError_t launch_qproj(const QprojParams& p, int D, cudaStream_t st);
+// Launch with programmatic stream serialization (the kernel may start while
+// the previous kernel of the stream finishes; see grid_dep_wait) and, when
+// cluster > 0, thread-block clusters of that many CTAs along x.
+template <typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       int cluster, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  int n = 0;
+  attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[n].val.programmaticStreamSerializationAllowed = 1;
+  ++n;
+  if (cluster > 0) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = cluster;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // how many clusters of `ns` tcgen05 attention CTAs fit on the current device at once
 int attn_tc_max_clusters(int D, int ns);
 cudaError_t launch_attn_tc(const AttnParams& p, int D, cudaStream_t st);

@@ -50,6 +50,8 @@ cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __
 // in float on |angle| <= pi.  The first threads also clear the split-K
 // arrival counters the Q-projection kernel uses in this call.
 __global__ void __launch_bounds__(256) prep_kernel(const __grid_constant__ PrepParams p) {
+  grid_dep_wait();     // the scratch it writes may be memory the previous kernel used
+  grid_dep_launch();   // the Q projection may start its main loop now
   const long long idx = (long long)blockIdx.x * 256 + threadIdx.x;
   if (p.counters != nullptr && idx < p.n_counters) p.counters[idx] = 0;
   const int half = p.D / 2;
@@ -67,8 +69,7 @@ __global__ void __launch_bounds__(256) prep_kernel(const __grid_constant__ PrepP
 
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st) {
   const long long n = std::max<long long>((long long)p.M * (p.D / 2), p.n_counters);
-  prep_kernel<<<(int)((n + 255) / 256), 256, 0, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(prep_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, 0, p);
 }
 
 }  // namespace att

@@ -279,7 +279,9 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
       }
     }
   } else {
-    // epilogue: warps 2..5 -> TMEM lane quadrants 2, 3, 0, 1
+    // epilogue: warps 2..5 -> TMEM lane quadrants 2, 3, 0, 1.  The RoPE table
+    // and the split-K counters come from the prep kernel just before this one.
+    grid_dep_wait();
     if (warp_wait(bar(QB_ACC), 0, abort_flag, p.wait_limit, p.status)) {
       tc_fence_after();
       const int nl = lora ? p.n_lora : 0;
@@ -289,6 +291,9 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
       else qproj_epilogue<D, 64>(p, sbase, tmem, bars, abort_flag, last_flag, head, ks, tile, m0);
     }
   }
+  // let the attention kernel launch once every CTA is here (triggering at the
+  // start measured slower: its early CTAs crowd the SMs the tail needs)
+  grid_dep_launch();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -303,8 +308,7 @@ static cudaError_t launch_qproj_t(const QprojParams& p, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(qproj_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
   dim3 grid(p.Hq * p.ksplit, (p.M + 127) / 128);
-  qproj_kernel<D><<<grid, 192, L::SMEM, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(qproj_kernel<D>, grid, dim3(192), (size_t)L::SMEM, st, 0, p);
 }
 
 cudaError_t launch_qproj(const QprojParams& p, int D, cudaStream_t st) {
