@@ -196,6 +196,34 @@ attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, 
                                     const void* suffix_k, const void* suffix_v, int32_t S,
                                     int32_t S_kv, void* out, float* lse_out, void* stream);
 
+/* Warm-cache load (the "CPU RAM cache lookup and GPU transfer" stage of the
+ * paper's time-to-first-token, Sec. 5 / App. A.3: encoded artifacts kept in
+ * host memory and moved to the GPU when a request needs them).  Registers n
+ * artifacts whose K/V live in PINNED host memory (cudaMallocHost /
+ * cudaHostAlloc / a pinned torch tensor) in one kernel that reads them over
+ * the CPU-GPU link and writes their paged pool blocks, on `stream`; run it on
+ * a second stream to overlap it with attuner_q_project, and make the attention
+ * stream wait for it.
+ *   k_host[i], v_host[i] : [L[i], Hkv, d] bf16, pinned host memory, 16-byte
+ *                          aligned; the caller keeps them alive and unchanged
+ *                          until the copy has run.
+ *   ids_out[i]           : artifact ids, allocated as by
+ *                          attuner_register_artifact, in order.
+ *   1 <= n <= ATTUNER_MAX_HOST_BATCH.
+ * Errors: INVALID_ARG (n out of range, L <= 0, NULL or unaligned pointers,
+ * memory that is not pinned host memory), OOM (pool full; nothing is
+ * registered then). */
+#define ATTUNER_MAX_HOST_BATCH 64
+attuner_status attuner_register_artifacts_host(attuner_ctx* ctx, int32_t n, const void* const* k_host,
+                                               const void* const* v_host, const int32_t* L,
+                                               void* stream, int32_t* ids_out);
+
+/* Forget every registered artifact: the pool is empty again and the next
+ * artifact gets id 0 and block 0 (a serving loop's eviction of the whole warm
+ * set).  Plans made before must not be used afterwards, and the caller must
+ * not reset while kernels that read the pool are still running. */
+attuner_status attuner_pool_reset(attuner_ctx* ctx);
+
 /* The paged pool: device base pointers of K and V ([pool_blocks][Hkv][64][d]
  * bf16 each), blocks in use and capacity.  Any output may be NULL. */
 attuner_status attuner_pool_info(const attuner_ctx* ctx, void** k_pool, void** v_pool,

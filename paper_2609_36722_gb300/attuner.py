@@ -41,7 +41,7 @@ EXPORTS = [
     "attuner_plan_export", "attuner_plan_t_art", "attuner_plan_free", "attuner_q_project",
     "attuner_attend", "attuner_query_attend", "attuner_pool_info", "attuner_sync_status",
     "attuner_set_option", "attuner_last_launch_count", "attuner_last_error",
-    "attuner_attend_static_scratch",
+    "attuner_attend_static_scratch", "attuner_register_artifacts_host", "attuner_pool_reset",
 ]
 
 
@@ -88,6 +88,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "attuner_set_option": ([_vp, _i32, ctypes.c_int64], _i32),
         "attuner_last_launch_count": ([_vp], _i32),
         "attuner_last_error": ([], ctypes.c_char_p),
+        "attuner_register_artifacts_host": ([_vp, _i32, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _p_i32, _vp,
+                                             _p_i32], _i32),
+        "attuner_pool_reset": ([_vp], _i32),
     }
     for name, (args, ret) in sig.items():
         f = getattr(lib, name)
@@ -204,6 +207,30 @@ class Context:
         _check(lib().attuner_register_artifact(self.handle, _ptr(k, "k"), _ptr(v, "v"), k.shape[0],
                                                _stream(stream), ctypes.byref(aid)))
         return aid.value
+
+    def register_artifacts_host(self, ks: Sequence[torch.Tensor], vs: Sequence[torch.Tensor], stream=None) -> list:
+        """Warm-cache load: artifacts whose K/V are pinned CPU tensors [L, Hkv, d]
+        bf16, copied into the pool by one kernel on `stream`.  Keep the tensors
+        alive and unchanged until that stream has run the copy."""
+        n = len(ks)
+        if n != len(vs) or n == 0:
+            raise ValueError("ks and vs must be non-empty lists of the same length")
+        for k, v in zip(ks, vs):
+            if k.is_cuda or v.is_cuda or not (k.is_pinned() and v.is_pinned()):
+                raise ValueError("ks and vs must be pinned CPU tensors")
+            if k.dtype != torch.bfloat16 or v.dtype != torch.bfloat16 or k.shape != v.shape or k.dim() != 3:
+                raise ValueError("each k, v must be bf16 [L, Hkv, d] of the same shape")
+            if not (k.is_contiguous() and v.is_contiguous()):
+                raise ValueError("ks and vs must be contiguous")
+        kp = (_vp * n)(*[k.data_ptr() for k in ks])
+        vp = (_vp * n)(*[v.data_ptr() for v in vs])
+        lens = (ctypes.c_int32 * n)(*[k.shape[0] for k in ks])
+        ids = (ctypes.c_int32 * n)()
+        _check(lib().attuner_register_artifacts_host(self.handle, n, kp, vp, lens, _stream(stream), ids))
+        return list(ids)
+
+    def pool_reset(self) -> None:
+        _check(lib().attuner_pool_reset(self.handle))
 
     def assemble(self, requests: Sequence[Sequence[int]]) -> Plan:
         reqs = [list(map(int, r)) for r in requests]

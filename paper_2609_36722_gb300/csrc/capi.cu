@@ -196,6 +196,63 @@ extern "C" attuner_status attuner_register_artifact(attuner_ctx* ctx, const void
   return ATTUNER_OK;
 }
 
+extern "C" attuner_status attuner_register_artifacts_host(attuner_ctx* ctx, int32_t n, const void* const* k_host,
+                                                          const void* const* v_host, const int32_t* L,
+                                                          void* stream, int32_t* ids_out) {
+  CHECK_ARG(ctx != nullptr, "ctx must not be NULL");
+  CHECK_ARG(n >= 1 && n <= ATTUNER_MAX_HOST_BATCH,
+            "n must be in [1, " + std::to_string(ATTUNER_MAX_HOST_BATCH) + "]");
+  CHECK_ARG(k_host != nullptr && v_host != nullptr && L != nullptr, "k_host, v_host and L must not be NULL");
+  attuner_status s = set_device(ctx);
+  if (s != ATTUNER_OK) return s;
+  HostBatch* b = new HostBatch();
+  auto done = [&](attuner_status st) { delete b; return st; };
+  const int Hkv = ctx->cfg.n_kv_heads, D = ctx->cfg.head_dim;
+  long long blocks = 0, chunks = 0;
+  for (int i = 0; i < n; ++i) {
+    if (L[i] <= 0) return done(fail(ATTUNER_ERR_INVALID_ARG, "artifact length L must be > 0"));
+    if (!k_host[i] || !v_host[i] || !aligned16(k_host[i]) || !aligned16(v_host[i]))
+      return done(fail(ATTUNER_ERR_INVALID_ARG, "k_host and v_host must be non-NULL and 16-byte aligned"));
+    for (const void* ptr : {k_host[i], v_host[i]}) {
+      cudaPointerAttributes at{};
+      if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess || at.type != cudaMemoryTypeHost) {
+        cudaGetLastError();
+        return done(fail(ATTUNER_ERR_INVALID_ARG, "k_host and v_host must be pinned host memory"));
+      }
+    }
+    b->k[i] = static_cast<const uint4*>(k_host[i]);
+    b->v[i] = static_cast<const uint4*>(v_host[i]);
+    b->first[i] = ctx->used_blocks + (int)blocks;
+    b->L[i] = L[i];
+    blocks += (L[i] + 63) / 64;
+    chunks += (long long)L[i] * Hkv * (D / 8);
+    b->chunk_end[i] = chunks;
+  }
+  if (ctx->used_blocks + blocks > ctx->cfg.pool_blocks)
+    return done(fail(ATTUNER_ERR_OOM, "artifact pool is full: " + std::to_string(ctx->used_blocks) + " of " +
+                                          std::to_string(ctx->cfg.pool_blocks) + " blocks used, " +
+                                          std::to_string(blocks) + " more needed"));
+  b->n = n;
+  b->Hkv = Hkv;
+  b->D = D;
+  CUDA_TRY(launch_pool_write_host(*b, ctx->kpool, ctx->vpool, ctx->num_sms, static_cast<cudaStream_t>(stream)));
+  for (int i = 0; i < n; ++i) {
+    ctx->arts.push_back(Artifact{b->first[i], L[i], (L[i] + 63) / 64});
+    if (ids_out) ids_out[i] = (int32_t)ctx->arts.size() - 1;
+  }
+  ctx->used_blocks += (int32_t)blocks;
+  ctx->last_launches = 1;
+  return done(ATTUNER_OK);
+}
+
+extern "C" attuner_status attuner_pool_reset(attuner_ctx* ctx) {
+  CHECK_ARG(ctx != nullptr, "ctx must not be NULL");
+  ctx->arts.clear();
+  ctx->used_blocks = 0;
+  ctx->last_launches = 0;
+  return ATTUNER_OK;
+}
+
 // ---------------------------------------------------------------------------
 // plans
 // ---------------------------------------------------------------------------

@@ -72,6 +72,19 @@ struct CombineParams {
 };
 
 // Pool repack: caller K/V [L, Hkv, D] -> pool blocks [first + p/64][h][p%64][:]
+// Batched pool write from host memory: artifact i copies [L[i], Hkv, D] K/V
+// from k[i], v[i] (pinned host memory, read by the kernel over the CPU-GPU
+// link) into pool blocks first[i] ...
+struct HostBatch {
+  const uint4* k[ATTUNER_MAX_HOST_BATCH];
+  const uint4* v[ATTUNER_MAX_HOST_BATCH];
+  long long chunk_end[ATTUNER_MAX_HOST_BATCH];   // inclusive prefix sums of L[i] * Hkv * D / 8
+  int32_t L[ATTUNER_MAX_HOST_BATCH];
+  int32_t first[ATTUNER_MAX_HOST_BATCH];
+  int32_t n, Hkv, D;
+};
+cudaError_t launch_pool_write_host(const HostBatch& b, __nv_bfloat16* kpool, __nv_bfloat16* vpool,
+                                   int num_sms, cudaStream_t st);
 cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __nv_bfloat16* kpool,
                               __nv_bfloat16* vpool, int L, int Hkv, int D, int first_block,
                               cudaStream_t st);

@@ -29,6 +29,20 @@ __global__ void pool_write_kernel(const uint4* __restrict__ k, const uint4* __re
     kpool[dst] = k[i];
     vpool[dst] = v[i];
   }
+  // unused tail slots of the last block read as zeros (see pool_write_host_kernel)
+  const int tail = L % kBlockTokens;
+  if (tail != 0) {
+    const long long nt = (long long)(kBlockTokens - tail) * Hkv * cpr;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < nt;
+         i += (long long)gridDim.x * blockDim.x) {
+      const int c = (int)(i % cpr);
+      const int h = (int)((i / cpr) % Hkv);
+      const int slot = tail + (int)(i / ((long long)cpr * Hkv));
+      const long long dst = (((long long)(first_block + L / kBlockTokens) * Hkv + h) * kBlockTokens + slot) * cpr + c;
+      kpool[dst] = make_uint4(0, 0, 0, 0);
+      vpool[dst] = make_uint4(0, 0, 0, 0);
+    }
+  }
 }
 
 cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __nv_bfloat16* kpool,
@@ -41,6 +55,58 @@ cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __
                                           reinterpret_cast<const uint4*>(v),
                                           reinterpret_cast<uint4*>(kpool),
                                           reinterpret_cast<uint4*>(vpool), L, Hkv, D, first_block);
+  return cudaGetLastError();
+}
+
+// The warm-cache load: one pass over every 16-byte chunk of a batch of host
+// artifacts.  Consecutive threads read consecutive chunks of one artifact
+// (coalesced reads over the CPU-GPU link); each chunk lands in its pool slot
+// [block][h][token % 64][:] as in pool_write_kernel.
+__global__ void __launch_bounds__(256) pool_write_host_kernel(const __grid_constant__ HostBatch b,
+                                                              uint4* __restrict__ kpool,
+                                                              uint4* __restrict__ vpool) {
+  const int cpr = b.D / 8;
+  const long long total = b.chunk_end[b.n - 1];
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+       i += (long long)gridDim.x * blockDim.x) {
+    int a = 0;
+    while (b.chunk_end[a] <= i) ++a;                    // n <= 64: a short scan
+    const long long li = i - (a > 0 ? b.chunk_end[a - 1] : 0);
+    const int c = (int)(li % cpr);
+    const long long ph = li / cpr;
+    const int h = (int)(ph % b.Hkv);
+    const int t = (int)(ph / b.Hkv);
+    const long long dst =
+        (((long long)(b.first[a] + t / kBlockTokens) * b.Hkv + h) * kBlockTokens + t % kBlockTokens) * cpr + c;
+    kpool[dst] = b.k[a][li];
+    vpool[dst] = b.v[a][li];
+  }
+  // zero the unused tail slots of each artifact's last block: the pool may
+  // hold an earlier artifact there after attuner_pool_reset, and a masked key
+  // still multiplies its V row by 0
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < (long long)b.n * kBlockTokens * b.Hkv * cpr;
+       i += (long long)gridDim.x * blockDim.x) {
+    const int c = (int)(i % cpr);
+    const long long r = i / cpr;
+    const int h = (int)(r % b.Hkv);
+    const int slot = (int)((r / b.Hkv) % kBlockTokens);
+    const int a = (int)(r / ((long long)b.Hkv * kBlockTokens));
+    const int tail = b.L[a] % kBlockTokens;
+    if (tail == 0 || slot < tail) continue;
+    const int blk = b.first[a] + b.L[a] / kBlockTokens;
+    const long long dst = (((long long)blk * b.Hkv + h) * kBlockTokens + slot) * cpr + c;
+    kpool[dst] = make_uint4(0, 0, 0, 0);
+    vpool[dst] = make_uint4(0, 0, 0, 0);
+  }
+}
+
+cudaError_t launch_pool_write_host(const HostBatch& b, __nv_bfloat16* kpool, __nv_bfloat16* vpool,
+                                   int num_sms, cudaStream_t st) {
+  const long long total = b.chunk_end[b.n - 1];
+  long long grid = (total + 255) / 256;
+  if (grid > (long long)num_sms * 8) grid = (long long)num_sms * 8;
+  pool_write_host_kernel<<<(int)grid, 256, 0, st>>>(b, reinterpret_cast<uint4*>(kpool),
+                                                    reinterpret_cast<uint4*>(vpool));
   return cudaGetLastError();
 }
 
