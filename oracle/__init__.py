@@ -13,7 +13,10 @@ Every function is a plain restatement of the paper's definitions in float64:
     assembled in prompt order;
   * Sec. 2.2, Eq. (routing-oracle): softmax(q K^T / sqrt(d_k) + M_t) V;
   * App. A.5 (Deployment): merged W^Q + (alpha/r) B A, SDPA with causal masks
-    and position ids for the assembled context.
+    and position ids for the assembled context;
+  * the suffix tokens' own keys and values: base k_proj / v_proj (the
+    adaptation touches W^Q only, Sec. 3), key normalisation and RoPE at their
+    assembled positions.
 
 Parity status: every function is pinned by the tests in
 ``tests/test_oracle_pins.py`` (closed forms, hand-derived fixtures under
@@ -30,6 +33,7 @@ from .attuner_oracle import (  # noqa: F401
     rms_norm_heads,
     rope_rotate_half,
     query_positions,
+    kv_projection,
     assemble,
     attention,
     request_forward,

@@ -89,6 +89,25 @@ def query_positions(t_art: int, S: int, S_kv: int) -> np.ndarray:
 
 
 # ---------------------------------------------------------------------------
+# Online K/V of the suffix tokens.  The adaptation changes W^Q only (Sec. 3:
+# the keys and values keep the base model's projections, which is what keeps
+# the cached artifact KV valid); the base model normalises each key head
+# (Qwen3 k_norm) and rotates it at the token's assembled position (App. A.5).
+# ---------------------------------------------------------------------------
+def kv_projection(x: np.ndarray, w_k: np.ndarray, w_v: np.ndarray, k_norm_w: np.ndarray, eps: float,
+                  theta: float, positions: np.ndarray, n_kv_heads: int) -> Tuple[np.ndarray, np.ndarray]:
+    """x [S_new, d_model]; w_k, w_v [Hkv*d, d_model]; k_norm_w [d]; positions [S_new].
+
+    K [S_new, Hkv, d] = RoPE(RMSNorm(x W_k^T per head) * w, pos);  V = x W_v^T.
+    """
+    d = w_k.shape[0] // n_kv_heads
+    k = rms_norm_heads((x @ w_k.T).reshape(-1, n_kv_heads, d), k_norm_w, eps)
+    k = rope_rotate_half(k, positions, theta)
+    v = (x @ w_v.T).reshape(-1, n_kv_heads, d)
+    return k, v
+
+
+# ---------------------------------------------------------------------------
 # Sec. 2 (PIC box, Eq. full-vs-pic) and App. A.3 "Cache construction and
 # reuse": cached blocks are assembled in prompt order without re-encoding.
 # Paging in 64-token blocks is this library's storage, not the paper's.

@@ -137,6 +137,49 @@ def test_rope_invariants():
                                O.rope_rotate_half(q, p + p2, theta), atol=1e-9)
 
 
+def test_kv_projection_invariants():
+    # The suffix tokens' keys and values (base k_proj / v_proj, Sec. 3: only
+    # W^Q is adapted), pinned by properties a dropped term, a transposed
+    # operand, a wrong axis or a wrong position would break.
+    rng = np.random.default_rng(21)
+    hkv, d, hidden, theta = 2, 8, 6, 1.0e6
+    w_k = rng.standard_normal((hkv * d, hidden))
+    w_v = rng.standard_normal((hkv * d, hidden))
+    ones = np.ones(d)
+    # a basis input selects one column of each weight: V is that column, K its
+    # per-head unit-RMS normalisation (position 0: no rotation, eps = 0)
+    for i in range(hidden):
+        x = np.zeros((1, hidden))
+        x[0, i] = 1.0
+        k, v = O.kv_projection(x, w_k, w_v, ones, 0.0, theta, np.array([0]), hkv)
+        np.testing.assert_allclose(v.reshape(-1), w_v[:, i], rtol=1e-14)
+        col = w_k[:, i].reshape(hkv, d)
+        np.testing.assert_allclose(k[0], col / np.sqrt(np.mean(col * col, axis=-1, keepdims=True)), rtol=1e-12)
+    x = rng.standard_normal((5, hidden))
+    pos = np.array([3, 40, 41, 700, 131000])
+    k, v = O.kv_projection(x, w_k, w_v, ones, 0.0, theta, pos, hkv)
+    # unit RMS per head survives the rotation: |k| = sqrt(d)
+    np.testing.assert_allclose(np.linalg.norm(k, axis=-1), np.sqrt(d), rtol=1e-12)
+    # V is linear in x and ignores positions and the key weights
+    k2, v2 = O.kv_projection(2.0 * x, w_k, w_v, ones, 0.0, theta, pos + 5, hkv)
+    np.testing.assert_allclose(v2, 2.0 * v, rtol=1e-13)
+    # the key normalisation is scale-invariant (eps = 0), so 2x only moves the rotation:
+    # shifting every position by 5 rotates each pair by 5 * inv_freq, preserving <k_t, k_u>
+    np.testing.assert_allclose(np.einsum("thd,uhd->thu", k2, k2), np.einsum("thd,uhd->thu", k, k), atol=1e-9)
+    # query . key depends only on the position difference (the property RoPE exists for)
+    q = rng.standard_normal((5, hkv, d))
+    for c in (1, 64, 4096):
+        kc, _ = O.kv_projection(x, w_k, w_v, ones, 0.0, theta, pos + c, hkv)
+        lhs = np.sum(O.rope_rotate_half(q, pos[::-1], theta) * k, axis=-1)
+        rhs = np.sum(O.rope_rotate_half(q, pos[::-1] + c, theta) * kc, axis=-1)
+        np.testing.assert_allclose(lhs, rhs, rtol=1e-9, atol=1e-9)
+    # the key-norm weight scales each channel after the normalisation
+    w = rng.standard_normal(d)
+    kw, _ = O.kv_projection(x, w_k, w_v, w, 0.0, theta, np.zeros(5, dtype=np.int64), hkv)
+    k0, _ = O.kv_projection(x, w_k, w_v, ones, 0.0, theta, np.zeros(5, dtype=np.int64), hkv)
+    np.testing.assert_allclose(kw, k0 * w, rtol=1e-12)
+
+
 def test_query_positions():
     # tiny workload: 201 artifact tokens, S = S_kv = 16 -> positions 201..216
     np.testing.assert_array_equal(O.query_positions(201, 16, 16), np.arange(201, 217))
