@@ -185,7 +185,7 @@ def cpu_baseline(wl, budget_s: float = 12.0, seed: int = 0):
 def run_ours(args, rank, world, local_rank):
     import torch
     import paper_2609_36722_gb300 as pkg
-    from gen import make_workload
+    from gen import make_kv_weights, make_workload
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
@@ -257,6 +257,20 @@ def run_ours(args, rank, world, local_rank):
         attn_ms.append(ev_a.elapsed_time(ev_b))
         qproj_ms.append(ev_q.elapsed_time(ev_a))
     torch.cuda.synchronize()
+    # the suffix tokens' K/V projection (§8(f) row 2), its own line: same x,
+    # base k_proj / v_proj weights of the geometry, into scratch suffix buffers
+    wk, wv, kn = make_kv_weights(g, 0, device=dev)
+    sk_s, sv_s = wl.suffix_k.clone(), wl.suffix_v.clone()
+    kv_ms = []
+    for i in range(args.steps + 3):
+        flush.zero_()
+        ev_q.record(stream)
+        ctx.kv_project(plan, wl.x, wk, wv, kn, sk_s, sv_s)
+        ev_a.record(stream)
+        ev_a.synchronize()
+        if i >= 3:
+            kv_ms.append(ev_q.elapsed_time(ev_a))
+    kv_flops = 2.0 * wl.n_req * wl.S * g.hidden * 2 * g.n_kv_heads * g.head_dim
     total_ms = sum(step_ms)
     if world > 1:
         t = torch.tensor([total_ms], device=dev)
@@ -389,6 +403,8 @@ def run_ours(args, rank, world, local_rank):
         "path_work": {"attention_flops": attention_flops(wl), "qproj_flops": qproj_flops(wl),
                       "kv_bytes": kv_bytes(wl)},
         # the Q projection (steps a1-a3: prep + qproj kernels) as its own line, from the same pass
+        "kv_project": {"avg_call_ms": round(statistics.mean(kv_ms), 5),
+                       "tflops": round(kv_flops / (statistics.mean(kv_ms) * 1e-3) / 1e12, 3)},
         "qproj": {"avg_call_ms": round(statistics.mean(qproj_ms), 5),
                   "tflops": round(qproj_flops(wl) / (statistics.mean(qproj_ms) * 1e-3) / 1e12, 3),
                   "frac_of_bf16_peak": round(qproj_flops(wl) / (statistics.mean(qproj_ms) * 1e-3) / 1e12 / peaks["bf16"], 4)},

@@ -11,5 +11,6 @@ from .workloads import (  # noqa: F401
     WORKLOADS,
     make_workload,
     make_custom,
+    make_kv_weights,
     layout,
 )

@@ -135,6 +135,19 @@ QWEN3_8B = Geometry(hidden=4096, n_q_heads=32, n_kv_heads=8, head_dim=128, rank=
 TINY = Geometry(hidden=256, n_q_heads=4, n_kv_heads=2, head_dim=64, rank=8)
 
 
+def make_kv_weights(geom: Geometry, seed: int, device="cpu"):
+    """Base k_proj / v_proj weights [Hkv*d, hidden] ~ N(0, 1/hidden) and a key
+    norm weight 1 + 0.1 N(0, 1), bf16, from a generator of their own seed."""
+    device = torch.device(device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed) + 1000)
+    n_out = geom.n_kv_heads * geom.head_dim
+    w_k = _normal((n_out, geom.hidden), geom.hidden ** -0.5, gen, device).to(torch.bfloat16)
+    w_v = _normal((n_out, geom.hidden), geom.hidden ** -0.5, gen, device).to(torch.bfloat16)
+    k_norm_w = (1.0 + 0.1 * _normal((geom.head_dim,), 1.0, gen, device)).to(torch.bfloat16)
+    return w_k, w_v, k_norm_w
+
+
 def _layout(name: str):
     """Lengths / requests / S / S_kv of the named workload (numpy-seeded)."""
     if name == "tiny":

@@ -188,6 +188,23 @@ attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const attuner_pla
                                              const void* suffix_v, int32_t S, int32_t S_kv,
                                              void* out, float* lse_out, void* stream);
 
+/* The suffix tokens' own keys and values (the layer's remaining online
+ * computation).  The adaptation changes W^Q only (Sec. 3), so K and V come
+ * from the base model's projections: for request r and new suffix token i < S
+ * (query position T_art(r) + S_kv - S + i, App. A.5)
+ *   suffix_k[r, S_kv - S + i, h, :] = RoPE(RMSNorm(x[r, i] W_k,h^T) * k_norm_w, pos)
+ *   suffix_v[r, S_kv - S + i, h, :] = x[r, i] W_v,h^T
+ *   x        [n_req, S, hidden] bf16
+ *   w_k, w_v [Hkv*d, hidden] bf16 (output x input)
+ *   k_norm_w [d] bf16
+ *   suffix_k, suffix_v [n_req, S_kv, Hkv, d] bf16: only the last S token rows
+ *            of each request are written, so a decode step (S = 1) appends
+ *            one token to KV the caller keeps.
+ * Errors: INVALID_ARG, CUDA. */
+attuner_status attuner_kv_project(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
+                                  const void* w_k, const void* w_v, const void* k_norm_w, int32_t S,
+                                  int32_t S_kv, void* suffix_k, void* suffix_v, void* stream);
+
 /* The whole path: attuner_q_project into stream-ordered scratch, then
  * attuner_attend.  Arguments as in those two calls. */
 attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, const void* x,

@@ -42,6 +42,7 @@ EXPORTS = [
     "attuner_attend", "attuner_query_attend", "attuner_pool_info", "attuner_sync_status",
     "attuner_set_option", "attuner_last_launch_count", "attuner_last_error",
     "attuner_attend_static_scratch", "attuner_register_artifacts_host", "attuner_pool_reset",
+    "attuner_kv_project",
 ]
 
 
@@ -91,6 +92,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "attuner_register_artifacts_host": ([_vp, _i32, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _p_i32, _vp,
                                              _p_i32], _i32),
         "attuner_pool_reset": ([_vp], _i32),
+        "attuner_kv_project": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
     }
     for name, (args, ret) in sig.items():
         f = getattr(lib, name)
@@ -256,6 +258,17 @@ class Context:
                                        _ptr(lora_a, "lora_a"), _ptr(lora_b, "lora_b"), r, float(s),
                                        _ptr(q_norm_w, "q_norm_w"), S, S_kv, _ptr(out, "out"), _stream(stream)))
         return out
+
+    def kv_project(self, plan: Plan, x, w_k, w_v, k_norm_w, suffix_k, suffix_v, stream=None) -> None:
+        """Write the new suffix tokens' K and V (the last S token rows of each
+        request in suffix_k / suffix_v [n_req, S_kv, Hkv, d]) from x [n_req, S, hidden]."""
+        n_req, S, hidden = x.shape
+        S_kv = suffix_k.shape[1]
+        if suffix_k.shape != suffix_v.shape or suffix_k.shape[0] != n_req:
+            raise ValueError("suffix_k and suffix_v must both be [n_req, S_kv, Hkv, d]")
+        _check(lib().attuner_kv_project(self.handle, plan.handle, _ptr(x, "x"), _ptr(w_k, "w_k"), _ptr(w_v, "w_v"),
+                                        _ptr(k_norm_w, "k_norm_w"), S, S_kv, _ptr(suffix_k, "suffix_k"),
+                                        _ptr(suffix_v, "suffix_v"), _stream(stream)))
 
     def attend(self, plan: Plan, q, suffix_k, suffix_v, out: Optional[torch.Tensor] = None,
                lse: Optional[torch.Tensor] = None, want_lse: bool = True, stream=None):

@@ -476,10 +476,82 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
   qp.M = M;
   qp.hidden = c.hidden;
   qp.Hq = Hq;
+  qp.kv = 0;
+  qp.Hout = Hq;
+  qp.S = S;
+  qp.S_out = S;
   qp.r = lora ? r : 0;
   qp.n_lora = n_lora;
   qp.ksplit = ksplit;
   qp.s = s;
+  qp.eps = c.rms_eps;
+  qp.status = ctx->d_status;
+  qp.wait_limit = ctx->wait_limit;
+  CUDA_TRY(launch_qproj(qp, D, st));
+  ++launches;
+  return ATTUNER_OK;
+}
+
+// The suffix tokens' own K and V: one launch of the Q-projection kernel in
+// K/V mode (grid heads 0..Hkv-1 project K with the key norm and RoPE, Hkv..
+// 2 Hkv-1 project V), after the prep kernel's RoPE table of the same positions.
+static attuner_status kv_project_impl(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
+                                      const void* w_k, const void* w_v, const void* k_norm_w, int32_t S,
+                                      int32_t S_kv, void* suffix_k, void* suffix_v, cudaStream_t st,
+                                      Scratch& sc, int& launches) {
+  const attuner_config& c = ctx->cfg;
+  CHECK_ARG(x && w_k && w_v && k_norm_w && suffix_k && suffix_v,
+            "x, w_k, w_v, k_norm_w, suffix_k and suffix_v must not be NULL");
+  CHECK_ARG(aligned16(x) && aligned16(w_k) && aligned16(w_v) && aligned16(k_norm_w) && aligned16(suffix_k) &&
+                aligned16(suffix_v),
+            "x, w_k, w_v, k_norm_w, suffix_k and suffix_v must be 16-byte aligned");
+  const int M = plan->n_req * S;
+  const int D = c.head_dim, Hkv = c.n_kv_heads, dkv = Hkv * D;
+  const size_t off_rope = sc.take((size_t)M * (D / 2) * 8);
+  char* base = static_cast<char*>(sc.base);
+  float2* rope = reinterpret_cast<float2*>(base + off_rope);
+
+  PrepParams pp{};
+  pp.rope = rope;
+  pp.t_art = plan_dev(plan).t_art;
+  pp.M = M;
+  pp.D = D;
+  pp.S = S;
+  pp.S_kv = S_kv;
+  for (int j = 0; j < D / 2; ++j) pp.inv_freq[j] = std::pow((double)c.rope_theta, -2.0 * j / (double)D);
+  CUDA_TRY(launch_prep(pp, st));
+  ++launches;
+
+  QprojParams qp{};
+  attuner_status e;
+  {
+    const uint64_t dims[2] = {(uint64_t)c.hidden, (uint64_t)M};
+    const uint64_t strides[1] = {(uint64_t)c.hidden * 2};
+    const uint32_t box[2] = {64, 128};
+    if ((e = make_map(&qp.tm_x, x, 2, dims, strides, box, "x")) != ATTUNER_OK) return e;
+  }
+  {
+    const uint64_t dims[2] = {(uint64_t)c.hidden, (uint64_t)dkv};
+    const uint64_t strides[1] = {(uint64_t)c.hidden * 2};
+    const uint32_t box[2] = {64, (uint32_t)D};
+    if ((e = make_map(&qp.tm_w, w_k, 2, dims, strides, box, "w_k")) != ATTUNER_OK) return e;
+    if ((e = make_map(&qp.tm_w2, w_v, 2, dims, strides, box, "w_v")) != ATTUNER_OK) return e;
+  }
+  qp.q_out = static_cast<__nv_bfloat16*>(suffix_k);
+  qp.out2 = static_cast<__nv_bfloat16*>(suffix_v);
+  qp.qnorm_w = static_cast<const __nv_bfloat16*>(k_norm_w);
+  qp.rope = rope;
+  qp.M = M;
+  qp.hidden = c.hidden;
+  qp.Hq = 2 * Hkv;
+  qp.kv = 1;
+  qp.Hout = Hkv;
+  qp.S = S;
+  qp.S_out = S_kv;
+  qp.r = 0;
+  qp.n_lora = 0;
+  qp.ksplit = 1;
+  qp.s = 0.f;
   qp.eps = c.rms_eps;
   qp.status = ctx->d_status;
   qp.wait_limit = ctx->wait_limit;
@@ -721,6 +793,24 @@ extern "C" attuner_status attuner_q_project(attuner_ctx* ctx, const attuner_plan
   CUDA_TRY(cudaMallocFromPoolAsync(&sc.base, sc.cap, ctx->mempool, st));
   int launches = 0;
   e = q_project_impl(ctx, plan, x, w_q, lora_a, lora_b, r, s, q_norm_w, S, S_kv, q_out, st, sc, launches);
+  cudaFreeAsync(sc.base, st);
+  ctx->last_launches = launches;
+  return e;
+}
+
+extern "C" attuner_status attuner_kv_project(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
+                                             const void* w_k, const void* w_v, const void* k_norm_w, int32_t S,
+                                             int32_t S_kv, void* suffix_k, void* suffix_v, void* stream) {
+  attuner_status e = check_common(ctx, plan, S, S_kv);
+  if (e != ATTUNER_OK) return e;
+  if ((e = set_device(ctx)) != ATTUNER_OK) return e;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  Scratch sc{ctx, st};
+  auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
+  sc.cap = al((size_t)plan->n_req * S * (ctx->cfg.head_dim / 2) * 8);
+  CUDA_TRY(cudaMallocFromPoolAsync(&sc.base, sc.cap, ctx->mempool, st));
+  int launches = 0;
+  e = kv_project_impl(ctx, plan, x, w_k, w_v, k_norm_w, S, S_kv, suffix_k, suffix_v, st, sc, launches);
   cudaFreeAsync(sc.base, st);
   ctx->last_launches = launches;
   return e;

@@ -29,12 +29,19 @@ struct QprojParams {
   CUtensorMap tm_w;    // W_q [d_q, hidden], box 64 x D, SW128
   CUtensorMap tm_a;    // A [r, hidden], box 64 x n_lora, SW128 (rows past r read as zeros)
   CUtensorMap tm_b;    // B [d_q, r], box 8 x D, no swizzle (columns past r read as zeros)
-  __nv_bfloat16* q_out;            // [M, Hq, D]
-  const __nv_bfloat16* qnorm_w;    // [D]
+  CUtensorMap tm_w2;   // K/V mode: W_v [Hkv*D, hidden], box 64 x D, SW128
+  __nv_bfloat16* q_out;            // Q mode: [M, Hq, D]; K/V mode: suffix K [n_req, S_kv, Hkv, D]
+  __nv_bfloat16* out2;             // K/V mode: suffix V [n_req, S_kv, Hkv, D]
+  const __nv_bfloat16* qnorm_w;    // [D] (q_norm, or k_norm in K/V mode)
   const float2* rope;              // [D/2, M] (cos, sin), pair-major
   float* part;                     // split-K partials [tiles][ksplit][128][D + n_lora]
   int32_t* counters;               // [tiles] arrivals per output tile (zero on entry)
-  int32_t M, hidden, Hq, r, n_lora, ksplit;
+  int32_t M, hidden, Hq, r, n_lora, ksplit;   // Hq: heads of the grid (2 Hkv in K/V mode)
+  // K/V mode (kv = 1): grid heads [0, Hout) project K (W = tm_w, key norm and
+  // RoPE), [Hout, 2 Hout) project V (W = tm_w2, stored as is).  Row m of the
+  // GEMM is token m % S of request m / S, written to output token row
+  // (m / S) * S_out + (S_out - S) + m % S (Q mode: S_out = S).
+  int32_t kv, Hout, S, S_out;
   float s, eps;
   int* status;
   long long wait_limit;

@@ -59,8 +59,8 @@ enum : int { QB_ACC = 0, QB_LORA = 1, QB_LUP = 2, QB_DRAIN = 3, QB_FULL = 4 };  
 template <int D, int R>
 __device__ __forceinline__ void qproj_epilogue(const QprojParams& p, uint32_t sbase, uint32_t tmem,
                                                uint64_t* bars, volatile int* abort_flag,
-                                               volatile int* last_flag, int head, int ks, int tile,
-                                               int m0) {
+                                               volatile int* last_flag, int head, bool is_v, int ks,
+                                               int tile, int m0) {
   using L = QpLayout<D>;
   constexpr int RU = R > 0 ? R : 1;
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -157,23 +157,28 @@ __device__ __forceinline__ void qproj_epilogue(const QprojParams& p, uint32_t sb
       for (int k = 0; k < 32; ++k) v[c * 32 + k] += t[k];
     }
   }
-  // RMSNorm * w, RoPE on pairs (j, j + D/2), bf16 store; rows past M store nothing
+  // RMSNorm * w, RoPE on pairs (j, j + D/2), bf16 store; rows past M store
+  // nothing; V (K/V mode) is stored as projected
   const bool row_ok = m < p.M;
   const int mr = row_ok ? m : p.M - 1;
-  float ss = 0.f;
+  if (!is_v) {
+    float ss = 0.f;
 #pragma unroll
-  for (int j = 0; j < D; ++j) ss = fmaf(v[j], v[j], ss);
-  const float rinv = rsqrtf(ss * (1.0f / D) + p.eps);
+    for (int j = 0; j < D; ++j) ss = fmaf(v[j], v[j], ss);
+    const float rinv = rsqrtf(ss * (1.0f / D) + p.eps);
 #pragma unroll
-  for (int j = 0; j < D / 2; ++j) {
-    const float2 cs = p.rope[(long long)j * p.M + mr];
-    const float a = v[j] * rinv * __bfloat162float(p.qnorm_w[j]);
-    const float b = v[j + D / 2] * rinv * __bfloat162float(p.qnorm_w[j + D / 2]);
-    v[j] = a * cs.x - b * cs.y;
-    v[j + D / 2] = b * cs.x + a * cs.y;
+    for (int j = 0; j < D / 2; ++j) {
+      const float2 cs = p.rope[(long long)j * p.M + mr];
+      const float a = v[j] * rinv * __bfloat162float(p.qnorm_w[j]);
+      const float b = v[j + D / 2] * rinv * __bfloat162float(p.qnorm_w[j + D / 2]);
+      v[j] = a * cs.x - b * cs.y;
+      v[j + D / 2] = b * cs.x + a * cs.y;
+    }
   }
   if (row_ok) {
-    uint4* dst = reinterpret_cast<uint4*>(p.q_out + ((long long)m * p.Hq + head) * D);
+    const long long t = (long long)(m / p.S) * p.S_out + (p.S_out - p.S) + m % p.S;   // output token row
+    __nv_bfloat16* base = is_v ? p.out2 : p.q_out;
+    uint4* dst = reinterpret_cast<uint4*>(base + (t * p.Hout + head) * D);
 #pragma unroll
     for (int c = 0; c < D / 8; ++c)
       dst[c] = make_uint4(pack_bf16(v[8 * c], v[8 * c + 1]), pack_bf16(v[8 * c + 2], v[8 * c + 3]),
@@ -199,7 +204,10 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
   const int ks = blockIdx.x % p.ksplit;
   const int tile = blockIdx.y * p.Hq + head;
   const int m0 = blockIdx.y * 128;
-  const int n0 = head * D;
+  const bool is_v = p.kv && head >= p.Hout;             // K/V mode: this CTA projects V
+  const int oh = is_v ? head - p.Hout : head;            // head within its output
+  const CUtensorMap* tm_w = is_v ? &p.tm_w2 : &p.tm_w;
+  const int n0 = oh * D;
   const int nk = p.hidden / 64;
   const int kb0 = ks * nk / p.ksplit, kb1 = (ks + 1) * nk / p.ksplit;
   const bool lora = p.n_lora > 0;
@@ -224,7 +232,7 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
   if (warp == 0) {
     if (lane == 0) {
       tma_prefetch_desc(&p.tm_x);
-      tma_prefetch_desc(&p.tm_w);
+      tma_prefetch_desc(tm_w);
       if (lora) {
         // B_h: r/8 boxes of [D rows][8 columns] (columns past r read as zeros)
         mbar_expect_tx(bar(QB_LORA), (p.n_lora / 8) * D * 16);
@@ -240,7 +248,7 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
         const uint32_t x_dst = sbase + st * L::STAGE;
         mbar_expect_tx(bar(B_FULL + st), stage_tx);
         tma_load_2d(x_dst, &p.tm_x, bar(B_FULL + st), kb * 64, m0);
-        tma_load_2d(x_dst + L::X_BYTES, &p.tm_w, bar(B_FULL + st), kb * 64, n0);
+        tma_load_2d(x_dst + L::X_BYTES, tm_w, bar(B_FULL + st), kb * 64, n0);
         if (lora) tma_load_2d(x_dst + L::X_BYTES + L::W_BYTES, &p.tm_a, bar(B_FULL + st), kb * 64, 0);
         issued = it + 1;
       }
@@ -285,10 +293,10 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
     if (warp_wait(bar(QB_ACC), 0, abort_flag, p.wait_limit, p.status)) {
       tc_fence_after();
       const int nl = lora ? p.n_lora : 0;
-      if (nl == 0) qproj_epilogue<D, 0>(p, sbase, tmem, bars, abort_flag, last_flag, head, ks, tile, m0);
-      else if (nl <= 16) qproj_epilogue<D, 16>(p, sbase, tmem, bars, abort_flag, last_flag, head, ks, tile, m0);
-      else if (nl <= 32) qproj_epilogue<D, 32>(p, sbase, tmem, bars, abort_flag, last_flag, head, ks, tile, m0);
-      else qproj_epilogue<D, 64>(p, sbase, tmem, bars, abort_flag, last_flag, head, ks, tile, m0);
+      if (nl == 0) qproj_epilogue<D, 0>(p, sbase, tmem, bars, abort_flag, last_flag, oh, is_v, ks, tile, m0);
+      else if (nl <= 16) qproj_epilogue<D, 16>(p, sbase, tmem, bars, abort_flag, last_flag, oh, is_v, ks, tile, m0);
+      else if (nl <= 32) qproj_epilogue<D, 32>(p, sbase, tmem, bars, abort_flag, last_flag, oh, is_v, ks, tile, m0);
+      else qproj_epilogue<D, 64>(p, sbase, tmem, bars, abort_flag, last_flag, oh, is_v, ks, tile, m0);
     }
   }
   // let the attention kernel launch once every CTA is here (triggering at the
