@@ -16,7 +16,9 @@ Every function is a plain restatement of the paper's definitions in float64:
     and position ids for the assembled context;
   * the suffix tokens' own keys and values: base k_proj / v_proj (the
     adaptation touches W^Q only, Sec. 3), key normalisation and RoPE at their
-    assembled positions.
+    assembled positions;
+  * prompt layouts whose online text (instructions, separators, the question)
+    interleaves with the cached artifact spans (App. prompt construction).
 
 Parity status: every function is pinned by the tests in
 ``tests/test_oracle_pins.py`` (closed forms, hand-derived fixtures under
@@ -37,5 +39,7 @@ from .attuner_oracle import (  # noqa: F401
     assemble,
     attention,
     request_forward,
+    layout_online_positions,
+    layout_forward,
     workload_reference,
 )

@@ -225,6 +225,58 @@ def request_forward(x, w_q, a, b, s, q_norm_w, eps, theta, art_k: List[np.ndarra
     return attention(q, k_all, v_all, n_visible, pairs)
 
 
+# ---------------------------------------------------------------------------
+# App. "Prompt Construction and Artifact Boundaries" (Tab. prompt layouts):
+# text outside the cached artifact spans -- instructions, separators, the
+# question -- is processed online, so online spans interleave with the cached
+# artifacts in prompt order.  Online tokens are laid out in assembled order in
+# one online buffer; item >= 0 is an artifact id, item < 0 an online span of
+# -item tokens, and online rows left after the items form the final span.
+# Every token sits at its index in the assembled sequence (App. A.5 position
+# ids); a query sees the assembled prefix up to its own position.
+# ---------------------------------------------------------------------------
+def layout_online_positions(items: Sequence[int], art_lengths: Sequence[int], S_kv: int) -> np.ndarray:
+    """Assembled position of each of the S_kv online rows."""
+    pos = []
+    at = 0
+    for it in items:
+        if it >= 0:
+            at += int(art_lengths[it])
+        else:
+            pos.extend(range(at, at - it))
+            at += -it
+    pos.extend(range(at, at + S_kv - len(pos)))
+    return np.asarray(pos, dtype=np.int64)
+
+
+def layout_forward(x, w_q, a, b, s, q_norm_w, eps, theta, items: Sequence[int], art_k: dict, art_v: dict,
+                   online_k, online_v, n_q_heads: int, pairs=None):
+    """x [S, d_model]: the last S online rows; art_k/art_v: artifact id ->
+    [L, Hkv, d]; online_k/online_v [S_kv, Hkv, d] in assembled order."""
+    S = x.shape[0]
+    S_kv = online_k.shape[0]
+    d = online_k.shape[2]
+    ks, vs = [], []
+    row = 0
+    for it in items:
+        if it >= 0:
+            ks.append(art_k[it])
+            vs.append(art_v[it])
+        else:
+            ks.append(online_k[row:row - it])
+            vs.append(online_v[row:row - it])
+            row += -it
+    ks.append(online_k[row:])
+    vs.append(online_v[row:])
+    lengths = {i: art_k[i].shape[0] for i in art_k}
+    pos_all = layout_online_positions(items, [lengths.get(i, 0) for i in range(max(lengths) + 1)] if lengths else [],
+                                      S_kv)
+    pos_q = pos_all[S_kv - S:]
+    q_raw = lora_q_projection(x, w_q, a, b, s).reshape(S, n_q_heads, d)
+    q = rope_rotate_half(rms_norm_heads(q_raw, q_norm_w, eps), pos_q, theta)
+    return attention(q, np.concatenate(ks, axis=0), np.concatenate(vs, axis=0), pos_q + 1, pairs)
+
+
 def workload_reference(wl, req: int, pairs=None, q_only: bool = False):
     """Run request_forward on request `req` of a seeded workload object."""
     g = wl.geom

@@ -180,6 +180,85 @@ def test_kv_projection_invariants():
     np.testing.assert_allclose(kw, k0 * w, rtol=1e-12)
 
 
+def test_layout_online_positions_hand_example():
+    # online 3, artifact of 5, online 2, artifact of 4, then the final online rows
+    pos = O.layout_online_positions([-3, 0, -2, 1], [5, 4], 12)
+    np.testing.assert_array_equal(pos, [0, 1, 2, 8, 9, 14, 15, 16, 17, 18, 19, 20])
+
+
+def _layout_case(seed=5, items=(-3, 1, -2, 0, -4, 2), S=9, S_kv=16):
+    rng = np.random.default_rng(seed)
+    hkv, G, d, hidden, r = 2, 2, 8, 12, 4
+    lens = {0: 7, 1: 5, 2: 9}
+    art_k = {i: rng.standard_normal((L, hkv, d)) for i, L in lens.items()}
+    art_v = {i: rng.standard_normal((L, hkv, d)) for i, L in lens.items()}
+    ok, ov = rng.standard_normal((S_kv, hkv, d)), rng.standard_normal((S_kv, hkv, d))
+    x = rng.standard_normal((S, hidden))
+    w_q = rng.standard_normal((hkv * G * d, hidden)) / math.sqrt(hidden)
+    a = rng.standard_normal((r, hidden)) / math.sqrt(hidden)
+    b = rng.standard_normal((hkv * G * d, r)) / math.sqrt(r)
+    qn = 1.0 + 0.1 * rng.standard_normal(d)
+    return dict(x=x, w_q=w_q, a=a, b=b, s=2.0, q_norm_w=qn, eps=1e-6, theta=1.0e4, items=list(items),
+                art_k=art_k, art_v=art_v, online_k=ok, online_v=ov, n_q_heads=hkv * G)
+
+
+def test_layout_without_online_items_is_the_classic_layout():
+    c = _layout_case(items=(1, 0, 2))
+    o1, l1 = O.layout_forward(**c)
+    o2, l2 = O.request_forward(c["x"], c["w_q"], c["a"], c["b"], c["s"], c["q_norm_w"], c["eps"], c["theta"],
+                               [c["art_k"][i] for i in (1, 0, 2)], [c["art_v"][i] for i in (1, 0, 2)],
+                               c["online_k"], c["online_v"], c["n_q_heads"])
+    np.testing.assert_allclose(o1, o2, rtol=1e-13, atol=1e-13)
+    np.testing.assert_allclose(l1, l2, rtol=1e-13, atol=1e-13)
+
+
+def test_layout_against_sdpa_over_the_assembled_sequence():
+    # the assembled sequence built token by token, queries rotated at their
+    # positions, and fp64 SDPA with an explicit boolean mask key <= query
+    c = _layout_case()
+    S, S_kv = c["x"].shape[0], c["online_k"].shape[0]
+    seq_k, seq_v, online_pos = [], [], []
+    row = 0
+    for it in c["items"]:
+        n = c["art_k"][it].shape[0] if it >= 0 else -it
+        for t in range(n):
+            if it >= 0:
+                seq_k.append(c["art_k"][it][t]); seq_v.append(c["art_v"][it][t])
+            else:
+                online_pos.append(len(seq_k)); seq_k.append(c["online_k"][row]); seq_v.append(c["online_v"][row])
+                row += 1
+    while row < S_kv:
+        online_pos.append(len(seq_k)); seq_k.append(c["online_k"][row]); seq_v.append(c["online_v"][row])
+        row += 1
+    K, V = np.stack(seq_k), np.stack(seq_v)
+    pos_q = np.asarray(online_pos[S_kv - S:])
+    d = K.shape[-1]
+    q_raw = O.lora_q_projection(c["x"], c["w_q"], c["a"], c["b"], c["s"]).reshape(S, c["n_q_heads"], d)
+    q = O.rope_rotate_half(O.rms_norm_heads(q_raw, c["q_norm_w"], c["eps"]), pos_q, c["theta"])
+    G = c["n_q_heads"] // K.shape[1]
+    mask = torch.as_tensor(np.arange(K.shape[0])[None, :] <= pos_q[:, None])
+    qt = torch.as_tensor(q).permute(1, 0, 2)
+    kt = torch.as_tensor(K).permute(1, 0, 2).repeat_interleave(G, dim=0)
+    vt = torch.as_tensor(V).permute(1, 0, 2).repeat_interleave(G, dim=0)
+    ref = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, attn_mask=mask).permute(1, 0, 2).numpy()
+    o, _ = O.layout_forward(**c)
+    np.testing.assert_allclose(o, ref, rtol=1e-10, atol=1e-12)
+
+
+def test_layout_queries_do_not_see_later_artifacts():
+    # queries in the first online span come before every artifact: replacing
+    # the artifacts' K/V must not change them; queries after an artifact must change
+    c = _layout_case(items=(-6, 1, -2, 0), S=16, S_kv=16)
+    o1, _ = O.layout_forward(**c)
+    rng = np.random.default_rng(99)
+    c2 = dict(c)
+    c2["art_k"] = {i: rng.standard_normal(t.shape) for i, t in c["art_k"].items()}
+    c2["art_v"] = {i: rng.standard_normal(t.shape) for i, t in c["art_v"].items()}
+    o2, _ = O.layout_forward(**c2)
+    np.testing.assert_array_equal(o1[:6], o2[:6])
+    assert np.abs(o1[6:] - o2[6:]).max() > 1e-3
+
+
 def test_query_positions():
     # tiny workload: 201 artifact tokens, S = S_kv = 16 -> positions 201..216
     np.testing.assert_array_equal(O.query_positions(201, 16, 16), np.arange(201, 217))
