@@ -109,6 +109,24 @@ attuner_status attuner_assemble(attuner_ctx* ctx, const int32_t* artifact_ids_ho
                                 const int32_t* req_offsets_host, int32_t n_req,
                                 attuner_plan** out);
 
+/* A plan for a prompt layout whose online text interleaves with the cached
+ * artifacts (App. "Prompt Construction and Artifact Boundaries": instructions,
+ * separators and the question are processed online, only artifact spans are
+ * cached).  items[] per request in prompt order: item >= 0 is an artifact id,
+ * item < 0 an online span of -item tokens.  The request's online tokens live
+ * in one online buffer in prompt order (x rows and suffix K/V rows): the spans'
+ * rows first, then the final span (online rows sum(spans) .. S_kv - 1, the
+ * suffix), so S_kv must be at least the spans' total.  The queries are the
+ * last S online rows (S = S_kv for a whole prefill layer); each sits at its
+ * index in the assembled sequence (App. A.5 position ids) and sees exactly the
+ * assembled tokens up to it, and suffix K/V rows must be rotated at those same
+ * positions (attuner_kv_project does so).  With no negative item this is
+ * attuner_assemble.  Errors: as attuner_assemble, plus INVALID_ARG for more
+ * than 2^22 online rows in the spans of one request. */
+attuner_status attuner_assemble_layout(attuner_ctx* ctx, const int32_t* items_host,
+                                       const int32_t* req_offsets_host, int32_t n_req,
+                                       attuner_plan** out);
+
 /* Copy a plan's layout to host arrays (for bit-exact tests).
  * sizes_inout[0..4] on input: capacities of block_table, valid_len,
  * index_map, token_art, token_off (elements); on output: the lengths used,

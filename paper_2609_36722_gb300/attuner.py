@@ -42,7 +42,7 @@ EXPORTS = [
     "attuner_attend", "attuner_query_attend", "attuner_pool_info", "attuner_sync_status",
     "attuner_set_option", "attuner_last_launch_count", "attuner_last_error",
     "attuner_attend_static_scratch", "attuner_register_artifacts_host", "attuner_pool_reset",
-    "attuner_kv_project",
+    "attuner_kv_project", "attuner_assemble_layout",
 ]
 
 
@@ -93,6 +93,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
                                              _p_i32], _i32),
         "attuner_pool_reset": ([_vp], _i32),
         "attuner_kv_project": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
+        "attuner_assemble_layout": ([_vp, _p_i32, _p_i32, _i32, ctypes.POINTER(_vp)], _i32),
     }
     for name, (args, ret) in sig.items():
         f = getattr(lib, name)
@@ -245,6 +246,21 @@ class Context:
         h = ctypes.c_void_p()
         _check(lib().attuner_assemble(self.handle, ids, off_arr, len(reqs), ctypes.byref(h)))
         return Plan(self, h, reqs)
+
+    def assemble_layout(self, layouts: Sequence[Sequence[int]]) -> Plan:
+        """Plans of prompt layouts: per request, items in prompt order, item >= 0
+        an artifact id, item < 0 an online span of -item tokens (the online
+        rows after the last item form the final span)."""
+        reqs = [list(map(int, r)) for r in layouts]
+        flat = [a for r in reqs for a in r]
+        offs = [0]
+        for r in reqs:
+            offs.append(offs[-1] + len(r))
+        items = (ctypes.c_int32 * max(len(flat), 1))(*flat)
+        off_arr = (ctypes.c_int32 * len(offs))(*offs)
+        h = ctypes.c_void_p()
+        _check(lib().attuner_assemble_layout(self.handle, items, off_arr, len(reqs), ctypes.byref(h)))
+        return Plan(self, h, [[a for a in r if a >= 0] for r in reqs])
 
     # --- compute
     def q_project(self, plan: Plan, x, w_q, lora_a, lora_b, s: float, q_norm_w, S_kv: Optional[int] = None,

@@ -32,7 +32,8 @@ struct MmaLayout {
   static_assert(MERGE_BYTES <= BAR_OFF, "merge area aliases the stage ring");
 };
 
-template <int D>
+// kLayout: some request has online spans before artifacts (general visibility rule)
+template <int D, bool kLayout>
 __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ AttnParams p) {
   using L = MmaLayout<D>;
   grid_dep_wait();     // Q and the suffix K/V may come from the previous kernel
@@ -60,10 +61,11 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
   const int nsplit = p.work.nsplit[req];
   const int boff = p.plan.blk_off[req];
   const int nab = p.plan.blk_off[req + 1] - boff;
-  const int nsuf = (p.S_kv + kBlockTokens - 1) / kBlockTokens;
+  const int o_rows = plan_o_rows(p.plan, req);           // online rows in the plan's spans
+  const int nsuf = (p.S_kv - o_rows + kBlockTokens - 1) / kBlockTokens;
   const int row0 = rt * kMmaRows;
   const int last_row = min(row0 + kMmaRows - 1, p.S * G - 1);
-  const int last_vis = nab + ((p.S_kv - p.S) + last_row / G) / kBlockTokens;
+  const int last_vis = row_visibility(p.plan, req, (p.S_kv - p.S) + last_row / G, nab).slot;
   const int b0 = split * p.work.chunk_blocks;
   const int b1 = min(min(b0 + p.work.chunk_blocks, nab + nsuf), last_vis + 1);
   const int nblk = max(0, b1 - b0);
@@ -73,13 +75,14 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
     int e;
     if (b < nab) {
       e = p.plan.blocks[boff + b];
-      const int blk = e >> 7, valid = e & 127;
-      if (blk < 0 || blk >= p.plan.pool_blocks || valid < 1 || valid > kBlockTokens) {
+      const bool bad = e > 0 ? ((e >> 7) >= p.plan.pool_blocks || (e & 127) < 1 || (e & 127) > kBlockTokens)
+                             : (slot_rows(e) < 1 || slot_rows(e) > kBlockTokens || slot_row0(e) + slot_rows(e) > o_rows);
+      if (bad) {
         set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
         e = 0;
       }
     } else {
-      e = -(b - nab + 1);
+      e = online_entry(o_rows + (b - nab) * kBlockTokens, kBlockTokens);
     }
     list[i] = e;
   }
@@ -111,7 +114,7 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
 #pragma unroll
         for (int h = 0; h < L::NH; ++h) {
           if (e < 0) {
-            const int c = (-e - 1) * kBlockTokens;
+            const int c = slot_row0(e);
             tma_load_4d(dst + h * L::BLK, &p.tm_ksuf, fb, h * 64, kvh, c, req);
             tma_load_4d(dst + (L::NH + h) * L::BLK, &p.tm_vsuf, fb, h * 64, kvh, c, req);
           } else {
@@ -155,8 +158,13 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
       }
     }
   }
+  // the thread's two query rows: online rows lim0 / lim1; with online spans
+  // before artifacts, also their own slots vs0 / vs1 (artifact slots after
+  // them are not visible)
   const int lim0 = (p.S_kv - p.S) + tok_r[0];
   const int lim1 = (p.S_kv - p.S) + tok_r[1];
+  const int vs0 = kLayout ? row_visibility(p.plan, req, (p.S_kv - p.S) + min(tok_r[0], p.S - 1), nab).slot - b0 : 0;
+  const int vs1 = kLayout ? row_visibility(p.plan, req, (p.S_kv - p.S) + min(tok_r[1], p.S - 1), nab).slot - b0 : 0;
 
   float o[NT][4];
 #pragma unroll
@@ -195,8 +203,8 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
       for (int c = 0; c < 4; ++c) {
         const int kb = 16 * warp + 8 * n + 2 * t + (c & 1);
         bool vis;
-        if (e > 0) vis = kb < (e & 127);
-        else if (e < 0) vis = ((-e - 1) * kBlockTokens + kb) <= ((c < 2) ? lim0 : lim1);
+        if (e > 0) vis = kb < (e & 127) && (!kLayout || j < ((c < 2) ? vs0 : vs1));
+        else if (e < 0) vis = (slot_row0(e) + kb) <= ((c < 2) ? lim0 : lim1) && (!kLayout || kb < slot_rows(e));
         else vis = false;
         if (!vis) s[n][c] = -INFINITY;
       }
@@ -321,17 +329,18 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
   }
 }
 
-template <int D>
+template <int D, bool kLayout>
 static cudaError_t launch_attn_mma_t(const AttnParams& p, cudaStream_t st) {
   using L = MmaLayout<D>;
-  cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
+  cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<D, kLayout>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
-  return launch_pdl(attn_mma_kernel<D>, dim3(p.work.n_cta), dim3(160), (size_t)L::SMEM, st, 0, p);
+  return launch_pdl(attn_mma_kernel<D, kLayout>, dim3(p.work.n_cta), dim3(160), (size_t)L::SMEM, st, 0, p);
 }
 
 cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st) {
-  if (D == 128) return launch_attn_mma_t<128>(p, st);
-  if (D == 64) return launch_attn_mma_t<64>(p, st);
+  const bool layout = p.plan.has_spans != 0;
+  if (D == 128) return layout ? launch_attn_mma_t<128, true>(p, st) : launch_attn_mma_t<128, false>(p, st);
+  if (D == 64) return layout ? launch_attn_mma_t<64, true>(p, st) : launch_attn_mma_t<64, false>(p, st);
   return cudaErrorInvalidValue;
 }
 

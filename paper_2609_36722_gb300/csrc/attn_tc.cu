@@ -87,8 +87,7 @@ __device__ __forceinline__ void load_slot(uint32_t dst, int e, const CUtensorMap
 #pragma unroll
   for (int h = 0; h < L::NH; ++h) {
     if (e < 0) {
-      const int chunk = -e - 1;
-      tma_load_4d(dst + h * L::HALF, suf, bar, h * 64, kvh, chunk * kBlockTokens, req);
+      tma_load_4d(dst + h * L::HALF, suf, bar, h * 64, kvh, slot_row0(e), req);
     } else if ((e & 127) != 0) {
       const int blk = e >> 7;
       tma_load_2d(dst + h * L::HALF, pool, bar, h * 64, (blk * Hkv + kvh) * kBlockTokens);
@@ -97,15 +96,6 @@ __device__ __forceinline__ void load_slot(uint32_t dst, int e, const CUtensorMap
       tma_load_2d(dst + h * L::HALF, pool, bar, h * 64, pool_rows);
     }
   }
-}
-
-// Visible keys of one 64-key block slot for a query row: every slot reduces
-// to "the first n keys are visible" -- an artifact block's valid length, the
-// causal prefix of a suffix chunk (keys <= lim), or 0 for an empty slot.
-__device__ __forceinline__ int slot_visible(int e, int lim) {
-  if (e > 0) return e & 127;
-  if (e < 0) return min(max(lim - (-e - 1) * kBlockTokens + 1, 0), kBlockTokens);
-  return 0;
 }
 
 // -inf for keys past n_vis in a 64-key slot
@@ -131,7 +121,8 @@ __device__ __forceinline__ TcCta tc_cta(const AttnParams& p, int cta) {
     const int rem = unit % per_req;
     c.rt = rem % p.work.row_tiles;
     c.kvh = rem / p.work.row_tiles;
-    const int nv = p.plan.blk_off[c.req + 1] - p.plan.blk_off[c.req] + (p.S_kv + kBlockTokens - 1) / kBlockTokens;
+    const int nv = p.plan.blk_off[c.req + 1] - p.plan.blk_off[c.req] +
+                   (p.S_kv - plan_o_rows(p.plan, c.req) + kBlockTokens - 1) / kBlockTokens;
     c.chunk = (((nv + ns - 1) / ns) + 1) & ~1;
   } else {
     c.req = find_req(p.work, cta);
@@ -398,7 +389,9 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
   }
 }
 
-template <int D>
+// kLayout: some request of the plan has online spans before artifacts (the
+// general visibility rule); false keeps the plain rule of the common layout.
+template <int D, bool kLayout>
 __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__ AttnParams p) {
   using L = TcLayout<D>;
   extern __shared__ uint8_t smem_raw[];
@@ -420,30 +413,32 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
   const int req = cw.req, rt = cw.rt, kvh = cw.kvh;
   const int boff = p.plan.blk_off[req];
   const int nab = p.plan.blk_off[req + 1] - boff;
-  const int nsuf = (p.S_kv + kBlockTokens - 1) / kBlockTokens;
+  const int o_rows = plan_o_rows(p.plan, req);           // online rows in the plan's spans
+  const int nsuf = (p.S_kv - o_rows + kBlockTokens - 1) / kBlockTokens;
   const int row0 = rt * kTcRows;
   const int last_row = min(row0 + kTcRows - 1, p.S * G - 1);
-  const int last_vis = nab + ((p.S_kv - p.S) + last_row / G) / kBlockTokens;
+  const int last_vis = row_visibility(p.plan, req, (p.S_kv - p.S) + last_row / G, nab).slot;
   const int b0 = cw.split * cw.chunk;
   const int b1 = min(min(b0 + cw.chunk, nab + nsuf), last_vis + 1);
   const int nblk = max(0, b1 - b0);
   const int ntile = (nblk + 1) / 2;
   const int pool_rows = p.plan.pool_blocks * p.Hkv * kBlockTokens;
 
-  // ---- block list of this chunk: >0 artifact (block << 7 | valid), <0 suffix chunk, 0 none
+  // ---- slots of this chunk: >0 artifact block, <0 online chunk, 0 none
   for (int i = threadIdx.x; i < 2 * ntile; i += blockDim.x) {
     int e = 0;
     if (i < nblk) {
       const int b = b0 + i;
       if (b < nab) {
         e = p.plan.blocks[boff + b];
-        const int blk = e >> 7, valid = e & 127;
-        if (blk < 0 || blk >= p.plan.pool_blocks || valid < 1 || valid > kBlockTokens) {
+        const bool bad = e > 0 ? ((e >> 7) >= p.plan.pool_blocks || (e & 127) < 1 || (e & 127) > kBlockTokens)
+                               : (slot_rows(e) < 1 || slot_rows(e) > kBlockTokens || slot_row0(e) + slot_rows(e) > o_rows);
+        if (bad) {
           set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
           e = 0;
         }
       } else {
-        e = -(b - nab + 1);
+        e = online_entry(o_rows + (b - nab) * kBlockTokens, kBlockTokens);
       }
     }
     list[i] = e;
@@ -597,7 +592,16 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
     const int r = qt * kTcTileRows + quad * 32 + lane;   // CTA row
     const int pr = row0 + r;                             // packed row
     const int tok = pr / G;
-    const int lim = (p.S_kv - p.S) + tok;                // last visible suffix key
+    // What this query (online row lim) sees: online keys up to its own online
+    // row (online rows are in assembled order) and, with online spans before
+    // artifacts, only the artifact slots before its own slot vs (chunk-relative).
+    const int lim = (p.S_kv - p.S) + tok;
+    const int vs = kLayout ? row_visibility(p.plan, req, lim, nab).slot - b0 : 0;
+    auto visible = [&](int s, int e) {
+      if (e > 0) return (kLayout && s >= vs) ? 0 : (e & 127);
+      if (e < 0) return min(max(lim - slot_row0(e) + 1, 0), kLayout ? slot_rows(e) : kBlockTokens);
+      return 0;
+    };
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const uint32_t s_col = tmem + lane_base + s_col_of(qt);
     const uint32_t o_col = tmem + lane_base + o_col_of(qt);
@@ -613,7 +617,7 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
       for (int c = 0; c < 4; ++c) tmem_ld32(s_col + c * 32, sc + c * 32);
       // while the TMEM loads are in flight: visible keys of the two slots, and
       // one warp vote (most tiles are fully visible and skip the masking code)
-      const int nv0 = slot_visible(list[2 * j], lim), nv1 = slot_visible(list[2 * j + 1], lim);
+      const int nv0 = visible(2 * j, list[2 * j]), nv1 = visible(2 * j + 1, list[2 * j + 1]);
       const bool need_mask = __any_sync(0xffffffffu, min(nv0, nv1) < kBlockTokens);
       tc_wait_ld();
       if (need_mask) {
@@ -689,25 +693,25 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
   }
 }
 
-template <int D>
+template <int D, bool kLayout>
 static cudaError_t launch_attn_tc_t(const AttnParams& p, cudaStream_t st) {
   using L = TcLayout<D>;
   // setmaxnreg.inc waits until the registers it asks for are free in the
   // block's launch budget: never launch a split that exceeds that budget.
   cudaFuncAttributes fa{};
-  cudaError_t e = cudaFuncGetAttributes(&fa, attn_tc_kernel<D>);
+  cudaError_t e = cudaFuncGetAttributes(&fa, attn_tc_kernel<D, kLayout>);
   if (e != cudaSuccess) return e;
   if (fa.numRegs * 384 < 128 * kCtrlRegs + 256 * kSoftRegs) return cudaErrorLaunchOutOfResources;
-  e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
+  e = cudaFuncSetAttribute(attn_tc_kernel<D, kLayout>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
-  return launch_pdl(attn_tc_kernel<D>, dim3(p.work.n_cta), dim3(384), (size_t)L::SMEM, st, p.work.cluster, p);
+  return launch_pdl(attn_tc_kernel<D, kLayout>, dim3(p.work.n_cta), dim3(384), (size_t)L::SMEM, st, p.work.cluster, p);
 }
 
 // clusters of `ns` CTAs of this kernel that fit on the device at once (0: none)
 template <int D>
 static int attn_tc_max_clusters_t(int ns) {
   using L = TcLayout<D>;
-  if (cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM) != cudaSuccess)
+  if (cudaFuncSetAttribute(attn_tc_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM) != cudaSuccess)
     return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(ns);
@@ -721,7 +725,7 @@ static int attn_tc_max_clusters_t(int ns) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<D>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<D, false>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
@@ -735,8 +739,9 @@ int attn_tc_max_clusters(int D, int ns) {
 }
 
 cudaError_t launch_attn_tc(const AttnParams& p, int D, cudaStream_t st) {
-  if (D == 128) return launch_attn_tc_t<128>(p, st);
-  if (D == 64) return launch_attn_tc_t<64>(p, st);
+  const bool layout = p.plan.has_spans != 0;
+  if (D == 128) return layout ? launch_attn_tc_t<128, true>(p, st) : launch_attn_tc_t<128, false>(p, st);
+  if (D == 64) return layout ? launch_attn_tc_t<64, true>(p, st) : launch_attn_tc_t<64, false>(p, st);
   return cudaErrorInvalidValue;
 }
 

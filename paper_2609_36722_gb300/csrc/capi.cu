@@ -256,8 +256,10 @@ extern "C" attuner_status attuner_pool_reset(attuner_ctx* ctx) {
 // ---------------------------------------------------------------------------
 // plans
 // ---------------------------------------------------------------------------
-extern "C" attuner_status attuner_assemble(attuner_ctx* ctx, const int32_t* ids, const int32_t* offs,
-                                           int32_t n_req, attuner_plan** out) {
+// Plans of both entry points: items >= 0 are artifact ids, items < 0 (layouts
+// only) online spans of -item rows, in prompt order.
+static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const int32_t* offs, int32_t n_req,
+                                    bool layout, attuner_plan** out) {
   CHECK_ARG(ctx != nullptr && out != nullptr, "ctx and out must not be NULL");
   *out = nullptr;
   CHECK_ARG(n_req >= 1 && n_req <= kMaxReq, "n_req must be in [1, " + std::to_string(kMaxReq) + "]");
@@ -270,43 +272,72 @@ extern "C" attuner_status attuner_assemble(attuner_ctx* ctx, const int32_t* ids,
   p->device = ctx->cfg.device;
   p->pool_blocks = ctx->cfg.pool_blocks;
   p->req_off.assign(offs, offs + n_req + 1);
-  p->art_ids.assign(ids, ids + offs[n_req]);
   p->blk_off.push_back(0);
+  p->span_off.push_back(0);
   for (int r = 0; r < n_req; ++r) {
-    long long t = 0;
+    long long t = 0, o = 0;
+    const int32_t first_slot = (int32_t)p->blocks.size();
     for (int i = offs[r]; i < offs[r + 1]; ++i) {
       const int a = ids[i];
+      if (a < 0 && layout) {
+        const long long n = -(long long)a;
+        p->spans.insert(p->spans.end(), {(int32_t)o, (int32_t)n, (int32_t)p->blocks.size() - first_slot, (int32_t)t});
+        for (long long c = 0; c < n; c += 64)
+          p->blocks.push_back(-((int32_t)(((o + c) << 7) | std::min<long long>(64, n - c)) + 1));
+        o += n;
+        if (o >= (1 << 22)) {
+          delete p;
+          return fail(ATTUNER_ERR_INVALID_ARG, "online rows of a request must be < 2^22");
+        }
+        continue;
+      }
       if (a < 0 || a >= (int)ctx->arts.size()) {
         delete p;
         return fail(ATTUNER_ERR_UNKNOWN_ARTIFACT, "artifact id " + std::to_string(a) + " was never registered");
       }
+      p->art_ids.push_back(a);
       const Artifact& A = ctx->arts[a];
       for (int b = 0; b < A.n_blocks; ++b)
         p->blocks.push_back(((A.first_block + b) << 7) | std::min(64, A.L - 64 * b));
       t += A.L;
     }
-    if (t >= (1ll << 30)) {
+    if (t + o >= (1ll << 30)) {
       delete p;
       return fail(ATTUNER_ERR_INVALID_ARG, "assembled length of a request must be < 2^30 tokens");
     }
     p->blk_off.push_back((int32_t)p->blocks.size());
     p->t_art.push_back((int32_t)t);
+    p->o_rows.push_back((int32_t)o);
+    p->span_off.push_back((int32_t)(p->spans.size() / 4));
+    p->max_o_rows = std::max(p->max_o_rows, (int32_t)o);
+  }
+  p->req_art_off.push_back(0);
+  {
+    int k = 0;
+    for (int r = 0; r < n_req; ++r) {
+      for (int i = offs[r]; i < offs[r + 1]; ++i) k += ids[i] >= 0;
+      p->req_art_off.push_back(k);
+    }
   }
   p->arts = ctx->arts;
   attuner_status s = set_device(ctx);
   if (s != ATTUNER_OK) { delete p; return s; }
-  const size_t n = p->blk_off.size() + p->blocks.size() + p->t_art.size();
   std::vector<int32_t> h;
-  h.reserve(n);
   h.insert(h.end(), p->blk_off.begin(), p->blk_off.end());
   h.insert(h.end(), p->blocks.begin(), p->blocks.end());
   h.insert(h.end(), p->t_art.begin(), p->t_art.end());
-  if (cudaMalloc(&p->d_buf, n * sizeof(int32_t)) != cudaSuccess) {
+  h.insert(h.end(), p->o_rows.begin(), p->o_rows.end());
+  h.insert(h.end(), p->span_off.begin(), p->span_off.end());
+  while (h.size() % 4) h.push_back(0);   // int4 spans start 16-byte aligned
+  p->spans_at = h.size();
+  h.insert(h.end(), p->spans.begin(), p->spans.end());
+  if (h.empty()) h.push_back(0);
+  if (cudaMalloc(&p->d_buf, h.size() * sizeof(int32_t)) != cudaSuccess) {
     cudaGetLastError();
     delete p;
     return fail(ATTUNER_ERR_OOM, "plan allocation failed");
   }
-  if (cudaMemcpy(p->d_buf, h.data(), n * sizeof(int32_t), cudaMemcpyHostToDevice) != cudaSuccess) {
+  if (cudaMemcpy(p->d_buf, h.data(), h.size() * sizeof(int32_t), cudaMemcpyHostToDevice) != cudaSuccess) {
     cudaFree(p->d_buf);
     delete p;
     return fail(ATTUNER_ERR_CUDA, "plan upload failed");
@@ -315,11 +346,22 @@ extern "C" attuner_status attuner_assemble(attuner_ctx* ctx, const int32_t* ids,
   return ATTUNER_OK;
 }
 
+extern "C" attuner_status attuner_assemble(attuner_ctx* ctx, const int32_t* ids, const int32_t* offs,
+                                           int32_t n_req, attuner_plan** out) {
+  return assemble_impl(ctx, ids, offs, n_req, false, out);
+}
+
+extern "C" attuner_status attuner_assemble_layout(attuner_ctx* ctx, const int32_t* items, const int32_t* offs,
+                                                  int32_t n_req, attuner_plan** out) {
+  return assemble_impl(ctx, items, offs, n_req, true, out);
+}
+
 extern "C" attuner_status attuner_plan_export(const attuner_plan* p, int32_t* block_table, int32_t* valid_len,
                                               int32_t* index_map, int32_t* token_art, int32_t* token_off,
                                               int64_t* sizes) {
   CHECK_ARG(p != nullptr && sizes != nullptr, "plan and sizes_inout must not be NULL");
-  const int64_t nb = (int64_t)p->blocks.size();
+  int64_t nb = 0;
+  for (int32_t e : p->blocks) nb += e > 0;   // artifact blocks (online chunks are not exported)
   int64_t nt = 0;
   for (int32_t t : p->t_art) nt += t;
   CHECK_ARG(!block_table || sizes[0] >= nb, "block_table capacity too small");
@@ -327,13 +369,18 @@ extern "C" attuner_status attuner_plan_export(const attuner_plan* p, int32_t* bl
   CHECK_ARG(!index_map || sizes[2] >= nt, "index_map capacity too small");
   CHECK_ARG(!token_art || sizes[3] >= nt, "token_art capacity too small");
   CHECK_ARG(!token_off || sizes[4] >= nt, "token_off capacity too small");
-  for (int64_t i = 0; i < nb; ++i) {
-    if (block_table) block_table[i] = p->blocks[i] >> 7;
-    if (valid_len) valid_len[i] = p->blocks[i] & 127;
+  {
+    int64_t i = 0;
+    for (int32_t e : p->blocks) {
+      if (e <= 0) continue;
+      if (block_table) block_table[i] = e >> 7;
+      if (valid_len) valid_len[i] = e & 127;
+      ++i;
+    }
   }
   int64_t t = 0;
   for (int r = 0; r < p->n_req; ++r) {
-    for (int i = p->req_off[r]; i < p->req_off[r + 1]; ++i) {
+    for (int i = p->req_art_off[r]; i < p->req_art_off[r + 1]; ++i) {
       const int a = p->art_ids[i];
       const Artifact& A = p->arts[a];
       for (int q = 0; q < A.L; ++q, ++t) {
@@ -377,7 +424,11 @@ PlanDev att::plan_dev(const attuner_plan* p) {
   d.blk_off = p->d_buf;
   d.blocks = p->d_buf + p->blk_off.size();
   d.t_art = p->d_buf + p->blk_off.size() + p->blocks.size();
+  d.o_rows = d.t_art + p->t_art.size();
+  d.span_off = d.o_rows + p->o_rows.size();
+  d.spans = reinterpret_cast<const int4*>(p->d_buf + p->spans_at);
   d.pool_blocks = p->pool_blocks;
+  d.has_spans = p->max_o_rows > 0 ? 1 : 0;
   return d;
 }
 
@@ -389,8 +440,9 @@ attuner_status att::check_common(attuner_ctx* ctx, const attuner_plan* plan, int
   CHECK_ARG(plan->device == ctx->cfg.device && plan->pool_blocks == ctx->cfg.pool_blocks,
             "plan belongs to another context");
   CHECK_ARG(S >= 1 && S_kv >= S, "need 1 <= S <= S_kv");
-  CHECK_ARG((long long)plan->n_req * S * ctx->cfg.n_q_heads < (1ll << 31) && S_kv < (1 << 30),
-            "n_req * S * n_q_heads must be < 2^31");
+  CHECK_ARG((long long)plan->n_req * S * ctx->cfg.n_q_heads < (1ll << 31) && S_kv < (1 << 22),
+            "n_req * S * n_q_heads must be < 2^31 and S_kv < 2^22");
+  CHECK_ARG(S_kv >= plan->max_o_rows, "S_kv must cover the online rows of the plan's spans");
   return ATTUNER_OK;
 }
 
@@ -433,7 +485,7 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
 
   PrepParams pp{};
   pp.rope = rope;
-  pp.t_art = plan_dev(plan).t_art;
+  pp.plan = plan_dev(plan);
   pp.counters = ksplit > 1 ? reinterpret_cast<int32_t*>(base + off_cnt) : nullptr;
   pp.n_counters = ksplit > 1 ? tiles : 0;
   pp.M = M;
@@ -513,7 +565,7 @@ static attuner_status kv_project_impl(attuner_ctx* ctx, const attuner_plan* plan
 
   PrepParams pp{};
   pp.rope = rope;
-  pp.t_art = plan_dev(plan).t_art;
+  pp.plan = plan_dev(plan);
   pp.M = M;
   pp.D = D;
   pp.S = S;
@@ -583,11 +635,14 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
   const int G = ctx->cfg.n_q_heads / ctx->cfg.n_kv_heads, Hkv = ctx->cfg.n_kv_heads;
   const int rows = tc ? kTcRows : kMmaRows;
   const int row_tiles = (S * G + rows - 1) / rows;
-  const int nsuf = (S_kv + 63) / 64;
+  // slots of request r: the plan's, then the chunks of its final online span
+  auto nslots = [&](int r) {
+    return plan->blk_off[r + 1] - plan->blk_off[r] + (S_kv - plan->o_rows[r] + 63) / 64;
+  };
   long long total = 0;
   int maxv = 0;
   for (int r = 0; r < plan->n_req; ++r) {
-    const int nv = plan->blk_off[r + 1] - plan->blk_off[r] + nsuf;
+    const int nv = nslots(r);
     total += (long long)nv * Hkv * row_tiles;
     maxv = std::max(maxv, nv);
   }
@@ -624,7 +679,7 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
         const int ct = (maxt + sp - 1) / sp;
         long long ncta = 0;
         for (int r = 0; r < plan->n_req; ++r) {
-          const int nv = plan->blk_off[r + 1] - plan->blk_off[r] + nsuf;
+          const int nv = nslots(r);
           ncta += (long long)((nv + 2 * ct - 1) / (2 * ct)) * Hkv * row_tiles;
         }
         const long long waves = (ncta + ctx->num_sms - 1) / ctx->num_sms;
@@ -672,7 +727,7 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
   w.chunk_blocks = chunk;
   int base = 0;
   for (int r = 0; r < plan->n_req; ++r) {
-    const int nv = plan->blk_off[r + 1] - plan->blk_off[r] + nsuf;
+    const int nv = nslots(r);
     const int ns = (nv + chunk - 1) / chunk;
     w.base[r] = base;
     w.nsplit[r] = ns;

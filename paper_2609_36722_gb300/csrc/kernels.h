@@ -15,7 +15,7 @@ namespace att {
 // counters of K1b for this call.
 struct PrepParams {
   float2* rope;                  // [D/2, M] (cos, sin), pair-major
-  const int32_t* t_art;          // [n_req]
+  PlanDev plan;                  // assembled positions of the online rows
   int32_t* counters;             // [n_counters] split-K arrival counters, or nullptr
   int32_t n_counters;
   int32_t M, D, S, S_kv;

@@ -124,7 +124,7 @@ __global__ void __launch_bounds__(256) prep_kernel(const __grid_constant__ PrepP
   if (idx >= (long long)p.M * half) return;
   const int j = (int)(idx / p.M), m = (int)(idx % p.M);   // pair-major: coalesced in the epilogue
   const int req = m / p.S, i = m % p.S;
-  const long long pos = (long long)p.t_art[req] + (p.S_kv - p.S) + i;
+  const long long pos = online_position(p.plan, req, (p.S_kv - p.S) + i);   // assembled position
   const double ang = (double)pos * p.inv_freq[j];
   const double k = rint(ang * 0.15915494309189533577);   // 1 / (2 pi)
   const double red = fma(-k, 6.283185307179586232, ang);
