@@ -271,6 +271,38 @@ def run_ours(args, rank, world, local_rank):
         if i >= 3:
             kv_ms.append(ev_q.elapsed_time(ev_a))
     kv_flops = 2.0 * wl.n_req * wl.S * g.hidden * 2 * g.n_kv_heads * g.head_dim
+    # the paper's skills layout (§8(f) row 3): a 16-token online system span,
+    # 5-token online separators between the artifacts, the rest of the online
+    # rows (the task) last; every online row is a query (S = S_kv)
+    lay_ms, lay_flops = [], 0.0
+    if wl.S == wl.S_kv:
+        layouts = []
+        for r in wl.requests:
+            lay = [-16]
+            for k, a in enumerate(r):
+                lay += ([a] if k == 0 else [-5, a])
+            layouts.append(lay)
+        if all(16 + 5 * (len(r) - 1) <= wl.S_kv for r in wl.requests):
+            lplan = ctx.assemble_layout(layouts)
+            for r, lay in enumerate(layouts):
+                at, online_pos = 0, []
+                for it in lay:
+                    if it >= 0:
+                        at += wl.art_lengths[it]
+                    else:
+                        online_pos += list(range(at, at - it))
+                        at += -it
+                online_pos += list(range(at, at + wl.S_kv - len(online_pos)))
+                lay_flops += 4.0 * g.head_dim * g.n_q_heads * sum(p_ + 1 for p_ in online_pos[wl.S_kv - wl.S:])
+            for i in range(args.steps + 3):
+                flush.zero_()
+                ev_q.record(stream)
+                ctx.attend(lplan, q, wl.suffix_k, wl.suffix_v, out=out, lse=lse)
+                ev_a.record(stream)
+                ev_a.synchronize()
+                if i >= 3:
+                    lay_ms.append(ev_q.elapsed_time(ev_a))
+            lplan.free()
     total_ms = sum(step_ms)
     if world > 1:
         t = torch.tensor([total_ms], device=dev)
@@ -403,6 +435,10 @@ def run_ours(args, rank, world, local_rank):
         "path_work": {"attention_flops": attention_flops(wl), "qproj_flops": qproj_flops(wl),
                       "kv_bytes": kv_bytes(wl)},
         # the Q projection (steps a1-a3: prep + qproj kernels) as its own line, from the same pass
+        "layout_attention": ({"avg_call_ms": round(statistics.mean(lay_ms), 5),
+                              "tflops": round(lay_flops / (statistics.mean(lay_ms) * 1e-3) / 1e12, 3),
+                              "layout": "online system span 16, artifacts with 5-token online separators, task last"}
+                             if lay_ms else None),
         "kv_project": {"avg_call_ms": round(statistics.mean(kv_ms), 5),
                        "tflops": round(kv_flops / (statistics.mean(kv_ms) * 1e-3) / 1e12, 3)},
         "qproj": {"avg_call_ms": round(statistics.mean(qproj_ms), 5),
