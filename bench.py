@@ -208,51 +208,71 @@ def run_ours(args, rank, world, local_rank):
         # from starting while the projection finishes (programmatic dependent
         # launch needs kernel after kernel), so the step timing runs without.
         if attn_events:
-            ev_q.record(stream)
+            ev_q.record()
         ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv, out=q)
         n1 = ctx.last_launch_count()
         if attn_events:
-            ev_a.record(stream)
+            ev_a.record()
         ctx.attend(plan, q, wl.suffix_k, wl.suffix_v, out=out, lse=lse)
         if attn_events:
-            ev_b.record(stream)
+            ev_b.record()
         return n1 + ctx.last_launch_count()
 
-    ev_q = torch.cuda.Event(enable_timing=True)
-    ev_a = torch.cuda.Event(enable_timing=True)
-    ev_b = torch.cuda.Event(enable_timing=True)
+    def graphed(fn):
+        # The timed work replays a CUDA graph of the calls: one launch for the
+        # host, so the GPU never waits on the Python binding or the per-call
+        # host setup between kernels.  Events inside the graph time it on the
+        # device.
+        e0, e1 = gevent(), gevent()
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr):
+            e0.record()
+            fn()
+            e1.record()
+        torch.cuda.synchronize()
+        return gr, e0, e1
+
+    def gevent():
+        # an event that a captured graph records as a node of its own
+        return torch.cuda.Event(enable_timing=True, external=True)
+
+    ev_q, ev_a, ev_b = gevent(), gevent(), gevent()
     for _ in range(args.warmup):
-        step()
+        launches_per_step = step()
     torch.cuda.synchronize()
+    assert ctx.sync_status() == 0
+    g_step, ev_s, ev_e = graphed(step)
+    g_parts, _, _ = graphed(lambda: step(attn_events=True))
     assert ctx.sync_status() == 0
 
     sampler = ClockSampler(local_rank) if rank == 0 else None
     # keep the GPU busy ~1 s before timing so the clock samples describe the timed region
     t_end = time.perf_counter() + 1.0
     while time.perf_counter() < t_end:
-        step()
+        g_step.replay()
         torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     attn_ms = []
     qproj_ms = []
+    step_ms = []
     launches = 0
     for i in range(args.steps):
         flush.zero_()                                   # L2 flush between steps, outside the timed events
-        starts[i].record(stream)
-        launches += step()
-        ends[i].record(stream)
-        ends[i].synchronize()
+        g_step.replay()
+        ev_e.synchronize()
+        step_ms.append(ev_s.elapsed_time(ev_e))
+        launches += launches_per_step
     torch.cuda.synchronize()
-    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     # the same steps again with events around the attention call: its launch
     # duration for the roofline
     for i in range(args.steps):
         flush.zero_()
-        step(attn_events=True)
+        g_parts.replay()
         ev_b.synchronize()
         attn_ms.append(ev_a.elapsed_time(ev_b))
         qproj_ms.append(ev_q.elapsed_time(ev_a))
@@ -262,14 +282,12 @@ def run_ours(args, rank, world, local_rank):
     wk, wv, kn = make_kv_weights(g, 0, device=dev)
     sk_s, sv_s = wl.suffix_k.clone(), wl.suffix_v.clone()
     kv_ms = []
-    for i in range(args.steps + 3):
+    g_kv, e0, e1 = graphed(lambda: ctx.kv_project(plan, wl.x, wk, wv, kn, sk_s, sv_s))
+    for i in range(args.steps):
         flush.zero_()
-        ev_q.record(stream)
-        ctx.kv_project(plan, wl.x, wk, wv, kn, sk_s, sv_s)
-        ev_a.record(stream)
-        ev_a.synchronize()
-        if i >= 3:
-            kv_ms.append(ev_q.elapsed_time(ev_a))
+        g_kv.replay()
+        e1.synchronize()
+        kv_ms.append(e0.elapsed_time(e1))
     kv_flops = 2.0 * wl.n_req * wl.S * g.hidden * 2 * g.n_kv_heads * g.head_dim
     # the paper's skills layout (§8(f) row 3): a 16-token online system span,
     # 5-token online separators between the artifacts, the rest of the online
@@ -294,14 +312,13 @@ def run_ours(args, rank, world, local_rank):
                         at += -it
                 online_pos += list(range(at, at + wl.S_kv - len(online_pos)))
                 lay_flops += 4.0 * g.head_dim * g.n_q_heads * sum(p_ + 1 for p_ in online_pos[wl.S_kv - wl.S:])
-            for i in range(args.steps + 3):
+            g_lay, e0, e1 = graphed(lambda: ctx.attend(lplan, q, wl.suffix_k, wl.suffix_v, out=out, lse=lse))
+            for i in range(args.steps):
                 flush.zero_()
-                ev_q.record(stream)
-                ctx.attend(lplan, q, wl.suffix_k, wl.suffix_v, out=out, lse=lse)
-                ev_a.record(stream)
-                ev_a.synchronize()
-                if i >= 3:
-                    lay_ms.append(ev_q.elapsed_time(ev_a))
+                g_lay.replay()
+                e1.synchronize()
+                lay_ms.append(e0.elapsed_time(e1))
+            del g_lay
             lplan.free()
     total_ms = sum(step_ms)
     if world > 1:
