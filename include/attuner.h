@@ -281,7 +281,7 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
  *                               chunks of a row tile: 0 auto (cost model),
  *                               1 independent CTAs merged through global memory
  *                               by the last one to finish, 2 one thread-block
- *                               cluster per row tile (2..8 chunks) merged
+ *                               cluster per row tile (2 or 4 chunks) merged
  *                               through distributed shared memory
  *   ATTUNER_OPT_TEST_STUCK_WAIT see below */
 #define ATTUNER_OPT_PREFILL_KERNEL 1

@@ -46,7 +46,8 @@ struct TcLayout {
   static constexpr int V_OFF = K_OFF + NS * NH * HALF;
   static constexpr int BAR_OFF = V_OFF + NS * NH * HALF;
   static constexpr int LIST_OFF = BAR_OFF + 1024;
-  static constexpr int SMEM_MIN = LIST_OFF + kMaxChunkBlocks * 4 + 1024;
+  static constexpr int XLSE_OFF = LIST_OFF + kMaxChunkBlocks * 4;   // cluster merge: LSE out + 3 in
+  static constexpr int SMEM_MIN = XLSE_OFF + 4 * kTcRows * 4 + 1024;
   // at least 116 KiB so that two CTAs never share an SM (each holds all of TMEM)
   static constexpr int SMEM = SMEM_MIN > 118784 ? SMEM_MIN : 118784;
   static constexpr uint32_t TMEM_COLS = 512;        // S0/P0 | S1/P1 | O0 | O1
@@ -145,6 +146,130 @@ __device__ __forceinline__ int cta_index_fresh() {
   return v;
 }
 
+// bf16 store of N columns of one output row, from column c0 on, scaled
+template <int D, int N>
+__device__ __forceinline__ void store_cols(__nv_bfloat16* out, long long orow, int c0, const float* o, float scale) {
+  uint4* dst = reinterpret_cast<uint4*>(out + orow * D + c0);
+#pragma unroll
+  for (int k = 0; k < N / 8; ++k)
+    dst[k] = make_uint4(pack_bf16(o[8 * k] * scale, o[8 * k + 1] * scale),
+                        pack_bf16(o[8 * k + 2] * scale, o[8 * k + 3] * scale),
+                        pack_bf16(o[8 * k + 4] * scale, o[8 * k + 5] * scale),
+                        pack_bf16(o[8 * k + 6] * scale, o[8 * k + 7] * scale));
+}
+
+// Cluster-mode merge of the NS split-KV chunks of a row tile (one CTA per
+// chunk, cluster rank = split).  CTA `split` produces columns
+// [split, split + 1) x D/NS of all 256 rows.  Each CTA stages the other CTAs'
+// columns of its normalised O, [D/NS][256] fp32 per peer, and its LSE, and
+// pushes them into the peers' shared memory with bulk copies (the copy engine
+// moves distributed shared memory about twice as fast as loads from a peer
+// do); its own columns stay in tensor memory.  The chunks are summed in split
+// order with the same arithmetic for the own chunk as for the others, so no
+// partial result goes to global memory and the sum does not depend on timing.
+template <int D, int NS>
+__device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* smem, const TcCta& ce,
+                                                 uint32_t o_col, bool ok, int ntile, float inv_l, float lse,
+                                                 long long orow, bool row_ok) {
+  using L = TcLayout<D>;
+  constexpr int CW = D / NS;                            // output columns per CTA
+  constexpr uint32_t kSlot = kTcRows * CW * 4;          // one chunk's columns of all rows
+  static_assert(CW % 16 == 0 && 2 * (NS - 1) * kSlot <= (uint32_t)L::BAR_OFF, "staging and receive slots");
+  static_assert(NS <= 4, "LSE slots");
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 520);
+  const uint32_t mbar = smem_u32(&bars[B_MF]);
+  const int split = ce.split, erow = threadIdx.x;
+  float* src = reinterpret_cast<float*>(smem);           // NS-1 outgoing slots, peer order
+  float* rcv = src + (NS - 1) * (kSlot / 4);            // NS-1 incoming slots, split order
+  float* src_lse = reinterpret_cast<float*>(smem + L::XLSE_OFF);
+  float* rcv_lse = src_lse + kTcRows;
+  // columns [c0, c0 + CW) of this thread's row, normalised (zeros for an empty chunk)
+  auto own_cols = [&](int c0, float* v) {
+    if (ok && ntile > 0) {
+      if constexpr (CW >= 32) {
+#pragma unroll
+        for (int c = 0; c < CW; c += 32) tmem_ld32(o_col + c0 + c, v + c);
+        tc_wait_ld();
+      } else {
+        float t[32];
+        tmem_ld32(o_col + (c0 & ~31), t);
+        tc_wait_ld();
+        const bool hi = (c0 & 31) != 0;
+#pragma unroll
+        for (int k = 0; k < CW; ++k) v[k] = hi ? t[16 + k] : t[k];
+      }
+#pragma unroll
+      for (int k = 0; k < CW; ++k) v[k] *= inv_l;
+    } else {
+#pragma unroll
+      for (int k = 0; k < CW; ++k) v[k] = 0.f;
+    }
+  };
+  if (threadIdx.x == 0) mbar_expect_tx(mbar, (NS - 1) * (kSlot + kTcRows * 4));
+#pragma unroll
+  for (int t = 0; t < NS; ++t) {
+    if (t == split) continue;
+    float v[CW];
+    own_cols(t * CW, v);
+    float* dst = src + (t < split ? t : t - 1) * (kSlot / 4) + erow;
+#pragma unroll
+    for (int k = 0; k < CW; ++k) dst[k * kTcRows] = v[k];
+  }
+  src_lse[erow] = lse;
+  fence_proxy_async_smem();
+  cluster_sync_all();   // 1: every CTA of the cluster has staged; all main loops are over
+  if (threadIdx.x == 0) {
+#pragma unroll
+    for (int t = 0; t < NS; ++t) {
+      if (t == split) continue;
+      const uint32_t at = (split < t ? split : split - 1);   // this CTA's slot at peer t
+      const uint32_t cbar = dsmem_addr(mbar, t);
+      bulk_push_dsmem(dsmem_addr(smem_u32(rcv) + at * kSlot, t), smem_u32(src) + (t < split ? t : t - 1) * kSlot,
+                      kSlot, cbar);
+      bulk_push_dsmem(dsmem_addr(smem_u32(rcv_lse) + at * kTcRows * 4, t), smem_u32(src_lse), kTcRows * 4, cbar);
+    }
+  }
+  // Every CTA waits for its incoming copies, also after an abort: the peers
+  // issue them unconditionally, and none may land after this CTA has exited.
+  const bool got = __all_sync(0xffffffffu, mbar_drain(mbar, 0, p.status));
+  if (got && !*abort_flag) {
+    float w[NS];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < NS; ++k) {
+      w[k] = (k == split) ? lse : rcv_lse[(k < split ? k : k - 1) * kTcRows + erow];
+      mx = fmaxf(mx, w[k]);
+    }
+    float wsum = 0.f;
+#pragma unroll
+    for (int k = 0; k < NS; ++k) {
+      w[k] = (w[k] == -INFINITY) ? 0.f : __expf(w[k] - mx);
+      wsum += w[k];
+    }
+    float own[CW], acc[CW];
+    own_cols(split * CW, own);
+#pragma unroll
+    for (int c = 0; c < CW; ++c) acc[c] = 0.f;
+#pragma unroll
+    for (int k = 0; k < NS; ++k) {
+      if (k == split) {
+#pragma unroll
+        for (int c = 0; c < CW; ++c) acc[c] = __fmaf_rn(w[k], own[c], acc[c]);
+      } else {
+        const float* r = rcv + (k < split ? k : k - 1) * (kSlot / 4) + erow;
+#pragma unroll
+        for (int c = 0; c < CW; ++c) acc[c] = __fmaf_rn(w[k], r[c * kTcRows], acc[c]);
+      }
+    }
+    if (row_ok) {
+      store_cols<D, CW>(p.out, orow, split * CW, acc, wsum > 0.f ? 1.f / wsum : 0.f);
+      if (split == 0 && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
+    }
+  }
+  cluster_sync_all();   // 2: every copy has landed; no CTA leaves while a peer may still read its slots
+}
+
 // Epilogue of the softmax warps (warps 0..7, one CTA row per thread): O from
 // tensor memory, normalised, written as bf16 -- directly, or after merging the
 // split-KV chunks of the row tile.  A separate (not inlined) function, so that
@@ -174,16 +299,6 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
   auto out_row = [&](int pr) {
     return ((long long)ce.req * p.S + pr / G) * p.Hq + ce.kvh * G + pr % G;
   };
-  // 32 columns of one output row, bf16
-  auto store_row32 = [&](long long orow, int c, const float* o, float scale) {
-    uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D) + c * 4;
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-      dst[k] = make_uint4(pack_bf16(o[8 * k] * scale, o[8 * k + 1] * scale),
-                          pack_bf16(o[8 * k + 2] * scale, o[8 * k + 3] * scale),
-                          pack_bf16(o[8 * k + 4] * scale, o[8 * k + 5] * scale),
-                          pack_bf16(o[8 * k + 6] * scale, o[8 * k + 7] * scale));
-  };
   // Split-KV partial results are staged in the Q/K/V area, free once the last
   // MMA has completed.  Global mode stages them column-major ([d][256 rows]
   // fp32): 32 columns are one contiguous 32 KiB piece for one bulk copy, and a
@@ -208,53 +323,10 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
     }
   };
   if (p.work.cluster > 0) {
-    // Cluster mode: the nsplit CTAs of this row tile form one cluster.  Each
-    // stages its normalised O and LSE, then merges a slice of the 256 rows
-    // (whole 32-row groups) from all of them through distributed shared
-    // memory, in split order, so no partial result goes to global memory.
-    float* slse = stage + D * kTcRows;
-    stage_own();
-    slse[erow] = lse;
-    cluster_sync_all();   // 1: every CTA of the cluster has staged
-    const int g_lo = (split * 8) / nsplit, g_hi = ((split + 1) * 8) / nsplit;
-    const int nrows = (g_hi - g_lo) * 32;
-    const uint32_t own_base = smem_u32(stage);
-    if (!*abort_flag) {
-      for (int item = erow; item < nrows * (D / 32); item += 256) {
-        const int lr = g_lo * 32 + item % nrows, cb = item / nrows;
-        float w[8];
-        float mx = -INFINITY;
-#pragma unroll
-        for (int sp = 0; sp < 8; ++sp) {
-          w[sp] = sp < nsplit ? ld_dsmem(dsmem_addr(own_base + (D * kTcRows + lr) * 4, sp)) : -INFINITY;
-          mx = fmaxf(mx, w[sp]);
-        }
-        float wsum = 0.f;
-#pragma unroll
-        for (int sp = 0; sp < 8; ++sp) {
-          w[sp] = (w[sp] == -INFINITY) ? 0.f : __expf(w[sp] - mx);
-          wsum += w[sp];
-        }
-        float acc[32];
-#pragma unroll
-        for (int k = 0; k < 32; ++k) acc[k] = 0.f;
-#pragma unroll
-        for (int sp = 0; sp < 8; ++sp) {
-          if (sp < nsplit) {
-            const uint32_t src = dsmem_addr(own_base + ((cb * 32) * kTcRows + lr) * 4, sp);
-#pragma unroll
-            for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w[sp], ld_dsmem(src + k * kTcRows * 4), acc[k]);
-          }
-        }
-        const int pr = ce.rt * kTcRows + lr;
-        if (pr / G < p.S) {
-          const long long orow = out_row(pr);
-          store_row32(orow, cb, acc, wsum > 0.f ? 1.f / wsum : 0.f);
-          if (cb == 0 && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
-        }
-      }
-    }
-    cluster_sync_all();   // 2: no CTA leaves while a peer may still read its shared memory
+    if (nsplit == 4)
+      tc_cluster_merge<D, 4>(p, smem, ce, o_col, ok, ntile, inv_l, lse, out_row(epr), row_ok);
+    else
+      tc_cluster_merge<D, 2>(p, smem, ce, o_col, ok, ntile, inv_l, lse, out_row(epr), row_ok);
   } else if (nsplit > 1) {
     // Independent splits: publish this chunk's normalised O and its
     // log-sum-exp through global memory; the last CTA of the (request, KV
@@ -262,7 +334,7 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
     const int cta = cta_index_fresh();
     const int r = erow;
     const long long orow = out_row(epr);
-    auto store_row32o = [&](int c, const float* o, float scale) { store_row32(orow, c, o, scale); };
+    auto store_row32o = [&](int c, const float* o, float scale) { store_cols<D, 32>(p.out, orow, c * 32, o, scale); };
     const int req = ce.req, kvh = ce.kvh, rt = ce.rt;
     constexpr int kBufs = L::BAR_OFF / kPiece;       // 6 (d = 128) or 3 (d = 64)
     constexpr int kRing = kBufs - 1;                 // the last one holds the merge weights
@@ -383,7 +455,7 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
       float o[32];
       tmem_ld32(o_col + c * 32, o);
       tc_wait_ld();
-      if (row_ok) store_row32(orow, c, o, inv_l);
+      if (row_ok) store_cols<D, 32>(p.out, orow, c * 32, o, inv_l);
     }
     if (row_ok && p.lse_out) p.lse_out[orow] = lse;
   }

@@ -627,7 +627,8 @@ static size_t q_project_scratch(const attuner_ctx* ctx, int M) {
 // ---------------------------------------------------------------------------
 void att::query_cluster_occupancy(attuner_ctx* ctx) {
   if (ctx->tc_clusters[2] >= 0) return;
-  for (int ns = 0; ns <= 8; ++ns) ctx->tc_clusters[ns] = ns >= 2 ? attn_tc_max_clusters(ctx->cfg.head_dim, ns) : 0;
+  for (int ns = 0; ns <= 8; ++ns)
+    ctx->tc_clusters[ns] = (ns == 2 || ns == 4) ? attn_tc_max_clusters(ctx->cfg.head_dim, ns) : 0;
 }
 
 void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc,
@@ -647,8 +648,8 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
     maxv = std::max(maxv, nv);
   }
   const long long units = (long long)plan->n_req * Hkv * row_tiles;
-  // Cluster mode (tcgen05 kernel): every row tile cut into ns chunks, one
-  // cluster of ns CTAs per row tile.  Cost in 128-key tile times: waves of
+  // Cluster mode (tcgen05 kernel): every row tile cut into ns (2 or 4)
+  // chunks, one cluster of ns CTAs per row tile.  Cost in 128-key tile times: waves of
   // co-resident clusters x (largest chunk + ~4 tiles of prologue and epilogue
   // + ~1 for the merge).
   auto cluster_cost = [&](int ns) -> double {
@@ -663,8 +664,10 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
   int chunk;
   if (ctx->opt_split > 0) {
     chunk = ctx->opt_split;
+    // a cluster merges 2 or 4 chunks (whole column blocks per CTA)
     if (tc && ctx->opt_merge == 2 && maxv > chunk) {
-      cluster_ns = std::min(8, std::max(2, (maxv + chunk - 1) / chunk));
+      cluster_ns = (maxv + chunk - 1) / chunk <= 2 ? 2 : 4;
+      if ((((maxv + cluster_ns - 1) / cluster_ns) + 1) / 2 * 2 > kMaxChunkBlocks) cluster_ns = 0;
     }
   } else if (tc) {
     // Independent splits, one CTA per SM.  Cost of a chunk size = waves x
@@ -691,7 +694,7 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
       }
     }
     if (ctx->opt_merge != 1) {
-      for (int ns = 2; ns <= 8; ++ns) {
+      for (int ns = 2; ns <= 4; ns += 2) {   // a cluster merges 2 or 4 chunks
         const double cost = cluster_cost(ns);
         if (cost < best - 1e-9) {
           best = cost;

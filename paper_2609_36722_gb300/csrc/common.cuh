@@ -175,13 +175,15 @@ ATT_DEV bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort, long 
 }
 
 // Drain wait used on the abort path: waits for work this CTA itself issued
-// (TMA copies, MMAs), which completes without any other role's help.
+// (TMA copies, MMAs), or copies that peers issue unconditionally, which
+// complete without any other role's help.  False after a timeout.
 constexpr long long kDrainLimit = 1ll << 32;   // ~2 s at 2 GHz
-ATT_DEV void mbar_drain(uint32_t bar, uint32_t parity, int* status) {
+ATT_DEV bool mbar_drain(uint32_t bar, uint32_t parity, int* status) {
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > kDrainLimit) { set_status(status, ATTUNER_ERR_TIMEOUT); return; }
+    if (clock64() - t0 > kDrainLimit) { set_status(status, ATTUNER_ERR_TIMEOUT); return false; }
   }
+  return true;
 }
 
 // ---------------------------------------------------------------------------
@@ -265,10 +267,13 @@ ATT_DEV uint32_t dsmem_addr(uint32_t saddr, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(saddr), "r"(rank));
   return d;
 }
-ATT_DEV float ld_dsmem(uint32_t caddr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
-  return v;
+// bulk copy of `bytes` from this CTA's shared memory into a peer's (both
+// addresses 16-byte aligned, size a multiple of 16); completes on the peer's
+// mbarrier `cbar` (a shared::cluster address)
+ATT_DEV void bulk_push_dsmem(uint32_t cdst, uint32_t src, uint32_t bytes, uint32_t cbar) {
+  asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(cdst), "r"(src), "r"(bytes), "r"(cbar)
+               : "memory");
 }
 ATT_DEV uint32_t cluster_rank() {
   uint32_t r;

@@ -107,7 +107,8 @@ def test_ragged_multi_request(kernel, split):
 def test_split_merge_modes(merge, split, S, S_kv):
     # tcgen05 kernel, split-KV chunks merged through global memory (1) or inside
     # one thread-block cluster per row tile (2); 300 suffix tokens x G = 4 give
-    # ragged 256-row tiles, and 2..8 chunks per row tile with uneven row slices
+    # ragged 256-row tiles; clusters of 2 or 4 chunks per row tile (each CTA
+    # producing whole column blocks), global mode with up to 6 chunks
     import paper_2609_36722_gb300 as pkg
     wl = _ragged(seed=17, S=S, S_kv=S_kv, lengths=(37, 700, 64, 1, 1290))
     o_ref, lse_ref = _full_reference(wl)
