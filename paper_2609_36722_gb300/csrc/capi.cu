@@ -450,6 +450,16 @@ attuner_status att::check_common(attuner_ctx* ctx, const attuner_plan* plan, int
 // (row tile, head) when those tiles alone would leave SMs idle.  Off by
 // default: on GB300 the partial-sum traffic costs more than the extra SMs
 // bring for the Qwen3-4B and decode shapes.
+// CTAs per head of the projection kernel: when the tiles (grid heads x
+// 128-row blocks) cannot fill half the GPU, 2 or 4 CTAs share a head's
+// columns so that more SMs stream the weights (at least 32 columns each).
+static int qproj_parts(const attuner_ctx* ctx, int heads, int M) {
+  const long long tiles = (long long)heads * ((M + 127) / 128);
+  int parts = 1;
+  while (parts < 4 && 2 * parts * 32 <= ctx->cfg.head_dim && tiles * 2 * parts <= ctx->num_sms) parts *= 2;
+  return parts;
+}
+
 static int qproj_ksplit(const attuner_ctx* ctx, int M) {
   const int tiles = ctx->cfg.n_q_heads * ((M + 127) / 128);
   const int nk = ctx->cfg.hidden / 64;
@@ -504,10 +514,11 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
     const uint32_t box[2] = {64, 128};
     if ((e = make_map(&qp.tm_x, x, 2, dims, strides, box, "x")) != ATTUNER_OK) return e;
   }
+  const int parts = ksplit > 1 ? 1 : qproj_parts(ctx, Hq, M);
   {
     const uint64_t dims[2] = {(uint64_t)c.hidden, (uint64_t)dq};
     const uint64_t strides[1] = {(uint64_t)c.hidden * 2};
-    const uint32_t box[2] = {64, (uint32_t)D};
+    const uint32_t box[2] = {64, (uint32_t)(D / 2 / parts)};
     if ((e = make_map(&qp.tm_w, w_q, 2, dims, strides, box, "w_q")) != ATTUNER_OK) return e;
   }
   if (lora) {
@@ -517,7 +528,7 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
     if ((e = make_map(&qp.tm_a, lora_a, 2, dims, strides, box, "lora_a")) != ATTUNER_OK) return e;
     const uint64_t bdims[2] = {(uint64_t)r, (uint64_t)dq};
     const uint64_t bstrides[1] = {(uint64_t)r * 2};
-    const uint32_t bbox[2] = {8, (uint32_t)D};
+    const uint32_t bbox[2] = {8, (uint32_t)(D / 2 / parts)};
     if ((e = make_map(&qp.tm_b, lora_b, 2, bdims, bstrides, bbox, "lora_b", false)) != ATTUNER_OK) return e;
   }
   qp.q_out = static_cast<__nv_bfloat16*>(q_out);
@@ -535,6 +546,7 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
   qp.r = lora ? r : 0;
   qp.n_lora = n_lora;
   qp.ksplit = ksplit;
+  qp.parts = parts;
   qp.s = s;
   qp.eps = c.rms_eps;
   qp.status = ctx->d_status;
@@ -582,10 +594,11 @@ static attuner_status kv_project_impl(attuner_ctx* ctx, const attuner_plan* plan
     const uint32_t box[2] = {64, 128};
     if ((e = make_map(&qp.tm_x, x, 2, dims, strides, box, "x")) != ATTUNER_OK) return e;
   }
+  const int parts = qproj_parts(ctx, 2 * Hkv, M);
   {
     const uint64_t dims[2] = {(uint64_t)c.hidden, (uint64_t)dkv};
     const uint64_t strides[1] = {(uint64_t)c.hidden * 2};
-    const uint32_t box[2] = {64, (uint32_t)D};
+    const uint32_t box[2] = {64, (uint32_t)(D / 2 / parts)};
     if ((e = make_map(&qp.tm_w, w_k, 2, dims, strides, box, "w_k")) != ATTUNER_OK) return e;
     if ((e = make_map(&qp.tm_w2, w_v, 2, dims, strides, box, "w_v")) != ATTUNER_OK) return e;
   }
@@ -603,6 +616,7 @@ static attuner_status kv_project_impl(attuner_ctx* ctx, const attuner_plan* plan
   qp.r = 0;
   qp.n_lora = 0;
   qp.ksplit = 1;
+  qp.parts = parts;
   qp.s = 0.f;
   qp.eps = c.rms_eps;
   qp.status = ctx->d_status;

@@ -267,6 +267,11 @@ ATT_DEV uint32_t dsmem_addr(uint32_t saddr, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(saddr), "r"(rank));
   return d;
 }
+ATT_DEV float ld_dsmem(uint32_t caddr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
+  return v;
+}
 // bulk copy of `bytes` from this CTA's shared memory into a peer's (both
 // addresses 16-byte aligned, size a multiple of 16); completes on the peer's
 // mbarrier `cbar` (a shared::cluster address)

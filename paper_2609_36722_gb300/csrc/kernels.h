@@ -26,10 +26,10 @@ struct PrepParams {
 // GEMM (A stacked under W_q: one MMA of N = D + r) with a fused epilogue.
 struct QprojParams {
   CUtensorMap tm_x;    // x [M, hidden], box 64 x 128, SW128
-  CUtensorMap tm_w;    // W_q [d_q, hidden], box 64 x D, SW128
+  CUtensorMap tm_w;    // W_q [d_q, hidden], box 64 x D/2parts, SW128
   CUtensorMap tm_a;    // A [r, hidden], box 64 x n_lora, SW128 (rows past r read as zeros)
-  CUtensorMap tm_b;    // B [d_q, r], box 8 x D, no swizzle (columns past r read as zeros)
-  CUtensorMap tm_w2;   // K/V mode: W_v [Hkv*D, hidden], box 64 x D, SW128
+  CUtensorMap tm_b;    // B [d_q, r], box 8 x D/2parts, no swizzle (columns past r read as zeros)
+  CUtensorMap tm_w2;   // K/V mode: W_v [Hkv*D, hidden], box 64 x D/2parts, SW128
   __nv_bfloat16* q_out;            // Q mode: [M, Hq, D]; K/V mode: suffix K [n_req, S_kv, Hkv, D]
   __nv_bfloat16* out2;             // K/V mode: suffix V [n_req, S_kv, Hkv, D]
   const __nv_bfloat16* qnorm_w;    // [D] (q_norm, or k_norm in K/V mode)
@@ -37,6 +37,9 @@ struct QprojParams {
   float* part;                     // split-K partials [tiles][ksplit][128][D + n_lora]
   int32_t* counters;               // [tiles] arrivals per output tile (zero on entry)
   int32_t M, hidden, Hq, r, n_lora, ksplit;   // Hq: heads of the grid (2 Hkv in K/V mode)
+  // CTAs per head (1, 2 or 4; a cluster): each computes D/parts of the head's
+  // columns, two halves of D/2parts (tm_w, tm_w2 and tm_b boxes of D/2parts rows)
+  int32_t parts;
   // K/V mode (kv = 1): grid heads [0, Hout) project K (W = tm_w, key norm and
   // RoPE), [Hout, 2 Hout) project V (W = tm_w2, stored as is).  Row m of the
   // GEMM is token m % S of request m / S, written to output token row
