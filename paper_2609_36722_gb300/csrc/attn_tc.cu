@@ -32,6 +32,8 @@
 // <= 64512, so every score of a tile stays in registers.
 #include <math.h>
 
+#include <cuda_fp16.h>
+
 #include "kernels.h"
 
 namespace att {
@@ -161,10 +163,14 @@ __device__ __forceinline__ void store_cols(__nv_bfloat16* out, long long orow, i
 // Cluster-mode merge of the NS split-KV chunks of a row tile (one CTA per
 // chunk, cluster rank = split).  CTA `split` produces columns
 // [split, split + 1) x D/NS of all 256 rows.  Each CTA stages the other CTAs'
-// columns of its normalised O, [D/NS][256] fp32 per peer, and its LSE, and
-// pushes them into the peers' shared memory with bulk copies (the copy engine
-// moves distributed shared memory about twice as fast as loads from a peer
-// do); its own columns stay in tensor memory.  The chunks are summed in split
+// columns of its normalised O and its LSE, and pushes them into the peers'
+// shared memory with bulk copies (the copy engine moves distributed shared
+// memory about twice as fast as loads from a peer do); its own columns stay
+// in tensor memory.  The pushed columns travel as fp16 pairs divided by a
+// power of 2 per row (the one just above the row's largest magnitude, sent
+// beside them), so no value overflows and each keeps 11 bits relative to its
+// row's largest, finer than the bf16 rounding of the output; half the bytes
+// of fp32 halve the transfer, the epilogue's largest part.  The chunks are summed in split
 // order with the same arithmetic for the own chunk as for the others, so no
 // partial result goes to global memory and the sum does not depend on timing.
 template <int D, int NS>
@@ -173,18 +179,19 @@ __device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* s
                                                  long long orow, bool row_ok) {
   using L = TcLayout<D>;
   constexpr int CW = D / NS;                            // output columns per CTA
-  constexpr uint32_t kSlot = kTcRows * CW * 4;          // one chunk's columns of all rows
+  // one chunk's columns of all rows as fp16 pairs [CW/2][256], then a power-of-2 scale per row
+  constexpr uint32_t kVals = kTcRows * CW * 2;
+  constexpr uint32_t kSlot = kVals + kTcRows * 4;
   static_assert(CW % 16 == 0 && 2 * (NS - 1) * kSlot <= (uint32_t)L::BAR_OFF, "staging and receive slots");
   static_assert(NS <= 4, "LSE slots");
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 520);
   const uint32_t mbar = smem_u32(&bars[B_MF]);
   const int split = ce.split, erow = threadIdx.x;
-  float* src = reinterpret_cast<float*>(smem);           // NS-1 outgoing slots, peer order
-  float* rcv = src + (NS - 1) * (kSlot / 4);            // NS-1 incoming slots, split order
+  uint8_t* src = smem;                                  // NS-1 outgoing slots, peer order
+  uint8_t* rcv = smem + (NS - 1) * kSlot;               // NS-1 incoming slots, split order
   float* src_lse = reinterpret_cast<float*>(smem + L::XLSE_OFF);
   float* rcv_lse = src_lse + kTcRows;
-  // columns [c0, c0 + CW) of this thread's row, normalised (zeros for an empty chunk)
   auto own_cols = [&](int c0, float* v) {
     if (ok && ntile > 0) {
       if constexpr (CW >= 32) {
@@ -212,9 +219,21 @@ __device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* s
     if (t == split) continue;
     float v[CW];
     own_cols(t * CW, v);
-    float* dst = src + (t < split ? t : t - 1) * (kSlot / 4) + erow;
+    float amax = 0.f;
 #pragma unroll
-    for (int k = 0; k < CW; ++k) dst[k * kTcRows] = v[k];
+    for (int k = 0; k < CW; ++k) amax = fmaxf(amax, fabsf(v[k]));
+    // scale = the power of 2 just above the row's largest magnitude: v / scale in [-1, 1]
+    const int ex = (__float_as_int(amax) >> 23) & 0xff;
+    const float scale = (amax > 0.f && ex < 254) ? __int_as_float((ex + 1) << 23) : 1.f;
+    const float inv = 1.f / scale;
+    uint8_t* slot = src + (t < split ? t : t - 1) * kSlot;
+    uint32_t* dst = reinterpret_cast<uint32_t*>(slot) + erow;
+#pragma unroll
+    for (int c = 0; c < CW / 2; ++c) {
+      const __half2 h = __floats2half2_rn(v[2 * c] * inv, v[2 * c + 1] * inv);
+      dst[c * kTcRows] = *reinterpret_cast<const uint32_t*>(&h);
+    }
+    reinterpret_cast<float*>(slot + kVals)[erow] = scale;
   }
   src_lse[erow] = lse;
   fence_proxy_async_smem();
@@ -230,8 +249,6 @@ __device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* s
       bulk_push_dsmem(dsmem_addr(smem_u32(rcv_lse) + at * kTcRows * 4, t), smem_u32(src_lse), kTcRows * 4, cbar);
     }
   }
-  // Every CTA waits for its incoming copies, also after an abort: the peers
-  // issue them unconditionally, and none may land after this CTA has exited.
   const bool got = __all_sync(0xffffffffu, mbar_drain(mbar, 0, p.status));
   if (got && !*abort_flag) {
     float w[NS];
@@ -257,9 +274,16 @@ __device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* s
 #pragma unroll
         for (int c = 0; c < CW; ++c) acc[c] = __fmaf_rn(w[k], own[c], acc[c]);
       } else {
-        const float* r = rcv + (k < split ? k : k - 1) * (kSlot / 4) + erow;
+        const uint8_t* slot = rcv + (k < split ? k : k - 1) * kSlot;
+        const uint32_t* r = reinterpret_cast<const uint32_t*>(slot) + erow;
+        const float wk = w[k] * reinterpret_cast<const float*>(slot + kVals)[erow];
 #pragma unroll
-        for (int c = 0; c < CW; ++c) acc[c] = __fmaf_rn(w[k], r[c * kTcRows], acc[c]);
+        for (int c = 0; c < CW / 2; ++c) {
+          const uint32_t bits = r[c * kTcRows];
+          const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&bits));
+          acc[2 * c] = __fmaf_rn(wk, f.x, acc[2 * c]);
+          acc[2 * c + 1] = __fmaf_rn(wk, f.y, acc[2 * c + 1]);
+        }
       }
     }
     if (row_ok) {
