@@ -107,6 +107,9 @@ extern "C" attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const 
     if ((e = make_map(&ap.tm_ksuf, suffix_k, 4, dims, strides, box, "suffix_k")) != ATTUNER_OK) return e;
     if ((e = make_map(&ap.tm_vsuf, suffix_v, 4, dims, strides, box, "suffix_v")) != ATTUNER_OK) return e;
   }
+  if (tc && ap.work.cluster > 0 &&
+      (e = make_out_map(&ap.tm_out, out, D, Hq, G, S, plan->n_req, ap.work.cluster)) != ATTUNER_OK)
+    return e;
   ap.tm_kpool = ctx->tm_kpool;
   ap.tm_vpool = ctx->tm_vpool;
   ap.plan = plan_dev(plan);

@@ -170,9 +170,12 @@ __device__ __forceinline__ void store_cols(__nv_bfloat16* out, long long orow, i
 // power of 2 per row (the one just above the row's largest magnitude, sent
 // beside them), so no value overflows and each keeps 11 bits relative to its
 // row's largest, finer than the bf16 rounding of the output; half the bytes
-// of fp32 halve the transfer, the epilogue's largest part.  The chunks are summed in split
-// order with the same arithmetic for the own chunk as for the others, so no
-// partial result goes to global memory and the sum does not depend on timing.
+// of fp32 halve the transfer, the epilogue's largest part.  The chunks are
+// summed in split order with the same arithmetic whichever CTA finishes
+// first, and the merged [256][D/NS] bf16 tile leaves through one TMA tensor
+// store (rows past the last token clipped by the map) instead of 64-byte
+// pieces per row.  The loops over peers stay rolled: this code runs once per
+// CTA, cold, and its instruction fetch costs more than its arithmetic.
 template <int D, int NS>
 __device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* smem, const TcCta& ce,
                                                  uint32_t o_col, bool ok, int ntile, float inv_l, float lse,
@@ -214,7 +217,7 @@ __device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* s
     }
   };
   if (threadIdx.x == 0) mbar_expect_tx(mbar, (NS - 1) * (kSlot + kTcRows * 4));
-#pragma unroll
+#pragma unroll 1
   for (int t = 0; t < NS; ++t) {
     if (t == split) continue;
     float v[CW];
@@ -239,7 +242,7 @@ __device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* s
   fence_proxy_async_smem();
   cluster_sync_all();   // 1: every CTA of the cluster has staged; all main loops are over
   if (threadIdx.x == 0) {
-#pragma unroll
+#pragma unroll 1
     for (int t = 0; t < NS; ++t) {
       if (t == split) continue;
       const uint32_t at = (split < t ? split : split - 1);   // this CTA's slot at peer t
@@ -249,34 +252,42 @@ __device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* s
       bulk_push_dsmem(dsmem_addr(smem_u32(rcv_lse) + at * kTcRows * 4, t), smem_u32(src_lse), kTcRows * 4, cbar);
     }
   }
+  // this CTA's own columns while the peers' arrive
+  float acc[CW];
+  own_cols(split * CW, acc);
+  // Every CTA waits for its incoming copies, also after an abort: the peers
+  // issue them unconditionally, and none may land after this CTA has exited.
+  // One answer for the whole CTA, so the barrier below is passed by all.
   const bool got = __all_sync(0xffffffffu, mbar_drain(mbar, 0, p.status));
-  if (got && !*abort_flag) {
-    float w[NS];
+  if (!got && (threadIdx.x & 31) == 0) *abort_flag = 1;
+  asm volatile("bar.sync 1, 256;" ::: "memory");
+  const bool merge = *abort_flag == 0;
+  // output tile [256 rows][CW] bf16 after the slots, in the tensor map's swizzle
+  constexpr uint32_t kOutOff = (2 * (NS - 1) * kSlot + 1023) & ~1023u;
+  static_assert(kOutOff + kTcRows * CW * 2 <= (uint32_t)L::BAR_OFF, "output tile");
+  if (merge) {
+    auto lse_of = [&](int k) { return (k == split) ? lse : rcv_lse[(k < split ? k : k - 1) * kTcRows + erow]; };
     float mx = -INFINITY;
+#pragma unroll 1
+    for (int k = 0; k < NS; ++k) mx = fmaxf(mx, lse_of(k));
+    // chunks in split order; the own chunk's term first computed into acc[] is
+    // rebuilt in order: acc = sum_k w_k * chunk_k
+    float own[CW];
 #pragma unroll
-    for (int k = 0; k < NS; ++k) {
-      w[k] = (k == split) ? lse : rcv_lse[(k < split ? k : k - 1) * kTcRows + erow];
-      mx = fmaxf(mx, w[k]);
-    }
+    for (int c = 0; c < CW; ++c) { own[c] = acc[c]; acc[c] = 0.f; }
     float wsum = 0.f;
-#pragma unroll
+#pragma unroll 1
     for (int k = 0; k < NS; ++k) {
-      w[k] = (w[k] == -INFINITY) ? 0.f : __expf(w[k] - mx);
-      wsum += w[k];
-    }
-    float own[CW], acc[CW];
-    own_cols(split * CW, own);
-#pragma unroll
-    for (int c = 0; c < CW; ++c) acc[c] = 0.f;
-#pragma unroll
-    for (int k = 0; k < NS; ++k) {
+      const float lk = lse_of(k);
+      const float w = (lk == -INFINITY) ? 0.f : __expf(lk - mx);
+      wsum += w;
       if (k == split) {
 #pragma unroll
-        for (int c = 0; c < CW; ++c) acc[c] = __fmaf_rn(w[k], own[c], acc[c]);
+        for (int c = 0; c < CW; ++c) acc[c] = __fmaf_rn(w, own[c], acc[c]);
       } else {
         const uint8_t* slot = rcv + (k < split ? k : k - 1) * kSlot;
         const uint32_t* r = reinterpret_cast<const uint32_t*>(slot) + erow;
-        const float wk = w[k] * reinterpret_cast<const float*>(slot + kVals)[erow];
+        const float wk = w * reinterpret_cast<const float*>(slot + kVals)[erow];
 #pragma unroll
         for (int c = 0; c < CW / 2; ++c) {
           const uint32_t bits = r[c * kTcRows];
@@ -286,12 +297,29 @@ __device__ __forceinline__ void tc_cluster_merge(const AttnParams& p, uint8_t* s
         }
       }
     }
-    if (row_ok) {
-      store_cols<D, CW>(p.out, orow, split * CW, acc, wsum > 0.f ? 1.f / wsum : 0.f);
-      if (split == 0 && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
+    const float sc = wsum > 0.f ? 1.f / wsum : 0.f;
+    // row erow of the tile: 16-byte chunk j at j ^ (bits 7.. of its offset), as the
+    // tensor map's swizzle of CW * 2 bytes places it
+    constexpr uint32_t kSwzMask = CW * 2 / 16 - 1;
+    const uint32_t tile = smem_u32(smem) + kOutOff;
+#pragma unroll
+    for (int j = 0; j < CW / 8; ++j) {
+      const uint32_t off = erow * (CW * 2) + j * 16;
+      st_shared_v4(tile + (off ^ (((off >> 7) & kSwzMask) << 4)),
+                   pack_bf16(acc[8 * j] * sc, acc[8 * j + 1] * sc), pack_bf16(acc[8 * j + 2] * sc, acc[8 * j + 3] * sc),
+                   pack_bf16(acc[8 * j + 4] * sc, acc[8 * j + 5] * sc), pack_bf16(acc[8 * j + 6] * sc, acc[8 * j + 7] * sc));
+    }
+    if (row_ok && split == 0 && p.lse_out) p.lse_out[orow] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
+    fence_proxy_async_smem();
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+    if (threadIdx.x == 0) {
+      // rows past the last token are clipped by the tensor map
+      tma_store_4d(&p.tm_out, tile, split * CW, ce.kvh * p.G, ce.rt * (kTcRows / p.G), ce.req);
+      bulk_commit();
     }
   }
   cluster_sync_all();   // 2: every copy has landed; no CTA leaves while a peer may still read its slots
+  if (threadIdx.x == 0) bulk_wait_read_all();   // the output tile has been read
 }
 
 // Epilogue of the softmax warps (warps 0..7, one CTA row per thread): O from

@@ -49,7 +49,7 @@ static EncodeTiledFn encode_fn() {
 // stride of dims[i+1].
 attuner_status att::make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
                                const uint64_t* strides, const uint32_t* box, const char* what,
-                               bool swizzle128) {
+                               int swizzle_bytes) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return fail(ATTUNER_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
   if ((reinterpret_cast<uintptr_t>(base) & 15) != 0)
@@ -65,12 +65,24 @@ attuner_status att::make_map(CUtensorMap* m, const void* base, int rank, const u
   }
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base), d, s, b, e,
                   CU_TENSOR_MAP_INTERLEAVE_NONE,
-                  swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                  swizzle_bytes == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                  : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                  : swizzle_bytes == 32 ? CU_TENSOR_MAP_SWIZZLE_32B
+                                        : CU_TENSOR_MAP_SWIZZLE_NONE,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS)
     return fail(ATTUNER_ERR_CUDA, std::string("cuTensorMapEncodeTiled failed for ") + what +
                                       " (CUresult " + std::to_string((int)r) + ")");
   return ATTUNER_OK;
+}
+
+attuner_status att::make_out_map(CUtensorMap* m, void* out, int D, int Hq, int G, int S, int n_req,
+                                 int cluster) {
+  const int cw = D / cluster;   // columns one CTA writes: one box row of cw * 2 bytes
+  const uint64_t dims[4] = {(uint64_t)D, (uint64_t)Hq, (uint64_t)S, (uint64_t)n_req};
+  const uint64_t strides[3] = {(uint64_t)D * 2, (uint64_t)Hq * D * 2, (uint64_t)S * Hq * D * 2};
+  const uint32_t box[4] = {(uint32_t)cw, (uint32_t)G, (uint32_t)(kTcRows / G), 1};
+  return make_map(m, out, 4, dims, strides, box, "out", cw * 2);
 }
 
 attuner_status att::set_device(const attuner_ctx* ctx) {
@@ -529,7 +541,7 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
     const uint64_t bdims[2] = {(uint64_t)r, (uint64_t)dq};
     const uint64_t bstrides[1] = {(uint64_t)r * 2};
     const uint32_t bbox[2] = {8, (uint32_t)(D / 2 / parts)};
-    if ((e = make_map(&qp.tm_b, lora_b, 2, bdims, bstrides, bbox, "lora_b", false)) != ATTUNER_OK) return e;
+    if ((e = make_map(&qp.tm_b, lora_b, 2, bdims, bstrides, bbox, "lora_b", 0)) != ATTUNER_OK) return e;
   }
   qp.q_out = static_cast<__nv_bfloat16*>(q_out);
   qp.qnorm_w = static_cast<const __nv_bfloat16*>(q_norm_w);
@@ -791,6 +803,9 @@ static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, co
     if ((e = make_map(&ap->tm_ksuf, suffix_k, 4, dims, strides, box, "suffix_k")) != ATTUNER_OK) return done(e);
     if ((e = make_map(&ap->tm_vsuf, suffix_v, 4, dims, strides, box, "suffix_v")) != ATTUNER_OK) return done(e);
   }
+  if (tc && w->cluster > 0 &&
+      (e = make_out_map(&ap->tm_out, out, D, Hq, G, S, plan->n_req, w->cluster)) != ATTUNER_OK)
+    return done(e);
   ap->tm_kpool = ctx->tm_kpool;
   ap->tm_vpool = ctx->tm_vpool;
   ap->plan = plan_dev(plan);

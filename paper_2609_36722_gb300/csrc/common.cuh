@@ -216,6 +216,16 @@ ATT_DEV void tma_load_5d(uint32_t dst, const CUtensorMap* m, uint32_t bar, int c
       : "memory");
 }
 
+// tiled tensor store shared -> global (bulk group of the issuing thread); boxes
+// past the tensor's bounds are clipped.  Coordinates must not be negative.
+ATT_DEV void tma_store_4d(const CUtensorMap* m, uint32_t src, int c0, int c1, int c2, int c3) {
+  asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.tile.bulk_group [%0, {%2, %3, %4, %5}], [%1];"
+               ::"l"(reinterpret_cast<uint64_t>(m)), "r"(src), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+               : "memory");
+}
+// waits until the bulk copies of this thread have read their shared-memory source
+ATT_DEV void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+
 // generic-proxy shared-memory writes -> visible to the async proxy (UMMA, TMA)
 ATT_DEV void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");

@@ -70,10 +70,13 @@ namespace att {
 
 // record `msg` as this thread's last error and return `s`
 attuner_status fail(attuner_status s, const std::string& msg);
-// bf16 tensor map with zero fill out of bounds; 128-byte swizzle unless swizzle128 is false
+// bf16 tensor map with zero fill out of bounds; swizzle_bytes 128 (default),
+// 64, 32 or 0 (none)
 attuner_status make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
                         const uint64_t* strides, const uint32_t* box, const char* what,
-                        bool swizzle128 = true);
+                        int swizzle_bytes = 128);
+// the cluster-mode output map of the tcgen05 attention kernel (see AttnParams::tm_out)
+attuner_status make_out_map(CUtensorMap* m, void* out, int D, int Hq, int G, int S, int n_req, int cluster);
 attuner_status set_device(const attuner_ctx* ctx);
 bool aligned16(const void* p);
 PlanDev plan_dev(const attuner_plan* p);

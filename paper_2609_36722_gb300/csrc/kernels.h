@@ -57,6 +57,9 @@ struct AttnParams {
   CUtensorMap tm_vpool;
   CUtensorMap tm_ksuf;   // suffix K viewed 4-D (D, Hkv, S_kv, n_req), box 64 x 1 x 64 x 1
   CUtensorMap tm_vsuf;
+  // cluster mode of K2 only: out viewed 4-D (D, Hq, S, n_req), box (D/cluster,
+  // G, 256/G, 1), swizzle = the box row's bytes (32, 64 or 128)
+  CUtensorMap tm_out;
   PlanDev plan;
   WorkTable work;
   const __nv_bfloat16* q;        // (K3 reads Q directly)
