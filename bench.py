@@ -218,11 +218,25 @@ def run_ours(args, rank, world, local_rank):
             ev_b.record()
         return n1 + ctx.last_launch_count()
 
+    class Eager:
+        # --eager: the same calls launched directly, with the events around them
+        # (profilers step through graph replays very slowly)
+        def __init__(self, fn, e0, e1):
+            self.fn, self.e0, self.e1 = fn, e0, e1
+
+        def replay(self):
+            self.e0.record()
+            self.fn()
+            self.e1.record()
+
     def graphed(fn):
         # The timed work replays a CUDA graph of the calls: one launch for the
         # host, so the GPU never waits on the Python binding or the per-call
         # host setup between kernels.  Events inside the graph time it on the
         # device.
+        if args.eager:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            return Eager(fn, e0, e1), e0, e1
         e0, e1 = gevent(), gevent()
         for _ in range(3):
             fn()
@@ -237,7 +251,7 @@ def run_ours(args, rank, world, local_rank):
 
     def gevent():
         # an event that a captured graph records as a node of its own
-        return torch.cuda.Event(enable_timing=True, external=True)
+        return torch.cuda.Event(enable_timing=True, external=not args.eager)
 
     ev_q, ev_a, ev_b = gevent(), gevent(), gevent()
     for _ in range(args.warmup):
@@ -443,7 +457,8 @@ def run_ours(args, rank, world, local_rank):
                    "artifacts_per_req": [len(r) for r in wl.requests][:8],
                    "parallelism": f"replicas x{world}",
                    "l2": f"flushed between timed steps ({L2_FLUSH_BYTES >> 20} MiB write, outside the events)",
-                   "attention_kernel": "tcgen05 (attn_tc)" if not decode else "split-KV warp-MMA (attn_mma)"},
+                   "attention_kernel": "tcgen05 (attn_tc)" if not decode else "split-KV warp-MMA (attn_mma)",
+                   "launch": "eager calls" if args.eager else "CUDA graph replay of the calls"},
         "roofline": {"bound": "hbm" if decode else "tensor", "achieved": round(achieved, 3), "peak": peak,
                      "unit": unit, "frac": round(achieved / peak, 4), "traffic": traffic,
                      "kernel": ("attn_mma_kernel + combine_kernel" if decode else "attn_tc_kernel (split-KV chunks merged inside it)"),
@@ -544,6 +559,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="qwen3_4b_prefill")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--eager", action="store_true",
+                    help="launch the timed calls directly instead of replaying CUDA graphs (for profilers)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
