@@ -120,6 +120,25 @@ def test_split_merge_modes(merge, split, S, S_kv):
     compare(_np(out), o_ref, _np(lse), lse_ref, label=f"merge={merge} split={split} S={S}")
 
 
+G64 = Geometry(hidden=256, n_q_heads=8, n_kv_heads=2, head_dim=64, rank=8)
+
+
+@pytest.mark.parametrize("merge", [1, 2])
+@pytest.mark.parametrize("split,S,S_kv", [(4, 300, 300), (16, 130, 200)])
+def test_split_merge_modes_head_dim_64(merge, split, S, S_kv):
+    # head_dim 64: clusters of 4 (16 output columns per CTA, a 32-byte row of
+    # the output tile) and of 2 (32 columns, 64-byte rows), and the global mode
+    import paper_2609_36722_gb300 as pkg
+    wl = _ragged(seed=19, S=S, S_kv=S_kv, geom=G64, lengths=(37, 700, 64, 1, 1290))
+    o_ref, lse_ref = _full_reference(wl)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, 1)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, split)
+    ctx.set_option(pkg.OPT_SPLIT_MERGE, merge)
+    out, lse = run_path(ctx, plan, wl)
+    compare(_np(out), o_ref, _np(lse), lse_ref, label=f"d=64 merge={merge} split={split} S={S}")
+
+
 @pytest.mark.parametrize("G", [1, 2, 8])
 def test_group_sizes(G):
     geom = Geometry(hidden=256, n_q_heads=4 * G, n_kv_heads=4, head_dim=128, rank=8)

@@ -58,6 +58,28 @@ def test_static_scratch_matches_attend_twice(kernel, split, S, S_kv):
         assert (lse - ref_l).abs().max().item() <= LSE_MAX_ABS
 
 
+@pytest.mark.parametrize("split", [4, 24])
+def test_static_scratch_cluster_merge(split):
+    # split-KV chunks merged inside thread-block clusters (4 and 2 CTAs): no
+    # partial results in any scratch, the output leaves by the kernel's tensor
+    # store; the result equals attuner_attend's
+    import paper_2609_36722_gb300 as pkg
+    geom = Geometry(hidden=256, n_q_heads=16, n_kv_heads=4, head_dim=128, rank=16)
+    wl = make_custom("noalloc_cl", geom, 43, [700, 333, 1200, 64], [[2, 0, 3], [1, 3], [0, 1, 2, 3]], 96, 96,
+                     device=DEV)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, 1)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, split)
+    ctx.set_option(pkg.OPT_SPLIT_MERGE, 2)
+    g = wl.geom
+    q = ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=96)
+    ref_o, ref_l = ctx.attend(plan, q, wl.suffix_k, wl.suffix_v)
+    assert ctx.sync_status() == 0 and ctx.last_launch_count() == 1
+    out, lse = ctx.attend_static_scratch(plan, q, wl.suffix_k, wl.suffix_v)
+    assert ctx.sync_status() == 0 and ctx.last_launch_count() == 1
+    assert torch.equal(out, ref_o) and torch.equal(lse, ref_l)
+
+
 def test_static_scratch_rejects_calls_beyond_its_size():
     import paper_2609_36722_gb300 as pkg
     geom = Geometry(hidden=256, n_q_heads=32, n_kv_heads=8, head_dim=128, rank=16)
