@@ -80,8 +80,10 @@ typedef struct attuner_plan attuner_plan;
 attuner_status attuner_create(const attuner_config* cfg, attuner_ctx** out);
 
 /* Free the context, its pool and every stream-ordered scratch it cached.
- * The caller must have finished all work it enqueued with this context and
- * freed its plans first. NULL is accepted. */
+ * The caller must have finished all work it enqueued with this context.
+ * Plans of the context not yet freed must not be used afterwards; freeing
+ * them later is allowed (each releases its own device buffer then). NULL is
+ * accepted. */
 attuner_status attuner_destroy(attuner_ctx* ctx);
 
 /* Register one artifact (Sec. 2, Eq. full-vs-pic: Z^PIC = C(A | P_cache),
@@ -142,7 +144,9 @@ attuner_status attuner_plan_export(const attuner_plan* plan, int32_t* block_tabl
 /* Per-request assembled artifact length T_art (host array of n_req). */
 attuner_status attuner_plan_t_art(const attuner_plan* plan, int32_t* t_art_host, int32_t n_req);
 
-/* Free a plan. The caller must have finished all work that reads it. */
+/* Free a plan. The caller must have finished all work that reads it. Its
+ * device buffer goes back to the context, which reuses a few such buffers
+ * for later assemblies instead of allocating. */
 attuner_status attuner_plan_free(attuner_plan* plan);
 
 /* Adapted query of the online tokens (Sec. 3, Eq. query-adaptation, then

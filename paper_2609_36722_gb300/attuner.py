@@ -8,7 +8,9 @@ shared library is missing, importing this module raises.
 
 from __future__ import annotations
 
+import array
 import ctypes
+import itertools
 import os
 from typing import List, Optional, Sequence
 
@@ -235,14 +237,22 @@ class Context:
     def pool_reset(self) -> None:
         _check(lib().attuner_pool_reset(self.handle))
 
+    @staticmethod
+    def _csr(reqs):
+        # int32 arrays of the flattened items and their offsets (array.array fills
+        # them in C; ctypes views their buffers without copying)
+        flat = array.array("i", itertools.chain.from_iterable(reqs))
+        if not flat:
+            flat.append(0)
+        offs = array.array("i", [0])
+        offs.extend(itertools.accumulate(len(r) for r in reqs))
+        c_flat = (ctypes.c_int32 * len(flat)).from_buffer(flat)
+        c_offs = (ctypes.c_int32 * len(offs)).from_buffer(offs)
+        return (flat, offs), c_flat, c_offs
+
     def assemble(self, requests: Sequence[Sequence[int]]) -> Plan:
         reqs = [list(map(int, r)) for r in requests]
-        flat = [a for r in reqs for a in r]
-        offs = [0]
-        for r in reqs:
-            offs.append(offs[-1] + len(r))
-        ids = (ctypes.c_int32 * max(len(flat), 1))(*flat)
-        off_arr = (ctypes.c_int32 * len(offs))(*offs)
+        keep, ids, off_arr = self._csr(reqs)
         h = ctypes.c_void_p()
         _check(lib().attuner_assemble(self.handle, ids, off_arr, len(reqs), ctypes.byref(h)))
         return Plan(self, h, reqs)
@@ -252,12 +262,7 @@ class Context:
         an artifact id, item < 0 an online span of -item tokens (the online
         rows after the last item form the final span)."""
         reqs = [list(map(int, r)) for r in layouts]
-        flat = [a for r in reqs for a in r]
-        offs = [0]
-        for r in reqs:
-            offs.append(offs[-1] + len(r))
-        items = (ctypes.c_int32 * max(len(flat), 1))(*flat)
-        off_arr = (ctypes.c_int32 * len(offs))(*offs)
+        keep, items, off_arr = self._csr(reqs)
         h = ctypes.c_void_p()
         _check(lib().attuner_assemble_layout(self.handle, items, off_arr, len(reqs), ctypes.byref(h)))
         return Plan(self, h, [[a for a in r if a >= 0] for r in reqs])

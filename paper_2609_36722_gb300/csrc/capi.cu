@@ -181,6 +181,11 @@ extern "C" attuner_status attuner_destroy(attuner_ctx* ctx) {
   if (ctx->vpool) cudaFree(ctx->vpool);
   if (ctx->d_status) cudaFree(ctx->d_status);
   if (ctx->mempool) cudaMemPoolDestroy(ctx->mempool);
+  {
+    std::lock_guard<std::mutex> lk(ctx->plan_mu);
+    for (attuner_plan* p : ctx->live_plans) p->ctx = nullptr;
+    for (auto& b : ctx->plan_bufs) cudaFree(b.second);
+  }
   delete ctx;
   return ATTUNER_OK;
 }
@@ -344,15 +349,39 @@ static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const 
   p->spans_at = h.size();
   h.insert(h.end(), p->spans.begin(), p->spans.end());
   if (h.empty()) h.push_back(0);
-  if (cudaMalloc(&p->d_buf, h.size() * sizeof(int32_t)) != cudaSuccess) {
-    cudaGetLastError();
-    delete p;
-    return fail(ATTUNER_ERR_OOM, "plan allocation failed");
+  // a buffer of a freed plan when one is large enough (no allocation per assembly)
+  const size_t bytes = h.size() * sizeof(int32_t);
+  p->ctx = ctx;
+  {
+    std::lock_guard<std::mutex> lk(ctx->plan_mu);
+    size_t best = ctx->plan_bufs.size();
+    for (size_t i = 0; i < ctx->plan_bufs.size(); ++i)
+      if (ctx->plan_bufs[i].first >= bytes && (best == ctx->plan_bufs.size() || ctx->plan_bufs[i].first < ctx->plan_bufs[best].first))
+        best = i;
+    if (best < ctx->plan_bufs.size()) {
+      p->d_cap = ctx->plan_bufs[best].first;
+      p->d_buf = ctx->plan_bufs[best].second;
+      ctx->plan_bufs.erase(ctx->plan_bufs.begin() + best);
+    }
   }
-  if (cudaMemcpy(p->d_buf, h.data(), h.size() * sizeof(int32_t), cudaMemcpyHostToDevice) != cudaSuccess) {
+  if (!p->d_buf) {
+    size_t cap = 4096;
+    while (cap < bytes) cap *= 2;
+    if (cudaMalloc(&p->d_buf, cap) != cudaSuccess) {
+      cudaGetLastError();
+      delete p;
+      return fail(ATTUNER_ERR_OOM, "plan allocation failed");
+    }
+    p->d_cap = cap;
+  }
+  if (cudaMemcpy(p->d_buf, h.data(), bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
     cudaFree(p->d_buf);
     delete p;
     return fail(ATTUNER_ERR_CUDA, "plan upload failed");
+  }
+  {
+    std::lock_guard<std::mutex> lk(ctx->plan_mu);
+    ctx->live_plans.insert(p);
   }
   *out = p;
   return ATTUNER_OK;
@@ -420,6 +449,16 @@ extern "C" attuner_status attuner_plan_t_art(const attuner_plan* p, int32_t* t_a
 
 extern "C" attuner_status attuner_plan_free(attuner_plan* p) {
   if (!p) return ATTUNER_OK;
+  // keep the buffer for the context's next assemblies (a few at most)
+  constexpr size_t kCachedPlanBufs = 8;
+  if (p->ctx) {
+    std::lock_guard<std::mutex> lk(p->ctx->plan_mu);
+    p->ctx->live_plans.erase(p);
+    if (p->d_buf && p->ctx->plan_bufs.size() < kCachedPlanBufs) {
+      p->ctx->plan_bufs.emplace_back(p->d_cap, p->d_buf);
+      p->d_buf = nullptr;
+    }
+  }
   if (p->d_buf) {
     int cur = -1;
     cudaGetDevice(&cur);

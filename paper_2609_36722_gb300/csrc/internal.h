@@ -3,7 +3,10 @@
 // public boundary, which is include/attuner.h.
 #pragma once
 
+#include <mutex>
 #include <string>
+#include <unordered_set>
+#include <utility>
 #include <vector>
 
 #include "kernels.h"
@@ -44,9 +47,17 @@ struct attuner_ctx {
   long long wait_limit = 1ll << 32;
   int inject_stuck = 0;
   int last_launches = 0;
+  // device buffers of freed plans, reused by the next assemblies (capacity,
+  // pointer), and the plans not yet freed (detached when the context goes, so
+  // a plan freed after its context frees its own buffer)
+  std::mutex plan_mu;
+  std::vector<std::pair<size_t, int32_t*>> plan_bufs;
+  std::unordered_set<attuner_plan*> live_plans;
 };
 
 struct attuner_plan {
+  attuner_ctx* ctx = nullptr;     // owner of d_buf's cache; null once the context is destroyed
+  size_t d_cap = 0;               // bytes of d_buf
   int32_t n_req = 0;
   int32_t device = 0;
   int32_t pool_blocks = 0;

@@ -121,3 +121,23 @@ def test_repeated_calls_are_bit_identical(S, S_kv, merge):
     o1, l1 = run_path(ctx, plan, wl)
     o2, l2 = run_path(ctx, plan, wl)
     assert torch.equal(o1, o2) and torch.equal(l1, l2)
+
+
+def test_plan_buffers_reused_and_plans_freed_after_their_context():
+    # freed plans hand their device buffers back to the context, which reuses
+    # them for later assemblies of other sizes: results stay bit-identical to
+    # a first assembly; a plan freed after its context releases its own buffer
+    import paper_2609_36722_gb300 as pkg
+    wl = make_custom("reuse", GEOM, 29, [150, 64, 333, 20, 900], [[3, 0, 2, 1], [1, 2, 4]], 40, 48, device=DEV)
+    ctx, plan = load_context(wl)
+    o1, l1 = run_path(ctx, plan, wl)
+    plan.free()
+    for reqs in ([[4, 4, 4, 4], [0]], [[1]], [[0, 1, 2, 3, 4], [4, 3, 2, 1, 0]]):
+        ctx.assemble(reqs).free()
+    again = ctx.assemble(wl.requests)
+    o2, l2 = run_path(ctx, again, wl)
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    late = ctx.assemble(wl.requests)
+    again.free()
+    ctx.close()
+    late.free()   # after the context: must not touch it
