@@ -339,7 +339,7 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
   const int G = p.G;
   grid_dep_wait();   // before the first global write (the producer thread has waited already)
   const TcCta ce = tc_cta(p, blockIdx.x);
-  const int split = ce.split, nsplit = ce.nsplit;
+  const int nsplit = ce.nsplit;
   const int erow = threadIdx.x;                               // CTA row = thread (warps 0..7)
   const int epr = ce.rt * kTcRows + erow;                     // packed row
   const bool row_ok = epr / G < p.S;
@@ -351,29 +351,6 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
   auto out_row = [&](int pr) {
     return ((long long)ce.req * p.S + pr / G) * p.Hq + ce.kvh * G + pr % G;
   };
-  // Split-KV partial results are staged in the Q/K/V area, free once the last
-  // MMA has completed.  Global mode stages them column-major ([d][256 rows]
-  // fp32): 32 columns are one contiguous 32 KiB piece for one bulk copy, and a
-  // warp's accesses to one column are 128 consecutive bytes.
-  constexpr int kPiece = 32 * kTcRows * 4;
-  float* stage = reinterpret_cast<float*>(smem);
-  auto stage_own = [&]() {
-    if (!ok) return;
-#pragma unroll
-    for (int c = 0; c < D / 32; ++c) {
-      float* sb = stage + c * (kPiece / 4);
-      if (ntile > 0) {
-        float o[32];
-        tmem_ld32(o_col + c * 32, o);
-        tc_wait_ld();
-#pragma unroll
-        for (int k = 0; k < 32; ++k) sb[k * kTcRows + erow] = o[k] * inv_l;
-      } else {
-#pragma unroll
-        for (int k = 0; k < 32; ++k) sb[k * kTcRows + erow] = 0.f;
-      }
-    }
-  };
   if (p.work.cluster > 0) {
     if (nsplit == 4)
       tc_cluster_merge<D, 4>(p, smem, ce, o_col, ok, ntile, inv_l, lse, out_row(epr), row_ok);
@@ -382,24 +359,54 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
   } else if (nsplit > 1) {
     // Independent splits: publish this chunk's normalised O and its
     // log-sum-exp through global memory; the last CTA of the (request, KV
-    // head, row tile) to arrive merges all chunks.
+    // head, row tile) to arrive merges all chunks.  A published piece is 32
+    // columns of the 256 rows as fp16 pairs [16][256] (each row divided by the
+    // power of 2 just above its largest magnitude in those columns), then the
+    // 256 scales: half the bytes of fp32, and a warp's accesses to one pair
+    // are 128 consecutive bytes.  The merge reads every chunk back, the
+    // merging CTA's own too, so the sum is the same whichever CTA is last.
     const int cta = cta_index_fresh();
     const int r = erow;
     const long long orow = out_row(epr);
-    auto store_row32o = [&](int c, const float* o, float scale) { store_cols<D, 32>(p.out, orow, c * 32, o, scale); };
     const int req = ce.req, kvh = ce.kvh, rt = ce.rt;
-    constexpr int kBufs = L::BAR_OFF / kPiece;       // 6 (d = 128) or 3 (d = 64)
-    constexpr int kRing = kBufs - 1;                 // the last one holds the merge weights
-    static_assert(D / 32 <= kRing && kRing <= 8, "staging buffers");
-    static_assert(kMaxSplits * kTcRows * 4 <= kPiece, "merge weights buffer");
-    float* po = p.part_o + (long long)cta * kTcRows * D;
-    stage_own();
+    constexpr int kVals = 16 * kTcRows * 4;                 // 16 KiB of fp16 pairs
+    constexpr int kPiece = kVals + kTcRows * 4;             // + 1 KiB of scales
+    constexpr int kWtsOff = L::BAR_OFF - kMaxSplits * kTcRows * 4;   // merge weights [kMaxSplits][256]
+    constexpr int kRing = (kWtsOff / kPiece) < 8 ? (kWtsOff / kPiece) : 8;
+    static_assert(D / 32 * kPiece <= kWtsOff && kRing >= 2, "staging buffers");
+    uint8_t* const part = reinterpret_cast<uint8_t*>(p.part_o);
+    auto piece_of = [&](int c_idx, int c) { return part + ((long long)c_idx * (D / 32) + c) * kPiece; };
+#pragma unroll 1
+    for (int c = 0; c < D / 32; ++c) {
+      float o[32];
+      if (ok && ntile > 0) {
+        tmem_ld32(o_col + c * 32, o);
+        tc_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) o[k] *= inv_l;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 32; ++k) o[k] = 0.f;
+      }
+      float amax = 0.f;
+#pragma unroll
+      for (int k = 0; k < 32; ++k) amax = fmaxf(amax, fabsf(o[k]));
+      const int ex = (__float_as_int(amax) >> 23) & 0xff;
+      const float scale = (amax > 0.f && ex < 254) ? __int_as_float((ex + 1) << 23) : 1.f;
+      const float inv = 1.f / scale;
+      uint32_t* dst = reinterpret_cast<uint32_t*>(smem + c * kPiece) + r;
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const __half2 h = __floats2half2_rn(o[2 * k] * inv, o[2 * k + 1] * inv);
+        dst[k * kTcRows] = *reinterpret_cast<const uint32_t*>(&h);
+      }
+      reinterpret_cast<float*>(smem + c * kPiece + kVals)[r] = scale;
+    }
     p.part_lse[(long long)cta * kTcRows + r] = lse;
     fence_proxy_async_smem();
     asm volatile("bar.sync 1, 256;" ::: "memory");
     if (threadIdx.x == 0) {
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) bulk_store(po + c * 32 * kTcRows, sbase + c * kPiece, kPiece);
+      bulk_store(piece_of(cta, 0), sbase, (D / 32) * kPiece);
       bulk_commit();
       bulk_wait_all();
       fence_proxy_async_all();
@@ -422,8 +429,8 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
       fence_proxy_async_all();
       const int c0 = p.work.base[req] + kvh * p.work.row_tiles + rt;   // CTA of split 0
       const int cstride = p.Hkv * p.work.row_tiles;
-      // merge weights exp(lse_s - max) of this row, one per split, in the last buffer
-      float* wt = stage + kRing * (kPiece / 4);
+      // merge weights exp(lse_s - max) of this row, one per split
+      float* wt = reinterpret_cast<float*>(smem + kWtsOff);
       float mx = -INFINITY;
       for (int sp = 0; sp < nsplit; ++sp)
         mx = fmaxf(mx, __ldcg(p.part_lse + (long long)(c0 + sp * cstride) * kTcRows + r));
@@ -435,19 +442,13 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
         wt[sp * kTcRows + r] = w;
       }
       const float inv_w = wsum > 0.f ? 1.f / wsum : 0.f;
-      // the other splits' pieces stream through the ring: piece i = (column
-      // block i / (nsplit-1), i-th other split); warp 0 issues the copies.
-      // Splits are summed in split order with the same arithmetic for the
-      // own chunk (tensor memory) as for the others, so the result does not
-      // depend on which CTA arrived last.
-      const int others = nsplit - 1, n_pieces = (D / 32) * others;
+      // piece i = (column block i / nsplit, split i % nsplit) streams through the
+      // ring of kRing buffers; warp 0 issues the copies
+      const int n_pieces = (D / 32) * nsplit;
       auto issue = [&](int i) {
-        const int t = i % others, sp = t < split ? t : t + 1;
         const int b = i % kRing;
         mbar_expect_tx(bar(B_MF + b), kPiece);
-        bulk_load(sbase + b * kPiece,
-                  p.part_o + (long long)(c0 + sp * cstride) * kTcRows * D + (long long)(i / others) * 32 * kTcRows,
-                  kPiece, bar(B_MF + b));
+        bulk_load(sbase + b * kPiece, piece_of(c0 + (i % nsplit) * cstride, i / nsplit), kPiece, bar(B_MF + b));
       };
       int issued = 0;
       if (warp == 0) {
@@ -459,31 +460,23 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
       bool mok = true;
 #pragma unroll 1
       for (int c = 0; mok && c < D / 32; ++c) {
-        float own[32], acc[32];
-        if (ntile > 0) {
-          tmem_ld32(o_col + c * 32, own);
-          tc_wait_ld();
-#pragma unroll
-          for (int k = 0; k < 32; ++k) own[k] = own[k] * inv_l;   // the value the other CTAs would read
-        } else {
-#pragma unroll
-          for (int k = 0; k < 32; ++k) own[k] = 0.f;
-        }
+        float acc[32];
 #pragma unroll
         for (int k = 0; k < 32; ++k) acc[k] = 0.f;
 #pragma unroll 1
         for (int sp = 0; sp < nsplit; ++sp) {
-          const float w = wt[sp * kTcRows + r];
-          if (sp == split) {
-#pragma unroll
-            for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w, own[k], acc[k]);
-            continue;
-          }
-          const int i = c * others + (sp < split ? sp : sp - 1), b = i % kRing;
+          const int i = c * nsplit + sp, b = i % kRing;
           if (!(mok = warp_wait(bar(B_MF + b), (i / kRing) & 1, abort_flag, p.wait_limit, p.status))) break;
-          const float* src = stage + b * (kPiece / 4) + r;
+          const uint8_t* pc = smem + b * kPiece;
+          const float wk = wt[sp * kTcRows + r] * reinterpret_cast<const float*>(pc + kVals)[r];
+          const uint32_t* src = reinterpret_cast<const uint32_t*>(pc) + r;
 #pragma unroll
-          for (int k = 0; k < 32; ++k) acc[k] = __fmaf_rn(w, src[k * kTcRows], acc[k]);
+          for (int k = 0; k < 16; ++k) {
+            const uint32_t bits = src[k * kTcRows];
+            const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&bits));
+            acc[2 * k] = __fmaf_rn(wk, f.x, acc[2 * k]);
+            acc[2 * k + 1] = __fmaf_rn(wk, f.y, acc[2 * k + 1]);
+          }
           __syncwarp();
           if (lane == 0) mbar_arrive(bar(B_ME + b));
           if (warp == 0 && i + kRing < n_pieces) {
@@ -492,7 +485,7 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
             ++issued;
           }
         }
-        if (mok && row_ok) store_row32o(c, acc, inv_w);
+        if (mok && row_ok) store_cols<D, 32>(p.out, orow, c * 32, acc, inv_w);
       }
       if (warp == 0 && !mok && lane == 0) {   // let the copies this CTA issued land
         for (int i = max(0, issued - kRing); i < issued; ++i)
