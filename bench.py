@@ -334,6 +334,30 @@ def run_ours(args, rank, world, local_rank):
                 lay_ms.append(e0.elapsed_time(e1))
             del g_lay
             lplan.free()
+    # the 131k-key layer's analogue: the same attention kernel on full causal
+    # attention over the whole assembled sequence (an empty plan: every token a
+    # query), i.e. the prefill the cached artifacts avoid; reported with the
+    # wall-time ratio full / cached
+    full_ms, full_flops, n_full = [], 0.0, 0
+    if args.workload == "qwen3_8b_long_131k":
+        n_full = wl.t_art(0) + wl.S_kv
+        gen = torch.Generator(device=dev).manual_seed(4)
+        qf = torch.randn(1, n_full, g.n_q_heads, g.head_dim, device=dev, dtype=torch.bfloat16, generator=gen)
+        kf = torch.randn(1, n_full, g.n_kv_heads, g.head_dim, device=dev, dtype=torch.bfloat16, generator=gen)
+        vf = torch.randn(1, n_full, g.n_kv_heads, g.head_dim, device=dev, dtype=torch.bfloat16, generator=gen)
+        of = torch.empty_like(qf)
+        fplan = ctx.assemble([[]])
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for i in range(5):
+            e0.record()
+            ctx.attend(fplan, qf, kf, vf, out=of, want_lse=False)
+            e1.record()
+            e1.synchronize()
+            if i >= 2:
+                full_ms.append(e0.elapsed_time(e1))
+        full_flops = 4.0 * g.head_dim * g.n_q_heads * n_full * (n_full + 1) / 2
+        fplan.free()
+        del qf, kf, vf, of
     total_ms = sum(step_ms)
     if world > 1:
         t = torch.tensor([total_ms], device=dev)
@@ -471,6 +495,10 @@ def run_ours(args, rank, world, local_rank):
                               "tflops": round(lay_flops / (statistics.mean(lay_ms) * 1e-3) / 1e12, 3),
                               "layout": "online system span 16, artifacts with 5-token online separators, task last"}
                              if lay_ms else None),
+        "full_causal_analogue": ({"tokens": n_full, "avg_call_ms": round(statistics.mean(full_ms), 3),
+                                  "tflops": round(full_flops / (statistics.mean(full_ms) * 1e-3) / 1e12, 3),
+                                  "wall_ratio_full_over_cached": round(statistics.mean(full_ms) / attn_avg_ms, 2)}
+                                 if full_ms else None),
         "kv_project": {"avg_call_ms": round(statistics.mean(kv_ms), 5),
                        "tflops": round(kv_flops / (statistics.mean(kv_ms) * 1e-3) / 1e12, 3)},
         "qproj": {"avg_call_ms": round(statistics.mean(qproj_ms), 5),
