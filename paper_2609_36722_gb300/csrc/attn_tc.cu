@@ -542,7 +542,7 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
   const int pool_rows = p.plan.pool_blocks * p.Hkv * kBlockTokens;
 
   // ---- slots of this chunk: >0 artifact block, <0 online chunk, 0 none
-  for (int i = threadIdx.x; i < 2 * ntile; i += blockDim.x) {
+  auto slot_entry = [&](int i) {
     int e = 0;
     if (i < nblk) {
       const int b = b0 + i;
@@ -558,14 +558,42 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
         e = online_entry(o_rows + (b - nab) * kBlockTokens, kBlockTokens);
       }
     }
-    list[i] = e;
-  }
-  if (threadIdx.x == 0) {
+    return e;
+  };
+  constexpr uint32_t tile_bytes = 2 * L::NH * (kBlockTokens * 128);
+  // The producer thread initialises the barriers and starts the first K tile
+  // and Q before the block's first barrier, so their loads overlap the slot
+  // list, the TMEM allocation and the first fetches of the other roles' code.
+  if (warp == kProducerWarp && lane == 0) {
     for (int i = 0; i < B_COUNT; ++i)
       mbar_init(bar(i), (i == B_PF || i == B_PF + 1) ? 4u : (i >= B_ME ? 8u : 1u));
     *abort_flag = 0;
     fence_mbar_init();
+    if (ntile > 0) {
+      tma_prefetch_desc(&p.tm_q);
+      tma_prefetch_desc(&p.tm_kpool);
+      tma_prefetch_desc(&p.tm_vpool);
+      const int e0 = slot_entry(0), e1 = slot_entry(1);
+      // Only kernels that never signal an early launch write the paged pool,
+      // so pool blocks may load while the previous kernel of the stream is
+      // still running; Q and suffix K/V wait for it.
+      if (e0 < 0 || e1 < 0) grid_dep_wait();
+      const uint32_t kd = sbase + L::K_OFF;
+      mbar_expect_tx(bar(B_KF), tile_bytes);
+      load_slot<D>(kd, e0, &p.tm_kpool, &p.tm_ksuf, bar(B_KF), kvh, p.Hkv, req, pool_rows);
+      load_slot<D>(kd + kBlockTokens * 128, e1, &p.tm_kpool, &p.tm_ksuf, bar(B_KF), kvh, p.Hkv, req, pool_rows);
+      grid_dep_wait();
+      mbar_expect_tx(bar(B_Q), 2 * L::NH * L::HALF);
+#pragma unroll
+      for (int qt = 0; qt < 2; ++qt) {
+#pragma unroll
+        for (int h = 0; h < L::NH; ++h)
+          tma_load_5d(sbase + L::Q_OFF + (qt * L::NH + h) * L::HALF, &p.tm_q, bar(B_Q), h * 64, 0, kvh,
+                      (row0 + qt * kTcTileRows) / G, req);
+      }
+    }
   }
+  for (int i = threadIdx.x; i < 2 * ntile; i += blockDim.x) list[i] = slot_entry(i);
   if (warp == kMmaWarp) {
     tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
     tmem_relinquish();
@@ -579,44 +607,22 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
   if (warp == kProducerWarp) {
     // ================= TMA producer =================
     if (lane == 0 && ntile > 0) {
-      tma_prefetch_desc(&p.tm_q);
-      tma_prefetch_desc(&p.tm_kpool);
-      tma_prefetch_desc(&p.tm_vpool);
-      // Only kernels that never signal an early launch write the paged pool,
-      // so its blocks of the first tile may load while the previous kernel of
-      // the stream is still running; Q and suffix K/V wait for it.
-      bool dep_done = false;
-      auto dep = [&]() {
-        if (!dep_done) grid_dep_wait();
-        dep_done = true;
-      };
-      auto load_q = [&]() {
-        dep();
-        mbar_expect_tx(bar(B_Q), 2 * L::NH * L::HALF);
-#pragma unroll
-        for (int qt = 0; qt < 2; ++qt) {
-#pragma unroll
-          for (int h = 0; h < L::NH; ++h)
-            tma_load_5d(sbase + L::Q_OFF + (qt * L::NH + h) * L::HALF, &p.tm_q, bar(B_Q), h * 64, 0, kvh,
-                        (row0 + qt * kTcTileRows) / G, req);
-        }
-      };
-      int issued_k = 0, issued_v = 0;
-      constexpr uint32_t tile_bytes = 2 * L::NH * (kBlockTokens * 128);
+      // K0 and Q are in flight (issued before the block's first barrier)
+      int issued_k = 1, issued_v = 0;
       for (int j = 0; j < ntile; ++j) {
         const int st = j % L::NS;
         const int e0 = list[2 * j], e1 = list[2 * j + 1];
-        if (e0 < 0 || e1 < 0) dep();
-        if (j >= L::NS &&
-            !mbar_wait(bar(B_KE + st), ((j / L::NS) - 1) & 1, abort_flag, p.wait_limit, p.status))
-          break;
-        const uint32_t kd = sbase + L::K_OFF + st * L::NH * L::HALF;
-        mbar_expect_tx(bar(B_KF + st), tile_bytes);
-        load_slot<D>(kd, e0, &p.tm_kpool, &p.tm_ksuf, bar(B_KF + st), kvh, p.Hkv, req, pool_rows);
-        load_slot<D>(kd + kBlockTokens * 128, e1, &p.tm_kpool, &p.tm_ksuf, bar(B_KF + st), kvh,
-                     p.Hkv, req, pool_rows);
-        issued_k = j + 1;
-        if (j == 0) load_q();
+        if (j > 0) {
+          if (j >= L::NS &&
+              !mbar_wait(bar(B_KE + st), ((j / L::NS) - 1) & 1, abort_flag, p.wait_limit, p.status))
+            break;
+          const uint32_t kd = sbase + L::K_OFF + st * L::NH * L::HALF;
+          mbar_expect_tx(bar(B_KF + st), tile_bytes);
+          load_slot<D>(kd, e0, &p.tm_kpool, &p.tm_ksuf, bar(B_KF + st), kvh, p.Hkv, req, pool_rows);
+          load_slot<D>(kd + kBlockTokens * 128, e1, &p.tm_kpool, &p.tm_ksuf, bar(B_KF + st), kvh,
+                       p.Hkv, req, pool_rows);
+          issued_k = j + 1;
+        }
         if (j >= L::NS &&
             !mbar_wait(bar(B_VE + st), ((j / L::NS) - 1) & 1, abort_flag, p.wait_limit, p.status))
           break;
