@@ -291,7 +291,7 @@ def run_ours(args, rank, world, local_rank):
         attn_ms.append(ev_a.elapsed_time(ev_b))
         qproj_ms.append(ev_q.elapsed_time(ev_a))
     torch.cuda.synchronize()
-    # the suffix tokens' K/V projection (§8(f) row 2), its own line: same x,
+    # the suffix tokens' K/V projection, its own line: same x,
     # base k_proj / v_proj weights of the geometry, into scratch suffix buffers
     wk, wv, kn = make_kv_weights(g, 0, device=dev)
     sk_s, sv_s = wl.suffix_k.clone(), wl.suffix_v.clone()
@@ -303,7 +303,7 @@ def run_ours(args, rank, world, local_rank):
         e1.synchronize()
         kv_ms.append(e0.elapsed_time(e1))
     kv_flops = 2.0 * wl.n_req * wl.S * g.hidden * 2 * g.n_kv_heads * g.head_dim
-    # the paper's skills layout (§8(f) row 3): a 16-token online system span,
+    # the paper's skills layout: a 16-token online system span,
     # 5-token online separators between the artifacts, the rest of the online
     # rows (the task) last; every online row is a query (S = S_kv)
     lay_ms, lay_flops = [], 0.0
