@@ -46,6 +46,23 @@ def _peaks():
 # ---------------------------------------------------------------------------
 # work accounting (algorithmic, per step)
 # ---------------------------------------------------------------------------
+def max_over_ranks(x: float, world: int, device="cpu") -> float:
+    """The largest of every rank's value (the job is as slow as its slowest
+    replica); the identity on one rank.  `device` is where the collective's
+    buffer lives: the GPU under NCCL, the CPU under gloo."""
+    if world <= 1:
+        return x
+    import torch
+    t = torch.tensor([x], device=device, dtype=torch.float64)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(work_per_rank_step: float, world: int, steps: int, seconds: float) -> float:
+    """Whole-job throughput: the work all ranks did over the slowest rank's time."""
+    return work_per_rank_step * world * steps / seconds
+
+
 def attention_flops(wl) -> float:
     """4 d Hq per visible (query, key) pair: 2d for q.k and 2d for p.v."""
     g = wl.geom
@@ -359,10 +376,7 @@ def run_ours(args, rank, world, local_rank):
         fplan.free()
         del qf, kf, vf, of
     total_ms = sum(step_ms)
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, world, dev)
     clocks = sampler.stop() if sampler else None
     st = ctx.sync_status()
     if st != 0:
@@ -398,10 +412,7 @@ def run_ours(args, rank, world, local_rank):
         e2e_step()
         e2e_times.append(time.perf_counter() - t0)
     e2e_s = sum(e2e_times)
-    if world > 1:
-        t = torch.tensor([e2e_s], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks(e2e_s, world, dev)
     h2d = (x_h.numel() + sk_h.numel() + sv_h.numel()) * 2
     d2h = out_h.numel() * 2
 
@@ -455,17 +466,14 @@ def run_ours(args, rank, world, local_rank):
     if wctx.sync_status() != 0:
         raise RuntimeError("device status after the warm-cache steps")
     warm_s = sum(warm_times)
-    if world > 1:
-        t = torch.tensor([warm_s], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        warm_s = float(t.item())
+    warm_s = max_over_ranks(warm_s, world, dev)
     wctx.close()
 
     peaks = _peaks()
     work = kv_bytes(wl) if decode else attention_flops(wl)
     scale = 1e9 if decode else 1e12
     unit = "GB/s" if decode else "TFLOP/s"
-    value = work * world * args.steps / (total_ms * 1e-3) / scale
+    value = job_throughput(work, world, args.steps, total_ms * 1e-3) / scale
     attn_avg_ms = statistics.mean(attn_ms)
     achieved = work / (attn_avg_ms * 1e-3) / scale
     peak = peaks["hbm"] if decode else peaks["bf16"]
@@ -504,10 +512,10 @@ def run_ours(args, rank, world, local_rank):
         "qproj": {"avg_call_ms": round(statistics.mean(qproj_ms), 5),
                   "tflops": round(qproj_flops(wl) / (statistics.mean(qproj_ms) * 1e-3) / 1e12, 3),
                   "frac_of_bf16_peak": round(qproj_flops(wl) / (statistics.mean(qproj_ms) * 1e-3) / 1e12 / peaks["bf16"], 4)},
-        "e2e": {"value": round(work * world * args.steps / e2e_s / scale, 3), "unit": unit,
+        "e2e": {"value": round(job_throughput(work, world, args.steps, e2e_s) / scale, 3), "unit": unit,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "includes": "assemble (host block table + H2D), H2D of x and suffix K/V, query_attend, D2H of O"},
-        "e2e_warm_cache": {"value": round(work * world * args.steps / warm_s / scale, 3), "unit": unit,
+        "e2e_warm_cache": {"value": round(job_throughput(work, world, args.steps, warm_s) / scale, 3), "unit": unit,
                            "h2d_bytes_per_step": h2d + art_bytes, "d2h_bytes_per_step": d2h,
                            "artifact_load_ms": round(statistics.mean(load_ms), 4),
                            "artifact_load_gbs": round(art_bytes / (statistics.mean(load_ms) * 1e-3) / 1e9, 1),
