@@ -286,7 +286,9 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
  *                               1 independent CTAs merged through global memory
  *                               by the last one to finish, 2 one thread-block
  *                               cluster per row tile (2 or 4 chunks) merged
- *                               through distributed shared memory
+ *                               through distributed shared memory (global
+ *                               memory where such clusters cannot be
+ *                               co-resident on the device)
  *   ATTUNER_OPT_TEST_STUCK_WAIT see below */
 #define ATTUNER_OPT_PREFILL_KERNEL 1
 #define ATTUNER_OPT_SPLIT_BLOCKS   2

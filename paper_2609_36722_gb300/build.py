@@ -20,7 +20,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libattuner.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
-SOURCES = ["capi.cu", "prep.cu", "qproj.cu", "attn_tc.cu", "attn_mma.cu", "attend_static.cu"]
+SOURCES = ["capi.cu", "plan.cpp", "prep.cu", "qproj.cu", "attn_tc.cu", "attn_mma.cu", "attend_static.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE]
 
@@ -38,6 +38,10 @@ def _deps():
     return hdrs
 
 
+def _obj(src: str) -> str:
+    return os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
+
+
 def _stale(target: str, inputs) -> bool:
     if not os.path.exists(target):
         return True
@@ -52,7 +56,7 @@ def build(verbose: bool = False, ptxas_verbose: bool = False, force: bool = Fals
     jobs = []
     for src in SOURCES:
         s = os.path.join(CSRC, src)
-        o = os.path.join(BUILD, src.replace(".cu", ".o"))
+        o = _obj(src)
         if force or _stale(o, [s] + deps):
             cmd = [nvcc] + ARCH + FLAGS + (["-Xptxas", "-v"] if ptxas_verbose else []) + ["-c", s, "-o", o]
             jobs.append((src, cmd))
@@ -69,7 +73,7 @@ def build(verbose: bool = False, ptxas_verbose: bool = False, force: bool = Fals
                     sys.stderr.write(f"[build] {' '.join(cmd)}\n{r.stdout}{r.stderr}")
                 if r.returncode != 0:
                     raise RuntimeError(f"nvcc failed on {src}")
-    objs = [os.path.join(BUILD, s.replace(".cu", ".o")) for s in SOURCES]
+    objs = [_obj(s) for s in SOURCES]
     if force or jobs or _stale(LIB, objs):
         cmd = [nvcc] + ARCH + ["-shared", "-o", LIB] + objs
         r = subprocess.run(cmd, capture_output=True, text=True)

@@ -279,63 +279,15 @@ static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const 
                                     bool layout, attuner_plan** out) {
   CHECK_ARG(ctx != nullptr && out != nullptr, "ctx and out must not be NULL");
   *out = nullptr;
-  CHECK_ARG(n_req >= 1 && n_req <= kMaxReq, "n_req must be in [1, " + std::to_string(kMaxReq) + "]");
-  CHECK_ARG(offs != nullptr, "req_offsets_host must not be NULL");
-  CHECK_ARG(offs[0] == 0, "req_offsets_host[0] must be 0");
-  for (int i = 0; i < n_req; ++i) CHECK_ARG(offs[i + 1] >= offs[i], "req_offsets_host must be non-decreasing");
-  CHECK_ARG(offs[n_req] == 0 || ids != nullptr, "artifact_ids_host must not be NULL");
   attuner_plan* p = new attuner_plan();
-  p->n_req = n_req;
+  std::string err;
+  const attuner_status bs = build_plan_tables(ctx->arts, ids, offs, n_req, layout, *p, err);
+  if (bs != ATTUNER_OK) {
+    delete p;
+    return fail(bs, err);
+  }
   p->device = ctx->cfg.device;
   p->pool_blocks = ctx->cfg.pool_blocks;
-  p->req_off.assign(offs, offs + n_req + 1);
-  p->blk_off.push_back(0);
-  p->span_off.push_back(0);
-  for (int r = 0; r < n_req; ++r) {
-    long long t = 0, o = 0;
-    const int32_t first_slot = (int32_t)p->blocks.size();
-    for (int i = offs[r]; i < offs[r + 1]; ++i) {
-      const int a = ids[i];
-      if (a < 0 && layout) {
-        const long long n = -(long long)a;
-        p->spans.insert(p->spans.end(), {(int32_t)o, (int32_t)n, (int32_t)p->blocks.size() - first_slot, (int32_t)t});
-        for (long long c = 0; c < n; c += 64)
-          p->blocks.push_back(-((int32_t)(((o + c) << 7) | std::min<long long>(64, n - c)) + 1));
-        o += n;
-        if (o >= (1 << 22)) {
-          delete p;
-          return fail(ATTUNER_ERR_INVALID_ARG, "online rows of a request must be < 2^22");
-        }
-        continue;
-      }
-      if (a < 0 || a >= (int)ctx->arts.size()) {
-        delete p;
-        return fail(ATTUNER_ERR_UNKNOWN_ARTIFACT, "artifact id " + std::to_string(a) + " was never registered");
-      }
-      p->art_ids.push_back(a);
-      const Artifact& A = ctx->arts[a];
-      for (int b = 0; b < A.n_blocks; ++b)
-        p->blocks.push_back(((A.first_block + b) << 7) | std::min(64, A.L - 64 * b));
-      t += A.L;
-    }
-    if (t + o >= (1ll << 30)) {
-      delete p;
-      return fail(ATTUNER_ERR_INVALID_ARG, "assembled length of a request must be < 2^30 tokens");
-    }
-    p->blk_off.push_back((int32_t)p->blocks.size());
-    p->t_art.push_back((int32_t)t);
-    p->o_rows.push_back((int32_t)o);
-    p->span_off.push_back((int32_t)(p->spans.size() / 4));
-    p->max_o_rows = std::max(p->max_o_rows, (int32_t)o);
-  }
-  p->req_art_off.push_back(0);
-  {
-    int k = 0;
-    for (int r = 0; r < n_req; ++r) {
-      for (int i = offs[r]; i < offs[r + 1]; ++i) k += ids[i] >= 0;
-      p->req_art_off.push_back(k);
-    }
-  }
   p->arts = ctx->arts;
   attuner_status s = set_device(ctx);
   if (s != ATTUNER_OK) { delete p; return s; }
@@ -401,43 +353,10 @@ extern "C" attuner_status attuner_plan_export(const attuner_plan* p, int32_t* bl
                                               int32_t* index_map, int32_t* token_art, int32_t* token_off,
                                               int64_t* sizes) {
   CHECK_ARG(p != nullptr && sizes != nullptr, "plan and sizes_inout must not be NULL");
-  int64_t nb = 0;
-  for (int32_t e : p->blocks) nb += e > 0;   // artifact blocks (online chunks are not exported)
-  int64_t nt = 0;
-  for (int32_t t : p->t_art) nt += t;
-  CHECK_ARG(!block_table || sizes[0] >= nb, "block_table capacity too small");
-  CHECK_ARG(!valid_len || sizes[1] >= nb, "valid_len capacity too small");
-  CHECK_ARG(!index_map || sizes[2] >= nt, "index_map capacity too small");
-  CHECK_ARG(!token_art || sizes[3] >= nt, "token_art capacity too small");
-  CHECK_ARG(!token_off || sizes[4] >= nt, "token_off capacity too small");
-  {
-    int64_t i = 0;
-    for (int32_t e : p->blocks) {
-      if (e <= 0) continue;
-      if (block_table) block_table[i] = e >> 7;
-      if (valid_len) valid_len[i] = e & 127;
-      ++i;
-    }
-  }
-  int64_t t = 0;
-  for (int r = 0; r < p->n_req; ++r) {
-    for (int i = p->req_art_off[r]; i < p->req_art_off[r + 1]; ++i) {
-      const int a = p->art_ids[i];
-      const Artifact& A = p->arts[a];
-      for (int q = 0; q < A.L; ++q, ++t) {
-        if (index_map) index_map[t] = (A.first_block + q / 64) * 64 + q % 64;
-        if (token_art) token_art[t] = a;
-        if (token_off) token_off[t] = q;
-      }
-    }
-  }
-  sizes[0] = nb;
-  sizes[1] = nb;
-  sizes[2] = nt;
-  sizes[3] = nt;
-  sizes[4] = nt;
-  sizes[5] = p->n_req;
-  return ATTUNER_OK;
+  std::string err;
+  const attuner_status s = export_plan_tables(*p, p->arts, block_table, valid_len, index_map, token_art, token_off,
+                                              sizes, err);
+  return s == ATTUNER_OK ? s : fail(s, err);
 }
 
 extern "C" attuner_status attuner_plan_t_art(const attuner_plan* p, int32_t* t_art, int32_t n_req) {
@@ -698,110 +617,14 @@ void att::query_cluster_occupancy(attuner_ctx* ctx) {
 
 void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc,
                       WorkTable& w) {
-  const int G = ctx->cfg.n_q_heads / ctx->cfg.n_kv_heads, Hkv = ctx->cfg.n_kv_heads;
-  const int rows = tc ? kTcRows : kMmaRows;
-  const int row_tiles = (S * G + rows - 1) / rows;
-  // slots of request r: the plan's, then the chunks of its final online span
-  auto nslots = [&](int r) {
-    return plan->blk_off[r + 1] - plan->blk_off[r] + (S_kv - plan->o_rows[r] + 63) / 64;
-  };
-  long long total = 0;
-  int maxv = 0;
-  for (int r = 0; r < plan->n_req; ++r) {
-    const int nv = nslots(r);
-    total += (long long)nv * Hkv * row_tiles;
-    maxv = std::max(maxv, nv);
-  }
-  const long long units = (long long)plan->n_req * Hkv * row_tiles;
-  // Cluster mode (tcgen05 kernel): every row tile cut into ns (2 or 4)
-  // chunks, one cluster of ns CTAs per row tile.  Cost in 128-key tile times: waves of
-  // co-resident clusters x (largest chunk + ~4 tiles of prologue and epilogue
-  // + ~1 for the merge).
-  auto cluster_cost = [&](int ns) -> double {
-    const int maxc = ctx->tc_clusters[ns];
-    if (maxc <= 0) return 1e30;
-    const int chunk = (((maxv + ns - 1) / ns) + 1) & ~1;
-    if (chunk > kMaxChunkBlocks) return 1e30;
-    const long long waves = (units + maxc - 1) / maxc;
-    return (double)waves * (chunk / 2 + 5.0);
-  };
-  int cluster_ns = 0;
-  int chunk;
-  if (ctx->opt_split > 0) {
-    chunk = ctx->opt_split;
-    // a cluster merges 2 or 4 chunks (whole column blocks per CTA)
-    if (tc && ctx->opt_merge == 2 && maxv > chunk) {
-      cluster_ns = (maxv + chunk - 1) / chunk <= 2 ? 2 : 4;
-      if ((((maxv + cluster_ns - 1) / cluster_ns) + 1) / 2 * 2 > kMaxChunkBlocks) cluster_ns = 0;
-    }
-  } else if (tc) {
-    // Independent splits, one CTA per SM.  Cost of a chunk size = waves x
-    // (tiles per CTA + ~4 tiles for the prologue and epilogue + ~2 for the
-    // merge through global memory); pick the number of splits of the
-    // longest request that minimises it.
-    const int maxt = (maxv + 1) / 2;
-    double best = 1e30;
-    chunk = maxv;
-    if (ctx->opt_merge != 2) {
-      for (int sp = 1; sp <= kMaxSplits; ++sp) {
-        const int ct = (maxt + sp - 1) / sp;
-        long long ncta = 0;
-        for (int r = 0; r < plan->n_req; ++r) {
-          const int nv = nslots(r);
-          ncta += (long long)((nv + 2 * ct - 1) / (2 * ct)) * Hkv * row_tiles;
-        }
-        const long long waves = (ncta + ctx->num_sms - 1) / ctx->num_sms;
-        const double cost = (double)waves * (ct + 4.0 + (sp > 1 ? 2.0 : 0.0));
-        if (cost < best - 1e-9) {
-          best = cost;
-          chunk = 2 * ct;
-        }
-      }
-    }
-    if (ctx->opt_merge != 1) {
-      for (int ns = 2; ns <= 4; ns += 2) {   // a cluster merges 2 or 4 chunks
-        const double cost = cluster_cost(ns);
-        if (cost < best - 1e-9) {
-          best = cost;
-          cluster_ns = ns;
-        }
-      }
-    }
-  } else {
-    // decode: several small CTAs per SM keep the HBM queues full and balance
-    // requests of different lengths
-    const long long target = 8ll * ctx->num_sms;
-    chunk = (int)std::max<long long>(16, (total + target - 1) / target);
-  }
-  w.n_req = plan->n_req;
-  w.row_tiles = row_tiles;
-  if (cluster_ns > 0) {
-    w.cluster = cluster_ns;
-    w.chunk_blocks = 0;   // per request, ceil(blocks / cluster) rounded up to whole tiles
-    for (int r = 0; r < plan->n_req; ++r) {
-      w.base[r] = (int)(r * (long long)Hkv * row_tiles * cluster_ns);
-      w.nsplit[r] = cluster_ns;
-    }
-    w.n_cta = (int)(units * cluster_ns);
-    return;
-  }
-  w.cluster = 0;
-  chunk = std::min(chunk, kMaxChunkBlocks);
-  if (tc) {
-    // the kernel merges at most kMaxSplits chunks of one row tile
-    chunk = std::max(chunk, (maxv + kMaxSplits - 1) / kMaxSplits);
-    chunk = (chunk + 1) & ~1;   // whole 128-key tiles per split
-  }
-  w.chunk_blocks = chunk;
-  int base = 0;
-  for (int r = 0; r < plan->n_req; ++r) {
-    const int nv = nslots(r);
-    const int ns = (nv + chunk - 1) / chunk;
-    w.base[r] = base;
-    w.nsplit[r] = ns;
-    base += ns * Hkv * row_tiles;
-  }
-  w.n_cta = base;
+  SplitPolicy pol;
+  pol.n_q_heads = ctx->cfg.n_q_heads;
+  pol.n_kv_heads = ctx->cfg.n_kv_heads;
+  pol.num_sms = ctx->num_sms;
+  pol.opt_split = ctx->opt_split;
+  pol.opt_merge = ctx->opt_merge;
+  for (int i = 0; i < 9; ++i) pol.tc_clusters[i] = ctx->tc_clusters[i];
+  split_work(pol, *plan, S, S_kv, tc, w);
 }
 
 static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, const void* q,

@@ -11,35 +11,11 @@
 #include <stdint.h>
 
 #include "../../include/attuner.h"
+#include "plan.h"
 
 #define ATT_DEV __device__ __forceinline__
 
 namespace att {
-
-constexpr int kBlockTokens = ATTUNER_BLOCK_TOKENS;   // 64 tokens per paged block
-constexpr int kMaxReq = 512;                         // requests per launch (kernel-param tables)
-
-// ---------------------------------------------------------------------------
-// Work decomposition shared by the attention kernels (passed by value).
-// A request's KV sequence is a list of "virtual blocks": its artifact blocks
-// (from the plan's block table, runtime order) followed by ceil(S_kv/64)
-// suffix chunks.  Each CTA owns one (request, kv head, row tile) and a
-// contiguous range of virtual blocks (one split-KV chunk).
-// CTA index = base[req] + (split * n_kv_heads + kv_head) * row_tiles + row_tile
-// ---------------------------------------------------------------------------
-struct WorkTable {
-  int32_t n_req;
-  int32_t row_tiles;      // row tiles per (request, kv head)
-  int32_t chunk_blocks;   // virtual blocks per split
-  int32_t n_cta;
-  // tcgen05 kernel only: 0 = splits of a row tile are independent CTAs merged
-  // through global memory; > 0 = every row tile has exactly this many splits,
-  // launched as one thread-block cluster (split = rank in the cluster) and
-  // merged through distributed shared memory.
-  int32_t cluster;
-  int32_t base[kMaxReq];
-  int32_t nsplit[kMaxReq];
-};
 
 // Plan arrays on the device.
 // A request's virtual block list ("slots", assembled order): artifact blocks

@@ -23,11 +23,7 @@
     if (!(cond)) return att::fail(ATTUNER_ERR_INVALID_ARG, msg);   \
   } while (0)
 
-struct Artifact {
-  int32_t first_block;
-  int32_t L;
-  int32_t n_blocks;
-};
+using att::Artifact;
 
 struct attuner_ctx {
   attuner_config cfg{};
@@ -55,23 +51,12 @@ struct attuner_ctx {
   std::unordered_set<attuner_plan*> live_plans;
 };
 
-struct attuner_plan {
+// An assembled plan: the host tables (att::PlanTables) and their device copy.
+struct attuner_plan : att::PlanTables {
   attuner_ctx* ctx = nullptr;     // owner of d_buf's cache; null once the context is destroyed
   size_t d_cap = 0;               // bytes of d_buf
-  int32_t n_req = 0;
   int32_t device = 0;
   int32_t pool_blocks = 0;
-  std::vector<int32_t> req_off;   // CSR over the items given to assembly
-  std::vector<int32_t> req_art_off;   // CSR over art_ids
-  std::vector<int32_t> art_ids;   // artifact ids in prompt order
-  std::vector<int32_t> blk_off;   // CSR over blocks
-  std::vector<int32_t> blocks;    // (pool block << 7) | valid
-  std::vector<int32_t> t_art;
-  // prompt layouts with online spans between artifacts (attuner_assemble_layout):
-  std::vector<int32_t> o_rows;    // online rows of each request's explicit spans
-  std::vector<int32_t> span_off;  // CSR over spans
-  std::vector<int32_t> spans;     // 4 per span: online row0, rows, first slot, artifact tokens before
-  int32_t max_o_rows = 0;
   size_t spans_at = 0;            // int32 offset of spans in d_buf
   std::vector<Artifact> arts;     // snapshot of the registry entries used
   int32_t* d_buf = nullptr;       // blk_off | blocks | t_art | o_rows | span_off | spans

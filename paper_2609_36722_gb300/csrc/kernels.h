@@ -137,13 +137,4 @@ cudaError_t launch_attn_tc(const AttnParams& p, int D, cudaStream_t st);
 cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st);
 cudaError_t launch_combine(const CombineParams& p, cudaStream_t st);
 
-// rows per CTA of each attention kernel
-constexpr int kTcRows = 256;      // packed query rows per CTA of attn_tc (two tiles)
-constexpr int kTcTileRows = 128;  // rows per query tile (one MMA M)
-constexpr int kMmaRows = 16;
-// largest split chunk (virtual blocks) the kernels' shared-memory block list holds
-constexpr int kMaxChunkBlocks = 4096;
-// most split-KV chunks of one (request, KV head, row tile) in the tcgen05 kernel
-constexpr int kMaxSplits = 32;
-
 }  // namespace att

@@ -1,0 +1,223 @@
+// plan.cpp - host-only planning (see plan.h): request assembly into a block
+// table (the runtime-order concatenation of independently stored artifact
+// caches, Sec. 2.1) and the split-KV decomposition of an attention launch.
+#include "plan.h"
+
+#include <algorithm>
+
+namespace att {
+
+namespace {
+attuner_status bad(attuner_status s, std::string& err, const std::string& msg) {
+  err = msg;
+  return s;
+}
+}  // namespace
+
+attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_t* items, const int32_t* offs,
+                                 int32_t n_req, bool layout, PlanTables& t, std::string& err) {
+  if (n_req < 1 || n_req > kMaxReq)
+    return bad(ATTUNER_ERR_INVALID_ARG, err, "n_req must be in [1, " + std::to_string(kMaxReq) + "]");
+  if (offs == nullptr) return bad(ATTUNER_ERR_INVALID_ARG, err, "req_offsets_host must not be NULL");
+  if (offs[0] != 0) return bad(ATTUNER_ERR_INVALID_ARG, err, "req_offsets_host[0] must be 0");
+  for (int i = 0; i < n_req; ++i)
+    if (offs[i + 1] < offs[i]) return bad(ATTUNER_ERR_INVALID_ARG, err, "req_offsets_host must be non-decreasing");
+  if (offs[n_req] != 0 && items == nullptr)
+    return bad(ATTUNER_ERR_INVALID_ARG, err, "artifact_ids_host must not be NULL");
+  t = PlanTables();
+  t.n_req = n_req;
+  t.req_off.assign(offs, offs + n_req + 1);
+  t.blk_off.push_back(0);
+  t.span_off.push_back(0);
+  for (int r = 0; r < n_req; ++r) {
+    long long tok = 0, o = 0;
+    const int32_t first_slot = (int32_t)t.blocks.size();
+    for (int i = offs[r]; i < offs[r + 1]; ++i) {
+      const int a = items[i];
+      if (a < 0 && layout) {
+        const long long n = -(long long)a;
+        t.spans.insert(t.spans.end(), {(int32_t)o, (int32_t)n, (int32_t)t.blocks.size() - first_slot, (int32_t)tok});
+        for (long long c = 0; c < n; c += kBlockTokens)
+          t.blocks.push_back(-((int32_t)(((o + c) << 7) | std::min<long long>(kBlockTokens, n - c)) + 1));
+        o += n;
+        if (o >= (1 << 22)) return bad(ATTUNER_ERR_INVALID_ARG, err, "online rows of a request must be < 2^22");
+        continue;
+      }
+      if (a < 0 || a >= (int)arts.size())
+        return bad(ATTUNER_ERR_UNKNOWN_ARTIFACT, err, "artifact id " + std::to_string(a) + " was never registered");
+      t.art_ids.push_back(a);
+      const Artifact& A = arts[a];
+      for (int b = 0; b < A.n_blocks; ++b)
+        t.blocks.push_back(((A.first_block + b) << 7) | std::min(kBlockTokens, A.L - kBlockTokens * b));
+      tok += A.L;
+    }
+    if (tok + o >= (1ll << 30))
+      return bad(ATTUNER_ERR_INVALID_ARG, err, "assembled length of a request must be < 2^30 tokens");
+    t.blk_off.push_back((int32_t)t.blocks.size());
+    t.t_art.push_back((int32_t)tok);
+    t.o_rows.push_back((int32_t)o);
+    t.span_off.push_back((int32_t)(t.spans.size() / 4));
+    t.max_o_rows = std::max(t.max_o_rows, (int32_t)o);
+  }
+  t.req_art_off.push_back(0);
+  int k = 0;
+  for (int r = 0; r < n_req; ++r) {
+    for (int i = offs[r]; i < offs[r + 1]; ++i) k += items[i] >= 0;
+    t.req_art_off.push_back(k);
+  }
+  return ATTUNER_OK;
+}
+
+attuner_status export_plan_tables(const PlanTables& t, const std::vector<Artifact>& arts, int32_t* block_table,
+                                  int32_t* valid_len, int32_t* index_map, int32_t* token_art, int32_t* token_off,
+                                  int64_t* sizes, std::string& err) {
+  if (sizes == nullptr) return bad(ATTUNER_ERR_INVALID_ARG, err, "plan and sizes_inout must not be NULL");
+  int64_t nb = 0;
+  for (int32_t e : t.blocks) nb += e > 0;   // artifact blocks (online chunks are not exported)
+  int64_t nt = 0;
+  for (int32_t v : t.t_art) nt += v;
+  if (block_table && sizes[0] < nb) return bad(ATTUNER_ERR_INVALID_ARG, err, "block_table capacity too small");
+  if (valid_len && sizes[1] < nb) return bad(ATTUNER_ERR_INVALID_ARG, err, "valid_len capacity too small");
+  if (index_map && sizes[2] < nt) return bad(ATTUNER_ERR_INVALID_ARG, err, "index_map capacity too small");
+  if (token_art && sizes[3] < nt) return bad(ATTUNER_ERR_INVALID_ARG, err, "token_art capacity too small");
+  if (token_off && sizes[4] < nt) return bad(ATTUNER_ERR_INVALID_ARG, err, "token_off capacity too small");
+  {
+    int64_t i = 0;
+    for (int32_t e : t.blocks) {
+      if (e <= 0) continue;
+      if (block_table) block_table[i] = e >> 7;
+      if (valid_len) valid_len[i] = e & 127;
+      ++i;
+    }
+  }
+  int64_t tok = 0;
+  for (int r = 0; r < t.n_req; ++r) {
+    for (int i = t.req_art_off[r]; i < t.req_art_off[r + 1]; ++i) {
+      const int a = t.art_ids[i];
+      const Artifact& A = arts[a];
+      for (int q = 0; q < A.L; ++q, ++tok) {
+        if (index_map) index_map[tok] = (A.first_block + q / kBlockTokens) * kBlockTokens + q % kBlockTokens;
+        if (token_art) token_art[tok] = a;
+        if (token_off) token_off[tok] = q;
+      }
+    }
+  }
+  sizes[0] = nb;
+  sizes[1] = nb;
+  sizes[2] = nt;
+  sizes[3] = nt;
+  sizes[4] = nt;
+  sizes[5] = t.n_req;
+  return ATTUNER_OK;
+}
+
+void split_work(const SplitPolicy& pol, const PlanTables& t, int S, int S_kv, bool tc, WorkTable& w) {
+  const int G = pol.n_q_heads / pol.n_kv_heads, Hkv = pol.n_kv_heads;
+  const int rows = tc ? kTcRows : kMmaRows;
+  const int row_tiles = (S * G + rows - 1) / rows;
+  // slots of request r: the plan's, then the chunks of its final online span
+  auto nslots = [&](int r) {
+    return t.blk_off[r + 1] - t.blk_off[r] + (S_kv - t.o_rows[r] + kBlockTokens - 1) / kBlockTokens;
+  };
+  long long total = 0;
+  int maxv = 0;
+  for (int r = 0; r < t.n_req; ++r) {
+    const int nv = nslots(r);
+    total += (long long)nv * Hkv * row_tiles;
+    maxv = std::max(maxv, nv);
+  }
+  const long long units = (long long)t.n_req * Hkv * row_tiles;
+  // Cluster mode (tcgen05 kernel): every row tile cut into ns (2 or 4)
+  // chunks, one cluster of ns CTAs per row tile.  Cost in 128-key tile times: waves of
+  // co-resident clusters x (largest chunk + ~4 tiles of prologue and epilogue
+  // + ~1 for the merge).
+  auto cluster_cost = [&](int ns) -> double {
+    const int maxc = pol.tc_clusters[ns];
+    if (maxc <= 0) return 1e30;
+    const int chunk = (((maxv + ns - 1) / ns) + 1) & ~1;
+    if (chunk > kMaxChunkBlocks) return 1e30;
+    const long long waves = (units + maxc - 1) / maxc;
+    return (double)waves * (chunk / 2 + 5.0);
+  };
+  int cluster_ns = 0;
+  int chunk;
+  if (pol.opt_split > 0) {
+    chunk = pol.opt_split;
+    // a cluster merges 2 or 4 chunks (whole column blocks per CTA); where such
+    // clusters cannot be co-resident the chunks merge through global memory
+    if (tc && pol.opt_merge == 2 && maxv > chunk) {
+      cluster_ns = (maxv + chunk - 1) / chunk <= 2 ? 2 : 4;
+      if ((((maxv + cluster_ns - 1) / cluster_ns) + 1) / 2 * 2 > kMaxChunkBlocks || pol.tc_clusters[cluster_ns] <= 0)
+        cluster_ns = 0;
+    }
+  } else if (tc) {
+    // Independent splits, one CTA per SM.  Cost of a chunk size = waves x
+    // (tiles per CTA + ~4 tiles for the prologue and epilogue + ~2 for the
+    // merge through global memory); pick the number of splits of the
+    // longest request that minimises it.
+    const int maxt = (maxv + 1) / 2;
+    double best = 1e30;
+    chunk = maxv;
+    if (pol.opt_merge != 2) {
+      for (int sp = 1; sp <= kMaxSplits; ++sp) {
+        const int ct = (maxt + sp - 1) / sp;
+        long long ncta = 0;
+        for (int r = 0; r < t.n_req; ++r) {
+          const int nv = nslots(r);
+          ncta += (long long)((nv + 2 * ct - 1) / (2 * ct)) * Hkv * row_tiles;
+        }
+        const long long waves = (ncta + pol.num_sms - 1) / pol.num_sms;
+        const double cost = (double)waves * (ct + 4.0 + (sp > 1 ? 2.0 : 0.0));
+        if (cost < best - 1e-9) {
+          best = cost;
+          chunk = 2 * ct;
+        }
+      }
+    }
+    if (pol.opt_merge != 1) {
+      for (int ns = 2; ns <= 4; ns += 2) {   // a cluster merges 2 or 4 chunks
+        const double cost = cluster_cost(ns);
+        if (cost < best - 1e-9) {
+          best = cost;
+          cluster_ns = ns;
+        }
+      }
+    }
+  } else {
+    // decode: several small CTAs per SM keep the HBM queues full and balance
+    // requests of different lengths
+    const long long target = 8ll * pol.num_sms;
+    chunk = (int)std::max<long long>(16, (total + target - 1) / target);
+  }
+  w.n_req = t.n_req;
+  w.row_tiles = row_tiles;
+  if (cluster_ns > 0) {
+    w.cluster = cluster_ns;
+    w.chunk_blocks = 0;   // per request, ceil(blocks / cluster) rounded up to whole tiles
+    for (int r = 0; r < t.n_req; ++r) {
+      w.base[r] = (int)(r * (long long)Hkv * row_tiles * cluster_ns);
+      w.nsplit[r] = cluster_ns;
+    }
+    w.n_cta = (int)(units * cluster_ns);
+    return;
+  }
+  w.cluster = 0;
+  chunk = std::min(chunk, kMaxChunkBlocks);
+  if (tc) {
+    // the kernel merges at most kMaxSplits chunks of one row tile
+    chunk = std::max(chunk, (maxv + kMaxSplits - 1) / kMaxSplits);
+    chunk = (chunk + 1) & ~1;   // whole 128-key tiles per split
+  }
+  w.chunk_blocks = chunk;
+  int base = 0;
+  for (int r = 0; r < t.n_req; ++r) {
+    const int nv = nslots(r);
+    const int ns = (nv + chunk - 1) / chunk;
+    w.base[r] = base;
+    w.nsplit[r] = ns;
+    base += ns * Hkv * row_tiles;
+  }
+  w.n_cta = base;
+}
+
+}  // namespace att

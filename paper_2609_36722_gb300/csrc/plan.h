@@ -1,0 +1,101 @@
+// plan.h - host-only planning of the attention path (plain C++, no CUDA):
+// the block table of an assembled request list and the split-KV decomposition
+// of one attention launch.  Compiled into libattuner and, on its own, into the
+// CPU tests of this logic.
+#pragma once
+
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/attuner.h"
+
+namespace att {
+
+constexpr int kBlockTokens = ATTUNER_BLOCK_TOKENS;   // 64 tokens per paged block
+constexpr int kMaxReq = 512;                         // requests per launch (kernel-param tables)
+
+// rows per CTA of each attention kernel
+constexpr int kTcRows = 256;      // packed query rows per CTA of attn_tc (two tiles)
+constexpr int kTcTileRows = 128;  // rows per query tile (one MMA M)
+constexpr int kMmaRows = 16;
+// largest split chunk (virtual blocks) the kernels' shared-memory block list holds
+constexpr int kMaxChunkBlocks = 4096;
+// most split-KV chunks of one (request, KV head, row tile) in the tcgen05 kernel
+constexpr int kMaxSplits = 32;
+
+// ---------------------------------------------------------------------------
+// Work decomposition shared by the attention kernels (passed by value).
+// A request's KV sequence is a list of "virtual blocks": its artifact blocks
+// (from the plan's block table, runtime order) followed by ceil(S_kv/64)
+// suffix chunks.  Each CTA owns one (request, kv head, row tile) and a
+// contiguous range of virtual blocks (one split-KV chunk).
+// CTA index = base[req] + (split * n_kv_heads + kv_head) * row_tiles + row_tile
+// ---------------------------------------------------------------------------
+struct WorkTable {
+  int32_t n_req;
+  int32_t row_tiles;      // row tiles per (request, kv head)
+  int32_t chunk_blocks;   // virtual blocks per split
+  int32_t n_cta;
+  // tcgen05 kernel only: 0 = splits of a row tile are independent CTAs merged
+  // through global memory; > 0 = every row tile has exactly this many splits,
+  // launched as one thread-block cluster (split = rank in the cluster) and
+  // merged through distributed shared memory.
+  int32_t cluster;
+  int32_t base[kMaxReq];
+  int32_t nsplit[kMaxReq];
+};
+
+// A registered artifact: ceil(L/64) consecutive pool blocks from first_block
+// (local token p in block first_block + p/64, row p%64).
+struct Artifact {
+  int32_t first_block;
+  int32_t L;
+  int32_t n_blocks;
+};
+
+// The host side of an assembled plan.  Items >= 0 given to assembly are
+// artifact ids; items < 0 (prompt layouts only) are online spans of -item rows.
+struct PlanTables {
+  int32_t n_req = 0;
+  std::vector<int32_t> req_off;       // CSR over the items given to assembly
+  std::vector<int32_t> req_art_off;   // CSR over art_ids
+  std::vector<int32_t> art_ids;       // artifact ids in prompt order
+  std::vector<int32_t> blk_off;       // CSR over blocks
+  // slot entries in prompt order: artifact block (pool_block << 7 | valid) > 0,
+  // online chunk -((online_row0 << 7 | rows) + 1) < 0 (at most 64 rows)
+  std::vector<int32_t> blocks;
+  std::vector<int32_t> t_art;         // artifact tokens of each request
+  std::vector<int32_t> o_rows;        // online rows of each request's explicit spans
+  std::vector<int32_t> span_off;      // CSR over spans
+  std::vector<int32_t> spans;         // 4 per span: online row0, rows, first slot, artifact tokens before
+  int32_t max_o_rows = 0;
+};
+
+// Fills `t` from the request lists (items[offs[r] .. offs[r+1]) of request r)
+// against the registry `arts`.  Returns ATTUNER_OK, or an error status with
+// `err` set and `t` unspecified.
+attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_t* items, const int32_t* offs,
+                                 int32_t n_req, bool layout, PlanTables& t, std::string& err);
+
+// The artifact blocks and the token index map of a plan, as the public
+// attuner_plan_export describes them (sizes_inout: capacities in, counts out).
+attuner_status export_plan_tables(const PlanTables& t, const std::vector<Artifact>& arts, int32_t* block_table,
+                                  int32_t* valid_len, int32_t* index_map, int32_t* token_art, int32_t* token_off,
+                                  int64_t* sizes, std::string& err);
+
+// What the split-KV choice depends on besides the plan.
+struct SplitPolicy {
+  int32_t n_q_heads, n_kv_heads;
+  int32_t num_sms;
+  int32_t opt_split;          // virtual blocks per chunk, 0 = chosen here
+  int32_t opt_merge;          // 0 = chosen here, 1 = through global memory, 2 = cluster
+  int32_t tc_clusters[9];     // co-resident clusters of n tcgen05 CTAs (n = 2, 4)
+};
+
+// Split-KV decomposition of one attention launch over S query rows and S_kv
+// online rows per request (tc: the tcgen05 kernel, else the warp-MMA kernel).
+void split_work(const SplitPolicy& pol, const PlanTables& t, int S, int S_kv, bool tc, WorkTable& w);
+
+}  // namespace att

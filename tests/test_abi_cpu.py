@@ -74,7 +74,7 @@ def test_product_path_does_not_import_oracle():
     pkg_dir = os.path.join(ROOT, "paper_2609_36722_gb300")
     for dirpath, _, files in os.walk(pkg_dir):
         for f in files:
-            if f.endswith((".py", ".cu", ".cuh", ".h")):
+            if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp")):
                 with open(os.path.join(dirpath, f)) as fh:
                     src = fh.read()
                 assert not re.search(r"^\s*(import|from)\s+oracle\b", src, re.M), f

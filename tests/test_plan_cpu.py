@@ -1,0 +1,366 @@
+"""Host planning logic of the library on the CPU: request assembly (block tables,
+index maps, prompt layouts with online spans) and the split-KV decomposition of
+an attention launch.
+
+The library's own planning source (csrc/plan.cpp) is compiled here with the host
+compiler alone, behind a small C shim (tests/plan_shim.cpp), so the code that
+runs inside `attuner_assemble`, `attuner_assemble_layout`, `attuner_plan_export`
+and every attention launch is checked without a GPU: block tables and index maps
+bit-exact against the oracle's storage rule (Sec. 2.1: independently stored
+artifact caches concatenated in runtime order), online positions against the
+oracle's prompt-layout positions, and the work table against the CTA mapping the
+kernels decode (every virtual block of every (request, KV head, row tile) in
+exactly one split, every CTA index used once).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import shutil
+import subprocess
+
+import numpy as np
+import pytest
+
+from oracle import attuner_oracle as orc
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+CSRC = os.path.join(ROOT, "paper_2609_36722_gb300", "csrc")
+BUILD = os.path.join(ROOT, "tests", "_build")
+
+OK, ERR_ARG, ERR_UNKNOWN = 0, -1, -3
+K_MAX_SPLITS, K_MAX_CHUNK, K_MAX_REQ = 32, 4096, 512
+I32P = ctypes.POINTER(ctypes.c_int32)
+I64P = ctypes.POINTER(ctypes.c_int64)
+
+
+@pytest.fixture(scope="module")
+def shim():
+    cxx = shutil.which("g++") or shutil.which("c++")
+    if cxx is None:
+        pytest.skip("no host C++ compiler")
+    os.makedirs(BUILD, exist_ok=True)
+    lib = os.path.join(BUILD, "libplan_shim.so")
+    cmd = [cxx, "-std=c++17", "-O1", "-shared", "-fPIC", "-Wall", "-Werror",
+           "-I", CSRC, os.path.join(ROOT, "tests", "plan_shim.cpp"), os.path.join(CSRC, "plan.cpp"), "-o", lib]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    h = ctypes.CDLL(lib)
+    h.shim_last_error.restype = ctypes.c_char_p
+    return h
+
+
+def _i32(a):
+    a = np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+    return a, a.ctypes.data_as(I32P)
+
+
+def bump_firsts(lengths):
+    """Bump allocation in registration order (the pool writer's rule)."""
+    first, nxt = [], 0
+    for L in lengths:
+        first.append(nxt)
+        nxt += -(-L // 64)
+    return first
+
+
+def assemble(shim, lengths, requests, layout=False, firsts=None):
+    """Tables of a plan over `requests` (lists of items); returns (status, dict)."""
+    firsts = bump_firsts(lengths) if firsts is None else firsts
+    n_req = len(requests)
+    items = [it for r in requests for it in r]
+    offs = np.cumsum([0] + [len(r) for r in requests])
+    fa, fp = _i32(firsts)
+    la, lp = _i32(lengths)
+    ia, ip = _i32(items if items else [0])
+    oa, op = _i32(offs)
+    cap = 1 << 20
+    out = np.zeros(cap, dtype=np.int32)
+    lens = np.zeros(4, dtype=np.int64)
+    st = shim.shim_assemble(fp, lp, len(lengths), ip, op, n_req, int(layout), out.ctypes.data_as(I32P),
+                            ctypes.c_int64(cap), lens.ctypes.data_as(I64P))
+    if st != OK:
+        return st, None
+    nb, ns, na = int(lens[0]), int(lens[1]), int(lens[2])
+    sizes = [n_req + 1, nb, n_req, n_req, n_req + 1, ns, n_req + 1, na]
+    names = ["blk_off", "blocks", "t_art", "o_rows", "span_off", "spans", "req_art_off", "art_ids"]
+    t, at = {}, 0
+    for nm, sz in zip(names, sizes):
+        t[nm] = out[at:at + sz].copy()
+        at += sz
+    t["max_o_rows"] = int(lens[3])
+    return st, t
+
+
+def export(shim, lengths, requests, layout=False, caps=None):
+    firsts = bump_firsts(lengths)
+    n_req = len(requests)
+    items = [it for r in requests for it in r]
+    offs = np.cumsum([0] + [len(r) for r in requests])
+    fa, fp = _i32(firsts)
+    la, lp = _i32(lengths)
+    ia, ip = _i32(items if items else [0])
+    oa, op = _i32(offs)
+    n = 1 << 18
+    bufs = [np.full(n, -7, dtype=np.int32) for _ in range(5)]
+    sizes = np.array(caps if caps is not None else [n] * 5 + [0], dtype=np.int64)
+    st = shim.shim_export(fp, lp, len(lengths), ip, op, n_req, int(layout),
+                          *[b.ctypes.data_as(I32P) for b in bufs], sizes.ctypes.data_as(I64P))
+    return st, bufs, sizes
+
+
+# ---------------------------------------------------------------------------
+# assembly
+# ---------------------------------------------------------------------------
+def _random_registry(rng, n):
+    # lengths across block boundaries: 1, 63, 64, 65, 128 ... and random
+    special = [1, 63, 64, 65, 127, 128, 129]
+    return [int(special[i]) if i < len(special) and rng.random() < 0.5 else int(rng.integers(1, 400))
+            for i in range(n)]
+
+
+def test_export_matches_oracle_storage_rule(shim):
+    rng = np.random.default_rng(11)
+    for trial in range(40):
+        lengths = _random_registry(rng, int(rng.integers(1, 9)))
+        n_req = int(rng.integers(1, 6))
+        # runtime order, repeats allowed, empty requests allowed
+        requests = [[int(a) for a in rng.integers(0, len(lengths), size=int(rng.integers(0, 6)))]
+                    for _ in range(n_req)]
+        st, bufs, sizes = export(shim, lengths, requests)
+        assert st == OK, shim.shim_last_error()
+        bt, vl, im, ta, to = bufs
+        nb, nt = int(sizes[0]), int(sizes[2])
+        want = {k: [] for k in ("block_table", "valid_len", "index_map", "token_art", "token_off")}
+        for req in requests:
+            ref = orc.assemble(lengths, req)
+            for k in want:
+                want[k].append(ref[k])
+        cat = {k: np.concatenate(v) if v else np.zeros(0, np.int32) for k, v in want.items()}
+        assert nb == len(cat["block_table"]) and nt == len(cat["index_map"])
+        assert sizes[5] == n_req
+        np.testing.assert_array_equal(bt[:nb], cat["block_table"])
+        np.testing.assert_array_equal(vl[:nb], cat["valid_len"])
+        np.testing.assert_array_equal(im[:nt], cat["index_map"])
+        np.testing.assert_array_equal(ta[:nt], cat["token_art"])
+        np.testing.assert_array_equal(to[:nt], cat["token_off"])
+        # nothing written past the counts
+        assert (bt[nb:nb + 4] == -7).all() and (im[nt:nt + 4] == -7).all()
+
+
+def test_plan_tables_of_artifact_lists(shim):
+    rng = np.random.default_rng(12)
+    for trial in range(30):
+        lengths = _random_registry(rng, int(rng.integers(1, 7)))
+        firsts = bump_firsts(lengths)
+        requests = [[int(a) for a in rng.integers(0, len(lengths), size=int(rng.integers(0, 5)))]
+                    for _ in range(int(rng.integers(1, 5)))]
+        st, t = assemble(shim, lengths, requests)
+        assert st == OK
+        assert t["max_o_rows"] == 0 and (t["o_rows"] == 0).all() and len(t["spans"]) == 0
+        for r, req in enumerate(requests):
+            ents = t["blocks"][t["blk_off"][r]:t["blk_off"][r + 1]]
+            want = [((firsts[a] + b) << 7) | min(64, lengths[a] - 64 * b)
+                    for a in req for b in range(-(-lengths[a] // 64))]
+            np.testing.assert_array_equal(ents, np.asarray(want, np.int32))
+            assert (ents > 0).all()
+            assert t["t_art"][r] == sum(lengths[a] for a in req)
+            ids = t["art_ids"][t["req_art_off"][r]:t["req_art_off"][r + 1]]
+            assert ids.tolist() == req
+
+
+def test_plan_tables_of_prompt_layouts(shim):
+    """Online spans between artifacts: slot entries, span records and the assembled
+    position of every online row against the oracle's layout positions."""
+    rng = np.random.default_rng(13)
+    for trial in range(40):
+        lengths = _random_registry(rng, int(rng.integers(1, 6)))
+        firsts = bump_firsts(lengths)
+        requests = []
+        for _ in range(int(rng.integers(1, 4))):
+            items = []
+            for _ in range(int(rng.integers(1, 7))):
+                if rng.random() < 0.4:
+                    items.append(-int(rng.choice([1, 5, 63, 64, 65, 130, int(rng.integers(1, 300))])))
+                else:
+                    items.append(int(rng.integers(0, len(lengths))))
+            requests.append(items)
+        st, t = assemble(shim, lengths, requests, layout=True)
+        assert st == OK, shim.shim_last_error()
+        for r, items in enumerate(requests):
+            ents = t["blocks"][t["blk_off"][r]:t["blk_off"][r + 1]].tolist()
+            spans = t["spans"][4 * t["span_off"][r]:4 * t["span_off"][r + 1]].reshape(-1, 4)
+            online = [-it for it in items if it < 0]
+            assert t["o_rows"][r] == sum(online)
+            assert len(spans) == len(online)
+            # walk the items in prompt order: slot entries and span records
+            slot, orow, tok, si = 0, 0, 0, 0
+            for it in items:
+                if it >= 0:
+                    L = lengths[it]
+                    for b in range(-(-L // 64)):
+                        assert ents[slot] == ((firsts[it] + b) << 7) | min(64, L - 64 * b)
+                        slot += 1
+                    tok += L
+                else:
+                    n = -it
+                    assert spans[si].tolist() == [orow, n, slot, tok]
+                    for c in range(0, n, 64):
+                        e = -ents[slot] - 1
+                        assert (e >> 7, e & 127) == (orow + c, min(64, n - c))
+                        slot += 1
+                    orow += n
+                    si += 1
+            assert slot == len(ents) and tok == t["t_art"][r]
+            # assembled positions: an online row sits after every artifact token and
+            # online row before it in the prompt (the oracle's layout rule)
+            S_kv = orow + 3
+            pos = orc.layout_online_positions(items, lengths, S_kv)
+            for row0, n, _, before in spans.tolist():
+                np.testing.assert_array_equal(pos[row0:row0 + n], before + row0 + np.arange(n))
+            # the rows after the explicit spans follow the whole prompt
+            assert pos[orow] == tok + orow
+        assert t["max_o_rows"] == max(t["o_rows"].tolist())
+
+
+def test_assembly_errors(shim):
+    lengths = [10, 70]
+    assert assemble(shim, lengths, [[0, 2]])[0] == ERR_UNKNOWN
+    assert assemble(shim, lengths, [[0, -5]])[0] == ERR_UNKNOWN          # online span outside a layout
+    assert assemble(shim, lengths, [[0, -5]], layout=True)[0] == OK
+    assert assemble(shim, lengths, [])[0] == ERR_ARG                      # n_req = 0
+    assert assemble(shim, lengths, [[0]] * (K_MAX_REQ + 1))[0] == ERR_ARG
+    assert assemble(shim, lengths, [[0]] * K_MAX_REQ)[0] == OK
+    assert assemble(shim, lengths, [[-(1 << 22)]], layout=True)[0] == ERR_ARG
+    assert assemble(shim, lengths, [[-((1 << 22) - 1)]], layout=True)[0] == OK
+
+    def raw(offs, n_req, items=(0,)):
+        fa, fp = _i32(bump_firsts(lengths))
+        la, lp = _i32(lengths)
+        ia, ip = _i32(list(items))
+        oa, op = _i32(offs)
+        out = np.zeros(1024, np.int32)
+        lens = np.zeros(4, np.int64)
+        return shim.shim_assemble(fp, lp, 2, ip, op, n_req, 0, out.ctypes.data_as(I32P), ctypes.c_int64(1024),
+                                  lens.ctypes.data_as(I64P))
+    assert raw([1, 1], 1) == ERR_ARG                                       # offs[0] != 0
+    assert raw([0, 1, 0], 2) == ERR_ARG                                    # decreasing offsets
+    assert raw([0, 1], 1) == OK
+
+
+def test_export_capacity_checks(shim):
+    lengths = [100, 30]
+    st, _, sizes = export(shim, lengths, [[0, 1]])
+    assert st == OK and sizes[:5].tolist() == [3, 3, 130, 130, 130]
+    for i, small in enumerate([2, 2, 129, 129, 129]):
+        caps = [1 << 18] * 5 + [0]
+        caps[i] = small
+        assert export(shim, lengths, [[0, 1]], caps=caps)[0] == ERR_ARG
+
+
+# ---------------------------------------------------------------------------
+# split-KV decomposition
+# ---------------------------------------------------------------------------
+def split(shim, n_q, n_kv, nv_art, o_rows, S, S_kv, tc, num_sms=152, opt_split=0, opt_merge=0,
+          clusters=(0, 0, 37, 0, 18, 0, 0, 0, 0)):
+    n_req = len(nv_art)
+    pol = _i32([n_q, n_kv, num_sms, opt_split, opt_merge] + list(clusters))
+    blk = _i32(np.cumsum([0] + list(nv_art)))
+    orow = _i32(o_rows)
+    out = np.zeros(5 + 2 * n_req, np.int32)
+    st = shim.shim_split(pol[1], blk[1], orow[1], n_req, S, S_kv, int(tc), out.ctypes.data_as(I32P))
+    assert st == OK
+    w = dict(n_req=int(out[0]), row_tiles=int(out[1]), chunk=int(out[2]), n_cta=int(out[3]), cluster=int(out[4]),
+             base=out[5:5 + n_req].tolist(), nsplit=out[5 + n_req:].tolist())
+    nv = [nv_art[r] + -(-(S_kv - o_rows[r]) // 64) for r in range(n_req)]
+    return w, nv
+
+
+def check_work(w, nv, n_kv, S, G, tc):
+    """The decomposition the kernels decode (CTA -> request, KV head, row tile,
+    split; split -> a range of virtual blocks) covers every block once."""
+    rows = 256 if tc else 16
+    assert w["row_tiles"] == -(-S * G // rows)
+    rt = w["row_tiles"]
+    if w["cluster"]:
+        ns = w["cluster"]
+        assert tc and ns in (2, 4)
+        assert w["n_cta"] == len(nv) * n_kv * rt * ns
+        for r, n in enumerate(nv):
+            chunk = ((-(-n // ns)) + 1) & ~1      # per request, whole 128-key tiles
+            assert chunk <= K_MAX_CHUNK and ns * chunk >= n
+            assert w["nsplit"][r] == ns and w["base"][r] == r * n_kv * rt * ns
+        return
+    chunk = w["chunk"]
+    assert chunk >= 1
+    if tc:
+        assert chunk % 2 == 0
+    seen = np.zeros(w["n_cta"], np.int32)
+    at = 0
+    for r, n in enumerate(nv):
+        ns = w["nsplit"][r]
+        assert w["base"][r] == at
+        assert ns == -(-n // chunk)                       # no empty split, nothing left over
+        if tc:
+            assert ns <= K_MAX_SPLITS
+        covered = np.zeros(n, np.int32)
+        for s in range(ns):
+            covered[s * chunk:min(n, (s + 1) * chunk)] += 1
+            for h in range(n_kv):
+                for t in range(rt):
+                    seen[w["base"][r] + (s * n_kv + h) * rt + t] += 1
+        assert (covered == 1).all()
+        at += ns * n_kv * rt
+    assert w["n_cta"] == at and (seen == 1).all()
+
+
+def test_split_work_covers_every_block_once(shim):
+    rng = np.random.default_rng(21)
+    for trial in range(300):
+        n_kv = int(rng.choice([1, 2, 4, 8]))
+        G = int(rng.choice([1, 2, 4, 8]))
+        n_req = int(rng.integers(1, 7))
+        tc = bool(rng.random() < 0.6)
+        S = int(rng.integers(1, 300)) if tc else int(rng.integers(1, 3))
+        nv_art = [int(rng.integers(0, 400)) for _ in range(n_req)]
+        o_rows = [int(rng.integers(0, 100)) if rng.random() < 0.3 else 0 for _ in range(n_req)]
+        S_kv = max(o_rows) + S + int(rng.integers(0, 64))
+        opt_merge = int(rng.integers(0, 3))
+        opt_split = int(rng.choice([0, 0, 2, 6, 64]))
+        clusters = (0, 0, int(rng.choice([0, 37, 76])), 0, int(rng.choice([0, 18, 38])), 0, 0, 0, 0)
+        w, nv = split(shim, G * n_kv, n_kv, nv_art, o_rows, S, S_kv, tc, num_sms=int(rng.choice([20, 148, 152])),
+                      opt_split=opt_split, opt_merge=opt_merge, clusters=clusters)
+        check_work(w, nv, n_kv, S, G, tc)
+        if opt_merge == 1 or not tc or not any(clusters):
+            assert w["cluster"] == 0
+        if not tc:
+            assert w["chunk"] >= (opt_split if opt_split else 16)
+
+
+def test_split_work_choices(shim):
+    # one long request on 152 SMs with 32 (KV head, row tile) units: split
+    w, nv = split(shim, 32, 8, [400], [0], 256, 256, True, opt_merge=1)
+    check_work(w, nv, 8, 256, 4, True)
+    assert w["nsplit"][0] > 1 and w["n_cta"] >= 152 // 2
+    # a short request is not split
+    w, nv = split(shim, 32, 8, [2], [0], 256, 256, True, opt_merge=1)
+    assert w["nsplit"][0] == 1
+    # merge option 2 with co-resident clusters: cluster mode
+    w, nv = split(shim, 32, 8, [400], [0], 256, 256, True, opt_merge=2)
+    check_work(w, nv, 8, 256, 4, True)
+    assert w["cluster"] in (2, 4)
+    # a fixed chunk: that many blocks per split (tcgen05: rounded to whole tiles)
+    w, nv = split(shim, 32, 8, [100, 37], [0, 0], 256, 256, True, opt_split=20, opt_merge=1)
+    assert w["chunk"] == 20 and w["nsplit"] == [-(-nv[0] // 20), -(-nv[1] // 20)]
+    # more blocks than 32 chunks of the fixed size hold: the chunk grows to 32 splits
+    w, nv = split(shim, 32, 8, [2000], [0], 256, 256, True, opt_split=4, opt_merge=1)
+    check_work(w, nv, 8, 256, 4, True)
+    assert w["nsplit"][0] == K_MAX_SPLITS
+    # decode: CTAs of at least 16 blocks, about 8 per SM
+    w, nv = split(shim, 32, 8, [700] * 64, [0] * 64, 1, 1, False)
+    check_work(w, nv, 8, 1, 4, False)
+    assert w["chunk"] >= 16 and w["n_cta"] >= 4 * 152
+    # the same inputs give the same table
+    a, _ = split(shim, 32, 8, [333, 12, 90], [0, 5, 0], 128, 200, True)
+    b, _ = split(shim, 32, 8, [333, 12, 90], [0, 5, 0], 128, 200, True)
+    assert a == b
