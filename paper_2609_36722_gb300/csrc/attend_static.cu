@@ -78,7 +78,7 @@ extern "C" attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const 
 
   AttnParams ap{};   // on the stack: this entry point touches no heap
   if (tc) query_cluster_occupancy(ctx);
-  make_work(ctx, plan, S, S_kv, tc, ap.work);
+  if ((e = make_work(ctx, plan, S, S_kv, tc, ap.work)) != ATTUNER_OK) return e;
   bool need_combine = false;   // split partial results in global memory
   for (int r = 0; r < plan->n_req; ++r) need_combine |= (ap.work.nsplit[r] > 1);
   if (ap.work.cluster > 0) need_combine = false;

@@ -615,8 +615,8 @@ void att::query_cluster_occupancy(attuner_ctx* ctx) {
     ctx->tc_clusters[ns] = (ns == 2 || ns == 4) ? attn_tc_max_clusters(ctx->cfg.head_dim, ns) : 0;
 }
 
-void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc,
-                      WorkTable& w) {
+attuner_status att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc,
+                              WorkTable& w) {
   SplitPolicy pol;
   pol.n_q_heads = ctx->cfg.n_q_heads;
   pol.n_kv_heads = ctx->cfg.n_kv_heads;
@@ -624,7 +624,9 @@ void att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int
   pol.opt_split = ctx->opt_split;
   pol.opt_merge = ctx->opt_merge;
   for (int i = 0; i < 9; ++i) pol.tc_clusters[i] = ctx->tc_clusters[i];
-  split_work(pol, *plan, S, S_kv, tc, w);
+  std::string err;
+  const attuner_status s = split_work(pol, *plan, S, S_kv, tc, w, err);
+  return s == ATTUNER_OK ? s : fail(s, err);
 }
 
 static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
@@ -642,7 +644,10 @@ static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, co
   else tc = (S * G > kMmaRows);
   WorkTable* w = new WorkTable();
   if (tc) query_cluster_occupancy(ctx);
-  make_work(ctx, plan, S, S_kv, tc, *w);
+  if (const attuner_status ws = make_work(ctx, plan, S, S_kv, tc, *w); ws != ATTUNER_OK) {
+    delete w;
+    return ws;
+  }
   bool need_combine = false;   // split partial results in global memory
   for (int r = 0; r < plan->n_req; ++r) need_combine |= (w->nsplit[r] > 1);
   if (w->cluster > 0) need_combine = false;

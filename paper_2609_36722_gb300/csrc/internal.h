@@ -78,7 +78,7 @@ bool aligned16(const void* p);
 PlanDev plan_dev(const attuner_plan* p);
 attuner_status check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv);
 // split-KV decomposition of one attention launch (tc: tcgen05 kernel, else warp-MMA kernel)
-void make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc, WorkTable& w);
+attuner_status make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc, WorkTable& w);
 // fills ctx->tc_clusters on first use (queries the device)
 void query_cluster_occupancy(attuner_ctx* ctx);
 

@@ -53,6 +53,8 @@ attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_
     }
     if (tok + o >= (1ll << 30))
       return bad(ATTUNER_ERR_INVALID_ARG, err, "assembled length of a request must be < 2^30 tokens");
+    if (t.blocks.size() >= (size_t)1 << 30)
+      return bad(ATTUNER_ERR_INVALID_ARG, err, "a plan must hold < 2^30 blocks in all");
     t.blk_off.push_back((int32_t)t.blocks.size());
     t.t_art.push_back((int32_t)tok);
     t.o_rows.push_back((int32_t)o);
@@ -111,7 +113,9 @@ attuner_status export_plan_tables(const PlanTables& t, const std::vector<Artifac
   return ATTUNER_OK;
 }
 
-void split_work(const SplitPolicy& pol, const PlanTables& t, int S, int S_kv, bool tc, WorkTable& w) {
+attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, int S_kv, bool tc, WorkTable& w,
+                          std::string& err) {
+  constexpr long long kMaxCta = 0x7fffffffll;
   const int G = pol.n_q_heads / pol.n_kv_heads, Hkv = pol.n_kv_heads;
   const int rows = tc ? kTcRows : kMmaRows;
   const int row_tiles = (S * G + rows - 1) / rows;
@@ -198,8 +202,9 @@ void split_work(const SplitPolicy& pol, const PlanTables& t, int S, int S_kv, bo
       w.base[r] = (int)(r * (long long)Hkv * row_tiles * cluster_ns);
       w.nsplit[r] = cluster_ns;
     }
+    if (units * cluster_ns > kMaxCta) return bad(ATTUNER_ERR_INVALID_ARG, err, "attention launch needs >= 2^31 CTAs");
     w.n_cta = (int)(units * cluster_ns);
-    return;
+    return ATTUNER_OK;
   }
   w.cluster = 0;
   chunk = std::min(chunk, kMaxChunkBlocks);
@@ -209,15 +214,18 @@ void split_work(const SplitPolicy& pol, const PlanTables& t, int S, int S_kv, bo
     chunk = (chunk + 1) & ~1;   // whole 128-key tiles per split
   }
   w.chunk_blocks = chunk;
-  int base = 0;
+  long long base = 0;
   for (int r = 0; r < t.n_req; ++r) {
     const int nv = nslots(r);
     const int ns = (nv + chunk - 1) / chunk;
-    w.base[r] = base;
+    w.base[r] = (int32_t)base;
     w.nsplit[r] = ns;
-    base += ns * Hkv * row_tiles;
+    base += (long long)ns * Hkv * row_tiles;
+    if (base > kMaxCta)
+      return bad(ATTUNER_ERR_INVALID_ARG, err, "attention launch needs >= 2^31 CTAs (use larger split chunks)");
   }
-  w.n_cta = base;
+  w.n_cta = (int32_t)base;
+  return ATTUNER_OK;
 }
 
 }  // namespace att

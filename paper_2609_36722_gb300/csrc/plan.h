@@ -96,6 +96,8 @@ struct SplitPolicy {
 
 // Split-KV decomposition of one attention launch over S query rows and S_kv
 // online rows per request (tc: the tcgen05 kernel, else the warp-MMA kernel).
-void split_work(const SplitPolicy& pol, const PlanTables& t, int S, int S_kv, bool tc, WorkTable& w);
+// Fails (INVALID_ARG, `err` set) only where the launch would need 2^31 or more CTAs.
+attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, int S_kv, bool tc, WorkTable& w,
+                          std::string& err);
 
 }  // namespace att

@@ -76,7 +76,8 @@ extern "C" int shim_split(const int32_t* pol, const int32_t* blk_off, const int3
   t.blk_off.assign(blk_off, blk_off + n_req + 1);
   t.o_rows.assign(o_rows, o_rows + n_req);
   att::WorkTable w;
-  att::split_work(p, t, S, S_kv, tc != 0, w);
+  const attuner_status s = att::split_work(p, t, S, S_kv, tc != 0, w, g_err);
+  if (s != ATTUNER_OK) return s;
   out[0] = w.n_req;
   out[1] = w.row_tiles;
   out[2] = w.chunk_blocks;

@@ -364,3 +364,18 @@ def test_split_work_choices(shim):
     a, _ = split(shim, 32, 8, [333, 12, 90], [0, 5, 0], 128, 200, True)
     b, _ = split(shim, 32, 8, [333, 12, 90], [0, 5, 0], 128, 200, True)
     assert a == b
+
+
+def test_split_work_rejects_a_launch_of_2_31_ctas(shim):
+    n_req = 512
+    pol = _i32([64, 8, 152, 1, 1] + [0] * 9)                 # one block per split (forced)
+    blk = _i32(np.arange(n_req + 1) * 20000)
+    orow = _i32([0] * n_req)
+    out = np.zeros(5 + 2 * n_req, np.int32)
+    # warp-MMA kernel: 32 row tiles x 8 KV heads x 512 requests x 20001 splits > 2^31
+    st = shim.shim_split(pol[1], blk[1], orow[1], n_req, 64, 64, 0, out.ctypes.data_as(I32P))
+    assert st == ERR_ARG and b"2^31" in shim.shim_last_error()
+    # the automatic chunk keeps the same plan well inside the limit
+    pol_auto = _i32([64, 8, 152, 0, 1] + [0] * 9)
+    st = shim.shim_split(pol_auto[1], blk[1], orow[1], n_req, 64, 64, 0, out.ctypes.data_as(I32P))
+    assert st == OK and 0 < out[3] < 1 << 31
