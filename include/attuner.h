@@ -94,7 +94,7 @@ attuner_status attuner_destroy(attuner_ctx* ctx);
  *   Blocks are handed out in registration order by a bump allocator:
  *   artifact j owns blocks first_j .. first_j + ceil(L_j/64) - 1 with
  *   first_j = sum_{i<j} ceil(L_i/64), and artifact ids are 0, 1, 2, ...
- * Errors: INVALID_ARG (L <= 0, NULL pointers), OOM (pool full). */
+ * Errors: INVALID_ARG (L outside [1, 2^30), NULL pointers), OOM (pool full). */
 attuner_status attuner_register_artifact(attuner_ctx* ctx, const void* k, const void* v,
                                          int32_t L, void* stream, int32_t* artifact_id_out);
 
@@ -105,7 +105,9 @@ attuner_status attuner_register_artifact(attuner_ctx* ctx, const void* k, const 
  * request then attends to its suffix only).  The plan holds, per request,
  * the block table (pool block, valid length) and the assembled index map
  * index_map[t] = block * 64 + slot for t in [0, T_art).  Synchronous: the
- * plan is on the device when the call returns.
+ * plan is on the device when the call returns.  A plan serves only the
+ * context that assembled it, and only until that context's next
+ * attuner_pool_reset: calls given another plan fail with INVALID_ARG.
  * Errors: INVALID_ARG, UNKNOWN_ARTIFACT, OOM, CUDA. */
 attuner_status attuner_assemble(attuner_ctx* ctx, const int32_t* artifact_ids_host,
                                 const int32_t* req_offsets_host, int32_t n_req,
@@ -249,7 +251,7 @@ attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, 
  *   ids_out[i]           : artifact ids, allocated as by
  *                          attuner_register_artifact, in order.
  *   1 <= n <= ATTUNER_MAX_HOST_BATCH.
- * Errors: INVALID_ARG (n out of range, L <= 0, NULL or unaligned pointers,
+ * Errors: INVALID_ARG (n out of range, L outside [1, 2^30), NULL or unaligned pointers,
  * memory that is not pinned host memory), OOM (pool full; nothing is
  * registered then). */
 #define ATTUNER_MAX_HOST_BATCH 64
@@ -259,8 +261,8 @@ attuner_status attuner_register_artifacts_host(attuner_ctx* ctx, int32_t n, cons
 
 /* Forget every registered artifact: the pool is empty again and the next
  * artifact gets id 0 and block 0 (a serving loop's eviction of the whole warm
- * set).  Plans made before must not be used afterwards, and the caller must
- * not reset while kernels that read the pool are still running. */
+ * set).  Plans made before are rejected afterwards (INVALID_ARG), and the
+ * caller must not reset while kernels that read the pool are still running. */
 attuner_status attuner_pool_reset(attuner_ctx* ctx);
 
 /* The paged pool: device base pointers of K and V ([pool_blocks][Hkv][64][d]

@@ -194,7 +194,7 @@ extern "C" attuner_status attuner_register_artifact(attuner_ctx* ctx, const void
                                                     int32_t L, void* stream, int32_t* artifact_id_out) {
   CHECK_ARG(ctx != nullptr, "ctx must not be NULL");
   CHECK_ARG(k != nullptr && v != nullptr, "k and v must not be NULL");
-  CHECK_ARG(L > 0, "artifact length L must be > 0");
+  CHECK_ARG(L > 0 && L < (1 << 30), "artifact length L must be in [1, 2^30)");
   CHECK_ARG(aligned16(k) && aligned16(v), "k and v must be 16-byte aligned");
   const int nb = (L + 63) / 64;
   if ((long long)ctx->used_blocks + nb > ctx->cfg.pool_blocks)
@@ -227,7 +227,8 @@ extern "C" attuner_status attuner_register_artifacts_host(attuner_ctx* ctx, int3
   const int Hkv = ctx->cfg.n_kv_heads, D = ctx->cfg.head_dim;
   long long blocks = 0, chunks = 0;
   for (int i = 0; i < n; ++i) {
-    if (L[i] <= 0) return done(fail(ATTUNER_ERR_INVALID_ARG, "artifact length L must be > 0"));
+    if (L[i] <= 0 || L[i] >= (1 << 30))
+      return done(fail(ATTUNER_ERR_INVALID_ARG, "artifact length L must be in [1, 2^30)"));
     if (!k_host[i] || !v_host[i] || !aligned16(k_host[i]) || !aligned16(v_host[i]))
       return done(fail(ATTUNER_ERR_INVALID_ARG, "k_host and v_host must be non-NULL and 16-byte aligned"));
     for (const void* ptr : {k_host[i], v_host[i]}) {
@@ -252,7 +253,10 @@ extern "C" attuner_status attuner_register_artifacts_host(attuner_ctx* ctx, int3
   b->n = n;
   b->Hkv = Hkv;
   b->D = D;
-  CUDA_TRY(launch_pool_write_host(*b, ctx->kpool, ctx->vpool, ctx->num_sms, static_cast<cudaStream_t>(stream)));
+  const cudaError_t ce = launch_pool_write_host(*b, ctx->kpool, ctx->vpool, ctx->num_sms,
+                                                static_cast<cudaStream_t>(stream));
+  if (ce != cudaSuccess)
+    return done(fail(ATTUNER_ERR_CUDA, std::string("pool write launch failed: ") + cudaGetErrorString(ce)));
   for (int i = 0; i < n; ++i) {
     ctx->arts.push_back(Artifact{b->first[i], L[i], (L[i] + 63) / 64});
     if (ids_out) ids_out[i] = (int32_t)ctx->arts.size() - 1;
@@ -266,6 +270,7 @@ extern "C" attuner_status attuner_pool_reset(attuner_ctx* ctx) {
   CHECK_ARG(ctx != nullptr, "ctx must not be NULL");
   ctx->arts.clear();
   ctx->used_blocks = 0;
+  ++ctx->pool_gen;
   ctx->last_launches = 0;
   return ATTUNER_OK;
 }
@@ -288,6 +293,7 @@ static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const 
   }
   p->device = ctx->cfg.device;
   p->pool_blocks = ctx->cfg.pool_blocks;
+  p->pool_gen = ctx->pool_gen;
   p->arts = ctx->arts;
   attuner_status s = set_device(ctx);
   if (s != ATTUNER_OK) { delete p; return s; }
@@ -407,8 +413,8 @@ PlanDev att::plan_dev(const attuner_plan* p) {
 // ---------------------------------------------------------------------------
 attuner_status att::check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv) {
   CHECK_ARG(ctx != nullptr && plan != nullptr, "ctx and plan must not be NULL");
-  CHECK_ARG(plan->device == ctx->cfg.device && plan->pool_blocks == ctx->cfg.pool_blocks,
-            "plan belongs to another context");
+  CHECK_ARG(plan->ctx == ctx, "plan belongs to another context");
+  CHECK_ARG(plan->pool_gen == ctx->pool_gen, "plan was assembled before the last attuner_pool_reset");
   CHECK_ARG(S >= 1 && S_kv >= S, "need 1 <= S <= S_kv");
   CHECK_ARG((long long)plan->n_req * S * ctx->cfg.n_q_heads < (1ll << 31) && S_kv < (1 << 22),
             "n_req * S * n_q_heads must be < 2^31 and S_kv < 2^22");

@@ -30,6 +30,7 @@ struct attuner_ctx {
   __nv_bfloat16* kpool = nullptr;
   __nv_bfloat16* vpool = nullptr;
   int32_t used_blocks = 0;
+  uint64_t pool_gen = 0;          // attuner_pool_reset calls so far (plans record it)
   std::vector<Artifact> arts;
   CUtensorMap tm_kpool{}, tm_vpool{};
   int* d_status = nullptr;
@@ -57,6 +58,7 @@ struct attuner_plan : att::PlanTables {
   size_t d_cap = 0;               // bytes of d_buf
   int32_t device = 0;
   int32_t pool_blocks = 0;
+  uint64_t pool_gen = 0;          // the context's pool generation at assembly
   size_t spans_at = 0;            // int32 offset of spans in d_buf
   std::vector<Artifact> arts;     // snapshot of the registry entries used
   int32_t* d_buf = nullptr;       // blk_off | blocks | t_art | o_rows | span_off | spans

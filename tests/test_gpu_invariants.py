@@ -108,6 +108,28 @@ def test_error_paths_leave_context_usable():
     assert torch.isfinite(out.float()).all()
 
 
+def test_plans_serve_only_their_context_and_pool_generation():
+    import paper_2609_36722_gb300 as pkg
+    wl = _wl()
+    ctx, plan = load_context(wl)
+    other, other_plan = load_context(wl)
+    # a plan of another context (same geometry, same pool) is refused before any launch
+    with pytest.raises(pkg.AttunerError) as e:
+        run_path(other, plan, wl)
+    assert e.value.status == pkg.attuner.ERR_INVALID_ARG
+    # after a reset the old plan is refused; one assembled afterwards works
+    ctx.pool_reset()
+    for k, v in zip(wl.art_k, wl.art_v):
+        ctx.register_artifact(k, v)
+    with pytest.raises(pkg.AttunerError) as e:
+        run_path(ctx, plan, wl)
+    assert e.value.status == pkg.attuner.ERR_INVALID_ARG
+    fresh = ctx.assemble(wl.requests)
+    out_a, _ = run_path(ctx, fresh, wl)
+    out_b, _ = run_path(other, other_plan, wl)
+    assert torch.equal(out_a.view(torch.int16), out_b.view(torch.int16))
+
+
 @pytest.mark.parametrize("merge", [1, 2])
 @pytest.mark.parametrize("S,S_kv", [(1, 129), (40, 48), (300, 300)])
 def test_repeated_calls_are_bit_identical(S, S_kv, merge):
