@@ -1,0 +1,251 @@
+"""Planted mistakes in the oracle, on the CPU.
+
+Each mutant replaces one oracle function with a plausible error -- a dropped
+term, a wrong sign, a wrong index or axis, an off-by-one position or mask, a
+transposed operand, a swapped output -- and the pins of test_oracle_pins.py
+are run against it: at least one must fail.  A mutant that no pin catches
+means a mistake of that kind could hide in the oracle, so the pins (not the
+mutant) would have to grow.  Nothing here touches the CUDA path.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import pytest
+
+from oracle import attuner_oracle as O
+import test_oracle_pins as pins
+
+ORIG = {n: getattr(O, n) for n in ("lora_q_projection", "merged_q_weight", "rms_norm_heads", "rope_rotate_half",
+                                  "query_positions", "kv_projection", "assemble", "attention", "request_forward",
+                                  "layout_online_positions", "layout_forward")}
+PINS = {n: f for n, f in vars(pins).items() if n.startswith("test_") and callable(f)}
+
+
+# --- Eq. query-adaptation and the merged form -------------------------------
+def lora_without_update(x, w_q, a, b, s):
+    return x @ w_q.T
+
+
+def lora_without_scale(x, w_q, a, b, s):
+    return ORIG["lora_q_projection"](x, w_q, a, b, 1.0)
+
+
+def lora_scale_on_base(x, w_q, a, b, s):
+    base = ORIG["lora_q_projection"](x, w_q, None, None, s)
+    return s * base + (ORIG["lora_q_projection"](x, w_q, a, b, s) - base)
+
+
+def merged_without_scale(w_q, a, b, s):
+    return w_q + b @ a
+
+
+def merged_transposed_update(w_q, a, b, s):
+    return w_q + s * (a.T @ b.T)                                     # (B A)^T
+
+
+# --- RMSNorm -----------------------------------------------------------------
+def rms_without_eps(q, w, eps):
+    return q / np.sqrt(np.mean(q * q, axis=-1, keepdims=True)) * w
+
+
+def rms_sum_not_mean(q, w, eps):
+    return q / np.sqrt(np.sum(q * q, axis=-1, keepdims=True) + eps) * w
+
+
+def rms_over_heads(q, w, eps):
+    return q / np.sqrt(np.mean(q * q, axis=-2, keepdims=True) + eps) * w
+
+
+def rms_without_weight(q, w, eps):
+    return ORIG["rms_norm_heads"](q, np.ones_like(w), eps)
+
+
+# --- RoPE --------------------------------------------------------------------
+def rope_wrong_sign(q, pos, theta):
+    return ORIG["rope_rotate_half"](q, -np.asarray(pos), theta)
+
+
+def rope_interleaved_pairs(q, pos, theta):
+    d = q.shape[-1]
+    perm = np.concatenate([np.arange(0, d, 2), np.arange(1, d, 2)])   # (2j, 2j+1) paired
+    inv = np.argsort(perm)
+    return ORIG["rope_rotate_half"](q[..., perm], pos, theta)[..., inv]
+
+
+def rope_half_frequency_exponent(q, pos, theta):
+    return ORIG["rope_rotate_half"](q, pos, theta ** 0.5)             # theta^(-j/d)
+
+
+def rope_position_plus_one(q, pos, theta):
+    return ORIG["rope_rotate_half"](q, np.asarray(pos) + 1, theta)
+
+
+# --- positions -----------------------------------------------------------------
+def qpos_off_by_one(t_art, S, S_kv):
+    return ORIG["query_positions"](t_art, S, S_kv) + 1
+
+
+def qpos_without_prior_suffix(t_art, S, S_kv):
+    return t_art + np.arange(S, dtype=np.int64)
+
+
+def layout_pos_ignoring_artifacts(items, art_lengths, S_kv):
+    return ORIG["layout_online_positions"](items, [0] * len(art_lengths), S_kv)
+
+
+def layout_pos_final_span_shifted(items, art_lengths, S_kv):
+    p = ORIG["layout_online_positions"](items, art_lengths, S_kv).copy()
+    p[sum(-it for it in items if it < 0):] += 1
+    return p
+
+
+# --- assembly ------------------------------------------------------------------
+def assemble_first_block_plus_one(art_lengths, request, block_tokens=64):
+    r = ORIG["assemble"](art_lengths, request, block_tokens)
+    r["block_table"] = r["block_table"] + 1
+    r["index_map"] = r["index_map"] + block_tokens
+    return r
+
+
+def assemble_block_and_slot_swapped(art_lengths, request, block_tokens=64):
+    r = ORIG["assemble"](art_lengths, request, block_tokens)
+    first = r["first_block"]
+    r["index_map"] = np.asarray([(first[a] + p % block_tokens) * block_tokens + p // block_tokens
+                                 for a in request for p in range(int(art_lengths[a]))], dtype=np.int32)
+    return r
+
+
+def assemble_valid_len_full_blocks(art_lengths, request, block_tokens=64):
+    r = ORIG["assemble"](art_lengths, request, block_tokens)
+    r["valid_len"] = np.full_like(r["valid_len"], block_tokens)
+    return r
+
+
+# --- attention -----------------------------------------------------------------
+def attention_without_scale(q, k, v, n_visible, pairs=None):
+    return ORIG["attention"](q * math.sqrt(q.shape[-1]), k, v, n_visible, pairs)
+
+
+def attention_mask_off_by_one(q, k, v, n_visible, pairs=None):
+    return ORIG["attention"](q, k, v, np.maximum(np.asarray(n_visible) - 1, 1), pairs)
+
+
+def attention_heads_modulo(q, k, v, n_visible, pairs=None):
+    Hq, Hkv = q.shape[1], k.shape[1]
+    idx = [h % Hkv for h in range(Hq)]                               # h % Hkv instead of h // G
+    return ORIG["attention"](q, k[:, idx], v[:, idx], n_visible, pairs)
+
+
+def attention_lse_base_two(q, k, v, n_visible, pairs=None):
+    o, lse = ORIG["attention"](q, k, v, n_visible, pairs)
+    return o, lse / math.log(2.0)
+
+
+def attention_swapped_kv(q, k, v, n_visible, pairs=None):
+    return ORIG["attention"](q, v, k, n_visible, pairs)
+
+
+# --- suffix K/V ----------------------------------------------------------------
+def kv_without_rope(x, w_k, w_v, k_norm_w, eps, theta, positions, n_kv_heads):
+    return ORIG["kv_projection"](x, w_k, w_v, k_norm_w, eps, theta, np.zeros_like(positions), n_kv_heads)
+
+
+def kv_value_normalised(x, w_k, w_v, k_norm_w, eps, theta, positions, n_kv_heads):
+    k, v = ORIG["kv_projection"](x, w_k, w_v, k_norm_w, eps, theta, positions, n_kv_heads)
+    return k, ORIG["rms_norm_heads"](v, np.ones(v.shape[-1]), eps)
+
+
+def kv_outputs_swapped(x, w_k, w_v, k_norm_w, eps, theta, positions, n_kv_heads):
+    k, v = ORIG["kv_projection"](x, w_k, w_v, k_norm_w, eps, theta, positions, n_kv_heads)
+    return v, k
+
+
+# --- one request -------------------------------------------------------------------
+def _request(x, w_q, a, b, s, q_norm_w, eps, theta, art_k, art_v, suffix_k, suffix_v, n_q_heads,
+             pairs=None, q_only=False, *, self_visible=1, causal=True, t_art_in_pos=True):
+    S, S_kv, d = x.shape[0], suffix_k.shape[0], suffix_k.shape[2]
+    t_art = int(sum(t.shape[0] for t in art_k))
+    q_raw = ORIG["lora_q_projection"](x, w_q, a, b, s).reshape(S, n_q_heads, d)
+    pos = ORIG["query_positions"](t_art if t_art_in_pos else 0, S, S_kv)
+    q = ORIG["rope_rotate_half"](ORIG["rms_norm_heads"](q_raw, q_norm_w, eps), pos, theta)
+    if q_only:
+        return q
+    k_all = np.concatenate(list(art_k) + [suffix_k], axis=0)
+    v_all = np.concatenate(list(art_v) + [suffix_v], axis=0)
+    n_vis = (t_art + (S_kv - S) + np.arange(S) + self_visible) if causal else np.full(S, t_art + S_kv)
+    return ORIG["attention"](q, k_all, v_all, np.maximum(n_vis, 1), pairs)
+
+
+def request_query_not_self_visible(*a, **kw):
+    return _request(*a, self_visible=0, **kw)
+
+
+def request_suffix_not_causal(*a, **kw):
+    return _request(*a, causal=False, **kw)
+
+
+def request_positions_without_artifacts(*a, **kw):
+    return _request(*a, t_art_in_pos=False, **kw)
+
+
+def layout_query_not_self_visible(x, w_q, a, b, s, q_norm_w, eps, theta, items, art_k, art_v, online_k, online_v,
+                                  n_q_heads, pairs=None):
+    # the layout forward with every query's mask one key short (its own key hidden)
+    real_attention = O.attention
+    try:
+        O.attention = lambda q, k, v, n_vis, p=None: ORIG["attention"](q, k, v, np.asarray(n_vis) - 1, p)
+        return ORIG["layout_forward"](x, w_q, a, b, s, q_norm_w, eps, theta, items, art_k, art_v, online_k,
+                                      online_v, n_q_heads, pairs)
+    finally:
+        O.attention = real_attention
+
+
+MUTANTS = [
+    ("lora_q_projection", lora_without_update), ("lora_q_projection", lora_without_scale),
+    ("lora_q_projection", lora_scale_on_base),
+    ("merged_q_weight", merged_without_scale), ("merged_q_weight", merged_transposed_update),
+    ("rms_norm_heads", rms_without_eps), ("rms_norm_heads", rms_sum_not_mean),
+    ("rms_norm_heads", rms_over_heads), ("rms_norm_heads", rms_without_weight),
+    ("rope_rotate_half", rope_wrong_sign), ("rope_rotate_half", rope_interleaved_pairs),
+    ("rope_rotate_half", rope_half_frequency_exponent), ("rope_rotate_half", rope_position_plus_one),
+    ("query_positions", qpos_off_by_one), ("query_positions", qpos_without_prior_suffix),
+    ("layout_online_positions", layout_pos_ignoring_artifacts),
+    ("layout_online_positions", layout_pos_final_span_shifted),
+    ("assemble", assemble_first_block_plus_one), ("assemble", assemble_block_and_slot_swapped),
+    ("assemble", assemble_valid_len_full_blocks),
+    ("attention", attention_without_scale), ("attention", attention_mask_off_by_one),
+    ("attention", attention_heads_modulo), ("attention", attention_lse_base_two),
+    ("attention", attention_swapped_kv),
+    ("kv_projection", kv_without_rope), ("kv_projection", kv_value_normalised),
+    ("kv_projection", kv_outputs_swapped),
+    ("request_forward", request_query_not_self_visible), ("request_forward", request_suffix_not_causal),
+    ("request_forward", request_positions_without_artifacts),
+    ("layout_forward", layout_query_not_self_visible),
+]
+
+
+def _pin_order(name):
+    # the pins that exercise the mutated function first (stop at the first failure)
+    key = {"lora_q_projection": "lora", "merged_q_weight": "merged", "rms_norm_heads": "rmsnorm",
+           "rope_rotate_half": "rope", "query_positions": "query_positions", "kv_projection": "kv_projection",
+           "assemble": "assemble", "attention": "attention", "request_forward": "artifact",
+           "layout_online_positions": "layout", "layout_forward": "layout"}[name]
+    names = sorted(PINS)
+    return [n for n in names if key in n] + [n for n in names if key not in n]
+
+
+@pytest.mark.parametrize("target,mutant", MUTANTS, ids=[m.__name__ for _, m in MUTANTS])
+def test_some_pin_catches_the_mutant(target, mutant, monkeypatch):
+    monkeypatch.setattr(O, target, mutant)
+    for name in _pin_order(target):
+        try:
+            PINS[name]()
+        except Exception:           # an assertion or a shape error: the pin caught it
+            return
+    pytest.fail(f"no pin fails when {target} is replaced by {mutant.__name__}")
+
+
+def test_every_oracle_function_has_a_mutant():
+    assert {t for t, _ in MUTANTS} == set(ORIG)
