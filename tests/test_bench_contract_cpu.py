@@ -1,0 +1,88 @@
+"""The benchmark's contract on the CPU: the reference arm's JSON line, and the
+algorithmic work the metric divides by, counted independently.
+
+The attention FLOPs are 4 d Hq per (query, key) pair the mask allows (2 d for
+q.k, 2 d for p.v); the decode bytes are each request's assembled K and V read
+once.  Both are checked here against a brute-force count of the visible pairs
+(the oracle's own mask rule, query i of S sees T_art + (S_kv - S) + i + 1 keys)
+and against the figure worked out for the tiny configuration (3 artifacts of
+37, 64, 100 tokens, 16 suffix tokens, d = 64, 4 query heads: 3.43 MFLOP).
+"""
+from __future__ import annotations
+
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+from gen import Geometry, make_custom, make_workload  # noqa: E402
+
+
+def _visible_pairs(wl):
+    n = 0
+    for r in range(wl.n_req):
+        t_art = wl.t_art(r)
+        for i in range(wl.S):
+            n += t_art + (wl.S_kv - wl.S) + i + 1
+    return n
+
+
+def test_tiny_attention_flops():
+    wl = make_workload("tiny")
+    assert _visible_pairs(wl) == 16 * 201 + 16 * 17 // 2
+    assert bench.attention_flops(wl) == 4 * 64 * 4 * (16 * 201 + 136) == 3_432_448
+
+
+def test_work_of_multi_request_decode_and_prefill_shapes():
+    g = Geometry(hidden=128, n_q_heads=8, n_kv_heads=2, head_dim=64, rank=8)
+    lengths = [70, 5, 130, 64]
+    reqs = [[0, 2], [], [3, 1, 3], [2]]
+    for S, S_kv in ((1, 9), (5, 5), (3, 40)):
+        wl = make_custom("c", g, 7, lengths, reqs, S, S_kv)
+        assert bench.attention_flops(wl) == 4 * 64 * 8 * _visible_pairs(wl)
+        # K and V, Hkv heads of d bf16 values, for every assembled and suffix token
+        toks = sum(sum(lengths[a] for a in r) + S_kv for r in reqs)
+        assert bench.kv_bytes(wl) == toks * 2 * 2 * 64 * 2
+        assert bench.is_decode(wl) == (S * g.group <= 16)
+
+
+def test_qproj_flops_counts_base_and_low_rank_products():
+    wl = make_workload("tiny")
+    g = wl.geom
+    M = wl.S
+    assert bench.qproj_flops(wl) == 2 * M * 256 * 256 + 2 * M * 256 * 8 + 2 * M * 8 * 256
+    assert g.d_q == 256 and g.rank == 8
+
+
+def test_reference_arm_line_keeps_the_contract():
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "tiny",
+                        "--steps", "2", "--warmup", "3"], capture_output=True, text=True, timeout=300, cwd=ROOT,
+                       env=dict(os.environ, RANK="0", WORLD_SIZE="1"))
+    assert r.returncode == 0, r.stderr
+    lines = [ln for ln in r.stdout.splitlines() if ln.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+              "vs_baseline", "dtype", "data", "impl", "config", "cpu_baseline", "e2e"):
+        assert k in d, k
+    assert d["impl"] == "reference" and d["unit"] == "TFLOP/s" and d["higher_is_better"] is True
+    assert d["steps"] == 2 and d["warmup"] == 3 and d["n_gpus"] == 1
+    assert d["config"]["workload"] == "tiny" and d["dtype"] == "f64"
+    assert d["value"] > 0 and d["cpu_baseline"]["value"] == d["value"] and d["e2e"]["value"] == d["value"]
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1 and d["cpu_baseline"]["sample"]
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
+    assert d["vs_baseline"] is None
+
+
+def test_warmup_below_three_is_raised_to_three():
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "tiny",
+                        "--steps", "1", "--warmup", "0"], capture_output=True, text=True, timeout=300, cwd=ROOT,
+                       env=dict(os.environ, RANK="0", WORLD_SIZE="1"))
+    assert r.returncode == 0, r.stderr
+    assert json.loads(r.stdout)["warmup"] == 3
