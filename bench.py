@@ -382,20 +382,36 @@ def run_ours(args, rank, world, local_rank):
     if st != 0:
         raise RuntimeError(f"device status {st} after the timed region")
 
-    # ---- end to end through the public API with host buffers
+    # ---- end to end through the public API with host buffers.  A step's inputs
+    # are its S new tokens: their hidden states and their own K/V rows (the last S
+    # of each request's S_kv suffix rows).  The S_kv - S earlier suffix rows of a
+    # decode step are the request's resident cache, written by earlier steps: they
+    # stay on the device, as the artifact pool does.
     x_h = wl.x.cpu().pin_memory()
-    sk_h = wl.suffix_k.cpu().pin_memory()
-    sv_h = wl.suffix_v.cpu().pin_memory()
+    S_old = wl.S_kv - wl.S
+    sk_h = wl.suffix_k[:, S_old:].cpu().contiguous().pin_memory()
+    sv_h = wl.suffix_v[:, S_old:].cpu().contiguous().pin_memory()
     out_h = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
     x_d = torch.empty_like(wl.x)
-    sk_d = torch.empty_like(wl.suffix_k)
-    sv_d = torch.empty_like(wl.suffix_v)
+    sk_d = wl.suffix_k.clone()
+    sv_d = wl.suffix_v.clone()
+    sk_new = torch.empty(sk_h.shape, dtype=sk_h.dtype, device=dev)
+    sv_new = torch.empty(sv_h.shape, dtype=sv_h.dtype, device=dev)
+
+    def copy_inputs():
+        x_d.copy_(x_h, non_blocking=True)
+        if S_old:
+            sk_new.copy_(sk_h, non_blocking=True)
+            sv_new.copy_(sv_h, non_blocking=True)
+            sk_d[:, S_old:].copy_(sk_new)
+            sv_d[:, S_old:].copy_(sv_new)
+        else:
+            sk_d.copy_(sk_h, non_blocking=True)
+            sv_d.copy_(sv_h, non_blocking=True)
 
     def e2e_step():
         p = ctx.assemble(wl.requests)
-        x_d.copy_(x_h, non_blocking=True)
-        sk_d.copy_(sk_h, non_blocking=True)
-        sv_d.copy_(sv_h, non_blocking=True)
+        copy_inputs()
         ctx.query_attend(p, x_d, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, sk_d, sv_d, out=out,
                          want_lse=False)
         out_h.copy_(out, non_blocking=True)
@@ -443,9 +459,7 @@ def run_ours(args, rank, world, local_rank):
     def warm_step():
         load_warm()
         p = wctx.assemble(reqs_w)
-        x_d.copy_(x_h, non_blocking=True)
-        sk_d.copy_(sk_h, non_blocking=True)
-        sv_d.copy_(sv_h, non_blocking=True)
+        copy_inputs()
         wctx.q_project(p, x_d, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv, out=q_w)
         stream.wait_stream(side)
         wctx.attend(p, q_w, sk_d, sv_d, out=out, want_lse=False)
@@ -514,14 +528,17 @@ def run_ours(args, rank, world, local_rank):
                   "frac_of_bf16_peak": round(qproj_flops(wl) / (statistics.mean(qproj_ms) * 1e-3) / 1e12 / peaks["bf16"], 4)},
         "e2e": {"value": round(job_throughput(work, world, args.steps, e2e_s) / scale, 3), "unit": unit,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "includes": "assemble (host block table + H2D), H2D of x and suffix K/V, query_attend, D2H of O"},
+                "includes": "assemble (host block table + H2D), H2D of the step's new tokens (x and their own "
+                            "suffix K/V rows; a decode step's earlier suffix rows stay resident), query_attend, "
+                            "D2H of O"},
         "e2e_warm_cache": {"value": round(job_throughput(work, world, args.steps, warm_s) / scale, 3), "unit": unit,
                            "h2d_bytes_per_step": h2d + art_bytes, "d2h_bytes_per_step": d2h,
                            "artifact_load_ms": round(statistics.mean(load_ms), 4),
                            "artifact_load_gbs": round(art_bytes / (statistics.mean(load_ms) * 1e-3) / 1e9, 1),
                            "includes": "pool reset, load of the requests' artifact K/V from pinned host memory "
                                        "(one kernel over the CPU-GPU link, second stream, overlapping the Q "
-                                       "projection), assemble, H2D of x and suffix K/V, Q projection, "
+                                       "projection), assemble, H2D of the step's new tokens (x and their "
+                                       "own suffix K/V rows), Q projection, "
                                        "attention, D2H of O"},
         "gpu_launches": launches,
         "clocks": clocks,
