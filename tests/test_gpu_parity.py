@@ -166,6 +166,31 @@ def test_decode_shape():
     compare(_np(out), o_ref, _np(lse), lse_ref, label="decode")
 
 
+@pytest.mark.parametrize("kernel,S,S_kv", [(2, 1, 9), (1, 8, 12)])
+def test_most_requests_per_call(kernel, S, S_kv):
+    # 512 requests, as many as one call takes (the kernels' per-request tables);
+    # ragged artifact lists, some empty, every request its own suffix
+    import paper_2609_36722_gb300 as pkg
+    rng = np.random.default_rng(29)
+    lengths = rng.integers(1, 200, size=16).tolist()
+    reqs = [rng.choice(16, size=int(rng.integers(0, 4)), replace=False).tolist() for _ in range(512)]
+    wl = make_custom("max_req", G128, 29, lengths, reqs, S, S_kv, device=DEV)
+    # the oracle per request, the shared weights and artifacts widened once
+    f, g = oracle.bf16_to_f64, wl.geom
+    w_q, a, b, qn = f(wl.w_q), f(wl.lora_a), f(wl.lora_b), f(wl.q_norm_w)
+    ak, av = [f(t) for t in wl.art_k], [f(t) for t in wl.art_v]
+    x, sk, sv = f(wl.x), f(wl.suffix_k), f(wl.suffix_v)
+    refs = [oracle.request_forward(x[r], w_q, a, b, g.scale, qn, g.rms_eps, g.rope_theta, [ak[i] for i in ids],
+                                   [av[i] for i in ids], sk[r], sv[r], g.n_q_heads) for r, ids in enumerate(reqs)]
+    o_ref, lse_ref = np.stack([o for o, _ in refs]), np.stack([l for _, l in refs])
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, kernel)
+    out, lse = run_path(ctx, plan, wl)
+    compare(_np(out), o_ref, _np(lse), lse_ref, label=f"512 requests kernel={kernel}")
+    with pytest.raises(pkg.AttunerError):
+        ctx.assemble(reqs + [[0]])
+
+
 @pytest.mark.parametrize("split_k", [2, 4])
 def test_q_project_split_k_matches_oracle(split_k):
     import paper_2609_36722_gb300 as pkg
