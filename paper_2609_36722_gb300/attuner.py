@@ -119,11 +119,13 @@ def _check(status: int):
         raise AttunerError(status, lib().attuner_last_error().decode())
 
 
-def _ptr(t: Optional[torch.Tensor], name: str, dtype=torch.bfloat16) -> Optional[int]:
+def _ptr(t: Optional[torch.Tensor], name: str, dtype=torch.bfloat16, device=None) -> Optional[int]:
     if t is None:
         return None
     if not t.is_cuda:
         raise ValueError(f"{name} must be a CUDA tensor")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, the context on {device}")
     if t.dtype != dtype:
         raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
     if not t.is_contiguous():
@@ -131,9 +133,12 @@ def _ptr(t: Optional[torch.Tensor], name: str, dtype=torch.bfloat16) -> Optional
     return t.data_ptr()
 
 
-def _stream(stream) -> Optional[int]:
+def _stream(stream, device=None) -> Optional[int]:
+    # the caller's stream, else the current stream of the context's device
     if stream is None:
-        stream = torch.cuda.current_stream()
+        stream = torch.cuda.current_stream(device)
+    elif device is not None and getattr(stream, "device", device) != device:
+        raise ValueError(f"stream is on {stream.device}, the context on {device}")
     return stream.cuda_stream
 
 
@@ -209,8 +214,8 @@ class Context:
         if k.shape != v.shape or k.dim() != 3:
             raise ValueError("k and v must both be [L, Hkv, d]")
         aid = ctypes.c_int32(-1)
-        _check(lib().attuner_register_artifact(self.handle, _ptr(k, "k"), _ptr(v, "v"), k.shape[0],
-                                               _stream(stream), ctypes.byref(aid)))
+        _check(lib().attuner_register_artifact(self.handle, self._p(k, "k"), self._p(v, "v"), k.shape[0],
+                                               self._s(stream), ctypes.byref(aid)))
         return aid.value
 
     def register_artifacts_host(self, ks: Sequence[torch.Tensor], vs: Sequence[torch.Tensor], stream=None) -> list:
@@ -227,15 +232,21 @@ class Context:
                 raise ValueError("each k, v must be bf16 [L, Hkv, d] of the same shape")
             if not (k.is_contiguous() and v.is_contiguous()):
                 raise ValueError("ks and vs must be contiguous")
-        kp = (_vp * n)(*[k.data_ptr() for k in ks])
-        vp = (_vp * n)(*[v.data_ptr() for v in vs])
+        kp = (_vp * n)(*[k.dataself._p() for k in ks])
+        vp = (_vp * n)(*[v.dataself._p() for v in vs])
         lens = (ctypes.c_int32 * n)(*[k.shape[0] for k in ks])
         ids = (ctypes.c_int32 * n)()
-        _check(lib().attuner_register_artifacts_host(self.handle, n, kp, vp, lens, _stream(stream), ids))
+        _check(lib().attuner_register_artifacts_host(self.handle, n, kp, vp, lens, self._s(stream), ids))
         return list(ids)
 
     def pool_reset(self) -> None:
         _check(lib().attuner_pool_reset(self.handle))
+
+    def _p(self, t, name, dtype=torch.bfloat16):
+        return _ptr(t, name, dtype, self.device)
+
+    def _s(self, stream):
+        return _stream(stream, self.device)
 
     @staticmethod
     def _csr(reqs):
@@ -275,9 +286,9 @@ class Context:
         r = 0 if lora_a is None else lora_a.shape[0]
         if out is None:
             out = torch.empty(n_req, S, self.cfg.n_q_heads, self.cfg.head_dim, dtype=torch.bfloat16, device=x.device)
-        _check(lib().attuner_q_project(self.handle, plan.handle, _ptr(x, "x"), _ptr(w_q, "w_q"),
-                                       _ptr(lora_a, "lora_a"), _ptr(lora_b, "lora_b"), r, float(s),
-                                       _ptr(q_norm_w, "q_norm_w"), S, S_kv, _ptr(out, "out"), _stream(stream)))
+        _check(lib().attuner_q_project(self.handle, plan.handle, self._p(x, "x"), self._p(w_q, "w_q"),
+                                       self._p(lora_a, "lora_a"), self._p(lora_b, "lora_b"), r, float(s),
+                                       self._p(q_norm_w, "q_norm_w"), S, S_kv, self._p(out, "out"), self._s(stream)))
         return out
 
     def kv_project(self, plan: Plan, x, w_k, w_v, k_norm_w, suffix_k, suffix_v, stream=None) -> None:
@@ -287,9 +298,9 @@ class Context:
         S_kv = suffix_k.shape[1]
         if suffix_k.shape != suffix_v.shape or suffix_k.shape[0] != n_req:
             raise ValueError("suffix_k and suffix_v must both be [n_req, S_kv, Hkv, d]")
-        _check(lib().attuner_kv_project(self.handle, plan.handle, _ptr(x, "x"), _ptr(w_k, "w_k"), _ptr(w_v, "w_v"),
-                                        _ptr(k_norm_w, "k_norm_w"), S, S_kv, _ptr(suffix_k, "suffix_k"),
-                                        _ptr(suffix_v, "suffix_v"), _stream(stream)))
+        _check(lib().attuner_kv_project(self.handle, plan.handle, self._p(x, "x"), self._p(w_k, "w_k"), self._p(w_v, "w_v"),
+                                        self._p(k_norm_w, "k_norm_w"), S, S_kv, self._p(suffix_k, "suffix_k"),
+                                        self._p(suffix_v, "suffix_v"), self._s(stream)))
 
     def attend(self, plan: Plan, q, suffix_k, suffix_v, out: Optional[torch.Tensor] = None,
                lse: Optional[torch.Tensor] = None, want_lse: bool = True, stream=None):
@@ -299,9 +310,9 @@ class Context:
             out = torch.empty_like(q)
         if lse is None and want_lse:
             lse = torch.empty(n_req, S, Hq, dtype=torch.float32, device=q.device)
-        _check(lib().attuner_attend(self.handle, plan.handle, _ptr(q, "q"), _ptr(suffix_k, "suffix_k"),
-                                    _ptr(suffix_v, "suffix_v"), S, S_kv, _ptr(out, "out"),
-                                    _ptr(lse, "lse", torch.float32), _stream(stream)))
+        _check(lib().attuner_attend(self.handle, plan.handle, self._p(q, "q"), self._p(suffix_k, "suffix_k"),
+                                    self._p(suffix_v, "suffix_v"), S, S_kv, self._p(out, "out"),
+                                    self._p(lse, "lse", torch.float32), self._s(stream)))
         return out, lse
 
     def attend_static_scratch(self, plan: Plan, q, suffix_k, suffix_v, out: Optional[torch.Tensor] = None,
@@ -313,10 +324,10 @@ class Context:
             out = torch.empty_like(q)
         if lse is None and want_lse:
             lse = torch.empty(n_req, S, Hq, dtype=torch.float32, device=q.device)
-        _check(lib().attuner_attend_static_scratch(self.handle, plan.handle, _ptr(q, "q"),
-                                                   _ptr(suffix_k, "suffix_k"), _ptr(suffix_v, "suffix_v"), S,
-                                                   S_kv, _ptr(out, "out"), _ptr(lse, "lse", torch.float32),
-                                                   _stream(stream)))
+        _check(lib().attuner_attend_static_scratch(self.handle, plan.handle, self._p(q, "q"),
+                                                   self._p(suffix_k, "suffix_k"), self._p(suffix_v, "suffix_v"), S,
+                                                   S_kv, self._p(out, "out"), self._p(lse, "lse", torch.float32),
+                                                   self._s(stream)))
         return out, lse
 
     def query_attend(self, plan: Plan, x, w_q, lora_a, lora_b, s: float, q_norm_w, suffix_k, suffix_v,
@@ -329,11 +340,11 @@ class Context:
             out = torch.empty(n_req, S, self.cfg.n_q_heads, self.cfg.head_dim, dtype=torch.bfloat16, device=x.device)
         if lse is None and want_lse:
             lse = torch.empty(n_req, S, self.cfg.n_q_heads, dtype=torch.float32, device=x.device)
-        _check(lib().attuner_query_attend(self.handle, plan.handle, _ptr(x, "x"), _ptr(w_q, "w_q"),
-                                          _ptr(lora_a, "lora_a"), _ptr(lora_b, "lora_b"), r, float(s),
-                                          _ptr(q_norm_w, "q_norm_w"), _ptr(suffix_k, "suffix_k"),
-                                          _ptr(suffix_v, "suffix_v"), S, S_kv, _ptr(out, "out"),
-                                          _ptr(lse, "lse", torch.float32), _stream(stream)))
+        _check(lib().attuner_query_attend(self.handle, plan.handle, self._p(x, "x"), self._p(w_q, "w_q"),
+                                          self._p(lora_a, "lora_a"), self._p(lora_b, "lora_b"), r, float(s),
+                                          self._p(q_norm_w, "q_norm_w"), self._p(suffix_k, "suffix_k"),
+                                          self._p(suffix_v, "suffix_v"), S, S_kv, self._p(out, "out"),
+                                          self._p(lse, "lse", torch.float32), self._s(stream)))
         return out, lse
 
     # --- misc
@@ -350,7 +361,7 @@ class Context:
 
     def sync_status(self, stream=None) -> int:
         """Synchronise and return the device status (0 = OK) without raising."""
-        return lib().attuner_sync_status(self.handle, _stream(stream))
+        return lib().attuner_sync_status(self.handle, self._s(stream))
 
     def set_option(self, option: int, value: int):
         _check(lib().attuner_set_option(self.handle, option, int(value)))
