@@ -294,7 +294,6 @@ static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const 
   p->device = ctx->cfg.device;
   p->pool_blocks = ctx->cfg.pool_blocks;
   p->pool_gen = ctx->pool_gen;
-  p->arts = ctx->arts;
   attuner_status s = set_device(ctx);
   if (s != ATTUNER_OK) { delete p; return s; }
   std::vector<int32_t> h;
@@ -360,8 +359,8 @@ extern "C" attuner_status attuner_plan_export(const attuner_plan* p, int32_t* bl
                                               int64_t* sizes) {
   CHECK_ARG(p != nullptr && sizes != nullptr, "plan and sizes_inout must not be NULL");
   std::string err;
-  const attuner_status s = export_plan_tables(*p, p->arts, block_table, valid_len, index_map, token_art, token_off,
-                                              sizes, err);
+  const attuner_status s = export_plan_tables(*p, block_table, valid_len, index_map, token_art, token_off, sizes,
+                                              err);
   return s == ATTUNER_OK ? s : fail(s, err);
 }
 

@@ -60,7 +60,6 @@ struct attuner_plan : att::PlanTables {
   int32_t pool_blocks = 0;
   uint64_t pool_gen = 0;          // the context's pool generation at assembly
   size_t spans_at = 0;            // int32 offset of spans in d_buf
-  std::vector<Artifact> arts;     // snapshot of the registry entries used
   int32_t* d_buf = nullptr;       // blk_off | blocks | t_art | o_rows | span_off | spans
 };
 

@@ -25,6 +25,22 @@ attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_
   if (offs[n_req] != 0 && items == nullptr)
     return bad(ATTUNER_ERR_INVALID_ARG, err, "artifact_ids_host must not be NULL");
   t = PlanTables();
+  {
+    // sizes first: the tables grow once
+    size_t nblk = 0, nids = 0;
+    for (int i = 0; i < offs[n_req]; ++i) {
+      const long long a = items[i];
+      if (a >= 0 && a < (long long)arts.size()) {
+        nblk += arts[a].n_blocks;
+        ++nids;
+      } else if (a < 0 && layout && -a < (1 << 22)) {
+        nblk += (-a + kBlockTokens - 1) / kBlockTokens;
+      }
+    }
+    t.blocks.reserve(nblk);
+    t.art_ids.reserve(nids);
+    t.art_used.reserve(nids);
+  }
   t.n_req = n_req;
   t.req_off.assign(offs, offs + n_req + 1);
   t.blk_off.push_back(0);
@@ -47,6 +63,7 @@ attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_
         return bad(ATTUNER_ERR_UNKNOWN_ARTIFACT, err, "artifact id " + std::to_string(a) + " was never registered");
       t.art_ids.push_back(a);
       const Artifact& A = arts[a];
+      t.art_used.push_back(A);
       for (int b = 0; b < A.n_blocks; ++b)
         t.blocks.push_back(((A.first_block + b) << 7) | std::min(kBlockTokens, A.L - kBlockTokens * b));
       tok += A.L;
@@ -70,9 +87,9 @@ attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_
   return ATTUNER_OK;
 }
 
-attuner_status export_plan_tables(const PlanTables& t, const std::vector<Artifact>& arts, int32_t* block_table,
-                                  int32_t* valid_len, int32_t* index_map, int32_t* token_art, int32_t* token_off,
-                                  int64_t* sizes, std::string& err) {
+attuner_status export_plan_tables(const PlanTables& t, int32_t* block_table, int32_t* valid_len,
+                                  int32_t* index_map, int32_t* token_art, int32_t* token_off, int64_t* sizes,
+                                  std::string& err) {
   if (sizes == nullptr) return bad(ATTUNER_ERR_INVALID_ARG, err, "plan and sizes_inout must not be NULL");
   int64_t nb = 0;
   for (int32_t e : t.blocks) nb += e > 0;   // artifact blocks (online chunks are not exported)
@@ -96,7 +113,7 @@ attuner_status export_plan_tables(const PlanTables& t, const std::vector<Artifac
   for (int r = 0; r < t.n_req; ++r) {
     for (int i = t.req_art_off[r]; i < t.req_art_off[r + 1]; ++i) {
       const int a = t.art_ids[i];
-      const Artifact& A = arts[a];
+      const Artifact& A = t.art_used[i];
       for (int q = 0; q < A.L; ++q, ++tok) {
         if (index_map) index_map[tok] = (A.first_block + q / kBlockTokens) * kBlockTokens + q % kBlockTokens;
         if (token_art) token_art[tok] = a;

@@ -62,6 +62,7 @@ struct PlanTables {
   std::vector<int32_t> req_off;       // CSR over the items given to assembly
   std::vector<int32_t> req_art_off;   // CSR over art_ids
   std::vector<int32_t> art_ids;       // artifact ids in prompt order
+  std::vector<Artifact> art_used;     // their registry entries (the plan's own copy)
   std::vector<int32_t> blk_off;       // CSR over blocks
   // slot entries in prompt order: artifact block (pool_block << 7 | valid) > 0,
   // online chunk -((online_row0 << 7 | rows) + 1) < 0 (at most 64 rows)
@@ -81,9 +82,9 @@ attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_
 
 // The artifact blocks and the token index map of a plan, as the public
 // attuner_plan_export describes them (sizes_inout: capacities in, counts out).
-attuner_status export_plan_tables(const PlanTables& t, const std::vector<Artifact>& arts, int32_t* block_table,
-                                  int32_t* valid_len, int32_t* index_map, int32_t* token_art, int32_t* token_off,
-                                  int64_t* sizes, std::string& err);
+attuner_status export_plan_tables(const PlanTables& t, int32_t* block_table, int32_t* valid_len,
+                                  int32_t* index_map, int32_t* token_art, int32_t* token_off, int64_t* sizes,
+                                  std::string& err);
 
 // What the split-KV choice depends on besides the plan.
 struct SplitPolicy {

@@ -54,7 +54,7 @@ extern "C" int shim_export(const int32_t* first, const int32_t* L, int32_t n_art
   att::PlanTables t;
   const attuner_status s = att::build_plan_tables(arts, items, offs, n_req, layout != 0, t, g_err);
   if (s != ATTUNER_OK) return s;
-  return att::export_plan_tables(t, arts, block_table, valid_len, index_map, token_art, token_off, sizes, g_err);
+  return att::export_plan_tables(t, block_table, valid_len, index_map, token_art, token_off, sizes, g_err);
 }
 
 // Split-KV decomposition of a launch over a plan given by its blk_off and
