@@ -86,3 +86,26 @@ def test_warmup_below_three_is_raised_to_three():
                        env=dict(os.environ, RANK="0", WORLD_SIZE="1"))
     assert r.returncode == 0, r.stderr
     assert json.loads(r.stdout)["warmup"] == 3
+
+
+def test_clock_record_parsing():
+    # nvidia-smi --format=csv,noheader,nounits lines of ClockSampler.FIELDS:
+    # index, sm, max sm, power, active mask, hw_slowdown, hw_thermal, sw_thermal, sw_power_cap
+    idle = "0, 345, 2070, 180.1, 0x0000000000000001, Not Active, Not Active, Not Active, Not Active"
+    busy = "0, 2070, 2070, 900.5, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active"
+    capped = "0, 1965, 2070, 1399.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active"
+    hot = "0, 1800, 2070, 1200.0, 0x0000000000000040, Not Active, Active, Not Active, Not Active"
+    r = bench.parse_clocks("\n".join([idle, busy, busy, busy]))
+    assert r == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 4}   # idle sample left out
+    r = bench.parse_clocks("\n".join([busy, capped, capped]))
+    assert r["reasons"] == ["sw_power_cap"] and r["sm_mhz"] == 1965.0
+    r = bench.parse_clocks("\n".join([busy, hot, "garbage", "0, N/A, 2070, x, y, a, b, c, d"]))
+    assert r["reasons"] == ["hw_thermal_slowdown"] and r["samples"] == 2
+    assert bench.parse_clocks("") is None and bench.parse_clocks("no samples here") is None
+
+
+def test_clock_sampler_without_nvidia_smi(monkeypatch):
+    # a host without the tool records no clocks instead of failing the run
+    monkeypatch.setenv("PATH", "")
+    s = bench.ClockSampler(0)
+    assert s.stop() is None
