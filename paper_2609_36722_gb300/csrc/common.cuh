@@ -266,11 +266,6 @@ ATT_DEV void bulk_push_dsmem(uint32_t cdst, uint32_t src, uint32_t bytes, uint32
                ::"r"(cdst), "r"(src), "r"(bytes), "r"(cbar)
                : "memory");
 }
-ATT_DEV uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
 
 // ---------------------------------------------------------------------------
 // tcgen05: tensor memory and the 5th-generation MMA (cta_group::1)
@@ -389,11 +384,6 @@ ATT_DEV uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
 ATT_DEV uint64_t f2_add(uint64_t a, uint64_t b) {
   uint64_t d;
   asm("add.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-ATT_DEV uint64_t f2_mul(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("mul.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
 ATT_DEV uint32_t pack_bf16(float lo, float hi) {
