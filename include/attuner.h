@@ -291,12 +291,20 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
  *                               through distributed shared memory (global
  *                               memory where such clusters cannot be
  *                               co-resident on the device)
+ *   ATTUNER_OPT_SYNC_CHECK      0 off, 1 every compute call reports the device
+ *                               status itself (see below)
  *   ATTUNER_OPT_TEST_STUCK_WAIT see below */
 #define ATTUNER_OPT_PREFILL_KERNEL 1
 #define ATTUNER_OPT_SPLIT_BLOCKS   2
 #define ATTUNER_OPT_WAIT_LIMIT     3
 #define ATTUNER_OPT_QPROJ_SPLIT_K  4
 #define ATTUNER_OPT_SPLIT_MERGE    5
+/* Debug check: while non-zero, attuner_q_project, attuner_kv_project,
+ * attuner_attend, attuner_attend_static_scratch and attuner_query_attend
+ * synchronise their stream before returning and return the device status as
+ * their own (TIMEOUT, DEVICE_CHECK; the status word is cleared), as
+ * attuner_sync_status would.  Not for calls captured into a CUDA graph. */
+#define ATTUNER_OPT_SYNC_CHECK     6
 /* Test hook (failure detection without a GPU fault): while non-zero, one
  * role of every attention launch waits on an mbarrier that nothing arrives
  * at; its bounded wait runs out, the kernel drains its own copies, frees its

@@ -155,5 +155,5 @@ extern "C" attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const 
   }
   ctx->last_launches = launches;
   if (ce != cudaSuccess) return fail(ATTUNER_ERR_CUDA, std::string("attention launch failed: ") + cudaGetErrorString(ce));
-  return ATTUNER_OK;
+  return finish_call(ctx, ATTUNER_OK, st);
 }

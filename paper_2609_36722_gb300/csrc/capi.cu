@@ -754,7 +754,7 @@ extern "C" attuner_status attuner_q_project(attuner_ctx* ctx, const attuner_plan
   e = q_project_impl(ctx, plan, x, w_q, lora_a, lora_b, r, s, q_norm_w, S, S_kv, q_out, st, sc, launches);
   cudaFreeAsync(sc.base, st);
   ctx->last_launches = launches;
-  return e;
+  return finish_call(ctx, e, st);
 }
 
 extern "C" attuner_status attuner_kv_project(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
@@ -772,7 +772,7 @@ extern "C" attuner_status attuner_kv_project(attuner_ctx* ctx, const attuner_pla
   e = kv_project_impl(ctx, plan, x, w_k, w_v, k_norm_w, S, S_kv, suffix_k, suffix_v, st, sc, launches);
   cudaFreeAsync(sc.base, st);
   ctx->last_launches = launches;
-  return e;
+  return finish_call(ctx, e, st);
 }
 
 extern "C" attuner_status attuner_attend(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
@@ -782,10 +782,10 @@ extern "C" attuner_status attuner_attend(attuner_ctx* ctx, const attuner_plan* p
   if (e != ATTUNER_OK) return e;
   if ((e = set_device(ctx)) != ATTUNER_OK) return e;
   int launches = 0;
-  e = attend_impl(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, static_cast<cudaStream_t>(stream),
-                  nullptr, launches);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  e = attend_impl(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, st, nullptr, launches);
   ctx->last_launches = launches;
-  return e;
+  return finish_call(ctx, e, st);
 }
 
 extern "C" attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
@@ -810,7 +810,7 @@ extern "C" attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_p
     e = attend_impl(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, st, &sc, launches);
   cudaFreeAsync(sc.base, st);
   ctx->last_launches = launches;
-  return e;
+  return finish_call(ctx, e, st);
 }
 
 // ---------------------------------------------------------------------------
@@ -840,6 +840,11 @@ extern "C" attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream) {
   return ATTUNER_OK;
 }
 
+attuner_status att::finish_call(attuner_ctx* ctx, attuner_status e, cudaStream_t st) {
+  if (e != ATTUNER_OK || !ctx->opt_sync_check) return e;
+  return attuner_sync_status(ctx, st);
+}
+
 extern "C" attuner_status attuner_set_option(attuner_ctx* ctx, int32_t option, int64_t value) {
   CHECK_ARG(ctx != nullptr, "ctx must not be NULL");
   switch (option) {
@@ -862,6 +867,9 @@ extern "C" attuner_status attuner_set_option(attuner_ctx* ctx, int32_t option, i
     case ATTUNER_OPT_SPLIT_MERGE:
       CHECK_ARG(value >= 0 && value <= 2, "split merge must be 0, 1 or 2");
       ctx->opt_merge = (int)value;
+      return ATTUNER_OK;
+    case ATTUNER_OPT_SYNC_CHECK:
+      ctx->opt_sync_check = value ? 1 : 0;
       return ATTUNER_OK;
     case ATTUNER_OPT_TEST_STUCK_WAIT:
       ctx->inject_stuck = value ? 1 : 0;

@@ -40,6 +40,7 @@ struct attuner_ctx {
   int opt_split = 0;
   int opt_qproj_split = 1;
   int opt_merge = 0;
+  int opt_sync_check = 0;
   int tc_clusters[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};   // co-resident clusters of n tcgen05 CTAs
   long long wait_limit = 1ll << 32;
   int inject_stuck = 0;
@@ -82,5 +83,8 @@ attuner_status check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, i
 attuner_status make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc, WorkTable& w);
 // fills ctx->tc_clusters on first use (queries the device)
 void query_cluster_occupancy(attuner_ctx* ctx);
+// the status a compute call returns: `e`, or with ATTUNER_OPT_SYNC_CHECK set
+// and nothing failed on the host, the device status after `st` drains
+attuner_status finish_call(attuner_ctx* ctx, attuner_status e, cudaStream_t st);
 
 }  // namespace att
