@@ -11,7 +11,8 @@ Every function is a plain restatement of the paper's definitions in float64:
     model's original query normalisation and RoPE;
   * Sec. 2, Eq. (1) and Eq. (full-vs-pic): artifacts cached independently and
     assembled in prompt order;
-  * Sec. 2.2, Eq. (routing-oracle): softmax(q K^T / sqrt(d_k) + M_t) V;
+  * Sec. 2.2, Eq. (routing-oracle): softmax(q K^T / sqrt(d_k) + M_t) V, and
+    the combination of its value over parts of the key set (split-KV);
   * App. A.5 (Deployment): merged W^Q + (alpha/r) B A, SDPA with causal masks
     and position ids for the assembled context;
   * the suffix tokens' own keys and values: base k_proj / v_proj (the
@@ -38,6 +39,7 @@ from .attuner_oracle import (  # noqa: F401
     kv_projection,
     assemble,
     attention,
+    merge_partials,
     request_forward,
     layout_online_positions,
     layout_forward,

@@ -198,6 +198,24 @@ def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, n_visible: Sequence[i
 
 
 # ---------------------------------------------------------------------------
+# Split-KV combine (an implementation step, not the paper's): attention over a
+# key set is the softmax-weighted combination of attention over its parts.
+# With o_i, lse_i the output and log-denominator of part i,
+#   lse = log sum_i exp(lse_i),   o = sum_i exp(lse_i - lse) o_i.
+# A part with no visible key has lse_i = -inf and weight 0.
+# ---------------------------------------------------------------------------
+def merge_partials(o_parts: Sequence[np.ndarray], lse_parts: Sequence[np.ndarray]):
+    """o_parts: P arrays [..., d]; lse_parts: P arrays [...] (-inf for an empty
+    part).  Returns (o [..., d], lse [...])."""
+    lse_stack = np.stack([np.asarray(l, dtype=np.float64) for l in lse_parts])      # [P, ...]
+    m = np.max(lse_stack, axis=0)
+    w = np.exp(lse_stack - m)                                                       # [P, ...]
+    z = np.sum(w, axis=0)
+    o = sum(w[i][..., None] * np.asarray(o_parts[i], dtype=np.float64) for i in range(len(o_parts))) / z[..., None]
+    return o, m + np.log(z)
+
+
+# ---------------------------------------------------------------------------
 # One request end to end: adapted Q -> q_norm -> RoPE -> attention over the
 # assembled artifact KV followed by the suffix's own KV.
 # ---------------------------------------------------------------------------

@@ -19,7 +19,7 @@ import test_oracle_pins as pins
 
 ORIG = {n: getattr(O, n) for n in ("lora_q_projection", "merged_q_weight", "rms_norm_heads", "rope_rotate_half",
                                   "query_positions", "kv_projection", "assemble", "attention", "request_forward",
-                                  "layout_online_positions", "layout_forward")}
+                                  "layout_online_positions", "layout_forward", "merge_partials")}
 PINS = {n: f for n, f in vars(pins).items() if n.startswith("test_") and callable(f)}
 
 
@@ -147,6 +147,22 @@ def attention_swapped_kv(q, k, v, n_visible, pairs=None):
     return ORIG["attention"](q, v, k, n_visible, pairs)
 
 
+# --- split-KV combine ----------------------------------------------------------
+def merge_unnormalised(o_parts, lse_parts):
+    o, lse = ORIG["merge_partials"](o_parts, lse_parts)
+    return o * np.exp(lse)[..., None], lse
+
+
+def merge_plain_mean(o_parts, lse_parts):
+    _, lse = ORIG["merge_partials"](o_parts, lse_parts)
+    return sum(np.asarray(o) for o in o_parts) / len(o_parts), lse
+
+
+def merge_lse_of_the_largest_part(o_parts, lse_parts):
+    o, _ = ORIG["merge_partials"](o_parts, lse_parts)
+    return o, np.max(np.stack([np.asarray(l) for l in lse_parts]), axis=0)
+
+
 # --- suffix K/V ----------------------------------------------------------------
 def kv_without_rope(x, w_k, w_v, k_norm_w, eps, theta, positions, n_kv_heads):
     return ORIG["kv_projection"](x, w_k, w_v, k_norm_w, eps, theta, np.zeros_like(positions), n_kv_heads)
@@ -218,6 +234,8 @@ MUTANTS = [
     ("attention", attention_without_scale), ("attention", attention_mask_off_by_one),
     ("attention", attention_heads_modulo), ("attention", attention_lse_base_two),
     ("attention", attention_swapped_kv),
+    ("merge_partials", merge_unnormalised), ("merge_partials", merge_plain_mean),
+    ("merge_partials", merge_lse_of_the_largest_part),
     ("kv_projection", kv_without_rope), ("kv_projection", kv_value_normalised),
     ("kv_projection", kv_outputs_swapped),
     ("request_forward", request_query_not_self_visible), ("request_forward", request_suffix_not_causal),
@@ -231,7 +249,7 @@ def _pin_order(name):
     key = {"lora_q_projection": "lora", "merged_q_weight": "merged", "rms_norm_heads": "rmsnorm",
            "rope_rotate_half": "rope", "query_positions": "query_positions", "kv_projection": "kv_projection",
            "assemble": "assemble", "attention": "attention", "request_forward": "artifact",
-           "layout_online_positions": "layout", "layout_forward": "layout"}[name]
+           "layout_online_positions": "layout", "layout_forward": "layout", "merge_partials": "merge"}[name]
     names = sorted(PINS)
     return [n for n in names if key in n] + [n for n in names if key not in n]
 

@@ -375,6 +375,55 @@ def test_gqa_equals_mha_with_duplicated_heads():
 
 
 # --------------------------------------------------------------------------
+# Split-KV combine: attention over a key set from attention over its parts
+# --------------------------------------------------------------------------
+def test_merge_hand_example():
+    # parts with denominators 1 and 3 (lse 0 and ln 3) weigh 1/4 and 3/4; lse = ln 4
+    o, lse = O.merge_partials([np.array([4.0, 0.0]), np.array([0.0, 8.0])], [np.array(0.0), np.array(math.log(3.0))])
+    np.testing.assert_allclose(o, [1.0, 6.0], atol=1e-15)
+    assert abs(lse - math.log(4.0)) < 1e-15
+    # an empty part (lse = -inf) has weight 0
+    o, lse = O.merge_partials([np.array([4.0, 0.0]), np.array([9.0, 9.0])], [np.array(0.5), np.array(-np.inf)])
+    np.testing.assert_array_equal(o, [4.0, 0.0])
+    assert lse == 0.5
+
+
+def _part_attention(q, k, v, n_vis, a, b):
+    """Attention of every query over keys [a, b) it can see; o = 0, lse = -inf where it sees none."""
+    S, Hq, d = q.shape
+    cnt = np.clip(np.asarray(n_vis) - a, 0, b - a)
+    o, lse = np.zeros((S, Hq, d)), np.full((S, Hq), -np.inf)
+    rows = np.nonzero(cnt > 0)[0]
+    if len(rows):
+        o_r, l_r = O.attention(q[rows], k[a:b], v[a:b], cnt[rows])
+        o[rows], lse[rows] = o_r, l_r
+    return o, lse
+
+
+def test_merge_of_parts_equals_attention_over_all_keys():
+    rng = np.random.default_rng(23)
+    S, Hq, Hkv, d, T = 7, 4, 2, 16, 90
+    q = rng.standard_normal((S, Hq, d)) * 2
+    k = rng.standard_normal((T, Hkv, d))
+    v = rng.standard_normal((T, Hkv, d))
+    n_vis = T - S + np.arange(S) + 1                       # causal tail: later parts are ragged
+    o_full, lse_full = O.attention(q, k, v, n_vis)
+    for cuts in ([45], [10, 64], [1, 2, 89], [30, 60, 84, 88]):
+        edges = [0] + cuts + [T]
+        parts = [_part_attention(q, k, v, n_vis, a, b) for a, b in zip(edges[:-1], edges[1:])]
+        o, lse = O.merge_partials([p[0] for p in parts], [p[1] for p in parts])
+        np.testing.assert_allclose(o, o_full, atol=1e-12)
+        np.testing.assert_allclose(lse, lse_full, atol=1e-12)
+        # the order of the parts does not matter
+        o_r, lse_r = O.merge_partials([p[0] for p in parts[::-1]], [p[1] for p in parts[::-1]])
+        np.testing.assert_allclose(o_r, o_full, atol=1e-12)
+    # one part is the identity
+    o1, l1 = O.merge_partials([o_full], [lse_full])
+    np.testing.assert_allclose(o1, o_full, atol=1e-15)
+    np.testing.assert_allclose(l1, lse_full, atol=1e-15)
+
+
+# --------------------------------------------------------------------------
 # End-to-end properties of one request
 # --------------------------------------------------------------------------
 def _small_inputs(rng, hidden=32, hq=4, hkv=2, d=16, r=4):
