@@ -378,14 +378,13 @@ def test_gqa_equals_mha_with_duplicated_heads():
 # Split-KV combine: attention over a key set from attention over its parts
 # --------------------------------------------------------------------------
 def test_merge_hand_example():
-    # parts with denominators 1 and 3 (lse 0 and ln 3) weigh 1/4 and 3/4; lse = ln 4
-    o, lse = O.merge_partials([np.array([4.0, 0.0]), np.array([0.0, 8.0])], [np.array(0.0), np.array(math.log(3.0))])
-    np.testing.assert_allclose(o, [1.0, 6.0], atol=1e-15)
-    assert abs(lse - math.log(4.0)) < 1e-15
-    # an empty part (lse = -inf) has weight 0
-    o, lse = O.merge_partials([np.array([4.0, 0.0]), np.array([9.0, 9.0])], [np.array(0.5), np.array(-np.inf)])
-    np.testing.assert_array_equal(o, [4.0, 0.0])
-    assert lse == 0.5
+    g = _golden("merge_two_parts.json")
+    num = {"ln3": math.log(3.0), "ln4": math.log(4.0), "-inf": -np.inf}
+    val = lambda x: num[x] if isinstance(x, str) else x
+    for c in g["cases"]:
+        o, lse = O.merge_partials([np.array(p) for p in c["o_parts"]], [np.array(val(l)) for l in c["lse_parts"]])
+        np.testing.assert_allclose(o, c["o"], atol=1e-15)
+        assert abs(lse - val(c["lse"])) < 1e-15
 
 
 def _part_attention(q, k, v, n_vis, a, b):
