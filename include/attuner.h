@@ -83,7 +83,7 @@ attuner_status attuner_create(const attuner_config* cfg, attuner_ctx** out);
  * The caller must have finished all work it enqueued with this context.
  * Plans of the context not yet freed must not be used afterwards; freeing
  * them later is allowed (each releases its own device buffer then). NULL is
- * accepted. */
+ * accepted.  Errors: none (always OK). */
 attuner_status attuner_destroy(attuner_ctx* ctx);
 
 /* Register one artifact (Sec. 2, Eq. full-vs-pic: Z^PIC = C(A | P_cache),
@@ -143,12 +143,15 @@ attuner_status attuner_plan_export(const attuner_plan* plan, int32_t* block_tabl
                                    int32_t* token_art_host, int32_t* token_off_host,
                                    int64_t* sizes_inout);
 
-/* Per-request assembled artifact length T_art (host array of n_req). */
+/* Per-request assembled artifact length T_art (host array of n_req), the
+ * offset of the suffix positions (App. A.5).  Errors: INVALID_ARG for NULL
+ * pointers or an n_req other than the plan's. */
 attuner_status attuner_plan_t_art(const attuner_plan* plan, int32_t* t_art_host, int32_t n_req);
 
 /* Free a plan. The caller must have finished all work that reads it. Its
  * device buffer goes back to the context, which reuses a few such buffers
- * for later assemblies instead of allocating. */
+ * for later assemblies instead of allocating.  NULL is accepted.  Errors:
+ * none (always OK). */
 attuner_status attuner_plan_free(attuner_plan* plan);
 
 /* Adapted query of the online tokens (Sec. 3, Eq. query-adaptation, then
@@ -229,8 +232,10 @@ attuner_status attuner_kv_project(attuner_ctx* ctx, const attuner_plan* plan, co
                                   const void* w_k, const void* w_v, const void* k_norm_w, int32_t S,
                                   int32_t S_kv, void* suffix_k, void* suffix_v, void* stream);
 
-/* The whole path: attuner_q_project into stream-ordered scratch, then
- * attuner_attend.  Arguments as in those two calls. */
+/* The whole path (Sec. 3, Eq. query-adaptation, then Sec. 2.2, Eq.
+ * routing-oracle): attuner_q_project into stream-ordered scratch, then
+ * attuner_attend.  Arguments as in those two calls.  Errors: as those two
+ * calls, plus CUDA when the scratch cannot be drawn from the context's pool. */
 attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
                                     const void* w_q, const void* lora_a, const void* lora_b,
                                     int32_t r, float s, const void* q_norm_w,
@@ -262,17 +267,20 @@ attuner_status attuner_register_artifacts_host(attuner_ctx* ctx, int32_t n, cons
 /* Forget every registered artifact: the pool is empty again and the next
  * artifact gets id 0 and block 0 (a serving loop's eviction of the whole warm
  * set).  Plans made before are rejected afterwards (INVALID_ARG), and the
- * caller must not reset while kernels that read the pool are still running. */
+ * caller must not reset while kernels that read the pool are still running.
+ * Errors: INVALID_ARG for a NULL context. */
 attuner_status attuner_pool_reset(attuner_ctx* ctx);
 
 /* The paged pool: device base pointers of K and V ([pool_blocks][Hkv][64][d]
- * bf16 each), blocks in use and capacity.  Any output may be NULL. */
+ * bf16 each), blocks in use and capacity.  Any output may be NULL.  The
+ * pointers stay owned by the context.  Errors: INVALID_ARG for a NULL context. */
 attuner_status attuner_pool_info(const attuner_ctx* ctx, void** k_pool, void** v_pool,
                                  int32_t* used_blocks, int32_t* capacity_blocks);
 
-/* Synchronise `stream`, then return and clear the device status word:
- * OK, TIMEOUT (a bounded wait ran out) or DEVICE_CHECK (an index failed a
- * bounds check), or CUDA if the synchronisation itself failed. */
+/* Synchronise `stream`, then return and clear the device status word.
+ * Errors: TIMEOUT (a bounded wait ran out), DEVICE_CHECK (an index failed a
+ * bounds check), CUDA if the synchronisation itself failed, INVALID_ARG for a
+ * NULL context. */
 attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
 
 /* Tuning and test options (value 0 restores the default):
@@ -310,9 +318,13 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
  * at; its bounded wait runs out, the kernel drains its own copies, frees its
  * tensor memory and returns, and attuner_sync_status() reports TIMEOUT. */
 #define ATTUNER_OPT_TEST_STUCK_WAIT 1000
+/* Set one option of the context; it applies to the calls that follow.
+ * Errors: INVALID_ARG for a NULL context, an unknown option or a value out of
+ * its range. */
 attuner_status attuner_set_option(attuner_ctx* ctx, int32_t option, int64_t value);
 
-/* Number of kernel launches the last call on this context enqueued. */
+/* Number of kernel launches the last call on this context enqueued (0 for a
+ * NULL context). */
 int32_t attuner_last_launch_count(const attuner_ctx* ctx);
 
 /* Message of the last error on this host thread ("" if none). */

@@ -79,3 +79,13 @@ def test_product_path_does_not_import_oracle():
                     src = fh.read()
                 assert not re.search(r"^\s*(import|from)\s+oracle\b", src, re.M), f
                 assert "oracle/" not in src and "oracle." not in src, f
+
+
+def test_every_status_entry_point_documents_its_errors():
+    # the header states, above each declaration, what the call returns on error
+    import re
+    with open(os.path.join(ROOT, "include", "attuner.h")) as f:
+        src = f.read()
+    for m in re.finditer(r"attuner_status\s+(attuner_\w+)\s*\(", src):
+        comment = src[:m.start()].rsplit("/*", 1)[-1]
+        assert "Errors" in comment, m.group(1)
