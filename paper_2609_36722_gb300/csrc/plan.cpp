@@ -205,8 +205,8 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
       }
     }
   } else {
-    // decode: several small CTAs per SM keep the HBM queues full and balance
-    // requests of different lengths
+    // decode: about eight small CTAs per SM, run in turn (shared memory holds
+    // one at a time), balance requests of different lengths
     const long long target = 8ll * pol.num_sms;
     chunk = (int)std::max<long long>(16, (total + target - 1) / target);
   }
