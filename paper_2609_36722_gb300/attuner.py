@@ -69,36 +69,39 @@ _p_i32 = ctypes.POINTER(ctypes.c_int32)
 _p_i64 = ctypes.POINTER(ctypes.c_int64)
 
 
+# argument and return types of every entry point, in the order include/attuner.h gives
+SIGNATURES = {
+    "attuner_create": ([ctypes.POINTER(Config), ctypes.POINTER(_vp)], _i32),
+    "attuner_destroy": ([_vp], _i32),
+    "attuner_register_artifact": ([_vp, _vp, _vp, _i32, _vp, _p_i32], _i32),
+    "attuner_assemble": ([_vp, _p_i32, _p_i32, _i32, ctypes.POINTER(_vp)], _i32),
+    "attuner_plan_export": ([_vp, _p_i32, _p_i32, _p_i32, _p_i32, _p_i32, _p_i64], _i32),
+    "attuner_plan_t_art": ([_vp, _p_i32, _i32], _i32),
+    "attuner_plan_free": ([_vp], _i32),
+    "attuner_q_project": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _i32, _i32, _vp, _vp], _i32),
+    "attuner_attend": ([_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
+    "attuner_attend_static_scratch": ([_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
+    "attuner_query_attend": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _vp, _vp, _i32, _i32,
+                              _vp, _vp, _vp], _i32),
+    "attuner_pool_info": ([_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _p_i32, _p_i32], _i32),
+    "attuner_sync_status": ([_vp, _vp], _i32),
+    "attuner_set_option": ([_vp, _i32, ctypes.c_int64], _i32),
+    "attuner_last_launch_count": ([_vp], _i32),
+    "attuner_last_error": ([], ctypes.c_char_p),
+    "attuner_register_artifacts_host": ([_vp, _i32, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _p_i32, _vp,
+                                         _p_i32], _i32),
+    "attuner_pool_reset": ([_vp], _i32),
+    "attuner_kv_project": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
+    "attuner_assemble_layout": ([_vp, _p_i32, _p_i32, _i32, ctypes.POINTER(_vp)], _i32),
+}
+
+
 def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     if not os.path.exists(path):
         raise ImportError(f"libattuner.so is not built ({path}); run __graft_entry__.build() "
                           "or python -m paper_2609_36722_gb300.build")
     lib = ctypes.CDLL(path)
-    sig = {
-        "attuner_create": ([ctypes.POINTER(Config), ctypes.POINTER(_vp)], _i32),
-        "attuner_destroy": ([_vp], _i32),
-        "attuner_register_artifact": ([_vp, _vp, _vp, _i32, _vp, _p_i32], _i32),
-        "attuner_assemble": ([_vp, _p_i32, _p_i32, _i32, ctypes.POINTER(_vp)], _i32),
-        "attuner_plan_export": ([_vp, _p_i32, _p_i32, _p_i32, _p_i32, _p_i32, _p_i64], _i32),
-        "attuner_plan_t_art": ([_vp, _p_i32, _i32], _i32),
-        "attuner_plan_free": ([_vp], _i32),
-        "attuner_q_project": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _i32, _i32, _vp, _vp], _i32),
-        "attuner_attend": ([_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
-        "attuner_attend_static_scratch": ([_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
-        "attuner_query_attend": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _vp, _vp, _i32, _i32,
-                                  _vp, _vp, _vp], _i32),
-        "attuner_pool_info": ([_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _p_i32, _p_i32], _i32),
-        "attuner_sync_status": ([_vp, _vp], _i32),
-        "attuner_set_option": ([_vp, _i32, ctypes.c_int64], _i32),
-        "attuner_last_launch_count": ([_vp], _i32),
-        "attuner_last_error": ([], ctypes.c_char_p),
-        "attuner_register_artifacts_host": ([_vp, _i32, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _p_i32, _vp,
-                                             _p_i32], _i32),
-        "attuner_pool_reset": ([_vp], _i32),
-        "attuner_kv_project": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
-        "attuner_assemble_layout": ([_vp, _p_i32, _p_i32, _i32, ctypes.POINTER(_vp)], _i32),
-    }
-    for name, (args, ret) in sig.items():
+    for name, (args, ret) in SIGNATURES.items():
         f = getattr(lib, name)
         f.argtypes = args
         f.restype = ret
@@ -233,8 +236,8 @@ class Context:
                 raise ValueError("each k, v must be bf16 [L, Hkv, d] of the same shape")
             if not (k.is_contiguous() and v.is_contiguous()):
                 raise ValueError("ks and vs must be contiguous")
-        kp = (_vp * n)(*[k.dataself._p() for k in ks])
-        vp = (_vp * n)(*[v.dataself._p() for v in vs])
+        kp = (_vp * n)(*[k.data_ptr() for k in ks])
+        vp = (_vp * n)(*[v.data_ptr() for v in vs])
         lens = (ctypes.c_int32 * n)(*[k.shape[0] for k in ks])
         ids = (ctypes.c_int32 * n)()
         _check(lib().attuner_register_artifacts_host(self.handle, n, kp, vp, lens, self._s(stream), ids))

@@ -18,16 +18,20 @@ from paper_2609_36722_gb300 import attuner as A
 
 
 class FakeTensor:
-    def __init__(self, shape, dtype=torch.bfloat16, device="cuda:0", ptr=0x1000, contiguous=True):
+    def __init__(self, shape, dtype=torch.bfloat16, device="cuda:0", ptr=0x1000, contiguous=True, pinned=False):
         self.shape = tuple(shape)
         self.dtype = dtype
         self.device = torch.device(device)
         self.is_cuda = self.device.type == "cuda"
         self._ptr = ptr
         self._contiguous = contiguous
+        self._pinned = pinned
 
     def is_contiguous(self):
         return self._contiguous
+
+    def is_pinned(self):
+        return self._pinned
 
     def data_ptr(self):
         return self._ptr
@@ -43,6 +47,10 @@ class FakeStream:
 
 
 class RecordingLib:
+    """Records each call after converting every argument through the ctypes
+    type the binding declares for it, so a wrong arity, a Python object where a
+    pointer belongs or a misspelt attribute fails here as it would in ctypes."""
+
     def __init__(self):
         self.calls = []
 
@@ -50,10 +58,17 @@ class RecordingLib:
         return b"recorded"
 
     def __getattr__(self, name):
-        if not name.startswith("attuner_"):
+        if name not in A.SIGNATURES:
             raise AttributeError(name)
+        argtypes, _ = A.SIGNATURES[name]
 
         def fn(*args):
+            assert len(args) == len(argtypes), f"{name}: {len(args)} arguments, header has {len(argtypes)}"
+            for i, (a, t) in enumerate(zip(args, argtypes)):
+                try:
+                    t.from_param(a)
+                except (TypeError, ctypes.ArgumentError) as e:
+                    raise AssertionError(f"{name} argument {i}: {a!r} is not a {t.__name__}: {e}")
             self.calls.append((name, args))
             return 0
         return fn
@@ -129,3 +144,100 @@ def test_a_failing_status_raises_with_the_library_message(ctx, monkeypatch):
     with pytest.raises(A.AttunerError, match="recorded") as e:
         c.set_option(A.OPT_SPLIT_BLOCKS, 3)
     assert e.value.status == A.ERR_INVALID_ARG
+
+
+def test_host_artifact_load_passes_host_pointers_lengths_and_stream(ctx):
+    c, plan, fake = ctx
+    ks = [FakeTensor((37, 2, 64), device="cpu", ptr=0x10000, pinned=True),
+          FakeTensor((100, 2, 64), device="cpu", ptr=0x20000, pinned=True)]
+    vs = [FakeTensor((37, 2, 64), device="cpu", ptr=0x30000, pinned=True),
+          FakeTensor((100, 2, 64), device="cpu", ptr=0x40000, pinned=True)]
+    ids = c.register_artifacts_host(ks, vs, stream=FakeStream())
+    name, args = fake.calls[-1]
+    assert name == "attuner_register_artifacts_host"
+    assert args[1] == 2
+    assert [args[2][i] for i in range(2)] == [0x10000, 0x20000]
+    assert [args[3][i] for i in range(2)] == [0x30000, 0x40000]
+    assert list(args[4]) == [37, 100]
+    assert args[5] == 0x77
+    assert ids == [0, 0]     # the stand-in library leaves the id array as allocated
+
+
+@pytest.mark.parametrize("bad", ["cuda", "pageable", "dtype", "shape", "empty"])
+def test_host_artifact_load_refuses_unusable_tensors(ctx, bad):
+    c, plan, fake = ctx
+    k = FakeTensor((37, 2, 64), device="cpu", pinned=True)
+    v = FakeTensor((37, 2, 64), device="cpu", pinned=True)
+    if bad == "cuda":
+        k = FakeTensor((37, 2, 64))
+    elif bad == "pageable":
+        v = FakeTensor((37, 2, 64), device="cpu")
+    elif bad == "dtype":
+        v = FakeTensor((37, 2, 64), dtype=torch.float16, device="cpu", pinned=True)
+    elif bad == "shape":
+        v = FakeTensor((36, 2, 64), device="cpu", pinned=True)
+    with pytest.raises(ValueError):
+        c.register_artifacts_host([] if bad == "empty" else [k], [] if bad == "empty" else [v], stream=FakeStream())
+    assert fake.calls == []
+
+
+def test_every_public_method_reaches_its_entry_point(ctx, monkeypatch):
+    """Each public method of Context and Plan, called once with matching
+    stand-ins, reaches the library with arguments its declared ctypes types
+    accept.  A public method missing from this table fails the test, so a new
+    method cannot skip the check."""
+    c, plan, fake = ctx
+    monkeypatch.setattr(A, "_wrap", lambda ptr, shape, device: ("view", ptr, shape))
+    plan.ctx = c
+    plan.n_req = 2
+    plan.requests = [[0], [1]]
+    dev = FakeTensor((4,))
+    q, sk, sv, out, lse = _attend_args()
+    x = FakeTensor((2, 3, 256), ptr=0x6000)
+    w = FakeTensor((256, 256), ptr=0x7000)
+    la, lb = FakeTensor((8, 256), ptr=0x8000), FakeTensor((256, 8), ptr=0x9000)
+    qn = FakeTensor((64,), ptr=0xA000)
+    wk, wv = FakeTensor((128, 256), ptr=0xB000), FakeTensor((128, 256), ptr=0xC000)
+    kn = FakeTensor((64,), ptr=0xD000)
+    hk = FakeTensor((5, 2, 64), device="cpu", pinned=True, ptr=0xE000)
+    hv = FakeTensor((5, 2, 64), device="cpu", pinned=True, ptr=0xF000)
+    st = FakeStream()
+    ctx_calls = {
+        "register_artifact": (lambda: c.register_artifact(FakeTensor((5, 2, 64)), FakeTensor((5, 2, 64)), stream=st),
+                              "attuner_register_artifact"),
+        "register_artifacts_host": (lambda: c.register_artifacts_host([hk], [hv], stream=st),
+                                    "attuner_register_artifacts_host"),
+        "pool_reset": (lambda: c.pool_reset(), "attuner_pool_reset"),
+        "assemble": (lambda: c.assemble([[0, 1], []]), "attuner_assemble"),
+        "assemble_layout": (lambda: c.assemble_layout([[-16, 0, -5, 1], [0]]), "attuner_assemble_layout"),
+        "q_project": (lambda: c.q_project(plan, x, w, la, lb, 2.0, qn, S_kv=5, out=q, stream=st),
+                      "attuner_q_project"),
+        "kv_project": (lambda: c.kv_project(plan, x, wk, wv, kn, sk, sv, stream=st), "attuner_kv_project"),
+        "attend": (lambda: c.attend(plan, q, sk, sv, out=out, lse=lse, stream=st), "attuner_attend"),
+        "attend_static_scratch": (lambda: c.attend_static_scratch(plan, q, sk, sv, out=out, lse=lse, stream=st),
+                                  "attuner_attend_static_scratch"),
+        "query_attend": (lambda: c.query_attend(plan, x, w, la, lb, 2.0, qn, sk, sv, out=q, lse=lse, stream=st),
+                         "attuner_query_attend"),
+        "pool_tensors": (lambda: c.pool_tensors(), "attuner_pool_info"),
+        "sync_status": (lambda: c.sync_status(stream=st), "attuner_sync_status"),
+        "set_option": (lambda: c.set_option(A.OPT_SPLIT_BLOCKS, 4), "attuner_set_option"),
+        "last_launch_count": (lambda: c.last_launch_count(), "attuner_last_launch_count"),
+    }
+    plan_calls = {
+        "t_art": (lambda: plan.t_art(), "attuner_plan_t_art"),
+        "export": (lambda: plan.export(), "attuner_plan_export"),
+    }
+    ignore = {"for_geometry", "close", "free"}   # a constructor and the two releases (checked last)
+    public = {n for n in dir(A.Context) if not n.startswith("_")} - ignore
+    assert public == set(ctx_calls), sorted(public ^ set(ctx_calls))
+    public_plan = {n for n in dir(A.Plan) if not n.startswith("_")} - ignore
+    assert public_plan == set(plan_calls), sorted(public_plan ^ set(plan_calls))
+    for method, (call, entry) in {**ctx_calls, **plan_calls}.items():
+        n = len(fake.calls)
+        call()
+        assert [name for name, _ in fake.calls[n:]][-1] == entry, method
+    plan.free()
+    assert fake.calls[-1][0] == "attuner_plan_free"
+    c.close()
+    assert fake.calls[-1][0] == "attuner_destroy"
+    assert dev.dim() == 1
