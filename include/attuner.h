@@ -197,14 +197,15 @@ attuner_status attuner_attend(attuner_ctx* ctx, const attuner_plan* plan, const 
  * partial results in one fixed 32 MiB array in device memory that the library
  * declares at file scope; it calls no allocator of any kind.
  *   - The array exists on every GPU that loads the library until the process
- *     exits.  The first call on a device looks up its device address once
- *     (cudaGetSymbolAddress), so make that first call outside any stream
- *     capture.
- *   - Every call shares the array and it keeps the last call's contents
- *     (nothing in it needs to start at zero; the call clears the arrival
- *     counters it keeps there with cudaMemsetAsync on `stream`).  Calls
- *     whose kernels overlap on the GPU race on it: order them (one stream,
- *     or events).
+ *     exits, one copy per CUDA context.  The first call in each context (so
+ *     once per device, and again after cudaDeviceReset) looks up its device
+ *     address (cudaGetSymbolAddress), which may load the library's module:
+ *     make that first call outside any stream capture.
+ *   - Every call in a context shares the array and it keeps the last call's
+ *     contents (nothing in it needs to start at zero; the call clears the
+ *     arrival counters it keeps there with cudaMemsetAsync on `stream`).
+ *     Calls whose kernels overlap on the GPU race on it: order them (one
+ *     stream, or events).
  *   - A call whose partial results would need more than 32 MiB
  *     (n_split_ctas * rows_per_cta * (d + 1) * 4 bytes, plus 4 bytes per
  *     (request, KV head, row tile) for the tcgen05 kernel) is rejected with

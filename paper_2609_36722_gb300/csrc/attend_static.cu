@@ -8,18 +8,19 @@
 // or fail at an arbitrary point of a request.  attuner_attend draws its
 // split-KV partial results from a stream-ordered pool, so it allocates on
 // first use and whenever a call needs more.  This entry point runs the same
-// kernels with the same work decomposition but keeps those partial results
-// in one file-scope device array of fixed size instead, and allocates
-// nothing: no cudaMalloc, no cudaFree, no pool allocation, no host heap.
+// launch code (att::attend_launch) with the same work decomposition, but
+// hands it one file-scope device array of fixed size for those partial
+// results, and allocates nothing: no cudaMalloc, no cudaFree, no pool
+// allocation.
 //
 // The array lives in every GPU that loads the library, until the process
-// exits.  All calls share it, so two calls whose kernels overlap on the GPU
-// (different streams, or different contexts on the same device) race on it;
-// the caller must order such calls.  It keeps the last call's contents:
-// nothing in it needs to start at zero, because every partial result a merge
-// reads is written earlier in the same call, and the call clears the few
-// arrival counters it keeps there itself (cudaMemsetAsync, which allocates
-// nothing).
+// exits; each CUDA context has its own copy.  All calls within one context
+// share it, so two calls whose kernels overlap on the GPU (different streams
+// of one context) race on it; the caller must order such calls.  It keeps the
+// last call's contents: nothing in it needs to start at zero, because every
+// partial result a merge reads is written earlier in the same call, and the
+// call clears the few arrival counters it keeps there itself
+// (cudaMemsetAsync, which allocates nothing).
 #include <mutex>
 
 #include "internal.h"
@@ -32,26 +33,64 @@ namespace {
 constexpr size_t kStaticScratchBytes = 32ull << 20;
 static __device__ __align__(256) unsigned char g_split_scratch[kStaticScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_setup_mutex;
-void* g_scratch_ptr[kMaxDevices] = {nullptr};
+// In host code the array's name is only a host-side stand-in for the symbol:
+// its device address has to be looked up (cudaGetSymbolAddress) with the
+// right context current.  A module, and so the array, exists once per CUDA
+// context, so the looked-up address is cached per context, keyed by the
+// context's unique id (a context created after cudaDeviceReset, or a
+// non-primary context, gets an id of its own and its own lookup).
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
 
-// Device address of g_split_scratch on the current device.  In host code the
-// array's name is only a host-side stand-in for the symbol, so the address
-// is looked up once per device (with that device current) and cached.
-attuner_status scratch_address(int device, void** out) {
-  if (device < 0 || device >= kMaxDevices)
-    return fail(ATTUNER_ERR_UNSUPPORTED, "attuner_attend_static_scratch: device ordinal >= 64");
+constexpr int kCacheSlots = 64;
+std::mutex g_setup_mutex;
+unsigned long long g_ctx_id[kCacheSlots] = {0};
+void* g_scratch_ptr[kCacheSlots] = {nullptr};
+int g_next_slot = 0;
+
+template <typename Fn>
+Fn driver_fn(const char* name) {
+  void* p = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion(name, &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+      q == cudaDriverEntryPointSuccess)
+    return reinterpret_cast<Fn>(p);
+  return nullptr;
+}
+
+// id of the calling thread's current context, or 0 if it cannot be told
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_cur = driver_fn<CtxGetCurrentFn>("cuCtxGetCurrent");
+  static CtxGetIdFn get_id = driver_fn<CtxGetIdFn>("cuCtxGetId");
+  CUcontext c = nullptr;
+  unsigned long long id = 0;
+  if (!get_cur || !get_id || get_cur(&c) != CUDA_SUCCESS || c == nullptr || get_id(c, &id) != CUDA_SUCCESS)
+    return 0;
+  return id + 1;   // 0 stays "unknown"
+}
+
+// Device address of g_split_scratch in the current context (set-up on the
+// first call in each context; later calls find it in the cache).
+attuner_status scratch_address(void** out) {
+  const unsigned long long id = current_context_id();
   std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (g_scratch_ptr[device] == nullptr) {
-    void* p = nullptr;
-    cudaError_t e = cudaGetSymbolAddress(&p, g_split_scratch);
-    if (e != cudaSuccess || p == nullptr)
-      return fail(ATTUNER_ERR_CUDA, std::string("cudaGetSymbolAddress(split scratch) failed: ") +
-                                        cudaGetErrorString(e));
-    g_scratch_ptr[device] = p;
+  if (id != 0)
+    for (int i = 0; i < kCacheSlots; ++i)
+      if (g_ctx_id[i] == id) {
+        *out = g_scratch_ptr[i];
+        return ATTUNER_OK;
+      }
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_split_scratch);
+  if (e != cudaSuccess || p == nullptr)
+    return fail(ATTUNER_ERR_CUDA,
+                std::string("cudaGetSymbolAddress(split scratch) failed: ") + cudaGetErrorString(e));
+  if (id != 0) {   // an unknown context is looked up on every call instead
+    g_ctx_id[g_next_slot] = id;
+    g_scratch_ptr[g_next_slot] = p;
+    g_next_slot = (g_next_slot + 1) % kCacheSlots;
   }
-  *out = g_scratch_ptr[device];
+  *out = p;
   return ATTUNER_OK;
 }
 
@@ -64,96 +103,11 @@ extern "C" attuner_status attuner_attend_static_scratch(attuner_ctx* ctx, const 
   attuner_status e = check_common(ctx, plan, S, S_kv);
   if (e != ATTUNER_OK) return e;
   if ((e = set_device(ctx)) != ATTUNER_OK) return e;
-  CHECK_ARG(q && suffix_k && suffix_v && out, "q, suffix_k, suffix_v and out must not be NULL");
-  CHECK_ARG(aligned16(q) && aligned16(suffix_k) && aligned16(suffix_v) && aligned16(out),
-            "q, suffix_k, suffix_v and out must be 16-byte aligned");
-  const attuner_config& c = ctx->cfg;
-  const int D = c.head_dim, Hq = c.n_q_heads, Hkv = c.n_kv_heads, G = Hq / Hkv;
+  FixedScratch fx{nullptr, kStaticScratchBytes};
+  if ((e = scratch_address(&fx.base)) != ATTUNER_OK) return e;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  bool tc;
-  if (ctx->opt_prefill == 1) tc = true;
-  else if (ctx->opt_prefill == 2) tc = false;
-  else tc = (S * G > kMmaRows);
-  const int rows = tc ? kTcRows : kMmaRows;
-
-  AttnParams ap{};   // on the stack: this entry point touches no heap
-  if (tc) query_cluster_occupancy(ctx);
-  if ((e = make_work(ctx, plan, S, S_kv, tc, ap.work)) != ATTUNER_OK) return e;
-  bool need_combine = false;   // split partial results in global memory
-  for (int r = 0; r < plan->n_req; ++r) need_combine |= (ap.work.nsplit[r] > 1);
-  if (ap.work.cluster > 0) need_combine = false;
-  const size_t pb = need_combine ? (size_t)ap.work.n_cta * rows * (D + 1) * 4 : 0;
-  const size_t units = (size_t)plan->n_req * Hkv * ap.work.row_tiles;
-  const size_t part_bytes = pb + ((need_combine && tc) ? units * 4 : 0);
-  if (part_bytes > kStaticScratchBytes)
-    return fail(ATTUNER_ERR_INVALID_ARG,
-                "attuner_attend_static_scratch: this call needs " + std::to_string(part_bytes) +
-                    " bytes of split-KV scratch, more than the fixed " +
-                    std::to_string(kStaticScratchBytes) + " bytes; use attuner_attend");
-  void* scratch = nullptr;
-  if (need_combine && (e = scratch_address(c.device, &scratch)) != ATTUNER_OK) return e;
-
-  if (tc) {
-    const uint64_t dims[5] = {(uint64_t)D, (uint64_t)G, (uint64_t)Hkv, (uint64_t)S, (uint64_t)plan->n_req};
-    const uint64_t strides[4] = {(uint64_t)D * 2, (uint64_t)G * D * 2, (uint64_t)Hq * D * 2,
-                                 (uint64_t)S * Hq * D * 2};
-    const uint32_t box[5] = {64, (uint32_t)G, 1, (uint32_t)(kTcTileRows / G), 1};
-    if ((e = make_map(&ap.tm_q, q, 5, dims, strides, box, "q")) != ATTUNER_OK) return e;
-  }
-  {
-    const uint64_t dims[4] = {(uint64_t)D, (uint64_t)Hkv, (uint64_t)S_kv, (uint64_t)plan->n_req};
-    const uint64_t strides[3] = {(uint64_t)D * 2, (uint64_t)Hkv * D * 2, (uint64_t)S_kv * Hkv * D * 2};
-    const uint32_t box[4] = {64, 1, 64, 1};
-    if ((e = make_map(&ap.tm_ksuf, suffix_k, 4, dims, strides, box, "suffix_k")) != ATTUNER_OK) return e;
-    if ((e = make_map(&ap.tm_vsuf, suffix_v, 4, dims, strides, box, "suffix_v")) != ATTUNER_OK) return e;
-  }
-  if (tc && ap.work.cluster > 0 &&
-      (e = make_out_map(&ap.tm_out, out, D, Hq, G, S, plan->n_req, ap.work.cluster)) != ATTUNER_OK)
-    return e;
-  ap.tm_kpool = ctx->tm_kpool;
-  ap.tm_vpool = ctx->tm_vpool;
-  ap.plan = plan_dev(plan);
-  ap.q = static_cast<const __nv_bfloat16*>(q);
-  ap.out = static_cast<__nv_bfloat16*>(out);
-  ap.lse_out = lse_out;
-  ap.S = S;
-  ap.S_kv = S_kv;
-  ap.Hq = Hq;
-  ap.Hkv = Hkv;
-  ap.G = G;
-  ap.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
-  ap.status = ctx->d_status;
-  ap.wait_limit = ctx->wait_limit;
-  ap.inject_stuck = ctx->inject_stuck;
-  cudaError_t ce = cudaSuccess;
-  if (need_combine) {
-    ap.part_o = static_cast<float*>(scratch);
-    ap.part_lse = static_cast<float*>(scratch) + (size_t)ap.work.n_cta * rows * D;
-    if (tc) {   // arrival counters of the in-kernel split merge
-      ap.unit_cnt = reinterpret_cast<int*>(static_cast<char*>(scratch) + pb);
-      ce = cudaMemsetAsync(ap.unit_cnt, 0, units * 4, st);
-    }
-  }
   int launches = 0;
-  if (ce == cudaSuccess) ce = tc ? launch_attn_tc(ap, D, st) : launch_attn_mma(ap, D, st);
-  if (ce == cudaSuccess) ++launches;
-  if (ce == cudaSuccess && need_combine && !tc) {
-    CombineParams cp{};
-    cp.work = ap.work;
-    cp.part_o = ap.part_o;
-    cp.part_lse = ap.part_lse;
-    cp.out = ap.out;
-    cp.lse_out = lse_out;
-    cp.S = S;
-    cp.Hq = Hq;
-    cp.Hkv = Hkv;
-    cp.G = G;
-    cp.D = D;
-    cp.rows_per_tile = rows;
-    ce = launch_combine(cp, st);
-    if (ce == cudaSuccess) ++launches;
-  }
+  e = attend_launch(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, st, &fx, launches);
   ctx->last_launches = launches;
-  if (ce != cudaSuccess) return fail(ATTUNER_ERR_CUDA, std::string("attention launch failed: ") + cudaGetErrorString(ce));
-  return finish_call(ctx, ATTUNER_OK, st);
+  return finish_call(ctx, e, st);
 }

@@ -634,9 +634,9 @@ attuner_status att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, 
   return s == ATTUNER_OK ? s : fail(s, err);
 }
 
-static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
+attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
                                   const void* suffix_k, const void* suffix_v, int32_t S, int32_t S_kv,
-                                  void* out, float* lse_out, cudaStream_t st, Scratch* sc_outer,
+                                  void* out, float* lse_out, cudaStream_t st, const FixedScratch* fixed,
                                   int& launches) {
   const attuner_config& c = ctx->cfg;
   CHECK_ARG(q && suffix_k && suffix_v && out, "q, suffix_k, suffix_v and out must not be NULL");
@@ -647,83 +647,83 @@ static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, co
   if (ctx->opt_prefill == 1) tc = true;
   else if (ctx->opt_prefill == 2) tc = false;
   else tc = (S * G > kMmaRows);
-  WorkTable* w = new WorkTable();
-  if (tc) query_cluster_occupancy(ctx);
-  if (const attuner_status ws = make_work(ctx, plan, S, S_kv, tc, *w); ws != ATTUNER_OK) {
-    delete w;
-    return ws;
-  }
-  bool need_combine = false;   // split partial results in global memory
-  for (int r = 0; r < plan->n_req; ++r) need_combine |= (w->nsplit[r] > 1);
-  if (w->cluster > 0) need_combine = false;
   const int rows = tc ? kTcRows : kMmaRows;
 
-  AttnParams* ap = new AttnParams();
+  AttnParams ap{};   // on the stack: the launch itself touches no heap
   attuner_status e = ATTUNER_OK;
-  auto done = [&](attuner_status s) { delete ap; delete w; return s; };
+  if (tc) query_cluster_occupancy(ctx);
+  if ((e = make_work(ctx, plan, S, S_kv, tc, ap.work)) != ATTUNER_OK) return e;
+  const WorkTable& w = ap.work;
+  bool need_combine = false;   // split partial results in global memory
+  for (int r = 0; r < plan->n_req; ++r) need_combine |= (w.nsplit[r] > 1);
+  if (w.cluster > 0) need_combine = false;
+  // partial O and LSE of every split CTA; for the tcgen05 kernel also one
+  // arrival counter per (request, KV head, row tile), zeroed below
+  const size_t pb = need_combine ? (size_t)w.n_cta * rows * (D + 1) * 4 : 0;
+  const size_t units = (size_t)plan->n_req * Hkv * w.row_tiles;
+  const size_t part_bytes = pb + ((need_combine && tc) ? units * 4 : 0);
+  if (fixed && part_bytes > fixed->cap)
+    return fail(ATTUNER_ERR_INVALID_ARG,
+                "this call needs " + std::to_string(part_bytes) + " bytes of split-KV scratch, more than the fixed " +
+                    std::to_string(fixed->cap) + " bytes of attuner_attend_static_scratch; use attuner_attend");
+
   if (tc) {
     const uint64_t dims[5] = {(uint64_t)D, (uint64_t)G, (uint64_t)Hkv, (uint64_t)S, (uint64_t)plan->n_req};
     const uint64_t strides[4] = {(uint64_t)D * 2, (uint64_t)G * D * 2, (uint64_t)Hq * D * 2,
                                  (uint64_t)S * Hq * D * 2};
     const uint32_t box[5] = {64, (uint32_t)G, 1, (uint32_t)(kTcTileRows / G), 1};
-    if ((e = make_map(&ap->tm_q, q, 5, dims, strides, box, "q")) != ATTUNER_OK) return done(e);
+    if ((e = make_map(&ap.tm_q, q, 5, dims, strides, box, "q")) != ATTUNER_OK) return e;
   }
   {
     const uint64_t dims[4] = {(uint64_t)D, (uint64_t)Hkv, (uint64_t)S_kv, (uint64_t)plan->n_req};
     const uint64_t strides[3] = {(uint64_t)D * 2, (uint64_t)Hkv * D * 2, (uint64_t)S_kv * Hkv * D * 2};
     const uint32_t box[4] = {64, 1, 64, 1};
-    if ((e = make_map(&ap->tm_ksuf, suffix_k, 4, dims, strides, box, "suffix_k")) != ATTUNER_OK) return done(e);
-    if ((e = make_map(&ap->tm_vsuf, suffix_v, 4, dims, strides, box, "suffix_v")) != ATTUNER_OK) return done(e);
+    if ((e = make_map(&ap.tm_ksuf, suffix_k, 4, dims, strides, box, "suffix_k")) != ATTUNER_OK) return e;
+    if ((e = make_map(&ap.tm_vsuf, suffix_v, 4, dims, strides, box, "suffix_v")) != ATTUNER_OK) return e;
   }
-  if (tc && w->cluster > 0 &&
-      (e = make_out_map(&ap->tm_out, out, D, Hq, G, S, plan->n_req, w->cluster)) != ATTUNER_OK)
-    return done(e);
-  ap->tm_kpool = ctx->tm_kpool;
-  ap->tm_vpool = ctx->tm_vpool;
-  ap->plan = plan_dev(plan);
-  ap->work = *w;
-  ap->q = static_cast<const __nv_bfloat16*>(q);
-  ap->out = static_cast<__nv_bfloat16*>(out);
-  ap->lse_out = lse_out;
-  ap->S = S;
-  ap->S_kv = S_kv;
-  ap->Hq = Hq;
-  ap->Hkv = Hkv;
-  ap->G = G;
-  ap->scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
-  ap->status = ctx->d_status;
-  ap->wait_limit = ctx->wait_limit;
-  ap->inject_stuck = ctx->inject_stuck;
+  if (tc && w.cluster > 0 &&
+      (e = make_out_map(&ap.tm_out, out, D, Hq, G, S, plan->n_req, w.cluster)) != ATTUNER_OK)
+    return e;
+  ap.tm_kpool = ctx->tm_kpool;
+  ap.tm_vpool = ctx->tm_vpool;
+  ap.plan = plan_dev(plan);
+  ap.q = static_cast<const __nv_bfloat16*>(q);
+  ap.out = static_cast<__nv_bfloat16*>(out);
+  ap.lse_out = lse_out;
+  ap.S = S;
+  ap.S_kv = S_kv;
+  ap.Hq = Hq;
+  ap.Hkv = Hkv;
+  ap.G = G;
+  ap.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
+  ap.status = ctx->d_status;
+  ap.wait_limit = ctx->wait_limit;
+  ap.inject_stuck = ctx->inject_stuck;
 
-  (void)sc_outer;
   void* part = nullptr;
-  size_t part_bytes = 0;
   cudaError_t ce = cudaSuccess;
   if (need_combine) {
-    // partial O and LSE of every split CTA; for the tcgen05 kernel also one
-    // arrival counter per (request, KV head, row tile), zeroed here
-    const size_t pb = (size_t)w->n_cta * rows * (D + 1) * 4;
-    const size_t units = (size_t)plan->n_req * Hkv * w->row_tiles;
-    part_bytes = pb + (tc ? units * 4 : 0);
-    if (cudaMallocFromPoolAsync(&part, part_bytes, ctx->mempool, st) != cudaSuccess) {
+    if (fixed) {
+      part = fixed->base;
+    } else if (cudaMallocFromPoolAsync(&part, part_bytes, ctx->mempool, st) != cudaSuccess) {
       cudaGetLastError();
-      return done(fail(ATTUNER_ERR_OOM, "split-KV scratch allocation failed"));
+      return fail(ATTUNER_ERR_OOM, "split-KV scratch allocation failed");
     }
-    ap->part_o = static_cast<float*>(part);
-    ap->part_lse = static_cast<float*>(part) + (size_t)w->n_cta * rows * D;
+    ap.part_o = static_cast<float*>(part);
+    ap.part_lse = static_cast<float*>(part) + (size_t)w.n_cta * rows * D;
     if (tc) {
-      ap->unit_cnt = reinterpret_cast<int*>(static_cast<char*>(part) + pb);
-      ce = cudaMemsetAsync(ap->unit_cnt, 0, units * 4, st);
+      ap.unit_cnt = reinterpret_cast<int*>(static_cast<char*>(part) + pb);
+      ce = cudaMemsetAsync(ap.unit_cnt, 0, units * 4, st);
     }
   }
-  if (ce == cudaSuccess) ce = tc ? launch_attn_tc(*ap, D, st) : launch_attn_mma(*ap, D, st);
+  if (ce == cudaSuccess) ce = tc ? launch_attn_tc(ap, D, st) : launch_attn_mma(ap, D, st);
   if (ce == cudaSuccess) ++launches;
   if (ce == cudaSuccess && need_combine && !tc) {   // the tcgen05 kernel merges its splits itself
     CombineParams cp{};
-    cp.work = *w;
-    cp.part_o = ap->part_o;
-    cp.part_lse = ap->part_lse;
-    cp.out = ap->out;
+    cp.work = w;
+    cp.part_o = ap.part_o;
+    cp.part_lse = ap.part_lse;
+    cp.out = ap.out;
     cp.lse_out = lse_out;
     cp.S = S;
     cp.Hq = Hq;
@@ -734,9 +734,9 @@ static attuner_status attend_impl(attuner_ctx* ctx, const attuner_plan* plan, co
     ce = launch_combine(cp, st);
     if (ce == cudaSuccess) ++launches;
   }
-  if (part) cudaFreeAsync(part, st);
-  if (ce != cudaSuccess) return done(fail(ATTUNER_ERR_CUDA, std::string("attention launch failed: ") + cudaGetErrorString(ce)));
-  return done(ATTUNER_OK);
+  if (part && !fixed) cudaFreeAsync(part, st);
+  if (ce != cudaSuccess) return fail(ATTUNER_ERR_CUDA, std::string("attention launch failed: ") + cudaGetErrorString(ce));
+  return ATTUNER_OK;
 }
 
 extern "C" attuner_status attuner_q_project(attuner_ctx* ctx, const attuner_plan* plan, const void* x,
@@ -783,7 +783,7 @@ extern "C" attuner_status attuner_attend(attuner_ctx* ctx, const attuner_plan* p
   if ((e = set_device(ctx)) != ATTUNER_OK) return e;
   int launches = 0;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  e = attend_impl(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, st, nullptr, launches);
+  e = attend_launch(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, st, nullptr, launches);
   ctx->last_launches = launches;
   return finish_call(ctx, e, st);
 }
@@ -807,7 +807,7 @@ extern "C" attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_p
   int launches = 0;
   e = q_project_impl(ctx, plan, x, w_q, lora_a, lora_b, r, s, q_norm_w, S, S_kv, q, st, sc, launches);
   if (e == ATTUNER_OK)
-    e = attend_impl(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, st, &sc, launches);
+    e = attend_launch(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, st, nullptr, launches);
   cudaFreeAsync(sc.base, st);
   ctx->last_launches = launches;
   return finish_call(ctx, e, st);

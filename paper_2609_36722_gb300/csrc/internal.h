@@ -83,6 +83,21 @@ attuner_status check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, i
 attuner_status make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc, WorkTable& w);
 // fills ctx->tc_clusters on first use (queries the device)
 void query_cluster_occupancy(attuner_ctx* ctx);
+// A caller-provided device region for the split-KV partial results of one
+// attention launch, used instead of an allocation from the context's pool.
+struct FixedScratch {
+  void* base;   // device address, 256-byte aligned
+  size_t cap;   // bytes
+};
+// The attention step of one call (attention and split-KV merge): work decomposition, tensor
+// maps, split-KV scratch and the kernel launches on `st`.  With `fixed` null
+// the scratch comes from the context's stream-ordered pool; otherwise from
+// `fixed`, and a call needing more than fixed->cap bytes fails with
+// INVALID_ARG before anything is launched.  Adds the kernels launched to
+// `launches`.
+attuner_status attend_launch(attuner_ctx* ctx, const attuner_plan* plan, const void* q, const void* suffix_k,
+                             const void* suffix_v, int32_t S, int32_t S_kv, void* out, float* lse_out,
+                             cudaStream_t st, const FixedScratch* fixed, int& launches);
 // the status a compute call returns: `e`, or with ATTUNER_OPT_SYNC_CHECK set
 // and nothing failed on the host, the device status after `st` drains
 attuner_status finish_call(attuner_ctx* ctx, attuner_status e, cudaStream_t st);
