@@ -2,17 +2,24 @@
 
 One step = one pass of the whole path over one batch: adapted Q projection
 (LoRA, RMSNorm, RoPE) and attention over the assembled artifact blocks plus
-the suffix KV (split-KV combine included).  Default workload: the Qwen3-4B
-layer (hidden 2560, 32/8 heads, d 128, r 16, 8 artifacts of 512-2048 tokens,
-256 suffix tokens).  Inputs are seeded synthetic tensors of that shape.
+the suffix KV (split-KV combine included).  Headline workload: the long
+assembled context of the Qwen3-8B layer geometry (hidden 4096, 32/8 heads,
+d 128, r 16; 64 artifacts of 2048 tokens = 131,072 cached keys plus a
+2048-token suffix, batch 1), with the same kernel timed on full causal
+attention over all 133,120 tokens beside it.  The Qwen3-4B prefill layer,
+the Qwen3-8B layer with 4 requests and the 64-request decode step follow as
+sub-objects of the same line, each with its own roofline.  Inputs are seeded
+synthetic tensors of those shapes.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--no-configs]
   python bench.py --impl reference ...   # the fp64 CPU oracle, timed on host cores
 
 Prints ONE JSON line (rank 0).  value = algorithmic attention FLOPs (or KV
 bytes for the decode workload) per step / device time per step, with the
 inputs resident in HBM; e2e = the same metric through the public API with
 the step's inputs copied from pinned host memory and its output copied back.
+The headline numbers are computed first; a later sub-object that fails
+records {"error": ...} in the line and the run exits non-zero.
 """
 
 from __future__ import annotations
@@ -32,6 +39,8 @@ if ROOT not in sys.path:
 
 METRIC = "artifact-KV attention TFLOP/s (prefill) & KV GB/s (decode), % of roofline"
 L2_FLUSH_BYTES = 512 << 20
+HEADLINE = "qwen3_8b_long_131k"
+SUB_CONFIGS = ("qwen3_4b_prefill", "qwen3_8b_prefill_4req", "qwen3_8b_decode_64req")
 
 
 def _peaks():
@@ -171,18 +180,51 @@ def oracle_sample(wl, inputs, tokens, decode: bool):
     vis = sum(t_art + (wl.S_kv - wl.S) + i + 1 for i in tokens)
     if decode:
         # every KV head's keys and values of the request are read once per token
-        work = float(sum(t_art + (wl.S_kv - wl.S) + i + 1 for i in tokens) * 2 * g.n_kv_heads * g.head_dim * 2)
+        work = float(vis * 2 * g.n_kv_heads * g.head_dim * 2)
     else:
         work = 4.0 * g.head_dim * g.n_q_heads * vis
     return dt, work
 
 
-def _single_thread_env():
+def host_threads_env():
+    """Let the oracle's BLAS use every host core: set before numpy loads."""
+    n = str(os.cpu_count() or 1)
     for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
-        os.environ.setdefault(k, "1")
+        os.environ[k] = n
+
+
+def blas_threads() -> int:
+    """Threads numpy's BLAS actually runs with (read from the loaded library),
+    else the thread count the environment asked for."""
+    try:
+        import threadpoolctl
+        info = [d for d in threadpoolctl.threadpool_info() if d.get("user_api") == "blas"]
+        if info:
+            return int(info[0]["num_threads"])
+    except Exception:
+        pass
+    try:
+        import ctypes
+        with open("/proc/self/maps") as f:
+            libs = sorted({ln.split()[-1] for ln in f
+                           if "openblas" in ln.split()[-1].lower() and ".so" in ln.split()[-1]})
+        for path in libs:
+            lib = ctypes.CDLL(path)
+            for sym in ("scipy_openblas_get_num_threads64_", "openblas_get_num_threads64_",
+                        "openblas_get_num_threads"):
+                fn = getattr(lib, sym, None)
+                if fn is not None:
+                    fn.restype = ctypes.c_int
+                    return int(fn())
+    except Exception:
+        pass
+    return int(os.environ.get("OPENBLAS_NUM_THREADS", "1"))
 
 
 def cpu_baseline(wl, budget_s: float = 12.0, seed: int = 0):
+    """The oracle on a bounded sample of request 0's suffix tokens (all q
+    heads), multithreaded BLAS on every host core; the metric is the sample's
+    work over its time, and the full step is extrapolated linearly by work."""
     import numpy as np
     decode = is_decode(wl)
     inputs = _oracle_inputs(wl, 0)
@@ -197,71 +239,78 @@ def cpu_baseline(wl, budget_s: float = 12.0, seed: int = 0):
         done_w += w
         n_tok += len(toks)
     scale = 1e9 if decode else 1e12
+    full = kv_bytes(wl) if decode else attention_flops(wl)
+    threads = blas_threads()
     return {"value": done_w / done_t / scale, "unit": "GB/s" if decode else "TFLOP/s",
-            "cores": int(os.environ.get("OPENBLAS_NUM_THREADS", "1")), "kind": "oracle",
-            "sample": f"request 0, {n_tok} suffix tokens x all {wl.geom.n_q_heads} q heads "
-                      f"(fp64 numpy, single-threaded BLAS), {done_t:.1f} s of CPU work"}
+            "cores": threads, "host_cpus": os.cpu_count(), "kind": "oracle",
+            "sample": f"request 0, {n_tok} random suffix tokens x all {wl.geom.n_q_heads} q heads of "
+                      f"{wl.n_req * wl.S} query tokens (fp64 numpy oracle, BLAS on {threads} threads), "
+                      f"{done_t:.1f} s of CPU work; the full step ({full / scale:.4g} "
+                      f"{'GB' if decode else 'TFLOP'}) extrapolated linearly by work: "
+                      f"{full * done_t / done_w:.4g} s"}
 
 
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
-def run_ours(args, rank, world, local_rank):
-    import torch
-    import paper_2609_36722_gb300 as pkg
-    from gen import make_kv_weights, make_workload
+class Bed:
+    """One workload loaded into a library context: registered artifacts, the
+    assembled plan and the step's output buffers, all resident on the GPU."""
 
-    dev = torch.device("cuda", local_rank)
-    torch.cuda.set_device(dev)
-    wl = make_workload(args.workload, device=dev)
-    g = wl.geom
-    decode = is_decode(wl)
-    ctx = pkg.Context.for_geometry(g, pool_blocks=sum(-(-L // 64) for L in wl.art_lengths) + 1, device=local_rank)
-    for k, v in zip(wl.art_k, wl.art_v):
-        ctx.register_artifact(k, v)
-    plan = ctx.assemble(wl.requests)
-    stream = torch.cuda.current_stream()
-    out = torch.empty(wl.n_req, wl.S, g.n_q_heads, g.head_dim, dtype=torch.bfloat16, device=dev)
-    lse = torch.empty(wl.n_req, wl.S, g.n_q_heads, dtype=torch.float32, device=dev)
-    q = torch.empty_like(out)
-    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    def __init__(self, name, dev, local_rank):
+        import torch
+        import paper_2609_36722_gb300 as pkg
+        from gen import make_workload
+        self.name = name
+        self.dev = dev
+        self.wl = wl = make_workload(name, device=dev)
+        self.g = g = wl.geom
+        self.decode = is_decode(wl)
+        self.ctx = pkg.Context.for_geometry(g, pool_blocks=sum(-(-L // 64) for L in wl.art_lengths) + 1,
+                                            device=local_rank)
+        for k, v in zip(wl.art_k, wl.art_v):
+            self.ctx.register_artifact(k, v)
+        self.plan = self.ctx.assemble(wl.requests)
+        self.out = torch.empty(wl.n_req, wl.S, g.n_q_heads, g.head_dim, dtype=torch.bfloat16, device=dev)
+        self.lse = torch.empty(wl.n_req, wl.S, g.n_q_heads, dtype=torch.float32, device=dev)
+        self.q = torch.empty_like(self.out)
+        self.work = kv_bytes(wl) if self.decode else attention_flops(wl)
+        self.scale = 1e9 if self.decode else 1e12
+        self.unit = "GB/s" if self.decode else "TFLOP/s"
 
-    def step(attn_events=False):
-        # attn_events: bracket the attention call with events (for the roofline).
-        # An event recorded between the two calls keeps the attention kernel
-        # from starting while the projection finishes (programmatic dependent
-        # launch needs kernel after kernel), so the step timing runs without.
-        if attn_events:
-            ev_q.record()
-        ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv, out=q)
-        n1 = ctx.last_launch_count()
-        if attn_events:
-            ev_a.record()
-        ctx.attend(plan, q, wl.suffix_k, wl.suffix_v, out=out, lse=lse)
-        if attn_events:
-            ev_b.record()
-        return n1 + ctx.last_launch_count()
+    def close(self):
+        import torch
+        self.plan.free()
+        self.ctx.close()
+        del self.wl, self.out, self.lse, self.q
+        torch.cuda.empty_cache()
 
-    class Eager:
-        # --eager: the same calls launched directly, with the events around them
-        # (profilers step through graph replays very slowly)
-        def __init__(self, fn, e0, e1):
-            self.fn, self.e0, self.e1 = fn, e0, e1
 
-        def replay(self):
-            self.e0.record()
-            self.fn()
-            self.e1.record()
+class Timer:
+    """Times callables on the device.  By default the calls are captured once
+    into a CUDA graph and every timed run replays it, with events recorded as
+    nodes inside the graph; with eager=True (for profilers, which step through
+    graph replays very slowly) the same calls are launched directly."""
 
-    def graphed(fn):
-        # The timed work replays a CUDA graph of the calls: one launch for the
-        # host, so the GPU never waits on the Python binding or the per-call
-        # host setup between kernels.  Events inside the graph time it on the
-        # device.
-        if args.eager:
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            return Eager(fn, e0, e1), e0, e1
-        e0, e1 = gevent(), gevent()
+    def __init__(self, eager, flush):
+        self.eager = eager
+        self.flush = flush
+
+    def event(self):
+        import torch
+        # an event that a captured graph records as a node of its own
+        return torch.cuda.Event(enable_timing=True, external=not self.eager)
+
+    def graphed(self, fn):
+        import torch
+        e0, e1 = self.event(), self.event()
+        if self.eager:
+            class Eager:
+                def replay(_):
+                    e0.record()
+                    fn()
+                    e1.record()
+            return Eager(), e0, e1
         for _ in range(3):
             fn()
         torch.cuda.synchronize()
@@ -273,288 +322,428 @@ def run_ours(args, rank, world, local_rank):
         torch.cuda.synchronize()
         return gr, e0, e1
 
-    def gevent():
-        # an event that a captured graph records as a node of its own
-        return torch.cuda.Event(enable_timing=True, external=not args.eager)
+    def time(self, fn, steps):
+        """ms of each of `steps` runs of fn, L2 flushed before each (outside the events)."""
+        gr, e0, e1 = self.graphed(fn)
+        ms = []
+        for _ in range(steps):
+            self.flush.zero_()
+            gr.replay()
+            e1.synchronize()
+            ms.append(e0.elapsed_time(e1))
+        return ms
 
-    ev_q, ev_a, ev_b = gevent(), gevent(), gevent()
+
+def measure_core(bed, args, world, timer, with_clocks=False, local_rank=0):
+    """Device-resident timing of one workload: the step (Q projection +
+    attention) for the value, and the same step with events around the
+    attention call for the roofline."""
+    import torch
+    wl, g, ctx, plan = bed.wl, bed.g, bed.ctx, bed.plan
+    ev_q, ev_a, ev_b = timer.event(), timer.event(), timer.event()
+
+    def step(attn_events=False):
+        # attn_events: bracket the attention call with events (for the roofline).
+        # An event recorded between the two calls keeps the attention kernel
+        # from starting while the projection finishes (programmatic dependent
+        # launch needs kernel after kernel), so the step timing runs without.
+        if attn_events:
+            ev_q.record()
+        ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv, out=bed.q)
+        n1 = ctx.last_launch_count()
+        if attn_events:
+            ev_a.record()
+        ctx.attend(plan, bed.q, wl.suffix_k, wl.suffix_v, out=bed.out, lse=bed.lse)
+        if attn_events:
+            ev_b.record()
+        return n1 + ctx.last_launch_count()
+
+    launches_per_step = 0
     for _ in range(args.warmup):
         launches_per_step = step()
     torch.cuda.synchronize()
-    assert ctx.sync_status() == 0
-    g_step, ev_s, ev_e = graphed(step)
-    g_parts, _, _ = graphed(lambda: step(attn_events=True))
-    assert ctx.sync_status() == 0
-
-    sampler = ClockSampler(local_rank) if rank == 0 else None
+    if ctx.sync_status() != 0:
+        raise RuntimeError(f"{bed.name}: device status after the warm-up steps")
+    g_step, ev_s, ev_e = timer.graphed(step)
+    g_parts, _, _ = timer.graphed(lambda: step(attn_events=True))
+    sampler = ClockSampler(local_rank) if with_clocks else None
     # keep the GPU busy ~1 s before timing so the clock samples describe the timed region
-    t_end = time.perf_counter() + 1.0
+    t_end = time.perf_counter() + (1.0 if with_clocks else 0.0)
     while time.perf_counter() < t_end:
         g_step.replay()
         torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    attn_ms = []
-    qproj_ms = []
     step_ms = []
-    launches = 0
-    for i in range(args.steps):
-        flush.zero_()                                   # L2 flush between steps, outside the timed events
+    for _ in range(args.steps):
+        timer.flush.zero_()                                   # L2 flush between steps, outside the events
         g_step.replay()
         ev_e.synchronize()
         step_ms.append(ev_s.elapsed_time(ev_e))
-        launches += launches_per_step
     torch.cuda.synchronize()
+    total_ms = max_over_ranks(sum(step_ms), world, bed.dev)
+    clocks = sampler.stop() if sampler else None
     # the same steps again with events around the attention call: its launch
     # duration for the roofline
-    for i in range(args.steps):
-        flush.zero_()
+    attn_ms, qproj_ms = [], []
+    for _ in range(args.steps):
+        timer.flush.zero_()
         g_parts.replay()
         ev_b.synchronize()
         attn_ms.append(ev_a.elapsed_time(ev_b))
         qproj_ms.append(ev_q.elapsed_time(ev_a))
     torch.cuda.synchronize()
-    # the suffix tokens' K/V projection, its own line: same x,
-    # base k_proj / v_proj weights of the geometry, into scratch suffix buffers
-    wk, wv, kn = make_kv_weights(g, 0, device=dev)
-    sk_s, sv_s = wl.suffix_k.clone(), wl.suffix_v.clone()
-    kv_ms = []
-    g_kv, e0, e1 = graphed(lambda: ctx.kv_project(plan, wl.x, wk, wv, kn, sk_s, sv_s))
-    for i in range(args.steps):
-        flush.zero_()
-        g_kv.replay()
-        e1.synchronize()
-        kv_ms.append(e0.elapsed_time(e1))
-    kv_flops = 2.0 * wl.n_req * wl.S * g.hidden * 2 * g.n_kv_heads * g.head_dim
-    # the paper's skills layout: a 16-token online system span,
-    # 5-token online separators between the artifacts, the rest of the online
-    # rows (the task) last; every online row is a query (S = S_kv)
-    lay_ms, lay_flops = [], 0.0
-    if wl.S == wl.S_kv:
-        layouts = []
-        for r in wl.requests:
-            lay = [-16]
-            for k, a in enumerate(r):
-                lay += ([a] if k == 0 else [-5, a])
-            layouts.append(lay)
-        if all(16 + 5 * (len(r) - 1) <= wl.S_kv for r in wl.requests):
-            lplan = ctx.assemble_layout(layouts)
-            for r, lay in enumerate(layouts):
-                at, online_pos = 0, []
-                for it in lay:
-                    if it >= 0:
-                        at += wl.art_lengths[it]
-                    else:
-                        online_pos += list(range(at, at - it))
-                        at += -it
-                online_pos += list(range(at, at + wl.S_kv - len(online_pos)))
-                lay_flops += 4.0 * g.head_dim * g.n_q_heads * sum(p_ + 1 for p_ in online_pos[wl.S_kv - wl.S:])
-            g_lay, e0, e1 = graphed(lambda: ctx.attend(lplan, q, wl.suffix_k, wl.suffix_v, out=out, lse=lse))
-            for i in range(args.steps):
-                flush.zero_()
-                g_lay.replay()
-                e1.synchronize()
-                lay_ms.append(e0.elapsed_time(e1))
-            del g_lay
-            lplan.free()
-    # the 131k-key layer's analogue: the same attention kernel on full causal
-    # attention over the whole assembled sequence (an empty plan: every token a
-    # query), i.e. the prefill the cached artifacts avoid; reported with the
-    # wall-time ratio full / cached
-    full_ms, full_flops, n_full = [], 0.0, 0
-    if args.workload == "qwen3_8b_long_131k":
-        n_full = wl.t_art(0) + wl.S_kv
-        gen = torch.Generator(device=dev).manual_seed(4)
-        qf = torch.randn(1, n_full, g.n_q_heads, g.head_dim, device=dev, dtype=torch.bfloat16, generator=gen)
-        kf = torch.randn(1, n_full, g.n_kv_heads, g.head_dim, device=dev, dtype=torch.bfloat16, generator=gen)
-        vf = torch.randn(1, n_full, g.n_kv_heads, g.head_dim, device=dev, dtype=torch.bfloat16, generator=gen)
-        of = torch.empty_like(qf)
-        fplan = ctx.assemble([[]])
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        for i in range(5):
-            e0.record()
-            ctx.attend(fplan, qf, kf, vf, out=of, want_lse=False)
-            e1.record()
-            e1.synchronize()
-            if i >= 2:
-                full_ms.append(e0.elapsed_time(e1))
-        full_flops = 4.0 * g.head_dim * g.n_q_heads * n_full * (n_full + 1) / 2
-        fplan.free()
-        del qf, kf, vf, of
-    total_ms = sum(step_ms)
-    total_ms = max_over_ranks(total_ms, world, dev)
-    clocks = sampler.stop() if sampler else None
     st = ctx.sync_status()
     if st != 0:
-        raise RuntimeError(f"device status {st} after the timed region")
+        raise RuntimeError(f"{bed.name}: device status {st} after the timed region")
+    del g_step, g_parts
+    peaks = _peaks()
+    attn_avg = statistics.mean(attn_ms)
+    achieved = bed.work / (attn_avg * 1e-3) / bed.scale
+    peak = peaks["hbm"] if bed.decode else peaks["bf16"]
+    qp_avg = statistics.mean(qproj_ms)
+    qp_tf = qproj_flops(wl) / (qp_avg * 1e-3) / 1e12
+    # the Q projection's own bound: its FLOPs at the bf16 peak, or its
+    # operand bytes (x, W_q, A, B, q_norm weight, Q out) at the copy bandwidth
+    qp_bytes = 2.0 * (wl.n_req * wl.S * g.hidden + g.d_q * g.hidden + g.rank * g.hidden + g.d_q * g.rank + g.head_dim
+                      + wl.n_req * wl.S * g.d_q)
+    qp_bound_ms = max(qproj_flops(wl) / (peaks["bf16"] * 1e12), qp_bytes / (peaks["hbm"] * 1e9)) * 1e3
+    return {
+        "value": round(job_throughput(bed.work, world, args.steps, total_ms * 1e-3) / bed.scale, 3),
+        "unit": bed.unit,
+        "ms_per_step": round(total_ms / args.steps, 5),
+        "roofline": {"bound": "hbm" if bed.decode else "tensor", "achieved": round(achieved, 3), "peak": peak,
+                     "unit": bed.unit, "frac": round(achieved / peak, 4), "traffic": load_traffic(bed.name),
+                     "kernel": ("attn_mma_kernel + combine_kernel" if bed.decode
+                                else "attn_tc_kernel (split-KV chunks merged inside it)"),
+                     "work_per_launch": bed.work,
+                     "work_unit": "bytes (each request's assembled K and V read once)" if bed.decode
+                                  else "FLOP (4 d Hq per visible query-key pair)",
+                     "peak_source": f"{peaks['src']} ({'hbm_gbs' if bed.decode else 'bf16_tflops burst'})",
+                     "avg_launch_ms": round(attn_avg, 5)},
+        "qproj": {"avg_call_ms": round(qp_avg, 5), "tflops": round(qp_tf, 3),
+                  "frac_of_bf16_peak": round(qp_tf / peaks["bf16"], 4),
+                  "bound_ms": round(qp_bound_ms, 5), "frac_of_bound": round(qp_bound_ms / qp_avg, 4)},
+        "path_work": {"attention_flops": attention_flops(wl), "qproj_flops": qproj_flops(wl),
+                      "kv_bytes": kv_bytes(wl)},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks,
+        "workload": {"hidden": g.hidden, "n_q_heads": g.n_q_heads, "n_kv_heads": g.n_kv_heads,
+                     "head_dim": g.head_dim, "lora_rank": g.rank, "s": g.scale, "n_req": wl.n_req, "S": wl.S,
+                     "S_kv": wl.S_kv, "t_art": [wl.t_art(r) for r in range(wl.n_req)][:8],
+                     "artifacts_per_req": [len(r) for r in wl.requests][:8]},
+    }
 
-    # ---- end to end through the public API with host buffers.  A step's inputs
-    # are its S new tokens: their hidden states and their own K/V rows (the last S
-    # of each request's S_kv suffix rows).  The S_kv - S earlier suffix rows of a
-    # decode step are the request's resident cache, written by earlier steps: they
-    # stay on the device, as the artifact pool does.
-    x_h = wl.x.cpu().pin_memory()
-    S_old = wl.S_kv - wl.S
-    sk_h = wl.suffix_k[:, S_old:].cpu().contiguous().pin_memory()
-    sv_h = wl.suffix_v[:, S_old:].cpu().contiguous().pin_memory()
-    out_h = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
-    x_d = torch.empty_like(wl.x)
-    sk_d = wl.suffix_k.clone()
-    sv_d = wl.suffix_v.clone()
-    sk_new = torch.empty(sk_h.shape, dtype=sk_h.dtype, device=dev)
-    sv_new = torch.empty(sv_h.shape, dtype=sv_h.dtype, device=dev)
 
-    def copy_inputs():
-        x_d.copy_(x_h, non_blocking=True)
-        if S_old:
-            sk_new.copy_(sk_h, non_blocking=True)
-            sv_new.copy_(sv_h, non_blocking=True)
-            sk_d[:, S_old:].copy_(sk_new)
-            sv_d[:, S_old:].copy_(sv_new)
+class HostInputs:
+    """A step's inputs in pinned host memory and their device buffers: the
+    new tokens' hidden states and their own suffix K/V rows (the last S of
+    each request's S_kv rows).  A decode step's earlier suffix rows are the
+    request's resident cache, written by earlier steps: they stay on the
+    device, as the artifact pool does."""
+
+    def __init__(self, bed):
+        import torch
+        wl = bed.wl
+        self.S_old = S_old = wl.S_kv - wl.S
+        self.x_h = wl.x.cpu().pin_memory()
+        self.sk_h = wl.suffix_k[:, S_old:].cpu().contiguous().pin_memory()
+        self.sv_h = wl.suffix_v[:, S_old:].cpu().contiguous().pin_memory()
+        self.out_h = torch.empty(bed.out.shape, dtype=bed.out.dtype, pin_memory=True)
+        self.x_d = torch.empty_like(wl.x)
+        self.sk_d = wl.suffix_k.clone()
+        self.sv_d = wl.suffix_v.clone()
+        self.sk_new = torch.empty(self.sk_h.shape, dtype=self.sk_h.dtype, device=bed.dev)
+        self.sv_new = torch.empty(self.sv_h.shape, dtype=self.sv_h.dtype, device=bed.dev)
+        self.h2d_bytes = (self.x_h.numel() + self.sk_h.numel() + self.sv_h.numel()) * 2
+        self.d2h_bytes = self.out_h.numel() * 2
+
+    def copy_in(self):
+        self.x_d.copy_(self.x_h, non_blocking=True)
+        if self.S_old:
+            self.sk_new.copy_(self.sk_h, non_blocking=True)
+            self.sv_new.copy_(self.sv_h, non_blocking=True)
+            self.sk_d[:, self.S_old:].copy_(self.sk_new)
+            self.sv_d[:, self.S_old:].copy_(self.sv_new)
         else:
-            sk_d.copy_(sk_h, non_blocking=True)
-            sv_d.copy_(sv_h, non_blocking=True)
+            self.sk_d.copy_(self.sk_h, non_blocking=True)
+            self.sv_d.copy_(self.sv_h, non_blocking=True)
 
+
+def measure_e2e(bed, args, world, flush):
+    """The same metric through the public API with host buffers: every step
+    assembles its plan, copies its new tokens' inputs from pinned host memory
+    (their hidden states and their own suffix K/V rows; a decode step's
+    earlier suffix rows are the request's resident cache, like the artifact
+    pool), runs attuner_query_attend and copies O back, all inside the
+    host-timed region."""
+    import torch
+    wl, g, ctx = bed.wl, bed.g, bed.ctx
+    io = HostInputs(bed)
     def e2e_step():
         p = ctx.assemble(wl.requests)
-        copy_inputs()
-        ctx.query_attend(p, x_d, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, sk_d, sv_d, out=out,
-                         want_lse=False)
-        out_h.copy_(out, non_blocking=True)
+        io.copy_in()
+        ctx.query_attend(p, io.x_d, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, io.sk_d, io.sv_d,
+                         out=bed.out, want_lse=False)
+        io.out_h.copy_(bed.out, non_blocking=True)
         torch.cuda.synchronize()
         p.free()
 
     for _ in range(max(3, args.warmup)):
         e2e_step()
-    e2e_times = []
+    times = []
     for _ in range(args.steps):
         flush.zero_()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         e2e_step()
-        e2e_times.append(time.perf_counter() - t0)
-    e2e_s = sum(e2e_times)
-    e2e_s = max_over_ranks(e2e_s, world, dev)
-    h2d = (x_h.numel() + sk_h.numel() + sv_h.numel()) * 2
-    d2h = out_h.numel() * 2
+        times.append(time.perf_counter() - t0)
+    e2e_s = max_over_ranks(sum(times), world, bed.dev)
+    if ctx.sync_status() != 0:
+        raise RuntimeError(f"{bed.name}: device status after the end-to-end steps")
+    return {"value": round(job_throughput(bed.work, world, args.steps, e2e_s) / bed.scale, 3), "unit": bed.unit,
+            "h2d_bytes_per_step": io.h2d_bytes, "d2h_bytes_per_step": io.d2h_bytes,
+            "ms_per_step": round(e2e_s * 1e3 / args.steps, 4),
+            "includes": "assemble (host block table + H2D), H2D of the step's new tokens (x and their own "
+                        "suffix K/V rows; a decode step's earlier suffix rows stay resident), query_attend, "
+                        "D2H of O"}
 
-    # ---- warm-cache end to end: the request's artifacts start in pinned host
-    # memory (the paper's CPU RAM cache) and are loaded into an emptied pool in
-    # every step, on a second stream that overlaps the Q projection
+
+def measure_full_causal(bed, reps=5):
+    """The 131k-key layer's analogue of the paper's reuse-vs-full-prefill
+    speedup: the same attention kernel on full causal attention over the
+    whole assembled sequence (an empty plan: every token a query), i.e. the
+    prefill the cached artifacts avoid."""
+    import torch
+    wl, g, ctx = bed.wl, bed.g, bed.ctx
+    n_full = wl.t_art(0) + wl.S_kv
+    gen = torch.Generator(device=bed.dev).manual_seed(4)
+    qf = torch.randn(1, n_full, g.n_q_heads, g.head_dim, device=bed.dev, dtype=torch.bfloat16, generator=gen)
+    kf = torch.randn(1, n_full, g.n_kv_heads, g.head_dim, device=bed.dev, dtype=torch.bfloat16, generator=gen)
+    vf = torch.randn(1, n_full, g.n_kv_heads, g.head_dim, device=bed.dev, dtype=torch.bfloat16, generator=gen)
+    of = torch.empty_like(qf)
+    fplan = ctx.assemble([[]])
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ms = []
+    for i in range(reps):
+        e0.record()
+        ctx.attend(fplan, qf, kf, vf, out=of, want_lse=False)
+        e1.record()
+        e1.synchronize()
+        if i >= 2:
+            ms.append(e0.elapsed_time(e1))
+    fplan.free()
+    if ctx.sync_status() != 0:
+        raise RuntimeError("device status after the full causal analogue")
+    flops = 4.0 * g.head_dim * g.n_q_heads * n_full * (n_full + 1) / 2
+    return n_full, statistics.mean(ms), flops
+
+
+def measure_kv_project(bed, args, timer):
+    """The suffix tokens' K/V projection: same x, base k_proj / v_proj weights
+    of the geometry, into scratch suffix buffers."""
+    from gen import make_kv_weights
+    wl, g, ctx = bed.wl, bed.g, bed.ctx
+    wk, wv, kn = make_kv_weights(g, 0, device=bed.dev)
+    sk_s, sv_s = wl.suffix_k.clone(), wl.suffix_v.clone()
+    ms = timer.time(lambda: ctx.kv_project(bed.plan, wl.x, wk, wv, kn, sk_s, sv_s), args.steps)
+    flops = 2.0 * wl.n_req * wl.S * g.hidden * 2 * g.n_kv_heads * g.head_dim
+    if ctx.sync_status() != 0:
+        raise RuntimeError("device status after kv_project")
+    return {"avg_call_ms": round(statistics.mean(ms), 5),
+            "tflops": round(flops / (statistics.mean(ms) * 1e-3) / 1e12, 3)}
+
+
+def measure_layout(bed, args, timer):
+    """The paper's skills layout: a 16-token online system span, 5-token
+    online separators between the artifacts, the rest of the online rows (the
+    task) last; every online row is a query (S = S_kv)."""
+    wl, g, ctx = bed.wl, bed.g, bed.ctx
+    if wl.S != wl.S_kv:
+        return None
+    layouts = []
+    for r in wl.requests:
+        lay = [-16]
+        for k, a in enumerate(r):
+            lay += ([a] if k == 0 else [-5, a])
+        layouts.append(lay)
+    if not all(16 + 5 * (len(r) - 1) <= wl.S_kv for r in wl.requests):
+        return None
+    lplan = ctx.assemble_layout(layouts)
+    flops = 0.0
+    for lay in layouts:
+        at, online_pos = 0, []
+        for it in lay:
+            if it >= 0:
+                at += wl.art_lengths[it]
+            else:
+                online_pos += list(range(at, at - it))
+                at += -it
+        online_pos += list(range(at, at + wl.S_kv - len(online_pos)))
+        flops += 4.0 * g.head_dim * g.n_q_heads * sum(p_ + 1 for p_ in online_pos[wl.S_kv - wl.S:])
+    ms = timer.time(lambda: ctx.attend(lplan, bed.q, wl.suffix_k, wl.suffix_v, out=bed.out, lse=bed.lse),
+                    args.steps)
+    lplan.free()
+    if ctx.sync_status() != 0:
+        raise RuntimeError("device status after the layout attention")
+    return {"avg_call_ms": round(statistics.mean(ms), 5),
+            "tflops": round(flops / (statistics.mean(ms) * 1e-3) / 1e12, 3),
+            "layout": "online system span 16, artifacts with 5-token online separators, task last"}
+
+
+def measure_warm_cache(bed, args, world, flush, local_rank):
+    """Warm-cache end to end: the request's artifacts start in pinned host
+    memory (the paper's CPU RAM cache) and are loaded into an emptied pool in
+    every step, on a second stream that overlaps the Q projection."""
+    import torch
+    import paper_2609_36722_gb300 as pkg
+    wl, g = bed.wl, bed.g
+    stream = torch.cuda.current_stream()
     used = sorted({a for r in wl.requests for a in r})
     remap = {a: i for i, a in enumerate(used)}
     reqs_w = [[remap[a] for a in r] for r in wl.requests]
     ak_h = [wl.art_k[a].cpu().pin_memory() for a in used]
     av_h = [wl.art_v[a].cpu().pin_memory() for a in used]
     art_bytes = sum(t.numel() * 2 for t in ak_h) * 2
+    io = HostInputs(bed)
     wctx = pkg.Context.for_geometry(g, pool_blocks=sum(-(-wl.art_lengths[a] // 64) for a in used) + 1,
                                     device=local_rank)
-    side = torch.cuda.Stream(device=dev)
-    q_w = torch.empty_like(q)
+    side = torch.cuda.Stream(device=bed.dev)
+    q_w = torch.empty_like(bed.q)
     ev_l0 = torch.cuda.Event(enable_timing=True)
     ev_l1 = torch.cuda.Event(enable_timing=True)
 
-    def load_warm():
+    def warm_step():
         wctx.pool_reset()
         side.wait_stream(stream)
         ev_l0.record(side)
         for i in range(0, len(used), 64):
             wctx.register_artifacts_host(ak_h[i:i + 64], av_h[i:i + 64], stream=side)
         ev_l1.record(side)
-
-    def warm_step():
-        load_warm()
         p = wctx.assemble(reqs_w)
-        copy_inputs()
-        wctx.q_project(p, x_d, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv, out=q_w)
+        io.copy_in()
+        wctx.q_project(p, io.x_d, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv, out=q_w)
         stream.wait_stream(side)
-        wctx.attend(p, q_w, sk_d, sv_d, out=out, want_lse=False)
-        out_h.copy_(out, non_blocking=True)
+        wctx.attend(p, q_w, io.sk_d, io.sv_d, out=bed.out, want_lse=False)
+        io.out_h.copy_(bed.out, non_blocking=True)
         torch.cuda.synchronize()
         p.free()
 
-    for _ in range(max(3, args.warmup)):
-        warm_step()
-    warm_times, load_ms = [], []
-    for _ in range(args.steps):
-        flush.zero_()
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        warm_step()
-        warm_times.append(time.perf_counter() - t0)
-        load_ms.append(ev_l0.elapsed_time(ev_l1))
-    if wctx.sync_status() != 0:
-        raise RuntimeError("device status after the warm-cache steps")
-    warm_s = sum(warm_times)
-    warm_s = max_over_ranks(warm_s, world, dev)
-    wctx.close()
+    try:
+        for _ in range(max(3, args.warmup)):
+            warm_step()
+        times, load_ms = [], []
+        for _ in range(args.steps):
+            flush.zero_()
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            warm_step()
+            times.append(time.perf_counter() - t0)
+            load_ms.append(ev_l0.elapsed_time(ev_l1))
+        if wctx.sync_status() != 0:
+            raise RuntimeError("device status after the warm-cache steps")
+    finally:
+        wctx.close()
+    warm_s = max_over_ranks(sum(times), world, bed.dev)
+    return {"value": round(job_throughput(bed.work, world, args.steps, warm_s) / bed.scale, 3), "unit": bed.unit,
+            "h2d_bytes_per_step": io.h2d_bytes + art_bytes, "d2h_bytes_per_step": io.d2h_bytes,
+            "artifact_load_ms": round(statistics.mean(load_ms), 4),
+            "artifact_load_gbs": round(art_bytes / (statistics.mean(load_ms) * 1e-3) / 1e9, 1),
+            "includes": "pool reset, load of the requests' artifact K/V from pinned host memory (one kernel "
+                        "over the CPU-GPU link, second stream, overlapping the Q projection), assemble, H2D of "
+                        "the step's new tokens (x and their own suffix K/V rows), Q projection, attention, D2H of O"}
 
-    peaks = _peaks()
-    work = kv_bytes(wl) if decode else attention_flops(wl)
-    scale = 1e9 if decode else 1e12
-    unit = "GB/s" if decode else "TFLOP/s"
-    value = job_throughput(work, world, args.steps, total_ms * 1e-3) / scale
-    attn_avg_ms = statistics.mean(attn_ms)
-    achieved = work / (attn_avg_ms * 1e-3) / scale
-    peak = peaks["hbm"] if decode else peaks["bf16"]
-    traffic = load_traffic(args.workload)
+
+def _guarded(fn, errors, label):
+    """Run an optional part of the line; a failure is recorded, not raised."""
+    import traceback
+    try:
+        return fn()
+    except Exception as e:  # noqa: BLE001 - reported in the line, and the run exits non-zero
+        traceback.print_exc()
+        errors.append(label)
+        return {"error": f"{type(e).__name__}: {e}"}
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    timer = Timer(args.eager, flush)
+    errors = []
+
+    # ---- the headline: computed first, and a failure here fails the run
+    bed = Bed(args.workload, dev, local_rank)
+    core = measure_core(bed, args, world, timer, with_clocks=(rank == 0), local_rank=local_rank)
+    e2e = measure_e2e(bed, args, world, flush)
+    full = None
+    if args.workload == HEADLINE:
+        n_full, full_ms, full_flops = measure_full_causal(bed)
+        full = {"tokens": n_full, "avg_call_ms": round(full_ms, 3),
+                "tflops": round(full_flops / (full_ms * 1e-3) / 1e12, 3),
+                "frac_of_bf16_peak": round(full_flops / (full_ms * 1e-3) / 1e12 / _peaks()["bf16"], 4),
+                "flops": full_flops,
+                "work_ratio_full_over_cached": round(full_flops / bed.work, 2),
+                "wall_ratio_full_over_cached": round(full_ms / core["roofline"]["avg_launch_ms"], 2)}
     result = {
-        "metric": METRIC, "value": round(value, 3), "unit": unit, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
+        "metric": METRIC, "value": core["value"], "unit": core["unit"], "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": core["ms_per_step"], "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": args.workload, "hidden": g.hidden, "n_q_heads": g.n_q_heads,
-                   "n_kv_heads": g.n_kv_heads, "head_dim": g.head_dim, "lora_rank": g.rank, "s": g.scale,
-                   "n_req": wl.n_req, "S": wl.S, "S_kv": wl.S_kv,
-                   "t_art": [wl.t_art(r) for r in range(wl.n_req)][:8],
-                   "artifacts_per_req": [len(r) for r in wl.requests][:8],
+        "config": {"workload": args.workload, **core["workload"],
                    "parallelism": f"replicas x{world}",
                    "l2": f"flushed between timed steps ({L2_FLUSH_BYTES >> 20} MiB write, outside the events)",
-                   "attention_kernel": "tcgen05 (attn_tc)" if not decode else "split-KV warp-MMA (attn_mma)",
+                   "attention_kernel": "split-KV warp-MMA (attn_mma)" if bed.decode else "tcgen05 (attn_tc)",
                    "launch": "eager calls" if args.eager else "CUDA graph replay of the calls"},
-        "roofline": {"bound": "hbm" if decode else "tensor", "achieved": round(achieved, 3), "peak": peak,
-                     "unit": unit, "frac": round(achieved / peak, 4), "traffic": traffic,
-                     "kernel": ("attn_mma_kernel + combine_kernel" if decode else "attn_tc_kernel (split-KV chunks merged inside it)"),
-                     "peak_source": f"{peaks['src']} ({'hbm_gbs' if decode else 'bf16_tflops burst'})",
-                     "avg_launch_ms": round(attn_avg_ms, 5)},
-        "path_work": {"attention_flops": attention_flops(wl), "qproj_flops": qproj_flops(wl),
-                      "kv_bytes": kv_bytes(wl)},
-        # the Q projection (steps a1-a3: prep + qproj kernels) as its own line, from the same pass
-        "layout_attention": ({"avg_call_ms": round(statistics.mean(lay_ms), 5),
-                              "tflops": round(lay_flops / (statistics.mean(lay_ms) * 1e-3) / 1e12, 3),
-                              "layout": "online system span 16, artifacts with 5-token online separators, task last"}
-                             if lay_ms else None),
-        "full_causal_analogue": ({"tokens": n_full, "avg_call_ms": round(statistics.mean(full_ms), 3),
-                                  "tflops": round(full_flops / (statistics.mean(full_ms) * 1e-3) / 1e12, 3),
-                                  "wall_ratio_full_over_cached": round(statistics.mean(full_ms) / attn_avg_ms, 2)}
-                                 if full_ms else None),
-        "kv_project": {"avg_call_ms": round(statistics.mean(kv_ms), 5),
-                       "tflops": round(kv_flops / (statistics.mean(kv_ms) * 1e-3) / 1e12, 3)},
-        "qproj": {"avg_call_ms": round(statistics.mean(qproj_ms), 5),
-                  "tflops": round(qproj_flops(wl) / (statistics.mean(qproj_ms) * 1e-3) / 1e12, 3),
-                  "frac_of_bf16_peak": round(qproj_flops(wl) / (statistics.mean(qproj_ms) * 1e-3) / 1e12 / peaks["bf16"], 4)},
-        "e2e": {"value": round(job_throughput(work, world, args.steps, e2e_s) / scale, 3), "unit": unit,
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "includes": "assemble (host block table + H2D), H2D of the step's new tokens (x and their own "
-                            "suffix K/V rows; a decode step's earlier suffix rows stay resident), query_attend, "
-                            "D2H of O"},
-        "e2e_warm_cache": {"value": round(job_throughput(work, world, args.steps, warm_s) / scale, 3), "unit": unit,
-                           "h2d_bytes_per_step": h2d + art_bytes, "d2h_bytes_per_step": d2h,
-                           "artifact_load_ms": round(statistics.mean(load_ms), 4),
-                           "artifact_load_gbs": round(art_bytes / (statistics.mean(load_ms) * 1e-3) / 1e9, 1),
-                           "includes": "pool reset, load of the requests' artifact K/V from pinned host memory "
-                                       "(one kernel over the CPU-GPU link, second stream, overlapping the Q "
-                                       "projection), assemble, H2D of the step's new tokens (x and their "
-                                       "own suffix K/V rows), Q projection, "
-                                       "attention, D2H of O"},
-        "gpu_launches": launches,
-        "clocks": clocks,
+        "roofline": core["roofline"],
+        "e2e": e2e,
+        "gpu_launches": core["gpu_launches"],
+        "clocks": core["clocks"],
+        "qproj": core["qproj"],
+        "path_work": core["path_work"],
+        "full_causal_analogue": full,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        result["cpu_baseline"] = cpu_baseline(wl)
-    plan.free()
-    ctx.close()
-    return result
+        result["cpu_baseline"] = cpu_baseline(bed.wl)
+
+    # ---- optional parts: each failure is recorded in the line
+    def extras(b):
+        out = {}
+        if args.sub_lines:
+            out["kv_project"] = _guarded(lambda: measure_kv_project(b, args, timer), errors, f"{b.name}.kv_project")
+            out["layout_attention"] = _guarded(lambda: measure_layout(b, args, timer), errors,
+                                               f"{b.name}.layout_attention")
+            out["e2e_warm_cache"] = _guarded(lambda: measure_warm_cache(b, args, world, flush, local_rank), errors,
+                                             f"{b.name}.e2e_warm_cache")
+        return out
+
+    result.update(extras(bed))
+    bed.close()
+    del bed
+    configs = {}
+    if not args.no_configs:
+        for name in SUB_CONFIGS:
+            if name == args.workload:
+                continue
+
+            def one(name=name):
+                b = Bed(name, dev, local_rank)
+                try:
+                    c = measure_core(b, args, world, timer, local_rank=local_rank)
+                    d = {"value": c["value"], "unit": c["unit"], "ms_per_step": c["ms_per_step"],
+                         "roofline": c["roofline"], "qproj": c["qproj"], "gpu_launches": c["gpu_launches"],
+                         "config": c["workload"], "path_work": c["path_work"]}
+                    d["e2e"] = _guarded(lambda: measure_e2e(b, args, world, flush), errors, f"{name}.e2e")
+                    d.update(extras(b))
+                    return d
+                finally:
+                    b.close()
+            configs[name] = _guarded(one, errors, name)
+    result["configs"] = configs
+    if errors:
+        result["errors"] = errors
+    return result, (1 if errors else 0)
 
 
 def load_traffic(workload):
@@ -589,7 +778,8 @@ def run_reference(args):
     decode = is_decode(wl)
     inputs = _oracle_inputs(wl, 0)
     rng = np.random.default_rng(0)
-    toks_per_step = max(1, min(4, wl.S))
+    # a bounded sample per step: fewer tokens where every query row sees more keys
+    toks_per_step = max(1, min(4, wl.S, int(4 * 16384 / max(1, wl.t_art(0) + wl.S_kv)) or 1))
     for _ in range(args.warmup):
         oracle_sample(wl, inputs, sorted(rng.choice(wl.S, size=toks_per_step, replace=False).tolist()), decode)
     tot_t, tot_w = 0.0, 0.0
@@ -601,13 +791,17 @@ def run_reference(args):
     scale = 1e9 if decode else 1e12
     unit = "GB/s" if decode else "TFLOP/s"
     value = tot_w / tot_t / scale
-    sample = (f"per step: request 0, {toks_per_step} random suffix tokens x all {wl.geom.n_q_heads} q heads "
-              f"(fp64 numpy oracle, single-threaded BLAS)")
+    threads = blas_threads()
+    full = kv_bytes(wl) if decode else attention_flops(wl)
+    sample = (f"per step: request 0, {toks_per_step} random suffix tokens x all {wl.geom.n_q_heads} q heads of "
+              f"{wl.n_req * wl.S} query tokens (fp64 numpy oracle, BLAS on {threads} threads); the full step "
+              f"extrapolated linearly by work: {full * tot_t / tot_w:.4g} s")
     return {"metric": METRIC, "value": value, "unit": unit, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": tot_t * 1e3 / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
             "config": {"workload": args.workload, "parallelism": "host cores"},
-            "cpu_baseline": {"value": value, "unit": unit, "cores": 1, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": unit, "cores": threads, "host_cpus": os.cpu_count(),
+                             "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
@@ -617,8 +811,12 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="qwen3_4b_prefill")
+    ap.add_argument("--workload", default=HEADLINE)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="time the headline workload only (no per-config sub-objects)")
+    ap.add_argument("--no-sub-lines", dest="sub_lines", action="store_false",
+                    help="skip the kv_project, layout_attention and e2e_warm_cache sub-lines")
     ap.add_argument("--eager", action="store_true",
                     help="launch the timed calls directly instead of replaying CUDA graphs (for profilers)")
     args = ap.parse_args()
@@ -629,25 +827,26 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
 
+    host_threads_env()
     if args.impl == "reference":
-        _single_thread_env()
         if rank != 0:
             return
         print(json.dumps(run_reference(args)))
         return
 
-    _single_thread_env()
     if world > 1:
         import torch
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
-    res = run_ours(args, rank, world, local_rank)
+    res, rc = run_ours(args, rank, world, local_rank)
     if rank == 0:
         print(json.dumps(res))
     if world > 1:
         import torch
         torch.distributed.barrier()
         torch.distributed.destroy_process_group()
+    if rc:
+        sys.exit(rc)
 
 
 if __name__ == "__main__":
