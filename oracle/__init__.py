@@ -19,7 +19,12 @@ Every function is a plain restatement of the paper's definitions in float64:
     adaptation touches W^Q only, Sec. 3), key normalisation and RoPE at their
     assembled positions;
   * prompt layouts whose online text (instructions, separators, the question)
-    interleaves with the cached artifact spans (App. prompt construction).
+    interleaves with the cached artifact spans (App. prompt construction);
+  * two variants of the read from the paper's training-free baselines
+    (App. C.2): keys stored before RoPE and rotated to their assembled
+    positions at assembly (EPIC), and separate attention over the cached
+    context (temperature T) and the online tokens combined by calibrated
+    log-sum-exp terms (APE).
 
 Parity status: every function is pinned by the tests in
 ``tests/test_oracle_pins.py`` (closed forms, hand-derived fixtures under
@@ -43,5 +48,9 @@ from .attuner_oracle import (  # noqa: F401
     request_forward,
     layout_online_positions,
     layout_forward,
+    rotate_at_assembly,
+    epic_request_forward,
+    ape_combine,
+    ape_request_forward,
     workload_reference,
 )

@@ -244,6 +244,79 @@ def request_forward(x, w_q, a, b, s, q_norm_w, eps, theta, art_k: List[np.ndarra
 
 
 # ---------------------------------------------------------------------------
+# App. C.2 "Training-Free Baselines", EPIC paragraph: the cached keys are
+# stored before RoPE and rotated to their target positions when the request
+# is assembled.  Here the target of artifact token t is its index in the
+# assembled sequence (artifacts in runtime order from position 0, App. A.5),
+# and the read that follows is the PIC read of Eq. (routing-oracle) over the
+# rotated keys: every artifact token visible, the suffix causal.
+# ---------------------------------------------------------------------------
+def rotate_at_assembly(art_k_raw: Sequence[np.ndarray], theta: float) -> np.ndarray:
+    """art_k_raw: per-artifact keys before RoPE [L_a, Hkv, d], runtime order.
+    Returns the assembled keys [T_art, Hkv, d], token t rotated at position t."""
+    k = np.concatenate(list(art_k_raw), axis=0)
+    return rope_rotate_half(k, np.arange(k.shape[0], dtype=np.int64), theta)
+
+
+def epic_request_forward(x, w_q, a, b, s, q_norm_w, eps, theta, art_k_raw: List[np.ndarray],
+                         art_v: List[np.ndarray], suffix_k, suffix_v, n_q_heads: int, pairs=None):
+    """request_forward with the artifact keys stored before RoPE and rotated
+    at their assembled positions; queries and suffix keys as there."""
+    k_art = rotate_at_assembly(art_k_raw, theta)
+    v_art = np.concatenate(list(art_v), axis=0)
+    return request_forward(x, w_q, a, b, s, q_norm_w, eps, theta, [k_art], [v_art], suffix_k, suffix_v,
+                           n_q_heads, pairs=pairs)
+
+
+# ---------------------------------------------------------------------------
+# App. C.2, APE paragraph: attention over the cached context and over the
+# online tokens is computed separately, the context's logits divided by a
+# temperature T, and the two results are combined through calibrated
+# log-sum-exp terms.  The paper fixes T = 0.9 and a scale of 0.9 but not how
+# the scale enters; the reading taken here multiplies the context's
+# log-sum-exp by it (its softmax denominator Z_c counts as Z_c^scale).
+# With no prefix of online text before the artifacts (a prompt that begins
+# with cached artifacts), the online part is the suffix, causal.
+# ---------------------------------------------------------------------------
+def ape_combine(o_ctx: np.ndarray, lse_ctx: np.ndarray, o_on: np.ndarray, lse_on: np.ndarray, scale: float):
+    """o = w_c o_ctx + w_o o_on with (w_c, w_o) proportional to
+    (exp(scale * lse_ctx), exp(lse_on)); lse = log of their sum.  An empty
+    context (lse_ctx = -inf) has weight 0.  Shapes: o [..., d], lse [...]."""
+    lc = np.where(np.isneginf(lse_ctx), -np.inf, scale * np.asarray(lse_ctx, dtype=np.float64))
+    lo = np.asarray(lse_on, dtype=np.float64)
+    m = np.maximum(lc, lo)
+    wc = np.exp(lc - m)
+    wo = np.exp(lo - m)
+    z = wc + wo
+    oc = np.where(np.isneginf(lc)[..., None], 0.0, o_ctx)
+    o = (wc[..., None] * oc + wo[..., None] * o_on) / z[..., None]
+    return o, m + np.log(z)
+
+
+def ape_request_forward(x, w_q, a, b, s, q_norm_w, eps, theta, art_k: List[np.ndarray], art_v: List[np.ndarray],
+                        suffix_k, suffix_v, n_q_heads: int, temperature: float, scale: float, pairs=None):
+    """Queries as in request_forward (positions of the assembled context);
+    context part = attention over every artifact token with logits divided by
+    `temperature`; online part = causal attention over the suffix keys;
+    combined by ape_combine."""
+    S = x.shape[0]
+    S_kv = suffix_k.shape[0]
+    d = suffix_k.shape[2]
+    t_art = int(sum(t.shape[0] for t in art_k))
+    q_raw = lora_q_projection(x, w_q, a, b, s).reshape(S, n_q_heads, d)
+    q = rope_rotate_half(rms_norm_heads(q_raw, q_norm_w, eps), query_positions(t_art, S, S_kv), theta)
+    o_on, lse_on = attention(q, suffix_k, suffix_v, (S_kv - S) + np.arange(S) + 1, pairs)
+    if t_art == 0:
+        o_ctx, lse_ctx = np.zeros_like(o_on), np.full(lse_on.shape, -np.inf)
+    else:
+        k_art = np.concatenate(list(art_k), axis=0)
+        v_art = np.concatenate(list(art_v), axis=0)
+        # logits q.k / (T sqrt(d)) = (q / T).k / sqrt(d)
+        o_ctx, lse_ctx = attention(q / temperature, k_art, v_art, np.full(S, t_art), pairs)
+    return ape_combine(o_ctx, lse_ctx, o_on, lse_on, scale)
+
+
+# ---------------------------------------------------------------------------
 # App. "Prompt Construction and Artifact Boundaries" (Tab. prompt layouts):
 # text outside the cached artifact spans -- instructions, separators, the
 # question -- is processed online, so online spans interleave with the cached

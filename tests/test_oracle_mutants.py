@@ -19,7 +19,9 @@ import test_oracle_pins as pins
 
 ORIG = {n: getattr(O, n) for n in ("lora_q_projection", "merged_q_weight", "rms_norm_heads", "rope_rotate_half",
                                   "query_positions", "kv_projection", "assemble", "attention", "request_forward",
-                                  "layout_online_positions", "layout_forward", "merge_partials")}
+                                  "layout_online_positions", "layout_forward", "merge_partials",
+                                  "rotate_at_assembly", "epic_request_forward", "ape_combine",
+                                  "ape_request_forward")}
 PINS = {n: f for n, f in vars(pins).items() if n.startswith("test_") and callable(f)}
 
 
@@ -218,6 +220,71 @@ def layout_query_not_self_visible(x, w_q, a, b, s, q_norm_w, eps, theta, items, 
         O.attention = real_attention
 
 
+# --- App. C.2 variants: EPIC (rotate at assembly) and APE (calibrated combine)
+def rotate_at_local_positions(art_k_raw, theta):
+    # each artifact rotated at its own positions 0..L-1 (the PIC cache)
+    return np.concatenate([ORIG["rope_rotate_half"](k, np.arange(k.shape[0]), theta) for k in art_k_raw], axis=0)
+
+
+def rotate_positions_plus_one(art_k_raw, theta):
+    k = np.concatenate(list(art_k_raw), axis=0)
+    return ORIG["rope_rotate_half"](k, np.arange(k.shape[0]) + 1, theta)
+
+
+def epic_values_unordered(x, w_q, a, b, s, q_norm_w, eps, theta, art_k_raw, art_v, suffix_k, suffix_v, n_q_heads,
+                          pairs=None):
+    # values taken in reverse artifact order against keys in runtime order
+    return ORIG["epic_request_forward"](x, w_q, a, b, s, q_norm_w, eps, theta, art_k_raw, list(art_v)[::-1],
+                                        suffix_k, suffix_v, n_q_heads, pairs)
+
+
+def epic_queries_at_local_positions(x, w_q, a, b, s, q_norm_w, eps, theta, art_k_raw, art_v, suffix_k, suffix_v,
+                                    n_q_heads, pairs=None):
+    # queries rotated as if the artifacts were not there
+    k_art = O.rotate_at_assembly(art_k_raw, theta)
+    v_art = np.concatenate(list(art_v), axis=0)
+    S, S_kv, d = x.shape[0], suffix_k.shape[0], suffix_k.shape[2]
+    q_raw = O.lora_q_projection(x, w_q, a, b, s).reshape(S, n_q_heads, d)
+    q = O.rope_rotate_half(O.rms_norm_heads(q_raw, q_norm_w, eps), (S_kv - S) + np.arange(S), theta)
+    return O.attention(q, np.concatenate([k_art, suffix_k]), np.concatenate([v_art, suffix_v]),
+                       k_art.shape[0] + (S_kv - S) + np.arange(S) + 1, pairs)
+
+
+def ape_scale_additive(o_ctx, lse_ctx, o_on, lse_on, scale):
+    # the scale as a factor on Z_c (log scale added) instead of a power
+    return ORIG["ape_combine"](o_ctx, np.asarray(lse_ctx) + math.log(scale) / scale, o_on, lse_on, scale)
+
+
+def ape_scale_on_online(o_ctx, lse_ctx, o_on, lse_on, scale):
+    return ORIG["ape_combine"](o_on, lse_on, o_ctx, lse_ctx, scale)
+
+
+def ape_combine_without_normalising(o_ctx, lse_ctx, o_on, lse_on, scale):
+    lc = scale * np.asarray(lse_ctx, dtype=np.float64)
+    m = np.maximum(lc, lse_on)
+    o = np.exp(lc - m)[..., None] * o_ctx + np.exp(np.asarray(lse_on) - m)[..., None] * o_on
+    return o, m + np.log(np.exp(lc - m) + np.exp(np.asarray(lse_on) - m))
+
+
+def ape_temperature_multiplied(x, w_q, a, b, s, q_norm_w, eps, theta, art_k, art_v, suffix_k, suffix_v, n_q_heads,
+                               temperature, scale, pairs=None):
+    return ORIG["ape_request_forward"](x, w_q, a, b, s, q_norm_w, eps, theta, art_k, art_v, suffix_k, suffix_v,
+                                       n_q_heads, 1.0 / temperature, scale, pairs)
+
+
+def ape_online_not_causal(x, w_q, a, b, s, q_norm_w, eps, theta, art_k, art_v, suffix_k, suffix_v, n_q_heads,
+                          temperature, scale, pairs=None):
+    real_attention = O.attention
+    S_kv = suffix_k.shape[0]
+    try:
+        O.attention = lambda q, k, v, n_vis, p=None: ORIG["attention"](
+            q, k, v, np.full(len(n_vis), S_kv) if k.shape[0] == S_kv else n_vis, p)
+        return ORIG["ape_request_forward"](x, w_q, a, b, s, q_norm_w, eps, theta, art_k, art_v, suffix_k, suffix_v,
+                                           n_q_heads, temperature, scale, pairs)
+    finally:
+        O.attention = real_attention
+
+
 MUTANTS = [
     ("lora_q_projection", lora_without_update), ("lora_q_projection", lora_without_scale),
     ("lora_q_projection", lora_scale_on_base),
@@ -241,6 +308,11 @@ MUTANTS = [
     ("request_forward", request_query_not_self_visible), ("request_forward", request_suffix_not_causal),
     ("request_forward", request_positions_without_artifacts),
     ("layout_forward", layout_query_not_self_visible),
+    ("rotate_at_assembly", rotate_at_local_positions), ("rotate_at_assembly", rotate_positions_plus_one),
+    ("epic_request_forward", epic_values_unordered), ("epic_request_forward", epic_queries_at_local_positions),
+    ("ape_combine", ape_scale_additive), ("ape_combine", ape_scale_on_online),
+    ("ape_combine", ape_combine_without_normalising),
+    ("ape_request_forward", ape_temperature_multiplied), ("ape_request_forward", ape_online_not_causal),
 ]
 
 
@@ -249,7 +321,9 @@ def _pin_order(name):
     key = {"lora_q_projection": "lora", "merged_q_weight": "merged", "rms_norm_heads": "rmsnorm",
            "rope_rotate_half": "rope", "query_positions": "query_positions", "kv_projection": "kv_projection",
            "assemble": "assemble", "attention": "attention", "request_forward": "artifact",
-           "layout_online_positions": "layout", "layout_forward": "layout", "merge_partials": "merge"}[name]
+           "layout_online_positions": "layout", "layout_forward": "layout", "merge_partials": "merge",
+           "rotate_at_assembly": "epic", "epic_request_forward": "epic", "ape_combine": "ape",
+           "ape_request_forward": "ape"}[name]
     names = sorted(PINS)
     return [n for n in names if key in n] + [n for n in names if key not in n]
 

@@ -491,3 +491,186 @@ def test_tiny_workload_against_sdpa():
     n_vis = 201 + np.arange(16) + 1
     np.testing.assert_allclose(o, _sdpa_f64(q, k, v, n_vis), atol=1e-12)
     assert o.shape == (16, 4, 64) and np.all(np.isfinite(lse))
+
+
+# --------------------------------------------------------------------------
+# App. C.2, EPIC paragraph: keys stored before RoPE, rotated to their
+# assembled positions at assembly
+# --------------------------------------------------------------------------
+def _variant_case(rng, lens=(13, 64, 40), S=6, S_kv=9, hidden=32, hq=4, hkv=2, d=16, theta=1.0e4):
+    w = _small_inputs(rng, hidden, hq, hkv, d)
+    return dict(
+        x=rng.standard_normal((S, hidden)), w_q=w["w_q"], a=w["a"], b=w["b"], s=2.0, q_norm_w=w["qn"], eps=1e-6,
+        theta=theta, art_k=[rng.standard_normal((L, hkv, d)) for L in lens],
+        art_v=[rng.standard_normal((L, hkv, d)) for L in lens], suffix_k=rng.standard_normal((S_kv, hkv, d)),
+        suffix_v=rng.standard_normal((S_kv, hkv, d)), n_q_heads=hq)
+
+
+def _queries(c):
+    # the queries of request_forward, step by step through the pinned functions
+    S, S_kv, d = c["x"].shape[0], c["suffix_k"].shape[0], c["suffix_k"].shape[2]
+    t_art = sum(k.shape[0] for k in c["art_k"])
+    q_raw = O.lora_q_projection(c["x"], c["w_q"], c["a"], c["b"], c["s"]).reshape(S, c["n_q_heads"], d)
+    pos = t_art + (S_kv - S) + np.arange(S)
+    return O.rope_rotate_half(O.rms_norm_heads(q_raw, c["q_norm_w"], c["eps"]), pos, c["theta"]), pos
+
+
+def _epic(c, **kw):
+    return O.epic_request_forward(c["x"], c["w_q"], c["a"], c["b"], c["s"], c["q_norm_w"], c["eps"], c["theta"],
+                                  c["art_k"], c["art_v"], c["suffix_k"], c["suffix_v"], c["n_q_heads"], **kw)
+
+
+def test_epic_equals_full_causal_over_the_assembled_sequence():
+    # With the artifacts' raw keys rotated at their assembled positions, the
+    # suffix rows read exactly the keys a full prefill of the concatenation
+    # would hold: fp64 causal SDPA over the whole sequence, keys rotated at
+    # 0..T-1, in two runtime orders
+    rng = np.random.default_rng(31)
+    c = _variant_case(rng)
+    for order in ([0, 1, 2], [2, 0, 1]):
+        cc = dict(c, art_k=[c["art_k"][i] for i in order], art_v=[c["art_v"][i] for i in order])
+        S = cc["x"].shape[0]
+        q, _ = _queries(cc)
+        k_raw = np.concatenate(cc["art_k"])
+        T_art = k_raw.shape[0]
+        K = np.concatenate([O.rope_rotate_half(k_raw, np.arange(T_art), cc["theta"]), cc["suffix_k"]])
+        V = np.concatenate(cc["art_v"] + [cc["suffix_v"]])
+        T = K.shape[0]
+        q_full = np.concatenate([rng.standard_normal((T - S, cc["n_q_heads"], q.shape[2])), q])
+        G = cc["n_q_heads"] // K.shape[1]
+        qt = torch.from_numpy(q_full).permute(1, 0, 2)[None]
+        kt = torch.from_numpy(K).repeat_interleave(G, dim=1).permute(1, 0, 2)[None]
+        vt = torch.from_numpy(V).repeat_interleave(G, dim=1).permute(1, 0, 2)[None]
+        full = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True)[0].permute(1, 0, 2)
+        o, _ = _epic(cc)
+        np.testing.assert_allclose(o, full.numpy()[T - S:], atol=1e-12)
+
+
+def test_epic_relative_position_identity():
+    # <R(p) q, R(t + off_a) k> = <R(p - off_a) q, R(t) k>: the keys rotated at
+    # their assembled positions give the same logits as the PIC cache (keys
+    # at local positions t) read by queries rotated back by each artifact's
+    # offset.  Direct sums over that second form, query by query.
+    rng = np.random.default_rng(32)
+    c = _variant_case(rng, lens=(5, 11, 3), S=3, S_kv=4, hq=2, hkv=1, d=8)
+    o, lse = _epic(c)
+    S, S_kv, d = c["x"].shape[0], c["suffix_k"].shape[0], 8
+    t_art = sum(k.shape[0] for k in c["art_k"])
+    q_raw = O.lora_q_projection(c["x"], c["w_q"], c["a"], c["b"], c["s"]).reshape(S, 2, d)
+    qn = O.rms_norm_heads(q_raw, c["q_norm_w"], c["eps"])
+    for i in range(S):
+        p = t_art + (S_kv - S) + i
+        for h in range(2):
+            logits, vals = [], []
+            off = 0
+            for ka, va in zip(c["art_k"], c["art_v"]):
+                q_back = O.rope_rotate_half(qn[i:i + 1, h:h + 1], np.array([p - off]), c["theta"])[0, 0]
+                k_loc = O.rope_rotate_half(ka[:, 0:1], np.arange(ka.shape[0]), c["theta"])[:, 0]
+                for t in range(ka.shape[0]):
+                    logits.append(float(q_back @ k_loc[t]) / math.sqrt(d))
+                    vals.append(va[t, 0])
+                off += ka.shape[0]
+            q_here = O.rope_rotate_half(qn[i:i + 1, h:h + 1], np.array([p]), c["theta"])[0, 0]
+            for j in range(S_kv - S + i + 1):
+                logits.append(float(q_here @ c["suffix_k"][j, 0]) / math.sqrt(d))
+                vals.append(c["suffix_v"][j, 0])
+            e = [math.exp(z) for z in logits]
+            z = sum(e)
+            ref = sum(w * v for w, v in zip(e, vals)) / z
+            np.testing.assert_allclose(o[i, h], ref, atol=1e-12)
+            assert abs(lse[i, h] - math.log(z)) < 1e-12
+
+
+def test_epic_single_artifact_is_the_pic_read():
+    # the first artifact starts at position 0: rotating its raw keys at
+    # assembly equals caching them rotated at their local positions
+    rng = np.random.default_rng(33)
+    c = _variant_case(rng, lens=(70,))
+    o, lse = _epic(c)
+    k_loc = O.rope_rotate_half(c["art_k"][0], np.arange(70), c["theta"])
+    o2, lse2 = O.request_forward(c["x"], c["w_q"], c["a"], c["b"], c["s"], c["q_norm_w"], c["eps"], c["theta"],
+                                 [k_loc], c["art_v"], c["suffix_k"], c["suffix_v"], c["n_q_heads"])
+    np.testing.assert_allclose(o, o2, atol=1e-13)
+    np.testing.assert_allclose(lse, lse2, atol=1e-13)
+
+
+def test_rotate_at_assembly_positions():
+    # token t of the concatenation is rotated at t: a unit vector in pair 0
+    # turns by t * theta^0 = t radians
+    k = [np.zeros((2, 1, 4)), np.zeros((3, 1, 4))]
+    for a in k:
+        a[:, 0, 0] = 1.0
+    out = O.rotate_at_assembly(k, 1.0e4)
+    for t in range(5):
+        np.testing.assert_allclose(out[t, 0, [0, 2]], [math.cos(t), math.sin(t)], atol=1e-15)
+
+
+# --------------------------------------------------------------------------
+# App. C.2, APE paragraph: context (temperature T) and online attention
+# combined through calibrated log-sum-exp terms
+# --------------------------------------------------------------------------
+def _ape(c, T, scale, **kw):
+    return O.ape_request_forward(c["x"], c["w_q"], c["a"], c["b"], c["s"], c["q_norm_w"], c["eps"], c["theta"],
+                                 c["art_k"], c["art_v"], c["suffix_k"], c["suffix_v"], c["n_q_heads"], T, scale, **kw)
+
+
+def test_ape_combine_hand_example():
+    g = _golden("ape_combine.json")
+    num = {"ln3": math.log(3.0), "ln4": math.log(4.0), "ln5": math.log(5.0), "ln8": math.log(8.0),
+           "ln16": math.log(16.0), "-inf": -np.inf}
+    val = lambda x: num[x] if isinstance(x, str) else x
+    for cs in g["cases"]:
+        o, lse = O.ape_combine(np.array(cs["o_ctx"]), np.array(val(cs["lse_ctx"])), np.array(cs["o_on"]),
+                               np.array(val(cs["lse_on"])), cs["scale"])
+        np.testing.assert_allclose(o, cs["o"], atol=1e-14)
+        assert abs(lse - val(cs["lse"])) < 1e-14
+
+
+def test_ape_with_unit_temperature_and_scale_is_the_pic_read():
+    rng = np.random.default_rng(34)
+    c = _variant_case(rng)
+    o, lse = _ape(c, 1.0, 1.0)
+    o2, lse2 = O.request_forward(c["x"], c["w_q"], c["a"], c["b"], c["s"], c["q_norm_w"], c["eps"], c["theta"],
+                                 c["art_k"], c["art_v"], c["suffix_k"], c["suffix_v"], c["n_q_heads"])
+    np.testing.assert_allclose(o, o2, atol=1e-12)
+    np.testing.assert_allclose(lse, lse2, atol=1e-12)
+
+
+@pytest.mark.parametrize("T,scale", [(0.9, 0.9), (0.5, 1.3)])
+def test_ape_against_direct_sums(T, scale):
+    # no max subtraction and no log-sum-exp machinery: Z_c = sum over context
+    # keys of exp(l / T), Z_o = sum over visible online keys of exp(l), and
+    # o = (Z_c^(scale - 1) N_c + N_o) / (Z_c^scale + Z_o) with N the
+    # exp-weighted value sums; lse = log(Z_c^scale + Z_o)
+    rng = np.random.default_rng(35)
+    c = _variant_case(rng, lens=(7, 4), S=3, S_kv=5, hq=2, hkv=1, d=8)
+    o, lse = _ape(c, T, scale)
+    q, _ = _queries(c)
+    S, S_kv, d = 3, 5, 8
+    k_art, v_art = np.concatenate(c["art_k"]), np.concatenate(c["art_v"])
+    for i in range(S):
+        for h in range(2):
+            zc, nc = 0.0, np.zeros(d)
+            for t in range(k_art.shape[0]):
+                e = math.exp(float(q[i, h] @ k_art[t, 0]) / math.sqrt(d) / T)
+                zc += e
+                nc += e * v_art[t, 0]
+            zo, no = 0.0, np.zeros(d)
+            for j in range(S_kv - S + i + 1):
+                e = math.exp(float(q[i, h] @ c["suffix_k"][j, 0]) / math.sqrt(d))
+                zo += e
+                no += e * c["suffix_v"][j, 0]
+            ref = (zc ** (scale - 1.0) * nc + no) / (zc ** scale + zo)
+            np.testing.assert_allclose(o[i, h], ref, rtol=1e-11, atol=1e-13)
+            assert abs(lse[i, h] - math.log(zc ** scale + zo)) < 1e-11
+
+
+def test_ape_without_artifacts_is_online_attention():
+    rng = np.random.default_rng(36)
+    c = _variant_case(rng, lens=())
+    o, lse = _ape(c, 0.9, 0.9)
+    q, _ = _queries(c)
+    S, S_kv = c["x"].shape[0], c["suffix_k"].shape[0]
+    o2, lse2 = O.attention(q, c["suffix_k"], c["suffix_v"], (S_kv - S) + np.arange(S) + 1)
+    np.testing.assert_allclose(o, o2, atol=1e-14)
+    np.testing.assert_allclose(lse, lse2, atol=1e-14)
