@@ -243,6 +243,48 @@ attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, 
                                     const void* suffix_k, const void* suffix_v, int32_t S,
                                     int32_t S_kv, void* out, float* lse_out, void* stream);
 
+/* Keys stored before RoPE, rotated to their target positions at assembly:
+ * the read of the paper's EPIC baseline (App. C.2 "Training-Free Baselines",
+ * EPIC paragraph: cached keys kept un-rotated and rotated to their place in
+ * the assembled prompt).  The plan's artifacts must have been registered
+ * with keys BEFORE RoPE; artifact token t of a request is rotated at its
+ * assembled position (the request's artifact tokens before it, in runtime
+ * order from 0: the position a full prefill would give it).  One kernel on
+ * `stream` writes the rotated keys into a buffer the plan owns
+ * ([n_blocks][Hkv][64][d] bf16, freed by attuner_plan_free); from then on
+ * every attention call with this plan reads its artifact keys there (values
+ * still from the pool), and queries and suffix keys are as for the plain
+ * read.  Calling it again re-rotates into the same buffer.  The call
+ * allocates the buffer (cudaMalloc) on first use and returns once the
+ * rotation has finished (it synchronises `stream`).
+ * Errors: INVALID_ARG (NULL, foreign or stale plan), UNSUPPORTED (a plan with
+ * online spans between artifacts), OOM, CUDA; DEVICE_CHECK through
+ * attuner_sync_status when a block id is out of the pool. */
+attuner_status attuner_plan_rotate_keys(attuner_ctx* ctx, attuner_plan* plan, void* stream);
+
+/* The read of the paper's APE baseline (App. C.2, APE paragraph): attention
+ * over the cached context and over the online tokens computed separately,
+ * the context's logits divided by `temperature`, and the two results
+ * combined through calibrated log-sum-exp terms.  The paper uses
+ * temperature 0.9 and scale 0.9 without stating how the scale enters; here
+ * it multiplies the context's log-sum-exp (its softmax denominator Z_c counts
+ * as Z_c^scale):
+ *   (o_c, lse_c) = softmax(q k_art^T / (temperature sqrt(d))) v_art, every
+ *                  artifact token visible;
+ *   (o_o, lse_o) = causal attention over the suffix keys j <= (S_kv - S) + i;
+ *   out = (e^(scale lse_c) o_c + e^(lse_o) o_o) / (e^(scale lse_c) + e^(lse_o)),
+ *   lse_out = log(e^(scale lse_c) + e^(lse_o)); a request without artifacts
+ *   takes o_o and lse_o.
+ * Arguments and layouts as in attuner_attend; temperature = scale = 1 gives
+ * attuner_attend's result.  Three launches (context part, online part,
+ * combine) with their two partial results in stream-ordered scratch.
+ * Errors: INVALID_ARG (also temperature or scale not positive and finite),
+ * UNSUPPORTED (a plan with online spans between artifacts), CUDA. */
+attuner_status attuner_attend_ape(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
+                                  const void* suffix_k, const void* suffix_v, int32_t S, int32_t S_kv,
+                                  float temperature, float scale, void* out, float* lse_out,
+                                  void* stream);
+
 /* Warm-cache load (the "CPU RAM cache lookup and GPU transfer" stage of the
  * paper's time-to-first-token, Sec. 5 / App. A.3: encoded artifacts kept in
  * host memory and moved to the GPU when a request needs them).  Registers n

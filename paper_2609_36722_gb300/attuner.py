@@ -45,7 +45,7 @@ EXPORTS = [
     "attuner_attend", "attuner_query_attend", "attuner_pool_info", "attuner_sync_status",
     "attuner_set_option", "attuner_last_launch_count", "attuner_last_error",
     "attuner_attend_static_scratch", "attuner_register_artifacts_host", "attuner_pool_reset",
-    "attuner_kv_project", "attuner_assemble_layout",
+    "attuner_kv_project", "attuner_assemble_layout", "attuner_plan_rotate_keys", "attuner_attend_ape",
 ]
 
 
@@ -93,6 +93,9 @@ SIGNATURES = {
     "attuner_pool_reset": ([_vp], _i32),
     "attuner_kv_project": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
     "attuner_assemble_layout": ([_vp, _p_i32, _p_i32, _i32, ctypes.POINTER(_vp)], _i32),
+    "attuner_plan_rotate_keys": ([_vp, _vp, _vp], _i32),
+    "attuner_attend_ape": ([_vp, _vp, _vp, _vp, _vp, _i32, _i32, ctypes.c_float, ctypes.c_float, _vp, _vp, _vp],
+                           _i32),
 }
 
 
@@ -332,6 +335,27 @@ class Context:
                                                    self._p(suffix_k, "suffix_k"), self._p(suffix_v, "suffix_v"), S,
                                                    S_kv, self._p(out, "out"), self._p(lse, "lse", torch.float32),
                                                    self._s(stream)))
+        return out, lse
+
+    def rotate_keys(self, plan: Plan, stream=None) -> None:
+        """Rotate the plan's artifact keys (registered before RoPE) to their
+        assembled positions; later attention calls with the plan read them."""
+        _check(lib().attuner_plan_rotate_keys(self.handle, plan.handle, self._s(stream)))
+
+    def attend_ape(self, plan: Plan, q, suffix_k, suffix_v, temperature: float = 0.9, scale: float = 0.9,
+                   out: Optional[torch.Tensor] = None, lse: Optional[torch.Tensor] = None, want_lse: bool = True,
+                   stream=None):
+        """Context (logits / temperature) and online attention combined by
+        calibrated log-sum-exp terms (scale on the context's)."""
+        n_req, S, Hq, d = q.shape
+        S_kv = suffix_k.shape[1]
+        if out is None:
+            out = torch.empty_like(q)
+        if lse is None and want_lse:
+            lse = torch.empty(n_req, S, Hq, dtype=torch.float32, device=q.device)
+        _check(lib().attuner_attend_ape(self.handle, plan.handle, self._p(q, "q"), self._p(suffix_k, "suffix_k"),
+                                        self._p(suffix_v, "suffix_v"), S, S_kv, float(temperature), float(scale),
+                                        self._p(out, "out"), self._p(lse, "lse", torch.float32), self._s(stream)))
         return out, lse
 
     def query_attend(self, plan: Plan, x, w_q, lora_a, lora_b, s: float, q_norm_w, suffix_k, suffix_v,

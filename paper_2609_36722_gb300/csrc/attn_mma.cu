@@ -66,8 +66,10 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
   const int row0 = rt * kMmaRows;
   const int last_row = min(row0 + kMmaRows - 1, p.S * G - 1);
   const int last_vis = row_visibility(p.plan, req, (p.S_kv - p.S) + last_row / G, nab).slot;
-  const int b0 = split * p.work.chunk_blocks;
-  const int b1 = min(min(b0 + p.work.chunk_blocks, nab + nsuf), last_vis + 1);
+  int v_lo, v_hi;
+  kv_part_range(p.kv_part, nab, nsuf, v_lo, v_hi);
+  const int b0 = v_lo + split * p.work.chunk_blocks;
+  const int b1 = min(min(b0 + p.work.chunk_blocks, v_hi), last_vis + 1);
   const int nblk = max(0, b1 - b0);
 
   for (int i = threadIdx.x; i < nblk; i += blockDim.x) {
@@ -119,7 +121,10 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
             tma_load_4d(dst + (L::NH + h) * L::BLK, &p.tm_vsuf, fb, h * 64, kvh, c, req);
           } else {
             const int row = (e == 0) ? pool_rows : ((e >> 7) * p.Hkv + kvh) * kBlockTokens;
-            tma_load_2d(dst + h * L::BLK, &p.tm_kpool, fb, h * 64, row);
+            if (e != 0 && p.k_by_slot)   // keys rotated at assembly, by the plan's slot index
+              tma_load_2d(dst + h * L::BLK, &p.tm_kslot, fb, h * 64, ((boff + b0 + j) * p.Hkv + kvh) * kBlockTokens);
+            else
+              tma_load_2d(dst + h * L::BLK, &p.tm_kpool, fb, h * 64, row);
             tma_load_2d(dst + (L::NH + h) * L::BLK, &p.tm_vpool, fb, h * 64, row);
           }
         }
@@ -399,6 +404,44 @@ __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ Co
     *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc.x * inv, acc.y * inv);
   }
   if (lane == 0 && p.lse_out) p.lse_out[orow] = (W > 0.f) ? M + logf(W) : -INFINITY;
+}
+
+// APE's calibrated combination of the context and online parts (see
+// ApeParams): one warp per output row (request, token, head), each lane D/32
+// consecutive columns.
+__global__ void __launch_bounds__(256) ape_combine_kernel(const __grid_constant__ ApeParams p, long long rows) {
+  grid_dep_wait();   // the online part comes from the attention launch just before
+  const long long row = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const int req = (int)(row / ((long long)p.S * p.Hq));
+  const float lo = p.lse_on[row];
+  const float lc = (p.t_art[req] > 0 && p.lse_ctx[row] != -INFINITY) ? p.scale * p.lse_ctx[row] : -INFINITY;
+  const float m = fmaxf(lc, lo);
+  const float wc = (lc == -INFINITY) ? 0.f : expf(lc - m);
+  const float wo = expf(lo - m);
+  const float inv = 1.f / (wc + wo);
+  const int cpl = p.D / 32;   // 2 or 4
+  const long long at = row * p.D + lane * cpl;
+  float y[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    if (k < cpl) {
+      const float c = (wc > 0.f) ? __bfloat162float(p.o_ctx[at + k]) : 0.f;
+      y[k] = (wc * c + wo * __bfloat162float(p.o_on[at + k])) * inv;
+    }
+  }
+  if (cpl == 4)
+    *reinterpret_cast<uint2*>(p.out + at) = make_uint2(pack_bf16(y[0], y[1]), pack_bf16(y[2], y[3]));
+  else
+    *reinterpret_cast<uint32_t*>(p.out + at) = pack_bf16(y[0], y[1]);
+  if (lane == 0 && p.lse_out) p.lse_out[row] = m + logf(wc + wo);
+}
+
+cudaError_t launch_ape_combine(const ApeParams& p, cudaStream_t st) {
+  const long long rows = (long long)p.n_req * p.S * p.Hq;
+  if (rows == 0) return cudaSuccess;
+  return launch_pdl(ape_combine_kernel, dim3((unsigned)((rows * 32 + 255) / 256)), dim3(256), 0, st, 0, p, rows);
 }
 
 cudaError_t launch_combine(const CombineParams& p, cudaStream_t st) {

@@ -81,19 +81,26 @@ ATT_DEV void umma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uin
       : "memory");
 }
 
-// load the K (or V) half-tiles of block slot `e` into `dst` (64-column halves at +HALF)
+// load the K (or V) half-tiles of block slot `e` into `dst` (64-column halves
+// at +HALF); an artifact slot reads rows kslot_row.. of `kslot` instead of its
+// pool block when `kslot` is given (keys rotated at assembly)
 template <int D>
 __device__ __forceinline__ void load_slot(uint32_t dst, int e, const CUtensorMap* pool,
                                           const CUtensorMap* suf, uint32_t bar, int kvh, int Hkv,
-                                          int req, int pool_rows) {
+                                          int req, int pool_rows, const CUtensorMap* kslot = nullptr,
+                                          int kslot_row = 0) {
   using L = TcLayout<D>;
 #pragma unroll
   for (int h = 0; h < L::NH; ++h) {
     if (e < 0) {
       tma_load_4d(dst + h * L::HALF, suf, bar, h * 64, kvh, slot_row0(e), req);
     } else if ((e & 127) != 0) {
-      const int blk = e >> 7;
-      tma_load_2d(dst + h * L::HALF, pool, bar, h * 64, (blk * Hkv + kvh) * kBlockTokens);
+      if (kslot != nullptr) {
+        tma_load_2d(dst + h * L::HALF, kslot, bar, h * 64, kslot_row);
+      } else {
+        const int blk = e >> 7;
+        tma_load_2d(dst + h * L::HALF, pool, bar, h * 64, (blk * Hkv + kvh) * kBlockTokens);
+      }
     } else {
       // no block: a box entirely past the end of the pool reads zeros
       tma_load_2d(dst + h * L::HALF, pool, bar, h * 64, pool_rows);
@@ -124,8 +131,10 @@ __device__ __forceinline__ TcCta tc_cta(const AttnParams& p, int cta) {
     const int rem = unit % per_req;
     c.rt = rem % p.work.row_tiles;
     c.kvh = rem / p.work.row_tiles;
-    const int nv = p.plan.blk_off[c.req + 1] - p.plan.blk_off[c.req] +
-                   (p.S_kv - plan_o_rows(p.plan, c.req) + kBlockTokens - 1) / kBlockTokens;
+    int lo, hi;
+    kv_part_range(p.kv_part, p.plan.blk_off[c.req + 1] - p.plan.blk_off[c.req],
+                  (p.S_kv - plan_o_rows(p.plan, c.req) + kBlockTokens - 1) / kBlockTokens, lo, hi);
+    const int nv = hi - lo;
     c.chunk = (((nv + ns - 1) / ns) + 1) & ~1;
   } else {
     c.req = find_req(p.work, cta);
@@ -535,11 +544,16 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
   const int row0 = rt * kTcRows;
   const int last_row = min(row0 + kTcRows - 1, p.S * G - 1);
   const int last_vis = row_visibility(p.plan, req, (p.S_kv - p.S) + last_row / G, nab).slot;
-  const int b0 = cw.split * cw.chunk;
-  const int b1 = min(min(b0 + cw.chunk, nab + nsuf), last_vis + 1);
+  int v_lo, v_hi;
+  kv_part_range(p.kv_part, nab, nsuf, v_lo, v_hi);
+  const int b0 = v_lo + cw.split * cw.chunk;
+  const int b1 = min(min(b0 + cw.chunk, v_hi), last_vis + 1);
   const int nblk = max(0, b1 - b0);
   const int ntile = (nblk + 1) / 2;
   const int pool_rows = p.plan.pool_blocks * p.Hkv * kBlockTokens;
+  // keys rotated at assembly: the K rows of this CTA's slot b0 + i
+  const CUtensorMap* kslot = p.k_by_slot ? &p.tm_kslot : nullptr;
+  auto kslot_row = [&](int i) { return ((boff + b0 + i) * p.Hkv + kvh) * kBlockTokens; };
 
   // ---- slots of this chunk: >0 artifact block, <0 online chunk, 0 none
   auto slot_entry = [&](int i) {
@@ -580,8 +594,9 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
       if (e0 < 0 || e1 < 0) grid_dep_wait();
       const uint32_t kd = sbase + L::K_OFF;
       mbar_expect_tx(bar(B_KF), tile_bytes);
-      load_slot<D>(kd, e0, &p.tm_kpool, &p.tm_ksuf, bar(B_KF), kvh, p.Hkv, req, pool_rows);
-      load_slot<D>(kd + kBlockTokens * 128, e1, &p.tm_kpool, &p.tm_ksuf, bar(B_KF), kvh, p.Hkv, req, pool_rows);
+      load_slot<D>(kd, e0, &p.tm_kpool, &p.tm_ksuf, bar(B_KF), kvh, p.Hkv, req, pool_rows, kslot, kslot_row(0));
+      load_slot<D>(kd + kBlockTokens * 128, e1, &p.tm_kpool, &p.tm_ksuf, bar(B_KF), kvh, p.Hkv, req, pool_rows,
+                   kslot, kslot_row(1));
       grid_dep_wait();
       mbar_expect_tx(bar(B_Q), 2 * L::NH * L::HALF);
 #pragma unroll
@@ -618,9 +633,10 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
             break;
           const uint32_t kd = sbase + L::K_OFF + st * L::NH * L::HALF;
           mbar_expect_tx(bar(B_KF + st), tile_bytes);
-          load_slot<D>(kd, e0, &p.tm_kpool, &p.tm_ksuf, bar(B_KF + st), kvh, p.Hkv, req, pool_rows);
+          load_slot<D>(kd, e0, &p.tm_kpool, &p.tm_ksuf, bar(B_KF + st), kvh, p.Hkv, req, pool_rows, kslot,
+                       kslot_row(2 * j));
           load_slot<D>(kd + kBlockTokens * 128, e1, &p.tm_kpool, &p.tm_ksuf, bar(B_KF + st), kvh,
-                       p.Hkv, req, pool_rows);
+                       p.Hkv, req, pool_rows, kslot, kslot_row(2 * j + 1));
           issued_k = j + 1;
         }
         if (j >= L::NS &&

@@ -383,15 +383,80 @@ extern "C" attuner_status attuner_plan_free(attuner_plan* p) {
       p->d_buf = nullptr;
     }
   }
-  if (p->d_buf) {
+  if (p->d_buf || p->k_rot) {
     int cur = -1;
     cudaGetDevice(&cur);
     if (cur != p->device) cudaSetDevice(p->device);
-    cudaFree(p->d_buf);
+    if (p->d_buf) cudaFree(p->d_buf);
+    if (p->k_rot) cudaFree(p->k_rot);
     if (cur != p->device && cur >= 0) cudaSetDevice(cur);
   }
   delete p;
   return ATTUNER_OK;
+}
+
+// ---------------------------------------------------------------------------
+// keys rotated at assembly (App. C.2, EPIC paragraph)
+// ---------------------------------------------------------------------------
+extern "C" attuner_status attuner_plan_rotate_keys(attuner_ctx* ctx, attuner_plan* plan, void* stream) {
+  CHECK_ARG(ctx != nullptr && plan != nullptr, "ctx and plan must not be NULL");
+  CHECK_ARG(plan->ctx == ctx, "plan belongs to another context");
+  CHECK_ARG(plan->pool_gen == ctx->pool_gen, "plan was assembled before the last attuner_pool_reset");
+  if (plan->max_o_rows > 0)
+    return fail(ATTUNER_ERR_UNSUPPORTED, "attuner_plan_rotate_keys: plans with online spans between artifacts");
+  attuner_status e = set_device(ctx);
+  if (e != ATTUNER_OK) return e;
+  const attuner_config& c = ctx->cfg;
+  const int D = c.head_dim, Hkv = c.n_kv_heads;
+  const size_t n_slots = plan->blocks.size();
+  if (n_slots == 0) return ATTUNER_OK;   // no artifact: nothing to rotate, the plain read is the same
+  CHECK_ARG((long long)n_slots * Hkv * kBlockTokens < (1ll << 31), "plan too large to rotate (slots * Hkv * 64 >= 2^31)");
+  // assembled position of each slot's first token: the request's artifact
+  // tokens before it, in runtime order from position 0
+  std::vector<int32_t> pos(n_slots, 0);
+  for (int r = 0; r < plan->n_req; ++r) {
+    int32_t at = 0;
+    for (int b = plan->blk_off[r]; b < plan->blk_off[r + 1]; ++b) {
+      pos[b] = at;
+      at += plan->blocks[b] & 127;
+    }
+  }
+  const size_t key_bytes = n_slots * Hkv * kBlockTokens * D * 2;
+  if (plan->k_rot == nullptr) {
+    if (cudaMalloc(&plan->k_rot, key_bytes + n_slots * 4) != cudaSuccess) {
+      cudaGetLastError();
+      plan->k_rot = nullptr;
+      return fail(ATTUNER_ERR_OOM, "rotated-key allocation failed");
+    }
+    const uint64_t dims[2] = {(uint64_t)D, (uint64_t)n_slots * Hkv * kBlockTokens};
+    const uint64_t strides[1] = {(uint64_t)D * 2};
+    const uint32_t box[2] = {64, 64};
+    if ((e = make_map(&plan->tm_krot, plan->k_rot, 2, dims, strides, box, "rotated keys")) != ATTUNER_OK) {
+      cudaFree(plan->k_rot);
+      plan->k_rot = nullptr;
+      return e;
+    }
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int32_t* d_pos = reinterpret_cast<int32_t*>(static_cast<char*>(plan->k_rot) + key_bytes);
+  CUDA_TRY(cudaMemcpyAsync(d_pos, pos.data(), n_slots * 4, cudaMemcpyHostToDevice, st));
+  RotateParams rp{};
+  rp.kpool = reinterpret_cast<const uint4*>(ctx->kpool);
+  rp.krot = reinterpret_cast<uint4*>(plan->k_rot);
+  rp.blocks = plan_dev(plan).blocks;
+  rp.slot_pos = d_pos;
+  rp.n_slots = (int32_t)n_slots;
+  rp.Hkv = Hkv;
+  rp.D = D;
+  rp.pool_blocks = c.pool_blocks;
+  rp.status = ctx->d_status;
+  for (int j = 0; j < D / 2; ++j) rp.inv_freq[j] = std::pow((double)c.rope_theta, -2.0 * j / D);
+  CUDA_TRY(launch_rotate_keys(rp, st));
+  // the positions are read by the kernel from pageable host memory's copy:
+  // keep `pos` alive until the copy has been made
+  CUDA_TRY(cudaStreamSynchronize(st));
+  ctx->last_launches = 1;
+  return finish_call(ctx, ATTUNER_OK, st);
 }
 
 PlanDev att::plan_dev(const attuner_plan* p) {
@@ -621,8 +686,9 @@ void att::query_cluster_occupancy(attuner_ctx* ctx) {
 }
 
 attuner_status att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc,
-                              WorkTable& w) {
+                              WorkTable& w, int kv_part) {
   SplitPolicy pol;
+  pol.kv_part = kv_part;
   pol.n_q_heads = ctx->cfg.n_q_heads;
   pol.n_kv_heads = ctx->cfg.n_kv_heads;
   pol.num_sms = ctx->num_sms;
@@ -637,7 +703,7 @@ attuner_status att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, 
 attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
                                   const void* suffix_k, const void* suffix_v, int32_t S, int32_t S_kv,
                                   void* out, float* lse_out, cudaStream_t st, const FixedScratch* fixed,
-                                  int& launches) {
+                                  int& launches, const AttendVariant& var) {
   const attuner_config& c = ctx->cfg;
   CHECK_ARG(q && suffix_k && suffix_v && out, "q, suffix_k, suffix_v and out must not be NULL");
   CHECK_ARG(aligned16(q) && aligned16(suffix_k) && aligned16(suffix_v) && aligned16(out),
@@ -652,8 +718,9 @@ attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, co
   AttnParams ap{};   // on the stack: the launch itself touches no heap
   attuner_status e = ATTUNER_OK;
   if (tc) query_cluster_occupancy(ctx);
-  if ((e = make_work(ctx, plan, S, S_kv, tc, ap.work)) != ATTUNER_OK) return e;
+  if ((e = make_work(ctx, plan, S, S_kv, tc, ap.work, var.kv_part)) != ATTUNER_OK) return e;
   const WorkTable& w = ap.work;
+  if (w.n_cta == 0) return ATTUNER_OK;   // no request has a slot of this part
   bool need_combine = false;   // split partial results in global memory
   for (int r = 0; r < plan->n_req; ++r) need_combine |= (w.nsplit[r] > 1);
   if (w.cluster > 0) need_combine = false;
@@ -695,10 +762,15 @@ attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, co
   ap.Hq = Hq;
   ap.Hkv = Hkv;
   ap.G = G;
-  ap.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D));
+  ap.scale_log2 = (float)(1.4426950408889634 / (std::sqrt((double)D) * (double)var.temperature));
   ap.status = ctx->d_status;
   ap.wait_limit = ctx->wait_limit;
   ap.inject_stuck = ctx->inject_stuck;
+  ap.kv_part = var.kv_part;
+  if (plan->k_rot != nullptr) {
+    ap.k_by_slot = 1;
+    ap.tm_kslot = plan->tm_krot;
+  }
 
   void* part = nullptr;
   cudaError_t ce = cudaSuccess;
@@ -809,6 +881,66 @@ extern "C" attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_p
   if (e == ATTUNER_OK)
     e = attend_launch(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse_out, st, nullptr, launches);
   cudaFreeAsync(sc.base, st);
+  ctx->last_launches = launches;
+  return finish_call(ctx, e, st);
+}
+
+// ---------------------------------------------------------------------------
+// APE-style read (App. C.2, APE paragraph): context and online attention
+// computed separately, combined through calibrated log-sum-exp terms
+// ---------------------------------------------------------------------------
+extern "C" attuner_status attuner_attend_ape(attuner_ctx* ctx, const attuner_plan* plan, const void* q,
+                                             const void* suffix_k, const void* suffix_v, int32_t S, int32_t S_kv,
+                                             float temperature, float scale, void* out, float* lse_out,
+                                             void* stream) {
+  attuner_status e = check_common(ctx, plan, S, S_kv);
+  if (e != ATTUNER_OK) return e;
+  if (plan->max_o_rows > 0)
+    return fail(ATTUNER_ERR_UNSUPPORTED, "attuner_attend_ape: plans with online spans between artifacts");
+  CHECK_ARG(temperature > 0.f && scale > 0.f && std::isfinite(temperature) && std::isfinite(scale),
+            "temperature and scale must be positive and finite");
+  CHECK_ARG(out != nullptr && aligned16(out), "out must not be NULL and must be 16-byte aligned");
+  if ((e = set_device(ctx)) != ATTUNER_OK) return e;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const attuner_config& c = ctx->cfg;
+  const size_t rows = (size_t)plan->n_req * S * c.n_q_heads;
+  auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
+  const size_t o_bytes = al(rows * c.head_dim * 2), l_bytes = al(rows * 4);
+  void* base = nullptr;
+  CUDA_TRY(cudaMallocFromPoolAsync(&base, 2 * (o_bytes + l_bytes), ctx->mempool, st));
+  char* b = static_cast<char*>(base);
+  void* o_ctx = b;
+  float* lse_ctx = reinterpret_cast<float*>(b + o_bytes);
+  void* o_on = b + o_bytes + l_bytes;
+  float* lse_on = reinterpret_cast<float*>(b + 2 * o_bytes + l_bytes);
+  int launches = 0;
+  AttendVariant ctx_part;
+  ctx_part.kv_part = 1;
+  ctx_part.temperature = temperature;
+  AttendVariant online_part;
+  online_part.kv_part = 2;
+  e = attend_launch(ctx, plan, q, suffix_k, suffix_v, S, S_kv, o_ctx, lse_ctx, st, nullptr, launches, ctx_part);
+  if (e == ATTUNER_OK)
+    e = attend_launch(ctx, plan, q, suffix_k, suffix_v, S, S_kv, o_on, lse_on, st, nullptr, launches, online_part);
+  if (e == ATTUNER_OK) {
+    ApeParams ap{};
+    ap.o_ctx = static_cast<const __nv_bfloat16*>(o_ctx);
+    ap.lse_ctx = lse_ctx;
+    ap.o_on = static_cast<const __nv_bfloat16*>(o_on);
+    ap.lse_on = lse_on;
+    ap.out = static_cast<__nv_bfloat16*>(out);
+    ap.lse_out = lse_out;
+    ap.t_art = plan_dev(plan).t_art;
+    ap.n_req = plan->n_req;
+    ap.S = S;
+    ap.Hq = c.n_q_heads;
+    ap.D = c.head_dim;
+    ap.scale = scale;
+    const cudaError_t ce = launch_ape_combine(ap, st);
+    if (ce != cudaSuccess) e = fail(ATTUNER_ERR_CUDA, std::string("APE combine launch failed: ") + cudaGetErrorString(ce));
+    else ++launches;
+  }
+  cudaFreeAsync(base, st);
   ctx->last_launches = launches;
   return finish_call(ctx, e, st);
 }

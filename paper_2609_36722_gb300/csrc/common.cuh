@@ -73,6 +73,18 @@ ATT_DEV int online_position(const PlanDev& pl, int req, int t) {
   return t;   // not reached for a valid plan
 }
 
+// cos and sin of the RoPE angle pos * inv_freq: the angle formed and reduced
+// modulo 2 pi in double (positions reach 2^22 and more), then sin / cos in
+// float on |angle| <= pi.
+ATT_DEV float2 rope_cos_sin(long long pos, double inv_freq) {
+  const double ang = (double)pos * inv_freq;
+  const double k = rint(ang * 0.15915494309189533577);   // 1 / (2 pi)
+  const double red = fma(-k, 6.283185307179586232, ang);
+  float sn, cs;
+  sincosf((float)red, &sn, &cs);
+  return make_float2(cs, sn);
+}
+
 ATT_DEV int find_req(const WorkTable& w, int cta) {
   int lo = 0, hi = w.n_req - 1;
   while (lo < hi) {

@@ -62,6 +62,10 @@ struct attuner_plan : att::PlanTables {
   uint64_t pool_gen = 0;          // the context's pool generation at assembly
   size_t spans_at = 0;            // int32 offset of spans in d_buf
   int32_t* d_buf = nullptr;       // blk_off | blocks | t_art | o_rows | span_off | spans
+  // keys rotated at assembly (attuner_plan_rotate_keys): [n_slots][Hkv][64][d]
+  // bf16, then the slots' assembled positions; null until rotated
+  void* k_rot = nullptr;
+  CUtensorMap tm_krot{};
 };
 
 namespace att {
@@ -80,7 +84,8 @@ bool aligned16(const void* p);
 PlanDev plan_dev(const attuner_plan* p);
 attuner_status check_common(attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv);
 // split-KV decomposition of one attention launch (tc: tcgen05 kernel, else warp-MMA kernel)
-attuner_status make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc, WorkTable& w);
+attuner_status make_work(const attuner_ctx* ctx, const attuner_plan* plan, int S, int S_kv, bool tc, WorkTable& w,
+                         int kv_part = 0);
 // fills ctx->tc_clusters on first use (queries the device)
 void query_cluster_occupancy(attuner_ctx* ctx);
 // A caller-provided device region for the split-KV partial results of one
@@ -95,9 +100,16 @@ struct FixedScratch {
 // `fixed`, and a call needing more than fixed->cap bytes fails with
 // INVALID_ARG before anything is launched.  Adds the kernels launched to
 // `launches`.
+// What a launch reads besides the plain read: which slots (kv_part as in
+// SplitPolicy) and the softmax temperature of the logits.
+struct AttendVariant {
+  int kv_part = 0;
+  float temperature = 1.f;
+};
 attuner_status attend_launch(attuner_ctx* ctx, const attuner_plan* plan, const void* q, const void* suffix_k,
                              const void* suffix_v, int32_t S, int32_t S_kv, void* out, float* lse_out,
-                             cudaStream_t st, const FixedScratch* fixed, int& launches);
+                             cudaStream_t st, const FixedScratch* fixed, int& launches,
+                             const AttendVariant& var = AttendVariant());
 // the status a compute call returns: `e`, or with ATTUNER_OPT_SYNC_CHECK set
 // and nothing failed on the host, the device status after `st` drains
 attuner_status finish_call(attuner_ctx* ctx, attuner_status e, cudaStream_t st);

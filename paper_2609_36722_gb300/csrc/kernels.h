@@ -69,10 +69,16 @@ struct AttnParams {
   float* part_lse;               // [n_cta, rows_per_tile]
   int* unit_cnt;                 // K2: arrivals per (request, KV head, row tile); zero on entry, left zero
   int32_t S, S_kv, Hq, Hkv, G;
-  float scale_log2;              // log2(e) / sqrt(D)
+  float scale_log2;              // log2(e) / (sqrt(D) * temperature), temperature 1 but for APE's context part
   int* status;
   long long wait_limit;
   int32_t inject_stuck;          // test hook: one role waits on a barrier nothing arrives at
+  // keys rotated at assembly (attuner_plan_rotate_keys): artifact slot s of
+  // the plan (global slot index blk_off[req] + slot) reads its K from rows
+  // (s * Hkv + kv head) * 64 of tm_kslot instead of the pool; V from the pool
+  CUtensorMap tm_kslot;
+  int32_t k_by_slot;
+  int32_t kv_part;               // slots read: 0 all, 1 the plan's (artifacts), 2 the final online span
 };
 
 struct CombineParams {
@@ -96,6 +102,41 @@ struct HostBatch {
   int32_t first[ATTUNER_MAX_HOST_BATCH];
   int32_t n, Hkv, D;
 };
+// Keys rotated at assembly (App. C.2, EPIC paragraph): for every artifact
+// slot s of a plan (entry blocks[s] > 0: pool block, valid tokens), token t
+// of the slot is rotated at assembled position slot_pos[s] + t and written
+// to krot[s][h][t][:] for every KV head h; rows t >= valid are zeroed.
+// Online slots are skipped.
+struct RotateParams {
+  const uint4* kpool;            // [pool_blocks][Hkv][64][D] bf16, keys stored before RoPE
+  uint4* krot;                   // [n_slots][Hkv][64][D] bf16
+  const int32_t* blocks;         // [n_slots] the plan's slot entries
+  const int32_t* slot_pos;       // [n_slots] assembled position of each slot's first token
+  int32_t n_slots, Hkv, D, pool_blocks;
+  int* status;
+  double inv_freq[64];           // theta^(-2j/D), j < D/2
+};
+cudaError_t launch_rotate_keys(const RotateParams& p, cudaStream_t st);
+
+// APE's calibrated combination (App. C.2, APE paragraph) of the context part
+// (attention over the artifacts, logits divided by the temperature) and the
+// online part (causal attention over the suffix), row by row:
+//   w_c : w_o = exp(scale * lse_ctx) : exp(lse_on), out = w_c o_ctx + w_o o_on
+//   (normalised), lse = log(exp(scale * lse_ctx) + exp(lse_on)).
+// A request without artifacts (t_art 0) takes the online part alone.
+struct ApeParams {
+  const __nv_bfloat16* o_ctx;    // [n_req, S, Hq, D]
+  const float* lse_ctx;          // [n_req, S, Hq]
+  const __nv_bfloat16* o_on;
+  const float* lse_on;
+  __nv_bfloat16* out;
+  float* lse_out;                // or nullptr
+  const int32_t* t_art;          // [n_req]
+  int32_t n_req, S, Hq, D;
+  float scale;
+};
+cudaError_t launch_ape_combine(const ApeParams& p, cudaStream_t st);
+
 cudaError_t launch_pool_write_host(const HostBatch& b, __nv_bfloat16* kpool, __nv_bfloat16* vpool,
                                    int num_sms, cudaStream_t st);
 cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __nv_bfloat16* kpool,

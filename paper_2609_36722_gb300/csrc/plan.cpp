@@ -136,9 +136,13 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
   const int G = pol.n_q_heads / pol.n_kv_heads, Hkv = pol.n_kv_heads;
   const int rows = tc ? kTcRows : kMmaRows;
   const int row_tiles = (S * G + rows - 1) / rows;
-  // slots of request r: the plan's, then the chunks of its final online span
+  // slots of request r the launch reads: the plan's, then the chunks of its
+  // final online span (or one of the two, kv_part)
   auto nslots = [&](int r) {
-    return t.blk_off[r + 1] - t.blk_off[r] + (S_kv - t.o_rows[r] + kBlockTokens - 1) / kBlockTokens;
+    int lo, hi;
+    kv_part_range(pol.kv_part, t.blk_off[r + 1] - t.blk_off[r],
+                  (S_kv - t.o_rows[r] + kBlockTokens - 1) / kBlockTokens, lo, hi);
+    return hi - lo;
   };
   long long total = 0;
   int maxv = 0;
@@ -148,6 +152,18 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
     maxv = std::max(maxv, nv);
   }
   const long long units = (long long)t.n_req * Hkv * row_tiles;
+  w.n_req = t.n_req;
+  w.row_tiles = row_tiles;
+  if (maxv == 0) {   // no request has a slot to read (a part-only launch): no CTA
+    w.cluster = 0;
+    w.chunk_blocks = tc ? 2 : 16;
+    for (int r = 0; r < t.n_req; ++r) {
+      w.base[r] = 0;
+      w.nsplit[r] = 0;
+    }
+    w.n_cta = 0;
+    return ATTUNER_OK;
+  }
   // Cluster mode (tcgen05 kernel): every row tile cut into ns (2 or 4)
   // chunks, one cluster of ns CTAs per row tile.  Cost in 128-key tile times: waves of
   // co-resident clusters x (largest chunk + ~4 tiles of prologue and epilogue

@@ -11,6 +11,13 @@
 
 #include "../../include/attuner.h"
 
+// functions that the kernels use too (plain inline C++ for the host-only build)
+#ifdef __CUDACC__
+#define ATT_HD __host__ __device__ __forceinline__
+#else
+#define ATT_HD inline
+#endif
+
 namespace att {
 
 constexpr int kBlockTokens = ATTUNER_BLOCK_TOKENS;   // 64 tokens per paged block
@@ -93,7 +100,18 @@ struct SplitPolicy {
   int32_t opt_split;          // virtual blocks per chunk, 0 = chosen here
   int32_t opt_merge;          // 0 = chosen here, 1 = through global memory, 2 = cluster
   int32_t tc_clusters[9];     // co-resident clusters of n tcgen05 CTAs (n = 2, 4)
+  // which slots of each request the launch reads: 0 every slot, 1 the plan's
+  // slots only (the artifacts of a plan without online spans), 2 the chunks
+  // of the final online span only (the suffix)
+  int32_t kv_part = 0;
 };
+
+// The slots [lo, hi) of a request that a launch reads, out of its nab plan
+// slots and nsuf chunks of the final online span (kv_part as in SplitPolicy).
+ATT_HD void kv_part_range(int kv_part, int nab, int nsuf, int& lo, int& hi) {
+  lo = (kv_part == 2) ? nab : 0;
+  hi = (kv_part == 1) ? nab : nab + nsuf;
+}
 
 // Split-KV decomposition of one attention launch over S query rows and S_kv
 // online rows per request (tc: the tcgen05 kernel, else the warp-MMA kernel).

@@ -3,7 +3,9 @@
 //     encoded alone at local positions, never changed afterwards) into its
 //     paged pool blocks [block][Hkv][64][D];
 //   * prep: the cos/sin table of every query row's RoPE angles (App. A.5
-//     position ids of the assembled context).
+//     position ids of the assembled context);
+//   * rotate_keys: keys stored before RoPE rotated to their assembled
+//     positions when a plan is assembled (App. C.2, EPIC paragraph).
 #include <math.h>
 
 #include <algorithm>
@@ -125,12 +127,64 @@ __global__ void __launch_bounds__(256) prep_kernel(const __grid_constant__ PrepP
   const int j = (int)(idx / p.M), m = (int)(idx % p.M);   // pair-major: coalesced in the epilogue
   const int req = m / p.S, i = m % p.S;
   const long long pos = online_position(p.plan, req, (p.S_kv - p.S) + i);   // assembled position
-  const double ang = (double)pos * p.inv_freq[j];
-  const double k = rint(ang * 0.15915494309189533577);   // 1 / (2 pi)
-  const double red = fma(-k, 6.283185307179586232, ang);
-  float sn, cs;
-  sincosf((float)red, &sn, &cs);
-  p.rope[(long long)j * p.M + m] = make_float2(cs, sn);
+  p.rope[(long long)j * p.M + m] = rope_cos_sin(pos, p.inv_freq[j]);
+}
+
+// One thread per (slot, token row, group of 8 rotary pairs): the cos/sin of
+// its 8 angles once, then for every KV head two 16-byte loads (columns
+// j0..j0+7 and their partners j0+D/2..) and two 16-byte stores; consecutive
+// threads take consecutive pair groups of a row, so each head's row is read
+// and written by D/16 neighbouring threads.
+__global__ void __launch_bounds__(256) rotate_keys_kernel(const __grid_constant__ RotateParams p) {
+  const int groups = p.D / 16;                          // 8-pair groups per row
+  const long long idx = (long long)blockIdx.x * 256 + threadIdx.x;
+  if (idx >= (long long)p.n_slots * kBlockTokens * groups) return;
+  const int g = (int)(idx % groups);
+  const int t = (int)((idx / groups) % kBlockTokens);
+  const int s = (int)(idx / ((long long)groups * kBlockTokens));
+  const int e = p.blocks[s];
+  if (e <= 0) return;                                   // online slot: its keys come from the suffix
+  const int valid = e & 127, blk = e >> 7;
+  if (blk >= p.pool_blocks || valid < 1 || valid > kBlockTokens) {
+    set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
+    return;
+  }
+  const int cpr = p.D / 8;                              // 16-byte chunks per row
+  const int j0 = 8 * g;                                 // first pair of the group
+  float2 cs[8];
+  if (t < valid) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) cs[k] = rope_cos_sin((long long)p.slot_pos[s] + t, p.inv_freq[j0 + k]);
+  }
+  for (int h = 0; h < p.Hkv; ++h) {
+    const long long src = (((long long)blk * p.Hkv + h) * kBlockTokens + t) * cpr;
+    const long long dst = (((long long)s * p.Hkv + h) * kBlockTokens + t) * cpr;
+    uint4 y1 = make_uint4(0, 0, 0, 0), y2 = make_uint4(0, 0, 0, 0);
+    if (t < valid) {
+      const uint4 a = p.kpool[src + g], b = p.kpool[src + g + cpr / 2];
+      const __nv_bfloat16* x1 = reinterpret_cast<const __nv_bfloat16*>(&a);
+      const __nv_bfloat16* x2 = reinterpret_cast<const __nv_bfloat16*>(&b);
+      uint32_t* o1 = reinterpret_cast<uint32_t*>(&y1);
+      uint32_t* o2 = reinterpret_cast<uint32_t*>(&y2);
+#pragma unroll
+      for (int k = 0; k < 8; k += 2) {
+        const float u0 = __bfloat162float(x1[k]), u1 = __bfloat162float(x1[k + 1]);
+        const float v0 = __bfloat162float(x2[k]), v1 = __bfloat162float(x2[k + 1]);
+        // rotate-half: (x_j, x_{j+D/2}) -> (x_j c - x_{j+D/2} s, x_{j+D/2} c + x_j s)
+        o1[k / 2] = pack_bf16(u0 * cs[k].x - v0 * cs[k].y, u1 * cs[k + 1].x - v1 * cs[k + 1].y);
+        o2[k / 2] = pack_bf16(v0 * cs[k].x + u0 * cs[k].y, v1 * cs[k + 1].x + u1 * cs[k + 1].y);
+      }
+    }
+    p.krot[dst + g] = y1;
+    p.krot[dst + g + cpr / 2] = y2;
+  }
+}
+
+cudaError_t launch_rotate_keys(const RotateParams& p, cudaStream_t st) {
+  const long long n = (long long)p.n_slots * kBlockTokens * (p.D / 16);
+  if (n == 0) return cudaSuccess;
+  rotate_keys_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(p);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st) {

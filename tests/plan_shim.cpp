@@ -61,10 +61,21 @@ extern "C" int shim_export(const int32_t* first, const int32_t* L, int32_t n_art
 // o_rows; out = n_req, row_tiles, chunk_blocks, n_cta, cluster, base[n_req],
 // nsplit[n_req].  pol = n_q_heads, n_kv_heads, num_sms, opt_split, opt_merge,
 // tc_clusters[9].
+extern "C" int shim_split_part(const int32_t* pol, const int32_t* blk_off, const int32_t* o_rows, int32_t n_req,
+                               int32_t S, int32_t S_kv, int32_t tc, int32_t kv_part, int32_t* out);
+
 extern "C" int shim_split(const int32_t* pol, const int32_t* blk_off, const int32_t* o_rows, int32_t n_req,
                           int32_t S, int32_t S_kv, int32_t tc, int32_t* out) {
+  return shim_split_part(pol, blk_off, o_rows, n_req, S, S_kv, tc, 0, out);
+}
+
+// As shim_split, for a launch that reads only some slots of each request:
+// kv_part 1 the plan's slots, 2 the chunks of the final online span.
+extern "C" int shim_split_part(const int32_t* pol, const int32_t* blk_off, const int32_t* o_rows, int32_t n_req,
+                               int32_t S, int32_t S_kv, int32_t tc, int32_t kv_part, int32_t* out) {
   if (n_req < 1 || n_req > att::kMaxReq) return ATTUNER_ERR_INVALID_ARG;
   att::SplitPolicy p;
+  p.kv_part = kv_part;
   p.n_q_heads = pol[0];
   p.n_kv_heads = pol[1];
   p.num_sms = pol[2];

@@ -218,6 +218,9 @@ def test_every_public_method_reaches_its_entry_point(ctx, monkeypatch):
                                   "attuner_attend_static_scratch"),
         "query_attend": (lambda: c.query_attend(plan, x, w, la, lb, 2.0, qn, sk, sv, out=q, lse=lse, stream=st),
                          "attuner_query_attend"),
+        "rotate_keys": (lambda: c.rotate_keys(plan, stream=st), "attuner_plan_rotate_keys"),
+        "attend_ape": (lambda: c.attend_ape(plan, q, sk, sv, 0.9, 0.9, out=out, lse=lse, stream=st),
+                       "attuner_attend_ape"),
         "pool_tensors": (lambda: c.pool_tensors(), "attuner_pool_info"),
         "sync_status": (lambda: c.sync_status(stream=st), "attuner_sync_status"),
         "set_option": (lambda: c.set_option(A.OPT_SPLIT_BLOCKS, 4), "attuner_set_option"),

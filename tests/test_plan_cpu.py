@@ -262,17 +262,19 @@ def test_export_capacity_checks(shim):
 # split-KV decomposition
 # ---------------------------------------------------------------------------
 def split(shim, n_q, n_kv, nv_art, o_rows, S, S_kv, tc, num_sms=152, opt_split=0, opt_merge=0,
-          clusters=(0, 0, 37, 0, 18, 0, 0, 0, 0)):
+          clusters=(0, 0, 37, 0, 18, 0, 0, 0, 0), kv_part=0):
     n_req = len(nv_art)
     pol = _i32([n_q, n_kv, num_sms, opt_split, opt_merge] + list(clusters))
     blk = _i32(np.cumsum([0] + list(nv_art)))
     orow = _i32(o_rows)
     out = np.zeros(5 + 2 * n_req, np.int32)
-    st = shim.shim_split(pol[1], blk[1], orow[1], n_req, S, S_kv, int(tc), out.ctypes.data_as(I32P))
+    st = shim.shim_split_part(pol[1], blk[1], orow[1], n_req, S, S_kv, int(tc), kv_part, out.ctypes.data_as(I32P))
     assert st == OK
     w = dict(n_req=int(out[0]), row_tiles=int(out[1]), chunk=int(out[2]), n_cta=int(out[3]), cluster=int(out[4]),
              base=out[5:5 + n_req].tolist(), nsplit=out[5 + n_req:].tolist())
-    nv = [nv_art[r] + -(-(S_kv - o_rows[r]) // 64) for r in range(n_req)]
+    # the slots the launch reads: the plan's, the final span's chunks, or both
+    nsuf = [-(-(S_kv - o_rows[r]) // 64) for r in range(n_req)]
+    nv = [(nv_art[r] if kv_part != 2 else 0) + (nsuf[r] if kv_part != 1 else 0) for r in range(n_req)]
     return w, nv
 
 
@@ -335,6 +337,27 @@ def test_split_work_covers_every_block_once(shim):
             assert w["cluster"] == 0
         if not tc:
             assert w["chunk"] >= (opt_split if opt_split else 16)
+
+
+def test_split_work_of_one_part_covers_its_slots_once(shim):
+    # a launch over the artifact slots only (kv_part 1: requests without
+    # artifacts get no CTA) or the suffix chunks only (kv_part 2), as the APE
+    # read makes them; plans without online spans
+    rng = np.random.default_rng(22)
+    for trial in range(200):
+        n_kv = int(rng.choice([1, 2, 4, 8]))
+        G = int(rng.choice([1, 2, 4, 8]))
+        n_req = int(rng.integers(1, 7))
+        tc = bool(rng.random() < 0.6)
+        S = int(rng.integers(1, 300)) if tc else int(rng.integers(1, 3))
+        nv_art = [int(rng.integers(0, 400)) if rng.random() < 0.8 else 0 for _ in range(n_req)]
+        S_kv = S + int(rng.integers(0, 64))
+        kv_part = int(rng.integers(1, 3))
+        clusters = (0, 0, int(rng.choice([0, 37, 76])), 0, int(rng.choice([0, 18, 38])), 0, 0, 0, 0)
+        w, nv = split(shim, G * n_kv, n_kv, nv_art, [0] * n_req, S, S_kv, tc, opt_split=int(rng.choice([0, 2, 6])),
+                      opt_merge=int(rng.integers(0, 3)), clusters=clusters, kv_part=kv_part)
+        assert nv == (nv_art if kv_part == 1 else [-(-S_kv // 64)] * n_req)
+        check_work(w, nv, n_kv, S, G, tc)
 
 
 def test_split_work_choices(shim):
