@@ -261,7 +261,11 @@ def rotate_at_assembly(art_k_raw: Sequence[np.ndarray], theta: float) -> np.ndar
 def epic_request_forward(x, w_q, a, b, s, q_norm_w, eps, theta, art_k_raw: List[np.ndarray],
                          art_v: List[np.ndarray], suffix_k, suffix_v, n_q_heads: int, pairs=None):
     """request_forward with the artifact keys stored before RoPE and rotated
-    at their assembled positions; queries and suffix keys as there."""
+    at their assembled positions; queries and suffix keys as there.  An empty
+    artifact list leaves nothing to rotate: the plain read of the suffix."""
+    if len(art_k_raw) == 0:
+        return request_forward(x, w_q, a, b, s, q_norm_w, eps, theta, [], [], suffix_k, suffix_v, n_q_heads,
+                               pairs=pairs)
     k_art = rotate_at_assembly(art_k_raw, theta)
     v_art = np.concatenate(list(art_v), axis=0)
     return request_forward(x, w_q, a, b, s, q_norm_w, eps, theta, [k_art], [v_art], suffix_k, suffix_v,

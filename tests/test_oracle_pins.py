@@ -594,6 +594,18 @@ def test_epic_single_artifact_is_the_pic_read():
     np.testing.assert_allclose(lse, lse2, atol=1e-13)
 
 
+def test_epic_without_artifacts_is_causal_attention_over_the_suffix():
+    # nothing to rotate: the suffix rows of plain causal attention, against
+    # fp64 SDPA with the queries at positions (S_kv - S) + i
+    rng = np.random.default_rng(37)
+    c = _variant_case(rng, lens=())
+    o, _ = _epic(c)
+    q, _ = _queries(c)
+    S, S_kv = c["x"].shape[0], c["suffix_k"].shape[0]
+    np.testing.assert_allclose(o, _sdpa_f64(q, c["suffix_k"], c["suffix_v"], (S_kv - S) + np.arange(S) + 1),
+                               atol=1e-12)
+
+
 def test_rotate_at_assembly_positions():
     # token t of the concatenation is rotated at t: a unit vector in pair 0
     # turns by t * theta^0 = t radians
