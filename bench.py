@@ -655,6 +655,52 @@ def measure_warm_cache(bed, args, world, flush, local_rank):
                         "the step's new tokens (x and their own suffix K/V rows), Q projection, attention, D2H of O"}
 
 
+def measure_variants(bed, args, timer):
+    """The two read variants of the paper's training-free baselines (App.
+    C.2) on the same layer: APE's separate context (temperature 0.9) and
+    online attention with the calibrated combine (scale 0.9), and EPIC's keys
+    stored before RoPE and rotated to their assembled positions at assembly
+    (the rotation kernel, then the attention over the rotated keys).  Both
+    count the same visible (query, key) pairs as the plain read."""
+    import torch
+    wl, ctx = bed.wl, bed.ctx
+    flops = attention_flops(wl)
+    ms = timer.time(lambda: ctx.attend_ape(bed.plan, bed.q, wl.suffix_k, wl.suffix_v, 0.9, 0.9, out=bed.out,
+                                           lse=bed.lse), args.steps)
+    ape_launches = ctx.last_launch_count()
+    ape = {"avg_call_ms": round(statistics.mean(ms), 5),
+           "tflops": round(flops / (statistics.mean(ms) * 1e-3) / 1e12, 3), "launches": ape_launches,
+           "temperature": 0.9, "scale": 0.9}
+    rplan = ctx.assemble(wl.requests)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    rot_ms = []
+    for i in range(max(3, min(args.steps, 10))):
+        timer.flush.zero_()
+        e0.record()
+        ctx.rotate_keys(rplan)
+        e1.record()
+        e1.synchronize()
+        if i >= 1:
+            rot_ms.append(e0.elapsed_time(e1))
+    g = bed.g
+    n_slots = sum(-(-wl.art_lengths[a] // 64) for r in wl.requests for a in r)
+    # the artifact tokens' keys read once, every slot's rows written once
+    rot_bytes = (sum(wl.t_art(r) for r in range(wl.n_req)) + n_slots * 64) * g.n_kv_heads * g.head_dim * 2
+    ms = timer.time(lambda: ctx.attend(rplan, bed.q, wl.suffix_k, wl.suffix_v, out=bed.out, lse=bed.lse),
+                    args.steps)
+    rplan.free()
+    if ctx.sync_status() != 0:
+        raise RuntimeError("device status after the read variants")
+    peaks = _peaks()
+    rot_gbs = rot_bytes / (statistics.mean(rot_ms) * 1e-3) / 1e9 if rot_ms else None
+    epic = {"rotate_ms": round(statistics.mean(rot_ms), 5) if rot_ms else None,
+            "rotate_gbs": round(rot_gbs, 1) if rot_gbs else None,
+            "rotate_frac_of_hbm": round(rot_gbs / peaks["hbm"], 4) if rot_gbs else None,
+            "attention_ms": round(statistics.mean(ms), 5),
+            "tflops": round(flops / (statistics.mean(ms) * 1e-3) / 1e12, 3)}
+    return {"ape": ape, "epic_rotated_keys": epic}
+
+
 def _guarded(fn, errors, label):
     """Run an optional part of the line; a failure is recorded, not raised."""
     import traceback
@@ -716,6 +762,8 @@ def run_ours(args, rank, world, local_rank):
                                                f"{b.name}.layout_attention")
             out["e2e_warm_cache"] = _guarded(lambda: measure_warm_cache(b, args, world, flush, local_rank), errors,
                                              f"{b.name}.e2e_warm_cache")
+            out["read_variants"] = _guarded(lambda: measure_variants(b, args, timer), errors,
+                                            f"{b.name}.read_variants")
         return out
 
     result.update(extras(bed))
@@ -816,7 +864,7 @@ def main():
     ap.add_argument("--no-configs", action="store_true",
                     help="time the headline workload only (no per-config sub-objects)")
     ap.add_argument("--no-sub-lines", dest="sub_lines", action="store_false",
-                    help="skip the kv_project, layout_attention and e2e_warm_cache sub-lines")
+                    help="skip the kv_project, layout_attention, e2e_warm_cache and read_variants sub-lines")
     ap.add_argument("--eager", action="store_true",
                     help="launch the timed calls directly instead of replaying CUDA graphs (for profilers)")
     args = ap.parse_args()
