@@ -59,7 +59,7 @@ __device__ __forceinline__ uint32_t s_col_of(int qt) { return qt ? 128u : 0u; }
 __device__ __forceinline__ uint32_t o_col_of(int qt) { return qt ? 384u : 256u; }
 
 constexpr int kProducerWarp = 8, kMmaWarp = 9;
-constexpr int kCtrlRegs = 80, kSoftRegs = 208;
+constexpr int kCtrlRegs = 96, kSoftRegs = 200;
 static_assert(128 * kCtrlRegs + 256 * kSoftRegs <= 384 * 168, "register split exceeds the launch budget");
 
 enum : int {
