@@ -837,11 +837,15 @@ static cudaError_t launch_attn_tc_t(const AttnParams& p, cudaStream_t st) {
   using L = TcLayout<D>;
   // setmaxnreg.inc waits until the registers it asks for are free in the
   // block's launch budget: never launch a split that exceeds that budget.
-  cudaFuncAttributes fa{};
-  cudaError_t e = cudaFuncGetAttributes(&fa, attn_tc_kernel<D, kLayout>);
-  if (e != cudaSuccess) return e;
-  if (fa.numRegs * 384 < 128 * kCtrlRegs + 256 * kSoftRegs) return cudaErrorLaunchOutOfResources;
-  e = cudaFuncSetAttribute(attn_tc_kernel<D, kLayout>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
+  // (checked once per instantiation: the register count is fixed at build time)
+  static const cudaError_t regs = [] {
+    cudaFuncAttributes fa{};
+    const cudaError_t r = cudaFuncGetAttributes(&fa, attn_tc_kernel<D, kLayout>);
+    if (r != cudaSuccess) return r;
+    return fa.numRegs * 384 < 128 * kCtrlRegs + 256 * kSoftRegs ? cudaErrorLaunchOutOfResources : cudaSuccess;
+  }();
+  if (regs != cudaSuccess) return regs;
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D, kLayout>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
   return launch_pdl(attn_tc_kernel<D, kLayout>, dim3(p.work.n_cta), dim3(384), (size_t)L::SMEM, st, p.work.cluster, p);
 }

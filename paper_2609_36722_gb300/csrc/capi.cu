@@ -158,6 +158,12 @@ extern "C" attuner_status attuner_create(const attuner_config* cfg, attuner_ctx*
   }
   uint64_t thresh = ~0ull;
   cudaMemPoolSetAttribute(ctx->mempool, cudaMemPoolAttrReleaseThreshold, &thresh);
+  if (cudaStreamCreateWithFlags(&ctx->upload_stream, cudaStreamNonBlocking) != cudaSuccess) {
+    attuner_destroy(ctx);
+    return fail(ATTUNER_ERR_CUDA, "cudaStreamCreateWithFlags failed");
+  }
+  for (int j = 0; j < cfg->head_dim / 2; ++j)
+    ctx->inv_freq[j] = std::pow((double)cfg->rope_theta, -2.0 * j / (double)cfg->head_dim);
 
   const uint64_t D = cfg->head_dim;
   const uint64_t rows = (uint64_t)cfg->pool_blocks * cfg->n_kv_heads * 64;
@@ -181,6 +187,8 @@ extern "C" attuner_status attuner_destroy(attuner_ctx* ctx) {
   if (ctx->vpool) cudaFree(ctx->vpool);
   if (ctx->d_status) cudaFree(ctx->d_status);
   if (ctx->mempool) cudaMemPoolDestroy(ctx->mempool);
+  if (ctx->upload_stream) cudaStreamDestroy(ctx->upload_stream);
+  if (ctx->staging) cudaFreeHost(ctx->staging);
   {
     std::lock_guard<std::mutex> lk(ctx->plan_mu);
     for (attuner_plan* p : ctx->live_plans) p->ctx = nullptr;
@@ -296,18 +304,35 @@ static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const 
   p->pool_gen = ctx->pool_gen;
   attuner_status s = set_device(ctx);
   if (s != ATTUNER_OK) { delete p; return s; }
-  std::vector<int32_t> h;
-  h.insert(h.end(), p->blk_off.begin(), p->blk_off.end());
-  h.insert(h.end(), p->blocks.begin(), p->blocks.end());
-  h.insert(h.end(), p->t_art.begin(), p->t_art.end());
-  h.insert(h.end(), p->o_rows.begin(), p->o_rows.end());
-  h.insert(h.end(), p->span_off.begin(), p->span_off.end());
-  while (h.size() % 4) h.push_back(0);   // int4 spans start 16-byte aligned
-  p->spans_at = h.size();
-  h.insert(h.end(), p->spans.begin(), p->spans.end());
-  if (h.empty()) h.push_back(0);
+  // the device image: blk_off | blocks | t_art | o_rows | span_off | (16-byte aligned) spans
+  const size_t head = p->blk_off.size() + p->blocks.size() + p->t_art.size() + p->o_rows.size() + p->span_off.size();
+  p->spans_at = (head + 3) & ~size_t(3);   // int4 spans start 16-byte aligned
+  const size_t n_words = std::max<size_t>(p->spans_at + p->spans.size(), 1);
+  const size_t bytes = n_words * sizeof(int32_t);
+  if (ctx->staging_cap < bytes) {
+    size_t cap = std::max<size_t>(ctx->staging_cap * 2, 1 << 16);
+    while (cap < bytes) cap *= 2;
+    void* st = nullptr;
+    if (cudaMallocHost(&st, cap) != cudaSuccess) {
+      cudaGetLastError();
+      delete p;
+      return fail(ATTUNER_ERR_OOM, "plan staging allocation failed");
+    }
+    if (ctx->staging) cudaFreeHost(ctx->staging);
+    ctx->staging = st;
+    ctx->staging_cap = cap;
+  }
+  {
+    int32_t* h = static_cast<int32_t*>(ctx->staging);
+    size_t at = 0;
+    for (const std::vector<int32_t>* v : {&p->blk_off, &p->blocks, &p->t_art, &p->o_rows, &p->span_off}) {
+      if (!v->empty()) std::memcpy(h + at, v->data(), v->size() * sizeof(int32_t));
+      at += v->size();
+    }
+    for (; at < p->spans_at; ++at) h[at] = 0;
+    if (!p->spans.empty()) std::memcpy(h + at, p->spans.data(), p->spans.size() * sizeof(int32_t));
+  }
   // a buffer of a freed plan when one is large enough (no allocation per assembly)
-  const size_t bytes = h.size() * sizeof(int32_t);
   p->ctx = ctx;
   {
     std::lock_guard<std::mutex> lk(ctx->plan_mu);
@@ -331,7 +356,9 @@ static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const 
     }
     p->d_cap = cap;
   }
-  if (cudaMemcpy(p->d_buf, h.data(), bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
+  if (cudaMemcpyAsync(p->d_buf, ctx->staging, bytes, cudaMemcpyHostToDevice, ctx->upload_stream) != cudaSuccess ||
+      cudaStreamSynchronize(ctx->upload_stream) != cudaSuccess) {
+    cudaGetLastError();
     cudaFree(p->d_buf);
     delete p;
     return fail(ATTUNER_ERR_CUDA, "plan upload failed");
@@ -450,7 +477,7 @@ extern "C" attuner_status attuner_plan_rotate_keys(attuner_ctx* ctx, attuner_pla
   rp.D = D;
   rp.pool_blocks = c.pool_blocks;
   rp.status = ctx->d_status;
-  for (int j = 0; j < D / 2; ++j) rp.inv_freq[j] = std::pow((double)c.rope_theta, -2.0 * j / D);
+  for (int j = 0; j < D / 2; ++j) rp.inv_freq[j] = ctx->inv_freq[j];
   CUDA_TRY(launch_rotate_keys(rp, st));
   // the positions are read by the kernel from pageable host memory's copy:
   // keep `pos` alive until the copy has been made
@@ -542,7 +569,7 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
   pp.D = D;
   pp.S = S;
   pp.S_kv = S_kv;
-  for (int j = 0; j < D / 2; ++j) pp.inv_freq[j] = std::pow((double)c.rope_theta, -2.0 * j / (double)D);
+  for (int j = 0; j < D / 2; ++j) pp.inv_freq[j] = ctx->inv_freq[j];
   CUDA_TRY(launch_prep(pp, st));
   ++launches;
 
@@ -622,7 +649,7 @@ static attuner_status kv_project_impl(attuner_ctx* ctx, const attuner_plan* plan
   pp.D = D;
   pp.S = S;
   pp.S_kv = S_kv;
-  for (int j = 0; j < D / 2; ++j) pp.inv_freq[j] = std::pow((double)c.rope_theta, -2.0 * j / (double)D);
+  for (int j = 0; j < D / 2; ++j) pp.inv_freq[j] = ctx->inv_freq[j];
   CUDA_TRY(launch_prep(pp, st));
   ++launches;
 

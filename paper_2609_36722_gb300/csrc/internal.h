@@ -45,6 +45,13 @@ struct attuner_ctx {
   long long wait_limit = 1ll << 32;
   int inject_stuck = 0;
   int last_launches = 0;
+  double inv_freq[64] = {};       // theta^(-2j/d), j < d/2
+  // plan uploads: a pinned staging buffer and a stream of the context's own
+  // that does not synchronise with other streams, so assembling a plan waits
+  // for its own copy only, never for kernels already running
+  cudaStream_t upload_stream = nullptr;
+  void* staging = nullptr;
+  size_t staging_cap = 0;
   // device buffers of freed plans, reused by the next assemblies (capacity,
   // pointer), and the plans not yet freed (detached when the context goes, so
   // a plan freed after its context frees its own buffer)
