@@ -499,20 +499,34 @@ def measure_e2e(bed, args, world, flush, local_rank=0):
     n_sets = max(1, -(-2 * L2_BYTES // working_set_bytes(bed)))
     beds = [bed] + [Bed(bed.name, bed.dev, local_rank) for _ in range(n_sets - 1)]
     try:
-        units = []   # (bed, host/device buffers, output) per step parity and set
+        # (bed, host/device buffers, output, inputs-copied / computed / output-on-host events)
+        units = []
         for b in beds:
             for _ in range(2):
-                units.append((b, HostInputs(b), torch.empty_like(b.out), torch.cuda.Event()))
+                units.append((b, HostInputs(b), torch.empty_like(b.out), torch.cuda.Event(), torch.cuda.Event(),
+                              torch.cuda.Event()))
         n_units = len(units)
+        compute = torch.cuda.current_stream()
+        h2d, d2h = torch.cuda.Stream(device=bed.dev), torch.cuda.Stream(device=bed.dev)
 
         def enqueue(i, plan):
-            b, io, out, ev = units[i % n_units]
+            # inputs on a copy stream, the call on the compute stream, the output
+            # on another copy stream: a step's copies overlap its neighbours'
+            # kernels.  Each unit's buffers are reused only after the step that
+            # last used them was waited for (two steps in flight at most).
+            b, io, out, ev_in, ev_comp, done = units[i % n_units]
             wl, g = b.wl, b.g
-            io.copy_in()
+            with torch.cuda.stream(h2d):
+                io.copy_in()
+                ev_in.record(h2d)
+            compute.wait_event(ev_in)
             b.ctx.query_attend(plan, io.x_d, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, io.sk_d, io.sv_d,
-                               out=out, want_lse=False)
-            io.out_h.copy_(out, non_blocking=True)
-            ev.record()
+                               out=out, want_lse=False, stream=compute)
+            ev_comp.record(compute)
+            with torch.cuda.stream(d2h):
+                d2h.wait_event(ev_comp)
+                io.out_h.copy_(out, non_blocking=True)
+                done.record(d2h)
 
         def assemble(i):
             b = units[i % n_units][0]
@@ -525,7 +539,7 @@ def measure_e2e(bed, args, world, flush, local_rank=0):
                 if i + 1 < n:
                     plans[i + 1] = assemble(i + 1)     # the next step, while step i runs
                     enqueue(i + 1, plans[i + 1])
-                units[i % n_units][3].synchronize()    # step i's output is on the host
+                units[i % n_units][5].synchronize()    # step i's output is on the host
                 plans.pop(i).free()
 
         run(max(3, args.warmup))
@@ -546,8 +560,9 @@ def measure_e2e(bed, args, world, flush, local_rank=0):
                        if n_sets > 1 else f"no flush in the loop; the {working_set_bytes(bed) / 1e6:.0f} MB working "
                                           "set of a step exceeds L2"),
                 "includes": "per step: assemble (host block table + upload), H2D of the step's new tokens (x and their "
-                            "own suffix K/V rows; a decode step's earlier suffix rows stay resident), query_attend, "
-                            "D2H of O and a wait for it; step i+1 assembled and enqueued while step i runs"}
+                            "own suffix K/V rows; a decode step's earlier suffix rows stay resident) on a copy stream, "
+                            "query_attend, D2H of O on a second copy stream and a wait for it; step i+1 assembled "
+                            "and enqueued while step i runs"}
     finally:
         for b in beds[1:]:
             b.close()

@@ -129,6 +129,11 @@ def _check(status: int):
 def _ptr(t: Optional[torch.Tensor], name: str, dtype=torch.bfloat16, device=None) -> Optional[int]:
     if t is None:
         return None
+    # the usual case in one test; which rule a tensor breaks is worked out
+    # only when it breaks one
+    if (t.dtype is dtype and t.is_cuda and (device is None or t.get_device() == device.index)
+            and t.is_contiguous()):
+        return t.data_ptr()
     if not t.is_cuda:
         raise ValueError(f"{name} must be a CUDA tensor")
     if device is not None and t.device != device:
@@ -140,9 +145,15 @@ def _ptr(t: Optional[torch.Tensor], name: str, dtype=torch.bfloat16, device=None
     return t.data_ptr()
 
 
+# the current stream of a device as a raw handle, without building a Stream object
+_RAW_STREAM = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+
+
 def _stream(stream, device=None) -> Optional[int]:
     # the caller's stream, else the current stream of the context's device
     if stream is None:
+        if _RAW_STREAM is not None and device is not None and torch.cuda.is_initialized():
+            return _RAW_STREAM(device.index)
         stream = torch.cuda.current_stream(device)
     elif device is not None and getattr(stream, "device", device) != device:
         raise ValueError(f"stream is on {stream.device}, the context on {device}")

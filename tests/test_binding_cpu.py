@@ -33,6 +33,9 @@ class FakeTensor:
     def is_pinned(self):
         return self._pinned
 
+    def get_device(self):
+        return self.device.index if self.is_cuda else -1
+
     def data_ptr(self):
         return self._ptr
 

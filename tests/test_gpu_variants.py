@@ -151,3 +151,46 @@ def test_variants_refuse_prompt_layouts_and_bad_parameters():
             ctx.attend_ape(plan, q, wl.suffix_k, wl.suffix_v, T, sc)
         assert e.value.status == pkg.attuner.ERR_INVALID_ARG
     assert ctx.sync_status() == 0
+
+
+def _sampled_variant_check(wl, out, lse, fn, label, **kw):
+    from helpers import sample_pairs
+    f = oracle.bf16_to_f64
+    g = wl.geom
+    trip = sample_pairs(wl, n=256, seed=7)
+    o_sel, l_sel, o_ref, l_ref = [], [], [], []
+    for r, ids in enumerate(wl.requests):
+        pairs = [(i, h) for (rr, i, h) in trip if rr == r]
+        if not pairs:
+            continue
+        o, l = fn(f(wl.x[r]), f(wl.w_q), f(wl.lora_a), f(wl.lora_b), g.scale, f(wl.q_norm_w), g.rms_eps,
+                  g.rope_theta, [f(wl.art_k[i]) for i in ids], [f(wl.art_v[i]) for i in ids], f(wl.suffix_k[r]),
+                  f(wl.suffix_v[r]), g.n_q_heads, pairs=pairs, **kw)
+        o_ref.append(o)
+        l_ref.append(l)
+        idx_i = torch.tensor([i for i, _ in pairs], device=DEV)
+        idx_h = torch.tensor([h for _, h in pairs], device=DEV)
+        o_sel.append(_np(out[r][idx_i, idx_h]))
+        l_sel.append(_np(lse[r][idx_i, idx_h]))
+    compare(np.concatenate(o_sel), np.concatenate(o_ref), np.concatenate(l_sel), np.concatenate(l_ref),
+            label=f"{label} ({len(trip)} sampled rows)")
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", ["qwen3_4b_prefill", "qwen3_8b_decode_64req"])
+def test_variants_at_full_size(name):
+    # the two variants on full workloads, in the launch configuration the
+    # bench times (automatic kernel, split and merge choice), on sampled rows
+    from gen import make_workload
+    from helpers import load_context
+    wl = make_workload(name, device=DEV)
+    ctx, plan = load_context(wl)
+    g = wl.geom
+    q = ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv)
+    out, lse = ctx.attend_ape(plan, q, wl.suffix_k, wl.suffix_v, 0.9, 0.9)
+    assert ctx.sync_status() == 0
+    _sampled_variant_check(wl, out, lse, oracle.ape_request_forward, f"ape {name}", temperature=0.9, scale=0.9)
+    ctx.rotate_keys(plan)
+    out, lse = ctx.attend(plan, q, wl.suffix_k, wl.suffix_v)
+    assert ctx.sync_status() == 0
+    _sampled_variant_check(wl, out, lse, oracle.epic_request_forward, f"epic {name}")
