@@ -415,7 +415,7 @@ def measure_core(bed, args, world, timer, with_clocks=False, local_rank=0):
         "ms_per_step": round(total_ms / args.steps, 5),
         "roofline": {"bound": "hbm" if bed.decode else "tensor", "achieved": round(achieved, 3), "peak": peak,
                      "unit": bed.unit, "frac": round(achieved / peak, 4), "traffic": load_traffic(bed.name),
-                     "kernel": ("attn_mma_kernel + combine_kernel" if bed.decode
+                     "kernel": ("attn_mma_kernel (split-KV chunks merged inside it)" if bed.decode
                                 else "attn_tc_kernel (split-KV chunks merged inside it)"),
                      "work_per_launch": bed.work,
                      "work_unit": "bytes (each request's assembled K and V read once)" if bed.decode

@@ -1,8 +1,9 @@
 // attn_mma.cu - K3: split-KV attention for few query rows per (request, KV
 // head), the decode step of Sec. 3 (generated tokens read the frozen
 // artifact KV plus the online KV through the adapted query) and, as a
-// second kernel for any S, the same attention as attn_tc.cu;
-// K4: the log-sum-exp merge of split-KV partial results.
+// second kernel for any S, the same attention as attn_tc.cu, with K4, the
+// log-sum-exp merge of its split-KV chunks, done by the last CTA of each row
+// tile to finish; and APE's calibrated combination of two partial results.
 //
 // K3 is bound by HBM: every (request, KV head) streams its assembled K/V
 // once (4 KiB per token at Hkv = 8, d = 128).  One CTA owns 16 packed query
@@ -37,7 +38,6 @@ template <int D, bool kLayout>
 __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ AttnParams p) {
   using L = MmaLayout<D>;
   grid_dep_wait();     // Q and the suffix K/V may come from the previous kernel
-  grid_dep_launch();   // the combine kernel may be scheduled as CTAs finish
   constexpr int NT = D / 8;           // n8 tiles of the output
   constexpr int KS = D / 16;          // k16 steps of QK^T
   extern __shared__ uint8_t smem_raw[];
@@ -309,7 +309,8 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
   const float lse = (wsum > 0.f) ? (Mu + log2f(wsum)) * 0.69314718055994531f : -INFINITY;
   const int pr = row0 + row;
   const int tok = pr / G;
-  if (tok >= p.S) return;
+  const bool row_ok = tok < p.S;
+  const long long orow = ((long long)req * p.S + (row_ok ? tok : 0)) * p.Hq + kvh * G + pr % G;
   float acc[CPT];
 #pragma unroll
   for (int c = 0; c < CPT; ++c) {
@@ -318,20 +319,62 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
     for (int w = 0; w < 4; ++w) a += wt[w] * mb[(w * 16 + row) * (D + 2) + c0 + c];
     acc[c] = a * inv;
   }
-  if (nsplit > 1) {
-    float* po = p.part_o + ((long long)cta * kMmaRows + row) * D + c0;
-#pragma unroll
-    for (int c = 0; c < CPT; c += 4) *reinterpret_cast<float4*>(po + c) = make_float4(acc[c], acc[c + 1], acc[c + 2], acc[c + 3]);
-    if ((tid & 7) == 0) p.part_lse[(long long)cta * kMmaRows + row] = lse;
-  } else {
-    const long long orow = ((long long)req * p.S + tok) * p.Hq + kvh * G + pr % G;
+  if (nsplit <= 1) {
+    if (!row_ok) return;
     uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D + c0);
 #pragma unroll
     for (int c = 0; c < CPT; c += 8)
       dst[c / 8] = make_uint4(pack_bf16(acc[c], acc[c + 1]), pack_bf16(acc[c + 2], acc[c + 3]),
                               pack_bf16(acc[c + 4], acc[c + 5]), pack_bf16(acc[c + 6], acc[c + 7]));
     if ((tid & 7) == 0 && p.lse_out) p.lse_out[orow] = lse;
+    return;
   }
+  // Split-KV chunks (K4): publish this chunk's normalised O and log-sum-exp;
+  // the last CTA of the (request, KV head, row tile) to arrive merges every
+  // chunk, its own included, in split order (the same arithmetic whichever
+  // CTA is last):  lse = log sum_s exp(lse_s),  O = sum_s exp(lse_s - lse) O_s.
+  // Every consumer thread passes the two barriers, rows past the last token too.
+  float* po = p.part_o + ((long long)cta * kMmaRows + row) * D + c0;
+#pragma unroll
+  for (int c = 0; c < CPT; c += 4) *reinterpret_cast<float4*>(po + c) = make_float4(acc[c], acc[c + 1], acc[c + 2], acc[c + 3]);
+  if ((tid & 7) == 0) p.part_lse[(long long)cta * kMmaRows + row] = lse;
+  __threadfence();
+  volatile int* last_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 8 * (2 * L::NS + 1) + 4);
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+  if (tid == 0) {
+    const int unit = (req * p.Hkv + kvh) * p.work.row_tiles + rt;
+    *last_flag = (atomicAdd(&p.unit_cnt[unit], 1) == nsplit - 1) ? 1 : 0;
+  }
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+  if (*last_flag == 0 || !row_ok) return;
+  __threadfence();
+  const long long c_0 = p.work.base[req] + (long long)kvh * p.work.row_tiles + rt;   // CTA of split 0
+  const long long c_stride = (long long)p.Hkv * p.work.row_tiles;
+  float Ms = -INFINITY;
+  for (int sp = 0; sp < nsplit; ++sp) Ms = fmaxf(Ms, __ldcg(p.part_lse + (c_0 + sp * c_stride) * kMmaRows + row));
+  float W = 0.f;
+#pragma unroll
+  for (int c = 0; c < CPT; ++c) acc[c] = 0.f;
+  for (int sp = 0; sp < nsplit; ++sp) {
+    const long long cs = c_0 + sp * c_stride;
+    const float ls = __ldcg(p.part_lse + cs * kMmaRows + row);
+    if (ls == -INFINITY) continue;
+    const float w = __expf(ls - Ms);
+    W += w;
+    const float* q = p.part_o + (cs * kMmaRows + row) * D + c0;
+#pragma unroll
+    for (int c = 0; c < CPT; c += 4) {
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(q + c));
+      acc[c] += w * v.x; acc[c + 1] += w * v.y; acc[c + 2] += w * v.z; acc[c + 3] += w * v.w;
+    }
+  }
+  const float invW = (W > 0.f) ? 1.f / W : 0.f;
+  uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D + c0);
+#pragma unroll
+  for (int c = 0; c < CPT; c += 8)
+    dst[c / 8] = make_uint4(pack_bf16(acc[c] * invW, acc[c + 1] * invW), pack_bf16(acc[c + 2] * invW, acc[c + 3] * invW),
+                            pack_bf16(acc[c + 4] * invW, acc[c + 5] * invW), pack_bf16(acc[c + 6] * invW, acc[c + 7] * invW));
+  if ((tid & 7) == 0 && p.lse_out) p.lse_out[orow] = (W > 0.f) ? Ms + logf(W) : -INFINITY;
 }
 
 template <int D, bool kLayout>
@@ -347,63 +390,6 @@ cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st) {
   if (D == 128) return layout ? launch_attn_mma_t<128, true>(p, st) : launch_attn_mma_t<128, false>(p, st);
   if (D == 64) return layout ? launch_attn_mma_t<64, true>(p, st) : launch_attn_mma_t<64, false>(p, st);
   return cudaErrorInvalidValue;
-}
-
-// ---------------------------------------------------------------------------
-// K4: merge split-KV partials: lse = log sum_s exp(lse_s),
-// O = sum_s exp(lse_s - lse) O_s.  One warp per output row.
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ CombineParams p,
-                                                      long long total_rows) {
-  grid_dep_wait();   // the partial results of the attention kernel just before
-  const long long gw = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (gw >= total_rows) return;
-  const int R = p.rows_per_tile;
-  const long long per_req = (long long)p.Hkv * p.work.row_tiles * R;
-  const int req = (int)(gw / per_req);
-  long long rem = gw % per_req;
-  const int r = (int)(rem % R);
-  rem /= R;
-  const int rt = (int)(rem % p.work.row_tiles);
-  const int kvh = (int)(rem / p.work.row_tiles);
-  const int ns = p.work.nsplit[req];
-  if (ns <= 1) return;
-  const int pr = rt * R + r;
-  const int tok = pr / p.G;
-  if (tok >= p.S) return;
-  float M = -INFINITY;
-  for (int s = 0; s < ns; ++s) {
-    const long long c = p.work.base[req] + ((long long)s * p.Hkv + kvh) * p.work.row_tiles + rt;
-    M = fmaxf(M, p.part_lse[c * R + r]);
-  }
-  float W = 0.f;
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  const int cpl = p.D / 32;   // columns per lane (2 or 4)
-  for (int s = 0; s < ns; ++s) {
-    const long long c = p.work.base[req] + ((long long)s * p.Hkv + kvh) * p.work.row_tiles + rt;
-    const float ls = p.part_lse[c * R + r];
-    if (ls == -INFINITY) continue;
-    const float w = __expf(ls - M);
-    W += w;
-    const float* po = p.part_o + (c * R + r) * p.D + lane * cpl;
-    if (cpl == 4) {
-      const float4 v = *reinterpret_cast<const float4*>(po);
-      acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
-    } else {
-      const float2 v = *reinterpret_cast<const float2*>(po);
-      acc.x += w * v.x; acc.y += w * v.y;
-    }
-  }
-  const float inv = (W > 0.f) ? 1.f / W : 0.f;
-  const long long orow = ((long long)req * p.S + tok) * p.Hq + kvh * p.G + pr % p.G;
-  __nv_bfloat16* dst = p.out + orow * p.D + lane * cpl;
-  if (cpl == 4) {
-    *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16(acc.x * inv, acc.y * inv), pack_bf16(acc.z * inv, acc.w * inv));
-  } else {
-    *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc.x * inv, acc.y * inv);
-  }
-  if (lane == 0 && p.lse_out) p.lse_out[orow] = (W > 0.f) ? M + logf(W) : -INFINITY;
 }
 
 // APE's calibrated combination of the context and online parts (see
@@ -442,13 +428,6 @@ cudaError_t launch_ape_combine(const ApeParams& p, cudaStream_t st) {
   const long long rows = (long long)p.n_req * p.S * p.Hq;
   if (rows == 0) return cudaSuccess;
   return launch_pdl(ape_combine_kernel, dim3((unsigned)((rows * 32 + 255) / 256)), dim3(256), 0, st, 0, p, rows);
-}
-
-cudaError_t launch_combine(const CombineParams& p, cudaStream_t st) {
-  const long long total_rows = (long long)p.work.n_req * p.Hkv * p.work.row_tiles * p.rows_per_tile;
-  const long long threads = total_rows * 32;
-  const int grid = (int)((threads + 255) / 256);
-  return launch_pdl(combine_kernel, dim3(grid), dim3(256), 0, st, 0, p, total_rows);
 }
 
 }  // namespace att

@@ -751,11 +751,12 @@ attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, co
   bool need_combine = false;   // split partial results in global memory
   for (int r = 0; r < plan->n_req; ++r) need_combine |= (w.nsplit[r] > 1);
   if (w.cluster > 0) need_combine = false;
-  // partial O and LSE of every split CTA; for the tcgen05 kernel also one
-  // arrival counter per (request, KV head, row tile), zeroed below
+  // partial O and LSE of every split CTA and one arrival counter per
+  // (request, KV head, row tile), zeroed below: the last CTA of a row tile
+  // to arrive merges its chunks, in either kernel
   const size_t pb = need_combine ? (size_t)w.n_cta * rows * (D + 1) * 4 : 0;
   const size_t units = (size_t)plan->n_req * Hkv * w.row_tiles;
-  const size_t part_bytes = pb + ((need_combine && tc) ? units * 4 : 0);
+  const size_t part_bytes = pb + (need_combine ? units * 4 : 0);
   if (fixed && part_bytes > fixed->cap)
     return fail(ATTUNER_ERR_INVALID_ARG,
                 "this call needs " + std::to_string(part_bytes) + " bytes of split-KV scratch, more than the fixed " +
@@ -810,29 +811,11 @@ attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, co
     }
     ap.part_o = static_cast<float*>(part);
     ap.part_lse = static_cast<float*>(part) + (size_t)w.n_cta * rows * D;
-    if (tc) {
-      ap.unit_cnt = reinterpret_cast<int*>(static_cast<char*>(part) + pb);
-      ce = cudaMemsetAsync(ap.unit_cnt, 0, units * 4, st);
-    }
+    ap.unit_cnt = reinterpret_cast<int*>(static_cast<char*>(part) + pb);
+    ce = cudaMemsetAsync(ap.unit_cnt, 0, units * 4, st);
   }
   if (ce == cudaSuccess) ce = tc ? launch_attn_tc(ap, D, st) : launch_attn_mma(ap, D, st);
   if (ce == cudaSuccess) ++launches;
-  if (ce == cudaSuccess && need_combine && !tc) {   // the tcgen05 kernel merges its splits itself
-    CombineParams cp{};
-    cp.work = w;
-    cp.part_o = ap.part_o;
-    cp.part_lse = ap.part_lse;
-    cp.out = ap.out;
-    cp.lse_out = lse_out;
-    cp.S = S;
-    cp.Hq = Hq;
-    cp.Hkv = Hkv;
-    cp.G = G;
-    cp.D = D;
-    cp.rows_per_tile = rows;
-    ce = launch_combine(cp, st);
-    if (ce == cudaSuccess) ++launches;
-  }
   if (part && !fixed) cudaFreeAsync(part, st);
   if (ce != cudaSuccess) return fail(ATTUNER_ERR_CUDA, std::string("attention launch failed: ") + cudaGetErrorString(ce));
   return ATTUNER_OK;

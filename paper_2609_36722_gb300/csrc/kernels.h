@@ -65,9 +65,9 @@ struct AttnParams {
   const __nv_bfloat16* q;        // (K3 reads Q directly)
   __nv_bfloat16* out;            // [n_req, S, Hq, D]
   float* lse_out;                // [n_req, S, Hq] or nullptr
-  float* part_o;                 // split chunks only: K3 [n_cta, 16, D]; K2 [n_cta, D, 256] (column-major)
+  float* part_o;                 // split chunks only: K3 [n_cta, 16, D]; K2 fp16 pieces (see attn_tc.cu)
   float* part_lse;               // [n_cta, rows_per_tile]
-  int* unit_cnt;                 // K2: arrivals per (request, KV head, row tile); zero on entry, left zero
+  int* unit_cnt;                 // arrivals per (request, KV head, row tile); zero on entry
   int32_t S, S_kv, Hq, Hkv, G;
   float scale_log2;              // log2(e) / (sqrt(D) * temperature), temperature 1 but for APE's context part
   int* status;
@@ -81,14 +81,6 @@ struct AttnParams {
   int32_t kv_part;               // slots read: 0 all, 1 the plan's (artifacts), 2 the final online span
 };
 
-struct CombineParams {
-  WorkTable work;
-  const float* part_o;
-  const float* part_lse;
-  __nv_bfloat16* out;
-  float* lse_out;
-  int32_t S, Hq, Hkv, G, D, rows_per_tile;
-};
 
 // Pool repack: caller K/V [L, Hkv, D] -> pool blocks [first + p/64][h][p%64][:]
 // Batched pool write from host memory: artifact i copies [L[i], Hkv, D] K/V
@@ -176,6 +168,5 @@ cudaError_t launch_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, size_t sm
 int attn_tc_max_clusters(int D, int ns);
 cudaError_t launch_attn_tc(const AttnParams& p, int D, cudaStream_t st);
 cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st);
-cudaError_t launch_combine(const CombineParams& p, cudaStream_t st);
 
 }  // namespace att

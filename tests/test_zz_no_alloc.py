@@ -43,15 +43,16 @@ def test_static_scratch_matches_attend_twice(kernel, split, S, S_kv):
     q = ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=S_kv)
     ref_o, ref_l = ctx.attend(plan, q, wl.suffix_k, wl.suffix_v)
     assert ctx.sync_status() == 0
+    # the KV must split so that the partial results go through the scratch:
+    # chunks of `split` blocks for the tcgen05 kernel, of at least 16 blocks
+    # (the decode chunk at this size) for the warp-MMA kernel; either kernel
+    # merges its chunks itself (one launch)
+    n_blocks = [sum(-(-wl.art_lengths[a] // 64) for a in req) + -(-S_kv // 64) for req in wl.requests]
     if kernel == 1:
-        # chunks of `split` blocks: every request has more blocks than that, so
-        # the KV splits and the partial results go through the scratch; the
-        # tcgen05 kernel merges its splits itself (one launch)
-        n_blocks = [sum(-(-wl.art_lengths[a] // 64) for a in req) + -(-S_kv // 64) for req in wl.requests]
         assert min(n_blocks) > split
-        launches = 1
     else:
-        launches = 2   # warp-MMA kernel + combine kernel: the layout must split the KV
+        assert max(n_blocks) > 16
+    launches = 1
     assert ctx.last_launch_count() == launches
     for _ in range(2):
         out, lse = ctx.attend_static_scratch(plan, q, wl.suffix_k, wl.suffix_v)
