@@ -331,9 +331,15 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
  *   ATTUNER_OPT_SPLIT_BLOCKS    KV blocks per split-KV chunk (0 = automatic)
  *   ATTUNER_OPT_WAIT_LIMIT      clock cycles a device wait may spin before it
  *                               gives up and sets TIMEOUT (0 = about 2 s)
- *   ATTUNER_OPT_QPROJ_SPLIT_K  most CTAs (1..4) that split the K dimension of one
- *                               Q-projection tile when the tiles alone leave SMs
- *                               idle (0 or 1 = no split, the default)
+ *   ATTUNER_OPT_QPROJ_SPLIT_K   CTAs (a thread-block cluster: 1, 2, 4 or 8) that
+ *                               split the K dimension of one projection tile
+ *                               (0 = chosen by the library's cost model)
+ *   ATTUNER_OPT_QPROJ_ROWS      query rows per projection CTA: 128 or 256
+ *                               (0 = chosen by the cost model).  A pair of these
+ *                               two options that no kernel shape supports for
+ *                               the context's head size and the call's LoRA
+ *                               rank makes the projection calls fail with
+ *                               INVALID_ARG
  *   ATTUNER_OPT_SPLIT_MERGE     how the tcgen05 kernel merges the split-KV
  *                               chunks of a row tile: 0 auto (cost model),
  *                               1 independent CTAs merged through global memory
@@ -350,6 +356,7 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
 #define ATTUNER_OPT_WAIT_LIMIT     3
 #define ATTUNER_OPT_QPROJ_SPLIT_K  4
 #define ATTUNER_OPT_SPLIT_MERGE    5
+#define ATTUNER_OPT_QPROJ_ROWS     7
 /* Debug check: while non-zero, attuner_q_project, attuner_kv_project,
  * attuner_attend, attuner_attend_static_scratch and attuner_query_attend
  * synchronise their stream before returning and return the device status as

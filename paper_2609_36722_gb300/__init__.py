@@ -17,6 +17,7 @@ from .attuner import (  # noqa: F401
     OPT_QPROJ_SPLIT_K,
     OPT_SPLIT_MERGE,
     OPT_SYNC_CHECK,
+    OPT_QPROJ_ROWS,
     OPT_TEST_STUCK_WAIT,
     lib,
     load_library,

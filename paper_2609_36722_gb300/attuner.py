@@ -34,6 +34,7 @@ OPT_WAIT_LIMIT = 3
 OPT_QPROJ_SPLIT_K = 4
 OPT_SPLIT_MERGE = 5
 OPT_SYNC_CHECK = 6
+OPT_QPROJ_ROWS = 7
 OPT_TEST_STUCK_WAIT = 1000
 
 BLOCK_TOKENS = 64

@@ -20,7 +20,8 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libattuner.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
-SOURCES = ["capi.cu", "plan.cpp", "prep.cu", "qproj.cu", "attn_tc.cu", "attn_mma.cu", "attend_static.cu"]
+SOURCES = ["capi.cu", "plan.cpp", "prep.cu", "qproj.cu", "qproj_mr2.cu", "qproj_d64.cu", "attn_tc.cu", "attn_mma.cu",
+           "attend_static.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE]
 

@@ -513,26 +513,41 @@ attuner_status att::check_common(attuner_ctx* ctx, const attuner_plan* plan, int
   return ATTUNER_OK;
 }
 
-// Split K of the Q projection over up to ATTUNER_OPT_QPROJ_SPLIT_K CTAs per
-// (row tile, head) when those tiles alone would leave SMs idle.  Off by
-// default: on GB300 the partial-sum traffic costs more than the extra SMs
-// bring for the Qwen3-4B and decode shapes.
-// CTAs per head of the projection kernel: when the tiles (grid heads x
-// 128-row blocks) cannot fill half the GPU, 2 or 4 CTAs share a head's
-// columns so that more SMs stream the weights (at least 32 columns each).
-static int qproj_parts(const attuner_ctx* ctx, int heads, int M) {
-  const long long tiles = (long long)heads * ((M + 127) / 128);
-  int parts = 1;
-  while (parts < 4 && 2 * parts * 32 <= ctx->cfg.head_dim && tiles * 2 * parts <= ctx->num_sms) parts *= 2;
-  return parts;
-}
-
-static int qproj_ksplit(const attuner_ctx* ctx, int M) {
-  const int tiles = ctx->cfg.n_q_heads * ((M + 127) / 128);
-  const int nk = ctx->cfg.hidden / 64;
-  int ks = 1;
-  while (ks < ctx->opt_qproj_split && (long long)tiles * (ks + 1) <= ctx->num_sms && nk / (ks + 1) >= 2) ++ks;
-  return ks;
+// Launch shape of the projection kernel: rows per CTA (mr x 128: one or two
+// TMEM accumulators sharing each W tile) and K slices per tile (ks CTAs of a
+// cluster exchanging fp32 partials through distributed shared memory).  The
+// estimate is waves x (start-up + operand bytes + epilogue), with constants
+// from per-CTA timelines on GB300: about 2.5 us from launch to the first full
+// stage; the operand stream, (mr*128 + D + r) * hidden/ks * 2 bytes per CTA
+// (out-of-range rows of a tile are filled, not skipped), at about 100 GB/s per
+// SM; an epilogue of about 3.5 us, plus 1.5 us and the exchanged partial rows
+// at about 20 GB/s when the K dimension is split.  ATTUNER_OPT_QPROJ_SPLIT_K
+// and ATTUNER_OPT_QPROJ_ROWS pin either choice.  {0, 0} when the options leave
+// no supported shape.
+struct QpShape {
+  int mr, ks;
+};
+static QpShape qproj_shape(const attuner_ctx* ctx, int heads, int M, int n_lora) {
+  const int D = ctx->cfg.head_dim, nk = ctx->cfg.hidden / 64;
+  QpShape best{0, 0};
+  double best_t = 0.0;
+  for (int mr = 1; mr <= 2; ++mr)
+    for (int ks = 1; ks <= 8; ks *= 2) {
+      if (ctx->opt_qproj_rows != 0 && ctx->opt_qproj_rows != 128 * mr) continue;
+      if (ctx->opt_qproj_split != 0 && ctx->opt_qproj_split != ks) continue;
+      if (ks > nk || !qproj_shape_supported(D, mr, ks, n_lora)) continue;
+      const long long tiles = (long long)heads * ((M + 128 * mr - 1) / (128 * mr));
+      const long long waves = (tiles * ks + ctx->num_sms - 1) / ctx->num_sms;
+      const double bytes = (double)(128 * mr + D + n_lora) * (double)(ctx->cfg.hidden / ks) * 2.0;
+      const double exch = (double)std::min(128 * mr, M) * (D + n_lora) * 4.0;
+      const double epi = ks > 1 ? 5.0e-6 + exch / 20e9 : 3.5e-6;
+      const double t = (double)waves * (2.5e-6 + bytes / 100e9 + epi);
+      if (best.mr == 0 || t < best_t) {
+        best = {mr, ks};
+        best_t = t;
+      }
+    }
+  return best;
 }
 
 static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan, const void* x, const void* w_q,
@@ -549,22 +564,16 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
   const int M = plan->n_req * S;
   const int D = c.head_dim, Hq = c.n_q_heads, dq = Hq * D;
   const int n_lora = lora ? ((r + 15) / 16) * 16 : 0;
-  const int ksplit = qproj_ksplit(ctx, M);
-  const int tiles = Hq * ((M + 127) / 128);
+  const QpShape shape = qproj_shape(ctx, Hq, M, n_lora);
+  CHECK_ARG(shape.mr != 0, "ATTUNER_OPT_QPROJ_SPLIT_K / ATTUNER_OPT_QPROJ_ROWS leave no supported "
+                           "projection shape for this head size, LoRA rank and hidden size");
   const size_t off_rope = sc.take((size_t)M * (D / 2) * 8);
-  size_t off_part = 0, off_cnt = 0;
-  if (ksplit > 1) {
-    off_part = sc.take((size_t)tiles * ksplit * 128 * (D + n_lora) * 4);
-    off_cnt = sc.take((size_t)tiles * 4);
-  }
   char* base = static_cast<char*>(sc.base);
   float2* rope = reinterpret_cast<float2*>(base + off_rope);
 
   PrepParams pp{};
   pp.rope = rope;
   pp.plan = plan_dev(plan);
-  pp.counters = ksplit > 1 ? reinterpret_cast<int32_t*>(base + off_cnt) : nullptr;
-  pp.n_counters = ksplit > 1 ? tiles : 0;
   pp.M = M;
   pp.D = D;
   pp.S = S;
@@ -581,11 +590,10 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
     const uint32_t box[2] = {64, 128};
     if ((e = make_map(&qp.tm_x, x, 2, dims, strides, box, "x")) != ATTUNER_OK) return e;
   }
-  const int parts = ksplit > 1 ? 1 : qproj_parts(ctx, Hq, M);
   {
     const uint64_t dims[2] = {(uint64_t)c.hidden, (uint64_t)dq};
     const uint64_t strides[1] = {(uint64_t)c.hidden * 2};
-    const uint32_t box[2] = {64, (uint32_t)(D / 2 / parts)};
+    const uint32_t box[2] = {64, (uint32_t)D};
     if ((e = make_map(&qp.tm_w, w_q, 2, dims, strides, box, "w_q")) != ATTUNER_OK) return e;
   }
   if (lora) {
@@ -595,14 +603,12 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
     if ((e = make_map(&qp.tm_a, lora_a, 2, dims, strides, box, "lora_a")) != ATTUNER_OK) return e;
     const uint64_t bdims[2] = {(uint64_t)r, (uint64_t)dq};
     const uint64_t bstrides[1] = {(uint64_t)r * 2};
-    const uint32_t bbox[2] = {8, (uint32_t)(D / 2 / parts)};
+    const uint32_t bbox[2] = {8, (uint32_t)D};
     if ((e = make_map(&qp.tm_b, lora_b, 2, bdims, bstrides, bbox, "lora_b", 0)) != ATTUNER_OK) return e;
   }
   qp.q_out = static_cast<__nv_bfloat16*>(q_out);
   qp.qnorm_w = static_cast<const __nv_bfloat16*>(q_norm_w);
   qp.rope = rope;
-  qp.part = ksplit > 1 ? reinterpret_cast<float*>(base + off_part) : nullptr;
-  qp.counters = pp.counters;
   qp.M = M;
   qp.hidden = c.hidden;
   qp.Hq = Hq;
@@ -612,13 +618,11 @@ static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan,
   qp.S_out = S;
   qp.r = lora ? r : 0;
   qp.n_lora = n_lora;
-  qp.ksplit = ksplit;
-  qp.parts = parts;
   qp.s = s;
   qp.eps = c.rms_eps;
   qp.status = ctx->d_status;
   qp.wait_limit = ctx->wait_limit;
-  CUDA_TRY(launch_qproj(qp, D, st));
+  CUDA_TRY(launch_qproj(qp, D, shape.mr, shape.ks, st));
   ++launches;
   return ATTUNER_OK;
 }
@@ -661,11 +665,13 @@ static attuner_status kv_project_impl(attuner_ctx* ctx, const attuner_plan* plan
     const uint32_t box[2] = {64, 128};
     if ((e = make_map(&qp.tm_x, x, 2, dims, strides, box, "x")) != ATTUNER_OK) return e;
   }
-  const int parts = qproj_parts(ctx, 2 * Hkv, M);
+  const QpShape shape = qproj_shape(ctx, 2 * Hkv, M, 0);
+  CHECK_ARG(shape.mr != 0, "ATTUNER_OPT_QPROJ_SPLIT_K / ATTUNER_OPT_QPROJ_ROWS leave no supported "
+                           "projection shape for this head size and hidden size");
   {
     const uint64_t dims[2] = {(uint64_t)c.hidden, (uint64_t)dkv};
     const uint64_t strides[1] = {(uint64_t)c.hidden * 2};
-    const uint32_t box[2] = {64, (uint32_t)(D / 2 / parts)};
+    const uint32_t box[2] = {64, (uint32_t)D};
     if ((e = make_map(&qp.tm_w, w_k, 2, dims, strides, box, "w_k")) != ATTUNER_OK) return e;
     if ((e = make_map(&qp.tm_w2, w_v, 2, dims, strides, box, "w_v")) != ATTUNER_OK) return e;
   }
@@ -682,25 +688,19 @@ static attuner_status kv_project_impl(attuner_ctx* ctx, const attuner_plan* plan
   qp.S_out = S_kv;
   qp.r = 0;
   qp.n_lora = 0;
-  qp.ksplit = 1;
-  qp.parts = parts;
   qp.s = 0.f;
   qp.eps = c.rms_eps;
   qp.status = ctx->d_status;
   qp.wait_limit = ctx->wait_limit;
-  CUDA_TRY(launch_qproj(qp, D, st));
+  CUDA_TRY(launch_qproj(qp, D, shape.mr, shape.ks, st));
   ++launches;
   return ATTUNER_OK;
 }
 
 static size_t q_project_scratch(const attuner_ctx* ctx, int M) {
-  const int D = ctx->cfg.head_dim, Hq = ctx->cfg.n_q_heads;
+  const int D = ctx->cfg.head_dim;
   auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
-  const int ksplit = qproj_ksplit(ctx, M);
-  const size_t tiles = (size_t)Hq * ((M + 127) / 128);
-  size_t bytes = al((size_t)M * (D / 2) * 8);
-  if (ksplit > 1) bytes += al(tiles * ksplit * 128 * (D + 64) * 4) + al(tiles * 4);
-  return bytes;
+  return al((size_t)M * (D / 2) * 8);
 }
 
 // ---------------------------------------------------------------------------
@@ -1003,8 +1003,13 @@ extern "C" attuner_status attuner_set_option(attuner_ctx* ctx, int32_t option, i
       ctx->wait_limit = value ? value : (1ll << 32);
       return ATTUNER_OK;
     case ATTUNER_OPT_QPROJ_SPLIT_K:
-      CHECK_ARG(value >= 0 && value <= 4, "Q-projection split-K must be in [0, 4]");
-      ctx->opt_qproj_split = value ? (int)value : 1;
+      CHECK_ARG(value == 0 || value == 1 || value == 2 || value == 4 || value == 8,
+                "Q-projection split-K must be 0, 1, 2, 4 or 8");
+      ctx->opt_qproj_split = (int)value;
+      return ATTUNER_OK;
+    case ATTUNER_OPT_QPROJ_ROWS:
+      CHECK_ARG(value == 0 || value == 128 || value == 256, "Q-projection rows per CTA must be 0, 128 or 256");
+      ctx->opt_qproj_rows = (int)value;
       return ATTUNER_OK;
     case ATTUNER_OPT_SPLIT_MERGE:
       CHECK_ARG(value >= 0 && value <= 2, "split merge must be 0, 1 or 2");

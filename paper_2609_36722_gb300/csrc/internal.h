@@ -38,7 +38,8 @@ struct attuner_ctx {
   int num_sms = 0;
   int opt_prefill = 0;
   int opt_split = 0;
-  int opt_qproj_split = 1;
+  int opt_qproj_split = 0;   // 0: the projection's shape from its cost model
+  int opt_qproj_rows = 0;
   int opt_merge = 0;
   int opt_sync_check = 0;
   int tc_clusters[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};   // co-resident clusters of n tcgen05 CTAs

@@ -11,35 +11,29 @@
 
 namespace att {
 
-// K1: the RoPE cos/sin table of every query row; also clears the split-K
-// counters of K1b for this call.
+// K1: the RoPE cos/sin table of every query row.
 struct PrepParams {
   float2* rope;                  // [D/2, M] (cos, sin), pair-major
   PlanDev plan;                  // assembled positions of the online rows
-  int32_t* counters;             // [n_counters] split-K arrival counters, or nullptr
-  int32_t n_counters;
   int32_t M, D, S, S_kv;
   double inv_freq[64];           // theta^(-2j/D), j < D/2 (computed on the host in double)
 };
 
 // K1b: Q = RoPE(RMSNorm(x W_q^T + s * bf16(x A^T) B^T) * w) as one tcgen05
 // GEMM (A stacked under W_q: one MMA of N = D + r) with a fused epilogue.
+// A CTA covers mr x 128 rows of one head and 1/ks of the K dimension (a
+// cluster of ks CTAs per tile; see qproj.cu).
 struct QprojParams {
   CUtensorMap tm_x;    // x [M, hidden], box 64 x 128, SW128
-  CUtensorMap tm_w;    // W_q [d_q, hidden], box 64 x D/2parts, SW128
+  CUtensorMap tm_w;    // W_q [d_q, hidden], box 64 x D, SW128
   CUtensorMap tm_a;    // A [r, hidden], box 64 x n_lora, SW128 (rows past r read as zeros)
-  CUtensorMap tm_b;    // B [d_q, r], box 8 x D/2parts, no swizzle (columns past r read as zeros)
-  CUtensorMap tm_w2;   // K/V mode: W_v [Hkv*D, hidden], box 64 x D/2parts, SW128
+  CUtensorMap tm_b;    // B [d_q, r], box 8 x D, no swizzle (columns past r read as zeros)
+  CUtensorMap tm_w2;   // K/V mode: W_v [Hkv*D, hidden], box 64 x D, SW128
   __nv_bfloat16* q_out;            // Q mode: [M, Hq, D]; K/V mode: suffix K [n_req, S_kv, Hkv, D]
   __nv_bfloat16* out2;             // K/V mode: suffix V [n_req, S_kv, Hkv, D]
   const __nv_bfloat16* qnorm_w;    // [D] (q_norm, or k_norm in K/V mode)
   const float2* rope;              // [D/2, M] (cos, sin), pair-major
-  float* part;                     // split-K partials [tiles][ksplit][128][D + n_lora]
-  int32_t* counters;               // [tiles] arrivals per output tile (zero on entry)
-  int32_t M, hidden, Hq, r, n_lora, ksplit;   // Hq: heads of the grid (2 Hkv in K/V mode)
-  // CTAs per head (1, 2 or 4; a cluster): each computes D/parts of the head's
-  // columns, two halves of D/2parts (tm_w, tm_w2 and tm_b boxes of D/2parts rows)
-  int32_t parts;
+  int32_t M, hidden, Hq, r, n_lora;   // Hq: heads of the grid (2 Hkv in K/V mode)
   // K/V mode (kv = 1): grid heads [0, Hout) project K (W = tm_w, key norm and
   // RoPE), [Hout, 2 Hout) project V (W = tm_w2, stored as is).  Row m of the
   // GEMM is token m % S of request m / S, written to output token row
@@ -135,7 +129,11 @@ cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __
                               __nv_bfloat16* vpool, int L, int Hkv, int D, int first_block,
                               cudaStream_t st);
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st);
-cudaError_t launch_qproj(const QprojParams& p, int D, cudaStream_t st);
+// Row tiles per CTA (mr = 1 or 2 accumulators of 128 rows) and K slices per
+// tile (ks = 1, 2, 4 or 8 CTAs, a cluster): shapes the kernel supports for a
+// head size and LoRA rank (rounded up to 16).
+bool qproj_shape_supported(int D, int mr, int ks, int n_lora);
+cudaError_t launch_qproj(const QprojParams& p, int D, int mr, int ks, cudaStream_t st);
 // Launch with programmatic stream serialization (the kernel may start while
 // the previous kernel of the stream finishes; see grid_dep_wait) and, when
 // cluster > 0, thread-block clusters of that many CTAs along x.

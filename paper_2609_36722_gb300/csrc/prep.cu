@@ -115,13 +115,11 @@ cudaError_t launch_pool_write_host(const HostBatch& b, __nv_bfloat16* kpool, __n
 // One thread per (query row, rotary pair): the RoPE angle pos * theta^(-2j/D)
 // with pos = T_art(req) + (S_kv - S) + i (App. A.5: positions of the
 // assembled context), formed and reduced modulo 2*pi in double, then sin/cos
-// in float on |angle| <= pi.  The first threads also clear the split-K
-// arrival counters the Q-projection kernel uses in this call.
+// in float on |angle| <= pi.
 __global__ void __launch_bounds__(256) prep_kernel(const __grid_constant__ PrepParams p) {
   grid_dep_wait();     // the scratch it writes may be memory the previous kernel used
   grid_dep_launch();   // the Q projection may start its main loop now
   const long long idx = (long long)blockIdx.x * 256 + threadIdx.x;
-  if (p.counters != nullptr && idx < p.n_counters) p.counters[idx] = 0;
   const int half = p.D / 2;
   if (idx >= (long long)p.M * half) return;
   const int j = (int)(idx / p.M), m = (int)(idx % p.M);   // pair-major: coalesced in the epilogue
@@ -188,7 +186,7 @@ cudaError_t launch_rotate_keys(const RotateParams& p, cudaStream_t st) {
 }
 
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st) {
-  const long long n = std::max<long long>((long long)p.M * (p.D / 2), p.n_counters);
+  const long long n = (long long)p.M * (p.D / 2);
   return launch_pdl(prep_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, 0, p);
 }
 

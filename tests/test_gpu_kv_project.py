@@ -52,6 +52,29 @@ def test_kv_project_matches_oracle(geom, S, S_kv):
         assert torch.equal(sv[r, :S_kv - S].view(torch.int16), wl.suffix_v[r, :S_kv - S].view(torch.int16))
 
 
+@pytest.mark.parametrize("rows,split", [(128, 1), (256, 2), (128, 8), (256, 4)])
+def test_kv_project_shapes_match_oracle(rows, split):
+    # the projection kernel's shapes pinned (rows per CTA, K slices per tile)
+    import paper_2609_36722_gb300 as pkg
+    geom, S, S_kv = G128, 300, 310
+    wl = make_custom("kvs", geom, 71, [37, 700], [[1, 0], [0]], S, S_kv, device=DEV)
+    wk, wv, kn = make_kv_weights(geom, 71, device=DEV)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_QPROJ_ROWS, rows)
+    ctx.set_option(pkg.OPT_QPROJ_SPLIT_K, split)
+    sk = wl.suffix_k.clone()
+    sv = wl.suffix_v.clone()
+    ctx.kv_project(plan, wl.x, wk, wv, kn, sk, sv)
+    assert ctx.sync_status() == 0
+    new = slice(S_kv - S, S_kv)
+    for r in range(wl.n_req):
+        k_ref, v_ref = _oracle_kv(wl, wk, wv, kn, r)
+        dk = np.abs(f64(sk[r, new]) - k_ref).max()
+        dv = np.abs(f64(sv[r, new]) - v_ref).max()
+        assert dk <= Q_MAX_ABS and dv <= Q_MAX_ABS, (r, dk, dv)
+        assert torch.equal(sk[r, :S_kv - S].view(torch.int16), wl.suffix_k[r, :S_kv - S].view(torch.int16))
+
+
 def test_decode_appends_one_token_per_step():
     # one request decoding three tokens into a buffer with room for 132 rows:
     # the prefix of S_kv rows is the call's contiguous [1, S_kv, Hkv, d] view,

@@ -191,15 +191,69 @@ def test_most_requests_per_call(kernel, S, S_kv):
         ctx.assemble(reqs + [[0]])
 
 
-@pytest.mark.parametrize("split_k", [2, 4])
-def test_q_project_split_k_matches_oracle(split_k):
+G64P = Geometry(hidden=512, n_q_heads=4, n_kv_heads=2, head_dim=64, rank=8)
+
+
+def _q_shape_case(geom, rank, rows, split, seed=13):
+    """Q projection with the kernel shape pinned (rows per CTA, K slices per
+    tile): two requests of 150 suffix tokens (M = 300: row tiles of 128 end
+    in a ragged 44-row tile, of 256 in a tile whose second accumulator holds
+    no row), against the oracle row by row."""
     import paper_2609_36722_gb300 as pkg
-    wl = make_custom("qsplit", G128, 13, [100], [[0]], 40, 40, device=DEV)
+    g = Geometry(hidden=geom.hidden, n_q_heads=geom.n_q_heads, n_kv_heads=geom.n_kv_heads,
+                 head_dim=geom.head_dim, rank=rank)
+    wl = make_custom("qshape", g, seed, [100, 37], [[0], [1, 0]], 150, 150, device=DEV)
     ctx, plan = load_context(wl)
-    ctx.set_option(pkg.OPT_QPROJ_SPLIT_K, split_k)
-    g = wl.geom
+    ctx.set_option(pkg.OPT_QPROJ_ROWS, rows)
+    ctx.set_option(pkg.OPT_QPROJ_SPLIT_K, split)
     q = ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv)
     assert ctx.sync_status() == 0
-    q_ref = oracle.workload_reference(wl, 0, q_only=True)
-    err = np.abs(_np(q[0]) - q_ref)
-    assert err.max() <= Q_MAX_ABS, err.max()
+    for r in range(wl.n_req):
+        q_ref = oracle.workload_reference(wl, r, q_only=True)
+        err = np.abs(_np(q[r]) - q_ref)
+        assert err.max() <= Q_MAX_ABS, (rows, split, r, err.max())
+    return ctx, plan, wl, q
+
+
+@pytest.mark.parametrize("rows", [128, 256])
+@pytest.mark.parametrize("split", [1, 2, 4, 8])
+def test_q_project_shapes_match_oracle(rows, split):
+    _q_shape_case(G128, 16, rows, split)
+
+
+@pytest.mark.parametrize("rows,split", [(128, 1), (128, 4), (256, 1), (128, 8)])
+def test_q_project_shapes_rank64(rows, split):
+    # LoRA rank 64: the widest partial rows (D + 64 columns) the exchange carries
+    # (256-row tiles with a K split do not fit this width in shared memory)
+    _q_shape_case(G128, 64, rows, split, seed=17)
+
+
+@pytest.mark.parametrize("rows,split", [(128, 1), (128, 2), (128, 4), (256, 1), (256, 2), (256, 8)])
+def test_q_project_shapes_head64(rows, split):
+    _q_shape_case(G64P, 8, rows, split, seed=19)
+
+
+def test_q_project_shapes_are_deterministic():
+    # the K slices are summed in slice order: two calls give the same bytes
+    ctx, plan, wl, q1 = _q_shape_case(G128, 16, 256, 4)
+    g = wl.geom
+    q2 = ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv)
+    assert ctx.sync_status() == 0
+    assert torch.equal(q1.view(torch.int16), q2.view(torch.int16))
+
+
+def test_q_project_unsupported_shape_refused():
+    # head size 64 with 8 K slices of 128-row tiles would leave 4 columns per
+    # thread: no kernel shape, so the call is refused before any launch
+    import paper_2609_36722_gb300 as pkg
+    wl = make_custom("qbad", G64P, 23, [40], [[0]], 16, 16, device=DEV)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_QPROJ_ROWS, 128)
+    ctx.set_option(pkg.OPT_QPROJ_SPLIT_K, 8)
+    g = wl.geom
+    with pytest.raises(pkg.AttunerError):
+        ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, S_kv=wl.S_kv)
+    with pytest.raises(pkg.AttunerError):
+        ctx.set_option(pkg.OPT_QPROJ_SPLIT_K, 3)
+    with pytest.raises(pkg.AttunerError):
+        ctx.set_option(pkg.OPT_QPROJ_ROWS, 64)
