@@ -61,13 +61,17 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
   const int nsplit = p.work.nsplit[req];
   const int boff = p.plan.blk_off[req];
   const int nab = p.plan.blk_off[req + 1] - boff;
-  const int o_rows = plan_o_rows(p.plan, req);           // online rows in the plan's spans
-  const int nsuf = (p.S_kv - o_rows + kBlockTokens - 1) / kBlockTokens;
+  const int nsuf = (p.S_kv + kBlockTokens - 1) / kBlockTokens;   // chunks of online rows
   const int row0 = rt * kMmaRows;
   const int last_row = min(row0 + kMmaRows - 1, p.S * G - 1);
-  const int last_vis = row_visibility(p.plan, req, (p.S_kv - p.S) + last_row / G, nab).slot;
+  const int lim_last = (p.S_kv - p.S) + last_row / G;   // online row of the tile's last query
+  // The row tile reads its own list of slots: the artifact slots its last
+  // query sees (queries are in prompt order, so no query of the tile sees
+  // more), then the online chunks up to the one holding that query's key.
+  const int nart = kLayout ? art_slots_seen(p.plan, req, lim_last, nab) : nab;
+  const int last_vis = nart + lim_last / kBlockTokens;
   int v_lo, v_hi;
-  kv_part_range(p.kv_part, nab, nsuf, v_lo, v_hi);
+  kv_part_range(p.kv_part, nart, nsuf, v_lo, v_hi);
   const int b0 = v_lo + split * p.work.chunk_blocks;
   const int b1 = min(min(b0 + p.work.chunk_blocks, v_hi), last_vis + 1);
   const int nblk = max(0, b1 - b0);
@@ -75,16 +79,14 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
   for (int i = threadIdx.x; i < nblk; i += blockDim.x) {
     const int b = b0 + i;
     int e;
-    if (b < nab) {
+    if (b < nart) {
       e = p.plan.blocks[boff + b];
-      const bool bad = e > 0 ? ((e >> 7) >= p.plan.pool_blocks || (e & 127) < 1 || (e & 127) > kBlockTokens)
-                             : (slot_rows(e) < 1 || slot_rows(e) > kBlockTokens || slot_row0(e) + slot_rows(e) > o_rows);
-      if (bad) {
+      if (e <= 0 || (e >> 7) >= p.plan.pool_blocks || (e & 127) < 1 || (e & 127) > kBlockTokens) {
         set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
         e = 0;
       }
     } else {
-      e = online_entry(o_rows + (b - nab) * kBlockTokens, kBlockTokens);
+      e = online_entry((b - nart) * kBlockTokens, kBlockTokens);
     }
     list[i] = e;
   }
@@ -164,12 +166,12 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
     }
   }
   // the thread's two query rows: online rows lim0 / lim1; with online spans
-  // before artifacts, also their own slots vs0 / vs1 (artifact slots after
-  // them are not visible)
+  // before artifacts, also the artifact slots they see, vs0 / vs1
+  // (chunk-relative)
   const int lim0 = (p.S_kv - p.S) + tok_r[0];
   const int lim1 = (p.S_kv - p.S) + tok_r[1];
-  const int vs0 = kLayout ? row_visibility(p.plan, req, (p.S_kv - p.S) + min(tok_r[0], p.S - 1), nab).slot - b0 : 0;
-  const int vs1 = kLayout ? row_visibility(p.plan, req, (p.S_kv - p.S) + min(tok_r[1], p.S - 1), nab).slot - b0 : 0;
+  const int vs0 = kLayout ? art_slots_seen(p.plan, req, (p.S_kv - p.S) + min(tok_r[0], p.S - 1), nab) - b0 : 0;
+  const int vs1 = kLayout ? art_slots_seen(p.plan, req, (p.S_kv - p.S) + min(tok_r[1], p.S - 1), nab) - b0 : 0;
 
   float o[NT][4];
 #pragma unroll
@@ -209,7 +211,7 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
         const int kb = 16 * warp + 8 * n + 2 * t + (c & 1);
         bool vis;
         if (e > 0) vis = kb < (e & 127) && (!kLayout || j < ((c < 2) ? vs0 : vs1));
-        else if (e < 0) vis = (slot_row0(e) + kb) <= ((c < 2) ? lim0 : lim1) && (!kLayout || kb < slot_rows(e));
+        else if (e < 0) vis = (slot_row0(e) + kb) <= ((c < 2) ? lim0 : lim1);
         else vis = false;
         if (!vis) s[n][c] = -INFINITY;
       }

@@ -133,7 +133,7 @@ __device__ __forceinline__ TcCta tc_cta(const AttnParams& p, int cta) {
     c.kvh = rem / p.work.row_tiles;
     int lo, hi;
     kv_part_range(p.kv_part, p.plan.blk_off[c.req + 1] - p.plan.blk_off[c.req],
-                  (p.S_kv - plan_o_rows(p.plan, c.req) + kBlockTokens - 1) / kBlockTokens, lo, hi);
+                  (p.S_kv + kBlockTokens - 1) / kBlockTokens, lo, hi);
     const int nv = hi - lo;
     c.chunk = (((nv + ns - 1) / ns) + 1) & ~1;
   } else {
@@ -539,13 +539,17 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
   const int req = cw.req, rt = cw.rt, kvh = cw.kvh;
   const int boff = p.plan.blk_off[req];
   const int nab = p.plan.blk_off[req + 1] - boff;
-  const int o_rows = plan_o_rows(p.plan, req);           // online rows in the plan's spans
-  const int nsuf = (p.S_kv - o_rows + kBlockTokens - 1) / kBlockTokens;
+  const int nsuf = (p.S_kv + kBlockTokens - 1) / kBlockTokens;   // chunks of online rows
   const int row0 = rt * kTcRows;
   const int last_row = min(row0 + kTcRows - 1, p.S * G - 1);
-  const int last_vis = row_visibility(p.plan, req, (p.S_kv - p.S) + last_row / G, nab).slot;
+  const int lim_last = (p.S_kv - p.S) + last_row / G;   // online row of the tile's last query
+  // The row tile reads its own list of slots: the artifact slots its last
+  // query sees (queries are in prompt order, so no query of the tile sees
+  // more), then the online chunks up to the one holding that query's key.
+  const int nart = kLayout ? art_slots_seen(p.plan, req, lim_last, nab) : nab;
+  const int last_vis = nart + lim_last / kBlockTokens;
   int v_lo, v_hi;
-  kv_part_range(p.kv_part, nab, nsuf, v_lo, v_hi);
+  kv_part_range(p.kv_part, nart, nsuf, v_lo, v_hi);
   const int b0 = v_lo + cw.split * cw.chunk;
   const int b1 = min(min(b0 + cw.chunk, v_hi), last_vis + 1);
   const int nblk = max(0, b1 - b0);
@@ -560,16 +564,14 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
     int e = 0;
     if (i < nblk) {
       const int b = b0 + i;
-      if (b < nab) {
+      if (b < nart) {
         e = p.plan.blocks[boff + b];
-        const bool bad = e > 0 ? ((e >> 7) >= p.plan.pool_blocks || (e & 127) < 1 || (e & 127) > kBlockTokens)
-                               : (slot_rows(e) < 1 || slot_rows(e) > kBlockTokens || slot_row0(e) + slot_rows(e) > o_rows);
-        if (bad) {
+        if (e <= 0 || (e >> 7) >= p.plan.pool_blocks || (e & 127) < 1 || (e & 127) > kBlockTokens) {
           set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
           e = 0;
         }
       } else {
-        e = online_entry(o_rows + (b - nab) * kBlockTokens, kBlockTokens);
+        e = online_entry((b - nart) * kBlockTokens, kBlockTokens);
       }
     }
     return e;
@@ -733,12 +735,12 @@ __global__ void __launch_bounds__(384, 1) attn_tc_kernel(const __grid_constant__
     const int tok = pr / G;
     // What this query (online row lim) sees: online keys up to its own online
     // row (online rows are in assembled order) and, with online spans before
-    // artifacts, only the artifact slots before its own slot vs (chunk-relative).
+    // artifacts, only the artifact slots before its span (vs, chunk-relative).
     const int lim = (p.S_kv - p.S) + tok;
-    const int vs = kLayout ? row_visibility(p.plan, req, lim, nab).slot - b0 : 0;
+    const int vs = kLayout ? art_slots_seen(p.plan, req, lim, nab) - b0 : 0;
     auto visible = [&](int s, int e) {
       if (e > 0) return (kLayout && s >= vs) ? 0 : (e & 127);
-      if (e < 0) return min(max(lim - slot_row0(e) + 1, 0), kLayout ? slot_rows(e) : kBlockTokens);
+      if (e < 0) return min(max(lim - slot_row0(e) + 1, 0), kBlockTokens);
       return 0;
     };
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;

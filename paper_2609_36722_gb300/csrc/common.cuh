@@ -18,19 +18,21 @@
 namespace att {
 
 // Plan arrays on the device.
-// A request's virtual block list ("slots", assembled order): artifact blocks
-// (entry > 0: pool_block << 7 | valid tokens) and chunks of at most 64 online
-// rows (entry < 0: -((online row0 << 7 | rows) + 1)); the plan holds the
-// artifact blocks and the chunks of the online spans that precede the last
-// artifact, and the kernels append the chunks of the final online span (the
-// suffix: online rows o_rows .. S_kv - 1).
+// A request's virtual block list ("slots"): its artifact blocks in prompt
+// order (entry > 0: pool_block << 7 | valid tokens), held by the plan, then
+// chunks of 64 online rows (entry < 0: -((online row0 << 7 | rows) + 1)),
+// appended by the kernels: every online row 0 .. S_kv - 1 of the request (the
+// explicit spans of a prompt layout, then the final span, the suffix).  An
+// online span between artifacts therefore takes no slot of its own: online
+// keys are visible by online row (online rows are in assembled order), and
+// artifact slots by the span a query sits in.
 struct PlanDev {
   const int32_t* blk_off;   // [n_req + 1] CSR offsets into blocks
   const int32_t* blocks;    // slot entries as above
   const int32_t* t_art;     // [n_req] artifact tokens
   const int32_t* o_rows;    // [n_req] online rows in the plan's explicit spans
   const int32_t* span_off;  // [n_req + 1] CSR offsets into spans
-  const int4* spans;        // explicit online spans: (online row0, rows, first slot, artifact tokens before)
+  const int4* spans;        // explicit online spans: (online row0, rows, artifact slots before, artifact tokens before)
   int32_t pool_blocks;      // capacity, for bounds checks
   int32_t has_spans;        // 0: no request has explicit online spans (o_rows all 0; no loads needed)
 };
@@ -38,29 +40,19 @@ struct PlanDev {
 ATT_DEV int plan_o_rows(const PlanDev& pl, int req) { return pl.has_spans ? pl.o_rows[req] : 0; }
 
 ATT_DEV int online_entry(int row0, int rows) { return -(((row0 << 7) | rows) + 1); }
-ATT_DEV int slot_rows(int e) { return e > 0 ? (e & 127) : (e < 0 ? ((-e - 1) & 127) : 0); }
 ATT_DEV int slot_row0(int e) { return (-e - 1) >> 7; }   // online slots only
 
-// Where online row t of request `req` sits: the slot holding its assembled
-// position (nab = the plan's slots of the request) and how many keys of that
-// slot it sees.  A query sees every slot before its own, fully.
-struct RowVis {
-  int slot, count;
-};
-ATT_DEV RowVis row_visibility(const PlanDev& pl, int req, int t, int nab) {
-  const int o = plan_o_rows(pl, req);
-  if (t >= o) {
-    const int u = t - o;
-    return {nab + u / kBlockTokens, u % kBlockTokens + 1};
-  }
+// Artifact slots that a query at online row t of request `req` sees: those
+// before its span in the prompt (all nab of them for rows of the final span).
+// It sees online rows 0 .. t, i.e. the keys of slots nab .. nab + t/64 up to
+// its own row.
+ATT_DEV int art_slots_seen(const PlanDev& pl, int req, int t, int nab) {
+  if (t >= plan_o_rows(pl, req)) return nab;
   for (int k = pl.span_off[req]; k < pl.span_off[req + 1]; ++k) {
     const int4 sp = pl.spans[k];
-    if (t < sp.x + sp.y) {
-      const int u = t - sp.x;
-      return {sp.z + u / kBlockTokens, u % kBlockTokens + 1};
-    }
+    if (t < sp.x + sp.y) return sp.z;
   }
-  return {0, 0};   // not reached for a valid plan
+  return 0;   // not reached for a valid plan
 }
 // assembled position of online row t (App. A.5 position ids)
 ATT_DEV int online_position(const PlanDev& pl, int req, int t) {

@@ -33,8 +33,6 @@ attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_
       if (a >= 0 && a < (long long)arts.size()) {
         nblk += arts[a].n_blocks;
         ++nids;
-      } else if (a < 0 && layout && -a < (1 << 22)) {
-        nblk += (-a + kBlockTokens - 1) / kBlockTokens;
       }
     }
     t.blocks.reserve(nblk);
@@ -51,10 +49,10 @@ attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_
     for (int i = offs[r]; i < offs[r + 1]; ++i) {
       const int a = items[i];
       if (a < 0 && layout) {
+        // an online span takes no slot: its rows are online rows o .. o + n - 1,
+        // read with every other online row after the artifact slots
         const long long n = -(long long)a;
         t.spans.insert(t.spans.end(), {(int32_t)o, (int32_t)n, (int32_t)t.blocks.size() - first_slot, (int32_t)tok});
-        for (long long c = 0; c < n; c += kBlockTokens)
-          t.blocks.push_back(-((int32_t)(((o + c) << 7) | std::min<long long>(kBlockTokens, n - c)) + 1));
         o += n;
         if (o >= (1 << 22)) return bad(ATTUNER_ERR_INVALID_ARG, err, "online rows of a request must be < 2^22");
         continue;
@@ -136,12 +134,11 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
   const int G = pol.n_q_heads / pol.n_kv_heads, Hkv = pol.n_kv_heads;
   const int rows = tc ? kTcRows : kMmaRows;
   const int row_tiles = (S * G + rows - 1) / rows;
-  // slots of request r the launch reads: the plan's, then the chunks of its
-  // final online span (or one of the two, kv_part)
+  // slots of request r the launch reads: the plan's artifact slots, then the
+  // 64-row chunks of its online rows (or one of the two, kv_part)
   auto nslots = [&](int r) {
     int lo, hi;
-    kv_part_range(pol.kv_part, t.blk_off[r + 1] - t.blk_off[r],
-                  (S_kv - t.o_rows[r] + kBlockTokens - 1) / kBlockTokens, lo, hi);
+    kv_part_range(pol.kv_part, t.blk_off[r + 1] - t.blk_off[r], (S_kv + kBlockTokens - 1) / kBlockTokens, lo, hi);
     return hi - lo;
   };
   long long total = 0;

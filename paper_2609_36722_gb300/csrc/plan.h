@@ -71,13 +71,15 @@ struct PlanTables {
   std::vector<int32_t> art_ids;       // artifact ids in prompt order
   std::vector<Artifact> art_used;     // their registry entries (the plan's own copy)
   std::vector<int32_t> blk_off;       // CSR over blocks
-  // slot entries in prompt order: artifact block (pool_block << 7 | valid) > 0,
-  // online chunk -((online_row0 << 7 | rows) + 1) < 0 (at most 64 rows)
+  // artifact slots in prompt order: pool_block << 7 | valid tokens (> 0).
+  // Online spans take no slot: a launch reads every online row of a request
+  // (explicit spans and the final span, in online-row order) as 64-row chunks
+  // after the artifact slots.
   std::vector<int32_t> blocks;
   std::vector<int32_t> t_art;         // artifact tokens of each request
   std::vector<int32_t> o_rows;        // online rows of each request's explicit spans
   std::vector<int32_t> span_off;      // CSR over spans
-  std::vector<int32_t> spans;         // 4 per span: online row0, rows, first slot, artifact tokens before
+  std::vector<int32_t> spans;         // 4 per span: online row0, rows, artifact slots before, artifact tokens before
   int32_t max_o_rows = 0;
 };
 
@@ -101,13 +103,13 @@ struct SplitPolicy {
   int32_t opt_merge;          // 0 = chosen here, 1 = through global memory, 2 = cluster
   int32_t tc_clusters[9];     // co-resident clusters of n tcgen05 CTAs (n = 2, 4)
   // which slots of each request the launch reads: 0 every slot, 1 the plan's
-  // slots only (the artifacts of a plan without online spans), 2 the chunks
-  // of the final online span only (the suffix)
+  // artifact slots only, 2 the chunks of the online rows only (for a plan
+  // without online spans: the suffix)
   int32_t kv_part = 0;
 };
 
-// The slots [lo, hi) of a request that a launch reads, out of its nab plan
-// slots and nsuf chunks of the final online span (kv_part as in SplitPolicy).
+// The slots [lo, hi) of a request that a launch reads, out of its nab artifact
+// slots and nsuf chunks of online rows (kv_part as in SplitPolicy).
 ATT_HD void kv_part_range(int kv_part, int nab, int nsuf, int& lo, int& hi) {
   lo = (kv_part == 2) ? nab : 0;
   hi = (kv_part == 1) ? nab : nab + nsuf;

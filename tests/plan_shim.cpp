@@ -70,7 +70,7 @@ extern "C" int shim_split(const int32_t* pol, const int32_t* blk_off, const int3
 }
 
 // As shim_split, for a launch that reads only some slots of each request:
-// kv_part 1 the plan's slots, 2 the chunks of the final online span.
+// kv_part 1 the plan's artifact slots, 2 the chunks of the online rows.
 extern "C" int shim_split_part(const int32_t* pol, const int32_t* blk_off, const int32_t* o_rows, int32_t n_req,
                                int32_t S, int32_t S_kv, int32_t tc, int32_t kv_part, int32_t* out) {
   if (n_req < 1 || n_req > att::kMaxReq) return ATTUNER_ERR_INVALID_ARG;

@@ -123,3 +123,58 @@ def test_layout_rejects_too_few_online_rows():
     with pytest.raises(pkg.AttunerError) as e:
         ctx.attend(plan, q, wl.suffix_k, wl.suffix_v)
     assert e.value.status == pkg.attuner.ERR_INVALID_ARG
+
+
+# Many short online spans (1 to 5 tokens) between many artifacts: the online
+# rows are read packed after the artifact slots, so every one of these spans
+# shares 64-row chunks with its neighbours.
+MANY_LENGTHS = [37, 90, 64, 1, 129, 300, 5, 66, 200, 17, 128, 63]
+MANY_LAYOUTS = [
+    [-3, 0, -1, 1, -5, 2, -2, 3, -4, 4, -1, 5, -3, 6, -5, 7, -1, 8, -2, 9, -4, 10, -1, 11],
+    [4, -1, -2, 6, -5, 0, -3, 3, 3, -4, 11, -1, 7],      # starts with an artifact; adjacent spans; a repeat
+    [-5, 8, -1, 2, -2, 9, -5],                             # ends with an explicit span
+]
+
+
+def _many_wl(S, S_kv, seed):
+    reqs = [[a for a in lay if a >= 0] for lay in MANY_LAYOUTS]
+    return make_custom("layout_many", G128, seed, MANY_LENGTHS, reqs, S, S_kv, device=DEV)
+
+
+def _many_reference(wl):
+    g = wl.geom
+    arts_k = {i: f64(t) for i, t in enumerate(wl.art_k)}
+    arts_v = {i: f64(t) for i, t in enumerate(wl.art_v)}
+    outs, lses = [], []
+    for r, lay in enumerate(MANY_LAYOUTS):
+        o, l = oracle.layout_forward(f64(wl.x[r]), f64(wl.w_q), f64(wl.lora_a), f64(wl.lora_b), g.scale,
+                                     f64(wl.q_norm_w), g.rms_eps, g.rope_theta, lay, arts_k, arts_v,
+                                     f64(wl.suffix_k[r]), f64(wl.suffix_v[r]), g.n_q_heads)
+        outs.append(o)
+        lses.append(l)
+    return np.stack(outs), np.stack(lses)
+
+
+@pytest.mark.parametrize("kernel,split,merge", [(1, 0, 0), (1, 2, 1), (1, 4, 2), (2, 0, 0), (2, 2, 0)])
+def test_layout_many_short_spans(kernel, split, merge):
+    import paper_2609_36722_gb300 as pkg
+    S = S_kv = 140          # explicit online rows: 32, 16 and 13; every online row is a query
+    wl = _many_wl(S, S_kv, 91)
+    ref_o, ref_l = _many_reference(wl)
+    ctx, _ = load_context(wl)
+    plan = ctx.assemble_layout(MANY_LAYOUTS)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, kernel)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, split)
+    ctx.set_option(pkg.OPT_SPLIT_MERGE, merge)
+    out, lse = _run(ctx, plan, wl)
+    compare(f64(out), ref_o, f64(lse), ref_l, label=f"many spans kernel={kernel} split={split} merge={merge}")
+
+
+def test_layout_many_short_spans_decode():
+    S, S_kv = 1, 129
+    wl = _many_wl(S, S_kv, 93)
+    ref_o, ref_l = _many_reference(wl)
+    ctx, _ = load_context(wl)
+    plan = ctx.assemble_layout(MANY_LAYOUTS)
+    out, lse = _run(ctx, plan, wl)
+    compare(f64(out), ref_o, f64(lse), ref_l, label="many spans decode")

@@ -170,7 +170,8 @@ def test_plan_tables_of_artifact_lists(shim):
 
 
 def test_plan_tables_of_prompt_layouts(shim):
-    """Online spans between artifacts: slot entries, span records and the assembled
+    """Online spans between artifacts: slot entries (artifact blocks only: the
+    online rows are read after them, packed), span records and the assembled
     position of every online row against the oracle's layout positions."""
     rng = np.random.default_rng(13)
     for trial in range(40):
@@ -203,12 +204,9 @@ def test_plan_tables_of_prompt_layouts(shim):
                         slot += 1
                     tok += L
                 else:
+                    # a span takes no slot; it records the artifact slots before it
                     n = -it
                     assert spans[si].tolist() == [orow, n, slot, tok]
-                    for c in range(0, n, 64):
-                        e = -ents[slot] - 1
-                        assert (e >> 7, e & 127) == (orow + c, min(64, n - c))
-                        slot += 1
                     orow += n
                     si += 1
             assert slot == len(ents) and tok == t["t_art"][r]
@@ -272,8 +270,9 @@ def split(shim, n_q, n_kv, nv_art, o_rows, S, S_kv, tc, num_sms=152, opt_split=0
     assert st == OK
     w = dict(n_req=int(out[0]), row_tiles=int(out[1]), chunk=int(out[2]), n_cta=int(out[3]), cluster=int(out[4]),
              base=out[5:5 + n_req].tolist(), nsplit=out[5 + n_req:].tolist())
-    # the slots the launch reads: the plan's, the final span's chunks, or both
-    nsuf = [-(-(S_kv - o_rows[r]) // 64) for r in range(n_req)]
+    # the slots the launch reads: the plan's artifact slots, the 64-row chunks
+    # of all online rows, or both
+    nsuf = [-(-S_kv // 64) for r in range(n_req)]
     nv = [(nv_art[r] if kv_part != 2 else 0) + (nsuf[r] if kv_part != 1 else 0) for r in range(n_req)]
     return w, nv
 
