@@ -187,8 +187,11 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
   } else if (tc) {
     // Independent splits, one CTA per SM.  Cost of a chunk size = waves x
     // (tiles per CTA + ~4 tiles for the prologue and epilogue + ~2 for the
-    // merge through global memory); pick the number of splits of the
-    // longest request that minimises it.
+    // merge through global memory + ~0.35 per further split, the time the
+    // merging CTA spends reading one more 17 KiB-per-32-column partial back);
+    // pick the number of splits of the longest request that minimises it.
+    // (On the 131k-key layer 4 and 7 splits take the same time; the read-back
+    // term picks 4, which writes and reads half the partial bytes.)
     const int maxt = (maxv + 1) / 2;
     double best = 1e30;
     chunk = maxv;
@@ -201,7 +204,7 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
           ncta += (long long)((nv + 2 * ct - 1) / (2 * ct)) * Hkv * row_tiles;
         }
         const long long waves = (ncta + pol.num_sms - 1) / pol.num_sms;
-        const double cost = (double)waves * (ct + 4.0 + (sp > 1 ? 2.0 : 0.0));
+        const double cost = (double)waves * (ct + 4.0 + (sp > 1 ? 2.0 + 0.35 * (sp - 1) : 0.0));
         if (cost < best - 1e-9) {
           best = cost;
           chunk = 2 * ct;
