@@ -191,7 +191,10 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
     // merging CTA spends reading one more 17 KiB-per-32-column partial back);
     // pick the number of splits of the longest request that minimises it.
     // (On the 131k-key layer 4 and 7 splits take the same time; the read-back
-    // term picks 4, which writes and reads half the partial bytes.)
+    // term picks 4, which writes and reads half the partial bytes.  Plans with
+    // online spans leave it out: their row tiles read different numbers of
+    // artifact slots, and finer chunks balance them - the 131k-key skills
+    // layout took 2.93 ms with 7 chunks per row tile, 3.04 ms with 4.)
     const int maxt = (maxv + 1) / 2;
     double best = 1e30;
     chunk = maxv;
@@ -204,7 +207,8 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
           ncta += (long long)((nv + 2 * ct - 1) / (2 * ct)) * Hkv * row_tiles;
         }
         const long long waves = (ncta + pol.num_sms - 1) / pol.num_sms;
-        const double cost = (double)waves * (ct + 4.0 + (sp > 1 ? 2.0 + 0.35 * (sp - 1) : 0.0));
+        const double readback = t.max_o_rows > 0 ? 0.0 : 0.35 * (sp - 1);
+        const double cost = (double)waves * (ct + 4.0 + (sp > 1 ? 2.0 + readback : 0.0));
         if (cost < best - 1e-9) {
           best = cost;
           chunk = 2 * ct;
