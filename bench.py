@@ -437,11 +437,11 @@ def measure_core(bed, args, world, timer, with_clocks=False, local_rank=0):
 
 
 class HostInputs:
-    """A step's inputs in pinned host memory and their device buffers: the
-    new tokens' hidden states and their own suffix K/V rows (the last S of
-    each request's S_kv rows).  A decode step's earlier suffix rows are the
-    request's resident cache, written by earlier steps: they stay on the
-    device, as the artifact pool does."""
+    """A step's inputs and output in pinned host memory, and the device suffix
+    K/V buffers they update: the new tokens' hidden states and their own
+    suffix K/V rows (the last S of each request's S_kv rows).  A decode step's
+    earlier suffix rows are the request's resident cache, written by earlier
+    steps: they stay on the device, as the artifact pool does."""
 
     def __init__(self, bed):
         import torch
@@ -454,21 +454,15 @@ class HostInputs:
         self.x_d = torch.empty_like(wl.x)
         self.sk_d = wl.suffix_k.clone()
         self.sv_d = wl.suffix_v.clone()
-        self.sk_new = torch.empty(self.sk_h.shape, dtype=self.sk_h.dtype, device=bed.dev)
-        self.sv_new = torch.empty(self.sv_h.shape, dtype=self.sv_h.dtype, device=bed.dev)
         self.h2d_bytes = (self.x_h.numel() + self.sk_h.numel() + self.sv_h.numel()) * 2
         self.d2h_bytes = self.out_h.numel() * 2
 
     def copy_in(self):
+        """The inputs' H2D copies as separate calls (the warm-cache step, whose
+        Q projection runs apart from the attention)."""
         self.x_d.copy_(self.x_h, non_blocking=True)
-        if self.S_old:
-            self.sk_new.copy_(self.sk_h, non_blocking=True)
-            self.sv_new.copy_(self.sv_h, non_blocking=True)
-            self.sk_d[:, self.S_old:].copy_(self.sk_new)
-            self.sv_d[:, self.S_old:].copy_(self.sv_new)
-        else:
-            self.sk_d.copy_(self.sk_h, non_blocking=True)
-            self.sv_d.copy_(self.sv_h, non_blocking=True)
+        self.sk_d[:, self.S_old:].copy_(self.sk_h, non_blocking=True)
+        self.sv_d[:, self.S_old:].copy_(self.sv_h, non_blocking=True)
 
 
 L2_BYTES = 129 << 20
@@ -485,48 +479,37 @@ def working_set_bytes(bed) -> int:
 
 def measure_e2e(bed, args, world, flush, local_rank=0):
     """The same metric through the public API with host buffers, as a serving
-    loop.  Every step assembles its plan, copies its new tokens' inputs from
-    pinned host memory (their hidden states and their own suffix K/V rows; a
-    decode step's earlier suffix rows are the request's resident cache, like
-    the artifact pool), runs attuner_query_attend and copies O back to pinned
-    host memory; a step counts as done once its output is on the host.  Step
-    i+1 is assembled and enqueued while step i runs (two sets of input and
-    output buffers), so host work overlaps device work as in a server.  No
-    flush runs inside the loop: a workload whose working set fits in L2
-    alternates between enough identical, separately loaded contexts that
-    every step reads data the others have evicted."""
+    loop.  Every step assembles its plan (attuner_assemble) and makes one
+    attuner_query_attend_host call, which copies the step's new inputs from
+    pinned host memory (the new tokens' hidden states and their own suffix K/V
+    rows; a decode step's earlier suffix rows are the request's resident cache,
+    like the artifact pool), runs the projection and the attention, and copies
+    O back to pinned host memory, all on the step's stream; a step counts as
+    done once its output is on the host.  Step i+1 is assembled and enqueued,
+    on another stream, while step i runs (two sets of buffers per context), so
+    host work and copies overlap device work as in a server.  No flush runs
+    inside the loop: a workload whose working set fits in L2 alternates between
+    enough identical, separately loaded contexts that every step reads data the
+    others have evicted."""
     import torch
     n_sets = max(1, -(-2 * L2_BYTES // working_set_bytes(bed)))
     beds = [bed] + [Bed(bed.name, bed.dev, local_rank) for _ in range(n_sets - 1)]
     try:
-        # (bed, host/device buffers, output, inputs-copied / computed / output-on-host events)
+        # (bed, host buffers and device suffix K/V, stream, output-on-host event)
         units = []
         for b in beds:
             for _ in range(2):
-                units.append((b, HostInputs(b), torch.empty_like(b.out), torch.cuda.Event(), torch.cuda.Event(),
-                              torch.cuda.Event()))
+                units.append((b, HostInputs(b), torch.cuda.Stream(device=bed.dev), torch.cuda.Event()))
         n_units = len(units)
-        compute = torch.cuda.current_stream()
-        h2d, d2h = torch.cuda.Stream(device=bed.dev), torch.cuda.Stream(device=bed.dev)
 
         def enqueue(i, plan):
-            # inputs on a copy stream, the call on the compute stream, the output
-            # on another copy stream: a step's copies overlap its neighbours'
-            # kernels.  Each unit's buffers are reused only after the step that
-            # last used them was waited for (two steps in flight at most).
-            b, io, out, ev_in, ev_comp, done = units[i % n_units]
+            # each unit's buffers are reused only after the step that last used
+            # them was waited for (two steps in flight at most)
+            b, io, stream, done = units[i % n_units]
             wl, g = b.wl, b.g
-            with torch.cuda.stream(h2d):
-                io.copy_in()
-                ev_in.record(h2d)
-            compute.wait_event(ev_in)
-            b.ctx.query_attend(plan, io.x_d, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, io.sk_d, io.sv_d,
-                               out=out, want_lse=False, stream=compute)
-            ev_comp.record(compute)
-            with torch.cuda.stream(d2h):
-                d2h.wait_event(ev_comp)
-                io.out_h.copy_(out, non_blocking=True)
-                done.record(d2h)
+            b.ctx.query_attend_host(plan, io.x_h, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, io.sk_d,
+                                    io.sv_d, io.sk_h, io.sv_h, out_host=io.out_h, stream=stream)
+            done.record(stream)
 
         def assemble(i):
             b = units[i % n_units][0]
@@ -539,7 +522,7 @@ def measure_e2e(bed, args, world, flush, local_rank=0):
                 if i + 1 < n:
                     plans[i + 1] = assemble(i + 1)     # the next step, while step i runs
                     enqueue(i + 1, plans[i + 1])
-                units[i % n_units][5].synchronize()    # step i's output is on the host
+                units[i % n_units][3].synchronize()    # step i's output is on the host
                 plans.pop(i).free()
 
         run(max(3, args.warmup))
@@ -559,10 +542,11 @@ def measure_e2e(bed, args, world, flush, local_rank=0):
                        f"{working_set_bytes(bed) / 1e6:.0f} MB working set is evicted before its next use"
                        if n_sets > 1 else f"no flush in the loop; the {working_set_bytes(bed) / 1e6:.0f} MB working "
                                           "set of a step exceeds L2"),
-                "includes": "per step: assemble (host block table + upload), H2D of the step's new tokens (x and their "
-                            "own suffix K/V rows; a decode step's earlier suffix rows stay resident) on a copy stream, "
-                            "query_attend, D2H of O on a second copy stream and a wait for it; step i+1 assembled "
-                            "and enqueued while step i runs"}
+                "includes": "per step: assemble (host block table + upload) and one attuner_query_attend_host call "
+                            "(H2D of the step's new tokens - x and their own suffix K/V rows; a decode step's earlier "
+                            "suffix rows stay resident - the Q projection, the attention and the D2H of O, on the "
+                            "step's stream) and a wait for the output; step i+1 assembled and enqueued on another "
+                            "stream while step i runs"}
     finally:
         for b in beds[1:]:
             b.close()

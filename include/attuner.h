@@ -243,6 +243,38 @@ attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_plan* plan, 
                                     const void* suffix_k, const void* suffix_v, int32_t S,
                                     int32_t S_kv, void* out, float* lse_out, void* stream);
 
+/* The whole path for a step whose new inputs and whose output live in HOST
+ * memory (the request-time path of Sec. 3 Eq. query-adaptation and Sec. 2.2
+ * Eq. routing-oracle, as attuner_query_attend).  On `stream`, in order: the
+ * new tokens' hidden states are copied from host memory into stream-ordered
+ * device scratch; when k_new_host and v_new_host are given, the new tokens'
+ * own K/V rows are copied into rows S_kv - S .. S_kv - 1 of each request of
+ * suffix_k / suffix_v; the projection and the attention run; O (and the LSE
+ * when lse_host is given) are copied back to host memory.
+ *   x_host      [n_req, S, hidden] bf16, host memory
+ *   k_new_host, v_new_host  [n_req, S, Hkv, d] bf16, host memory, RoPE'd at
+ *               the tokens' positions; both NULL when the caller's device
+ *               suffix K/V already hold them (e.g. from attuner_kv_project)
+ *   suffix_k, suffix_v  [n_req, S_kv, Hkv, d] bf16, device memory: the rows
+ *               before the new tokens are the request's resident online KV
+ *   out_host    [n_req, S, Hq, d] bf16, host memory; lse_host [n_req, S, Hq]
+ *               fp32, host memory, or NULL
+ *   w_q, lora_a, lora_b, q_norm_w: device memory, as in attuner_q_project
+ * The call returns once everything is enqueued; out_host and lse_host hold
+ * the result when the stream reaches the end of the call (an event recorded
+ * after it, or a stream synchronisation).  The host buffers must stay valid
+ * and unchanged until then.  Pinned (page-locked) host memory makes the
+ * copies asynchronous; with pageable memory the driver stages them and the
+ * call may block.  Errors: as attuner_query_attend, plus INVALID_ARG for a
+ * NULL x_host, out_host, suffix_k or suffix_v, or only one of k_new_host and
+ * v_new_host given. */
+attuner_status attuner_query_attend_host(attuner_ctx* ctx, const attuner_plan* plan,
+                                         const void* x_host, const void* w_q, const void* lora_a,
+                                         const void* lora_b, int32_t r, float s, const void* q_norm_w,
+                                         const void* k_new_host, const void* v_new_host,
+                                         void* suffix_k, void* suffix_v, int32_t S, int32_t S_kv,
+                                         void* out_host, float* lse_host, void* stream);
+
 /* Keys stored before RoPE, rotated to their target positions at assembly:
  * the read of the paper's EPIC baseline (App. C.2 "Training-Free Baselines",
  * EPIC paragraph: cached keys kept un-rotated and rotated to their place in

@@ -47,6 +47,7 @@ EXPORTS = [
     "attuner_set_option", "attuner_last_launch_count", "attuner_last_error",
     "attuner_attend_static_scratch", "attuner_register_artifacts_host", "attuner_pool_reset",
     "attuner_kv_project", "attuner_assemble_layout", "attuner_plan_rotate_keys", "attuner_attend_ape",
+    "attuner_query_attend_host",
 ]
 
 
@@ -84,6 +85,8 @@ SIGNATURES = {
     "attuner_attend_static_scratch": ([_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp], _i32),
     "attuner_query_attend": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _vp, _vp, _i32, _i32,
                               _vp, _vp, _vp], _i32),
+    "attuner_query_attend_host": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, ctypes.c_float, _vp, _vp, _vp, _vp, _vp,
+                                   _i32, _i32, _vp, _vp, _vp], _i32),
     "attuner_pool_info": ([_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _p_i32, _p_i32], _i32),
     "attuner_sync_status": ([_vp, _vp], _i32),
     "attuner_set_option": ([_vp, _i32, ctypes.c_int64], _i32),
@@ -139,6 +142,19 @@ def _ptr(t: Optional[torch.Tensor], name: str, dtype=torch.bfloat16, device=None
         raise ValueError(f"{name} must be a CUDA tensor")
     if device is not None and t.device != device:
         raise ValueError(f"{name} is on {t.device}, the context on {device}")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _host_ptr(t: Optional[torch.Tensor], name: str, dtype=torch.bfloat16) -> Optional[int]:
+    # a host (CPU) tensor's address; pinned memory keeps the library's copies asynchronous
+    if t is None:
+        return None
+    if t.is_cuda:
+        raise ValueError(f"{name} must be a CPU tensor")
     if t.dtype != dtype:
         raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
     if not t.is_contiguous():
@@ -386,6 +402,31 @@ class Context:
                                           self._p(suffix_v, "suffix_v"), S, S_kv, self._p(out, "out"),
                                           self._p(lse, "lse", torch.float32), self._s(stream)))
         return out, lse
+
+    def query_attend_host(self, plan: Plan, x_host, w_q, lora_a, lora_b, s: float, q_norm_w, suffix_k, suffix_v,
+                          k_new_host=None, v_new_host=None, out_host: Optional[torch.Tensor] = None,
+                          lse_host: Optional[torch.Tensor] = None, stream=None):
+        """attuner_query_attend_host: x_host [n_req, S, hidden], k_new_host / v_new_host
+        [n_req, S, Hkv, d] (or None) and out_host / lse_host are CPU tensors (pinned for
+        asynchronous copies); suffix_k / suffix_v [n_req, S_kv, Hkv, d] and the weights are
+        on the device.  The outputs are valid once `stream` has run the call."""
+        n_req, S, _ = x_host.shape
+        S_kv = suffix_k.shape[1]
+        r = 0 if lora_a is None else lora_a.shape[0]
+        if (k_new_host is None) != (v_new_host is None):
+            raise ValueError("k_new_host and v_new_host must both be given or both be None")
+        if k_new_host is not None and (k_new_host.shape != v_new_host.shape or k_new_host.shape[:2] != (n_req, S)):
+            raise ValueError("k_new_host and v_new_host must be [n_req, S, Hkv, d]")
+        if out_host is None:
+            out_host = torch.empty(n_req, S, self.cfg.n_q_heads, self.cfg.head_dim, dtype=torch.bfloat16,
+                                   pin_memory=True)
+        _check(lib().attuner_query_attend_host(
+            self.handle, plan.handle, _host_ptr(x_host, "x_host"), self._p(w_q, "w_q"), self._p(lora_a, "lora_a"),
+            self._p(lora_b, "lora_b"), r, float(s), self._p(q_norm_w, "q_norm_w"),
+            _host_ptr(k_new_host, "k_new_host"), _host_ptr(v_new_host, "v_new_host"),
+            self._p(suffix_k, "suffix_k"), self._p(suffix_v, "suffix_v"), S, S_kv, _host_ptr(out_host, "out_host"),
+            _host_ptr(lse_host, "lse_host", torch.float32), self._s(stream)))
+        return out_host, lse_host
 
     # --- misc
     def pool_tensors(self):

@@ -895,6 +895,64 @@ extern "C" attuner_status attuner_query_attend(attuner_ctx* ctx, const attuner_p
   return finish_call(ctx, e, st);
 }
 
+// The whole path with the step's new inputs and its output in host memory:
+// the copies in, the projection and attention of attuner_query_attend, and
+// the copies out, all enqueued on the caller's stream from one host call.
+extern "C" attuner_status attuner_query_attend_host(attuner_ctx* ctx, const attuner_plan* plan, const void* x_host,
+                                                    const void* w_q, const void* lora_a, const void* lora_b,
+                                                    int32_t r, float s, const void* q_norm_w, const void* k_new_host,
+                                                    const void* v_new_host, void* suffix_k, void* suffix_v, int32_t S,
+                                                    int32_t S_kv, void* out_host, float* lse_host, void* stream) {
+  attuner_status e = check_common(ctx, plan, S, S_kv);
+  if (e != ATTUNER_OK) return e;
+  CHECK_ARG(x_host != nullptr && out_host != nullptr && suffix_k != nullptr && suffix_v != nullptr,
+            "x_host, out_host, suffix_k and suffix_v must not be NULL");
+  CHECK_ARG((k_new_host == nullptr) == (v_new_host == nullptr),
+            "k_new_host and v_new_host must both be given or both be NULL");
+  if ((e = set_device(ctx)) != ATTUNER_OK) return e;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const attuner_config& c = ctx->cfg;
+  const int M = plan->n_req * S;
+  auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
+  const size_t x_bytes = (size_t)M * c.hidden * 2;
+  const size_t o_bytes = (size_t)M * c.n_q_heads * c.head_dim * 2;
+  const size_t l_bytes = lse_host ? (size_t)M * c.n_q_heads * 4 : 0;
+  Scratch sc{ctx, st};
+  sc.cap = al(x_bytes) + 2 * al(o_bytes) + al(l_bytes) + q_project_scratch(ctx, M);
+  CUDA_TRY(cudaMallocFromPoolAsync(&sc.base, sc.cap, ctx->mempool, st));
+  char* base = static_cast<char*>(sc.base);
+  void* x = base + sc.take(al(x_bytes));
+  void* q = base + sc.take(al(o_bytes));
+  void* out = base + sc.take(al(o_bytes));
+  float* lse = lse_host ? reinterpret_cast<float*>(base + sc.take(al(l_bytes))) : nullptr;
+  int launches = 0;
+  cudaError_t ce = cudaMemcpyAsync(x, x_host, x_bytes, cudaMemcpyHostToDevice, st);
+  if (ce == cudaSuccess && k_new_host != nullptr) {
+    // the S new rows of each request, into rows S_kv - S .. of its S_kv
+    const size_t row = (size_t)c.n_kv_heads * c.head_dim * 2;
+    const size_t off = (size_t)(S_kv - S) * row;
+    ce = cudaMemcpy2DAsync(static_cast<char*>(suffix_k) + off, (size_t)S_kv * row, k_new_host, (size_t)S * row,
+                           (size_t)S * row, plan->n_req, cudaMemcpyHostToDevice, st);
+    if (ce == cudaSuccess)
+      ce = cudaMemcpy2DAsync(static_cast<char*>(suffix_v) + off, (size_t)S_kv * row, v_new_host, (size_t)S * row,
+                             (size_t)S * row, plan->n_req, cudaMemcpyHostToDevice, st);
+  }
+  if (ce != cudaSuccess) e = fail(ATTUNER_ERR_CUDA, std::string("host-to-device copy: ") + cudaGetErrorString(ce));
+  if (e == ATTUNER_OK)
+    e = q_project_impl(ctx, plan, x, w_q, lora_a, lora_b, r, s, q_norm_w, S, S_kv, q, st, sc, launches);
+  if (e == ATTUNER_OK)
+    e = attend_launch(ctx, plan, q, suffix_k, suffix_v, S, S_kv, out, lse, st, nullptr, launches);
+  if (e == ATTUNER_OK) {
+    ce = cudaMemcpyAsync(out_host, out, o_bytes, cudaMemcpyDeviceToHost, st);
+    if (ce == cudaSuccess && lse_host != nullptr)
+      ce = cudaMemcpyAsync(lse_host, lse, l_bytes, cudaMemcpyDeviceToHost, st);
+    if (ce != cudaSuccess) e = fail(ATTUNER_ERR_CUDA, std::string("device-to-host copy: ") + cudaGetErrorString(ce));
+  }
+  cudaFreeAsync(sc.base, st);
+  ctx->last_launches = launches;
+  return finish_call(ctx, e, st);
+}
+
 // ---------------------------------------------------------------------------
 // APE-style read (App. C.2, APE paragraph): context and online attention
 // computed separately, combined through calibrated log-sum-exp terms

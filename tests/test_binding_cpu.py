@@ -204,6 +204,11 @@ def test_every_public_method_reaches_its_entry_point(ctx, monkeypatch):
     kn = FakeTensor((64,), ptr=0xD000)
     hk = FakeTensor((5, 2, 64), device="cpu", pinned=True, ptr=0xE000)
     hv = FakeTensor((5, 2, 64), device="cpu", pinned=True, ptr=0xF000)
+    xh = FakeTensor((2, 3, 256), device="cpu", pinned=True, ptr=0x10000)
+    kh = FakeTensor((2, 3, 2, 64), device="cpu", pinned=True, ptr=0x11000)
+    vh = FakeTensor((2, 3, 2, 64), device="cpu", pinned=True, ptr=0x12000)
+    oh = FakeTensor((2, 3, 4, 64), device="cpu", pinned=True, ptr=0x13000)
+    lh = FakeTensor((2, 3, 4), dtype=torch.float32, device="cpu", pinned=True, ptr=0x14000)
     st = FakeStream()
     ctx_calls = {
         "register_artifact": (lambda: c.register_artifact(FakeTensor((5, 2, 64)), FakeTensor((5, 2, 64)), stream=st),
@@ -221,6 +226,8 @@ def test_every_public_method_reaches_its_entry_point(ctx, monkeypatch):
                                   "attuner_attend_static_scratch"),
         "query_attend": (lambda: c.query_attend(plan, x, w, la, lb, 2.0, qn, sk, sv, out=q, lse=lse, stream=st),
                          "attuner_query_attend"),
+        "query_attend_host": (lambda: c.query_attend_host(plan, xh, w, la, lb, 2.0, qn, sk, sv, kh, vh, out_host=oh,
+                                                          lse_host=lh, stream=st), "attuner_query_attend_host"),
         "rotate_keys": (lambda: c.rotate_keys(plan, stream=st), "attuner_plan_rotate_keys"),
         "attend_ape": (lambda: c.attend_ape(plan, q, sk, sv, 0.9, 0.9, out=out, lse=lse, stream=st),
                        "attuner_attend_ape"),
@@ -247,3 +254,31 @@ def test_every_public_method_reaches_its_entry_point(ctx, monkeypatch):
     c.close()
     assert fake.calls[-1][0] == "attuner_destroy"
     assert dev.dim() == 1
+
+
+def test_query_attend_host_refuses_device_or_mismatched_host_buffers(ctx):
+    """The host-buffer call takes CPU tensors for the step's inputs and outputs
+    and device tensors for the resident state; the wrong kind, or only one of
+    the new K/V row buffers, is refused before the library is called."""
+    c, plan, fake = ctx
+    plan.ctx = c
+    plan.n_req = 2
+    q, sk, sv, out, lse = _attend_args()
+    w = FakeTensor((256, 256), ptr=0x7000)
+    qn = FakeTensor((64,), ptr=0xA000)
+    xh = FakeTensor((2, 3, 256), device="cpu", pinned=True, ptr=0x10000)
+    xd = FakeTensor((2, 3, 256), ptr=0x6000)
+    kh = FakeTensor((2, 3, 2, 64), device="cpu", pinned=True, ptr=0x11000)
+    oh = FakeTensor((2, 3, 4, 64), device="cpu", pinned=True, ptr=0x13000)
+    st = FakeStream()
+    with pytest.raises(ValueError):
+        c.query_attend_host(plan, xd, w, None, None, 2.0, qn, sk, sv, out_host=oh, stream=st)
+    with pytest.raises(ValueError):
+        c.query_attend_host(plan, xh, w, None, None, 2.0, qn, sk, sv, kh, None, out_host=oh, stream=st)
+    with pytest.raises(ValueError):
+        c.query_attend_host(plan, xh, w, None, None, 2.0, qn, sk, sv, out_host=out, stream=st)
+    assert fake.calls == []
+    c.query_attend_host(plan, xh, w, None, None, 2.0, qn, sk, sv, out_host=oh, stream=st)
+    name, args = fake.calls[-1]
+    assert name == "attuner_query_attend_host"
+    assert args[2] == 0x10000 and args[9] is None and args[10] is None and args[15] == 0x13000
