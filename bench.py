@@ -925,9 +925,13 @@ def main():
         return
 
     if world > 1:
+        import datetime
+
         import torch
         torch.cuda.set_device(local_rank)
-        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+        # a rank whose part failed must not hold the others at a collective for long
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank),
+                                             timeout=datetime.timedelta(minutes=5))
     res, rc = run_ours(args, rank, world, local_rank)
     if rank == 0:
         print(json.dumps(res))
