@@ -52,7 +52,7 @@ typedef int32_t attuner_status;
 #define ATTUNER_ERR_UNKNOWN_ARTIFACT (-3) /* an artifact id was never registered         */
 #define ATTUNER_ERR_CUDA             (-4) /* a CUDA runtime or driver call failed        */
 #define ATTUNER_ERR_TIMEOUT          (-5) /* a kernel's bounded wait ran out             */
-#define ATTUNER_ERR_UNSUPPORTED      (-6) /* geometry this build has no kernel for       */
+#define ATTUNER_ERR_UNSUPPORTED      (-6) /* geometry the library has no kernel for     */
 #define ATTUNER_ERR_DEVICE_CHECK     (-7) /* a kernel's bounds check rejected an index   */
 
 /* Tokens per paged KV block.  Paging is this library's storage; the paper
