@@ -513,41 +513,16 @@ attuner_status att::check_common(attuner_ctx* ctx, const attuner_plan* plan, int
   return ATTUNER_OK;
 }
 
-// Launch shape of the projection kernel: rows per CTA (mr x 128: one or two
-// TMEM accumulators sharing each W tile) and K slices per tile (ks CTAs of a
-// cluster exchanging fp32 partials through distributed shared memory).  The
-// estimate is waves x (start-up + operand bytes + epilogue), with constants
-// from per-CTA timelines on GB300: about 2.5 us from launch to the first full
-// stage; the operand stream, (mr*128 + D + r) * hidden/ks * 2 bytes per CTA
-// (out-of-range rows of a tile are filled, not skipped), at about 100 GB/s per
-// SM; an epilogue of about 3.5 us, plus 1.5 us and the exchanged partial rows
-// at about 20 GB/s when the K dimension is split.  ATTUNER_OPT_QPROJ_SPLIT_K
-// and ATTUNER_OPT_QPROJ_ROWS pin either choice.  {0, 0} when the options leave
-// no supported shape.
-struct QpShape {
-  int mr, ks;
-};
+// Launch shape of the projection kernel (choose_qproj_shape in plan.cpp):
+// rows per CTA and K slices per tile, from the context's options and SM count.
 static QpShape qproj_shape(const attuner_ctx* ctx, int heads, int M, int n_lora) {
-  const int D = ctx->cfg.head_dim, nk = ctx->cfg.hidden / 64;
-  QpShape best{0, 0};
-  double best_t = 0.0;
-  for (int mr = 1; mr <= 2; ++mr)
-    for (int ks = 1; ks <= 8; ks *= 2) {
-      if (ctx->opt_qproj_rows != 0 && ctx->opt_qproj_rows != 128 * mr) continue;
-      if (ctx->opt_qproj_split != 0 && ctx->opt_qproj_split != ks) continue;
-      if (ks > nk || !qproj_shape_supported(D, mr, ks, n_lora)) continue;
-      const long long tiles = (long long)heads * ((M + 128 * mr - 1) / (128 * mr));
-      const long long waves = (tiles * ks + ctx->num_sms - 1) / ctx->num_sms;
-      const double bytes = (double)(128 * mr + D + n_lora) * (double)(ctx->cfg.hidden / ks) * 2.0;
-      const double exch = (double)std::min(128 * mr, M) * (D + n_lora) * 4.0;
-      const double epi = ks > 1 ? 5.0e-6 + exch / 20e9 : 3.5e-6;
-      const double t = (double)waves * (2.5e-6 + bytes / 100e9 + epi);
-      if (best.mr == 0 || t < best_t) {
-        best = {mr, ks};
-        best_t = t;
-      }
-    }
-  return best;
+  QpPolicy pol;
+  pol.head_dim = ctx->cfg.head_dim;
+  pol.hidden = ctx->cfg.hidden;
+  pol.num_sms = ctx->num_sms;
+  pol.opt_rows = ctx->opt_qproj_rows;
+  pol.opt_split = ctx->opt_qproj_split;
+  return choose_qproj_shape(pol, heads, M, n_lora);
 }
 
 static attuner_status q_project_impl(attuner_ctx* ctx, const attuner_plan* plan, const void* x, const void* w_q,

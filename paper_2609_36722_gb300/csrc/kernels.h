@@ -129,10 +129,8 @@ cudaError_t launch_pool_write(const __nv_bfloat16* k, const __nv_bfloat16* v, __
                               __nv_bfloat16* vpool, int L, int Hkv, int D, int first_block,
                               cudaStream_t st);
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st);
-// Row tiles per CTA (mr = 1 or 2 accumulators of 128 rows) and K slices per
-// tile (ks = 1, 2, 4 or 8 CTAs, a cluster): shapes the kernel supports for a
-// head size and LoRA rank (rounded up to 16).
-bool qproj_shape_supported(int D, int mr, int ks, int n_lora);
+// Launch with mr accumulators of 128 rows per CTA and ks K slices per tile
+// (qproj_shape_supported in plan.h lists the shapes).
 cudaError_t launch_qproj(const QprojParams& p, int D, int mr, int ks, cudaStream_t st);
 // Launch with programmatic stream serialization (the kernel may start while
 // the previous kernel of the stream finishes; see grid_dep_wait) and, when

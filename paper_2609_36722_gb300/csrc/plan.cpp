@@ -265,4 +265,43 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
   return ATTUNER_OK;
 }
 
+bool qproj_shape_supported(int D, int mr, int ks, int n_lora) {
+  if (D != 64 && D != 128) return false;
+  if (mr != 1 && mr != 2) return false;
+  if (ks != 1 && ks != 2 && ks != 4 && ks != 8) return false;
+  if (ks == 1) return true;
+  const int tpr = ks / mr;
+  if (tpr < 1 || D / 2 / tpr < 8) return false;
+  return qp_recv_bytes(mr, D, qp_lora_width(n_lora)) <= qp_ring_bytes(D, mr);
+}
+
+// The estimate is waves x (start-up + operand bytes + epilogue), with
+// constants from per-CTA timelines on GB300: about 2.5 us from launch to the
+// first full stage; the operand stream, (mr*128 + D + r) * hidden/ks * 2 bytes
+// per CTA (out-of-range rows of a tile are filled, not skipped), at about
+// 100 GB/s per SM; an epilogue of about 3.5 us, plus 1.5 us and the exchanged
+// partial rows at about 20 GB/s when the K dimension is split.
+QpShape choose_qproj_shape(const QpPolicy& pol, int heads, int M, int n_lora) {
+  const int D = pol.head_dim, nk = pol.hidden / 64;
+  QpShape best{0, 0};
+  double best_t = 0.0;
+  for (int mr = 1; mr <= 2; ++mr)
+    for (int ks = 1; ks <= 8; ks *= 2) {
+      if (pol.opt_rows != 0 && pol.opt_rows != 128 * mr) continue;
+      if (pol.opt_split != 0 && pol.opt_split != ks) continue;
+      if (ks > nk || !qproj_shape_supported(D, mr, ks, n_lora)) continue;
+      const long long tiles = (long long)heads * ((M + 128 * mr - 1) / (128 * mr));
+      const long long waves = (tiles * ks + pol.num_sms - 1) / pol.num_sms;
+      const double bytes = (double)(128 * mr + D + n_lora) * (double)(pol.hidden / ks) * 2.0;
+      const double exch = (double)std::min(128 * mr, M) * (D + n_lora) * 4.0;
+      const double epi = ks > 1 ? 5.0e-6 + exch / 20e9 : 3.5e-6;
+      const double t = (double)waves * (2.5e-6 + bytes / 100e9 + epi);
+      if (best.mr == 0 || t < best_t) {
+        best = {mr, ks};
+        best_t = t;
+      }
+    }
+  return best;
+}
+
 }  // namespace att

@@ -33,6 +33,42 @@ constexpr int kMaxChunkBlocks = 4096;
 constexpr int kMaxSplits = 32;
 
 // ---------------------------------------------------------------------------
+// The Q-projection kernel's shared-memory geometry (qproj.cuh), which the
+// host's choice of its launch shape obeys too.  A stage of the TMA ring holds
+// MR x tiles (128 rows x 64 bf16), the head's D rows of W_q and up to 64 rows
+// of LoRA A; the ring takes as many stages as fit in 200 KiB.  With the K
+// dimension split over a cluster, the fp32 partial rows of the tile (D + R
+// columns, R = LoRA rank rounded up to 16) are exchanged in the ring, at a row
+// pitch that is 4 mod 8 floats.
+ATT_HD constexpr int qp_stage_bytes(int D, int MR) { return MR * 128 * 128 + D * 128 + 64 * 128; }
+ATT_HD constexpr int qp_ring_bytes(int D, int MR) {
+  return (200 * 1024) / qp_stage_bytes(D, MR) * qp_stage_bytes(D, MR);
+}
+ATT_HD constexpr int qp_pitch(int W) { return W + ((12 - W % 8) % 8); }
+ATT_HD constexpr int qp_recv_bytes(int MR, int D, int R) { return MR * 128 * qp_pitch(D + R) * 4; }
+ATT_HD constexpr int qp_lora_width(int n_lora) {
+  return n_lora == 0 ? 0 : (n_lora <= 16 ? 16 : (n_lora <= 32 ? 32 : 64));
+}
+
+// Launch shapes of the projection kernel: mr = 1 or 2 accumulators of 128
+// rows per CTA, ks = 1, 2, 4 or 8 CTAs (a cluster) splitting the K dimension
+// of a tile.  Supported where the K-split epilogue keeps at least 8 rotary
+// pairs per thread (ks/mr threads per row) and the exchange fits the ring.
+bool qproj_shape_supported(int D, int mr, int ks, int n_lora);
+
+struct QpPolicy {
+  int32_t head_dim, hidden, num_sms;
+  int32_t opt_rows;    // 128 or 256 pins the rows per CTA, 0 = chosen here
+  int32_t opt_split;   // 1, 2, 4 or 8 pins the K slices, 0 = chosen here
+};
+struct QpShape {
+  int mr, ks;          // {0, 0}: no supported shape under the options
+};
+// The shape for `heads` heads (grid heads: 2 Hkv in K/V mode) and M rows,
+// LoRA rank rounded up to 16 (n_lora, 0 without an adapter).
+QpShape choose_qproj_shape(const QpPolicy& pol, int heads, int M, int n_lora);
+
+// ---------------------------------------------------------------------------
 // Work decomposition shared by the attention kernels (passed by value).
 // A request's KV sequence is a list of "virtual blocks": its artifact blocks
 // (from the plan's block table, runtime order) followed by ceil(S_kv/64)

@@ -1,5 +1,5 @@
-// qproj.cu - launch of the Q-projection kernel (qproj.cuh): supported shapes,
-// the dispatch over (D, MR), and the D = 128, one-accumulator instantiations.
+// qproj.cu - launch of the Q-projection kernel (qproj.cuh): the dispatch over
+// (D, MR) and the D = 128, one-accumulator instantiations.
 #include "qproj.cuh"
 
 namespace att {
@@ -8,10 +8,6 @@ template cudaError_t launch_qproj_mr<128, 1>(const QprojParams&, int, cudaStream
 extern template cudaError_t launch_qproj_mr<128, 2>(const QprojParams&, int, cudaStream_t);
 extern template cudaError_t launch_qproj_mr<64, 1>(const QprojParams&, int, cudaStream_t);
 extern template cudaError_t launch_qproj_mr<64, 2>(const QprojParams&, int, cudaStream_t);
-
-bool qproj_shape_supported(int D, int mr, int ks, int n_lora) {
-  return qproj_shape_supported_impl(D, mr, ks, n_lora);
-}
 
 cudaError_t launch_qproj(const QprojParams& p, int D, int mr, int ks, cudaStream_t st) {
   if (!qproj_shape_supported(D, mr, ks, p.n_lora) || p.hidden / 64 < ks) return cudaErrorInvalidValue;

@@ -42,23 +42,16 @@ struct QpLayout {
   static constexpr int X_BYTES = 128 * 128;               // one x tile: 128 rows x 64 bf16 (SW128)
   static constexpr int W_OFF = MR * X_BYTES;               // the head's D rows of W_q x 64 bf16 ...
   static constexpr int A_OFF = W_OFF + D * 128;            // ... then up to 64 rows of LoRA A
-  static constexpr int STAGE = A_OFF + 64 * 128;
+  static constexpr int STAGE = qp_stage_bytes(D, MR);
   static constexpr int NS = (200 * 1024) / STAGE;          // 5/3 stages (D = 128), 6/4 (D = 64)
-  static constexpr int RING = NS * STAGE;
+  static constexpr int RING = qp_ring_bytes(D, MR);
+  static_assert(STAGE == A_OFF + 64 * 128 && RING == NS * STAGE, "stage layout");
   static constexpr int B_OFF = RING;                       // B_h: [r/8][D rows][8 bf16], no swizzle
   static constexpr int BAR_OFF = B_OFF + 64 * D * 2;
   static constexpr int SMEM = BAR_OFF + 256 + 1024;       // + alignment slack
   static constexpr uint32_t TMEM_COLS = MR == 2 ? 512 : 256;
   static constexpr uint32_t ACC_STRIDE = 256;              // accumulator a at TMEM column 256 a
 };
-
-// Row pitch (floats) of the partial rows exchanged between the K slices: the
-// smallest pitch >= W that is 4 mod 8, so the 16-byte stores of 8 consecutive
-// rows fall on distinct bank groups.
-__host__ __device__ constexpr int qp_pitch(int W) { return W + ((12 - W % 8) % 8); }
-
-// Bytes of the exchange buffer (all KS partial slots of the rows one CTA owns).
-__host__ __device__ constexpr int qp_recv_bytes(int MR, int D, int R) { return MR * 128 * qp_pitch(D + R) * 4; }
 
 // Shared-memory matrix descriptor, no swizzle (canonical K-major layout of
 // 8-row x 16-byte core matrices): lbo = byte distance between the two
@@ -478,19 +471,6 @@ __global__ void __launch_bounds__(192, 1) qproj_kernel(const __grid_constant__ Q
     tc_fence_after();
     tmem_dealloc(tmem, L::TMEM_COLS);
   }
-}
-
-inline bool qproj_shape_supported_impl(int D, int mr, int ks, int n_lora) {
-  if (D != 64 && D != 128) return false;
-  if (mr != 1 && mr != 2) return false;
-  if (ks != 1 && ks != 2 && ks != 4 && ks != 8) return false;
-  if (ks == 1) return true;
-  const int tpr = ks / mr;
-  if (tpr < 1 || D / 2 / tpr < 8) return false;
-  const int R = n_lora == 0 ? 0 : (n_lora <= 16 ? 16 : (n_lora <= 32 ? 32 : 64));
-  const int ring = D == 128 ? (mr == 2 ? QpLayout<128, 2>::RING : QpLayout<128, 1>::RING)
-                            : (mr == 2 ? QpLayout<64, 2>::RING : QpLayout<64, 1>::RING);
-  return qp_recv_bytes(mr, D, R) <= ring;
 }
 
 template <int D, int MR, int KS>

@@ -100,3 +100,21 @@ extern "C" int shim_split_part(const int32_t* pol, const int32_t* blk_off, const
   }
   return ATTUNER_OK;
 }
+
+// The Q projection's launch shape: pol = head_dim, hidden, num_sms, opt_rows,
+// opt_split; out = {mr, ks} ({0, 0}: no supported shape).
+extern "C" void shim_qproj_shape(const int32_t* pol, int32_t heads, int32_t M, int32_t n_lora, int32_t* out) {
+  att::QpPolicy p;
+  p.head_dim = pol[0];
+  p.hidden = pol[1];
+  p.num_sms = pol[2];
+  p.opt_rows = pol[3];
+  p.opt_split = pol[4];
+  const att::QpShape s = att::choose_qproj_shape(p, heads, M, n_lora);
+  out[0] = s.mr;
+  out[1] = s.ks;
+}
+
+extern "C" int shim_qproj_supported(int32_t D, int32_t mr, int32_t ks, int32_t n_lora) {
+  return att::qproj_shape_supported(D, mr, ks, n_lora) ? 1 : 0;
+}

@@ -401,3 +401,68 @@ def test_split_work_rejects_a_launch_of_2_31_ctas(shim):
     pol_auto = _i32([64, 8, 152, 0, 1] + [0] * 9)
     st = shim.shim_split(pol_auto[1], blk[1], orow[1], n_req, 64, 64, 0, out.ctypes.data_as(I32P))
     assert st == OK and 0 < out[3] < 1 << 31
+
+
+# ---------------------------------------------------------------------------
+# Q projection launch shape (rows per CTA, K slices per tile)
+# ---------------------------------------------------------------------------
+def qp_shape(shim, head_dim, hidden, heads, M, n_lora, num_sms=152, rows=0, split=0):
+    pol, pp = _i32([head_dim, hidden, num_sms, rows, split])
+    out = np.zeros(2, np.int32)
+    shim.shim_qproj_shape(pp, heads, M, n_lora, out.ctypes.data_as(I32P))
+    return int(out[0]), int(out[1])
+
+
+def test_qproj_supported_shapes(shim):
+    """The K-split epilogue needs at least 8 rotary pairs per thread (ks/mr
+    threads per row) and the exchanged fp32 rows must fit the stage ring."""
+    sup = lambda D, mr, ks, nl: bool(shim.shim_qproj_supported(D, mr, ks, nl))
+    for D in (64, 128):
+        for mr in (1, 2):
+            assert sup(D, mr, 1, 0) and sup(D, mr, 1, 64)           # no split: every rank
+    assert sup(128, 1, 8, 16) and sup(128, 2, 8, 16) and sup(64, 2, 8, 16)
+    assert not sup(64, 1, 8, 16)                                     # 32/8 = 4 pairs per thread
+    assert sup(128, 2, 2, 32) and not sup(128, 2, 2, 64)            # 256 rows x 196 floats > ring
+    assert sup(128, 1, 2, 64)
+    assert not sup(96, 1, 1, 0) and not sup(128, 3, 1, 0) and not sup(128, 1, 3, 0)
+
+
+def test_qproj_shape_of_the_measured_layers(shim):
+    """The cost model's picks on 152 SMs, measured best on GB300: Qwen3-4B
+    prefill (M = 256) 128 rows and 2 slices, decode (M = 64) 128 rows and 4
+    slices, the 2048-token layers 256 rows and no split; the K/V mode's 16
+    grid heads of a decode step 8 slices."""
+    assert qp_shape(shim, 128, 2560, 32, 256, 16) == (1, 2)
+    assert qp_shape(shim, 128, 4096, 32, 64, 16) == (1, 4)
+    assert qp_shape(shim, 128, 4096, 32, 2048, 16) == (2, 1)
+    assert qp_shape(shim, 128, 4096, 16, 64, 0) == (1, 8)
+    assert qp_shape(shim, 64, 256, 4, 16, 16) == (1, 1)
+
+
+def test_qproj_shape_options_and_limits(shim):
+    rng = np.random.default_rng(29)
+    for _ in range(300):
+        D = int(rng.choice([64, 128]))
+        hidden = 64 * int(rng.integers(1, 80))
+        heads = int(rng.integers(1, 70))
+        M = int(rng.integers(1, 5000))
+        nl = int(rng.choice([0, 16, 32, 64]))
+        sms = int(rng.choice([20, 148, 152]))
+        rows = int(rng.choice([0, 128, 256]))
+        split = int(rng.choice([0, 1, 2, 4, 8]))
+        mr, ks = qp_shape(shim, D, hidden, heads, M, nl, sms, rows, split)
+        if mr == 0:
+            # only pinned options can leave no shape
+            assert rows or split
+            assert ks == 0
+            continue
+        assert bool(shim.shim_qproj_supported(D, mr, ks, nl))
+        assert ks <= hidden // 64                       # every CTA has a K block
+        if rows:
+            assert mr * 128 == rows
+        if split:
+            assert ks == split
+    # one K block (hidden 64): no split
+    for D in (64, 128):
+        assert qp_shape(shim, D, 64, 8, 100, 16)[1] == 1
+    assert qp_shape(shim, 64, 512, 4, 300, 8, rows=128, split=8) == (0, 0)
