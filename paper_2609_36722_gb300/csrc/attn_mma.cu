@@ -5,15 +5,16 @@
 // log-sum-exp merge of its split-KV chunks, done by the last CTA of each row
 // tile to finish; and APE's calibrated combination of two partial results.
 //
-// K3 is bound by HBM: every (request, KV head) streams its assembled K/V
-// once (4 KiB per token at Hkv = 8, d = 128).  One CTA owns 16 packed query
-// rows (token * G + head_in_group) of one request and KV head, and one
-// chunk of its virtual block list.  Warp 4 streams 64-token K/V blocks with
-// TMA (128-byte swizzle) into a 4-stage ring; warps 0..3 each take 16 of the
-// 64 keys of every block (intra-CTA split over keys), run QK^T and PV with
-// m16n8k16 warp MMAs (tensor work is ~5% of the memory time here), keep an
-// online softmax in registers, and merge their partial results through
-// shared memory at the end.
+// K3 streams K/V: every (request, KV head) reads its assembled K/V once
+// (4 KiB per token at Hkv = 8, d = 128).  One CTA owns 16 packed query rows
+// (token * G + head_in_group) of one request and KV head, and one chunk of its
+// virtual block list; the CTAs launch KV-head-major, so requests that share
+// an artifact read its blocks from L2 after the first.  Warp 4 streams
+// 64-token K/V blocks with TMA (128-byte swizzle) into a 4-stage ring; warps
+// 0..3 each take 16 of the 64 keys of every block (intra-CTA split over
+// keys), run QK^T and PV with m16n8k16 warp MMAs (tensor work is ~5% of the
+// memory time here), keep an online softmax in registers, and merge their
+// partial results through shared memory at the end.
 #include <math.h>
 
 #include "kernels.h"
@@ -51,13 +52,27 @@ __global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ A
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int G = p.G;
-  const int cta = blockIdx.x;
-  const int req = find_req(p.work, cta);
-  int rel = cta - p.work.base[req];
+  // Launch order: KV head outermost, then request, split and row tile.  The
+  // CTAs resident at any one time read the blocks of one KV head (about an
+  // eighth of the pool), so requests that share an artifact find most of its
+  // blocks still in L2.  `cta` is the request-major index that numbers the
+  // split partials and the merge (base[r] + (split * Hkv + kvh) * row_tiles + rt).
+  const int per_head = p.work.n_cta / p.Hkv;
+  const int kvh = blockIdx.x / per_head;
+  const int in_head = blockIdx.x % per_head;
+  int req = 0;
+  {
+    int lo = 0, hi = p.work.n_req - 1;   // the per-head bases are base[r] / Hkv
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (p.work.base[mid] / p.Hkv <= in_head) lo = mid; else hi = mid - 1;
+    }
+    req = lo;
+  }
+  const int rel = in_head - p.work.base[req] / p.Hkv;
   const int rt = rel % p.work.row_tiles;
-  rel /= p.work.row_tiles;
-  const int kvh = rel % p.Hkv;
-  const int split = rel / p.Hkv;
+  const int split = rel / p.work.row_tiles;
+  const int cta = p.work.base[req] + (split * p.Hkv + kvh) * p.work.row_tiles + rt;
   const int nsplit = p.work.nsplit[req];
   const int boff = p.plan.blk_off[req];
   const int nab = p.plan.blk_off[req + 1] - boff;
