@@ -10,7 +10,8 @@
 // (token * G + head_in_group) of one request and KV head, and one chunk of its
 // virtual block list; the CTAs launch KV-head-major, so requests that share
 // an artifact read its blocks from L2 after the first.  Warp 4 streams
-// 64-token K/V blocks with TMA (128-byte swizzle) into a 4-stage ring; warps
+// 64-token K/V blocks with TMA (128-byte swizzle) into a 3-stage ring (two
+// CTAs share an SM, so one's prologue and merge overlap the other's loads); warps
 // 0..3 each take 16 of the 64 keys of every block (intra-CTA split over
 // keys), run QK^T and PV with m16n8k16 warp MMAs (tensor work is ~5% of the
 // memory time here), keep an online softmax in registers, and merge their
@@ -24,19 +25,19 @@ namespace att {
 template <int D>
 struct MmaLayout {
   static constexpr int NH = D / 64;
-  static constexpr int NS = 4;
+  static constexpr int NS = 3;
   static constexpr int BLK = kBlockTokens * 128;      // one 64-row x 128 B box
   static constexpr int STAGE = 2 * NH * BLK;          // K halves then V halves
   static constexpr int BAR_OFF = NS * STAGE;
   static constexpr int LIST_OFF = BAR_OFF + 256;
   static constexpr int MERGE_BYTES = 4 * 16 * (D + 2) * 4;   // per warp: O[16][D], m[16], l[16]
-  static constexpr int SMEM = LIST_OFF + kMaxChunkBlocks * 4 + 1024;
+  static constexpr int SMEM = LIST_OFF + kMmaMaxChunkBlocks * 4 + 1024;   // two CTAs per SM
   static_assert(MERGE_BYTES <= BAR_OFF, "merge area aliases the stage ring");
 };
 
 // kLayout: some request has online spans before artifacts (general visibility rule)
 template <int D, bool kLayout>
-__global__ void __launch_bounds__(160) attn_mma_kernel(const __grid_constant__ AttnParams p) {
+__global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant__ AttnParams p) {
   using L = MmaLayout<D>;
   grid_dep_wait();     // Q and the suffix K/V may come from the previous kernel
   constexpr int NT = D / 8;           // n8 tiles of the output

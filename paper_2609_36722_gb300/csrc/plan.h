@@ -29,6 +29,8 @@ constexpr int kTcTileRows = 128;  // rows per query tile (one MMA M)
 constexpr int kMmaRows = 16;
 // largest split chunk (virtual blocks) the kernels' shared-memory block list holds
 constexpr int kMaxChunkBlocks = 4096;
+// the warp-MMA kernel's list is shorter, so that two of its CTAs share an SM
+constexpr int kMmaMaxChunkBlocks = 1024;
 // most split-KV chunks of one (request, KV head, row tile) in the tcgen05 kernel
 constexpr int kMaxSplits = 32;
 
