@@ -94,6 +94,17 @@ def kv_bytes(wl) -> float:
     return float(sum((wl.t_art(r) + wl.S_kv) * 2 * g.n_kv_heads * g.head_dim * 2 for r in range(wl.n_req)))
 
 
+def kv_distinct_bytes(wl) -> float:
+    """The distinct K/V a step needs: every artifact the requests use, once, and
+    every request's own suffix rows.  Requests that share an artifact need its
+    bytes once, so a kernel that reads shared blocks once (or from L2) moves
+    fewer DRAM bytes than kv_bytes counts."""
+    g = wl.geom
+    used = {a for r in wl.requests for a in r}
+    tokens = sum(wl.art_lengths[a] for a in used) + wl.n_req * wl.S_kv
+    return float(tokens * 2 * g.n_kv_heads * g.head_dim * 2)
+
+
 def is_decode(wl) -> bool:
     return wl.S * wl.geom.group <= 16
 
@@ -421,7 +432,8 @@ def measure_core(bed, args, world, timer, with_clocks=False, local_rank=0):
                      "work_unit": "bytes (each request's assembled K and V read once)" if bed.decode
                                   else "FLOP (4 d Hq per visible query-key pair)",
                      "peak_source": f"{peaks['src']} ({'hbm_gbs' if bed.decode else 'bf16_tflops burst'})",
-                     "avg_launch_ms": round(attn_avg, 5)},
+                     "avg_launch_ms": round(attn_avg, 5),
+                     **(decode_read_fracs(wl, attn_avg, peak, load_traffic(bed.name)) if bed.decode else {})},
         "qproj": {"avg_call_ms": round(qp_avg, 5), "tflops": round(qp_tf, 3),
                   "frac_of_bf16_peak": round(qp_tf / peaks["bf16"], 4),
                   "bound_ms": round(qp_bound_ms, 5), "frac_of_bound": round(qp_bound_ms / qp_avg, 4)},
@@ -834,6 +846,17 @@ def run_ours(args, rank, world, local_rank):
     if errors:
         result["errors"] = errors
     return result, (1 if errors else 0)
+
+
+def decode_read_fracs(wl, attn_ms, peak_gbs, traffic):
+    """The decode roofline counted in the bytes the launch must move: the distinct
+    K/V (each shared artifact once) and, when an ncu capture of the current
+    kernel exists, the DRAM bytes it did move, each per second against the peak."""
+    d = kv_distinct_bytes(wl)
+    out = {"distinct_bytes": d, "distinct_frac": round(d / (attn_ms * 1e-3) / 1e9 / peak_gbs, 4)}
+    if traffic:
+        out["dram_frac"] = round(traffic / (attn_ms * 1e-3) / 1e9 / peak_gbs, 4)
+    return out
 
 
 def load_traffic(workload):

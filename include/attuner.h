@@ -380,6 +380,17 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
  *                               through distributed shared memory (global
  *                               memory where such clusters cannot be
  *                               co-resident on the device)
+ *   ATTUNER_OPT_SHARE_READS     shared artifact reads of the decode kernel
+ *                               (the warp-MMA kernel, at most 16 packed query
+ *                               rows per request): one CTA reads a chunk of an
+ *                               artifact for every request of a group of
+ *                               requests that use it, each request's partial
+ *                               results merged afterwards.  0 auto (where it
+ *                               saves 10 % or more of the block reads), 1 off,
+ *                               2 wherever it applies: plans without online
+ *                               spans whose keys were not rotated at assembly,
+ *                               at least two requests' rows per CTA, at most
+ *                               511 distinct artifacts in the plan
  *   ATTUNER_OPT_SYNC_CHECK      0 off, 1 every compute call reports the device
  *                               status itself (see below)
  *   ATTUNER_OPT_TEST_STUCK_WAIT see below */
@@ -389,6 +400,7 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
 #define ATTUNER_OPT_QPROJ_SPLIT_K  4
 #define ATTUNER_OPT_SPLIT_MERGE    5
 #define ATTUNER_OPT_QPROJ_ROWS     7
+#define ATTUNER_OPT_SHARE_READS    8
 /* Debug check: while non-zero, attuner_q_project, attuner_kv_project,
  * attuner_attend, attuner_attend_static_scratch and attuner_query_attend
  * synchronise their stream before returning and return the device status as

@@ -18,6 +18,7 @@ from .attuner import (  # noqa: F401
     OPT_SPLIT_MERGE,
     OPT_SYNC_CHECK,
     OPT_QPROJ_ROWS,
+    OPT_SHARE_READS,
     OPT_TEST_STUCK_WAIT,
     lib,
     load_library,

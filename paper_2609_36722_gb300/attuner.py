@@ -35,6 +35,7 @@ OPT_QPROJ_SPLIT_K = 4
 OPT_SPLIT_MERGE = 5
 OPT_SYNC_CHECK = 6
 OPT_QPROJ_ROWS = 7
+OPT_SHARE_READS = 8
 OPT_TEST_STUCK_WAIT = 1000
 
 BLOCK_TOKENS = 64

@@ -30,13 +30,53 @@ struct MmaLayout {
   static constexpr int STAGE = 2 * NH * BLK;          // K halves then V halves
   static constexpr int BAR_OFF = NS * STAGE;
   static constexpr int LIST_OFF = BAR_OFF + 256;
+  static constexpr int MEM_OFF = LIST_OFF + kMmaMaxChunkBlocks * 4;   // shared reads: [16][4] member table
   static constexpr int MERGE_BYTES = 4 * 16 * (D + 2) * 4;   // per warp: O[16][D], m[16], l[16]
-  static constexpr int SMEM = LIST_OFF + kMmaMaxChunkBlocks * 4 + 1024;   // two CTAs per SM
+  static constexpr int SMEM = MEM_OFF + 16 * 16 + 1024;   // two CTAs per SM
   static_assert(MERGE_BYTES <= BAR_OFF, "merge area aliases the stage ring");
 };
 
+// The merge of n partial results of one query row (K4): record k of the row
+// at part_lse[rec(k)] and part_o[rec(k) * D ...], in order k = 0 .. n - 1:
+// lse = log sum_k exp(lse_k),  O = sum_k exp(lse_k - lse) O_k.  The calling
+// thread writes its CPT = D / 8 columns from c0 of output row orow.
+template <int D, class Rec>
+ATT_DEV void merge_records(const AttnParams& p, int n, Rec rec, int c0, long long orow, int tid) {
+  constexpr int CPT = D / 8;
+  float Ms = -INFINITY;
+  for (int k = 0; k < n; ++k) Ms = fmaxf(Ms, __ldcg(p.part_lse + rec(k)));
+  float W = 0.f;
+  float acc[CPT];
+#pragma unroll
+  for (int c = 0; c < CPT; ++c) acc[c] = 0.f;
+  for (int k = 0; k < n; ++k) {
+    const long long at = rec(k);
+    const float ls = __ldcg(p.part_lse + at);
+    if (ls == -INFINITY) continue;
+    const float w = __expf(ls - Ms);
+    W += w;
+    const float* q = p.part_o + at * D + c0;
+#pragma unroll
+    for (int c = 0; c < CPT; c += 4) {
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(q + c));
+      acc[c] += w * v.x; acc[c + 1] += w * v.y; acc[c + 2] += w * v.z; acc[c + 3] += w * v.w;
+    }
+  }
+  const float invW = (W > 0.f) ? 1.f / W : 0.f;
+  uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D + c0);
+#pragma unroll
+  for (int c = 0; c < CPT; c += 8)
+    dst[c / 8] = make_uint4(pack_bf16(acc[c] * invW, acc[c + 1] * invW), pack_bf16(acc[c + 2] * invW, acc[c + 3] * invW),
+                            pack_bf16(acc[c + 4] * invW, acc[c + 5] * invW), pack_bf16(acc[c + 6] * invW, acc[c + 7] * invW));
+  if ((tid & 7) == 0 && p.lse_out) p.lse_out[orow] = (W > 0.f) ? Ms + logf(W) : -INFINITY;
+}
+
 // kLayout: some request has online spans before artifacts (general visibility rule)
-template <int D, bool kLayout>
+// kShare: the shared-read decomposition (WorkTable): a CTA reads one chunk of
+// an artifact for the requests of one group of its references, or one chunk
+// of a request's online rows, and every request's partials are merged by the
+// last CTA to finish one of them
+template <int D, bool kLayout, bool kShare>
 __global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant__ AttnParams p) {
   using L = MmaLayout<D>;
   grid_dep_wait();     // Q and the suffix K/V may come from the previous kernel
@@ -53,58 +93,125 @@ __global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant_
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int G = p.G;
-  // Launch order: KV head outermost, then request, split and row tile.  The
-  // CTAs resident at any one time read the blocks of one KV head (about an
-  // eighth of the pool), so requests that share an artifact find most of its
-  // blocks still in L2.  `cta` is the request-major index that numbers the
-  // split partials and the merge (base[r] + (split * Hkv + kvh) * row_tiles + rt).
-  const int per_head = p.work.n_cta / p.Hkv;
-  const int kvh = blockIdx.x / per_head;
-  const int in_head = blockIdx.x % per_head;
-  int req = 0;
-  {
-    int lo = 0, hi = p.work.n_req - 1;   // the per-head bases are base[r] / Hkv
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (p.work.base[mid] / p.Hkv <= in_head) lo = mid; else hi = mid - 1;
-    }
-    req = lo;
-  }
-  const int rel = in_head - p.work.base[req] / p.Hkv;
-  const int rt = rel % p.work.row_tiles;
-  const int split = rel / p.work.row_tiles;
-  const int cta = p.work.base[req] + (split * p.Hkv + kvh) * p.work.row_tiles + rt;
-  const int nsplit = p.work.nsplit[req];
-  const int boff = p.plan.blk_off[req];
-  const int nab = p.plan.blk_off[req + 1] - boff;
-  const int nsuf = (p.S_kv + kBlockTokens - 1) / kBlockTokens;   // chunks of online rows
-  const int row0 = rt * kMmaRows;
-  const int last_row = min(row0 + kMmaRows - 1, p.S * G - 1);
-  const int lim_last = (p.S_kv - p.S) + last_row / G;   // online row of the tile's last query
-  // The row tile reads its own list of slots: the artifact slots its last
-  // query sees (queries are in prompt order, so no query of the tile sees
-  // more), then the online chunks up to the one holding that query's key.
-  const int nart = kLayout ? art_slots_seen(p.plan, req, lim_last, nab) : nab;
-  const int last_vis = nart + lim_last / kBlockTokens;
-  int v_lo, v_hi;
-  kv_part_range(p.kv_part, nart, nsuf, v_lo, v_hi);
-  const int b0 = v_lo + split * p.work.chunk_blocks;
-  const int b1 = min(min(b0 + p.work.chunk_blocks, v_hi), last_vis + 1);
-  const int nblk = max(0, b1 - b0);
-
-  for (int i = threadIdx.x; i < nblk; i += blockDim.x) {
-    const int b = b0 + i;
-    int e;
-    if (b < nart) {
-      e = p.plan.blocks[boff + b];
-      if (e <= 0 || (e >> 7) >= p.plan.pool_blocks || (e & 127) < 1 || (e & 127) > kBlockTokens) {
-        set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
-        e = 0;
+  const int SG = p.S * G;                 // packed rows of one request
+  int* mem = reinterpret_cast<int*>(smem + L::MEM_OFF);   // shared reads: request, partial, partials, last
+  int kvh, req, row0, nblk, b0 = 0, boff = 0, nab = 0, cta = 0, nsplit = 1, rt = 0, n_mem = 1;
+  if constexpr (kShare) {
+    const int per_head = p.work.n_cta / p.Hkv;
+    kvh = blockIdx.x / per_head;
+    const int u = blockIdx.x % per_head;
+    const int C = p.work.chunk_blocks;
+    row0 = 0;
+    int chunk, src = 0, m_beg = 0;
+    const bool art = u < p.work.art_units;
+    if (art) {
+      int lo = 0, hi = p.work.n_dist - 1;   // distinct artifact d: nsplit[d] <= u < nsplit[d + 1]
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.work.nsplit[mid] <= u) lo = mid; else hi = mid - 1;
       }
+      const int r_beg = p.plan.dist_off[lo], r_end = p.plan.dist_off[lo + 1];
+      const int nb = p.plan.ref_nblk[p.plan.dist_refs[r_beg]];
+      const int nch = (nb + C - 1) / C;
+      const int local = u - p.work.nsplit[lo];
+      chunk = local % nch;
+      m_beg = r_beg + (local / nch) * p.work.members;
+      n_mem = min(p.work.members, r_end - m_beg);
+      const int i0 = p.plan.dist_refs[m_beg];
+      req = p.plan.ref_req[i0];
+      src = p.plan.blk_off[req] + p.plan.ref_slot[i0] + chunk * C;
+      nblk = min(C, nb - chunk * C);
     } else {
-      e = online_entry((b - nart) * kBlockTokens, kBlockTokens);
+      const int v = u - p.work.art_units;
+      req = v / p.work.suf_chunks;
+      chunk = v % p.work.suf_chunks;
+      const int nsuf = (p.S_kv + kBlockTokens - 1) / kBlockTokens;
+      nblk = min(C, nsuf - chunk * C);
     }
-    list[i] = e;
+    for (int i = threadIdx.x; i < nblk; i += blockDim.x) {
+      int e;
+      if (art) {
+        e = p.plan.blocks[src + i];
+        if (e <= 0 || (e >> 7) >= p.plan.pool_blocks || (e & 127) < 1 || (e & 127) > kBlockTokens) {
+          set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
+          e = 0;
+        }
+      } else {
+        e = online_entry((chunk * C + i) * kBlockTokens, kBlockTokens);
+      }
+      list[i] = e;
+    }
+    if (threadIdx.x < n_mem) {
+      // the member's request, the index of this chunk among the request's
+      // partials (its references' chunks in prompt order, then the suffix
+      // chunks) and their count
+      const int ir = art ? p.plan.dist_refs[m_beg + threadIdx.x] : -1;
+      const int r = art ? p.plan.ref_req[ir] : req;
+      int k = 0, P = 0;
+      for (int i = p.plan.req_art_off[r]; i < p.plan.req_art_off[r + 1]; ++i) {
+        const int n = (p.plan.ref_nblk[i] + C - 1) / C;
+        if (i < ir) k += n;
+        P += n;
+      }
+      mem[4 * threadIdx.x + 0] = r;
+      mem[4 * threadIdx.x + 1] = art ? k + chunk : P + chunk;
+      mem[4 * threadIdx.x + 2] = P + p.work.suf_chunks;
+      mem[4 * threadIdx.x + 3] = 0;
+    }
+  } else {
+    // Launch order: KV head outermost, then request, split and row tile.  The
+    // CTAs resident at any one time read the blocks of one KV head (about an
+    // eighth of the pool), so requests that share an artifact find most of its
+    // blocks still in L2.  `cta` is the request-major index that numbers the
+    // split partials and the merge (base[r] + (split * Hkv + kvh) * row_tiles + rt).
+    const int per_head = p.work.n_cta / p.Hkv;
+    kvh = blockIdx.x / per_head;
+    const int in_head = blockIdx.x % per_head;
+    req = 0;
+    {
+      int lo = 0, hi = p.work.n_req - 1;   // the per-head bases are base[r] / Hkv
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.work.base[mid] / p.Hkv <= in_head) lo = mid; else hi = mid - 1;
+      }
+      req = lo;
+    }
+    const int rel = in_head - p.work.base[req] / p.Hkv;
+    rt = rel % p.work.row_tiles;
+    const int split = rel / p.work.row_tiles;
+    cta = p.work.base[req] + (split * p.Hkv + kvh) * p.work.row_tiles + rt;
+    nsplit = p.work.nsplit[req];
+    boff = p.plan.blk_off[req];
+    nab = p.plan.blk_off[req + 1] - boff;
+    const int nsuf = (p.S_kv + kBlockTokens - 1) / kBlockTokens;   // chunks of online rows
+    row0 = rt * kMmaRows;
+    const int last_row = min(row0 + kMmaRows - 1, SG - 1);
+    const int lim_last = (p.S_kv - p.S) + last_row / G;   // online row of the tile's last query
+    // The row tile reads its own list of slots: the artifact slots its last
+    // query sees (queries are in prompt order, so no query of the tile sees
+    // more), then the online chunks up to the one holding that query's key.
+    const int nart = kLayout ? art_slots_seen(p.plan, req, lim_last, nab) : nab;
+    const int last_vis = nart + lim_last / kBlockTokens;
+    int v_lo, v_hi;
+    kv_part_range(p.kv_part, nart, nsuf, v_lo, v_hi);
+    b0 = v_lo + split * p.work.chunk_blocks;
+    const int b1 = min(min(b0 + p.work.chunk_blocks, v_hi), last_vis + 1);
+    nblk = max(0, b1 - b0);
+
+    for (int i = threadIdx.x; i < nblk; i += blockDim.x) {
+      const int b = b0 + i;
+      int e;
+      if (b < nart) {
+        e = p.plan.blocks[boff + b];
+        if (e <= 0 || (e >> 7) >= p.plan.pool_blocks || (e & 127) < 1 || (e & 127) > kBlockTokens) {
+          set_status(p.status, ATTUNER_ERR_DEVICE_CHECK);
+          e = 0;
+        }
+      } else {
+        e = online_entry((b - nart) * kBlockTokens, kBlockTokens);
+      }
+      list[i] = e;
+    }
   }
   if (threadIdx.x == 0) {
     for (int i = 0; i < L::NS; ++i) {
@@ -165,8 +272,14 @@ __global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant_
 #pragma unroll
   for (int hr = 0; hr < 2; ++hr) {
     const int pr = row0 + g + 8 * hr;
-    tok_r[hr] = pr / G;
-    qrow[hr] = (tok_r[hr] < p.S) ? (((long long)req * p.S + tok_r[hr]) * p.Hq + kvh * G + pr % G) : -1;
+    if constexpr (kShare) {   // member pr / SG, its packed row pr % SG
+      const int mi = pr / SG, wr = pr % SG;
+      tok_r[hr] = wr / G;
+      qrow[hr] = (mi < n_mem) ? (((long long)mem[4 * mi] * p.S + tok_r[hr]) * p.Hq + kvh * G + wr % G) : -1;
+    } else {
+      tok_r[hr] = pr / G;
+      qrow[hr] = (tok_r[hr] < p.S) ? (((long long)req * p.S + tok_r[hr]) * p.Hq + kvh * G + pr % G) : -1;
+    }
   }
 #pragma unroll
   for (int ks = 0; ks < KS; ++ks) {
@@ -337,6 +450,39 @@ __global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant_
     for (int w = 0; w < 4; ++w) a += wt[w] * mb[(w * 16 + row) * (D + 2) + c0 + c];
     acc[c] = a * inv;
   }
+  // Split-KV chunks (K4): publish this chunk's normalised O and log-sum-exp;
+  // the last CTA to finish a chunk of a (request, KV head, row tile) merges
+  // all its chunks, its own included, in a fixed order (the same arithmetic
+  // whichever CTA is last):  lse = log sum_s exp(lse_s),  O = sum_s exp(lse_s - lse) O_s.
+  // Every consumer thread passes the two barriers, rows past the last token too.
+  volatile int* last_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 8 * (2 * L::NS + 1) + 4);
+  if constexpr (kShare) {
+    // this row's member: its request's partial record k of P (records of
+    // request r: base[r] + k, each [Hkv][16 rows])
+    const int mi = row / SG, wr = row % SG;
+    const bool mine = mi < n_mem;
+    const int r = mine ? mem[4 * mi] : 0;
+    const long long rec0 = (long long)p.work.base[r] * p.Hkv + kvh;   // record k at rec0 + k * Hkv
+    if (mine) {
+      const long long at = (rec0 + (long long)mem[4 * mi + 1] * p.Hkv) * kMmaRows + wr;
+      float* po = p.part_o + at * D + c0;
+#pragma unroll
+      for (int c = 0; c < CPT; c += 4)
+        *reinterpret_cast<float4*>(po + c) = make_float4(acc[c], acc[c + 1], acc[c + 2], acc[c + 3]);
+      if ((tid & 7) == 0) p.part_lse[at] = lse;
+    }
+    __threadfence();
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (tid < n_mem)
+      mem[4 * tid + 3] = (atomicAdd(&p.unit_cnt[mem[4 * tid] * p.Hkv + kvh], 1) == mem[4 * tid + 2] - 1) ? 1 : 0;
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (!mine || mem[4 * mi + 3] == 0) return;
+    __threadfence();
+    const long long orow_m = ((long long)r * p.S + wr / G) * p.Hq + kvh * G + wr % G;
+    merge_records<D>(p, mem[4 * mi + 2], [&](int k) { return (rec0 + (long long)k * p.Hkv) * kMmaRows + wr; }, c0,
+                     orow_m, tid);
+    return;
+  }
   if (nsplit <= 1) {
     if (!row_ok) return;
     uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D + c0);
@@ -347,17 +493,11 @@ __global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant_
     if ((tid & 7) == 0 && p.lse_out) p.lse_out[orow] = lse;
     return;
   }
-  // Split-KV chunks (K4): publish this chunk's normalised O and log-sum-exp;
-  // the last CTA of the (request, KV head, row tile) to arrive merges every
-  // chunk, its own included, in split order (the same arithmetic whichever
-  // CTA is last):  lse = log sum_s exp(lse_s),  O = sum_s exp(lse_s - lse) O_s.
-  // Every consumer thread passes the two barriers, rows past the last token too.
   float* po = p.part_o + ((long long)cta * kMmaRows + row) * D + c0;
 #pragma unroll
   for (int c = 0; c < CPT; c += 4) *reinterpret_cast<float4*>(po + c) = make_float4(acc[c], acc[c + 1], acc[c + 2], acc[c + 3]);
   if ((tid & 7) == 0) p.part_lse[(long long)cta * kMmaRows + row] = lse;
   __threadfence();
-  volatile int* last_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 8 * (2 * L::NS + 1) + 4);
   asm volatile("bar.sync 1, 128;" ::: "memory");
   if (tid == 0) {
     const int unit = (req * p.Hkv + kvh) * p.work.row_tiles + rt;
@@ -368,45 +508,28 @@ __global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant_
   __threadfence();
   const long long c_0 = p.work.base[req] + (long long)kvh * p.work.row_tiles + rt;   // CTA of split 0
   const long long c_stride = (long long)p.Hkv * p.work.row_tiles;
-  float Ms = -INFINITY;
-  for (int sp = 0; sp < nsplit; ++sp) Ms = fmaxf(Ms, __ldcg(p.part_lse + (c_0 + sp * c_stride) * kMmaRows + row));
-  float W = 0.f;
-#pragma unroll
-  for (int c = 0; c < CPT; ++c) acc[c] = 0.f;
-  for (int sp = 0; sp < nsplit; ++sp) {
-    const long long cs = c_0 + sp * c_stride;
-    const float ls = __ldcg(p.part_lse + cs * kMmaRows + row);
-    if (ls == -INFINITY) continue;
-    const float w = __expf(ls - Ms);
-    W += w;
-    const float* q = p.part_o + (cs * kMmaRows + row) * D + c0;
-#pragma unroll
-    for (int c = 0; c < CPT; c += 4) {
-      const float4 v = __ldcg(reinterpret_cast<const float4*>(q + c));
-      acc[c] += w * v.x; acc[c + 1] += w * v.y; acc[c + 2] += w * v.z; acc[c + 3] += w * v.w;
-    }
-  }
-  const float invW = (W > 0.f) ? 1.f / W : 0.f;
-  uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D + c0);
-#pragma unroll
-  for (int c = 0; c < CPT; c += 8)
-    dst[c / 8] = make_uint4(pack_bf16(acc[c] * invW, acc[c + 1] * invW), pack_bf16(acc[c + 2] * invW, acc[c + 3] * invW),
-                            pack_bf16(acc[c + 4] * invW, acc[c + 5] * invW), pack_bf16(acc[c + 6] * invW, acc[c + 7] * invW));
-  if ((tid & 7) == 0 && p.lse_out) p.lse_out[orow] = (W > 0.f) ? Ms + logf(W) : -INFINITY;
+  merge_records<D>(p, nsplit, [&](int sp) { return (c_0 + sp * c_stride) * kMmaRows + row; }, c0, orow, tid);
 }
 
-template <int D, bool kLayout>
+template <int D, bool kLayout, bool kShare>
 static cudaError_t launch_attn_mma_t(const AttnParams& p, cudaStream_t st) {
   using L = MmaLayout<D>;
-  cudaError_t e = cudaFuncSetAttribute(attn_mma_kernel<D, kLayout>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
+  cudaError_t e =
+      cudaFuncSetAttribute(attn_mma_kernel<D, kLayout, kShare>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
-  return launch_pdl(attn_mma_kernel<D, kLayout>, dim3(p.work.n_cta), dim3(160), (size_t)L::SMEM, st, 0, p);
+  return launch_pdl(attn_mma_kernel<D, kLayout, kShare>, dim3(p.work.n_cta), dim3(160), (size_t)L::SMEM, st, 0, p);
+}
+
+template <int D>
+static cudaError_t launch_attn_mma_d(const AttnParams& p, cudaStream_t st) {
+  // shared reads are planned only for plans without online spans
+  if (p.work.share) return p.plan.has_spans ? cudaErrorInvalidValue : launch_attn_mma_t<D, false, true>(p, st);
+  return p.plan.has_spans ? launch_attn_mma_t<D, true, false>(p, st) : launch_attn_mma_t<D, false, false>(p, st);
 }
 
 cudaError_t launch_attn_mma(const AttnParams& p, int D, cudaStream_t st) {
-  const bool layout = p.plan.has_spans != 0;
-  if (D == 128) return layout ? launch_attn_mma_t<128, true>(p, st) : launch_attn_mma_t<128, false>(p, st);
-  if (D == 64) return layout ? launch_attn_mma_t<64, true>(p, st) : launch_attn_mma_t<64, false>(p, st);
+  if (D == 128) return launch_attn_mma_d<128>(p, st);
+  if (D == 64) return launch_attn_mma_d<64>(p, st);
   return cudaErrorInvalidValue;
 }
 

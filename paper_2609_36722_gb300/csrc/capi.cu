@@ -304,8 +304,12 @@ static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const 
   p->pool_gen = ctx->pool_gen;
   attuner_status s = set_device(ctx);
   if (s != ATTUNER_OK) { delete p; return s; }
-  // the device image: blk_off | blocks | t_art | o_rows | span_off | (16-byte aligned) spans
-  const size_t head = p->blk_off.size() + p->blocks.size() + p->t_art.size() + p->o_rows.size() + p->span_off.size();
+  // the device image: blk_off | blocks | t_art | o_rows | span_off | req_art_off | ref_req |
+  // ref_slot | ref_nblk | dist_off | dist_refs | (16-byte aligned) spans
+  const std::vector<int32_t>* parts[] = {&p->blk_off, &p->blocks, &p->t_art, &p->o_rows, &p->span_off, &p->req_art_off,
+                                         &p->ref_req, &p->ref_slot, &p->ref_nblk, &p->dist_off, &p->dist_refs};
+  size_t head = 0;
+  for (const std::vector<int32_t>* v : parts) head += v->size();
   p->spans_at = (head + 3) & ~size_t(3);   // int4 spans start 16-byte aligned
   const size_t n_words = std::max<size_t>(p->spans_at + p->spans.size(), 1);
   const size_t bytes = n_words * sizeof(int32_t);
@@ -325,7 +329,7 @@ static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const 
   {
     int32_t* h = static_cast<int32_t*>(ctx->staging);
     size_t at = 0;
-    for (const std::vector<int32_t>* v : {&p->blk_off, &p->blocks, &p->t_art, &p->o_rows, &p->span_off}) {
+    for (const std::vector<int32_t>* v : parts) {
       if (!v->empty()) std::memcpy(h + at, v->data(), v->size() * sizeof(int32_t));
       at += v->size();
     }
@@ -493,6 +497,12 @@ PlanDev att::plan_dev(const attuner_plan* p) {
   d.t_art = p->d_buf + p->blk_off.size() + p->blocks.size();
   d.o_rows = d.t_art + p->t_art.size();
   d.span_off = d.o_rows + p->o_rows.size();
+  d.req_art_off = d.span_off + p->span_off.size();
+  d.ref_req = d.req_art_off + p->req_art_off.size();
+  d.ref_slot = d.ref_req + p->ref_req.size();
+  d.ref_nblk = d.ref_slot + p->ref_slot.size();
+  d.dist_off = d.ref_nblk + p->ref_nblk.size();
+  d.dist_refs = d.dist_off + p->dist_off.size();
   d.spans = reinterpret_cast<const int4*>(p->d_buf + p->spans_at);
   d.pool_blocks = p->pool_blocks;
   d.has_spans = p->max_o_rows > 0 ? 1 : 0;
@@ -696,6 +706,8 @@ attuner_status att::make_work(const attuner_ctx* ctx, const attuner_plan* plan, 
   pol.num_sms = ctx->num_sms;
   pol.opt_split = ctx->opt_split;
   pol.opt_merge = ctx->opt_merge;
+  pol.opt_share = ctx->opt_share;
+  pol.k_by_slot = plan->k_rot != nullptr ? 1 : 0;
   for (int i = 0; i < 9; ++i) pol.tc_clusters[i] = ctx->tc_clusters[i];
   std::string err;
   const attuner_status s = split_work(pol, *plan, S, S_kv, tc, w, err);
@@ -723,13 +735,15 @@ attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, co
   if ((e = make_work(ctx, plan, S, S_kv, tc, ap.work, var.kv_part)) != ATTUNER_OK) return e;
   const WorkTable& w = ap.work;
   if (w.n_cta == 0) return ATTUNER_OK;   // no request has a slot of this part
-  bool need_combine = false;   // split partial results in global memory
-  for (int r = 0; r < plan->n_req; ++r) need_combine |= (w.nsplit[r] > 1);
+  bool need_combine = w.share != 0;   // split partial results in global memory
+  if (!w.share)
+    for (int r = 0; r < plan->n_req; ++r) need_combine |= (w.nsplit[r] > 1);
   if (w.cluster > 0) need_combine = false;
-  // partial O and LSE of every split CTA and one arrival counter per
-  // (request, KV head, row tile), zeroed below: the last CTA of a row tile
-  // to arrive merges its chunks, in either kernel
-  const size_t pb = need_combine ? (size_t)w.n_cta * rows * (D + 1) * 4 : 0;
+  // partial O and LSE of every split CTA (shared reads: of every partial
+  // record) and one arrival counter per (request, KV head, row tile), zeroed
+  // below: the last CTA of a row tile to arrive merges its chunks, in either kernel
+  const size_t records = w.share ? (size_t)w.n_part * Hkv : (size_t)w.n_cta;
+  const size_t pb = need_combine ? records * rows * (D + 1) * 4 : 0;
   const size_t units = (size_t)plan->n_req * Hkv * w.row_tiles;
   const size_t part_bytes = pb + (need_combine ? units * 4 : 0);
   if (fixed && part_bytes > fixed->cap)
@@ -785,7 +799,7 @@ attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, co
       return fail(ATTUNER_ERR_OOM, "split-KV scratch allocation failed");
     }
     ap.part_o = static_cast<float*>(part);
-    ap.part_lse = static_cast<float*>(part) + (size_t)w.n_cta * rows * D;
+    ap.part_lse = static_cast<float*>(part) + records * rows * D;
     ap.unit_cnt = reinterpret_cast<int*>(static_cast<char*>(part) + pb);
     ce = cudaMemsetAsync(ap.unit_cnt, 0, units * 4, st);
   }
@@ -1047,6 +1061,10 @@ extern "C" attuner_status attuner_set_option(attuner_ctx* ctx, int32_t option, i
     case ATTUNER_OPT_SPLIT_MERGE:
       CHECK_ARG(value >= 0 && value <= 2, "split merge must be 0, 1 or 2");
       ctx->opt_merge = (int)value;
+      return ATTUNER_OK;
+    case ATTUNER_OPT_SHARE_READS:
+      CHECK_ARG(value >= 0 && value <= 2, "shared reads must be 0, 1 or 2");
+      ctx->opt_share = (int)value;
       return ATTUNER_OK;
     case ATTUNER_OPT_SYNC_CHECK:
       ctx->opt_sync_check = value ? 1 : 0;

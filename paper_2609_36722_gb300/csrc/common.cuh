@@ -33,6 +33,13 @@ struct PlanDev {
   const int32_t* o_rows;    // [n_req] online rows in the plan's explicit spans
   const int32_t* span_off;  // [n_req + 1] CSR offsets into spans
   const int4* spans;        // explicit online spans: (online row0, rows, artifact slots before, artifact tokens before)
+  // artifact references and their grouping by artifact (PlanTables)
+  const int32_t* req_art_off;   // [n_req + 1] CSR offsets into the references
+  const int32_t* ref_req;
+  const int32_t* ref_slot;
+  const int32_t* ref_nblk;
+  const int32_t* dist_off;      // [n_dist + 1]
+  const int32_t* dist_refs;
   int32_t pool_blocks;      // capacity, for bounds checks
   int32_t has_spans;        // 0: no request has explicit online spans (o_rows all 0; no loads needed)
 };

@@ -41,6 +41,7 @@ struct attuner_ctx {
   int opt_qproj_split = 0;   // 0: the projection's shape from its cost model
   int opt_qproj_rows = 0;
   int opt_merge = 0;
+  int opt_share = 0;          // shared artifact reads of the warp-MMA kernel: 0 auto, 1 off, 2 on
   int opt_sync_check = 0;
   int tc_clusters[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};   // co-resident clusters of n tcgen05 CTAs
   long long wait_limit = 1ll << 32;

@@ -33,6 +33,9 @@ constexpr int kMaxChunkBlocks = 4096;
 constexpr int kMmaMaxChunkBlocks = 1024;
 // most split-KV chunks of one (request, KV head, row tile) in the tcgen05 kernel
 constexpr int kMaxSplits = 32;
+// most distinct artifacts of a launch whose reads are shared (WorkTable::nsplit
+// holds one unit offset per distinct artifact and the total)
+constexpr int kMaxShareArts = kMaxReq - 1;
 
 // ---------------------------------------------------------------------------
 // The Q-projection kernel's shared-memory geometry (qproj.cuh), which the
@@ -77,6 +80,20 @@ QpShape choose_qproj_shape(const QpPolicy& pol, int heads, int M, int n_lora);
 // suffix chunks.  Each CTA owns one (request, kv head, row tile) and a
 // contiguous range of virtual blocks (one split-KV chunk).
 // CTA index = base[req] + (split * n_kv_heads + kv_head) * row_tiles + row_tile
+//
+// Shared reads (warp-MMA kernel, share = 1): when several requests use the
+// same artifact, one CTA reads a chunk of it for up to `members` requests
+// (members x S x G <= 16 packed rows) instead of each request reading it on
+// its own.  Work units per KV head: first the artifact units - distinct
+// artifact d (the plan's dist_* tables) in chunks of chunk_blocks of its
+// blocks, times groups of `members` of its references - numbered from
+// nsplit[d] (nsplit[n_dist] = art_units), then suffix units: request r's
+// chunks of online rows, art_units + r * suf_chunks + chunk.  CTA index =
+// kv_head * (n_cta / n_kv_heads) + unit.  Every (reference, chunk) and every
+// suffix chunk leaves a partial result of its request; request r's partials
+// are records base[r] .. base[r] + P_r - 1 (the references' chunks in prompt
+// order, then the suffix chunks), n_part in all per KV head, and the last
+// CTA to finish one of them merges the request's P_r partials in that order.
 // ---------------------------------------------------------------------------
 struct WorkTable {
   int32_t n_req;
@@ -90,6 +107,13 @@ struct WorkTable {
   int32_t cluster;
   int32_t base[kMaxReq];
   int32_t nsplit[kMaxReq];
+  // shared reads (see above); share = 0 for the per-request decomposition
+  int32_t share;
+  int32_t members;        // requests per CTA
+  int32_t n_dist;         // distinct artifacts
+  int32_t art_units;      // artifact units per KV head
+  int32_t suf_chunks;     // suffix units of each request
+  int32_t n_part;         // partial records per KV head
 };
 
 // A registered artifact: ceil(L/64) consecutive pool blocks from first_block
@@ -119,6 +143,14 @@ struct PlanTables {
   std::vector<int32_t> span_off;      // CSR over spans
   std::vector<int32_t> spans;         // 4 per span: online row0, rows, artifact slots before, artifact tokens before
   int32_t max_o_rows = 0;
+  // artifact references (one per art_ids entry, CSR by req_art_off): the
+  // request, the slot of its first block in the request's slot list and its
+  // block count; and the references of each distinct artifact id (ascending
+  // id, references in plan order within one id), CSR by dist_off
+  std::vector<int32_t> ref_req, ref_slot, ref_nblk;
+  std::vector<int32_t> dist_off;      // [n_dist + 1]
+  std::vector<int32_t> dist_refs;
+  int n_dist() const { return dist_off.empty() ? 0 : (int)dist_off.size() - 1; }
 };
 
 // Fills `t` from the request lists (items[offs[r] .. offs[r+1]) of request r)
@@ -144,6 +176,12 @@ struct SplitPolicy {
   // artifact slots only, 2 the chunks of the online rows only (for a plan
   // without online spans: the suffix)
   int32_t kv_part = 0;
+  // shared reads of the warp-MMA kernel: 0 where they save 10 % or more of
+  // the block reads, 1 never, 2 wherever they apply (a plan without online
+  // spans whose keys are read from the pool, every slot, 2 or more requests'
+  // rows per CTA)
+  int32_t opt_share = 0;
+  int32_t k_by_slot = 0;      // keys rotated at assembly: reads cannot be shared
 };
 
 // The slots [lo, hi) of a request that a launch reads, out of its nab artifact

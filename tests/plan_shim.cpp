@@ -118,3 +118,46 @@ extern "C" void shim_qproj_shape(const int32_t* pol, int32_t heads, int32_t M, i
 extern "C" int shim_qproj_supported(int32_t D, int32_t mr, int32_t ks, int32_t n_lora) {
   return att::qproj_shape_supported(D, mr, ks, n_lora) ? 1 : 0;
 }
+
+// Shared reads: the plan of (first, L, items, offs) and the split-KV work of
+// one warp-MMA launch over it.  pol = n_q_heads, n_kv_heads, num_sms,
+// opt_split, opt_share, k_by_slot, kv_part.  out (capacity cap) = n_cta,
+// chunk_blocks, share, members, n_dist, art_units, suf_chunks, n_part,
+// base[n_req] | nsplit[n_dist + 1] | ref_req | ref_slot | ref_nblk |
+// dist_off[n_dist + 1] | dist_refs; lens = n_refs, n_dist.
+extern "C" int shim_share(const int32_t* pol, const int32_t* first, const int32_t* L, int32_t n_arts,
+                          const int32_t* items, const int32_t* offs, int32_t n_req, int32_t S, int32_t S_kv,
+                          int32_t* out, int64_t cap, int64_t* lens) {
+  std::vector<att::Artifact> arts;
+  for (int i = 0; i < n_arts; ++i)
+    arts.push_back(att::Artifact{first[i], L[i], (L[i] + att::kBlockTokens - 1) / att::kBlockTokens});
+  att::PlanTables t;
+  attuner_status s = att::build_plan_tables(arts, items, offs, n_req, false, t, g_err);
+  if (s != ATTUNER_OK) return s;
+  att::SplitPolicy p;
+  p.n_q_heads = pol[0];
+  p.n_kv_heads = pol[1];
+  p.num_sms = pol[2];
+  p.opt_split = pol[3];
+  p.opt_merge = 0;
+  p.opt_share = pol[4];
+  p.k_by_slot = pol[5];
+  p.kv_part = pol[6];
+  for (int i = 0; i < 9; ++i) p.tc_clusters[i] = 0;
+  att::WorkTable w;
+  s = att::split_work(p, t, S, S_kv, false, w, g_err);
+  if (s != ATTUNER_OK) return s;
+  std::vector<int32_t> h = {w.n_cta, w.chunk_blocks, w.share, w.members, w.n_dist, w.art_units, w.suf_chunks, w.n_part};
+  h.insert(h.end(), w.base, w.base + n_req);
+  if (w.share) h.insert(h.end(), w.nsplit, w.nsplit + w.n_dist + 1);
+  for (const auto* v : {&t.ref_req, &t.ref_slot, &t.ref_nblk, &t.dist_off, &t.dist_refs})
+    h.insert(h.end(), v->begin(), v->end());
+  if ((int64_t)h.size() > cap) {
+    g_err = "output capacity too small";
+    return ATTUNER_ERR_INVALID_ARG;
+  }
+  memcpy(out, h.data(), h.size() * sizeof(int32_t));
+  lens[0] = (int64_t)t.ref_req.size();
+  lens[1] = t.n_dist();
+  return ATTUNER_OK;
+}

@@ -50,6 +50,8 @@ def test_work_of_multi_request_decode_and_prefill_shapes():
         toks = sum(sum(lengths[a] for a in r) + S_kv for r in reqs)
         assert bench.kv_bytes(wl) == toks * 2 * 2 * 64 * 2
         assert bench.is_decode(wl) == (S * g.group <= 16)
+        # distinct K/V: artifacts 0, 1, 2, 3 once each (2 and 3 are used twice), and the suffixes
+        assert bench.kv_distinct_bytes(wl) == (70 + 5 + 130 + 64 + 4 * S_kv) * 2 * 2 * 64 * 2
 
 
 def test_qproj_flops_counts_base_and_low_rank_products():

@@ -1,0 +1,85 @@
+"""Shared artifact reads of the decode kernel against the fp64 oracle.
+
+When several requests of one call use the same artifact, the warp-MMA kernel
+can read each chunk of it once for a group of those requests (up to 16 packed
+query rows per CTA) and merge every request's partial results afterwards by
+their log-sum-exp (the split-KV identity of the attention over the assembled
+keys).  These cases force the mode on and off on plans with repeated
+artifacts (across requests and within one request), requests without
+artifacts, chunked artifacts and online chunks, every group size and both
+head sizes, and compare each with the oracle.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gen import Geometry, make_custom
+from helpers import compare, load_context, run_path
+
+pytestmark = pytest.mark.gpu
+
+DEV = torch.device("cuda", 0) if torch.cuda.is_available() else None
+
+LENGTHS = [300, 77, 640, 64, 1, 129, 1000]
+REQS = [[2, 0], [1], [3, 1, 0, 2], [], [6, 2, 2], [5, 4, 6, 0], [0, 2, 6], [4]]
+
+
+def _reference(wl):
+    outs, lses = [], []
+    for r in range(wl.n_req):
+        o, l = oracle.workload_reference(wl, r)
+        outs.append(o)
+        lses.append(l)
+    return np.stack(outs), np.stack(lses)
+
+
+def _np(t):
+    return t.double().cpu().numpy()
+
+
+def _case(G, D, S, S_kv, seed):
+    geom = Geometry(hidden=256, n_q_heads=2 * G, n_kv_heads=2, head_dim=D, rank=8)
+    return make_custom("share", geom, seed, LENGTHS, REQS, S, S_kv, device=DEV)
+
+
+@pytest.mark.parametrize("G,D,S", [(1, 128, 1), (2, 128, 1), (4, 128, 1), (8, 128, 1), (4, 64, 1), (4, 128, 2),
+                                   (2, 64, 4)])
+@pytest.mark.parametrize("share,split", [(1, 0), (2, 0), (2, 3), (2, 16)])
+def test_shared_reads_match_oracle(G, D, S, share, split):
+    import paper_2609_36722_gb300 as pkg
+    wl = _case(G, D, S, 200 + S, seed=31 + G + D + S)
+    o_ref, lse_ref = _reference(wl)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, 2)
+    ctx.set_option(pkg.OPT_SHARE_READS, share)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, split)
+    out, lse = run_path(ctx, plan, wl)
+    compare(_np(out), o_ref, _np(lse), lse_ref, label=f"share={share} split={split} G={G} D={D} S={S}")
+
+
+def test_shared_reads_are_deterministic():
+    import paper_2609_36722_gb300 as pkg
+    wl = _case(4, 128, 1, 129, seed=3)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_SHARE_READS, 2)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, 4)
+    o1, l1 = run_path(ctx, plan, wl)
+    o2, l2 = run_path(ctx, plan, wl)
+    assert torch.equal(o1.view(torch.int16), o2.view(torch.int16))
+    assert torch.equal(l1, l2)
+
+
+def test_shared_and_per_request_reads_agree():
+    # the two decompositions merge the same keys in different chunks: equal up
+    # to the rounding of the merge (bf16 outputs)
+    import paper_2609_36722_gb300 as pkg
+    wl = _case(4, 128, 1, 129, seed=5)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_SHARE_READS, 1)
+    o1, l1 = run_path(ctx, plan, wl)
+    ctx.set_option(pkg.OPT_SHARE_READS, 2)
+    o2, l2 = run_path(ctx, plan, wl)
+    assert (o1.float() - o2.float()).abs().max().item() <= 1.6e-2
+    assert (l1 - l2).abs().max().item() <= 1e-4

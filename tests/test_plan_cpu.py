@@ -466,3 +466,163 @@ def test_qproj_shape_options_and_limits(shim):
     for D in (64, 128):
         assert qp_shape(shim, D, 64, 8, 100, 16)[1] == 1
     assert qp_shape(shim, 64, 512, 4, 300, 8, rows=128, split=8) == (0, 0)
+
+
+# ---------------------------------------------------------------------------
+# shared reads of the decode kernel
+# ---------------------------------------------------------------------------
+def share_plan(shim, lengths, requests, S, S_kv, n_q=32, n_kv=8, num_sms=152, opt_split=0, opt_share=0,
+               k_by_slot=0, kv_part=0):
+    firsts = bump_firsts(lengths)
+    n_req = len(requests)
+    items = [it for r in requests for it in r]
+    offs = np.cumsum([0] + [len(r) for r in requests])
+    fa, fp = _i32(firsts)
+    la, lp = _i32(lengths)
+    ia, ip = _i32(items if items else [0])
+    oa, op = _i32(offs)
+    pol = _i32([n_q, n_kv, num_sms, opt_split, opt_share, k_by_slot, kv_part])
+    cap = 1 << 20
+    out = np.zeros(cap, np.int32)
+    lens = np.zeros(2, np.int64)
+    st = shim.shim_share(pol[1], fp, lp, len(lengths), ip, op, n_req, S, S_kv, out.ctypes.data_as(I32P),
+                         ctypes.c_int64(cap), lens.ctypes.data_as(I64P))
+    assert st == OK, shim.shim_last_error()
+    n_refs, n_dist = int(lens[0]), int(lens[1])
+    keys = ["n_cta", "chunk", "share", "members", "n_dist", "art_units", "suf_chunks", "n_part"]
+    w = {k: int(out[i]) for i, k in enumerate(keys)}
+    at = len(keys)
+    w["base"] = out[at:at + n_req].tolist()
+    at += n_req
+    if w["share"]:
+        w["nsplit"] = out[at:at + n_dist + 1].tolist()
+        at += n_dist + 1
+    t = {}
+    for nm, sz in (("ref_req", n_refs), ("ref_slot", n_refs), ("ref_nblk", n_refs), ("dist_off", n_dist + 1 if n_refs else 0),
+                   ("dist_refs", n_refs)):
+        t[nm] = out[at:at + sz].tolist()
+        at += sz
+    return w, t
+
+
+def check_share_tables(t, lengths, requests):
+    """References in plan order (request, first slot, blocks) and their grouping
+    by artifact id (ascending id, plan order within an id)."""
+    refs = [(r, a) for r, req in enumerate(requests) for a in req]
+    nb = [-(-lengths[a] // 64) for _, a in refs]
+    assert t["ref_req"] == [r for r, _ in refs]
+    assert t["ref_nblk"] == nb
+    slot, want = {}, []
+    for (r, a), n in zip(refs, nb):
+        want.append(slot.get(r, 0))
+        slot[r] = slot.get(r, 0) + n
+    assert t["ref_slot"] == want
+    ids = sorted(set(a for _, a in refs))
+    groups = [[i for i, (_, a) in enumerate(refs) if a == x] for x in ids]
+    assert t["dist_refs"] == [i for g in groups for i in g]
+    assert t["dist_off"] == (list(np.cumsum([0] + [len(g) for g in groups])) if refs else [])
+
+
+def check_share_work(w, t, lengths, requests, S, S_kv, n_q, n_kv):
+    """The CTA -> work mapping the shared-read kernel decodes, restated: every
+    (KV head, reference, block) and every (KV head, request, online chunk) is
+    read by exactly one CTA, a CTA's members are references of the artifact it
+    reads, and every request's partial records 0 .. P_r - 1 are written once
+    per KV head, P_r agreeing between all CTAs that write them."""
+    G = n_q // n_kv
+    R = 16 // (S * G)
+    C = w["chunk"]
+    assert w["share"] == 1 and w["members"] == R >= 2 and 1 <= C <= 1024
+    n_req = len(requests)
+    nsuf = -(-S_kv // 64)
+    assert w["suf_chunks"] == -(-nsuf // C)
+    per_head = w["art_units"] + n_req * w["suf_chunks"]
+    assert w["n_cta"] == per_head * n_kv
+    nd = w["n_dist"]
+    assert w["nsplit"][0] == 0 and w["nsplit"][nd] == w["art_units"]
+    req_refs = [[i for i, r in enumerate(t["ref_req"]) if r == q] for q in range(n_req)]
+    P = [sum(-(-t["ref_nblk"][i] // C) for i in req_refs[r]) + w["suf_chunks"] for r in range(n_req)]
+    assert w["base"] == list(np.cumsum([0] + P[:-1])) and w["n_part"] == sum(P)
+    refs = [(r, a) for r, req in enumerate(requests) for a in req]
+    for h in range(n_kv):
+        read = {}
+        parts = {}
+        for u in range(per_head):
+            cta = h * per_head + u
+            assert cta // per_head == h
+            if u < w["art_units"]:
+                d = max(x for x in range(nd) if w["nsplit"][x] <= u)
+                rb, re_ = t["dist_off"][d], t["dist_off"][d + 1]
+                nb = t["ref_nblk"][t["dist_refs"][rb]]
+                nch = -(-nb // C)
+                local = u - w["nsplit"][d]
+                chunk, m_beg = local % nch, rb + (local // nch) * R
+                n_mem = min(R, re_ - m_beg)
+                assert n_mem >= 1
+                blocks = range(chunk * C, min(nb, (chunk + 1) * C))
+                assert len(blocks) >= 1
+                for m in range(n_mem):
+                    i = t["dist_refs"][m_beg + m]
+                    assert refs[i][1] == refs[t["dist_refs"][rb]][1]      # the same artifact
+                    r = t["ref_req"][i]
+                    for b in blocks:
+                        read[("art", i, b)] = read.get(("art", i, b), 0) + 1
+                    k = sum(-(-t["ref_nblk"][j] // C) for j in req_refs[r] if j < i) + chunk
+                    parts[(r, k)] = parts.get((r, k), 0) + 1
+            else:
+                v = u - w["art_units"]
+                r, chunk = v // w["suf_chunks"], v % w["suf_chunks"]
+                for b in range(chunk * C, min(nsuf, (chunk + 1) * C)):
+                    read[("suf", r, b)] = read.get(("suf", r, b), 0) + 1
+                k = sum(-(-t["ref_nblk"][j] // C) for j in req_refs[r]) + chunk
+                parts[(r, k)] = parts.get((r, k), 0) + 1
+        want = {("art", i, b) for i in range(len(refs)) for b in range(t["ref_nblk"][i])}
+        want |= {("suf", r, b) for r in range(n_req) for b in range(nsuf)}
+        assert set(read) == want and all(c == 1 for c in read.values())
+        assert set(parts) == {(r, k) for r in range(n_req) for k in range(P[r])}
+        assert all(c == 1 for c in parts.values())
+
+
+def test_share_tables_and_work_cover_every_read_once(shim):
+    rng = np.random.default_rng(5)
+    for trial in range(60):
+        lengths = _random_registry(rng, int(rng.integers(1, 12)))
+        n_req = int(rng.integers(1, 9))
+        requests = []
+        for r in range(n_req):
+            k = int(rng.integers(0, 6))
+            # repeats across requests and now and then within one request
+            requests.append([int(a) for a in rng.integers(0, len(lengths), k)])
+        S = int(rng.choice([1, 1, 2]))
+        n_kv = int(rng.choice([1, 2, 8]))
+        G = int(rng.choice([1, 2, 4])) if S == 2 else int(rng.choice([1, 2, 4, 8]))
+        S_kv = S + int(rng.integers(0, 200))
+        opt_split = int(rng.choice([0, 1, 2, 5, 16]))
+        w, t = share_plan(shim, lengths, requests, S, S_kv, n_q=G * n_kv, n_kv=n_kv, opt_split=opt_split, opt_share=2)
+        check_share_tables(t, lengths, requests)
+        if not any(requests):
+            assert w["share"] == 0      # no artifact: nothing to share
+            continue
+        check_share_work(w, t, lengths, requests, S, S_kv, G * n_kv, n_kv)
+
+
+def test_share_choice(shim):
+    lengths = [640, 1280, 320, 2048, 700]
+    shared = [[0, 1, 3], [1, 3, 4], [0, 3], [2, 3, 1]]
+    distinct = [[0], [1], [2, 3], [4]]
+    plan = lambda req, S=1, **kw: share_plan(shim, lengths, req, S, 129, **kw)[0]
+    assert plan(shared)["share"] == 1                    # 25 % fewer block reads and more
+    assert plan(distinct)["share"] == 0                  # nothing shared
+    assert plan(distinct, opt_share=2)["share"] == 1     # forced
+    assert plan(shared, opt_share=1)["share"] == 0       # off
+    assert plan(shared, k_by_slot=1)["share"] == 0       # keys rotated per slot
+    assert plan(shared, kv_part=1)["share"] == 0         # one part only
+    assert plan(shared, S=3)["share"] == 0               # 12 rows per request: one request per CTA
+    assert plan(shared, S=2)["share"] == 1 and plan(shared, S=2)["members"] == 2
+    # the 64-request decode step: whole artifacts (4 to 32 blocks) per chunk
+    rng = np.random.default_rng(0)
+    pool = [int(x) for x in rng.integers(256, 2049, 256)]
+    reqs = [[int(a) for a in rng.choice(256, int(rng.integers(4, 13)), replace=False)] for _ in range(64)]
+    w, t = share_plan(shim, pool, reqs, 1, 129)
+    assert w["share"] == 1 and w["members"] == 4 and w["chunk"] == 32
+    check_share_work(w, t, pool, reqs, 1, 129, 32, 8)
