@@ -9,7 +9,12 @@
 // (4 KiB per token at Hkv = 8, d = 128).  One CTA owns 16 packed query rows
 // (token * G + head_in_group) of one request and KV head, and one chunk of its
 // virtual block list; the CTAs launch KV-head-major, so requests that share
-// an artifact read its blocks from L2 after the first.  Warp 4 streams
+// an artifact read its blocks from L2 after the first.  With shared reads
+// (kShare) the 16 rows are those of up to 16 / (S G) requests that use the
+// same artifact: a CTA reads one chunk of that artifact once for all of them
+// (or one chunk of a single request's online rows), and every request's
+// partial results - one per chunk of each artifact it lists, one per online
+// chunk - are merged by the last CTA to finish one of them.  Warp 4 streams
 // 64-token K/V blocks with TMA (128-byte swizzle) into a 3-stage ring (two
 // CTAs share an SM, so one's prologue and merge overlap the other's loads); warps
 // 0..3 each take 16 of the 64 keys of every block (intra-CTA split over
@@ -458,13 +463,13 @@ __global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant_
   volatile int* last_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 8 * (2 * L::NS + 1) + 4);
   if constexpr (kShare) {
     // this row's member: its request's partial record k of P (records of
-    // request r: base[r] + k, each [Hkv][16 rows])
+    // request r: base[r] + k, each [Hkv][S G rows])
     const int mi = row / SG, wr = row % SG;
     const bool mine = mi < n_mem;
     const int r = mine ? mem[4 * mi] : 0;
     const long long rec0 = (long long)p.work.base[r] * p.Hkv + kvh;   // record k at rec0 + k * Hkv
     if (mine) {
-      const long long at = (rec0 + (long long)mem[4 * mi + 1] * p.Hkv) * kMmaRows + wr;
+      const long long at = (rec0 + (long long)mem[4 * mi + 1] * p.Hkv) * SG + wr;
       float* po = p.part_o + at * D + c0;
 #pragma unroll
       for (int c = 0; c < CPT; c += 4)
@@ -479,7 +484,7 @@ __global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant_
     if (!mine || mem[4 * mi + 3] == 0) return;
     __threadfence();
     const long long orow_m = ((long long)r * p.S + wr / G) * p.Hq + kvh * G + wr % G;
-    merge_records<D>(p, mem[4 * mi + 2], [&](int k) { return (rec0 + (long long)k * p.Hkv) * kMmaRows + wr; }, c0,
+    merge_records<D>(p, mem[4 * mi + 2], [&](int k) { return (rec0 + (long long)k * p.Hkv) * SG + wr; }, c0,
                      orow_m, tid);
     return;
   }

@@ -740,10 +740,12 @@ attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, co
     for (int r = 0; r < plan->n_req; ++r) need_combine |= (w.nsplit[r] > 1);
   if (w.cluster > 0) need_combine = false;
   // partial O and LSE of every split CTA (shared reads: of every partial
-  // record) and one arrival counter per (request, KV head, row tile), zeroed
-  // below: the last CTA of a row tile to arrive merges its chunks, in either kernel
+  // record, the S G rows of one request) and one arrival counter per (request,
+  // KV head, row tile), zeroed below: the last CTA of a row tile to arrive
+  // merges its chunks, in either kernel
   const size_t records = w.share ? (size_t)w.n_part * Hkv : (size_t)w.n_cta;
-  const size_t pb = need_combine ? records * rows * (D + 1) * 4 : 0;
+  const size_t rec_rows = w.share ? (size_t)S * G : (size_t)rows;
+  const size_t pb = need_combine ? records * rec_rows * (D + 1) * 4 : 0;
   const size_t units = (size_t)plan->n_req * Hkv * w.row_tiles;
   const size_t part_bytes = pb + (need_combine ? units * 4 : 0);
   if (fixed && part_bytes > fixed->cap)
@@ -799,7 +801,7 @@ attuner_status att::attend_launch(attuner_ctx* ctx, const attuner_plan* plan, co
       return fail(ATTUNER_ERR_OOM, "split-KV scratch allocation failed");
     }
     ap.part_o = static_cast<float*>(part);
-    ap.part_lse = static_cast<float*>(part) + records * rows * D;
+    ap.part_lse = static_cast<float*>(part) + records * rec_rows * D;
     ap.unit_cnt = reinterpret_cast<int*>(static_cast<char*>(part) + pb);
     ce = cudaMemsetAsync(ap.unit_cnt, 0, units * 4, st);
   }

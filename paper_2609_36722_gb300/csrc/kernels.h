@@ -59,8 +59,9 @@ struct AttnParams {
   const __nv_bfloat16* q;        // (K3 reads Q directly)
   __nv_bfloat16* out;            // [n_req, S, Hq, D]
   float* lse_out;                // [n_req, S, Hq] or nullptr
-  float* part_o;                 // split chunks only: K3 [n_cta, 16, D]; K2 fp16 pieces (see attn_tc.cu)
-  float* part_lse;               // [n_cta, rows_per_tile]
+  float* part_o;                 // split chunks only: K3 [n_cta, 16, D] (shared reads: [n_part, Hkv, S G, D]);
+                                 // K2 fp16 pieces (see attn_tc.cu)
+  float* part_lse;               // [n_cta, rows_per_tile] (shared reads: [n_part, Hkv, S G])
   int* unit_cnt;                 // arrivals per (request, KV head, row tile); zero on entry
   int32_t S, S_kv, Hq, Hkv, G;
   float scale_log2;              // log2(e) / (sqrt(D) * temperature), temperature 1 but for APE's context part

@@ -83,3 +83,28 @@ def test_shared_and_per_request_reads_agree():
     o2, l2 = run_path(ctx, plan, wl)
     assert (o1.float() - o2.float()).abs().max().item() <= 1.6e-2
     assert (l1 - l2).abs().max().item() <= 1e-4
+
+
+def test_static_scratch_takes_a_64_request_shared_decode():
+    # 64 decode requests over a 32-artifact pool (the bench's decode recipe,
+    # smaller hidden size): the shared-read partials (S G rows per record) fit
+    # the allocation-free entry point's fixed scratch, and its result is the
+    # pool-backed call's, bit for bit (same decomposition, same arithmetic)
+    import paper_2609_36722_gb300 as pkg
+    rng = np.random.default_rng(61)
+    lengths = rng.integers(256, 2049, size=32).tolist()
+    reqs = [rng.choice(32, size=int(rng.integers(4, 13)), replace=False).tolist() for _ in range(64)]
+    geom = Geometry(hidden=256, n_q_heads=32, n_kv_heads=8, head_dim=128, rank=16)
+    wl = make_custom("dec64", geom, 61, lengths, reqs, 1, 129, device=DEV)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_SHARE_READS, 2)
+    q = ctx.q_project(plan, wl.x, wl.w_q, wl.lora_a, wl.lora_b, geom.scale, wl.q_norm_w, S_kv=wl.S_kv)
+    o1, l1 = ctx.attend(plan, q, wl.suffix_k, wl.suffix_v)
+    o2, l2 = ctx.attend_static_scratch(plan, q, wl.suffix_k, wl.suffix_v)
+    assert ctx.sync_status() == 0
+    assert torch.equal(o1.view(torch.int16), o2.view(torch.int16))
+    assert torch.equal(l1, l2)
+    # and both against the oracle on a sample of requests
+    for r in (0, 17, 63):
+        o_ref, lse_ref = oracle.workload_reference(wl, r)
+        compare(_np(o1[r:r + 1]), o_ref[None], _np(l1[r:r + 1]), lse_ref[None], label=f"dec64 request {r}")
