@@ -15,8 +15,9 @@
 // (or one chunk of a single request's online rows), and every request's
 // partial results - one per chunk of each artifact it lists, one per online
 // chunk - are merged by the last CTA to finish one of them.  Warp 4 streams
-// 64-token K/V blocks with TMA (128-byte swizzle) into a 3-stage ring (two
-// CTAs share an SM, so one's prologue and merge overlap the other's loads); warps
+// 64-token K/V blocks with TMA (128-byte swizzle) into a ring of 3 stages
+// (2 with shared reads; two or three CTAs share an SM, so one's prologue and
+// merge overlap the others' loads); warps
 // 0..3 each take 16 of the 64 keys of every block (intra-CTA split over
 // keys), run QK^T and PV with m16n8k16 warp MMAs (tensor work is ~5% of the
 // memory time here), keep an online softmax in registers, and merge their
@@ -27,17 +28,23 @@
 
 namespace att {
 
-template <int D>
+// Per-request reads: a 3-stage ring, two CTAs per SM.  Shared reads: a
+// 2-stage ring, three CTAs per SM (their CTAs are shorter, so a third CTA's
+// loads cover more of the others' prologues and merges: 0.210 against 0.213 ms
+// on the 64-request decode step, where the per-request kernel took 0.310
+// against 0.285 ms in that shape).
+template <int D, bool kShare>
 struct MmaLayout {
+  static constexpr int CTAS = kShare ? 3 : 2;        // resident CTAs per SM
   static constexpr int NH = D / 64;
-  static constexpr int NS = 3;
+  static constexpr int NS = kShare ? 2 : 3;
   static constexpr int BLK = kBlockTokens * 128;      // one 64-row x 128 B box
   static constexpr int STAGE = 2 * NH * BLK;          // K halves then V halves
   static constexpr int BAR_OFF = NS * STAGE;
   static constexpr int LIST_OFF = BAR_OFF + 256;
   static constexpr int MEM_OFF = LIST_OFF + kMmaMaxChunkBlocks * 4;   // shared reads: [16][4] member table
   static constexpr int MERGE_BYTES = 4 * 16 * (D + 2) * 4;   // per warp: O[16][D], m[16], l[16]
-  static constexpr int SMEM = MEM_OFF + 16 * 16 + 1024;   // two CTAs per SM
+  static constexpr int SMEM = MEM_OFF + 16 * 16 + 1024;   // CTAS of them fit in an SM's shared memory
   static_assert(MERGE_BYTES <= BAR_OFF, "merge area aliases the stage ring");
 };
 
@@ -82,8 +89,9 @@ ATT_DEV void merge_records(const AttnParams& p, int n, Rec rec, int c0, long lon
 // of a request's online rows, and every request's partials are merged by the
 // last CTA to finish one of them
 template <int D, bool kLayout, bool kShare>
-__global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant__ AttnParams p) {
-  using L = MmaLayout<D>;
+__global__ void __launch_bounds__(160, kShare ? 3 : 2) attn_mma_kernel(const __grid_constant__ AttnParams p) {
+  using L = MmaLayout<D, kShare>;
+  static_assert(L::CTAS == (kShare ? 3 : 2), "launch bounds and layout agree");
   grid_dep_wait();     // Q and the suffix K/V may come from the previous kernel
   constexpr int NT = D / 8;           // n8 tiles of the output
   constexpr int KS = D / 16;          // k16 steps of QK^T
@@ -518,7 +526,7 @@ __global__ void __launch_bounds__(160, 2) attn_mma_kernel(const __grid_constant_
 
 template <int D, bool kLayout, bool kShare>
 static cudaError_t launch_attn_mma_t(const AttnParams& p, cudaStream_t st) {
-  using L = MmaLayout<D>;
+  using L = MmaLayout<D, kShare>;
   cudaError_t e =
       cudaFuncSetAttribute(attn_mma_kernel<D, kLayout, kShare>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM);
   if (e != cudaSuccess) return e;
