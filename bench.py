@@ -478,6 +478,7 @@ class HostInputs:
 
 
 L2_BYTES = 129 << 20
+E2E_DEPTH = 3   # steps in flight in the end-to-end loop
 
 
 def working_set_bytes(bed) -> int:
@@ -497,9 +498,9 @@ def measure_e2e(bed, args, world, flush, local_rank=0):
     rows; a decode step's earlier suffix rows are the request's resident cache,
     like the artifact pool), runs the projection and the attention, and copies
     O back to pinned host memory, all on the step's stream; a step counts as
-    done once its output is on the host.  Step i+1 is assembled and enqueued,
-    on another stream, while step i runs (two sets of buffers per context), so
-    host work and copies overlap device work as in a server.  No flush runs
+    done once its output is on the host.  Steps i+1 and i+2 are assembled and
+    enqueued, on other streams, while step i runs (three sets of buffers per
+    context), so host work and copies overlap device work as in a server.  No flush runs
     inside the loop: a workload whose working set fits in L2 alternates between
     enough identical, separately loaded contexts that every step reads data the
     others have evicted."""
@@ -508,15 +509,16 @@ def measure_e2e(bed, args, world, flush, local_rank=0):
     beds = [bed] + [Bed(bed.name, bed.dev, local_rank) for _ in range(n_sets - 1)]
     try:
         # (bed, host buffers and device suffix K/V, stream, output-on-host event)
+        # interleaved, so that consecutive steps use different contexts
         units = []
-        for b in beds:
-            for _ in range(2):
+        for _ in range(E2E_DEPTH):
+            for b in beds:
                 units.append((b, HostInputs(b), torch.cuda.Stream(device=bed.dev), torch.cuda.Event()))
         n_units = len(units)
 
         def enqueue(i, plan):
             # each unit's buffers are reused only after the step that last used
-            # them was waited for (two steps in flight at most)
+            # them was waited for (E2E_DEPTH steps in flight at most)
             b, io, stream, done = units[i % n_units]
             wl, g = b.wl, b.g
             b.ctx.query_attend_host(plan, io.x_h, wl.w_q, wl.lora_a, wl.lora_b, g.scale, wl.q_norm_w, io.sk_d,
@@ -528,12 +530,15 @@ def measure_e2e(bed, args, world, flush, local_rank=0):
             return b.ctx.assemble(b.wl.requests)
 
         def run(n):
-            plans = {0: assemble(0)}
-            enqueue(0, plans[0])
+            plans = {}
+            for i in range(min(E2E_DEPTH - 1, n)):
+                plans[i] = assemble(i)
+                enqueue(i, plans[i])
             for i in range(n):
-                if i + 1 < n:
-                    plans[i + 1] = assemble(i + 1)     # the next step, while step i runs
-                    enqueue(i + 1, plans[i + 1])
+                nxt = i + E2E_DEPTH - 1
+                if nxt < n:
+                    plans[nxt] = assemble(nxt)         # a later step, while step i runs
+                    enqueue(nxt, plans[nxt])
                 units[i % n_units][3].synchronize()    # step i's output is on the host
                 plans.pop(i).free()
 
@@ -557,8 +562,8 @@ def measure_e2e(bed, args, world, flush, local_rank=0):
                 "includes": "per step: assemble (host block table + upload) and one attuner_query_attend_host call "
                             "(H2D of the step's new tokens - x and their own suffix K/V rows; a decode step's earlier "
                             "suffix rows stay resident - the Q projection, the attention and the D2H of O, on the "
-                            "step's stream) and a wait for the output; step i+1 assembled and enqueued on another "
-                            "stream while step i runs"}
+                            "step's stream) and a wait for the output; steps i+1 and i+2 assembled and enqueued on "
+                            "other streams while step i runs"}
     finally:
         for b in beds[1:]:
             b.close()
