@@ -51,28 +51,55 @@ struct MmaLayout {
 // The merge of n partial results of one query row (K4): record k of the row
 // at part_lse[rec(k)] and part_o[rec(k) * D ...], in order k = 0 .. n - 1:
 // lse = log sum_k exp(lse_k),  O = sum_k exp(lse_k - lse) O_k.  The calling
-// thread writes its CPT = D / 8 columns from c0 of output row orow.
+// thread writes its CPT = D / 8 columns from c0 of output row orow.  The
+// loads of eight log-sum-exps, then of two records, are issued before any is
+// used: the merge is bound by L2 latency, not by its few bytes (two records
+// and not four keep the three-CTAs-per-SM kernel within its registers).
 template <int D, class Rec>
 ATT_DEV void merge_records(const AttnParams& p, int n, Rec rec, int c0, long long orow, int tid) {
-  constexpr int CPT = D / 8;
+  constexpr int CPT = D / 8, NV = CPT / 4;
   float Ms = -INFINITY;
-  for (int k = 0; k < n; ++k) Ms = fmaxf(Ms, __ldcg(p.part_lse + rec(k)));
+  int k = 0;
+  for (; k + 8 <= n; k += 8) {
+    float l[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) l[i] = __ldcg(p.part_lse + rec(k + i));
+#pragma unroll
+    for (int i = 0; i < 8; ++i) Ms = fmaxf(Ms, l[i]);
+  }
+  for (; k < n; ++k) Ms = fmaxf(Ms, __ldcg(p.part_lse + rec(k)));
   float W = 0.f;
   float acc[CPT];
 #pragma unroll
   for (int c = 0; c < CPT; ++c) acc[c] = 0.f;
-  for (int k = 0; k < n; ++k) {
-    const long long at = rec(k);
-    const float ls = __ldcg(p.part_lse + at);
-    if (ls == -INFINITY) continue;
-    const float w = __expf(ls - Ms);
+  auto add = [&](float ls, const float4* v) {
+    const float w = (ls == -INFINITY) ? 0.f : __expf(ls - Ms);
     W += w;
-    const float* q = p.part_o + at * D + c0;
 #pragma unroll
-    for (int c = 0; c < CPT; c += 4) {
-      const float4 v = __ldcg(reinterpret_cast<const float4*>(q + c));
-      acc[c] += w * v.x; acc[c + 1] += w * v.y; acc[c + 2] += w * v.z; acc[c + 3] += w * v.w;
+    for (int c = 0; c < NV; ++c) {
+      acc[4 * c] += w * v[c].x; acc[4 * c + 1] += w * v[c].y; acc[4 * c + 2] += w * v[c].z; acc[4 * c + 3] += w * v[c].w;
     }
+  };
+  k = 0;
+  for (; k + 2 <= n; k += 2) {
+    float ls[2];
+    float4 v[2][NV];
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const long long at = rec(k + i);
+      ls[i] = __ldcg(p.part_lse + at);
+#pragma unroll
+      for (int c = 0; c < NV; ++c) v[i][c] = __ldcg(reinterpret_cast<const float4*>(p.part_o + at * D + c0) + c);
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) add(ls[i], v[i]);
+  }
+  for (; k < n; ++k) {
+    const long long at = rec(k);
+    float4 v[NV];
+#pragma unroll
+    for (int c = 0; c < NV; ++c) v[c] = __ldcg(reinterpret_cast<const float4*>(p.part_o + at * D + c0) + c);
+    add(__ldcg(p.part_lse + at), v);
   }
   const float invW = (W > 0.f) ? 1.f / W : 0.f;
   uint4* dst = reinterpret_cast<uint4*>(p.out + orow * D + c0);
@@ -110,9 +137,19 @@ __global__ void __launch_bounds__(160, kShare ? 3 : 2) attn_mma_kernel(const __g
   int* mem = reinterpret_cast<int*>(smem + L::MEM_OFF);   // shared reads: request, partial, partials, last
   int kvh, req, row0, nblk, b0 = 0, boff = 0, nab = 0, cta = 0, nsplit = 1, rt = 0, n_mem = 1;
   if constexpr (kShare) {
-    const int per_head = p.work.n_cta / p.Hkv;
-    kvh = blockIdx.x / per_head;
-    const int u = blockIdx.x % per_head;
+    // Launch order: the artifact units KV-head-major (the CTAs resident at any
+    // one time read one head's blocks), then every head's online-row units,
+    // short CTAs that fill the grid's last wave.
+    const int art_ctas = p.work.art_units * p.Hkv;
+    int u;
+    if ((int)blockIdx.x < art_ctas) {
+      kvh = blockIdx.x / p.work.art_units;
+      u = blockIdx.x % p.work.art_units;
+    } else {
+      const int v = blockIdx.x - art_ctas, per = p.work.n_req * p.work.suf_chunks;
+      kvh = v / per;
+      u = p.work.art_units + v % per;
+    }
     const int C = p.work.chunk_blocks;
     row0 = 0;
     int chunk, src = 0, m_beg = 0;
@@ -124,15 +161,14 @@ __global__ void __launch_bounds__(160, kShare ? 3 : 2) attn_mma_kernel(const __g
         if (p.work.nsplit[mid] <= u) lo = mid; else hi = mid - 1;
       }
       const int r_beg = p.plan.dist_off[lo], r_end = p.plan.dist_off[lo + 1];
-      const int nb = p.plan.ref_nblk[p.plan.dist_refs[r_beg]];
+      const int nb = p.plan.dist_nb[lo];
       const int nch = (nb + C - 1) / C;
       const int local = u - p.work.nsplit[lo];
       chunk = local % nch;
       m_beg = r_beg + (local / nch) * p.work.members;
       n_mem = min(p.work.members, r_end - m_beg);
-      const int i0 = p.plan.dist_refs[m_beg];
-      req = p.plan.ref_req[i0];
-      src = p.plan.blk_off[req] + p.plan.ref_slot[i0] + chunk * C;
+      req = p.plan.dref_req[m_beg];
+      src = p.plan.dist_src[lo] + chunk * C;
       nblk = min(C, nb - chunk * C);
     } else {
       const int v = u - p.work.art_units;
@@ -158,13 +194,26 @@ __global__ void __launch_bounds__(160, kShare ? 3 : 2) attn_mma_kernel(const __g
       // the member's request, the index of this chunk among the request's
       // partials (its references' chunks in prompt order, then the suffix
       // chunks) and their count
-      const int ir = art ? p.plan.dist_refs[m_beg + threadIdx.x] : -1;
-      const int r = art ? p.plan.ref_req[ir] : req;
-      int k = 0, P = 0;
-      for (int i = p.plan.req_art_off[r]; i < p.plan.req_art_off[r + 1]; ++i) {
-        const int n = (p.plan.ref_nblk[i] + C - 1) / C;
-        if (i < ir) k += n;
-        P += n;
+      int r, j, nref;
+      if (art) {
+        r = p.plan.dref_req[m_beg + threadIdx.x];
+        j = p.plan.dref_j[m_beg + threadIdx.x];
+        nref = p.plan.dref_nref[m_beg + threadIdx.x];
+      } else {
+        r = req;
+        j = 0;
+        nref = p.plan.req_art_off[r + 1] - p.plan.req_art_off[r];
+      }
+      int k = j, P = nref;   // every reference one chunk
+      if (!p.work.whole_refs) {
+        k = 0;
+        P = 0;
+        const int i0 = p.plan.req_art_off[r];
+        for (int i = 0; i < nref; ++i) {
+          const int n = (p.plan.ref_nblk[i0 + i] + C - 1) / C;
+          if (i < j) k += n;
+          P += n;
+        }
       }
       mem[4 * threadIdx.x + 0] = r;
       mem[4 * threadIdx.x + 1] = art ? k + chunk : P + chunk;

@@ -304,10 +304,11 @@ static attuner_status assemble_impl(attuner_ctx* ctx, const int32_t* ids, const 
   p->pool_gen = ctx->pool_gen;
   attuner_status s = set_device(ctx);
   if (s != ATTUNER_OK) { delete p; return s; }
-  // the device image: blk_off | blocks | t_art | o_rows | span_off | req_art_off | ref_req |
-  // ref_slot | ref_nblk | dist_off | dist_refs | (16-byte aligned) spans
-  const std::vector<int32_t>* parts[] = {&p->blk_off, &p->blocks, &p->t_art, &p->o_rows, &p->span_off, &p->req_art_off,
-                                         &p->ref_req, &p->ref_slot, &p->ref_nblk, &p->dist_off, &p->dist_refs};
+  // the device image: blk_off | blocks | t_art | o_rows | span_off | req_art_off | ref_nblk |
+  // dist_off | dist_src | dist_nb | dref_req | dref_j | dref_nref | (16-byte aligned) spans
+  const std::vector<int32_t>* parts[] = {&p->blk_off, &p->blocks,   &p->t_art,   &p->o_rows,   &p->span_off,
+                                         &p->req_art_off, &p->ref_nblk, &p->dist_off, &p->dist_src, &p->dist_nb,
+                                         &p->dref_req, &p->dref_j, &p->dref_nref};
   size_t head = 0;
   for (const std::vector<int32_t>* v : parts) head += v->size();
   p->spans_at = (head + 3) & ~size_t(3);   // int4 spans start 16-byte aligned
@@ -498,11 +499,13 @@ PlanDev att::plan_dev(const attuner_plan* p) {
   d.o_rows = d.t_art + p->t_art.size();
   d.span_off = d.o_rows + p->o_rows.size();
   d.req_art_off = d.span_off + p->span_off.size();
-  d.ref_req = d.req_art_off + p->req_art_off.size();
-  d.ref_slot = d.ref_req + p->ref_req.size();
-  d.ref_nblk = d.ref_slot + p->ref_slot.size();
+  d.ref_nblk = d.req_art_off + p->req_art_off.size();
   d.dist_off = d.ref_nblk + p->ref_nblk.size();
-  d.dist_refs = d.dist_off + p->dist_off.size();
+  d.dist_src = d.dist_off + p->dist_off.size();
+  d.dist_nb = d.dist_src + p->dist_src.size();
+  d.dref_req = d.dist_nb + p->dist_nb.size();
+  d.dref_j = d.dref_req + p->dref_req.size();
+  d.dref_nref = d.dref_j + p->dref_j.size();
   d.spans = reinterpret_cast<const int4*>(p->d_buf + p->spans_at);
   d.pool_blocks = p->pool_blocks;
   d.has_spans = p->max_o_rows > 0 ? 1 : 0;

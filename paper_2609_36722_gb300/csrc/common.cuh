@@ -35,11 +35,13 @@ struct PlanDev {
   const int4* spans;        // explicit online spans: (online row0, rows, artifact slots before, artifact tokens before)
   // artifact references and their grouping by artifact (PlanTables)
   const int32_t* req_art_off;   // [n_req + 1] CSR offsets into the references
-  const int32_t* ref_req;
-  const int32_t* ref_slot;
-  const int32_t* ref_nblk;
-  const int32_t* dist_off;      // [n_dist + 1]
-  const int32_t* dist_refs;
+  const int32_t* ref_nblk;      // blocks of each reference (plan order)
+  const int32_t* dist_off;      // [n_dist + 1] references of each distinct artifact
+  const int32_t* dist_src;      // [n_dist] plan slot of its first reference's first block
+  const int32_t* dist_nb;       // [n_dist] its blocks
+  const int32_t* dref_req;      // per reference in grouping order: its request,
+  const int32_t* dref_j;        //   its ordinal among the request's references,
+  const int32_t* dref_nref;     //   and the request's number of references
   int32_t pool_blocks;      // capacity, for bounds checks
   int32_t has_spans;        // 0: no request has explicit online spans (o_rows all 0; no loads needed)
 };

@@ -103,6 +103,23 @@ attuner_status build_plan_tables(const std::vector<Artifact>& arts, const int32_
   for (int i = 1; i < n_refs; ++i)
     if (t.art_ids[t.dist_refs[i]] != t.art_ids[t.dist_refs[i - 1]]) t.dist_off.push_back(i);
   if (n_refs > 0) t.dist_off.push_back(n_refs);
+  const int nd = t.n_dist();
+  t.dist_src.resize(nd);
+  t.dist_nb.resize(nd);
+  for (int d = 0; d < nd; ++d) {
+    const int i0 = t.dist_refs[t.dist_off[d]];
+    t.dist_src[d] = t.blk_off[t.ref_req[i0]] + t.ref_slot[i0];
+    t.dist_nb[d] = t.ref_nblk[i0];
+  }
+  t.dref_req.resize(n_refs);
+  t.dref_j.resize(n_refs);
+  t.dref_nref.resize(n_refs);
+  for (int k = 0; k < n_refs; ++k) {
+    const int i = t.dist_refs[k], r = t.ref_req[i];
+    t.dref_req[k] = r;
+    t.dref_j[k] = i - t.req_art_off[r];
+    t.dref_nref[k] = t.req_art_off[r + 1] - t.req_art_off[r];
+  }
   return ATTUNER_OK;
 }
 
@@ -178,11 +195,13 @@ attuner_status share_work(const SplitPolicy& pol, const PlanTables& t, int S_kv,
   w.share = 1;
   w.members = members;
   w.n_dist = nd;
+  w.whole_refs = 1;
+  for (int32_t nb : t.dist_nb) w.whole_refs &= (nb <= chunk) ? 1 : 0;
   long long u = 0;
   for (int d = 0; d < nd; ++d) {
     w.nsplit[d] = (int32_t)u;
     const int nref = t.dist_off[d + 1] - t.dist_off[d];
-    u += nch(t.ref_nblk[t.dist_refs[t.dist_off[d]]]) * ((nref + members - 1) / members);
+    u += nch(t.dist_nb[d]) * ((nref + members - 1) / members);
     if (u * Hkv > kMaxCta) return bad(ATTUNER_ERR_INVALID_ARG, err, "attention launch needs >= 2^31 CTAs");
   }
   w.nsplit[nd] = (int32_t)u;
@@ -211,6 +230,7 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
   w.art_units = 0;
   w.suf_chunks = 0;
   w.n_part = 0;
+  w.whole_refs = 0;
   const int G = pol.n_q_heads / pol.n_kv_heads, Hkv = pol.n_kv_heads;
   const int rows = tc ? kTcRows : kMmaRows;
   const int row_tiles = (S * G + rows - 1) / rows;
@@ -253,7 +273,7 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
       long long reads_req = 0, reads_share = 0;
       for (int d = 0; d < nd; ++d) {
         const int nref = t.dist_off[d + 1] - t.dist_off[d];
-        const long long nb = t.ref_nblk[t.dist_refs[t.dist_off[d]]];
+        const long long nb = t.dist_nb[d];
         reads_req += nb * nref;
         reads_share += nb * ((nref + members - 1) / members);
       }

@@ -88,8 +88,10 @@ QpShape choose_qproj_shape(const QpPolicy& pol, int heads, int M, int n_lora);
 // artifact d (the plan's dist_* tables) in chunks of chunk_blocks of its
 // blocks, times groups of `members` of its references - numbered from
 // nsplit[d] (nsplit[n_dist] = art_units), then suffix units: request r's
-// chunks of online rows, art_units + r * suf_chunks + chunk.  CTA index =
-// kv_head * (n_cta / n_kv_heads) + unit.  Every (reference, chunk) and every
+// chunks of online rows, art_units + r * suf_chunks + chunk.  CTA index:
+// artifact unit u of KV head h at h * art_units + u, then the suffix units of
+// every head, unit art_units + v of head h at Hkv * art_units + h * n_req *
+// suf_chunks + v (the short suffix CTAs last).  Every (reference, chunk) and every
 // suffix chunk leaves a partial result of its request; request r's partials
 // are records base[r] .. base[r] + P_r - 1 (the references' chunks in prompt
 // order, then the suffix chunks), n_part in all per KV head, and the last
@@ -114,6 +116,7 @@ struct WorkTable {
   int32_t art_units;      // artifact units per KV head
   int32_t suf_chunks;     // suffix units of each request
   int32_t n_part;         // partial records per KV head
+  int32_t whole_refs;     // every artifact fits one chunk: a reference's partial index is its ordinal
 };
 
 // A registered artifact: ceil(L/64) consecutive pool blocks from first_block
@@ -150,6 +153,13 @@ struct PlanTables {
   std::vector<int32_t> ref_req, ref_slot, ref_nblk;
   std::vector<int32_t> dist_off;      // [n_dist + 1]
   std::vector<int32_t> dist_refs;
+  // what the decode kernel reads of them, flattened so that one load (two for
+  // the blocks) reaches it: per distinct artifact the plan slot of its first
+  // reference's first block and its block count; per reference in dist_refs
+  // order its request, its ordinal among that request's references and the
+  // request's number of references
+  std::vector<int32_t> dist_src, dist_nb;
+  std::vector<int32_t> dref_req, dref_j, dref_nref;
   int n_dist() const { return dist_off.empty() ? 0 : (int)dist_off.size() - 1; }
 };
 

@@ -123,8 +123,9 @@ extern "C" int shim_qproj_supported(int32_t D, int32_t mr, int32_t ks, int32_t n
 // one warp-MMA launch over it.  pol = n_q_heads, n_kv_heads, num_sms,
 // opt_split, opt_share, k_by_slot, kv_part.  out (capacity cap) = n_cta,
 // chunk_blocks, share, members, n_dist, art_units, suf_chunks, n_part,
-// base[n_req] | nsplit[n_dist + 1] | ref_req | ref_slot | ref_nblk |
-// dist_off[n_dist + 1] | dist_refs; lens = n_refs, n_dist.
+// whole_refs, base[n_req] | nsplit[n_dist + 1] | ref_req | ref_slot |
+// ref_nblk | dist_off[n_dist + 1] | dist_refs | dist_src | dist_nb |
+// dref_req | dref_j | dref_nref; lens = n_refs, n_dist.
 extern "C" int shim_share(const int32_t* pol, const int32_t* first, const int32_t* L, int32_t n_arts,
                           const int32_t* items, const int32_t* offs, int32_t n_req, int32_t S, int32_t S_kv,
                           int32_t* out, int64_t cap, int64_t* lens) {
@@ -147,10 +148,12 @@ extern "C" int shim_share(const int32_t* pol, const int32_t* first, const int32_
   att::WorkTable w;
   s = att::split_work(p, t, S, S_kv, false, w, g_err);
   if (s != ATTUNER_OK) return s;
-  std::vector<int32_t> h = {w.n_cta, w.chunk_blocks, w.share, w.members, w.n_dist, w.art_units, w.suf_chunks, w.n_part};
+  std::vector<int32_t> h = {w.n_cta,     w.chunk_blocks, w.share,  w.members,   w.n_dist,
+                            w.art_units, w.suf_chunks,   w.n_part, w.whole_refs};
   h.insert(h.end(), w.base, w.base + n_req);
   if (w.share) h.insert(h.end(), w.nsplit, w.nsplit + w.n_dist + 1);
-  for (const auto* v : {&t.ref_req, &t.ref_slot, &t.ref_nblk, &t.dist_off, &t.dist_refs})
+  for (const auto* v : {&t.ref_req, &t.ref_slot, &t.ref_nblk, &t.dist_off, &t.dist_refs, &t.dist_src, &t.dist_nb,
+                        &t.dref_req, &t.dref_j, &t.dref_nref})
     h.insert(h.end(), v->begin(), v->end());
   if ((int64_t)h.size() > cap) {
     g_err = "output capacity too small";

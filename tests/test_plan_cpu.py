@@ -489,7 +489,7 @@ def share_plan(shim, lengths, requests, S, S_kv, n_q=32, n_kv=8, num_sms=152, op
                          ctypes.c_int64(cap), lens.ctypes.data_as(I64P))
     assert st == OK, shim.shim_last_error()
     n_refs, n_dist = int(lens[0]), int(lens[1])
-    keys = ["n_cta", "chunk", "share", "members", "n_dist", "art_units", "suf_chunks", "n_part"]
+    keys = ["n_cta", "chunk", "share", "members", "n_dist", "art_units", "suf_chunks", "n_part", "whole_refs"]
     w = {k: int(out[i]) for i, k in enumerate(keys)}
     at = len(keys)
     w["base"] = out[at:at + n_req].tolist()
@@ -499,7 +499,8 @@ def share_plan(shim, lengths, requests, S, S_kv, n_q=32, n_kv=8, num_sms=152, op
         at += n_dist + 1
     t = {}
     for nm, sz in (("ref_req", n_refs), ("ref_slot", n_refs), ("ref_nblk", n_refs), ("dist_off", n_dist + 1 if n_refs else 0),
-                   ("dist_refs", n_refs)):
+                   ("dist_refs", n_refs), ("dist_src", n_dist), ("dist_nb", n_dist), ("dref_req", n_refs),
+                   ("dref_j", n_refs), ("dref_nref", n_refs)):
         t[nm] = out[at:at + sz].tolist()
         at += sz
     return w, t
@@ -521,6 +522,15 @@ def check_share_tables(t, lengths, requests):
     groups = [[i for i, (_, a) in enumerate(refs) if a == x] for x in ids]
     assert t["dist_refs"] == [i for g in groups for i in g]
     assert t["dist_off"] == (list(np.cumsum([0] + [len(g) for g in groups])) if refs else [])
+    # the flattened forms the kernel reads
+    blk_off = list(np.cumsum([0] + [sum(-(-lengths[a] // 64) for a in req) for req in requests]))
+    first = [g[0] for g in groups]
+    assert t["dist_src"] == [blk_off[refs[i][0]] + want[i] for i in first]
+    assert t["dist_nb"] == [nb[i] for i in first]
+    order = t["dist_refs"]
+    assert t["dref_req"] == [refs[i][0] for i in order]
+    assert t["dref_j"] == [i - sum(len(requests[q]) for q in range(refs[i][0])) for i in order]
+    assert t["dref_nref"] == [len(requests[refs[i][0]]) for i in order]
 
 
 def check_share_work(w, t, lengths, requests, S, S_kv, n_q, n_kv):
@@ -533,6 +543,7 @@ def check_share_work(w, t, lengths, requests, S, S_kv, n_q, n_kv):
     R = 16 // (S * G)
     C = w["chunk"]
     assert w["share"] == 1 and w["members"] == R >= 2 and 1 <= C <= 1024
+    assert w["whole_refs"] == int(all(nb <= C for nb in t["ref_nblk"]))
     n_req = len(requests)
     nsuf = -(-S_kv // 64)
     assert w["suf_chunks"] == -(-nsuf // C)
@@ -544,16 +555,26 @@ def check_share_work(w, t, lengths, requests, S, S_kv, n_q, n_kv):
     P = [sum(-(-t["ref_nblk"][i] // C) for i in req_refs[r]) + w["suf_chunks"] for r in range(n_req)]
     assert w["base"] == list(np.cumsum([0] + P[:-1])) and w["n_part"] == sum(P)
     refs = [(r, a) for r, req in enumerate(requests) for a in req]
+    # CTA -> (KV head, unit): every head's artifact units, then every head's suffix units
+    units = {h: [] for h in range(n_kv)}
+    n_suf = n_req * w["suf_chunks"]
+    for cta in range(w["n_cta"]):
+        if cta < w["art_units"] * n_kv:
+            units[cta // w["art_units"]].append(cta % w["art_units"])
+        else:
+            v = cta - w["art_units"] * n_kv
+            units[v // n_suf].append(w["art_units"] + v % n_suf)
     for h in range(n_kv):
         read = {}
         parts = {}
-        for u in range(per_head):
-            cta = h * per_head + u
-            assert cta // per_head == h
+        assert sorted(units[h]) == list(range(per_head))
+        for u in units[h]:
             if u < w["art_units"]:
+                # as the kernel decodes it: from dist_off / dist_nb / dist_src
+                # and the dref_* tables of the members
                 d = max(x for x in range(nd) if w["nsplit"][x] <= u)
                 rb, re_ = t["dist_off"][d], t["dist_off"][d + 1]
-                nb = t["ref_nblk"][t["dist_refs"][rb]]
+                nb = t["dist_nb"][d]
                 nch = -(-nb // C)
                 local = u - w["nsplit"][d]
                 chunk, m_beg = local % nch, rb + (local // nch) * R
@@ -562,12 +583,17 @@ def check_share_work(w, t, lengths, requests, S, S_kv, n_q, n_kv):
                 blocks = range(chunk * C, min(nb, (chunk + 1) * C))
                 assert len(blocks) >= 1
                 for m in range(n_mem):
-                    i = t["dist_refs"][m_beg + m]
+                    r, jj, nref = t["dref_req"][m_beg + m], t["dref_j"][m_beg + m], t["dref_nref"][m_beg + m]
+                    i = req_refs[r][jj]                                   # the member's reference
                     assert refs[i][1] == refs[t["dist_refs"][rb]][1]      # the same artifact
-                    r = t["ref_req"][i]
+                    assert nref == len(req_refs[r])
                     for b in blocks:
                         read[("art", i, b)] = read.get(("art", i, b), 0) + 1
-                    k = sum(-(-t["ref_nblk"][j] // C) for j in req_refs[r] if j < i) + chunk
+                    if w["whole_refs"]:
+                        k = jj + chunk
+                    else:
+                        k = sum(-(-t["ref_nblk"][req_refs[r][q]] // C) for q in range(jj)) + chunk
+                    assert k == sum(-(-t["ref_nblk"][j] // C) for j in req_refs[r] if j < i) + chunk
                     parts[(r, k)] = parts.get((r, k), 0) + 1
             else:
                 v = u - w["art_units"]
