@@ -652,3 +652,15 @@ def test_share_choice(shim):
     w, t = share_plan(shim, pool, reqs, 1, 129)
     assert w["share"] == 1 and w["members"] == 4 and w["chunk"] == 32
     check_share_work(w, t, pool, reqs, 1, 129, 32, 8)
+
+
+def test_share_falls_back_beyond_the_distinct_artifact_table(shim):
+    # the work table holds 511 distinct artifacts' unit offsets: a plan with
+    # more reads per request even when shared reads are forced on
+    lengths = [64] * 600
+    reqs = [[i, (i + 1) % 600] for i in range(0, 600, 2)] + [[i] for i in range(1, 600, 2)]
+    w, _ = share_plan(shim, lengths, reqs[:512], 1, 9, opt_share=2)
+    assert w["share"] == 0
+    w, t = share_plan(shim, lengths[:511], [[i, (i + 7) % 511] for i in range(511)], 1, 9, opt_share=2)
+    assert w["share"] == 1 and w["n_dist"] == 511
+    check_share_work(w, t, lengths[:511], [[i, (i + 7) % 511] for i in range(511)], 1, 9, 32, 8)
