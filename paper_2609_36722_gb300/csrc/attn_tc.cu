@@ -438,14 +438,25 @@ __device__ __noinline__ void tc_epilogue(const AttnParams& p, uint8_t* smem, uin
       fence_proxy_async_all();
       const int c0 = p.work.base[req] + kvh * p.work.row_tiles + rt;   // CTA of split 0
       const int cstride = p.Hkv * p.work.row_tiles;
-      // merge weights exp(lse_s - max) of this row, one per split
+      // merge weights exp(lse_s - max) of this row, one per split; the
+      // splits' log-sum-exps are loaded together (one L2 round trip, not one
+      // per split), eight at a time
       float* wt = reinterpret_cast<float*>(smem + kWtsOff);
       float mx = -INFINITY;
-      for (int sp = 0; sp < nsplit; ++sp)
-        mx = fmaxf(mx, __ldcg(p.part_lse + (long long)(c0 + sp * cstride) * kTcRows + r));
+      for (int s0 = 0; s0 < nsplit; s0 += 8) {
+        float ls[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          ls[i] = (s0 + i < nsplit) ? __ldcg(p.part_lse + (long long)(c0 + (s0 + i) * cstride) * kTcRows + r) : -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          mx = fmaxf(mx, ls[i]);
+          if (s0 + i < nsplit) wt[(s0 + i) * kTcRows + r] = ls[i];
+        }
+      }
       float wsum = 0.f;
       for (int sp = 0; sp < nsplit; ++sp) {
-        const float ls = __ldcg(p.part_lse + (long long)(c0 + sp * cstride) * kTcRows + r);
+        const float ls = wt[sp * kTcRows + r];
         const float w = (ls == -INFINITY) ? 0.f : __expf(ls - mx);
         wsum += w;
         wt[sp * kTcRows + r] = w;
