@@ -108,3 +108,31 @@ def test_static_scratch_takes_a_64_request_shared_decode():
     for r in (0, 17, 63):
         o_ref, lse_ref = oracle.workload_reference(wl, r)
         compare(_np(o1[r:r + 1]), o_ref[None], _np(l1[r:r + 1]), lse_ref[None], label=f"dec64 request {r}")
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_random_decode_plans_both_decompositions(seed):
+    # random plans: artifacts repeated across and within requests, empty
+    # requests, lengths across block boundaries, random group size, head size,
+    # rows per request (S G <= 16) and chunk size; shared reads forced on and off
+    import paper_2609_36722_gb300 as pkg
+    rng = np.random.default_rng(100 + seed)
+    G = int(rng.choice([1, 2, 4, 8]))
+    D = int(rng.choice([64, 128]))
+    S = int(rng.choice([s for s in (1, 2, 3, 4) if s * G <= 16]))
+    n_kv = int(rng.choice([1, 2, 4]))
+    geom = Geometry(hidden=256, n_q_heads=G * n_kv, n_kv_heads=n_kv, head_dim=D, rank=8)
+    lengths = [int(x) for x in rng.integers(1, 400, size=int(rng.integers(2, 9)))]
+    n_req = int(rng.integers(1, 13))
+    reqs = [[int(a) for a in rng.integers(0, len(lengths), size=int(rng.integers(0, 6)))] for _ in range(n_req)]
+    S_kv = S + int(rng.integers(0, 150))
+    wl = make_custom(f"rand{seed}", geom, 200 + seed, lengths, reqs, S, S_kv, device=DEV)
+    o_ref, lse_ref = _reference(wl)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, 2)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, int(rng.choice([0, 1, 2, 5])))
+    for share in (1, 2):
+        ctx.set_option(pkg.OPT_SHARE_READS, share)
+        out, lse = run_path(ctx, plan, wl)
+        compare(_np(out), o_ref, _np(lse), lse_ref,
+                label=f"seed={seed} share={share} G={G} D={D} S={S} n_req={n_req} S_kv={S_kv}")
