@@ -257,3 +257,32 @@ def test_q_project_unsupported_shape_refused():
         ctx.set_option(pkg.OPT_QPROJ_SPLIT_K, 3)
     with pytest.raises(pkg.AttunerError):
         ctx.set_option(pkg.OPT_QPROJ_ROWS, 64)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_random_prefill_plans(seed):
+    # random plans for the tcgen05 kernel: artifacts repeated across and within
+    # requests, empty requests, lengths across block boundaries, ragged row
+    # tiles, random group size and head size; the split merge mode and split
+    # size forced at random
+    import paper_2609_36722_gb300 as pkg
+    rng = np.random.default_rng(300 + seed)
+    G = int(rng.choice([1, 2, 4, 8]))
+    D = int(rng.choice([64, 128]))
+    n_kv = int(rng.choice([1, 2, 4]))
+    geom = Geometry(hidden=256, n_q_heads=G * n_kv, n_kv_heads=n_kv, head_dim=D, rank=8)
+    lengths = [int(x) for x in rng.integers(1, 900, size=int(rng.integers(2, 7)))]
+    n_req = int(rng.integers(1, 4))
+    reqs = [[int(a) for a in rng.integers(0, len(lengths), size=int(rng.integers(0, 5)))] for _ in range(n_req)]
+    S = int(rng.integers(17, 260))
+    S_kv = S + int(rng.integers(0, 100))
+    wl = make_custom(f"randp{seed}", geom, 400 + seed, lengths, reqs, S, S_kv, device=DEV)
+    o_ref, lse_ref = _full_reference(wl)
+    ctx, plan = load_context(wl)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, 1)
+    merge, split = int(rng.choice([0, 1, 2])), int(rng.choice([0, 2, 4, 6]))
+    ctx.set_option(pkg.OPT_SPLIT_MERGE, merge)
+    ctx.set_option(pkg.OPT_SPLIT_BLOCKS, split)
+    out, lse = run_path(ctx, plan, wl)
+    compare(_np(out), o_ref, _np(lse), lse_ref,
+            label=f"seed={seed} G={G} D={D} S={S} S_kv={S_kv} n_req={n_req} merge={merge} split={split}")
