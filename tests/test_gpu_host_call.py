@@ -27,9 +27,12 @@ def _pinned(t):
     return t.cpu().contiguous().pin_memory()
 
 
-@pytest.mark.parametrize("S,S_kv", [(150, 150), (40, 70), (1, 129)])
-def test_host_call_matches_device_call(S, S_kv):
-    wl = make_custom("hostcall", G128, 101, [37, 700, 64, 129], [[1, 0], [3, 2, 0]], S, S_kv, device=DEV)
+@pytest.mark.parametrize("S,S_kv,reqs", [(150, 150, [[1, 0], [3, 2, 0]]), (40, 70, [[1, 0], [3, 2, 0]]),
+                                          (1, 129, [[1, 0], [3, 2, 0]]),
+                                          # decode whose requests share most artifacts: shared reads
+                                          (1, 129, [[1, 0], [1, 3, 2, 0], [0, 1], [3, 1]])])
+def test_host_call_matches_device_call(S, S_kv, reqs):
+    wl = make_custom("hostcall", G128, 101, [37, 700, 64, 129], reqs, S, S_kv, device=DEV)
     g = wl.geom
     ctx, plan = load_context(wl)
     stream = torch.cuda.Stream(device=DEV)
