@@ -387,8 +387,10 @@ attuner_status attuner_sync_status(attuner_ctx* ctx, void* stream);
  *                               requests that use it, each request's partial
  *                               results merged afterwards.  0 auto (where it
  *                               saves 10 % or more of the block reads), 1 off,
- *                               2 wherever it applies: plans without online
- *                               spans whose keys were not rotated at assembly,
+ *                               2 wherever it applies: every query sees every
+ *                               artifact (no online spans, or every query row
+ *                               in its request's final online span, as a
+ *                               decode token is), keys not rotated at assembly,
  *                               at least two requests' rows per CTA, at most
  *                               511 distinct artifacts in the plan
  *   ATTUNER_OPT_SYNC_CHECK      0 off, 1 every compute call reports the device

@@ -584,8 +584,9 @@ static cudaError_t launch_attn_mma_t(const AttnParams& p, cudaStream_t st) {
 
 template <int D>
 static cudaError_t launch_attn_mma_d(const AttnParams& p, cudaStream_t st) {
-  // shared reads are planned only for plans without online spans
-  if (p.work.share) return p.plan.has_spans ? cudaErrorInvalidValue : launch_attn_mma_t<D, false, true>(p, st);
+  // shared reads are planned only where every query sees every artifact slot
+  // (online spans, if any, all before the queries), so they need no layout rule
+  if (p.work.share) return launch_attn_mma_t<D, false, true>(p, st);
   return p.plan.has_spans ? launch_attn_mma_t<D, true, false>(p, st) : launch_attn_mma_t<D, false, false>(p, st);
 }
 

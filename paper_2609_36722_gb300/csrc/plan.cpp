@@ -263,12 +263,16 @@ attuner_status split_work(const SplitPolicy& pol, const PlanTables& t, int S, in
   }
   // Shared reads (warp-MMA kernel): a CTA reads a chunk of one artifact for up
   // to `members` requests that use it.  Taken where it saves 10 % or more of
-  // the block reads (or always, opt_share = 2, where it applies).
+  // the block reads (or always, opt_share = 2, where it applies).  Every query
+  // must see every artifact slot: in a prompt layout, every query row sits in
+  // its request's final online span (as a decode token does).
   {
     const int SG = S * G;
     const int members = SG <= kMmaRows ? kMmaRows / SG : 0;
     const int nd = t.n_dist();
-    if (!tc && pol.opt_share != 1 && members >= 2 && pol.kv_part == 0 && t.max_o_rows == 0 && !pol.k_by_slot &&
+    bool all_see_all = true;
+    for (int r = 0; r < t.n_req && t.max_o_rows > 0; ++r) all_see_all &= S <= S_kv - t.o_rows[r];
+    if (!tc && pol.opt_share != 1 && members >= 2 && pol.kv_part == 0 && all_see_all && !pol.k_by_slot &&
         nd > 0 && nd <= kMaxShareArts) {
       long long reads_req = 0, reads_share = 0;
       for (int d = 0; d < nd; ++d) {

@@ -187,8 +187,9 @@ struct SplitPolicy {
   // without online spans: the suffix)
   int32_t kv_part = 0;
   // shared reads of the warp-MMA kernel: 0 where they save 10 % or more of
-  // the block reads, 1 never, 2 wherever they apply (a plan without online
-  // spans whose keys are read from the pool, every slot, 2 or more requests'
+  // the block reads, 1 never, 2 wherever they apply (every query sees every
+  // artifact slot - no online spans, or every query in its request's final
+  // span -, keys read from the pool, every slot read, 2 or more requests'
   // rows per CTA)
   int32_t opt_share = 0;
   int32_t k_by_slot = 0;      // keys rotated at assembly: reads cannot be shared

@@ -121,7 +121,7 @@ extern "C" int shim_qproj_supported(int32_t D, int32_t mr, int32_t ks, int32_t n
 
 // Shared reads: the plan of (first, L, items, offs) and the split-KV work of
 // one warp-MMA launch over it.  pol = n_q_heads, n_kv_heads, num_sms,
-// opt_split, opt_share, k_by_slot, kv_part.  out (capacity cap) = n_cta,
+// opt_split, opt_share, k_by_slot, kv_part, layout (items < 0: online spans).  out (capacity cap) = n_cta,
 // chunk_blocks, share, members, n_dist, art_units, suf_chunks, n_part,
 // whole_refs, base[n_req] | nsplit[n_dist + 1] | ref_req | ref_slot |
 // ref_nblk | dist_off[n_dist + 1] | dist_refs | dist_src | dist_nb |
@@ -133,7 +133,7 @@ extern "C" int shim_share(const int32_t* pol, const int32_t* first, const int32_
   for (int i = 0; i < n_arts; ++i)
     arts.push_back(att::Artifact{first[i], L[i], (L[i] + att::kBlockTokens - 1) / att::kBlockTokens});
   att::PlanTables t;
-  attuner_status s = att::build_plan_tables(arts, items, offs, n_req, false, t, g_err);
+  attuner_status s = att::build_plan_tables(arts, items, offs, n_req, pol[7] != 0, t, g_err);
   if (s != ATTUNER_OK) return s;
   att::SplitPolicy p;
   p.n_q_heads = pol[0];

@@ -178,3 +178,21 @@ def test_layout_many_short_spans_decode():
     plan = ctx.assemble_layout(MANY_LAYOUTS)
     out, lse = _run(ctx, plan, wl)
     compare(f64(out), ref_o, f64(lse), ref_l, label="many spans decode")
+
+
+@pytest.mark.parametrize("share", [1, 2])
+def test_layout_decode_with_shared_reads(share):
+    # four decode tokens whose layouts share artifacts (and online spans before
+    # and between them): every query sits in its final span and sees every
+    # artifact, so the decode kernel may read each artifact once for all four
+    import paper_2609_36722_gb300 as pkg
+    layouts = [[-12, 1, -5, 0, -5, 3], [-7, 4, -5, 2, -70, 2, 0], [1, -5, 0], [-3, 3, 1, 0]]
+    reqs = [[a for a in lay if a >= 0] for lay in layouts]
+    wl = make_custom("layout_share", G128, 87, LENGTHS, reqs, 1, 129, device=DEV)
+    ref_o, ref_l = _reference(wl, layouts)
+    ctx, _ = load_context(wl)
+    plan = ctx.assemble_layout(layouts)
+    ctx.set_option(pkg.OPT_PREFILL_KERNEL, 2)
+    ctx.set_option(pkg.OPT_SHARE_READS, share)
+    out, lse = _run(ctx, plan, wl)
+    compare(f64(out), ref_o, f64(lse), ref_l, label=f"layout decode share={share}")

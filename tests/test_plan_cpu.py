@@ -472,7 +472,7 @@ def test_qproj_shape_options_and_limits(shim):
 # shared reads of the decode kernel
 # ---------------------------------------------------------------------------
 def share_plan(shim, lengths, requests, S, S_kv, n_q=32, n_kv=8, num_sms=152, opt_split=0, opt_share=0,
-               k_by_slot=0, kv_part=0):
+               k_by_slot=0, kv_part=0, layout=0):
     firsts = bump_firsts(lengths)
     n_req = len(requests)
     items = [it for r in requests for it in r]
@@ -481,7 +481,7 @@ def share_plan(shim, lengths, requests, S, S_kv, n_q=32, n_kv=8, num_sms=152, op
     la, lp = _i32(lengths)
     ia, ip = _i32(items if items else [0])
     oa, op = _i32(offs)
-    pol = _i32([n_q, n_kv, num_sms, opt_split, opt_share, k_by_slot, kv_part])
+    pol = _i32([n_q, n_kv, num_sms, opt_split, opt_share, k_by_slot, kv_part, layout])
     cap = 1 << 20
     out = np.zeros(cap, np.int32)
     lens = np.zeros(2, np.int64)
@@ -664,3 +664,24 @@ def test_share_falls_back_beyond_the_distinct_artifact_table(shim):
     w, t = share_plan(shim, lengths[:511], [[i, (i + 7) % 511] for i in range(511)], 1, 9, opt_share=2)
     assert w["share"] == 1 and w["n_dist"] == 511
     check_share_work(w, t, lengths[:511], [[i, (i + 7) % 511] for i in range(511)], 1, 9, 32, 8)
+
+
+def test_share_reads_of_prompt_layouts(shim):
+    # online spans before and between artifacts: a decode token (in the final
+    # span) sees every artifact, so the reads can be shared; queries that sit
+    # in an earlier span see only some artifacts, so they cannot
+    lengths = [640, 1280, 320, 2048]
+    layouts = [[-12, 1, -5, 0, -5, 3], [-7, 1, -5, 3, 0], [0, -9, 1, 3], [3, 1]]
+    w, t = share_plan(shim, lengths, layouts, 1, 129, layout=1)
+    assert w["share"] == 1
+    arts = [[a for a in lay if a >= 0] for lay in layouts]
+    check_share_work(w, t, lengths, arts, 1, 129, 32, 8)
+    # every query row in the final span: 2 rows of 129 - 22 (the largest explicit span total)
+    assert share_plan(shim, lengths, layouts, 2, 129, layout=1)[0]["share"] == 1
+    # G = 1, S = 8 (two requests per CTA): with 25 online rows, request 0's 22
+    # explicit rows leave 3 in its final span, so 8 queries reach into the
+    # spans and cannot share; 3 queries can
+    assert share_plan(shim, lengths, layouts, 8, 25, n_q=8, n_kv=8, opt_share=2, layout=1)[0]["share"] == 0
+    w3, t3 = share_plan(shim, lengths, layouts, 3, 25, n_q=8, n_kv=8, opt_share=2, layout=1)
+    assert w3["share"] == 1
+    check_share_work(w3, t3, lengths, arts, 3, 25, 8, 8)
