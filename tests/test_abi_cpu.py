@@ -89,3 +89,17 @@ def test_every_status_entry_point_documents_its_errors():
     for m in re.finditer(r"attuner_status\s+(attuner_\w+)\s*\(", src):
         comment = src[:m.start()].rsplit("/*", 1)[-1]
         assert "Errors" in comment, m.group(1)
+
+
+def test_binding_constants_match_the_header():
+    # every status code and option the header defines has the same value in
+    # the Python binding (a drift would silently pass the wrong option)
+    from paper_2609_36722_gb300 import attuner as A
+    with open(os.path.join(ROOT, "include", "attuner.h")) as f:
+        text = f.read()
+    defs = {m.group(1): int(m.group(2)) for m in
+            re.finditer(r"^#define ATTUNER_((?:OK|ERR_[A-Z_]+|OPT_[A-Z_]+))\s+\(?(-?\d+)\)?", text, re.M)}
+    assert len([k for k in defs if k.startswith("OPT_")]) >= 9 and len([k for k in defs if k.startswith("ERR_")]) >= 7
+    for name, value in defs.items():
+        assert getattr(A, name) == value, name
+    assert A.BLOCK_TOKENS == int(re.search(r"#define ATTUNER_BLOCK_TOKENS\s+(\d+)", text).group(1))
