@@ -111,3 +111,18 @@ def test_clock_sampler_without_nvidia_smi(monkeypatch):
     monkeypatch.setenv("PATH", "")
     s = bench.ClockSampler(0)
     assert s.stop() is None
+
+
+def test_decode_read_fractions():
+    # the decode roofline in the bytes a launch must move: distinct K/V per
+    # second against the peak, and the measured DRAM bytes when a current
+    # traffic record exists
+    g = Geometry(hidden=128, n_q_heads=8, n_kv_heads=2, head_dim=64, rank=8)
+    wl = make_custom("d", g, 7, [70, 5, 130, 64], [[0, 2], [2, 1], [3, 1, 3], [2]], 1, 9)
+    per_token = 2 * 2 * 64 * 2
+    distinct = (70 + 5 + 130 + 64 + 4 * 9) * per_token
+    f = bench.decode_read_fracs(wl, 0.5, 100.0, None)
+    assert f["distinct_bytes"] == distinct and "dram_frac" not in f
+    assert abs(f["distinct_frac"] - round(distinct / 0.5e-3 / 1e9 / 100.0, 4)) < 1e-12
+    f = bench.decode_read_fracs(wl, 0.5, 100.0, 10_000_000)
+    assert abs(f["dram_frac"] - round(1e7 / 0.5e-3 / 1e9 / 100.0, 4)) < 1e-12
